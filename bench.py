@@ -1,0 +1,423 @@
+"""Benchmark of the C2KV hot path: compose stored compressed chunks into one GQA cache
+(RoPE re-rotated) and run the suffix tokens' attention over it, through the C ABI.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                    [--workload NAME]
+
+A step is one pass of the whole path over one batch: c2kv_compose (all layers, one
+launch) + c2kv_attend (suffix RoPE/append + attention, all layers) + cache release.
+Metric: composed KV tokens/s = composed positions of the batch / step time.
+Prints one JSON line (rank 0).  Under torchrun every rank runs its own replica of the
+workload (requests are independent: weak scaling, no data-path collective); only the
+timing barrier and the max-over-ranks reduction cross ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+L2_FLUSH_BYTES = 256 << 20          # > 129 MB of L2
+METRIC = "composed KV tokens/s"
+
+
+# --------------------------------------------------------------------------- workload
+
+def workload_facts(wl):
+    """Sizes the metric and the rooflines are computed from."""
+    m = -(-wl.chunk_tokens // wl.ratio_k)
+    S = wl.chunks_per_request * m                          # composed slots / request
+    span = wl.chunks_per_request * (wl.chunk_tokens + wl.gap)
+    eb = 4 if wl.dtype == "f32" else 2
+    row_bytes = wl.n_kv_heads * wl.head_dim * eb
+    # compose: every stored slot read once (K and V) and written once, plus its position
+    compose_bytes = wl.layers * wl.batch * S * row_bytes * 2 * 2 + wl.batch * S * 4
+    sq = wl.n_suffix
+    keys = S * sq + sq * (sq + 1) // 2                     # visible (query, key) pairs
+    attn_flops = 4 * wl.head_dim * wl.n_q_heads * keys * wl.batch * wl.layers
+    return dict(slots=S, span=span, positions=wl.batch * span, row_bytes=row_bytes,
+                compose_bytes=compose_bytes, attn_flops=attn_flops, slots_per_chunk=m)
+
+
+def describe(wl):
+    f = workload_facts(wl)
+    return (f"{wl.name}: Hq{wl.n_q_heads}/Hkv{wl.n_kv_heads} d{wl.head_dim} {wl.dtype}, "
+            f"{wl.layers} layers, batch {wl.batch} x {wl.chunks_per_request} chunks x "
+            f"{wl.chunk_tokens} tok, k={wl.ratio_k} ({f['slots']} slots, {f['span']} "
+            f"positions/request), {wl.n_suffix} suffix tokens")
+
+
+def measured_peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as fh:
+            pk = json.load(fh)
+        return pk["hbm_gbs"], pk["bf16_tflops"], pk.get("bf16_tflops_sustained"), "measured"
+    return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+# --------------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi sampling of SM clocks and throttle reasons while the timed region runs."""
+
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.proc = None
+        self.gpu = gpu_index
+        self.path = os.path.join("/tmp", f"c2kv_clocks_{os.getpid()}.csv")
+
+    def __enter__(self):
+        try:
+            self.fh = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.QUERY}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=self.fh, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except (OSError, FileNotFoundError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.fh.close()
+
+    def summary(self):
+        if self.proc is None or not os.path.exists(self.path):
+            return None
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                smax.append(float(parts[2]))
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# --------------------------------------------------------------------------- our arm
+
+class Arm:
+    """One replica of the workload on this rank's GPU."""
+
+    def __init__(self, wl, seed, torch, c2kv):
+        self.wl, self.torch, self.c2kv = wl, torch, c2kv
+        f = self.facts = workload_facts(wl)
+        self.tdt = torch.float32 if wl.dtype == "f32" else torch.bfloat16
+        self.stream = torch.cuda.current_stream()
+        self.reqs = synth.requests(wl, seed)
+        pool_ids = sorted({c for ids, _ in self.reqs for c in ids})
+        m = f["slots_per_chunk"]
+        self.ctx = c2kv.c2kv_create(
+            wl.layers, wl.n_q_heads, wl.n_kv_heads, wl.head_dim, wl.rope_theta,
+            c2kv.DTYPE_F32 if wl.dtype == "f32" else c2kv.DTYPE_BF16,
+            pool_slots=len(pool_ids) * m * 2 + 64, stream=self.stream)
+        # stored compressed chunks, kept in pinned host memory (the storage tier) and
+        # loaded once into the device pool for the device-resident measurement
+        self.host_chunks = {}
+        self.dev_ids = {}
+        for cid in pool_ids:
+            ks, vs = synth.chunk_slots(wl, cid, m, seed)
+            kh = torch.from_numpy(ks).to(self.tdt).pin_memory()
+            vh = torch.from_numpy(vs).to(self.tdt).pin_memory()
+            self.host_chunks[cid] = (kh, vh)
+            self.dev_ids[cid] = c2kv.c2kv_compress_chunk(self.ctx, kh, vh, wl.chunk_tokens,
+                                                         wl.ratio_k, c2kv.MODE_STORED)
+        self.req_ptr = np.cumsum([0] + [len(ids) for ids, _ in self.reqs]).astype(np.int32)
+        self.positions = [o for _, offs in self.reqs for o in offs]
+        q, k, v = synth.suffix(wl, seed)
+        self.q_host = [torch.from_numpy(x).to(self.tdt).pin_memory() for x in (q, k, v)]
+        self.q_dev = [x.to("cuda") for x in self.q_host]
+        self.out = torch.empty_like(self.q_dev[0])
+        self.out_host = torch.empty(self.out.shape, dtype=self.tdt).pin_memory()
+        self.flush_buf = torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device="cuda")
+        c2kv.c2kv_sync(self.ctx)
+
+    def flush_l2(self):
+        self.flush_buf.fill_(1.0)
+
+    def launches_per_step(self):
+        n_occ = int(self.req_ptr[-1])
+        groups = -(-n_occ // 128)
+        return groups + 3 * (-(-self.wl.batch // 256))
+
+    def step_device(self, ev):
+        """compose + attend with inputs resident in HBM; ev = 4 events to record."""
+        c2kv, wl = self.c2kv, self.wl
+        ids = [self.dev_ids[c] for ids_, _ in self.reqs for c in ids_]
+        ev[0].record(self.stream)
+        cache = c2kv.c2kv_compose(self.ctx, self.req_ptr, ids, self.positions, wl.n_suffix)
+        ev[1].record(self.stream)
+        c2kv.c2kv_attend(self.ctx, cache, -1, *self.q_dev, wl.n_suffix, self.out)
+        ev[2].record(self.stream)
+        c2kv.c2kv_cache_release(self.ctx, cache)
+        ev[3].record(self.stream)
+
+    def step_e2e(self):
+        """The same step from host buffers: load the requested chunks from pinned host
+        memory into the pool, copy the suffix in, compose, attend, read the output back."""
+        c2kv, wl, torch = self.c2kv, self.wl, self.torch
+        loaded = {}
+        for cid, (kh, vh) in self.host_chunks.items():
+            loaded[cid] = c2kv.c2kv_compress_chunk(self.ctx, kh, vh, wl.chunk_tokens,
+                                                   wl.ratio_k, c2kv.MODE_STORED)
+        qd = [x.to("cuda", non_blocking=True) for x in self.q_host]
+        ids = [loaded[c] for ids_, _ in self.reqs for c in ids_]
+        cache = c2kv.c2kv_compose(self.ctx, self.req_ptr, ids, self.positions, wl.n_suffix)
+        c2kv.c2kv_attend(self.ctx, cache, -1, *qd, wl.n_suffix, self.out)
+        self.out_host.copy_(self.out, non_blocking=True)
+        c2kv.c2kv_cache_release(self.ctx, cache)
+        for cid in loaded.values():
+            c2kv.c2kv_free_chunk(self.ctx, cid)
+
+    def e2e_bytes(self):
+        h2d = sum(kh.numel() * kh.element_size() * 2 for kh, _ in self.host_chunks.values())
+        h2d += sum(x.numel() * x.element_size() for x in self.q_host)
+        d2h = self.out_host.numel() * self.out_host.element_size()
+        return h2d, d2h
+
+    def close(self):
+        self.c2kv.c2kv_destroy(self.ctx)
+
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def run_ours(args):
+    import torch
+    import __graft_entry__ as g
+    g.build()
+    from paper_2607_17715_gb300 import c2kv
+
+    world, rank, local = dist_setup()
+    torch.cuda.set_device(local)
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    wl = synth.workload(args.workload)
+    arm = Arm(wl, seed=rank, torch=torch, c2kv=c2kv)
+    f = arm.facts
+    E = torch.cuda.Event
+
+    def barrier():
+        torch.cuda.synchronize()
+        if world > 1:
+            torch.distributed.barrier()
+            torch.cuda.synchronize()
+
+    for _ in range(args.warmup):
+        arm.flush_l2()
+        arm.step_device([E(enable_timing=True) for _ in range(4)])
+    c2kv.c2kv_sync(arm.ctx)
+
+    events = [[E(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    barrier()
+    with ClockSampler(local) as clocks:
+        t0 = time.perf_counter()
+        for i in range(args.steps):
+            arm.flush_l2()           # untimed: L2 holds none of this step's inputs
+            arm.step_device(events[i])
+        torch.cuda.synchronize()
+        wall = time.perf_counter() - t0
+    barrier()
+    c2kv.c2kv_sync(arm.ctx)
+    step_ms = [ev[0].elapsed_time(ev[3]) for ev in events]
+    compose_ms = [ev[0].elapsed_time(ev[1]) for ev in events]
+    attend_ms = [ev[1].elapsed_time(ev[2]) for ev in events]
+    total_ms = sum(step_ms)
+
+    # end to end from host buffers (copies inside the timed region)
+    for _ in range(max(1, args.warmup // 2)):
+        arm.step_e2e()
+    barrier()
+    e0, e1 = E(enable_timing=True), E(enable_timing=True)
+    e0.record(arm.stream)
+    for _ in range(args.steps):
+        arm.step_e2e()
+    e1.record(arm.stream)
+    torch.cuda.synchronize()
+    c2kv.c2kv_sync(arm.ctx)
+    e2e_ms = e0.elapsed_time(e1)
+    h2d, d2h = arm.e2e_bytes()
+
+    times = torch.tensor([total_ms, e2e_ms], device="cuda", dtype=torch.float64)
+    if world > 1:
+        torch.distributed.all_reduce(times, op=torch.distributed.ReduceOp.MAX)
+    total_ms, e2e_ms = times.tolist()
+    arm.close()
+    if rank != 0:
+        if world > 1:
+            torch.distributed.destroy_process_group()
+        return
+
+    hbm, bf16, bf16_sus, src = measured_peaks()
+    positions = f["positions"] * world * args.steps
+    value = positions / (total_ms / 1e3)
+    c_ms = statistics.mean(compose_ms)
+    a_ms = statistics.mean(attend_ms)
+    comp_gbs = f["compose_bytes"] / (c_ms / 1e3) / 1e9
+    attn_tfs = f["attn_flops"] / (a_ms / 1e3) / 1e12
+    clk = clocks.summary()
+    line = {
+        "metric": METRIC, "value": round(value, 1), "unit": "tokens/s", "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(total_ms / args.steps, 5), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype, "data": "synthetic",
+        "config": {"workload": describe(wl), "parallelism": f"replicas x{world}",
+                   "l2": "flushed between timed steps (256 MB write, untimed)",
+                   "global_batch": wl.batch * world,
+                   "ttft_proxy_ms_per_layer": round(c_ms / wl.layers, 6),
+                   "compose_ms": round(c_ms, 5), "attend_ms": round(a_ms, 5),
+                   "compose_gbs": round(comp_gbs, 1), "attend_tflops": round(attn_tfs, 2),
+                   "compose_bytes": f["compose_bytes"], "attend_flops": f["attn_flops"],
+                   "wall_s": round(wall, 4)},
+        "roofline": {"bound": "hbm", "kernel": "compose_kernel", "achieved": round(comp_gbs, 1),
+                     "peak": hbm, "unit": "GB/s", "frac": round(comp_gbs / hbm, 4),
+                     "traffic": None, "peak_source": f"{src} hbm_gbs",
+                     "bytes_per_launch": f["compose_bytes"]},
+        "roofline_attend": {"bound": "tensor", "achieved": round(attn_tfs, 2), "peak": bf16,
+                            "unit": "TFLOP/s", "frac": round(attn_tfs / bf16, 4),
+                            "peak_source": f"{src} bf16_tflops (burst)",
+                            "note": "c2kv_attend call: suffix RoPE/append + attention"},
+        "e2e": {"value": round(f["positions"] * world * args.steps / (e2e_ms / 1e3), 1),
+                "unit": "tokens/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+                "ms_per_step": round(e2e_ms / args.steps, 4)},
+        "gpu_launches": arm.launches_per_step() * args.steps,
+        "clocks": clk,
+    }
+    if not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(wl, budget_s=args.cpu_budget)
+    print(json.dumps(line), flush=True)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+
+
+# --------------------------------------------------------------------------- oracle arm
+
+def cpu_threads():
+    try:
+        from threadpoolctl import threadpool_info
+        n = [i["num_threads"] for i in threadpool_info() if i.get("user_api") == "blas"]
+        if n:
+            return max(n)
+    except Exception:
+        pass
+    return len(os.sched_getaffinity(0))
+
+
+def oracle_sample(wl, layers, seed=0):
+    """Time the oracle's compose + attend for `layers` layers of request 0's workload."""
+    from oracle import c2kv_oracle as orc
+    sub = synth.scaled(wl, layers=1)
+    reqs = synth.requests(wl, seed)
+    m = -(-wl.chunk_tokens // wl.ratio_k)
+    ids, offs = reqs[0]
+    chunks = {}
+    for cid in sorted(set(ids)):
+        ks, vs = synth.chunk_slots(sub, cid, m, seed)
+        chunks[cid] = (ks.astype(np.float64), vs.astype(np.float64), wl.chunk_tokens,
+                       wl.ratio_k)
+    q, k, v = synth.suffix(sub, seed)
+    t0 = time.perf_counter()
+    for _ in range(layers):
+        orc.run_request(chunks, ids, offs, q[:, 0], k[:, 0], v[:, 0], wl.rope_theta, wl.dtype)
+    return time.perf_counter() - t0
+
+
+def cpu_baseline(wl, budget_s=15.0):
+    """The oracle as it stands on this host's cores, on a bounded sample: as many layers of
+    request 0 as fit in about `budget_s` seconds, scaled to the whole batch."""
+    f = workload_facts(wl)
+    t1 = oracle_sample(wl, 1)
+    n = int(max(1, min(wl.layers * wl.batch, budget_s // max(t1, 1e-3))))
+    t = oracle_sample(wl, n)
+    per_layer_req = t / n
+    step_s = per_layer_req * wl.layers * wl.batch
+    return {"value": round(f["positions"] / step_s, 1), "unit": "tokens/s",
+            "cores": cpu_threads(), "kind": "oracle",
+            "sample": f"{n} (layer, request) compose+attend passes of the oracle (fp64 numpy), "
+                      f"{t:.1f} s, scaled to {wl.layers} layers x {wl.batch} requests"}
+
+
+def run_reference(args):
+    world, rank, _ = dist_setup()
+    if rank != 0:
+        return
+    wl = synth.workload(args.workload)
+    f = workload_facts(wl)
+    for _ in range(args.warmup):
+        oracle_sample(wl, 1)
+    times = [oracle_sample(wl, 1) for _ in range(args.steps)]
+    step_s = statistics.mean(times) * wl.layers * wl.batch
+    value = f["positions"] / step_s
+    cores = cpu_threads()
+    line = {
+        "impl": "reference", "metric": METRIC, "value": round(value, 1), "unit": "tokens/s",
+        "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(step_s * 1e3, 3), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": describe(wl), "parallelism": "cpu oracle"},
+        "cpu_baseline": {"value": round(value, 1), "unit": "tokens/s", "cores": cores,
+                         "kind": "oracle",
+                         "sample": f"each step: compose+attend of 1 layer of request 0, "
+                                   f"scaled x{wl.layers * wl.batch}"},
+        "e2e": {"value": round(value, 1), "unit": "tokens/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="llama8b", choices=sorted(synth.WORKLOADS))
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-budget", type=float, default=15.0)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

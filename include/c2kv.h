@@ -1,0 +1,237 @@
+/*
+ * c2kv.h -- C ABI of the GB300 (sm_103a) library for C2KV compressed, composable KV-cache
+ * reuse (arXiv 2607.17715): store per-chunk compressed KV, compose the chunks a request
+ * asks for into one contiguous GQA cache (RoPE re-rotated to the request's positions),
+ * and run the request's suffix tokens' attention over it.
+ *
+ * The paper's generalized reuse pipeline (Sec. 2.2) has three steps, and the calls below
+ * follow them:
+ *   Encoding  M : KV_k     = M(x_k)                   -> c2kv_compress_chunk
+ *   Blending  B : KV_total = B(x_s, KV_1 .. KV_K)     -> c2kv_compose
+ *   Inference F : y        = F([KV_total, x_q])       -> c2kv_attend
+ *
+ * Conventions shared by every call
+ *   - Every call returns a c2kv_status at once: C2KV_OK (0) or a negative code.  No C++
+ *     exception and no abort ever crosses this boundary.
+ *   - GPU work is enqueued on the context's CUDA stream and runs asynchronously.  Errors
+ *     found by a kernel's own bounds checks surface at the next c2kv_sync().
+ *   - On any error status the library's state (pool, chunk table, caches) is unchanged
+ *     and c2kv_last_error() describes the failure.
+ *   - Tensors are dense, row-major, with the innermost dimension last.  "d" is head_dim,
+ *     "Hq"/"Hkv" the query / key-value head counts, "L" the layer count.  Element type is
+ *     the context dtype (bf16 or fp32) unless stated.
+ *   - The caller owns every buffer it passes in; the library owns the chunk pool and the
+ *     composed caches it returns.
+ *   - A context is used from one host thread at a time.
+ */
+#ifndef C2KV_H
+#define C2KV_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int32_t c2kv_status;
+
+#define C2KV_OK                  0
+#define C2KV_ERR_ARG            -1   /* null pointer, bad size or shape                  */
+#define C2KV_ERR_DTYPE          -2   /* dtype not supported for this call                */
+#define C2KV_ERR_NOMEM          -3   /* device or pinned host allocation failed          */
+#define C2KV_ERR_POOL_FULL      -4   /* no contiguous free slot range in the chunk pool  */
+#define C2KV_ERR_BAD_CHUNK      -5   /* unknown or freed chunk id                        */
+#define C2KV_ERR_POSITIONS      -6   /* offsets negative, decreasing or overlapping      */
+#define C2KV_ERR_CUDA           -7   /* a CUDA runtime call failed                       */
+#define C2KV_ERR_DEVICE_BOUNDS  -8   /* a kernel's bounds check refused an index         */
+#define C2KV_ERR_STATE          -9   /* object used in the wrong state / wrong context   */
+#define C2KV_ERR_UNSUPPORTED   -10   /* valid request this build does not implement      */
+
+#define C2KV_DTYPE_BF16 0
+#define C2KV_DTYPE_F32  1
+
+/* c2kv_compress_chunk modes */
+#define C2KV_MODE_MEANPOOL 0  /* tokens -> slots: block mean of pre-RoPE K/V rows            */
+#define C2KV_MODE_PROVIDED 1  /* slots given pre-RoPE by an external extractor               */
+#define C2KV_MODE_STORED   2  /* slots given already in stored form (load from host storage) */
+
+/* c2kv_attend kernel choice */
+#define C2KV_ATTN_AUTO   0    /* tensor-core kernel where it applies, SIMT otherwise */
+#define C2KV_ATTN_SIMT   1    /* CUDA-core fp32-accumulate kernel (any dtype)        */
+#define C2KV_ATTN_TC     2    /* tcgen05 / TMEM tensor-core kernel (bf16, d = 128)    */
+
+typedef struct c2kv_ctx c2kv_ctx;
+typedef struct c2kv_cache c2kv_cache;
+
+/* Model / pool shape.  head_dim must be 64 or 128; n_q_heads a multiple of n_kv_heads. */
+typedef struct c2kv_config {
+    int32_t layers;
+    int32_t n_q_heads;
+    int32_t n_kv_heads;
+    int32_t head_dim;
+    double  rope_theta;        /* RoPE base: pair (i, i + d/2) turns by pos * theta^(-2i/d) */
+    int32_t dtype;             /* C2KV_DTYPE_BF16 or C2KV_DTYPE_F32                           */
+    int32_t pool_slots;        /* capacity of the device chunk pool, in slots (all layers)    */
+    int32_t fixed_pos;         /* 1 = no re-rotation at compose ("Fixed-Pos." ablation,
+                                  Sec. 4.8): slots keep their chunk-local positions          */
+    int32_t attn_impl;         /* C2KV_ATTN_AUTO / _SIMT / _TC                                */
+} c2kv_config;
+
+/* Chunk metadata (c2kv_chunk_info). */
+typedef struct c2kv_chunk_desc {
+    int32_t n_tokens;          /* original chunk length n (the span it occupies when composed) */
+    int32_t ratio_k;           /* compression ratio k                                          */
+    int32_t n_slots;           /* m = ceil(n / k)                                              */
+    int32_t slot_base;         /* first pool slot                                              */
+    void*   k;                 /* device: pool K at (layer 0, slot_base); layer stride below   */
+    void*   v;                 /* device: pool V, same layout                                  */
+    int64_t layer_stride;      /* elements between layers = pool_slots * Hkv * d              */
+} c2kv_chunk_desc;
+
+/* Composed cache metadata (c2kv_cache_info).  Host arrays stay valid until release. */
+typedef struct c2kv_cache_desc {
+    int32_t batch;
+    int32_t layers;
+    int64_t rows;              /* rows per layer in k / v (all requests, padded)          */
+    void*   k;                 /* device [layers][rows][Hkv][d]                            */
+    void*   v;                 /* device [layers][rows][Hkv][d]                            */
+    int32_t* pos;              /* device [rows]: composed position of each row             */
+    const int32_t* row_base;   /* host [batch]: first row of each request (multiple of 128)*/
+    const int32_t* n_slots;    /* host [batch]: composed slots S_r of each request         */
+    const int32_t* l_req;      /* host [batch]: composed span L_r = max_i (o_i + n_i)      */
+    const int32_t* capacity;   /* host [batch]: rows reserved for the request              */
+    int32_t suffix_capacity;   /* suffix rows reserved after the slots of each request     */
+} c2kv_cache_desc;
+
+/* ABI version of this header (bumped on any incompatible change). */
+#define C2KV_ABI_VERSION 1
+int32_t c2kv_abi_version(void);
+
+/*
+ * c2kv_create -- make a context on the current CUDA device.
+ *   cfg     : shape and pool size (copied).
+ *   stream  : cudaStream_t to enqueue all work on (NULL = legacy default stream).
+ *   out     : receives the context.
+ * Allocates the chunk pool: 2 * layers * pool_slots * Hkv * d elements of device memory.
+ * Errors: ERR_ARG (bad shape / null out), ERR_DTYPE, ERR_NOMEM, ERR_CUDA.
+ */
+c2kv_status c2kv_create(const c2kv_config* cfg, void* stream, c2kv_ctx** out);
+
+/* c2kv_destroy -- synchronize the stream and free everything the context owns, including
+ * composed caches not yet released.  NULL is accepted. */
+c2kv_status c2kv_destroy(c2kv_ctx* ctx);
+
+/* c2kv_set_stream -- switch the stream later calls enqueue on (e.g. torch's current one). */
+c2kv_status c2kv_set_stream(c2kv_ctx* ctx, void* stream);
+
+/*
+ * c2kv_compress_chunk -- the encoding step M: store one chunk (document) as compressed
+ * slots in the device pool.  Sec. 3.2.1: a chunk of n tokens gets m = ceil(n/k) slots, one
+ * per block of k consecutive tokens; Sec. 3.3.1: slot j takes the position of the last
+ * token of its block, p_j = min((j+1)k, n) - 1.  The pool keeps K with RoPE applied at
+ * p_j (chunk-local positions) and V as is.
+ *
+ *   k, v     : MEANPOOL: device [L][n][Hkv][d] pre-RoPE per-token K/V.  Slot j is the mean
+ *              of block j's rows divided by the block's true size (a stand-in for the
+ *              trained extractor, adapted from the residual mean-pooling variant of
+ *              Sec. 3.2.3).
+ *              PROVIDED: device [L][m][Hkv][d] pre-RoPE slot K/V from an external
+ *              extractor (the paper's C2 token K/V, Sec. 3.2.2); K is turned to p_j.
+ *              STORED: host or device [L][m][Hkv][d] slots already in stored form (K at
+ *              p_j), copied verbatim -- the "load from host memory" step of Appendix C.
+ *   n_tokens : original chunk length n >= 1.
+ *   ratio_k  : compression ratio k >= 1 (k = 1: uncompressed control).
+ *   mode     : C2KV_MODE_*.
+ *   chunk_id_out : receives the new chunk's id (>= 0).
+ * The caller's buffers must stay valid until the stream reaches this call's work.
+ * Errors: ERR_ARG, ERR_POOL_FULL (state unchanged), ERR_CUDA.
+ */
+c2kv_status c2kv_compress_chunk(c2kv_ctx* ctx, const void* k, const void* v, int32_t n_tokens,
+                                int32_t ratio_k, int32_t mode, int32_t* chunk_id_out);
+
+/* c2kv_free_chunk -- return a chunk's slots to the pool.  Composed caches already made
+ * from it are unaffected (they hold copies).  Errors: ERR_BAD_CHUNK. */
+c2kv_status c2kv_free_chunk(c2kv_ctx* ctx, int32_t chunk_id);
+
+/* c2kv_chunk_info -- where a chunk lives in the pool.  Errors: ERR_BAD_CHUNK, ERR_ARG. */
+c2kv_status c2kv_chunk_info(const c2kv_ctx* ctx, int32_t chunk_id, c2kv_chunk_desc* out);
+
+/*
+ * c2kv_compose -- the blending step B for a batch of requests (Sec. 3.2.4): each chunk
+ * occurrence gets new positional embeddings for its placement -- offsets accumulate across
+ * the concatenated segments and a compressed segment occupies its original span -- and
+ * the slots are concatenated, without recomputation (Appendix C: load + position
+ * reassignment + RoPE re-rotation).
+ *
+ * Occurrence i of request r (chunk c_i, n_i tokens, m_i slots, offset o_i) fills rows
+ * row_base[r] + D_i + j, j < m_i, D_i = sum of earlier m, for every layer:
+ *     K' = R(o_i) K_stored   (turn from p_j to o_i + p_j),   V' = V_stored,
+ *     pos = o_i + p_j.
+ * With cfg.fixed_pos, K' = K_stored and pos = p_j.
+ *
+ *   batch           : number of requests B >= 1.
+ *   req_ptr         : host [B + 1], CSR offsets into chunk_ids (req_ptr[0] = 0,
+ *                     non-decreasing; a request may reuse no chunk).
+ *   chunk_ids       : host [req_ptr[B]] chunk ids; duplicates allowed.
+ *   positions       : host [req_ptr[B]] start offset o_i of each occurrence, or NULL for
+ *                     o_0 = 0, o_{i+1} = o_i + n_i within each request.  Must satisfy
+ *                     o_0 >= 0 and o_{i+1} >= o_i + n_i (gaps allowed: room for a static /
+ *                     system prompt, Sec. 4.1), else ERR_POSITIONS.
+ *   suffix_capacity : rows reserved after each request's slots for its suffix tokens.
+ *   out             : receives a library-owned cache; each request's region starts at a
+ *                     multiple of 128 rows and holds round_up(S_r + suffix_capacity, 128)
+ *                     rows.
+ * Errors: ERR_ARG, ERR_BAD_CHUNK, ERR_POSITIONS, ERR_NOMEM, ERR_CUDA.
+ */
+c2kv_status c2kv_compose(c2kv_ctx* ctx, int32_t batch, const int32_t* req_ptr,
+                         const int32_t* chunk_ids, const int32_t* positions,
+                         int32_t suffix_capacity, c2kv_cache** out);
+
+/* c2kv_cache_info -- pointers and per-request metadata of a composed cache. */
+c2kv_status c2kv_cache_info(const c2kv_cache* cache, c2kv_cache_desc* out);
+
+/*
+ * c2kv_attend -- the inference step F over [KV_total; x_q] (Sec. 2.2) with the model's
+ * standard attention operator (Sec. 3.2.2): for each request r, suffix token t sits at
+ * position L_r + t; its Q and K are RoPE'd there, its K/V written into the cache rows
+ * right after the S_r composed slots, and
+ *     O[t, h] = softmax_j( Q_t,h . K_j,h/G / sqrt(d) ) V_j,h/G     over keys j <= S_r + t
+ * (every composed slot visible; causal inside the suffix; G = Hq / Hkv, query head h uses
+ * KV head h / G).
+ *
+ *   layer    : layer index, or -1 for all layers in one launch.
+ *   q        : device [Lq][B][n_suffix][Hq][d] pre-RoPE queries (Lq = L if layer == -1,
+ *              else 1).
+ *   k_suf, v_suf : device [Lq][B][n_suffix][Hkv][d] pre-RoPE suffix K, V.
+ *   n_suffix : suffix tokens per request, 1 <= n_suffix <= the cache's suffix_capacity.
+ *   out      : device [Lq][B][n_suffix][Hq][d] attention output (context dtype).
+ *   lse      : device [Lq][B][Hq][n_suffix] fp32 natural-log softmax normaliser, or NULL.
+ * The call is idempotent: it always writes the suffix at rows S_r .. S_r + n_suffix - 1.
+ * Errors: ERR_ARG, ERR_STATE (cache from another context), ERR_NOMEM, ERR_CUDA.
+ */
+c2kv_status c2kv_attend(c2kv_ctx* ctx, c2kv_cache* cache, int32_t layer, const void* q,
+                        const void* k_suf, const void* v_suf, int32_t n_suffix, void* out,
+                        float* lse);
+
+/* c2kv_cache_release -- free a composed cache (stream-ordered). */
+c2kv_status c2kv_cache_release(c2kv_ctx* ctx, c2kv_cache* cache);
+
+/* c2kv_sync -- wait for the context's stream; returns ERR_DEVICE_BOUNDS if any kernel's
+ * bounds check refused an index since the last sync (the refused access was skipped), or
+ * ERR_CUDA for a CUDA error. */
+c2kv_status c2kv_sync(c2kv_ctx* ctx);
+
+/* c2kv_last_error -- message for the last failing call on this context ("" if none).
+ * Valid until the next call on the context.  NULL ctx gives the last create() failure. */
+const char* c2kv_last_error(const c2kv_ctx* ctx);
+
+/* c2kv_inject_fault -- host-side fault injection for tests.  what = 1: the next compose
+ * writes one out-of-range pool slot index into its slot map, which the compose kernel's
+ * bounds check must refuse (reported by c2kv_sync as ERR_DEVICE_BOUNDS).  what = 0 clears. */
+c2kv_status c2kv_inject_fault(c2kv_ctx* ctx, int32_t what);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* C2KV_H */

@@ -1,0 +1,588 @@
+// Host side of the C2KV library: the C ABI declared in include/c2kv.h.
+//
+// Owns the device chunk pool (a slot arena with a first-fit free list), validates every
+// request before anything is enqueued (so a failing call leaves no trace), packs the small
+// per-call metadata (chunk occurrences, per-request row layout, RoPE frequencies as 0.64
+// fixed-point turns) into the kernels' parameter blocks -- no host-to-device copy per call
+// -- and launches the kernels on the context's stream.  Composed caches and per-call
+// scratch come from a context-owned stream-ordered memory pool.
+#include "c2kv.h"
+#include "internal.cuh"
+
+#include <algorithm>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <new>
+#include <string>
+#include <vector>
+
+
+namespace {
+
+constexpr int64_t kTileRows = 128;   // composed-cache request regions align to this
+
+struct Chunk {
+    int32_t n = 0, k = 0, m = 0, base = 0;
+    bool live = false;
+};
+
+thread_local std::string g_create_error;
+
+}  // namespace
+
+struct c2kv_cache {
+    c2kv_ctx* owner = nullptr;
+    int32_t batch = 0, layers = 0;
+    int64_t rows = 0;
+    void* k = nullptr;
+    void* v = nullptr;
+    int32_t* pos = nullptr;        // device [rows]
+    std::vector<int32_t> row_base, n_slots, l_req, capacity;
+    int32_t suffix_capacity = 0;
+};
+
+struct c2kv_ctx {
+    c2kv_config cfg{};
+    cudaStream_t stream = nullptr;
+    int device = 0;
+    int eb = 2;
+    void* pool_k = nullptr;
+    void* pool_v = nullptr;
+    std::vector<Chunk> chunks;
+    std::map<int32_t, int32_t> free_ranges;   // start -> length
+    std::string err;
+    int32_t* d_err = nullptr;
+    cudaMemPool_t mempool = nullptr;
+    std::vector<c2kv_cache*> caches;
+    int32_t inject = 0;
+    c2kv::RopeTurns turns{};
+};
+
+namespace {
+
+c2kv_status fail(c2kv_ctx* ctx, c2kv_status code, const char* fmt, ...) {
+    char buf[512];
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(buf, sizeof(buf), fmt, ap);
+    va_end(ap);
+    if (ctx) ctx->err = buf;
+    else g_create_error = buf;
+    return code;
+}
+
+c2kv_status cuda_fail(c2kv_ctx* ctx, cudaError_t e, const char* what) {
+    return fail(ctx, e == cudaErrorMemoryAllocation ? C2KV_ERR_NOMEM : C2KV_ERR_CUDA,
+                "%s: %s", what, cudaGetErrorString(e));
+}
+
+int64_t row_elems(const c2kv_ctx* c) { return (int64_t)c->cfg.n_kv_heads * c->cfg.head_dim; }
+
+cudaError_t pool_alloc(c2kv_ctx* c, void** p, size_t bytes) {
+    *p = nullptr;
+    if (bytes == 0) bytes = 256;
+    return cudaMallocFromPoolAsync(p, bytes, c->mempool, c->stream);
+}
+
+void pool_free(c2kv_ctx* c, void* p) {
+    if (p) cudaFreeAsync(p, c->stream);
+}
+
+// RoPE frequency i = theta^(-2i/d) as a fraction of a turn in 0.64 fixed point, from
+// long-double arithmetic (the kernels' phase accumulator; see internal.cuh).
+void make_turns(c2kv::RopeTurns* t, double theta, int d) {
+    const long double two_pi = 6.283185307179586476925286766559005768L;
+    for (int i = 0; i < c2kv::kMaxHalf; ++i) {
+        if (i >= d / 2) {
+            t->turn[i] = 0;
+            continue;
+        }
+        const long double f = std::pow((long double)theta, -2.0L * i / d) / two_pi;
+        t->turn[i] = (uint64_t)std::llround(std::ldexp(f, 64));
+    }
+}
+
+bool take_range(c2kv_ctx* c, int32_t m, int32_t* base) {
+    for (auto it = c->free_ranges.begin(); it != c->free_ranges.end(); ++it) {
+        if (it->second >= m) {
+            *base = it->first;
+            const int32_t rest = it->second - m;
+            const int32_t start = it->first + m;
+            c->free_ranges.erase(it);
+            if (rest > 0) c->free_ranges[start] = rest;
+            return true;
+        }
+    }
+    return false;
+}
+
+void give_range(c2kv_ctx* c, int32_t base, int32_t m) {
+    if (m <= 0) return;
+    auto it = c->free_ranges.emplace(base, m).first;
+    auto next = std::next(it);
+    if (next != c->free_ranges.end() && it->first + it->second == next->first) {
+        it->second += next->second;
+        c->free_ranges.erase(next);
+    }
+    if (it != c->free_ranges.begin()) {
+        auto prev = std::prev(it);
+        if (prev->first + prev->second == it->first) {
+            prev->second += it->second;
+            c->free_ranges.erase(it);
+        }
+    }
+}
+
+bool is_device_ptr(const void* p) {
+    cudaPointerAttributes at{};
+    if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
+}
+
+bool own_cache(const c2kv_ctx* c, const c2kv_cache* cache) {
+    return cache && std::find(c->caches.begin(), c->caches.end(), cache) != c->caches.end();
+}
+
+void destroy_cache(c2kv_ctx* c, c2kv_cache* cache) {
+    pool_free(c, cache->k);
+    pool_free(c, cache->v);
+    pool_free(c, cache->pos);
+    delete cache;
+}
+
+}  // namespace
+
+extern "C" {
+
+int32_t c2kv_abi_version(void) { return C2KV_ABI_VERSION; }
+
+const char* c2kv_last_error(const c2kv_ctx* ctx) {
+    return ctx ? ctx->err.c_str() : g_create_error.c_str();
+}
+
+c2kv_status c2kv_create(const c2kv_config* cfg, void* stream, c2kv_ctx** out) {
+    try {
+        if (!cfg || !out) return fail(nullptr, C2KV_ERR_ARG, "create: null cfg or out");
+        *out = nullptr;
+        const c2kv_config& f = *cfg;
+        if (f.layers < 1 || f.n_q_heads < 1 || f.n_kv_heads < 1 || f.n_q_heads % f.n_kv_heads)
+            return fail(nullptr, C2KV_ERR_ARG, "create: bad layer/head counts");
+        if (f.head_dim != 64 && f.head_dim != 128)
+            return fail(nullptr, C2KV_ERR_ARG, "create: head_dim must be 64 or 128");
+        if (!(f.rope_theta > 1.0)) return fail(nullptr, C2KV_ERR_ARG, "create: rope_theta <= 1");
+        if (f.dtype != C2KV_DTYPE_BF16 && f.dtype != C2KV_DTYPE_F32)
+            return fail(nullptr, C2KV_ERR_DTYPE, "create: dtype must be BF16 or F32");
+        if (f.pool_slots < 1) return fail(nullptr, C2KV_ERR_ARG, "create: pool_slots < 1");
+        if (f.attn_impl < C2KV_ATTN_AUTO || f.attn_impl > C2KV_ATTN_TC)
+            return fail(nullptr, C2KV_ERR_ARG, "create: bad attn_impl");
+        if (f.attn_impl == C2KV_ATTN_TC &&
+            !c2kv::attn_tc_supported(f.dtype, f.head_dim, f.n_q_heads, f.n_kv_heads))
+            return fail(nullptr, C2KV_ERR_UNSUPPORTED,
+                        "create: tensor-core attention needs bf16, head_dim 128, Hq/Hkv in {1,2,4,8,16}");
+        auto* c = new c2kv_ctx();
+        c->cfg = f;
+        c->stream = static_cast<cudaStream_t>(stream);
+        c->eb = f.dtype == C2KV_DTYPE_BF16 ? 2 : 4;
+        cudaError_t e = cudaGetDevice(&c->device);
+        const size_t pool_bytes = (size_t)f.layers * (size_t)f.pool_slots * (size_t)row_elems(c) * c->eb;
+        if (e == cudaSuccess) e = cudaMalloc(&c->pool_k, pool_bytes);
+        if (e == cudaSuccess) e = cudaMalloc(&c->pool_v, pool_bytes);
+        if (e == cudaSuccess) e = cudaMalloc(&c->d_err, sizeof(int32_t));
+        if (e == cudaSuccess) e = cudaMemset(c->d_err, 0, sizeof(int32_t));
+        if (e == cudaSuccess) {
+            cudaMemPoolProps props{};
+            props.allocType = cudaMemAllocationTypePinned;
+            props.location.type = cudaMemLocationTypeDevice;
+            props.location.id = c->device;
+            e = cudaMemPoolCreate(&c->mempool, &props);
+            if (e == cudaSuccess) {
+                uint64_t keep = UINT64_MAX;
+                e = cudaMemPoolSetAttribute(c->mempool, cudaMemPoolAttrReleaseThreshold, &keep);
+            }
+        }
+        if (e != cudaSuccess) {
+            cuda_fail(nullptr, e, "create");
+            c2kv_destroy(c);
+            return e == cudaErrorMemoryAllocation ? C2KV_ERR_NOMEM : C2KV_ERR_CUDA;
+        }
+        c->free_ranges[0] = f.pool_slots;
+        make_turns(&c->turns, f.rope_theta, f.head_dim);
+        *out = c;
+        return C2KV_OK;
+    } catch (const std::bad_alloc&) {
+        return fail(nullptr, C2KV_ERR_NOMEM, "create: host allocation failed");
+    } catch (...) {
+        return fail(nullptr, C2KV_ERR_ARG, "create: unexpected failure");
+    }
+}
+
+c2kv_status c2kv_destroy(c2kv_ctx* c) {
+    if (!c) return C2KV_OK;
+    try {
+        if (c->stream || c->pool_k) cudaStreamSynchronize(c->stream);
+        for (c2kv_cache* cache : c->caches) destroy_cache(c, cache);
+        c->caches.clear();
+        cudaStreamSynchronize(c->stream);
+        if (c->mempool) cudaMemPoolDestroy(c->mempool);
+        if (c->pool_k) cudaFree(c->pool_k);
+        if (c->pool_v) cudaFree(c->pool_v);
+        if (c->d_err) cudaFree(c->d_err);
+        delete c;
+        return C2KV_OK;
+    } catch (...) {
+        return C2KV_ERR_STATE;
+    }
+}
+
+c2kv_status c2kv_set_stream(c2kv_ctx* c, void* stream) {
+    if (!c) return C2KV_ERR_ARG;
+    c->stream = static_cast<cudaStream_t>(stream);
+    c->err.clear();
+    return C2KV_OK;
+}
+
+c2kv_status c2kv_compress_chunk(c2kv_ctx* c, const void* k, const void* v, int32_t n_tokens,
+                                int32_t ratio_k, int32_t mode, int32_t* chunk_id_out) {
+    if (!c) return C2KV_ERR_ARG;
+    try {
+        c->err.clear();
+        if (!k || !v || !chunk_id_out) return fail(c, C2KV_ERR_ARG, "compress: null pointer");
+        if (n_tokens < 1 || ratio_k < 1) return fail(c, C2KV_ERR_ARG, "compress: need n >= 1, k >= 1");
+        if (mode != C2KV_MODE_MEANPOOL && mode != C2KV_MODE_PROVIDED && mode != C2KV_MODE_STORED)
+            return fail(c, C2KV_ERR_ARG, "compress: bad mode %d", mode);
+        if (mode != C2KV_MODE_STORED && (!is_device_ptr(k) || !is_device_ptr(v)))
+            return fail(c, C2KV_ERR_ARG, "compress: MEANPOOL/PROVIDED inputs must be device memory");
+        const int32_t m = (int32_t)(((int64_t)n_tokens + ratio_k - 1) / ratio_k);
+        int32_t base = 0;
+        if (!take_range(c, m, &base))
+            return fail(c, C2KV_ERR_POOL_FULL, "compress: no free range of %d slots", m);
+        const size_t rb = (size_t)row_elems(c) * c->eb;
+        cudaError_t e = cudaSuccess;
+        if (mode == C2KV_MODE_STORED) {
+            const size_t dpitch = (size_t)c->cfg.pool_slots * rb;
+            char* dk = static_cast<char*>(c->pool_k) + (size_t)base * rb;
+            char* dv = static_cast<char*>(c->pool_v) + (size_t)base * rb;
+            e = cudaMemcpy2DAsync(dk, dpitch, k, (size_t)m * rb, (size_t)m * rb, c->cfg.layers,
+                                  cudaMemcpyDefault, c->stream);
+            if (e == cudaSuccess)
+                e = cudaMemcpy2DAsync(dv, dpitch, v, (size_t)m * rb, (size_t)m * rb,
+                                      c->cfg.layers, cudaMemcpyDefault, c->stream);
+        } else {
+            c2kv::CompressParams a{};
+            a.in_k = k;
+            a.in_v = v;
+            a.pool_k = c->pool_k;
+            a.pool_v = c->pool_v;
+            a.pool_slots = c->cfg.pool_slots;
+            a.slot_base = base;
+            a.m = m;
+            a.n = n_tokens;
+            a.k = ratio_k;
+            a.one_row = mode == C2KV_MODE_PROVIDED ? 1 : 0;
+            a.rows_in = mode == C2KV_MODE_PROVIDED ? m : n_tokens;
+            a.layers = c->cfg.layers;
+            a.hkv = c->cfg.n_kv_heads;
+            a.rope = c->turns;
+            e = c2kv::launch_compress(a, c->cfg.dtype, c->cfg.head_dim, c->stream);
+        }
+        if (e != cudaSuccess) {
+            give_range(c, base, m);
+            return cuda_fail(c, e, "compress");
+        }
+        int32_t id = -1;
+        for (size_t i = 0; i < c->chunks.size(); ++i)
+            if (!c->chunks[i].live) { id = (int32_t)i; break; }
+        if (id < 0) {
+            c->chunks.emplace_back();
+            id = (int32_t)c->chunks.size() - 1;
+        }
+        Chunk& ch = c->chunks[id];
+        ch.n = n_tokens;
+        ch.k = ratio_k;
+        ch.m = m;
+        ch.base = base;
+        ch.live = true;
+        *chunk_id_out = id;
+        return C2KV_OK;
+    } catch (const std::bad_alloc&) {
+        return fail(c, C2KV_ERR_NOMEM, "compress: host allocation failed");
+    }
+}
+
+c2kv_status c2kv_free_chunk(c2kv_ctx* c, int32_t id) {
+    if (!c) return C2KV_ERR_ARG;
+    c->err.clear();
+    if (id < 0 || id >= (int32_t)c->chunks.size() || !c->chunks[id].live)
+        return fail(c, C2KV_ERR_BAD_CHUNK, "free_chunk: unknown chunk %d", id);
+    Chunk& ch = c->chunks[id];
+    give_range(c, ch.base, ch.m);
+    ch.live = false;
+    return C2KV_OK;
+}
+
+c2kv_status c2kv_chunk_info(const c2kv_ctx* c, int32_t id, c2kv_chunk_desc* out) {
+    if (!c || !out) return C2KV_ERR_ARG;
+    if (id < 0 || id >= (int32_t)c->chunks.size() || !c->chunks[id].live) return C2KV_ERR_BAD_CHUNK;
+    const Chunk& ch = c->chunks[id];
+    const size_t rb = (size_t)row_elems(c) * c->eb;
+    out->n_tokens = ch.n;
+    out->ratio_k = ch.k;
+    out->n_slots = ch.m;
+    out->slot_base = ch.base;
+    out->k = static_cast<char*>(c->pool_k) + (size_t)ch.base * rb;
+    out->v = static_cast<char*>(c->pool_v) + (size_t)ch.base * rb;
+    out->layer_stride = (int64_t)c->cfg.pool_slots * row_elems(c);
+    return C2KV_OK;
+}
+
+c2kv_status c2kv_compose(c2kv_ctx* c, int32_t batch, const int32_t* req_ptr,
+                         const int32_t* chunk_ids, const int32_t* positions,
+                         int32_t suffix_capacity, c2kv_cache** out) {
+    if (!c) return C2KV_ERR_ARG;
+    try {
+        c->err.clear();
+        if (!out || !req_ptr || batch < 1) return fail(c, C2KV_ERR_ARG, "compose: bad batch/out/req_ptr");
+        *out = nullptr;
+        if (suffix_capacity < 0) return fail(c, C2KV_ERR_ARG, "compose: suffix_capacity < 0");
+        if (req_ptr[0] != 0) return fail(c, C2KV_ERR_ARG, "compose: req_ptr[0] != 0");
+        for (int32_t r = 0; r < batch; ++r)
+            if (req_ptr[r + 1] < req_ptr[r]) return fail(c, C2KV_ERR_ARG, "compose: req_ptr decreases");
+        const int32_t n_occ = req_ptr[batch];
+        if (n_occ > 0 && !chunk_ids) return fail(c, C2KV_ERR_ARG, "compose: null chunk_ids");
+
+        // Validate everything and lay out the rows before touching the device.
+        std::vector<c2kv::OccParam> occ((size_t)n_occ);
+        auto* cache = new c2kv_cache();
+        cache->owner = c;
+        cache->batch = batch;
+        cache->layers = c->cfg.layers;
+        cache->suffix_capacity = suffix_capacity;
+        cache->row_base.resize(batch);
+        cache->n_slots.resize(batch);
+        cache->l_req.resize(batch);
+        cache->capacity.resize(batch);
+        int64_t row = 0;
+        for (int32_t r = 0; r < batch; ++r) {
+            int64_t slots = 0, prev_end = 0;
+            for (int32_t i = req_ptr[r]; i < req_ptr[r + 1]; ++i) {
+                const int32_t id = chunk_ids[i];
+                if (id < 0 || id >= (int32_t)c->chunks.size() || !c->chunks[id].live) {
+                    delete cache;
+                    return fail(c, C2KV_ERR_BAD_CHUNK, "compose: unknown chunk %d (occurrence %d)", id, i);
+                }
+                const Chunk& ch = c->chunks[id];
+                const int64_t o = positions ? positions[i] : prev_end;
+                if (o < 0 || o < prev_end) {
+                    delete cache;
+                    return fail(c, C2KV_ERR_POSITIONS,
+                                "compose: request %d occurrence %d starts at %lld before %lld", r, i,
+                                (long long)o, (long long)prev_end);
+                }
+                prev_end = o + ch.n;
+                if (prev_end > INT32_MAX) {
+                    delete cache;
+                    return fail(c, C2KV_ERR_POSITIONS, "compose: positions exceed int32");
+                }
+                c2kv::OccParam& rec = occ[i];
+                rec.src_base = ch.base;
+                rec.dest_row = (int32_t)(row + slots);
+                rec.delta = c->cfg.fixed_pos ? 0 : (int32_t)o;
+                rec.n = ch.n;
+                rec.k = ch.k;
+                rec.m = ch.m;
+                rec.tile_base = 0;
+                rec.pad = 0;
+                slots += ch.m;
+            }
+            const int64_t cap = (slots + suffix_capacity + kTileRows - 1) / kTileRows * kTileRows;
+            if (row + cap > INT32_MAX) {
+                delete cache;
+                return fail(c, C2KV_ERR_ARG, "compose: batch too large");
+            }
+            cache->row_base[r] = (int32_t)row;
+            cache->n_slots[r] = (int32_t)slots;
+            cache->l_req[r] = (int32_t)prev_end;
+            cache->capacity[r] = (int32_t)cap;
+            row += cap;
+        }
+        cache->rows = row;
+        if (c->inject == 1 && n_occ > 0) {
+            occ[0].src_base = c->cfg.pool_slots + 7;   // refused by the kernel's bounds check
+            c->inject = 0;
+        }
+
+        const size_t kv_bytes = (size_t)c->cfg.layers * (size_t)std::max<int64_t>(row, 1) *
+                                (size_t)row_elems(c) * c->eb;
+        const size_t pos_bytes = (size_t)std::max<int64_t>(row, 1) * sizeof(int32_t);
+        cudaError_t e = pool_alloc(c, &cache->k, kv_bytes);
+        if (e == cudaSuccess) e = pool_alloc(c, &cache->v, kv_bytes);
+        if (e == cudaSuccess) e = pool_alloc(c, reinterpret_cast<void**>(&cache->pos), pos_bytes);
+        // One launch per group of at most kMaxOcc occurrences, all layers at once.
+        for (int32_t g0 = 0; e == cudaSuccess && g0 < n_occ; g0 += c2kv::kMaxOcc) {
+            c2kv::ComposeParams pr{};
+            pr.pool_k = c->pool_k;
+            pr.pool_v = c->pool_v;
+            pr.out_k = cache->k;
+            pr.out_v = cache->v;
+            pr.pos = cache->pos;
+            pr.err = c->d_err;
+            pr.pool_slots = c->cfg.pool_slots;
+            pr.rows = row;
+            pr.hkv = c->cfg.n_kv_heads;
+            pr.rope = c->turns;
+            int32_t tiles = 0;
+            const int32_t g1 = std::min(n_occ, g0 + c2kv::kMaxOcc);
+            for (int32_t i = g0; i < g1; ++i) {
+                if (occ[i].m == 0) continue;
+                c2kv::OccParam rec = occ[i];
+                rec.tile_base = tiles;
+                pr.occ[pr.n_occ++] = rec;
+                tiles += (rec.m + c2kv::kComposeTile - 1) / c2kv::kComposeTile;
+            }
+            pr.n_tiles = tiles;
+            e = c2kv::launch_compose(pr, c->cfg.dtype, c->cfg.head_dim, c->cfg.layers, c->stream);
+        }
+        if (e != cudaSuccess) {
+            destroy_cache(c, cache);
+            return cuda_fail(c, e, "compose");
+        }
+        c->caches.push_back(cache);
+        *out = cache;
+        return C2KV_OK;
+    } catch (const std::bad_alloc&) {
+        return fail(c, C2KV_ERR_NOMEM, "compose: host allocation failed");
+    }
+}
+
+c2kv_status c2kv_cache_info(const c2kv_cache* cache, c2kv_cache_desc* out) {
+    if (!cache || !out) return C2KV_ERR_ARG;
+    out->batch = cache->batch;
+    out->layers = cache->layers;
+    out->rows = cache->rows;
+    out->k = cache->k;
+    out->v = cache->v;
+    out->pos = cache->pos;
+    out->row_base = cache->row_base.data();
+    out->n_slots = cache->n_slots.data();
+    out->l_req = cache->l_req.data();
+    out->capacity = cache->capacity.data();
+    out->suffix_capacity = cache->suffix_capacity;
+    return C2KV_OK;
+}
+
+c2kv_status c2kv_attend(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const void* q,
+                        const void* k_suf, const void* v_suf, int32_t n_suffix, void* out,
+                        float* lse) {
+    if (!c) return C2KV_ERR_ARG;
+    try {
+        c->err.clear();
+        if (!own_cache(c, cache)) return fail(c, C2KV_ERR_STATE, "attend: cache not owned by this context");
+        if (!q || !k_suf || !v_suf || !out) return fail(c, C2KV_ERR_ARG, "attend: null pointer");
+        if (layer < -1 || layer >= c->cfg.layers) return fail(c, C2KV_ERR_ARG, "attend: bad layer %d", layer);
+        if (n_suffix < 1 || n_suffix > cache->suffix_capacity)
+            return fail(c, C2KV_ERR_ARG, "attend: n_suffix %d outside [1, %d]", n_suffix,
+                        cache->suffix_capacity);
+        const int32_t lq = layer < 0 ? c->cfg.layers : 1;
+        const int32_t layer0 = layer < 0 ? 0 : layer;
+        const int32_t B = cache->batch;
+        const bool use_tc =
+            c->cfg.attn_impl != C2KV_ATTN_SIMT &&
+            c2kv::attn_tc_supported(c->cfg.dtype, c->cfg.head_dim, c->cfg.n_q_heads, c->cfg.n_kv_heads);
+
+        // scratch: the suffix queries after RoPE (the attention kernels' Q operand)
+        const size_t q_bytes =
+            (size_t)lq * B * n_suffix * c->cfg.n_q_heads * c->cfg.head_dim * c->eb;
+        void* q_rot = nullptr;
+        cudaError_t e = pool_alloc(c, &q_rot, q_bytes);
+        if (e != cudaSuccess) return cuda_fail(c, e, "attend: scratch allocation");
+        for (int32_t b0 = 0; e == cudaSuccess && b0 < B; b0 += c2kv::kMaxReq) {
+            const int32_t nb = std::min<int32_t>(c2kv::kMaxReq, B - b0);
+            c2kv::SuffixParams s{};
+            s.q = q;
+            s.k = k_suf;
+            s.v = v_suf;
+            s.q_rot = q_rot;
+            s.cache_k = cache->k;
+            s.cache_v = cache->v;
+            s.pos = cache->pos;
+            s.rows = cache->rows;
+            s.layer0 = layer0;
+            s.lq = lq;
+            s.batch = nb;
+            s.batch_total = B;
+            s.b0 = b0;
+            s.sq = n_suffix;
+            s.hq = c->cfg.n_q_heads;
+            s.hkv = c->cfg.n_kv_heads;
+            s.rope = c->turns;
+            for (int32_t i = 0; i < nb; ++i)
+                s.req[i] = c2kv::ReqParam{cache->row_base[b0 + i], cache->n_slots[b0 + i],
+                                          cache->l_req[b0 + i], 0};
+            e = c2kv::launch_suffix_prep(s, c->cfg.dtype, c->cfg.head_dim, c->stream);
+            if (e != cudaSuccess) break;
+            c2kv::AttnParams a{};
+            a.q_rot = q_rot;
+            a.cache_k = cache->k;
+            a.cache_v = cache->v;
+            a.out = out;
+            a.lse = lse;
+            a.rows = cache->rows;
+            a.layer0 = layer0;
+            a.lq = lq;
+            a.batch = nb;
+            a.batch_total = B;
+            a.b0 = b0;
+            a.sq = n_suffix;
+            a.hq = c->cfg.n_q_heads;
+            a.hkv = c->cfg.n_kv_heads;
+            a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)c->cfg.head_dim));
+            for (int32_t i = 0; i < nb; ++i) a.req[i] = s.req[i];
+            e = use_tc ? c2kv::launch_attn_tc(a, c->stream)
+                       : c2kv::launch_attn_simt(a, c->cfg.dtype, c->cfg.head_dim, c->stream);
+        }
+        pool_free(c, q_rot);
+        if (e != cudaSuccess) return cuda_fail(c, e, "attend");
+        return C2KV_OK;
+    } catch (const std::bad_alloc&) {
+        return fail(c, C2KV_ERR_NOMEM, "attend: host allocation failed");
+    }
+}
+
+c2kv_status c2kv_cache_release(c2kv_ctx* c, c2kv_cache* cache) {
+    if (!c) return C2KV_ERR_ARG;
+    c->err.clear();
+    if (!own_cache(c, cache)) return fail(c, C2KV_ERR_STATE, "cache_release: cache not owned by this context");
+    c->caches.erase(std::find(c->caches.begin(), c->caches.end(), cache));
+    destroy_cache(c, cache);
+    return C2KV_OK;
+}
+
+c2kv_status c2kv_sync(c2kv_ctx* c) {
+    if (!c) return C2KV_ERR_ARG;
+    c->err.clear();
+    cudaError_t e = cudaStreamSynchronize(c->stream);
+    if (e != cudaSuccess) return cuda_fail(c, e, "sync");
+    int32_t word = 0;
+    e = cudaMemcpy(&word, c->d_err, sizeof(word), cudaMemcpyDeviceToHost);
+    if (e != cudaSuccess) return cuda_fail(c, e, "sync: error word");
+    if (word != 0) {
+        cudaMemset(c->d_err, 0, sizeof(int32_t));
+        return fail(c, C2KV_ERR_DEVICE_BOUNDS, "sync: a kernel refused an out-of-range index (flags 0x%x)", word);
+    }
+    return C2KV_OK;
+}
+
+c2kv_status c2kv_inject_fault(c2kv_ctx* c, int32_t what) {
+    if (!c) return C2KV_ERR_ARG;
+    if (what < 0 || what > 1) return fail(c, C2KV_ERR_ARG, "inject_fault: unknown fault %d", what);
+    c->inject = what;
+    return C2KV_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,133 @@
+// Internal declarations shared by the C2KV library's translation units (not installed).
+//
+// Per-call metadata (chunk occurrences, per-request row layout, RoPE frequencies) travels
+// inside the kernel parameter block, so compose and attend need no host-to-device copy
+// and no device-side metadata buffer.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <cuda_bf16.h>
+#include <stdint.h>
+
+namespace c2kv {
+
+constexpr int kDtypeBf16 = 0;
+constexpr int kDtypeF32 = 1;
+constexpr int kMaxHalf = 64;        // head_dim / 2 for head_dim <= 128
+constexpr int kMaxOcc = 128;        // chunk occurrences per compose launch
+constexpr int kMaxReq = 256;        // requests per suffix / attention launch
+constexpr int kComposeTile = 16;    // composed slots per compose CTA (per layer)
+
+// RoPE frequency i as a fraction of a full turn in 0.64 fixed point:
+// turn[i] = round(theta^(-2i/d) / (2 pi) * 2^64).  For an integer position p the angle in
+// turns is the low 64 bits of p * turn[i] (a phase accumulator: wrap-around is the
+// reduction modulo 2 pi, exact in integers), so no large float angle is ever formed.
+struct RopeTurns {
+    uint64_t turn[kMaxHalf];
+};
+
+// One chunk occurrence of a compose launch.
+struct OccParam {
+    int32_t src_base;    // first pool slot of the chunk
+    int32_t dest_row;    // first composed row
+    int32_t delta;       // positions to turn by (o_i, or 0 under fixed_pos)
+    int32_t n;           // original chunk length
+    int32_t k;           // ratio
+    int32_t m;           // slots
+    int32_t tile_base;   // first compose tile of this occurrence (prefix over the launch)
+    int32_t pad;
+};
+
+struct ComposeParams {
+    const void* pool_k;      // [L][pool_slots][Hkv][d]
+    const void* pool_v;
+    void* out_k;             // [L][rows][Hkv][d]
+    void* out_v;
+    int32_t* pos;            // [rows]
+    int32_t* err;            // device error word: bit 0 = index refused
+    int64_t pool_slots;
+    int64_t rows;
+    int32_t n_occ;
+    int32_t n_tiles;
+    int32_t hkv;
+    int32_t pad;
+    RopeTurns rope;
+    OccParam occ[kMaxOcc];
+};
+
+struct CompressParams {
+    const void* in_k;        // [L][rows_in][Hkv][d]
+    const void* in_v;
+    void* pool_k;            // [L][pool_slots][Hkv][d]
+    void* pool_v;
+    int64_t pool_slots;
+    int32_t slot_base;
+    int32_t m;               // slots
+    int32_t n;               // tokens
+    int32_t k;               // ratio
+    int32_t rows_in;         // n (meanpool) or m (provided)
+    int32_t one_row;         // 1 = provided (slot j is input row j); 0 = block mean
+    int32_t layers;
+    int32_t hkv;
+    RopeTurns rope;
+};
+
+struct ReqParam {
+    int32_t row_base;        // first cache row of the request
+    int32_t n_slots;         // composed slots S_r
+    int32_t l_req;           // composed span L_r (suffix token t sits at L_r + t)
+    int32_t pad;
+};
+
+struct SuffixParams {
+    const void* q;           // [Lq][B][Sq][Hq][d]   (B = this launch's requests)
+    const void* k;           // [Lq][B][Sq][Hkv][d]
+    const void* v;
+    void* q_rot;             // [Lq][B][Sq][Hq][d]
+    void* cache_k;           // [L][rows][Hkv][d]
+    void* cache_v;
+    int32_t* pos;            // [rows]
+    int64_t rows;
+    int32_t layer0;          // first cache layer touched
+    int32_t lq;              // layers in this call
+    int32_t batch;           // requests in this launch
+    int32_t batch_total;     // requests in the q / out tensors
+    int32_t b0;              // first request of this launch
+    int32_t sq;
+    int32_t hq;
+    int32_t hkv;
+    RopeTurns rope;
+    ReqParam req[kMaxReq];
+};
+
+struct AttnParams {
+    const void* q_rot;       // [Lq][Btot][Sq][Hq][d]
+    const void* cache_k;     // [L][rows][Hkv][d]
+    const void* cache_v;
+    void* out;               // [Lq][Btot][Sq][Hq][d]
+    float* lse;              // [Lq][Btot][Hq][Sq] or null
+    int64_t rows;
+    int32_t layer0;
+    int32_t lq;
+    int32_t batch;
+    int32_t batch_total;
+    int32_t b0;
+    int32_t sq;
+    int32_t hq;
+    int32_t hkv;
+    float scale_log2;        // log2(e) / sqrt(d)
+    int32_t pad;
+    ReqParam req[kMaxReq];
+};
+
+// Launchers: return the launch error, never throw.  `d` is head_dim.
+cudaError_t launch_compose(const ComposeParams& p, int dtype, int d, int layers, cudaStream_t s);
+cudaError_t launch_compress(const CompressParams& p, int dtype, int d, cudaStream_t s);
+cudaError_t launch_suffix_prep(const SuffixParams& p, int dtype, int d, cudaStream_t s);
+cudaError_t launch_attn_simt(const AttnParams& p, int dtype, int d, cudaStream_t s);
+
+// Tensor-core attention (attn_tc.cu).
+bool attn_tc_supported(int dtype, int d, int hq, int hkv);
+cudaError_t launch_attn_tc(const AttnParams& p, cudaStream_t s);
+
+}  // namespace c2kv

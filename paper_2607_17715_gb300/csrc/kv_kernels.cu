@@ -1,0 +1,393 @@
+// Streaming KV kernels of the C2KV hot path: compose (re-rotate + gather), compress (block
+// mean + local RoPE), suffix preparation.  All are HBM-bound element-wise moves: each
+// thread moves 16-byte vectors, and one thread owns a RoPE pair of vectors (channels
+// [c, c+E) and [c + d/2, c + d/2 + E)) so the 2x2 rotation needs no exchange between
+// threads.
+//
+// Angles: cos/sin of p * theta^(-2i/d) come from the phase accumulator in RopeTurns (the
+// turn fraction is the low 64 bits of p * turn[i], exact integer wrap-around), converted
+// once to a float in [-1/2, 1/2) turns and handed to sincospif.  The error is about
+// 1e-7 rad at any position, where forming p * inv_freq in fp32 would lose p * 2^-24 rad.
+#include "internal.cuh"
+
+namespace c2kv {
+namespace {
+
+template <typename T>
+struct Vec16;
+
+template <>
+struct Vec16<__nv_bfloat16> {
+    static constexpr int N = 8;
+    __device__ __forceinline__ static void unpack(const uint4& r, float* f) {
+        const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&r);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            float2 t = __bfloat1622float2(h[i]);
+            f[2 * i] = t.x;
+            f[2 * i + 1] = t.y;
+        }
+    }
+    __device__ __forceinline__ static uint4 pack(const float* f) {
+        uint4 r;
+        __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&r);
+#pragma unroll
+        for (int i = 0; i < 4; ++i) h[i] = __floats2bfloat162_rn(f[2 * i], f[2 * i + 1]);
+        return r;
+    }
+};
+
+template <>
+struct Vec16<float> {
+    static constexpr int N = 4;
+    __device__ __forceinline__ static void unpack(const uint4& r, float* f) {
+        f[0] = __uint_as_float(r.x);
+        f[1] = __uint_as_float(r.y);
+        f[2] = __uint_as_float(r.z);
+        f[3] = __uint_as_float(r.w);
+    }
+    __device__ __forceinline__ static uint4 pack(const float* f) {
+        return make_uint4(__float_as_uint(f[0]), __float_as_uint(f[1]), __float_as_uint(f[2]),
+                          __float_as_uint(f[3]));
+    }
+};
+
+__device__ __forceinline__ uint4 ld16(const void* p) {
+    return __ldg(reinterpret_cast<const uint4*>(p));
+}
+__device__ __forceinline__ void st16(void* p, const uint4& v) {
+    *reinterpret_cast<uint4*>(p) = v;
+}
+
+// (cos, sin) of pos * theta^(-2i/d) from the 0.64 fixed-point turn of frequency i.
+__device__ __forceinline__ float2 turn_cs(uint64_t turn, int64_t pos) {
+    const uint64_t frac = (uint64_t)pos * turn;                 // turns mod 1, exact
+    const float x = (float)(long long)frac * 0x1p-63f;          // 2 * turns in [-1, 1)
+    float s, c;
+    sincospif(x, &s, &c);
+    return make_float2(c, s);
+}
+
+template <int E>
+__device__ __forceinline__ void rotate(const float* x, const float* y, const float2* cs,
+                                       float* ox, float* oy) {
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+        ox[e] = x[e] * cs[e].x - y[e] * cs[e].y;
+        oy[e] = x[e] * cs[e].y + y[e] * cs[e].x;
+    }
+}
+
+// ---------------------------------------------------------------------------------------
+// compose.  grid = (tiles, layers); a tile is kComposeTile consecutive slots of one chunk
+// occurrence.  The CTA forms the occurrence's d/2 (cos, sin) of delta once in shared
+// memory, then streams the tile: per item (slot, head, vector pair) four 16-byte loads of
+// stored K/V, K turned, four 16-byte stores into the composed cache.  IPT items per
+// thread are loaded before any is stored, so 16 loads per thread are in flight.
+// ---------------------------------------------------------------------------------------
+template <typename T, int VPH>
+__global__ void __launch_bounds__(256) compose_kernel(const __grid_constant__ ComposeParams P) {
+    using V = Vec16<T>;
+    constexpr int E = V::N;
+    constexpr int HALF = VPH * E;
+    constexpr int D = 2 * HALF;
+    constexpr int IPT = 4;
+    __shared__ float2 cs[HALF];
+
+    const int tile = blockIdx.x;
+    const int l = blockIdx.y;
+    int lo = 0, hi = P.n_occ - 1;
+    while (lo < hi) {                       // last occurrence whose tile_base <= tile
+        const int mid = (lo + hi + 1) >> 1;
+        if (P.occ[mid].tile_base <= tile) lo = mid;
+        else hi = mid - 1;
+    }
+    const OccParam& o = P.occ[lo];
+    const int j0 = (tile - o.tile_base) * kComposeTile;
+    const int ns = min(kComposeTile, o.m - j0);
+    if (threadIdx.x < HALF) cs[threadIdx.x] = turn_cs(P.rope.turn[threadIdx.x], o.delta);
+    __syncthreads();
+    if (ns <= 0) return;
+
+    const T* __restrict__ pk = static_cast<const T*>(P.pool_k);
+    const T* __restrict__ pv = static_cast<const T*>(P.pool_v);
+    T* __restrict__ ok = static_cast<T*>(P.out_k);
+    T* __restrict__ ov = static_cast<T*>(P.out_v);
+    const int pairs = P.hkv * VPH;
+    const int items = ns * pairs;
+    const int64_t row_elems = (int64_t)P.hkv * D;
+
+    for (int base = 0; base < items; base += 256 * IPT) {
+        uint4 kx[IPT], ky[IPT], vx[IPT], vy[IPT];
+        int64_t dof[IPT];
+        int civ[IPT];
+        bool live[IPT];
+#pragma unroll
+        for (int u = 0; u < IPT; ++u) {
+            const int it = base + u * 256 + (int)threadIdx.x;
+            live[u] = it < items;
+            if (!live[u]) continue;
+            const int s = it / pairs;
+            const int p = it - s * pairs;
+            const int h = p / VPH;
+            const int iv = p - h * VPH;
+            const int j = j0 + s;
+            const int64_t src = (int64_t)o.src_base + j;
+            const int64_t dst = (int64_t)o.dest_row + j;
+            if (src < 0 || src >= P.pool_slots || dst < 0 || dst >= P.rows) {
+                atomicOr(P.err, 1);
+                live[u] = false;
+                continue;
+            }
+            const int64_t so = ((int64_t)l * P.pool_slots + src) * row_elems + h * D + iv * E;
+            dof[u] = ((int64_t)l * P.rows + dst) * row_elems + h * D + iv * E;
+            civ[u] = iv * E;
+            kx[u] = ld16(pk + so);
+            ky[u] = ld16(pk + so + HALF);
+            vx[u] = ld16(pv + so);
+            vy[u] = ld16(pv + so + HALF);
+            if (l == 0 && p == 0) P.pos[dst] = o.delta + min((j + 1) * o.k, o.n) - 1;
+        }
+#pragma unroll
+        for (int u = 0; u < IPT; ++u) {
+            if (!live[u]) continue;
+            float fx[E], fy[E], gx[E], gy[E];
+            V::unpack(kx[u], fx);
+            V::unpack(ky[u], fy);
+            rotate<E>(fx, fy, cs + civ[u], gx, gy);
+            st16(ok + dof[u], V::pack(gx));
+            st16(ok + dof[u] + HALF, V::pack(gy));
+            st16(ov + dof[u], vx[u]);
+            st16(ov + dof[u] + HALF, vy[u]);
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------------------
+// compress: one item = (layer, slot, head, vector pair).  Mean of the block's rows (or the
+// provided slot row), K turned to the slot's local position, both stored in the pool.
+// ---------------------------------------------------------------------------------------
+template <typename T, int VPH>
+__global__ void __launch_bounds__(256) compress_kernel(const __grid_constant__ CompressParams P) {
+    using V = Vec16<T>;
+    constexpr int E = V::N;
+    constexpr int HALF = VPH * E;
+    constexpr int D = 2 * HALF;
+    const int pairs = P.hkv * VPH;
+    const int64_t per_layer = (int64_t)P.m * pairs;
+    const int64_t total = per_layer * P.layers;
+    const int64_t row_elems = (int64_t)P.hkv * D;
+    const T* ik = static_cast<const T*>(P.in_k);
+    const T* iv_ = static_cast<const T*>(P.in_v);
+    T* pk = static_cast<T*>(P.pool_k);
+    T* pv = static_cast<T*>(P.pool_v);
+    for (int64_t it = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; it < total;
+         it += (int64_t)gridDim.x * blockDim.x) {
+        const int l = (int)(it / per_layer);
+        const int64_t r = it - (int64_t)l * per_layer;
+        const int j = (int)(r / pairs);
+        const int p = (int)(r - (int64_t)j * pairs);
+        const int h = p / VPH;
+        const int iv = p - h * VPH;
+        int r0, r1;
+        if (P.one_row) {
+            r0 = j;
+            r1 = j + 1;
+        } else {
+            r0 = j * P.k;
+            r1 = min(r0 + P.k, P.n);
+        }
+        float sx[E], sy[E], tx[E], ty[E];
+#pragma unroll
+        for (int e = 0; e < E; ++e) sx[e] = sy[e] = tx[e] = ty[e] = 0.f;
+        for (int row = r0; row < r1; ++row) {
+            const int64_t off = ((int64_t)l * P.rows_in + row) * row_elems + h * D + iv * E;
+            float f[E];
+            V::unpack(ld16(ik + off), f);
+#pragma unroll
+            for (int e = 0; e < E; ++e) sx[e] += f[e];
+            V::unpack(ld16(ik + off + HALF), f);
+#pragma unroll
+            for (int e = 0; e < E; ++e) sy[e] += f[e];
+            V::unpack(ld16(iv_ + off), f);
+#pragma unroll
+            for (int e = 0; e < E; ++e) tx[e] += f[e];
+            V::unpack(ld16(iv_ + off + HALF), f);
+#pragma unroll
+            for (int e = 0; e < E; ++e) ty[e] += f[e];
+        }
+        const int cnt = r1 - r0;
+        if (cnt > 1) {
+            const float c = (float)cnt;
+#pragma unroll
+            for (int e = 0; e < E; ++e) {
+                sx[e] = sx[e] / c;
+                sy[e] = sy[e] / c;
+                tx[e] = tx[e] / c;
+                ty[e] = ty[e] / c;
+            }
+        }
+        // slot j sits at the last token of its block (provided slots: same rule)
+        const int64_t p_local = (int64_t)min((j + 1) * P.k, P.n) - 1;
+        float2 cs[E];
+#pragma unroll
+        for (int e = 0; e < E; ++e) cs[e] = turn_cs(P.rope.turn[iv * E + e], p_local);
+        float gx[E], gy[E];
+        rotate<E>(sx, sy, cs, gx, gy);
+        const int64_t dof =
+            ((int64_t)l * P.pool_slots + P.slot_base + j) * row_elems + h * D + iv * E;
+        st16(pk + dof, V::pack(gx));
+        st16(pk + dof + HALF, V::pack(gy));
+        st16(pv + dof, V::pack(tx));
+        st16(pv + dof + HALF, V::pack(ty));
+    }
+}
+
+// ---------------------------------------------------------------------------------------
+// suffix preparation.  Items per suffix row (layer, request, token): Hq query-head pairs
+// (RoPE at L_b + t into q_rot) then Hkv key-head pairs (RoPE into the cache row
+// row_base + S_b + t, V copied alongside, position recorded).
+// ---------------------------------------------------------------------------------------
+template <typename T, int VPH>
+__global__ void __launch_bounds__(256) suffix_kernel(const __grid_constant__ SuffixParams P) {
+    using V = Vec16<T>;
+    constexpr int E = V::N;
+    constexpr int HALF = VPH * E;
+    constexpr int D = 2 * HALF;
+    const int per_row = (P.hq + P.hkv) * VPH;
+    const int64_t n_rows = (int64_t)P.lq * P.batch * P.sq;
+    const int64_t total = n_rows * per_row;
+    for (int64_t it = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; it < total;
+         it += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t row = it / per_row;           // ((l * batch) + bl) * Sq + t
+        const int p = (int)(it - row * per_row);
+        const int t = (int)(row % P.sq);
+        const int64_t lb = row / P.sq;
+        const int bl = (int)(lb % P.batch);
+        const int l = (int)(lb / P.batch);
+        const ReqParam& rq = P.req[bl];
+        const int64_t grow = ((int64_t)l * P.batch_total + P.b0 + bl) * P.sq + t;  // tensor row
+        const int64_t position = (int64_t)rq.l_req + t;
+        const bool is_q = p < P.hq * VPH;
+        const int pp = is_q ? p : p - P.hq * VPH;
+        const int h = pp / VPH;
+        const int iv = pp - h * VPH;
+        float2 cs[E];
+#pragma unroll
+        for (int e = 0; e < E; ++e) cs[e] = turn_cs(P.rope.turn[iv * E + e], position);
+        float x[E], y[E], gx[E], gy[E];
+        if (is_q) {
+            const int64_t off = (grow * P.hq + h) * D + iv * E;
+            const T* src = static_cast<const T*>(P.q) + off;
+            V::unpack(ld16(src), x);
+            V::unpack(ld16(src + HALF), y);
+            rotate<E>(x, y, cs, gx, gy);
+            T* dst = static_cast<T*>(P.q_rot) + off;
+            st16(dst, V::pack(gx));
+            st16(dst + HALF, V::pack(gy));
+        } else {
+            const int64_t off = (grow * P.hkv + h) * D + iv * E;
+            const int64_t crow = (int64_t)rq.row_base + rq.n_slots + t;
+            if (crow < 0 || crow >= P.rows) continue;
+            const int64_t coff = (((int64_t)(P.layer0 + l) * P.rows + crow) * P.hkv + h) * D + iv * E;
+            const T* ks = static_cast<const T*>(P.k) + off;
+            const T* vs = static_cast<const T*>(P.v) + off;
+            V::unpack(ld16(ks), x);
+            V::unpack(ld16(ks + HALF), y);
+            rotate<E>(x, y, cs, gx, gy);
+            T* kd = static_cast<T*>(P.cache_k) + coff;
+            T* vd = static_cast<T*>(P.cache_v) + coff;
+            st16(kd, V::pack(gx));
+            st16(kd + HALF, V::pack(gy));
+            st16(vd, ld16(vs));
+            st16(vd + HALF, ld16(vs + HALF));
+            if (l == 0 && pp == 0) P.pos[crow] = (int32_t)position;
+        }
+    }
+}
+
+// Zero the cache rows between the end of the suffix and the next 128-row boundary, so a
+// key tile that straddles the end reads finite zeros (masked keys must not carry NaN/Inf
+// garbage into P.V).
+template <typename T>
+__global__ void __launch_bounds__(256) pad_zero_kernel(const __grid_constant__ SuffixParams P, int d) {
+    const int vec_per_row = P.hkv * d * (int)sizeof(T) / 16;
+    const int64_t total = (int64_t)P.lq * P.batch * 128 * vec_per_row;
+    for (int64_t it = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; it < total;
+         it += (int64_t)gridDim.x * blockDim.x) {
+        const int vi = (int)(it % vec_per_row);
+        const int64_t r = it / vec_per_row;
+        const int rr = (int)(r % 128);
+        const int64_t lb = r / 128;
+        const int bl = (int)(lb % P.batch);
+        const int l = (int)(lb / P.batch);
+        const int used = P.req[bl].n_slots + P.sq;
+        const int end = (used + 127) / 128 * 128;
+        const int row = used + rr;
+        if (row >= end) continue;
+        const int64_t crow = (int64_t)P.req[bl].row_base + row;
+        if (crow >= P.rows) continue;
+        const int64_t off = ((int64_t)(P.layer0 + l) * P.rows + crow) * P.hkv * d;
+        const uint4 z = make_uint4(0, 0, 0, 0);
+        st16(static_cast<T*>(P.cache_k) + off + vi * (16 / (int)sizeof(T)), z);
+        st16(static_cast<T*>(P.cache_v) + off + vi * (16 / (int)sizeof(T)), z);
+    }
+}
+
+int sm_count() {
+    int dev = 0, sms = 148;
+    if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    return sms;
+}
+
+int grid_for(int64_t items, int threads) {
+    const int64_t want = (items + threads - 1) / threads;
+    const int64_t cap = (int64_t)sm_count() * 8;   // grid-stride beyond 8 CTAs per SM
+    return (int)(want < 1 ? 1 : (want > cap ? cap : want));
+}
+
+int vph_of(int dtype, int d) { return d / 2 / (dtype == kDtypeBf16 ? 8 : 4); }
+
+}  // namespace
+
+// KERNEL<element type, vectors per half head> for the supported (dtype, head_dim).
+#define C2KV_DISPATCH(KERNEL, GRID, PARAMS, DTYPE, D, STREAM)                                  \
+    do {                                                                                       \
+        if ((DTYPE) == kDtypeBf16 && (D) == 128) KERNEL<__nv_bfloat16, 8><<<GRID, 256, 0, STREAM>>>(PARAMS); \
+        else if ((DTYPE) == kDtypeBf16 && (D) == 64) KERNEL<__nv_bfloat16, 4><<<GRID, 256, 0, STREAM>>>(PARAMS); \
+        else if ((DTYPE) == kDtypeF32 && (D) == 128) KERNEL<float, 16><<<GRID, 256, 0, STREAM>>>(PARAMS); \
+        else if ((DTYPE) == kDtypeF32 && (D) == 64) KERNEL<float, 8><<<GRID, 256, 0, STREAM>>>(PARAMS); \
+        else return cudaErrorInvalidValue;                                                     \
+    } while (0)
+
+cudaError_t launch_compose(const ComposeParams& p, int dtype, int d, int layers, cudaStream_t s) {
+    if (p.n_tiles == 0 || p.n_occ == 0) return cudaSuccess;
+    if (layers > 65535) return cudaErrorInvalidValue;
+    const dim3 grid(p.n_tiles, layers);
+    C2KV_DISPATCH(compose_kernel, grid, p, dtype, d, s);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_compress(const CompressParams& p, int dtype, int d, cudaStream_t s) {
+    if (p.m == 0) return cudaSuccess;
+    const int64_t items = (int64_t)p.m * p.layers * p.hkv * vph_of(dtype, d);
+    const int g = grid_for(items, 256);
+    C2KV_DISPATCH(compress_kernel, g, p, dtype, d, s);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_suffix_prep(const SuffixParams& p, int dtype, int d, cudaStream_t s) {
+    const int64_t items = (int64_t)p.lq * p.batch * p.sq * (p.hq + p.hkv) * vph_of(dtype, d);
+    const int g = grid_for(items, 256);
+    C2KV_DISPATCH(suffix_kernel, g, p, dtype, d, s);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const int eb = dtype == kDtypeBf16 ? 2 : 4;
+    const int64_t pad_items = (int64_t)p.lq * p.batch * 128 * (p.hkv * d * eb / 16);
+    const int gp = grid_for(pad_items, 256);
+    if (dtype == kDtypeBf16) pad_zero_kernel<__nv_bfloat16><<<gp, 256, 0, s>>>(p, d);
+    else pad_zero_kernel<float><<<gp, 256, 0, s>>>(p, d);
+    return cudaGetLastError();
+}
+
+}  // namespace c2kv
