@@ -149,6 +149,7 @@ __global__ void __launch_bounds__(NW * 32) attn_simt_kernel(const __grid_constan
 }  // namespace
 
 cudaError_t launch_attn_simt(const AttnParams& a, int dtype, int d, cudaStream_t s) {
+    (void)cudaGetLastError();   // report this launch's error only, not a stale one
     const int G = a.hq / a.hkv;
     dim3 grid((a.sq * G + RB - 1) / RB, a.hkv, a.lq * a.batch);
     if (grid.z > 65535u) return cudaErrorInvalidValue;

@@ -1,10 +1,548 @@
-// Tensor-core (tcgen05 / TMEM) attention over [composed cache; suffix]: not built yet.
+// Tensor-core attention over [composed cache; suffix] for sm_103a: tcgen05.mma with TMEM
+// accumulators, operands staged by TMA in 128-byte-swizzled shared memory.
+//
+// Work unit (one CTA): 128 packed query rows of one (layer, request, KV head).  Row
+// m = t * G + g is suffix token t0 + t, query head h_kv * G + g (G = Hq / Hkv), so the
+// G query heads that share a KV head form the M dimension of one MMA and every K/V tile
+// is fetched once for all of them.  The CTA walks the request's key tiles of 128 rows
+// (composed slots first, then its own suffix rows); only the tiles past S_r + t0 need
+// the causal mask.
+//
+// Warp roles (192 threads):
+//   warp 0      TMA producer: Q once, then K and V tiles into a 2-stage ring.
+//   warp 1      MMA issuer (one lane) and TMEM owner:  S_j = Q K_j^T into one of two
+//               TMEM S buffers, then O += P_{j-1} V_{j-1} into the TMEM O accumulator.
+//   warps 2..5  softmax / correction / epilogue: thread i owns TMEM lane (row) i.  Reads
+//               S_j, masks, keeps the running max and sum, writes P_j (bf16) into shared
+//               memory in the MMA's 128B-swizzled K-major layout, rescales O in TMEM only
+//               when its row max grew by more than 2^8 (otherwise the stale reference max
+//               is kept: the normaliser uses the same one, so the result is exact).
+//
+// Every mbarrier wait is bounded (kWaitCycles); on expiry the waiting thread sets bit 1
+// of the error word and carries on, so the kernel always terminates and the host reports
+// C2KV_ERR_DEVICE_BOUNDS at the next c2kv_sync.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <math_constants.h>
+
+#include <cstring>
+
 #include "internal.cuh"
 
 namespace c2kv {
+namespace {
 
-bool attn_tc_supported(int, int, int, int) { return false; }
+constexpr int BM = 128;                 // query rows per CTA (MMA M)
+constexpr int BN = 128;                 // keys per tile (MMA N of S, K of P.V)
+constexpr int HD = 128;                 // head dim
+constexpr int STAGES = 2;
+constexpr int TILE = BN * HD * 2;       // bytes of one 128 x 128 bf16 tile (32 KB)
+constexpr int HALF_TILE = TILE / 2;     // one 128-byte-wide swizzle column block
+constexpr int kThreads = 192;
+constexpr uint32_t kTmemCols = 512;     // S0 [0,128) S1 [128,256) O [256,384)
+constexpr uint32_t kColS = 0, kColO = 256;
+constexpr long long kWaitCycles = 4000000000LL;
 
-cudaError_t launch_attn_tc(const AttnParams&, cudaStream_t) { return cudaErrorNotSupported; }
+// barrier slots
+constexpr int B_Q = 0;
+constexpr int B_KF = 1;                  // + stage
+constexpr int B_VF = B_KF + STAGES;      // + stage
+constexpr int B_KVE = B_VF + STAGES;     // + stage: K and V stage free again
+constexpr int B_SF = B_KVE + STAGES;     // + buffer: S ready in TMEM
+constexpr int B_SFREE = B_SF + 2;        // + buffer: S read out by the softmax warps
+constexpr int B_PF = B_SFREE + 2;        // P written (and O corrected)
+constexpr int B_PVD = B_PF + 1;          // P.V finished (P buffer free, O current)
+constexpr int NBAR = B_PVD + 1;
+
+constexpr size_t kSmemBytes = 1024 /*align*/ + (size_t)TILE * (2 + 2 * STAGES) + 8 * NBAR + 16;
+
+struct alignas(64) TcParams {
+    CUtensorMap tm_q;        // q_rot   [Lq*Btot][Sq][Hq][128]  box {64, G, TQ, 1}
+    CUtensorMap tm_k;        // cache K [L*rows][Hkv][128]      box {64, 1, 128}
+    CUtensorMap tm_v;        // cache V, same
+    void* out;
+    float* lse;
+    int32_t* err;
+    int64_t rows;
+    int32_t layer0, lq, batch, batch_total, b0, sq, hq, hkv, group, tq;
+    float scale_log2;
+    int32_t pad;
+    ReqParam req[kMaxReq];
+};
+
+// ------------------------------------------------------------------ PTX wrappers
+
+__device__ __forceinline__ uint32_t smem_u32(const void* p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Bounded wait for the phase with the given parity to complete.
+__device__ __forceinline__ void mbar_wait(uint32_t bar, uint32_t parity, int32_t* err) {
+    if (mbar_try(bar, parity)) return;
+    const long long t0 = clock64();
+    while (!mbar_try(bar, parity)) {
+        if (clock64() - t0 > kWaitCycles) {
+            atomicOr(err, 2);
+            return;
+        }
+    }
+}
+
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* tm, int c0, int c1,
+                                            int c2, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(c2), "r"(bar)
+        : "memory");
+}
+
+__device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap* tm, int c0, int c1,
+                                            int c2, int c3, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(dst),
+        "l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(bar)
+        : "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() {
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// Shared-memory matrix descriptor, 128-byte swizzle (layout type 2), sm_100 version bit.
+// K-major operands: SBO = 1024 (8 rows of 128 B); LBO unused.  MN-major operands: LBO =
+// byte distance between 64-element column blocks, SBO = between 8-row K groups.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);
+    d |= (uint64_t)((lbo >> 4) & 0x3FFFu) << 16;
+    d |= (uint64_t)((sbo >> 4) & 0x3FFFu) << 32;
+    d |= (uint64_t)1 << 46;
+    d |= (uint64_t)2 << 61;
+    return d;
+}
+
+// Instruction descriptor, kind::f16: D fp32, A and B bf16, A K-major, B K- or MN-major.
+__host__ __device__ constexpr uint32_t idesc_bf16(int m, int n, bool b_mn_major) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((b_mn_major ? 1u : 0u) << 16) |
+           ((uint32_t)(n >> 3) << 17) | ((uint32_t)(m >> 4) << 24);
+}
+
+__device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b, uint32_t idesc,
+                                         uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(a), "l"(b), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+        : "memory");
+}
+
+// 32 consecutive TMEM columns of this thread's lane -> 32 registers.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, "
+        "%16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),
+          "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]),
+          "=r"(v[13]), "=r"(v[14]), "=r"(v[15]), "=r"(v[16]), "=r"(v[17]), "=r"(v[18]),
+          "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]), "=r"(v[24]),
+          "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]),
+          "=r"(v[31])
+        : "r"(taddr));
+}
+
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&v)[32]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
+        "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, "
+        "%17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(taddr),
+        "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
+        "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]),
+        "r"(v[15]), "r"(v[16]), "r"(v[17]), "r"(v[18]), "r"(v[19]), "r"(v[20]), "r"(v[21]),
+        "r"(v[22]), "r"(v[23]), "r"(v[24]), "r"(v[25]), "r"(v[26]), "r"(v[27]), "r"(v[28]),
+        "r"(v[29]), "r"(v[30]), "r"(v[31])
+        : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld_wait() {
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_st_wait() {
+    asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
+    __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<uint32_t*>(&v);
+}
+
+__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c,
+                                             uint32_t d) {
+    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c),
+                 "r"(d)
+                 : "memory");
+}
+
+// ------------------------------------------------------------------ kernel
+
+__global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_constant__ TcParams P) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                               ~uintptr_t(1023));
+    const uint32_t sQ = smem_u32(smem);
+    const uint32_t sK = sQ + TILE;
+    const uint32_t sV = sK + STAGES * TILE;
+    const uint32_t sP = sV + STAGES * TILE;
+    const uint32_t sBar = sP + TILE;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + (size_t)TILE * (2 + 2 * STAGES) + 8 * NBAR);
+    auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
+
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const int G = P.group;
+    const int hk = blockIdx.y;
+    const int l = blockIdx.z / P.batch;
+    const int bl = blockIdx.z - l * P.batch;
+    const int b = P.b0 + bl;
+    const int s_r = P.req[bl].n_slots;
+    const int t0 = blockIdx.x * P.tq;
+    const int t_last = min(P.sq - 1, t0 + P.tq - 1);
+    const int n_kv = (s_r + t_last + 1 + BN - 1) / BN;
+
+    if (threadIdx.x == 0) {
+        mbar_init(bar(B_Q), 1);
+        for (int s = 0; s < STAGES; ++s) {
+            mbar_init(bar(B_KF + s), 1);
+            mbar_init(bar(B_VF + s), 1);
+            mbar_init(bar(B_KVE + s), 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(bar(B_SF + i), 1);
+            mbar_init(bar(B_SFREE + i), 128);
+        }
+        mbar_init(bar(B_PF), 128);
+        mbar_init(bar(B_PVD), 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         smem_u32(tmem_slot)),
+                     "r"(kTmemCols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = *tmem_slot;
+
+    if (warp == 0) {
+        // ---------------------------------------------------------------- TMA producer
+        if (lane == 0) {
+            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&P.tm_q)) : "memory");
+            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&P.tm_k)) : "memory");
+            asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&P.tm_v)) : "memory");
+            const int qz = l * P.batch_total + b;
+            mbar_expect_tx(bar(B_Q), TILE);
+            tma_load_4d(sQ, &P.tm_q, 0, hk * G, t0, qz, bar(B_Q));
+            tma_load_4d(sQ + HALF_TILE, &P.tm_q, 64, hk * G, t0, qz, bar(B_Q));
+            const int key0 = (int)((int64_t)(P.layer0 + l) * P.rows + P.req[bl].row_base);
+            for (int j = 0; j < n_kv; ++j) {
+                const int s = j % STAGES;
+                if (j >= STAGES) mbar_wait(bar(B_KVE + s), (uint32_t)((j / STAGES) - 1) & 1u, P.err);
+                const int krow = key0 + j * BN;
+                mbar_expect_tx(bar(B_KF + s), TILE);
+                tma_load_3d(sK + s * TILE, &P.tm_k, 0, hk, krow, bar(B_KF + s));
+                tma_load_3d(sK + s * TILE + HALF_TILE, &P.tm_k, 64, hk, krow, bar(B_KF + s));
+                mbar_expect_tx(bar(B_VF + s), TILE);
+                tma_load_3d(sV + s * TILE, &P.tm_v, 0, hk, krow, bar(B_VF + s));
+                tma_load_3d(sV + s * TILE + HALF_TILE, &P.tm_v, 64, hk, krow, bar(B_VF + s));
+            }
+        }
+    } else if (warp == 1) {
+        // ---------------------------------------------------------------- MMA issuer
+        if (lane == 0) {
+            constexpr uint32_t idS = idesc_bf16(BM, BN, false);
+            constexpr uint32_t idO = idesc_bf16(BM, HD, true);
+            mbar_wait(bar(B_Q), 0, P.err);
+            tc_fence_after();
+            for (int j = 0; j <= n_kv; ++j) {
+                if (j < n_kv) {
+                    const int s = j % STAGES;
+                    const int sb = j & 1;
+                    mbar_wait(bar(B_KF + s), (uint32_t)(j / STAGES) & 1u, P.err);
+                    if (j >= 2) mbar_wait(bar(B_SFREE + sb), (uint32_t)((j - 2) >> 1) & 1u, P.err);
+                    tc_fence_after();
+                    const uint32_t kb = sK + s * TILE;
+#pragma unroll
+                    for (int kk = 0; kk < HD / 16; ++kk) {
+                        const uint32_t off = (uint32_t)(kk >> 2) * HALF_TILE + (uint32_t)(kk & 3) * 32u;
+                        mma_bf16(tmem + kColS + sb * BN, sw128_desc(sQ + off, 16, 1024),
+                                 sw128_desc(kb + off, 16, 1024), idS, kk > 0 ? 1u : 0u);
+                    }
+                    mma_commit(bar(B_SF + sb));
+                }
+                if (j >= 1) {
+                    const int jp = j - 1;
+                    const int s = jp % STAGES;
+                    mbar_wait(bar(B_PF), (uint32_t)jp & 1u, P.err);
+                    mbar_wait(bar(B_VF + s), (uint32_t)(jp / STAGES) & 1u, P.err);
+                    tc_fence_after();
+                    const uint32_t vb = sV + s * TILE;
+#pragma unroll
+                    for (int kk = 0; kk < BN / 16; ++kk) {
+                        const uint32_t aoff = (uint32_t)(kk >> 2) * HALF_TILE + (uint32_t)(kk & 3) * 32u;
+                        mma_bf16(tmem + kColO, sw128_desc(sP + aoff, 16, 1024),
+                                 sw128_desc(vb + (uint32_t)kk * 2048u, HALF_TILE, 1024), idO,
+                                 (jp > 0 || kk > 0) ? 1u : 0u);
+                    }
+                    mma_commit(bar(B_KVE + s));
+                    mma_commit(bar(B_PVD));
+                }
+            }
+        }
+    } else {
+        // ---------------------------------------------------------------- softmax warps
+        const int quad = warp & 3;
+        const int r = quad * 32 + lane;                 // row = TMEM lane
+        const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
+        const int t_row = min(t0 + r / G, P.sq - 1);   // rows past the suffix mirror its end
+        const int lim = s_r + t_row;                    // last key this row may see
+        const float sc = P.scale_log2;
+        float m_run = -CUDART_INF_F;
+        float l_run = 0.f;
+        const uint32_t p_row = sP + (uint32_t)r * 128u;
+        const uint32_t swz = (uint32_t)(r & 7);
+
+        for (int j = 0; j < n_kv; ++j) {
+            const int sb = j & 1;
+            mbar_wait(bar(B_SF + sb), (uint32_t)(j >> 1) & 1u, P.err);
+            tc_fence_after();
+            uint32_t sv[4][32];
+#pragma unroll
+            for (int c = 0; c < 4; ++c) tmem_ld32(tmem + lane_addr + kColS + sb * BN + c * 32, sv[c]);
+            tmem_ld_wait();
+            tc_fence_before();
+            mbar_arrive(bar(B_SFREE + sb));
+
+            const int kbase = j * BN;
+            if (kbase + BN - 1 > lim) {
+#pragma unroll
+                for (int c = 0; c < 4; ++c)
+#pragma unroll
+                    for (int e = 0; e < 32; ++e)
+                        if (kbase + c * 32 + e > lim) sv[c][e] = __float_as_uint(-CUDART_INF_F);
+            }
+            float mx = -CUDART_INF_F;
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+#pragma unroll
+                for (int e = 0; e < 32; ++e) mx = fmaxf(mx, __uint_as_float(sv[c][e]));
+            const float m_new = fmaxf(m_run, mx * sc);
+            const bool resc = m_new > m_run + 8.0f;       // also true on the first tile
+            const float m_use = resc ? m_new : m_run;
+            const float alpha = resc ? exp2f(m_run - m_new) : 1.0f;
+
+            if (j > 0) {
+                mbar_wait(bar(B_PVD), (uint32_t)(j - 1) & 1u, P.err);   // P buffer free, O current
+                if (__any_sync(0xffffffffu, resc)) {
+                    tc_fence_after();
+#pragma unroll
+                    for (int c = 0; c < 4; ++c) {
+                        uint32_t ov[32];
+                        tmem_ld32(tmem + lane_addr + kColO + c * 32, ov);
+                        tmem_ld_wait();
+#pragma unroll
+                        for (int e = 0; e < 32; ++e) ov[e] = __float_as_uint(__uint_as_float(ov[e]) * alpha);
+                        tmem_st32(tmem + lane_addr + kColO + c * 32, ov);
+                    }
+                    tmem_st_wait();
+                }
+            }
+            float sum = 0.f;
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+#pragma unroll
+                for (int q8 = 0; q8 < 4; ++q8) {
+                    uint32_t pk[4];
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const float a = exp2f(fmaf(__uint_as_float(sv[c][q8 * 8 + 2 * e]), sc, -m_use));
+                        const float bb = exp2f(fmaf(__uint_as_float(sv[c][q8 * 8 + 2 * e + 1]), sc, -m_use));
+                        sum += a + bb;
+                        pk[e] = pack_bf16(a, bb);
+                    }
+                    // keys c*32 + q8*8 .. +8: column block (c >> 1), 16-byte chunk within it
+                    const uint32_t chunk = (uint32_t)((c & 1) * 4 + q8);
+                    st_shared_v4(p_row + (uint32_t)(c >> 1) * HALF_TILE + ((chunk ^ swz) << 4),
+                                 pk[0], pk[1], pk[2], pk[3]);
+                }
+            }
+            l_run = l_run * alpha + sum;
+            m_run = m_use;
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+            tc_fence_before();
+            mbar_arrive(bar(B_PF));
+        }
+
+        // ---------------------------------------------------------------- epilogue
+        mbar_wait(bar(B_PVD), (uint32_t)(n_kv - 1) & 1u, P.err);
+        tc_fence_after();
+        const int t = t0 + r / G;
+        const int g = r - (r / G) * G;
+        const float inv = 1.0f / l_run;
+        __nv_bfloat16* orow = static_cast<__nv_bfloat16*>(P.out) +
+                              ((((int64_t)l * P.batch_total + b) * P.sq + t) * P.hq + hk * G + g) * HD;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            uint32_t ov[32];
+            tmem_ld32(tmem + lane_addr + kColO + c * 32, ov);
+            tmem_ld_wait();
+            if (t < P.sq) {
+#pragma unroll
+                for (int q8 = 0; q8 < 4; ++q8) {
+                    uint4 w;
+                    w.x = pack_bf16(__uint_as_float(ov[q8 * 8 + 0]) * inv, __uint_as_float(ov[q8 * 8 + 1]) * inv);
+                    w.y = pack_bf16(__uint_as_float(ov[q8 * 8 + 2]) * inv, __uint_as_float(ov[q8 * 8 + 3]) * inv);
+                    w.z = pack_bf16(__uint_as_float(ov[q8 * 8 + 4]) * inv, __uint_as_float(ov[q8 * 8 + 5]) * inv);
+                    w.w = pack_bf16(__uint_as_float(ov[q8 * 8 + 6]) * inv, __uint_as_float(ov[q8 * 8 + 7]) * inv);
+                    *reinterpret_cast<uint4*>(orow + c * 32 + q8 * 8) = w;
+                }
+            }
+        }
+        if (P.lse != nullptr && t < P.sq)
+            P.lse[(((int64_t)l * P.batch_total + b) * P.hq + hk * G + g) * P.sq + t] =
+                (m_run + log2f(l_run)) * 0.69314718055994531f;
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                     "r"(kTmemCols)
+                     : "memory");
+    }
+}
+
+// ------------------------------------------------------------------ host side
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+    if (!fn) {
+        void* p = nullptr;
+        cudaDriverEntryPointQueryResult q{};
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                             &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+    }
+    return fn;
+}
+
+bool encode(CUtensorMap* tm, const void* base, int rank, const cuuint64_t* dims,
+            const cuuint64_t* strides_bytes, const cuuint32_t* box) {
+    auto fn = encode_fn();
+    if (!fn) return false;
+    cuuint32_t estr[5] = {1, 1, 1, 1, 1};
+    const CUresult r = fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank,
+                          const_cast<void*>(base), dims, strides_bytes, box, estr,
+                          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                          CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    return r == CUDA_SUCCESS;
+}
+
+}  // namespace
+
+bool attn_tc_supported(int dtype, int d, int hq, int hkv) {
+    if (dtype != kDtypeBf16 || d != HD || hkv < 1 || hq % hkv) return false;
+    const int g = hq / hkv;
+    return g == 1 || g == 2 || g == 4 || g == 8 || g == 16;
+}
+
+cudaError_t launch_attn_tc(const AttnParams& a, cudaStream_t s) {
+    (void)cudaGetLastError();   // report this launch's error only, not a stale one
+    cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)kSmemBytes);
+    if (e != cudaSuccess) return e;
+    TcParams p;
+    std::memset(&p, 0, sizeof(p));
+    const int G = a.hq / a.hkv;
+    const int tq = BM / G;
+    {   // Q: q_rot [Lq*Btot][Sq][Hq][128] -> dims (d, Hq, Sq, Lq*Btot)
+        const cuuint64_t dims[4] = {HD, (cuuint64_t)a.hq, (cuuint64_t)a.sq,
+                                    (cuuint64_t)a.lq * a.batch_total};
+        const cuuint64_t str[3] = {(cuuint64_t)HD * 2, (cuuint64_t)a.hq * HD * 2,
+                                   (cuuint64_t)a.sq * a.hq * HD * 2};
+        const cuuint32_t box[4] = {64, (cuuint32_t)G, (cuuint32_t)tq, 1};
+        if (!encode(&p.tm_q, a.q_rot, 4, dims, str, box)) return cudaErrorInvalidValue;
+    }
+    {   // K, V: cache [L*rows][Hkv][128] -> dims (d, Hkv, L*rows); layer0 + lq <= L
+        const int64_t lrows = (int64_t)(a.layer0 + a.lq) * a.rows;
+        const cuuint64_t dims[3] = {HD, (cuuint64_t)a.hkv, (cuuint64_t)lrows};
+        const cuuint64_t str[2] = {(cuuint64_t)HD * 2, (cuuint64_t)a.hkv * HD * 2};
+        const cuuint32_t box[3] = {64, 1, (cuuint32_t)BN};
+        if (!encode(&p.tm_k, a.cache_k, 3, dims, str, box)) return cudaErrorInvalidValue;
+        if (!encode(&p.tm_v, a.cache_v, 3, dims, str, box)) return cudaErrorInvalidValue;
+    }
+    p.out = a.out;
+    p.lse = a.lse;
+    p.err = a.err;
+    p.rows = a.rows;
+    p.layer0 = a.layer0;
+    p.lq = a.lq;
+    p.batch = a.batch;
+    p.batch_total = a.batch_total;
+    p.b0 = a.b0;
+    p.sq = a.sq;
+    p.hq = a.hq;
+    p.hkv = a.hkv;
+    p.group = G;
+    p.tq = tq;
+    p.scale_log2 = a.scale_log2;
+    std::memcpy(p.req, a.req, sizeof(ReqParam) * (size_t)a.batch);
+    const dim3 grid((a.sq + tq - 1) / tq, a.hkv, a.lq * a.batch);
+    if (grid.z > 65535u || grid.y > 65535u) return cudaErrorInvalidValue;
+    attn_tc_kernel<<<grid, kThreads, kSmemBytes, s>>>(p);
+    return cudaGetLastError();
+}
 
 }  // namespace c2kv

@@ -75,6 +75,7 @@ c2kv_status fail(c2kv_ctx* ctx, c2kv_status code, const char* fmt, ...) {
 }
 
 c2kv_status cuda_fail(c2kv_ctx* ctx, cudaError_t e, const char* what) {
+    (void)cudaGetLastError();   // a non-sticky failure must not leak into later calls
     return fail(ctx, e == cudaErrorMemoryAllocation ? C2KV_ERR_NOMEM : C2KV_ERR_CUDA,
                 "%s: %s", what, cudaGetErrorString(e));
 }
@@ -532,6 +533,7 @@ c2kv_status c2kv_attend(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
             a.cache_v = cache->v;
             a.out = out;
             a.lse = lse;
+            a.err = c->d_err;
             a.rows = cache->rows;
             a.layer0 = layer0;
             a.lq = lq;

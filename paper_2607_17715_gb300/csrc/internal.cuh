@@ -106,6 +106,7 @@ struct AttnParams {
     const void* cache_v;
     void* out;               // [Lq][Btot][Sq][Hq][d]
     float* lse;              // [Lq][Btot][Hq][Sq] or null
+    int32_t* err;            // device error word: bit 1 = a bounded wait expired
     int64_t rows;
     int32_t layer0;
     int32_t lq;

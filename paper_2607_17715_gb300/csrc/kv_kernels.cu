@@ -362,6 +362,7 @@ int vph_of(int dtype, int d) { return d / 2 / (dtype == kDtypeBf16 ? 8 : 4); }
 
 cudaError_t launch_compose(const ComposeParams& p, int dtype, int d, int layers, cudaStream_t s) {
     if (p.n_tiles == 0 || p.n_occ == 0) return cudaSuccess;
+    (void)cudaGetLastError();   // report this launch's error only, not a stale one
     if (layers > 65535) return cudaErrorInvalidValue;
     const dim3 grid(p.n_tiles, layers);
     C2KV_DISPATCH(compose_kernel, grid, p, dtype, d, s);
@@ -370,6 +371,7 @@ cudaError_t launch_compose(const ComposeParams& p, int dtype, int d, int layers,
 
 cudaError_t launch_compress(const CompressParams& p, int dtype, int d, cudaStream_t s) {
     if (p.m == 0) return cudaSuccess;
+    (void)cudaGetLastError();
     const int64_t items = (int64_t)p.m * p.layers * p.hkv * vph_of(dtype, d);
     const int g = grid_for(items, 256);
     C2KV_DISPATCH(compress_kernel, g, p, dtype, d, s);
@@ -377,6 +379,7 @@ cudaError_t launch_compress(const CompressParams& p, int dtype, int d, cudaStrea
 }
 
 cudaError_t launch_suffix_prep(const SuffixParams& p, int dtype, int d, cudaStream_t s) {
+    (void)cudaGetLastError();
     const int64_t items = (int64_t)p.lq * p.batch * p.sq * (p.hq + p.hkv) * vph_of(dtype, d);
     const int g = grid_for(items, 256);
     C2KV_DISPATCH(suffix_kernel, g, p, dtype, d, s);

@@ -91,6 +91,17 @@ def pair_magnitude(k_stored: np.ndarray) -> np.ndarray:
     return np.concatenate([m, m], axis=-1)
 
 
+def check_rounded(got, want, scale, wl, what):
+    """At most one storage ulp from the fp64 result rounded once, or within fp32
+    arithmetic error, 2^-20 of `scale` (the magnitude of the operands the value was
+    computed from), where the result is much smaller than its operands."""
+    diff = np.abs(got - want)
+    allowed = np.maximum(ulp_of(want, wl), 2.0 ** -20 * scale)
+    bad = diff > allowed
+    assert not bad.any(), (f"{what}: {bad.sum()} elements off; worst diff "
+                           f"{diff.max():.3g}, ulps {np.max(np.abs(order_keys(got, wl) - order_keys(want, wl)))}")
+
+
 def check_rotated(got, want, k_stored, wl, what):
     """Rotated K: at most one storage ulp from the fp64 result rounded once, or within the
     fp32 arithmetic error of the rotation (2^-20 of the pair's magnitude) where a pair
