@@ -58,6 +58,23 @@ def describe(wl):
             f"positions/request), {wl.n_suffix} suffix tokens")
 
 
+def captured_traffic(kernel):
+    """DRAM bytes per launch from the committed ncu summary, if the kernel's source is still
+    the one that was captured (else None: the counters no longer describe this kernel)."""
+    import hashlib
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as fh:
+        rec = json.load(fh).get(kernel)
+    if not rec:
+        return None
+    src = os.path.join(ROOT, rec["source"])
+    with open(src, "rb") as fh:
+        digest = hashlib.sha256(fh.read()).hexdigest()[:16]
+    return rec["traffic_bytes"] if digest == rec["sha256_16"] else None
+
+
 def measured_peaks():
     path = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(path):
@@ -307,11 +324,12 @@ def run_ours(args):
                    "wall_s": round(wall, 4)},
         "roofline": {"bound": "hbm", "kernel": "compose_kernel", "achieved": round(comp_gbs, 1),
                      "peak": hbm, "unit": "GB/s", "frac": round(comp_gbs / hbm, 4),
-                     "traffic": None, "peak_source": f"{src} hbm_gbs",
+                     "traffic": captured_traffic("compose_kernel"), "peak_source": f"{src} hbm_gbs",
                      "bytes_per_launch": f["compose_bytes"]},
         "roofline_attend": {"bound": "tensor", "achieved": round(attn_tfs, 2), "peak": bf16,
                             "unit": "TFLOP/s", "frac": round(attn_tfs / bf16, 4),
                             "peak_source": f"{src} bf16_tflops (burst)",
+                            "traffic": captured_traffic("attn_tc_kernel"),
                             "note": "c2kv_attend call: suffix RoPE/append + attention"},
         "e2e": {"value": round(f["positions"] * world * args.steps / (e2e_ms / 1e3), 1),
                 "unit": "tokens/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
