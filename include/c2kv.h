@@ -213,6 +213,32 @@ c2kv_status c2kv_attend(c2kv_ctx* ctx, c2kv_cache* cache, int32_t layer, const v
                         const void* k_suf, const void* v_suf, int32_t n_suffix, void* out,
                         float* lse);
 
+/*
+ * c2kv_attend_noalloc -- the same computation and arguments as c2kv_attend, for callers
+ * that cannot let the library allocate device memory while they run: for example a
+ * serving engine that reserves all of HBM for its own cache pool at start-up and treats
+ * any later allocation as an error, or a host runtime whose allocator must own every
+ * device byte.  The paper has no counterpart; this is a deployment variant.
+ *
+ * c2kv_attend takes its scratch (the suffix queries after RoPE, which the attention
+ * kernels read) from the context's memory pool.  This call instead uses one fixed 16 MiB
+ * array that the library defines in device memory; it calls no allocator at all.
+ *   - Refused with C2KV_ERR_ARG (before anything is enqueued) when the rotated queries,
+ *     Lq * batch * n_suffix * Hq * head_dim * element size bytes, exceed 16 MiB; split
+ *     such a call by layer or by requests.
+ *   - Every GPU on which the library's device code is loaded holds the 16 MiB until the
+ *     process exits.
+ *   - The first call on a device looks up the array's device address (with that device
+ *     current) and keeps it; make that first call before any stream capture.
+ *   - All calls on a device share the array: calls whose GPU work overlaps (other
+ *     streams, other contexts on the same device) race on it.  It keeps the last call's
+ *     contents; nothing in it needs to start at zero.
+ * Errors: as c2kv_attend, plus ERR_ARG for the size limit.
+ */
+c2kv_status c2kv_attend_noalloc(c2kv_ctx* ctx, c2kv_cache* cache, int32_t layer,
+                                const void* q, const void* k_suf, const void* v_suf,
+                                int32_t n_suffix, void* out, float* lse);
+
 /* c2kv_cache_release -- free a composed cache (stream-ordered). */
 c2kv_status c2kv_cache_release(c2kv_ctx* ctx, c2kv_cache* cache);
 

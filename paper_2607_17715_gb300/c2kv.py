@@ -74,6 +74,7 @@ _SIGS = {
     "c2kv_compose": (_I32, [_VP, _I32, _P32, _P32, _P32, _I32, ctypes.POINTER(_VP)]),
     "c2kv_cache_info": (_I32, [_VP, ctypes.POINTER(c2kv_cache_desc)]),
     "c2kv_attend": (_I32, [_VP, _VP, _I32, _VP, _VP, _VP, _I32, _VP, _VP]),
+    "c2kv_attend_noalloc": (_I32, [_VP, _VP, _I32, _VP, _VP, _VP, _I32, _VP, _VP]),
     "c2kv_cache_release": (_I32, [_VP, _VP]),
     "c2kv_sync": (_I32, [_VP]),
     "c2kv_last_error": (ctypes.c_char_p, [_VP]),
@@ -194,6 +195,13 @@ def c2kv_cache_info(cache) -> dict:
 def c2kv_attend(ctx, cache, layer, q, k_suf, v_suf, n_suffix, out, lse=None):
     _check(_lib.c2kv_attend(ctx, cache, layer, _ptr(q), _ptr(k_suf), _ptr(v_suf), n_suffix,
                             _ptr(out), _ptr(lse)), ctx)
+
+
+def c2kv_attend_noalloc(ctx, cache, layer, q, k_suf, v_suf, n_suffix, out, lse=None):
+    """c2kv_attend without any device allocation (scratch in a fixed 16 MiB device array;
+    see include/c2kv.h for the limits)."""
+    _check(_lib.c2kv_attend_noalloc(ctx, cache, layer, _ptr(q), _ptr(k_suf), _ptr(v_suf),
+                                    n_suffix, _ptr(out), _ptr(lse)), ctx)
 
 
 def c2kv_cache_release(ctx, cache):

@@ -588,3 +588,35 @@ c2kv_status c2kv_inject_fault(c2kv_ctx* c, int32_t what) {
 }
 
 }  // extern "C"
+
+namespace c2kv {
+
+bool attend_view(const c2kv_ctx* c, const c2kv_cache* cache, AttendView* v) {
+    if (!c || !v || !own_cache(c, cache)) return false;
+    v->layers = c->cfg.layers;
+    v->n_q_heads = c->cfg.n_q_heads;
+    v->n_kv_heads = c->cfg.n_kv_heads;
+    v->head_dim = c->cfg.head_dim;
+    v->dtype = c->cfg.dtype;
+    v->attn_impl = c->cfg.attn_impl;
+    v->stream = c->stream;
+    v->err = c->d_err;
+    v->turns = c->turns;
+    v->cache_k = cache->k;
+    v->cache_v = cache->v;
+    v->pos = cache->pos;
+    v->rows = cache->rows;
+    v->batch = cache->batch;
+    v->suffix_capacity = cache->suffix_capacity;
+    v->row_base = cache->row_base.data();
+    v->n_slots = cache->n_slots.data();
+    v->l_req = cache->l_req.data();
+    return true;
+}
+
+int32_t set_last_error(c2kv_ctx* c, int32_t code, const char* msg) {
+    if (c) c->err = msg ? msg : "";
+    return code;
+}
+
+}  // namespace c2kv

@@ -131,4 +131,31 @@ cudaError_t launch_attn_simt(const AttnParams& p, int dtype, int d, cudaStream_t
 bool attn_tc_supported(int dtype, int d, int hq, int hkv);
 cudaError_t launch_attn_tc(const AttnParams& p, cudaStream_t s);
 
+// Read-only view of a context and one of its caches, for entry points defined outside
+// c2kv_api.cu (c2kv_attend_noalloc).
+struct AttendView {
+    int32_t layers, n_q_heads, n_kv_heads, head_dim, dtype, attn_impl;
+    cudaStream_t stream;
+    int32_t* err;
+    RopeTurns turns;
+    void* cache_k;
+    void* cache_v;
+    int32_t* pos;
+    int64_t rows;
+    int32_t batch;
+    int32_t suffix_capacity;
+    const int32_t* row_base;
+    const int32_t* n_slots;
+    const int32_t* l_req;
+};
+
+}  // namespace c2kv
+
+struct c2kv_ctx;
+struct c2kv_cache;
+namespace c2kv {
+// Fills `v` if `cache` belongs to `ctx` (returns false otherwise).
+bool attend_view(const c2kv_ctx* ctx, const c2kv_cache* cache, AttendView* v);
+// Records `msg` as the context's last error and returns `code`.
+int32_t set_last_error(c2kv_ctx* ctx, int32_t code, const char* msg);
 }  // namespace c2kv
