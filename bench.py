@@ -46,8 +46,12 @@ def workload_facts(wl):
     sq = wl.n_suffix
     keys = S * sq + sq * (sq + 1) // 2                     # visible (query, key) pairs
     attn_flops = 4 * wl.head_dim * wl.n_q_heads * keys * wl.batch * wl.layers
+    # attention bytes: every cache row (slots + suffix) read once, Q read, O written
+    attn_bytes = wl.layers * wl.batch * ((S + sq) * row_bytes * 2
+                                         + 2 * sq * wl.n_q_heads * wl.head_dim * eb)
     return dict(slots=S, span=span, positions=wl.batch * span, row_bytes=row_bytes,
-                compose_bytes=compose_bytes, attn_flops=attn_flops, slots_per_chunk=m)
+                compose_bytes=compose_bytes, attn_flops=attn_flops, attn_bytes=attn_bytes,
+                slots_per_chunk=m)
 
 
 def describe(wl):
@@ -269,6 +273,8 @@ def run_ours(args):
     c2kv.c2kv_sync(arm.ctx)
 
     events = [[E(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    c2kv.c2kv_profile_read(arm.ctx)            # drop anything recorded before the timed region
+    c2kv.c2kv_profile_enable(arm.ctx, True)     # per-kernel events on the library's stream
     barrier()
     with ClockSampler(local) as clocks:
         t0 = time.perf_counter()
@@ -279,6 +285,8 @@ def run_ours(args):
         wall = time.perf_counter() - t0
     barrier()
     c2kv.c2kv_sync(arm.ctx)
+    kern = c2kv.c2kv_profile_read(arm.ctx)      # mean device ms per kernel kind, timed steps
+    c2kv.c2kv_profile_enable(arm.ctx, False)
     step_ms = [ev[0].elapsed_time(ev[3]) for ev in events]
     compose_ms = [ev[0].elapsed_time(ev[1]) for ev in events]
     attend_ms = [ev[1].elapsed_time(ev[2]) for ev in events]
@@ -312,8 +320,10 @@ def run_ours(args):
     value = positions / (total_ms / 1e3)
     c_ms = statistics.mean(compose_ms)
     a_ms = statistics.mean(attend_ms)
-    comp_gbs = f["compose_bytes"] / (c_ms / 1e3) / 1e9
-    attn_tfs = f["attn_flops"] / (a_ms / 1e3) / 1e12
+    kc_ms = kern["compose"][0] or c_ms         # compose kernel alone (library events)
+    ka_ms = kern["attention"][0] or a_ms       # attention kernel alone
+    comp_gbs = f["compose_bytes"] / (kc_ms / 1e3) / 1e9
+    attn_tfs = f["attn_flops"] / (ka_ms / 1e3) / 1e12
     clk = clocks.summary()
     line = {
         "metric": METRIC, "value": round(value, 1), "unit": "tokens/s", "n_gpus": world,
@@ -323,8 +333,9 @@ def run_ours(args):
         "config": {"workload": describe(wl), "parallelism": f"dp{world}: requests sharded over ranks, no data-path collective",
                    "l2": "flushed between timed steps (256 MB write, untimed)",
                    "global_batch": wl.batch * world,
-                   "ttft_proxy_ms_per_layer": round(c_ms / wl.layers, 6),
-                   "compose_ms": round(c_ms, 5), "attend_ms": round(a_ms, 5),
+                   "ttft_proxy_ms_per_layer": round(kc_ms / wl.layers, 6),
+                   "compose_call_ms": round(c_ms, 5), "attend_call_ms": round(a_ms, 5),
+                   "kernel_ms": {k: round(v[0], 5) for k, v in kern.items() if v[1]},
                    "compose_gbs": round(comp_gbs, 1), "attend_tflops": round(attn_tfs, 2),
                    "compose_bytes": f["compose_bytes"], "attend_flops": f["attn_flops"],
                    "wall_s": round(wall, 4)},
@@ -332,11 +343,13 @@ def run_ours(args):
                      "peak": hbm, "unit": "GB/s", "frac": round(comp_gbs / hbm, 4),
                      "traffic": captured_traffic("compose_kernel"), "peak_source": f"{src} hbm_gbs",
                      "bytes_per_launch": f["compose_bytes"]},
-        "roofline_attend": {"bound": "tensor", "achieved": round(attn_tfs, 2), "peak": bf16,
+        "roofline_attend": {"bound": "tensor", "kernel": "attn_tc_kernel",
+                            "achieved": round(attn_tfs, 2), "peak": bf16,
                             "unit": "TFLOP/s", "frac": round(attn_tfs / bf16, 4),
                             "peak_source": f"{src} bf16_tflops (burst)",
                             "traffic": captured_traffic("attn_tc_kernel"),
-                            "note": "c2kv_attend call: suffix RoPE/append + attention"},
+                            "hbm_frac_of_cache_read": round(
+                                f["attn_bytes"] / (ka_ms / 1e3) / 1e9 / hbm, 4)},
         "e2e": {"value": round(positions / (e2e_ms / 1e3), 1),
                 "unit": "tokens/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "ms_per_step": round(e2e_ms / args.steps, 4)},

@@ -251,6 +251,23 @@ c2kv_status c2kv_sync(c2kv_ctx* ctx);
  * Valid until the next call on the context.  NULL ctx gives the last create() failure. */
 const char* c2kv_last_error(const c2kv_ctx* ctx);
 
+/*
+ * Tracing: per-kernel device time.  While enabled, each kernel launch the library makes
+ * (compose, compress, suffix RoPE/append, attention) is bracketed by CUDA events on the
+ * context's stream.  c2kv_profile_read synchronizes the stream and returns, per kind, the
+ * mean device time of the launches recorded since the previous read (or since enabling),
+ * then forgets them.  Kinds index the arrays:
+ */
+#define C2KV_PROF_COMPOSE  0
+#define C2KV_PROF_COMPRESS 1
+#define C2KV_PROF_SUFFIX   2   /* suffix RoPE + append + pad zeroing */
+#define C2KV_PROF_ATTN     3   /* the attention kernel alone */
+#define C2KV_PROF_KINDS    4
+c2kv_status c2kv_profile_enable(c2kv_ctx* ctx, int32_t on);
+/* mean_ms[C2KV_PROF_KINDS] receives mean milliseconds (0 where none), launches[] the
+ * counts; either may be NULL. */
+c2kv_status c2kv_profile_read(c2kv_ctx* ctx, float* mean_ms, int32_t* launches);
+
 /* c2kv_inject_fault -- host-side fault injection for tests.  what = 1: the next compose
  * writes one out-of-range pool slot index into its slot map, which the compose kernel's
  * bounds check must refuse (reported by c2kv_sync as ERR_DEVICE_BOUNDS).  what = 0 clears. */

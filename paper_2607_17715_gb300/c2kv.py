@@ -29,6 +29,8 @@ ERR_POSITIONS, ERR_CUDA, ERR_DEVICE_BOUNDS, ERR_STATE, ERR_UNSUPPORTED = -6, -7,
 DTYPE_BF16, DTYPE_F32 = 0, 1
 MODE_MEANPOOL, MODE_PROVIDED, MODE_STORED = 0, 1, 2
 ATTN_AUTO, ATTN_SIMT, ATTN_TC = 0, 1, 2
+PROF_COMPOSE, PROF_COMPRESS, PROF_SUFFIX, PROF_ATTN, PROF_KINDS = 0, 1, 2, 3, 4
+PROF_NAMES = ("compose", "compress", "suffix", "attention")
 
 STATUS_NAMES = {
     0: "OK", -1: "ERR_ARG", -2: "ERR_DTYPE", -3: "ERR_NOMEM", -4: "ERR_POOL_FULL",
@@ -79,6 +81,8 @@ _SIGS = {
     "c2kv_sync": (_I32, [_VP]),
     "c2kv_last_error": (ctypes.c_char_p, [_VP]),
     "c2kv_inject_fault": (_I32, [_VP, _I32]),
+    "c2kv_profile_enable": (_I32, [_VP, _I32]),
+    "c2kv_profile_read": (_I32, [_VP, ctypes.POINTER(ctypes.c_float), _P32]),
 }
 for _name, (_res, _args) in _SIGS.items():
     _fn = getattr(_lib, _name)
@@ -210,6 +214,18 @@ def c2kv_cache_release(ctx, cache):
 
 def c2kv_sync(ctx):
     _check(_lib.c2kv_sync(ctx), ctx)
+
+
+def c2kv_profile_enable(ctx, on=True):
+    _check(_lib.c2kv_profile_enable(ctx, int(bool(on))), ctx)
+
+
+def c2kv_profile_read(ctx) -> dict:
+    """{kind name: (mean ms, launches)} for the launches recorded since the last read."""
+    ms = (ctypes.c_float * PROF_KINDS)()
+    cnt = (ctypes.c_int32 * PROF_KINDS)()
+    _check(_lib.c2kv_profile_read(ctx, ms, cnt), ctx)
+    return {PROF_NAMES[k]: (ms[k], cnt[k]) for k in range(PROF_KINDS)}
 
 
 def c2kv_inject_fault(ctx, what):

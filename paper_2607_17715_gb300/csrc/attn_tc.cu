@@ -9,14 +9,18 @@
 // the causal mask.
 //
 // Warp roles (192 threads):
-//   warp 0      TMA producer: Q once, then K and V tiles into a 2-stage ring.
-//   warp 1      MMA issuer (one lane) and TMEM owner:  S_j = Q K_j^T into one of two
-//               TMEM S buffers, then O += P_{j-1} V_{j-1} into the TMEM O accumulator.
+//   warp 0      TMA producer: Q once, then K tiles into a 3-stage ring and V tiles into a
+//               3-stage ring, each issued as soon as its own stage is free (a K stage is
+//               refilled once S_j = Q K_j^T has read it, a V stage after P_j.V_j), so K
+//               loads never queue behind V releases.
+//   warp 1      MMA issuer (one lane) and TMEM owner:  S_j = Q K_j^T into one of two TMEM
+//               S buffers, then O += P_{j-1} V_{j-1}, P read from TMEM as the A operand.
 //   warps 2..5  softmax / correction / epilogue: thread i owns TMEM lane (row) i.  Reads
-//               S_j, masks, keeps the running max and sum, writes P_j (bf16) into shared
-//               memory in the MMA's 128B-swizzled K-major layout, rescales O in TMEM only
-//               when its row max grew by more than 2^8 (otherwise the stale reference max
-//               is kept: the normaliser uses the same one, so the result is exact).
+//               S_j, masks, keeps the running max and sum, writes P_j (bf16, two keys per
+//               32-bit column) into one of two TMEM P buffers (so P_{j+1} is written while
+//               P_j.V_j runs), rescales O in TMEM only when its row max grew by more than
+//               2^8 (otherwise the stale reference max is kept: the normaliser uses the
+//               same one, so the result is exact).
 //
 // Every mbarrier wait is bounded (kWaitCycles); on expiry the waiting thread sets bit 1
 // of the error word and carries on, so the kernel always terminates and the host reports
@@ -36,28 +40,32 @@ namespace {
 constexpr int BM = 128;                 // query rows per CTA (MMA M)
 constexpr int BN = 128;                 // keys per tile (MMA N of S, K of P.V)
 constexpr int HD = 128;                 // head dim
-constexpr int STAGES = 2;
+constexpr int KSTAGES = 3;              // K ring depth
+constexpr int VSTAGES = 3;              // V ring depth
 constexpr int TILE = BN * HD * 2;       // bytes of one 128 x 128 bf16 tile (32 KB)
 constexpr int HALF_TILE = TILE / 2;     // one 128-byte-wide swizzle column block
 constexpr int kThreads = 192;
-constexpr uint32_t kTmemCols = 512;     // S0 [0,128) S1 [128,256) O [256,384)
-constexpr uint32_t kColS = 0, kColO = 256;
+constexpr uint32_t kTmemCols = 512;     // S0 [0,128) S1 [128,256) O [256,384) P0, P1 [384,512)
+constexpr uint32_t kColS = 0, kColO = 256, kColP = 384;
 constexpr long long kWaitCycles = 4000000000LL;
 
 // barrier slots
 constexpr int B_Q = 0;
 constexpr int B_KF = 1;                  // + stage
-constexpr int B_VF = B_KF + STAGES;      // + stage
-constexpr int B_KVE = B_VF + STAGES;     // + stage: K and V stage free again
-constexpr int B_SF = B_KVE + STAGES;     // + buffer: S ready in TMEM
+constexpr int B_KE = B_KF + KSTAGES;     // + stage: K stage free (both S MMAs finished)
+constexpr int B_VF = B_KE + KSTAGES;     // + stage
+constexpr int B_VE = B_VF + VSTAGES;     // + stage: V stage free (both P.V MMAs finished)
+constexpr int B_SF = B_VE + VSTAGES;     // + buffer: S ready in TMEM
 constexpr int B_SFREE = B_SF + 2;        // + buffer: S read out by the softmax warps
-constexpr int B_PF = B_SFREE + 2;        // P written (and O corrected)
-constexpr int B_PVD = B_PF + 1;          // P.V finished (P buffer free, O current)
-constexpr int NBAR = B_PVD + 1;
+constexpr int B_PF = B_SFREE + 2;        // + buffer: P_j written (and O corrected)
+constexpr int B_PFREE = B_PF + 2;        // + buffer: P_j.V_j finished (buffer free, O current)
+constexpr int NBAR = B_PFREE + 2;
 
-constexpr size_t kSmemBytes = 1024 /*align*/ + (size_t)TILE * (2 + 2 * STAGES) + 8 * NBAR + 16;
+constexpr int kSmemTiles = 1 /*Q*/ + KSTAGES + VSTAGES;
+constexpr size_t kSmemBytes = 1024 /*align*/ + (size_t)TILE * kSmemTiles + 8 * NBAR + 16;
+static_assert(kSmemBytes <= 232448, "shared memory budget of one sm_100 CTA");
 
-struct alignas(64) TcParams {
+struct TcParams {                // CUtensorMap members carry their own alignment
     CUtensorMap tm_q;        // q_rot   [Lq*Btot][Sq][Hq][128]  box {64, G, TQ, 1}
     CUtensorMap tm_k;        // cache K [L*rows][Hkv][128]      box {64, 1, 128}
     CUtensorMap tm_v;        // cache V, same
@@ -168,6 +176,17 @@ __device__ __forceinline__ void mma_bf16(uint32_t d_tmem, uint64_t a, uint64_t b
         : "memory");
 }
 
+// Same, with A read from tensor memory (rows in lanes, K packed two bf16 per column).
+__device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t b,
+                                            uint32_t idesc, uint32_t accumulate) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "r"(a_tmem), "l"(b), "r"(idesc), "r"(accumulate)
+        : "memory");
+}
+
 __device__ __forceinline__ void mma_commit(uint32_t bar) {
     asm volatile(
         "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
@@ -209,16 +228,17 @@ __device__ __forceinline__ void tmem_st_wait() {
     asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 
+// 2^x on the MUFU pipe (ex2.approx: relative error ~2^-22, flushes subnormal results,
+// 2^-inf = +0).
+__device__ __forceinline__ float ex2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
     __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
     return *reinterpret_cast<uint32_t*>(&v);
-}
-
-__device__ __forceinline__ void st_shared_v4(uint32_t addr, uint32_t a, uint32_t b, uint32_t c,
-                                             uint32_t d) {
-    asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(addr), "r"(a), "r"(b), "r"(c),
-                 "r"(d)
-                 : "memory");
 }
 
 // ------------------------------------------------------------------ kernel
@@ -229,10 +249,9 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_const
                                                ~uintptr_t(1023));
     const uint32_t sQ = smem_u32(smem);
     const uint32_t sK = sQ + TILE;
-    const uint32_t sV = sK + STAGES * TILE;
-    const uint32_t sP = sV + STAGES * TILE;
-    const uint32_t sBar = sP + TILE;
-    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + (size_t)TILE * (2 + 2 * STAGES) + 8 * NBAR);
+    const uint32_t sV = sK + KSTAGES * TILE;
+    const uint32_t sBar = sV + VSTAGES * TILE;
+    uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + (size_t)TILE * kSmemTiles + 8 * NBAR);
     auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
 
     const int warp = threadIdx.x >> 5;
@@ -249,17 +268,20 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_const
 
     if (threadIdx.x == 0) {
         mbar_init(bar(B_Q), 1);
-        for (int s = 0; s < STAGES; ++s) {
+        for (int s = 0; s < KSTAGES; ++s) {
             mbar_init(bar(B_KF + s), 1);
+            mbar_init(bar(B_KE + s), 1);
+        }
+        for (int s = 0; s < VSTAGES; ++s) {
             mbar_init(bar(B_VF + s), 1);
-            mbar_init(bar(B_KVE + s), 1);
+            mbar_init(bar(B_VE + s), 1);
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(bar(B_SF + i), 1);
             mbar_init(bar(B_SFREE + i), 128);
+            mbar_init(bar(B_PF + i), 128);
+            mbar_init(bar(B_PFREE + i), 1);
         }
-        mbar_init(bar(B_PF), 128);
-        mbar_init(bar(B_PVD), 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (warp == 1) {
@@ -285,16 +307,34 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_const
             tma_load_4d(sQ, &P.tm_q, 0, hk * G, t0, qz, bar(B_Q));
             tma_load_4d(sQ + HALF_TILE, &P.tm_q, 64, hk * G, t0, qz, bar(B_Q));
             const int key0 = (int)((int64_t)(P.layer0 + l) * P.rows + P.req[bl].row_base);
-            for (int j = 0; j < n_kv; ++j) {
-                const int s = j % STAGES;
-                if (j >= STAGES) mbar_wait(bar(B_KVE + s), (uint32_t)((j / STAGES) - 1) & 1u, P.err);
-                const int krow = key0 + j * BN;
-                mbar_expect_tx(bar(B_KF + s), TILE);
-                tma_load_3d(sK + s * TILE, &P.tm_k, 0, hk, krow, bar(B_KF + s));
-                tma_load_3d(sK + s * TILE + HALF_TILE, &P.tm_k, 64, hk, krow, bar(B_KF + s));
-                mbar_expect_tx(bar(B_VF + s), TILE);
-                tma_load_3d(sV + s * TILE, &P.tm_v, 0, hk, krow, bar(B_VF + s));
-                tma_load_3d(sV + s * TILE + HALF_TILE, &P.tm_v, 64, hk, krow, bar(B_VF + s));
+            // two independent queues: a K load waits only for its own K stage
+            int jk = 0, jv = 0;
+            while (jk < n_kv || jv < n_kv) {
+                if (jk < n_kv && (jk < KSTAGES || mbar_try(bar(B_KE + jk % KSTAGES),
+                                                          (uint32_t)((jk / KSTAGES) - 1) & 1u))) {
+                    const int s = jk % KSTAGES;
+                    const int krow = key0 + jk * BN;
+                    mbar_expect_tx(bar(B_KF + s), TILE);
+                    tma_load_3d(sK + s * TILE, &P.tm_k, 0, hk, krow, bar(B_KF + s));
+                    tma_load_3d(sK + s * TILE + HALF_TILE, &P.tm_k, 64, hk, krow, bar(B_KF + s));
+                    ++jk;
+                    continue;
+                }
+                if (jv < n_kv && (jv < VSTAGES || mbar_try(bar(B_VE + jv % VSTAGES),
+                                                          (uint32_t)((jv / VSTAGES) - 1) & 1u))) {
+                    const int s = jv % VSTAGES;
+                    const int vrow = key0 + jv * BN;
+                    mbar_expect_tx(bar(B_VF + s), TILE);
+                    tma_load_3d(sV + s * TILE, &P.tm_v, 0, hk, vrow, bar(B_VF + s));
+                    tma_load_3d(sV + s * TILE + HALF_TILE, &P.tm_v, 64, hk, vrow, bar(B_VF + s));
+                    ++jv;
+                    continue;
+                }
+                // nothing issuable: wait (bounded) for the stage the next K load needs
+                if (jk < n_kv)
+                    mbar_wait(bar(B_KE + jk % KSTAGES), (uint32_t)((jk / KSTAGES) - 1) & 1u, P.err);
+                else
+                    mbar_wait(bar(B_VE + jv % VSTAGES), (uint32_t)((jv / VSTAGES) - 1) & 1u, P.err);
             }
         }
     } else if (warp == 1) {
@@ -306,12 +346,12 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_const
             tc_fence_after();
             for (int j = 0; j <= n_kv; ++j) {
                 if (j < n_kv) {
-                    const int s = j % STAGES;
+                    const int ks = j % KSTAGES;
                     const int sb = j & 1;
-                    mbar_wait(bar(B_KF + s), (uint32_t)(j / STAGES) & 1u, P.err);
+                    mbar_wait(bar(B_KF + ks), (uint32_t)(j / KSTAGES) & 1u, P.err);
                     if (j >= 2) mbar_wait(bar(B_SFREE + sb), (uint32_t)((j - 2) >> 1) & 1u, P.err);
                     tc_fence_after();
-                    const uint32_t kb = sK + s * TILE;
+                    const uint32_t kb = sK + ks * TILE;
 #pragma unroll
                     for (int kk = 0; kk < HD / 16; ++kk) {
                         const uint32_t off = (uint32_t)(kk >> 2) * HALF_TILE + (uint32_t)(kk & 3) * 32u;
@@ -319,23 +359,26 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_const
                                  sw128_desc(kb + off, 16, 1024), idS, kk > 0 ? 1u : 0u);
                     }
                     mma_commit(bar(B_SF + sb));
+                    mma_commit(bar(B_KE + ks));
                 }
                 if (j >= 1) {
                     const int jp = j - 1;
-                    const int s = jp % STAGES;
-                    mbar_wait(bar(B_PF), (uint32_t)jp & 1u, P.err);
-                    mbar_wait(bar(B_VF + s), (uint32_t)(jp / STAGES) & 1u, P.err);
+                    const int vs = jp % VSTAGES;
+                    const int pb = jp & 1;
+                    mbar_wait(bar(B_PF + pb), (uint32_t)(jp >> 1) & 1u, P.err);
+                    mbar_wait(bar(B_VF + vs), (uint32_t)(jp / VSTAGES) & 1u, P.err);
                     tc_fence_after();
-                    const uint32_t vb = sV + s * TILE;
+                    const uint32_t vb = sV + vs * TILE;
+                    const uint32_t pcol = tmem + kColP + (uint32_t)pb * (BN / 2);
 #pragma unroll
                     for (int kk = 0; kk < BN / 16; ++kk) {
-                        const uint32_t aoff = (uint32_t)(kk >> 2) * HALF_TILE + (uint32_t)(kk & 3) * 32u;
-                        mma_bf16(tmem + kColO, sw128_desc(sP + aoff, 16, 1024),
-                                 sw128_desc(vb + (uint32_t)kk * 2048u, HALF_TILE, 1024), idO,
-                                 (jp > 0 || kk > 0) ? 1u : 0u);
+                        // A = P_j from TMEM: 16 keys (8 packed columns) per instruction
+                        mma_bf16_ts(tmem + kColO, pcol + (uint32_t)kk * 8u,
+                                    sw128_desc(vb + (uint32_t)kk * 2048u, HALF_TILE, 1024), idO,
+                                    (jp > 0 || kk > 0) ? 1u : 0u);
                     }
-                    mma_commit(bar(B_KVE + s));
-                    mma_commit(bar(B_PVD));
+                    mma_commit(bar(B_VE + vs));
+                    mma_commit(bar(B_PFREE + pb));
                 }
             }
         }
@@ -349,8 +392,6 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_const
         const float sc = P.scale_log2;
         float m_run = -CUDART_INF_F;
         float l_run = 0.f;
-        const uint32_t p_row = sP + (uint32_t)r * 128u;
-        const uint32_t swz = (uint32_t)(r & 7);
 
         for (int j = 0; j < n_kv; ++j) {
             const int sb = j & 1;
@@ -371,60 +412,72 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_const
                     for (int e = 0; e < 32; ++e)
                         if (kbase + c * 32 + e > lim) sv[c][e] = __float_as_uint(-CUDART_INF_F);
             }
-            float mx = -CUDART_INF_F;
+            // row max with 8 independent chains (no 128-long dependency)
+            float mx8[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) mx8[e] = -CUDART_INF_F;
 #pragma unroll
             for (int c = 0; c < 4; ++c)
 #pragma unroll
-                for (int e = 0; e < 32; ++e) mx = fmaxf(mx, __uint_as_float(sv[c][e]));
+                for (int e = 0; e < 32; ++e)
+                    mx8[e & 7] = fmaxf(mx8[e & 7], __uint_as_float(sv[c][e]));
+            const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
+                                   fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
             const float m_new = fmaxf(m_run, mx * sc);
             const bool resc = m_new > m_run + 8.0f;       // also true on the first tile
             const float m_use = resc ? m_new : m_run;
-            const float alpha = resc ? exp2f(m_run - m_new) : 1.0f;
+            const float alpha = resc ? ex2(m_run - m_new) : 1.0f;
 
-            if (j > 0) {
-                mbar_wait(bar(B_PVD), (uint32_t)(j - 1) & 1u, P.err);   // P buffer free, O current
-                if (__any_sync(0xffffffffu, resc)) {
-                    tc_fence_after();
+            const int pb = j & 1;
+            // P buffer pb is free once P_{j-2}.V_{j-2} has finished
+            if (j >= 2) mbar_wait(bar(B_PFREE + pb), (uint32_t)((j - 2) >> 1) & 1u, P.err);
+            if (j >= 1 && __any_sync(0xffffffffu, resc)) {
+                // O must hold every P.V up to tile j-1 before it is rescaled
+                mbar_wait(bar(B_PFREE + (pb ^ 1)), (uint32_t)((j - 1) >> 1) & 1u, P.err);
+                tc_fence_after();
 #pragma unroll
-                    for (int c = 0; c < 4; ++c) {
-                        uint32_t ov[32];
-                        tmem_ld32(tmem + lane_addr + kColO + c * 32, ov);
-                        tmem_ld_wait();
+                for (int c = 0; c < 4; ++c) {
+                    uint32_t ov[32];
+                    tmem_ld32(tmem + lane_addr + kColO + c * 32, ov);
+                    tmem_ld_wait();
 #pragma unroll
-                        for (int e = 0; e < 32; ++e) ov[e] = __float_as_uint(__uint_as_float(ov[e]) * alpha);
-                        tmem_st32(tmem + lane_addr + kColO + c * 32, ov);
-                    }
-                    tmem_st_wait();
+                    for (int e = 0; e < 32; ++e) ov[e] = __float_as_uint(__uint_as_float(ov[e]) * alpha);
+                    tmem_st32(tmem + lane_addr + kColO + c * 32, ov);
                 }
+                tmem_st_wait();
             }
-            float sum = 0.f;
+            float ps[8];
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
+            for (int e = 0; e < 8; ++e) ps[e] = 0.f;
+            // P_j (bf16, keys 2c and 2c+1 packed in column c) into TMEM buffer pb
+            const uint32_t p_addr = tmem + lane_addr + kColP + (uint32_t)pb * (BN / 2);
 #pragma unroll
-                for (int q8 = 0; q8 < 4; ++q8) {
-                    uint32_t pk[4];
+            for (int half = 0; half < 2; ++half) {
+                uint32_t pk[32];
 #pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const float a = exp2f(fmaf(__uint_as_float(sv[c][q8 * 8 + 2 * e]), sc, -m_use));
-                        const float bb = exp2f(fmaf(__uint_as_float(sv[c][q8 * 8 + 2 * e + 1]), sc, -m_use));
-                        sum += a + bb;
-                        pk[e] = pack_bf16(a, bb);
+                for (int cc = 0; cc < 2; ++cc) {
+                    const int c = half * 2 + cc;
+#pragma unroll
+                    for (int e = 0; e < 32; e += 2) {
+                        const float a0 = ex2(fmaf(__uint_as_float(sv[c][e]), sc, -m_use));
+                        const float a1 = ex2(fmaf(__uint_as_float(sv[c][e + 1]), sc, -m_use));
+                        ps[e & 7] += a0;
+                        ps[(e + 1) & 7] += a1;
+                        pk[cc * 16 + (e >> 1)] = pack_bf16(a0, a1);
                     }
-                    // keys c*32 + q8*8 .. +8: column block (c >> 1), 16-byte chunk within it
-                    const uint32_t chunk = (uint32_t)((c & 1) * 4 + q8);
-                    st_shared_v4(p_row + (uint32_t)(c >> 1) * HALF_TILE + ((chunk ^ swz) << 4),
-                                 pk[0], pk[1], pk[2], pk[3]);
                 }
+                tmem_st32(p_addr + (uint32_t)half * 32u, pk);
             }
+            tmem_st_wait();
+            const float sum = ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
             l_run = l_run * alpha + sum;
             m_run = m_use;
-            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
             tc_fence_before();
-            mbar_arrive(bar(B_PF));
+            mbar_arrive(bar(B_PF + pb));
         }
 
         // ---------------------------------------------------------------- epilogue
-        mbar_wait(bar(B_PVD), (uint32_t)(n_kv - 1) & 1u, P.err);
+        mbar_wait(bar(B_PFREE + ((n_kv - 1) & 1)), (uint32_t)((n_kv - 1) >> 1) & 1u, P.err);
         tc_fence_after();
         const int t = t0 + r / G;
         const int g = r - (r / G) * G;

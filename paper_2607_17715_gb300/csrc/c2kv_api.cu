@@ -59,6 +59,11 @@ struct c2kv_ctx {
     std::vector<c2kv_cache*> caches;
     int32_t inject = 0;
     c2kv::RopeTurns turns{};
+    // tracing (c2kv_profile_enable): event pairs around launches, by kind
+    bool prof = false;
+    struct ProfRec { int kind; cudaEvent_t a, b; };
+    std::vector<ProfRec> prof_recs;
+    std::vector<cudaEvent_t> prof_free;
 };
 
 namespace {
@@ -157,6 +162,40 @@ void destroy_cache(c2kv_ctx* c, c2kv_cache* cache) {
     delete cache;
 }
 
+cudaEvent_t prof_event(c2kv_ctx* c) {
+    if (!c->prof_free.empty()) {
+        cudaEvent_t e = c->prof_free.back();
+        c->prof_free.pop_back();
+        return e;
+    }
+    cudaEvent_t e = nullptr;
+    if (cudaEventCreate(&e) != cudaSuccess) {
+        (void)cudaGetLastError();
+        return nullptr;
+    }
+    return e;
+}
+
+// Brackets the launches between begin() and end() with events when tracing is on.
+struct ProfScope {
+    c2kv_ctx* c;
+    int kind;
+    cudaEvent_t a = nullptr;
+    ProfScope(c2kv_ctx* ctx, int k) : c(ctx), kind(k) {
+        if (c->prof && (a = prof_event(c)) != nullptr) cudaEventRecord(a, c->stream);
+    }
+    ~ProfScope() {
+        if (!a) return;
+        cudaEvent_t b = prof_event(c);
+        if (!b) {
+            c->prof_free.push_back(a);
+            return;
+        }
+        cudaEventRecord(b, c->stream);
+        c->prof_recs.push_back({kind, a, b});
+    }
+};
+
 }  // namespace
 
 extern "C" {
@@ -230,6 +269,11 @@ c2kv_status c2kv_destroy(c2kv_ctx* c) {
         for (c2kv_cache* cache : c->caches) destroy_cache(c, cache);
         c->caches.clear();
         cudaStreamSynchronize(c->stream);
+        for (auto& r : c->prof_recs) {
+            cudaEventDestroy(r.a);
+            cudaEventDestroy(r.b);
+        }
+        for (cudaEvent_t e : c->prof_free) cudaEventDestroy(e);
         if (c->mempool) cudaMemPoolDestroy(c->mempool);
         if (c->pool_k) cudaFree(c->pool_k);
         if (c->pool_v) cudaFree(c->pool_v);
@@ -290,6 +334,7 @@ c2kv_status c2kv_compress_chunk(c2kv_ctx* c, const void* k, const void* v, int32
             a.layers = c->cfg.layers;
             a.hkv = c->cfg.n_kv_heads;
             a.rope = c->turns;
+            ProfScope prof_compress(c, C2KV_PROF_COMPRESS);
             e = c2kv::launch_compress(a, c->cfg.dtype, c->cfg.head_dim, c->stream);
         }
         if (e != cudaSuccess) {
@@ -425,6 +470,7 @@ c2kv_status c2kv_compose(c2kv_ctx* c, int32_t batch, const int32_t* req_ptr,
         if (e == cudaSuccess) e = pool_alloc(c, &cache->v, kv_bytes);
         if (e == cudaSuccess) e = pool_alloc(c, reinterpret_cast<void**>(&cache->pos), pos_bytes);
         // One launch per group of at most kMaxOcc occurrences, all layers at once.
+        ProfScope prof_compose(c, C2KV_PROF_COMPOSE);
         for (int32_t g0 = 0; e == cudaSuccess && g0 < n_occ; g0 += c2kv::kMaxOcc) {
             c2kv::ComposeParams pr{};
             pr.pool_k = c->pool_k;
@@ -525,7 +571,10 @@ c2kv_status c2kv_attend(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
             for (int32_t i = 0; i < nb; ++i)
                 s.req[i] = c2kv::ReqParam{cache->row_base[b0 + i], cache->n_slots[b0 + i],
                                           cache->l_req[b0 + i], 0};
-            e = c2kv::launch_suffix_prep(s, c->cfg.dtype, c->cfg.head_dim, c->stream);
+            {
+                ProfScope prof_suffix(c, C2KV_PROF_SUFFIX);
+                e = c2kv::launch_suffix_prep(s, c->cfg.dtype, c->cfg.head_dim, c->stream);
+            }
             if (e != cudaSuccess) break;
             c2kv::AttnParams a{};
             a.q_rot = q_rot;
@@ -545,6 +594,7 @@ c2kv_status c2kv_attend(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
             a.hkv = c->cfg.n_kv_heads;
             a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)c->cfg.head_dim));
             for (int32_t i = 0; i < nb; ++i) a.req[i] = s.req[i];
+            ProfScope prof_attn(c, C2KV_PROF_ATTN);
             e = use_tc ? c2kv::launch_attn_tc(a, c->stream)
                        : c2kv::launch_attn_simt(a, c->cfg.dtype, c->cfg.head_dim, c->stream);
         }
@@ -578,6 +628,42 @@ c2kv_status c2kv_sync(c2kv_ctx* c) {
         return fail(c, C2KV_ERR_DEVICE_BOUNDS, "sync: a kernel refused an out-of-range index (flags 0x%x)", word);
     }
     return C2KV_OK;
+}
+
+c2kv_status c2kv_profile_enable(c2kv_ctx* c, int32_t on) {
+    if (!c) return C2KV_ERR_ARG;
+    c->prof = on != 0;
+    return C2KV_OK;
+}
+
+c2kv_status c2kv_profile_read(c2kv_ctx* c, float* mean_ms, int32_t* launches) {
+    if (!c) return C2KV_ERR_ARG;
+    try {
+        c->err.clear();
+        cudaError_t e = cudaStreamSynchronize(c->stream);
+        if (e != cudaSuccess) return cuda_fail(c, e, "profile_read");
+        double sum[C2KV_PROF_KINDS] = {0};
+        int32_t cnt[C2KV_PROF_KINDS] = {0};
+        for (auto& r : c->prof_recs) {
+            float ms = 0.f;
+            if (cudaEventElapsedTime(&ms, r.a, r.b) == cudaSuccess && r.kind >= 0 &&
+                r.kind < C2KV_PROF_KINDS) {
+                sum[r.kind] += ms;
+                cnt[r.kind] += 1;
+            }
+            (void)cudaGetLastError();
+            c->prof_free.push_back(r.a);
+            c->prof_free.push_back(r.b);
+        }
+        c->prof_recs.clear();
+        for (int k = 0; k < C2KV_PROF_KINDS; ++k) {
+            if (mean_ms) mean_ms[k] = cnt[k] ? (float)(sum[k] / cnt[k]) : 0.f;
+            if (launches) launches[k] = cnt[k];
+        }
+        return C2KV_OK;
+    } catch (const std::bad_alloc&) {
+        return fail(c, C2KV_ERR_NOMEM, "profile_read: host allocation failed");
+    }
 }
 
 c2kv_status c2kv_inject_fault(c2kv_ctx* c, int32_t what) {

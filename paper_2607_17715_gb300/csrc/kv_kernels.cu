@@ -244,9 +244,12 @@ __global__ void __launch_bounds__(256) compress_kernel(const __grid_constant__ C
 }
 
 // ---------------------------------------------------------------------------------------
-// suffix preparation.  Items per suffix row (layer, request, token): Hq query-head pairs
-// (RoPE at L_b + t into q_rot) then Hkv key-head pairs (RoPE into the cache row
-// row_base + S_b + t, V copied alongside, position recorded).
+// suffix preparation.  grid = (batch * Sq suffix rows + batch pad blocks, layers).  A row
+// block forms the row's d/2 (cos, sin) at L_b + t once in shared memory, then turns the
+// Hq query heads into q_rot and the Hkv key heads into the cache row row_base + S_b + t
+// (V copied alongside) for its layer.  A pad block zeroes its request's cache rows from
+// the end of the suffix to the next 128-row boundary, so a key tile that straddles the end
+// reads finite zeros (masked keys must not carry NaN/Inf garbage into P.V).
 // ---------------------------------------------------------------------------------------
 template <typename T, int VPH>
 __global__ void __launch_bounds__(256) suffix_kernel(const __grid_constant__ SuffixParams P) {
@@ -254,83 +257,77 @@ __global__ void __launch_bounds__(256) suffix_kernel(const __grid_constant__ Suf
     constexpr int E = V::N;
     constexpr int HALF = VPH * E;
     constexpr int D = 2 * HALF;
-    const int per_row = (P.hq + P.hkv) * VPH;
-    const int64_t n_rows = (int64_t)P.lq * P.batch * P.sq;
-    const int64_t total = n_rows * per_row;
-    for (int64_t it = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; it < total;
-         it += (int64_t)gridDim.x * blockDim.x) {
-        const int64_t row = it / per_row;           // ((l * batch) + bl) * Sq + t
-        const int p = (int)(it - row * per_row);
-        const int t = (int)(row % P.sq);
-        const int64_t lb = row / P.sq;
-        const int bl = (int)(lb % P.batch);
-        const int l = (int)(lb / P.batch);
-        const ReqParam& rq = P.req[bl];
-        const int64_t grow = ((int64_t)l * P.batch_total + P.b0 + bl) * P.sq + t;  // tensor row
-        const int64_t position = (int64_t)rq.l_req + t;
-        const bool is_q = p < P.hq * VPH;
-        const int pp = is_q ? p : p - P.hq * VPH;
+    __shared__ float2 cs[HALF];
+    const int l = blockIdx.y;
+    const int n_rows = P.batch * P.sq;
+    const int64_t row_elems = (int64_t)P.hkv * D;
+    if ((int)blockIdx.x >= n_rows) {
+        const int bl = blockIdx.x - n_rows;
+        const int used = P.req[bl].n_slots + P.sq;
+        const int end = (used + 127) / 128 * 128;
+        constexpr int VPR_ELEMS = 16 / (int)sizeof(T);
+        const int vec_per_row = (int)(row_elems / VPR_ELEMS);
+        const int items = (end - used) * vec_per_row;
+        const uint4 z = make_uint4(0, 0, 0, 0);
+        for (int it = threadIdx.x; it < items; it += blockDim.x) {
+            const int rr = it / vec_per_row;
+            const int vi = it - rr * vec_per_row;
+            const int64_t crow = (int64_t)P.req[bl].row_base + used + rr;
+            if (crow >= P.rows) continue;
+            const int64_t off = ((int64_t)(P.layer0 + l) * P.rows + crow) * row_elems + (int64_t)vi * VPR_ELEMS;
+            st16(static_cast<T*>(P.cache_k) + off, z);
+            st16(static_cast<T*>(P.cache_v) + off, z);
+        }
+        return;
+    }
+    const int bl = blockIdx.x / P.sq;
+    const int t = blockIdx.x - bl * P.sq;
+    const ReqParam& rq = P.req[bl];
+    const int64_t position = (int64_t)rq.l_req + t;
+    if (threadIdx.x < HALF) cs[threadIdx.x] = turn_cs(P.rope.turn[threadIdx.x], position);
+    __syncthreads();
+    const int64_t crow = (int64_t)rq.row_base + rq.n_slots + t;
+    if (threadIdx.x == 0 && l == 0 && crow >= 0 && crow < P.rows) P.pos[crow] = (int32_t)position;
+    const int64_t grow = ((int64_t)l * P.batch_total + P.b0 + bl) * P.sq + t;  // tensor row
+    const int nq = P.hq * VPH;
+    const int items = (P.hq + P.hkv) * VPH;
+    for (int p = threadIdx.x; p < items; p += blockDim.x) {
+        const bool is_q = p < nq;
+        const int pp = is_q ? p : p - nq;
         const int h = pp / VPH;
         const int iv = pp - h * VPH;
-        float2 cs[E];
-#pragma unroll
-        for (int e = 0; e < E; ++e) cs[e] = turn_cs(P.rope.turn[iv * E + e], position);
         float x[E], y[E], gx[E], gy[E];
         if (is_q) {
             const int64_t off = (grow * P.hq + h) * D + iv * E;
             const T* src = static_cast<const T*>(P.q) + off;
-            V::unpack(ld16(src), x);
-            V::unpack(ld16(src + HALF), y);
-            rotate<E>(x, y, cs, gx, gy);
+            const uint4 a = ld16(src);
+            const uint4 b = ld16(src + HALF);
+            V::unpack(a, x);
+            V::unpack(b, y);
+            rotate<E>(x, y, cs + iv * E, gx, gy);
             T* dst = static_cast<T*>(P.q_rot) + off;
             st16(dst, V::pack(gx));
             st16(dst + HALF, V::pack(gy));
         } else {
-            const int64_t off = (grow * P.hkv + h) * D + iv * E;
-            const int64_t crow = (int64_t)rq.row_base + rq.n_slots + t;
             if (crow < 0 || crow >= P.rows) continue;
-            const int64_t coff = (((int64_t)(P.layer0 + l) * P.rows + crow) * P.hkv + h) * D + iv * E;
+            const int64_t off = (grow * P.hkv + h) * D + iv * E;
+            const int64_t coff = ((int64_t)(P.layer0 + l) * P.rows + crow) * row_elems + h * D + iv * E;
             const T* ks = static_cast<const T*>(P.k) + off;
             const T* vs = static_cast<const T*>(P.v) + off;
-            V::unpack(ld16(ks), x);
-            V::unpack(ld16(ks + HALF), y);
-            rotate<E>(x, y, cs, gx, gy);
+            const uint4 ka = ld16(ks);
+            const uint4 kb = ld16(ks + HALF);
+            const uint4 va = ld16(vs);
+            const uint4 vb = ld16(vs + HALF);
+            V::unpack(ka, x);
+            V::unpack(kb, y);
+            rotate<E>(x, y, cs + iv * E, gx, gy);
             T* kd = static_cast<T*>(P.cache_k) + coff;
             T* vd = static_cast<T*>(P.cache_v) + coff;
             st16(kd, V::pack(gx));
             st16(kd + HALF, V::pack(gy));
-            st16(vd, ld16(vs));
-            st16(vd + HALF, ld16(vs + HALF));
-            if (l == 0 && pp == 0) P.pos[crow] = (int32_t)position;
+            st16(vd, va);
+            st16(vd + HALF, vb);
         }
-    }
-}
-
-// Zero the cache rows between the end of the suffix and the next 128-row boundary, so a
-// key tile that straddles the end reads finite zeros (masked keys must not carry NaN/Inf
-// garbage into P.V).
-template <typename T>
-__global__ void __launch_bounds__(256) pad_zero_kernel(const __grid_constant__ SuffixParams P, int d) {
-    const int vec_per_row = P.hkv * d * (int)sizeof(T) / 16;
-    const int64_t total = (int64_t)P.lq * P.batch * 128 * vec_per_row;
-    for (int64_t it = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; it < total;
-         it += (int64_t)gridDim.x * blockDim.x) {
-        const int vi = (int)(it % vec_per_row);
-        const int64_t r = it / vec_per_row;
-        const int rr = (int)(r % 128);
-        const int64_t lb = r / 128;
-        const int bl = (int)(lb % P.batch);
-        const int l = (int)(lb / P.batch);
-        const int used = P.req[bl].n_slots + P.sq;
-        const int end = (used + 127) / 128 * 128;
-        const int row = used + rr;
-        if (row >= end) continue;
-        const int64_t crow = (int64_t)P.req[bl].row_base + row;
-        if (crow >= P.rows) continue;
-        const int64_t off = ((int64_t)(P.layer0 + l) * P.rows + crow) * P.hkv * d;
-        const uint4 z = make_uint4(0, 0, 0, 0);
-        st16(static_cast<T*>(P.cache_k) + off + vi * (16 / (int)sizeof(T)), z);
-        st16(static_cast<T*>(P.cache_v) + off + vi * (16 / (int)sizeof(T)), z);
     }
 }
 
@@ -379,17 +376,12 @@ cudaError_t launch_compress(const CompressParams& p, int dtype, int d, cudaStrea
 }
 
 cudaError_t launch_suffix_prep(const SuffixParams& p, int dtype, int d, cudaStream_t s) {
-    (void)cudaGetLastError();
-    const int64_t items = (int64_t)p.lq * p.batch * p.sq * (p.hq + p.hkv) * vph_of(dtype, d);
-    const int g = grid_for(items, 256);
-    C2KV_DISPATCH(suffix_kernel, g, p, dtype, d, s);
-    cudaError_t e = cudaGetLastError();
-    if (e != cudaSuccess) return e;
-    const int eb = dtype == kDtypeBf16 ? 2 : 4;
-    const int64_t pad_items = (int64_t)p.lq * p.batch * 128 * (p.hkv * d * eb / 16);
-    const int gp = grid_for(pad_items, 256);
-    if (dtype == kDtypeBf16) pad_zero_kernel<__nv_bfloat16><<<gp, 256, 0, s>>>(p, d);
-    else pad_zero_kernel<float><<<gp, 256, 0, s>>>(p, d);
+    (void)cudaGetLastError();   // report this launch's error only, not a stale one
+    if (p.batch < 1 || p.sq < 1 || p.lq < 1) return cudaSuccess;
+    const int64_t blocks = (int64_t)p.batch * p.sq + p.batch;
+    if (blocks > 0x7fffffffLL || p.lq > 65535) return cudaErrorInvalidValue;
+    const dim3 grid((unsigned)blocks, p.lq);
+    C2KV_DISPATCH(suffix_kernel, grid, p, dtype, d, s);
     return cudaGetLastError();
 }
 

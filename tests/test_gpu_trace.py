@@ -1,0 +1,37 @@
+"""Tracing: per-kernel device time through c2kv_profile_enable / c2kv_profile_read."""
+import numpy as np
+import pytest
+import torch
+
+import synth
+from tests import _gpu_helpers as H
+
+pytestmark = pytest.mark.gpu
+
+
+def test_profile_counts_and_times():
+    wl = synth.scaled(synth.workload("llama8b"), layers=2, chunks_per_request=3, pool_chunks=3)
+    c2kv = H.lib()
+    ctx = H.make_ctx(wl, pool_slots=1024)
+    try:
+        c2kv.c2kv_profile_enable(ctx, True)
+        kt, vt = synth.chunk_tokens(wl, 0)
+        ids = [c2kv.c2kv_compress_chunk(ctx, H.to_dev(kt, wl), H.to_dev(vt, wl),
+                                        wl.chunk_tokens, wl.ratio_k, c2kv.MODE_MEANPOOL)
+               for _ in range(3)]
+        cache = c2kv.c2kv_compose(ctx, [0, 3], ids, None, wl.n_suffix)
+        q, k, v = (H.to_dev(x, wl) for x in synth.suffix(wl))
+        out = torch.empty_like(q)
+        for _ in range(2):
+            c2kv.c2kv_attend(ctx, cache, -1, q, k, v, wl.n_suffix, out)
+        prof = c2kv.c2kv_profile_read(ctx)
+        assert prof["compress"][1] == 3 and prof["compose"][1] == 1
+        assert prof["suffix"][1] == 2 and prof["attention"][1] == 2
+        assert all(ms > 0 for ms, n in prof.values() if n)
+        assert c2kv.c2kv_profile_read(ctx)["attention"] == (0.0, 0)   # read clears
+        c2kv.c2kv_profile_enable(ctx, False)
+        c2kv.c2kv_attend(ctx, cache, -1, q, k, v, wl.n_suffix, out)
+        assert c2kv.c2kv_profile_read(ctx)["attention"][1] == 0
+        assert np.isfinite(out.float().cpu().numpy()).all()
+    finally:
+        c2kv.c2kv_destroy(ctx)
