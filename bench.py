@@ -151,7 +151,7 @@ class ClockSampler:
 class Arm:
     """This rank's share of the global batch (wl.batch requests per rank) on its GPU."""
 
-    def __init__(self, wl, rank, world, torch, c2kv):
+    def __init__(self, wl, rank, world, torch, c2kv, attn_split=0):
         from paper_2607_17715_gb300.shard import shard_range
         seed = 0
         gwl = synth.scaled(wl, batch=wl.batch * world)
@@ -168,7 +168,7 @@ class Arm:
         self.ctx = c2kv.c2kv_create(
             wl.layers, wl.n_q_heads, wl.n_kv_heads, wl.head_dim, wl.rope_theta,
             c2kv.DTYPE_F32 if wl.dtype == "f32" else c2kv.DTYPE_BF16,
-            pool_slots=len(pool_ids) * m * 2 + 64, stream=self.stream)
+            pool_slots=len(pool_ids) * m * 2 + 64, stream=self.stream, attn_split=attn_split)
         # stored compressed chunks, kept in pinned host memory (the storage tier) and
         # loaded once into the device pool for the device-resident measurement
         self.host_chunks = {}
@@ -257,7 +257,7 @@ def run_ours(args):
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=torch.device("cuda", local))
     wl = synth.workload(args.workload)
-    arm = Arm(wl, rank, world, torch=torch, c2kv=c2kv)
+    arm = Arm(wl, rank, world, torch=torch, c2kv=c2kv, attn_split=args.attn_split)
     f = arm.facts
     E = torch.cuda.Event
 
@@ -321,7 +321,8 @@ def run_ours(args):
     c_ms = statistics.mean(compose_ms)
     a_ms = statistics.mean(attend_ms)
     kc_ms = kern["compose"][0] or c_ms         # compose kernel alone (library events)
-    ka_ms = kern["attention"][0] or a_ms       # attention kernel alone
+    # attention kernel (plus the merge of its key-range splits, when it was split)
+    ka_ms = (kern["attention"][0] + kern["combine"][0]) or a_ms
     comp_gbs = f["compose_bytes"] / (kc_ms / 1e3) / 1e9
     attn_tfs = f["attn_flops"] / (ka_ms / 1e3) / 1e12
     clk = clocks.summary()
@@ -447,6 +448,8 @@ def main():
     ap.add_argument("--workload", default="llama8b", choices=sorted(synth.WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-budget", type=float, default=15.0)
+    ap.add_argument("--attn-split", type=int, default=0,
+                    help="key-range splits of the attention (0 = library's choice)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

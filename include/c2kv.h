@@ -75,6 +75,10 @@ typedef struct c2kv_config {
     int32_t fixed_pos;         /* 1 = no re-rotation at compose ("Fixed-Pos." ablation,
                                   Sec. 4.8): slots keep their chunk-local positions          */
     int32_t attn_impl;         /* C2KV_ATTN_AUTO / _SIMT / _TC                                */
+    int32_t attn_split;        /* tensor-core attention key-range splits per work unit:
+                                  0 = chosen per call (split only when the units would leave
+                                  most SMs idle), 1 = never, n <= 16 = always n (partials
+                                  merged by an exact log-sum-exp combine)                     */
 } c2kv_config;
 
 /* Chunk metadata (c2kv_chunk_info). */
@@ -262,7 +266,8 @@ const char* c2kv_last_error(const c2kv_ctx* ctx);
 #define C2KV_PROF_COMPRESS 1
 #define C2KV_PROF_SUFFIX   2   /* suffix RoPE + append + pad zeroing */
 #define C2KV_PROF_ATTN     3   /* the attention kernel alone */
-#define C2KV_PROF_KINDS    4
+#define C2KV_PROF_COMBINE  4   /* merge of key-range splits (when attention was split) */
+#define C2KV_PROF_KINDS    5
 c2kv_status c2kv_profile_enable(c2kv_ctx* ctx, int32_t on);
 /* mean_ms[C2KV_PROF_KINDS] receives mean milliseconds (0 where none), launches[] the
  * counts; either may be NULL. */

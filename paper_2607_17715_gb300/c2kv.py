@@ -29,8 +29,8 @@ ERR_POSITIONS, ERR_CUDA, ERR_DEVICE_BOUNDS, ERR_STATE, ERR_UNSUPPORTED = -6, -7,
 DTYPE_BF16, DTYPE_F32 = 0, 1
 MODE_MEANPOOL, MODE_PROVIDED, MODE_STORED = 0, 1, 2
 ATTN_AUTO, ATTN_SIMT, ATTN_TC = 0, 1, 2
-PROF_COMPOSE, PROF_COMPRESS, PROF_SUFFIX, PROF_ATTN, PROF_KINDS = 0, 1, 2, 3, 4
-PROF_NAMES = ("compose", "compress", "suffix", "attention")
+PROF_COMPOSE, PROF_COMPRESS, PROF_SUFFIX, PROF_ATTN, PROF_COMBINE, PROF_KINDS = 0, 1, 2, 3, 4, 5
+PROF_NAMES = ("compose", "compress", "suffix", "attention", "combine")
 
 STATUS_NAMES = {
     0: "OK", -1: "ERR_ARG", -2: "ERR_DTYPE", -3: "ERR_NOMEM", -4: "ERR_POOL_FULL",
@@ -44,7 +44,7 @@ class c2kv_config(ctypes.Structure):
                 ("n_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
                 ("rope_theta", ctypes.c_double), ("dtype", ctypes.c_int32),
                 ("pool_slots", ctypes.c_int32), ("fixed_pos", ctypes.c_int32),
-                ("attn_impl", ctypes.c_int32)]
+                ("attn_impl", ctypes.c_int32), ("attn_split", ctypes.c_int32)]
 
 
 class c2kv_chunk_desc(ctypes.Structure):
@@ -141,9 +141,9 @@ def c2kv_last_error(ctx=None) -> str:
 
 
 def c2kv_create(layers, n_q_heads, n_kv_heads, head_dim, rope_theta, dtype, pool_slots,
-                fixed_pos=0, attn_impl=ATTN_AUTO, stream=None):
+                fixed_pos=0, attn_impl=ATTN_AUTO, stream=None, attn_split=0):
     cfg = c2kv_config(layers, n_q_heads, n_kv_heads, head_dim, float(rope_theta), dtype,
-                      pool_slots, int(fixed_pos), attn_impl)
+                      pool_slots, int(fixed_pos), attn_impl, attn_split)
     out = _VP()
     _check(_lib.c2kv_create(ctypes.byref(cfg), _stream_handle(stream), ctypes.byref(out)))
     return out.value

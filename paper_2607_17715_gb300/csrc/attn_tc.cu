@@ -75,7 +75,9 @@ struct TcParams {                // CUtensorMap members carry their own alignmen
     int64_t rows;
     int32_t layer0, lq, batch, batch_total, b0, sq, hq, hkv, group, tq;
     float scale_log2;
-    int32_t pad;
+    int32_t n_split;
+    float* part_o;
+    float* part_lse;
     ReqParam req[kMaxReq];
 };
 
@@ -262,9 +264,15 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_const
     const int bl = blockIdx.z - l * P.batch;
     const int b = P.b0 + bl;
     const int s_r = P.req[bl].n_slots;
-    const int t0 = blockIdx.x * P.tq;
+    const int mt = blockIdx.x / P.n_split;          // Q tile
+    const int sp = blockIdx.x - mt * P.n_split;     // key-range split
+    const int t0 = mt * P.tq;
     const int t_last = min(P.sq - 1, t0 + P.tq - 1);
-    const int n_kv = (s_r + t_last + 1 + BN - 1) / BN;
+    const int n_kv_all = (s_r + t_last + 1 + BN - 1) / BN;
+    // this CTA's key tiles: [j_base, j_base + n_kv) of the request's n_kv_all
+    const int per_split = (n_kv_all + P.n_split - 1) / P.n_split;
+    const int j_base = sp * per_split;
+    const int n_kv = max(0, min(n_kv_all, j_base + per_split) - j_base);
 
     if (threadIdx.x == 0) {
         mbar_init(bar(B_Q), 1);
@@ -306,7 +314,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_const
             mbar_expect_tx(bar(B_Q), TILE);
             tma_load_4d(sQ, &P.tm_q, 0, hk * G, t0, qz, bar(B_Q));
             tma_load_4d(sQ + HALF_TILE, &P.tm_q, 64, hk * G, t0, qz, bar(B_Q));
-            const int key0 = (int)((int64_t)(P.layer0 + l) * P.rows + P.req[bl].row_base);
+            const int key0 = (int)((int64_t)(P.layer0 + l) * P.rows + P.req[bl].row_base) + j_base * BN;
             // two independent queues: a K load waits only for its own K stage
             int jk = 0, jv = 0;
             while (jk < n_kv || jv < n_kv) {
@@ -404,7 +412,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_const
             tc_fence_before();
             mbar_arrive(bar(B_SFREE + sb));
 
-            const int kbase = j * BN;
+            const int kbase = (j_base + j) * BN;
             if (kbase + BN - 1 > lim) {
 #pragma unroll
                 for (int c = 0; c < 4; ++c)
@@ -424,9 +432,10 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_const
             const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
                                    fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
             const float m_new = fmaxf(m_run, mx * sc);
-            const bool resc = m_new > m_run + 8.0f;       // also true on the first tile
+            const bool resc = m_new > m_run + 8.0f;       // false while nothing is visible
             const float m_use = resc ? m_new : m_run;
             const float alpha = resc ? ex2(m_run - m_new) : 1.0f;
+            const float m_sub = m_use == -CUDART_INF_F ? 0.f : m_use;   // all masked so far
 
             const int pb = j & 1;
             // P buffer pb is free once P_{j-2}.V_{j-2} has finished
@@ -459,8 +468,8 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_const
                     const int c = half * 2 + cc;
 #pragma unroll
                     for (int e = 0; e < 32; e += 2) {
-                        const float a0 = ex2(fmaf(__uint_as_float(sv[c][e]), sc, -m_use));
-                        const float a1 = ex2(fmaf(__uint_as_float(sv[c][e + 1]), sc, -m_use));
+                        const float a0 = ex2(fmaf(__uint_as_float(sv[c][e]), sc, -m_sub));
+                        const float a1 = ex2(fmaf(__uint_as_float(sv[c][e + 1]), sc, -m_sub));
                         ps[e & 7] += a0;
                         ps[(e + 1) & 7] += a1;
                         pk[cc * 16 + (e >> 1)] = pack_bf16(a0, a1);
@@ -477,33 +486,63 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_const
         }
 
         // ---------------------------------------------------------------- epilogue
-        mbar_wait(bar(B_PFREE + ((n_kv - 1) & 1)), (uint32_t)((n_kv - 1) >> 1) & 1u, P.err);
-        tc_fence_after();
+        if (n_kv > 0) {
+            mbar_wait(bar(B_PFREE + ((n_kv - 1) & 1)), (uint32_t)((n_kv - 1) >> 1) & 1u, P.err);
+            tc_fence_after();
+        }
         const int t = t0 + r / G;
         const int g = r - (r / G) * G;
-        const float inv = 1.0f / l_run;
-        __nv_bfloat16* orow = static_cast<__nv_bfloat16*>(P.out) +
-                              ((((int64_t)l * P.batch_total + b) * P.sq + t) * P.hq + hk * G + g) * HD;
+        const bool any = l_run > 0.f;                 // some key of this split was visible
+        const float inv = any ? 1.0f / l_run : 0.f;
+        const int64_t row_id = (((int64_t)l * P.batch_total + b) * P.sq + t) * P.hq + hk * G + g;
+        const int64_t lse_id = (((int64_t)l * P.batch_total + b) * P.hq + hk * G + g) * P.sq + t;
+        if (P.n_split == 1) {
+            __nv_bfloat16* orow = static_cast<__nv_bfloat16*>(P.out) + row_id * HD;
 #pragma unroll
-        for (int c = 0; c < 4; ++c) {
-            uint32_t ov[32];
-            tmem_ld32(tmem + lane_addr + kColO + c * 32, ov);
-            tmem_ld_wait();
-            if (t < P.sq) {
+            for (int c = 0; c < 4; ++c) {
+                uint32_t ov[32];
+                tmem_ld32(tmem + lane_addr + kColO + c * 32, ov);
+                tmem_ld_wait();
+                if (t < P.sq) {
 #pragma unroll
-                for (int q8 = 0; q8 < 4; ++q8) {
-                    uint4 w;
-                    w.x = pack_bf16(__uint_as_float(ov[q8 * 8 + 0]) * inv, __uint_as_float(ov[q8 * 8 + 1]) * inv);
-                    w.y = pack_bf16(__uint_as_float(ov[q8 * 8 + 2]) * inv, __uint_as_float(ov[q8 * 8 + 3]) * inv);
-                    w.z = pack_bf16(__uint_as_float(ov[q8 * 8 + 4]) * inv, __uint_as_float(ov[q8 * 8 + 5]) * inv);
-                    w.w = pack_bf16(__uint_as_float(ov[q8 * 8 + 6]) * inv, __uint_as_float(ov[q8 * 8 + 7]) * inv);
-                    *reinterpret_cast<uint4*>(orow + c * 32 + q8 * 8) = w;
+                    for (int q8 = 0; q8 < 4; ++q8) {
+                        uint4 w;
+                        w.x = pack_bf16(__uint_as_float(ov[q8 * 8 + 0]) * inv, __uint_as_float(ov[q8 * 8 + 1]) * inv);
+                        w.y = pack_bf16(__uint_as_float(ov[q8 * 8 + 2]) * inv, __uint_as_float(ov[q8 * 8 + 3]) * inv);
+                        w.z = pack_bf16(__uint_as_float(ov[q8 * 8 + 4]) * inv, __uint_as_float(ov[q8 * 8 + 5]) * inv);
+                        w.w = pack_bf16(__uint_as_float(ov[q8 * 8 + 6]) * inv, __uint_as_float(ov[q8 * 8 + 7]) * inv);
+                        *reinterpret_cast<uint4*>(orow + c * 32 + q8 * 8) = w;
+                    }
                 }
             }
+            if (P.lse != nullptr && t < P.sq)
+                P.lse[lse_id] = (m_run + log2f(l_run)) * 0.69314718055994531f;
+        } else {
+            // partial over this split's keys: normalised O (fp32) and its log2-domain lse
+            const int64_t part_rows = (int64_t)P.lq * P.batch_total * P.sq * P.hq;
+            float* orow = P.part_o + ((int64_t)sp * part_rows + row_id) * HD;
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                uint32_t ov[32];
+                if (n_kv > 0) {
+                    tmem_ld32(tmem + lane_addr + kColO + c * 32, ov);
+                    tmem_ld_wait();
+                } else {
+#pragma unroll
+                    for (int e = 0; e < 32; ++e) ov[e] = 0u;
+                }
+                if (t < P.sq) {
+#pragma unroll
+                    for (int q4 = 0; q4 < 8; ++q4) {
+                        float4 w = make_float4(__uint_as_float(ov[q4 * 4 + 0]) * inv, __uint_as_float(ov[q4 * 4 + 1]) * inv,
+                                               __uint_as_float(ov[q4 * 4 + 2]) * inv, __uint_as_float(ov[q4 * 4 + 3]) * inv);
+                        *reinterpret_cast<float4*>(orow + c * 32 + q4 * 4) = w;
+                    }
+                }
+            }
+            if (t < P.sq)
+                P.part_lse[(int64_t)sp * part_rows + lse_id] = any ? m_run + log2f(l_run) : -CUDART_INF_F;
         }
-        if (P.lse != nullptr && t < P.sq)
-            P.lse[(((int64_t)l * P.batch_total + b) * P.hq + hk * G + g) * P.sq + t] =
-                (m_run + log2f(l_run)) * 0.69314718055994531f;
     }
 
     tc_fence_before();
@@ -514,6 +553,55 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_const
                      "r"(kTmemCols)
                      : "memory");
     }
+}
+
+// Merge the splits: lse = log2 sum_s 2^lse_s, O = sum_s 2^(lse_s - lse) O_s.  One warp per
+// (layer, request, suffix token, query head) row; lane i owns head channels 4i .. 4i+3.
+// Every split's lse and O slice is loaded before any is used (at most kMaxSplit), so the
+// loads of one row are all in flight together.
+constexpr int kMaxSplit = 16;
+
+__global__ void __launch_bounds__(256) attn_combine_kernel(const __grid_constant__ AttnParams P) {
+    const int64_t rows = (int64_t)P.lq * P.batch_total * P.sq * P.hq;
+    const int64_t row = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+    const int lane = threadIdx.x & 31;
+    if (row >= rows) return;
+    const int h = (int)(row % P.hq);
+    const int64_t lbt = row / P.hq;                 // (l * Btot + b) * Sq + t
+    const int t = (int)(lbt % P.sq);
+    const int64_t lb = lbt / P.sq;
+    const int64_t lse_id = (lb * P.hq + h) * P.sq + t;
+    float ls[kMaxSplit];
+    float4 o[kMaxSplit];
+#pragma unroll
+    for (int s = 0; s < kMaxSplit; ++s) {
+        ls[s] = -CUDART_INF_F;
+        o[s] = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (s < P.n_split) {
+            ls[s] = P.part_lse[(int64_t)s * rows + lse_id];
+            o[s] = *reinterpret_cast<const float4*>(P.part_o + ((int64_t)s * rows + row) * HD + lane * 4);
+        }
+    }
+    float mx = -CUDART_INF_F;
+#pragma unroll
+    for (int s = 0; s < kMaxSplit; ++s) mx = fmaxf(mx, ls[s]);
+    float wsum = 0.f;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+    for (int s = 0; s < kMaxSplit; ++s) {
+        const float w = ls[s] == -CUDART_INF_F ? 0.f : ex2(ls[s] - mx);
+        acc.x += w * o[s].x;
+        acc.y += w * o[s].y;
+        acc.z += w * o[s].z;
+        acc.w += w * o[s].w;
+        wsum += w;
+    }
+    const float inv = 1.0f / wsum;
+    uint2 pk;
+    pk.x = pack_bf16(acc.x * inv, acc.y * inv);
+    pk.y = pack_bf16(acc.z * inv, acc.w * inv);
+    *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(P.out) + row * HD + lane * 4) = pk;
+    if (P.lse != nullptr && lane == 0) P.lse[lse_id] = (mx + log2f(wsum)) * 0.69314718055994531f;
 }
 
 // ------------------------------------------------------------------ host side
@@ -544,6 +632,21 @@ bool encode(CUtensorMap* tm, const void* base, int rank, const cuuint64_t* dims,
 }
 
 }  // namespace
+
+int64_t attn_tc_units(const AttnParams& a) {
+    const int tq = BM / (a.hq / a.hkv);
+    return (int64_t)((a.sq + tq - 1) / tq) * a.hkv * a.lq * a.batch;
+}
+
+cudaError_t launch_attn_combine(const AttnParams& a, cudaStream_t s) {
+    (void)cudaGetLastError();
+    if (a.n_split > kMaxSplit) return cudaErrorInvalidValue;
+    const int64_t rows = (int64_t)a.lq * a.batch_total * a.sq * a.hq;
+    const int64_t blocks = (rows + 7) / 8;
+    if (blocks > 0x7fffffffLL) return cudaErrorInvalidValue;
+    attn_combine_kernel<<<(unsigned)blocks, 256, 0, s>>>(a);
+    return cudaGetLastError();
+}
 
 bool attn_tc_supported(int dtype, int d, int hq, int hkv) {
     if (dtype != kDtypeBf16 || d != HD || hkv < 1 || hq % hkv) return false;
@@ -591,8 +694,13 @@ cudaError_t launch_attn_tc(const AttnParams& a, cudaStream_t s) {
     p.group = G;
     p.tq = tq;
     p.scale_log2 = a.scale_log2;
+    p.n_split = a.n_split < 1 ? 1 : a.n_split;
+    p.part_o = a.part_o;
+    p.part_lse = a.part_lse;
     std::memcpy(p.req, a.req, sizeof(ReqParam) * (size_t)a.batch);
-    const dim3 grid((a.sq + tq - 1) / tq, a.hkv, a.lq * a.batch);
+    const int64_t gx = (int64_t)((a.sq + tq - 1) / tq) * p.n_split;
+    if (gx > 0x7fffffffLL) return cudaErrorInvalidValue;
+    const dim3 grid((unsigned)gx, a.hkv, a.lq * a.batch);
     if (grid.z > 65535u || grid.y > 65535u) return cudaErrorInvalidValue;
     attn_tc_kernel<<<grid, kThreads, kSmemBytes, s>>>(p);
     return cudaGetLastError();

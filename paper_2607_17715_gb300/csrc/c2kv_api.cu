@@ -58,6 +58,7 @@ struct c2kv_ctx {
     cudaMemPool_t mempool = nullptr;
     std::vector<c2kv_cache*> caches;
     int32_t inject = 0;
+    int sms = 148;
     c2kv::RopeTurns turns{};
     // tracing (c2kv_profile_enable): event pairs around launches, by kind
     bool prof = false;
@@ -221,6 +222,8 @@ c2kv_status c2kv_create(const c2kv_config* cfg, void* stream, c2kv_ctx** out) {
         if (f.pool_slots < 1) return fail(nullptr, C2KV_ERR_ARG, "create: pool_slots < 1");
         if (f.attn_impl < C2KV_ATTN_AUTO || f.attn_impl > C2KV_ATTN_TC)
             return fail(nullptr, C2KV_ERR_ARG, "create: bad attn_impl");
+        if (f.attn_split < 0 || f.attn_split > 16)
+            return fail(nullptr, C2KV_ERR_ARG, "create: attn_split outside [0, 16]");
         if (f.attn_impl == C2KV_ATTN_TC &&
             !c2kv::attn_tc_supported(f.dtype, f.head_dim, f.n_q_heads, f.n_kv_heads))
             return fail(nullptr, C2KV_ERR_UNSUPPORTED,
@@ -230,6 +233,7 @@ c2kv_status c2kv_create(const c2kv_config* cfg, void* stream, c2kv_ctx** out) {
         c->stream = static_cast<cudaStream_t>(stream);
         c->eb = f.dtype == C2KV_DTYPE_BF16 ? 2 : 4;
         cudaError_t e = cudaGetDevice(&c->device);
+        if (e == cudaSuccess) e = cudaDeviceGetAttribute(&c->sms, cudaDevAttrMultiProcessorCount, c->device);
         const size_t pool_bytes = (size_t)f.layers * (size_t)f.pool_slots * (size_t)row_elems(c) * c->eb;
         if (e == cudaSuccess) e = cudaMalloc(&c->pool_k, pool_bytes);
         if (e == cudaSuccess) e = cudaMalloc(&c->pool_v, pool_bytes);
@@ -548,6 +552,37 @@ c2kv_status c2kv_attend(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
         void* q_rot = nullptr;
         cudaError_t e = pool_alloc(c, &q_rot, q_bytes);
         if (e != cudaSuccess) return cuda_fail(c, e, "attend: scratch allocation");
+        // Key-range split of the tensor-core attention: when its work units would leave most
+        // SMs idle (a single layer of a small batch), each unit's key tiles are split and the
+        // partials merged; at a wave or more the split only adds the merge.
+        int32_t n_split = 1;
+        float* part = nullptr;
+        if (use_tc) {
+            const int64_t tq = 128 / (c->cfg.n_q_heads / c->cfg.n_kv_heads);
+            const int64_t units = (n_suffix + tq - 1) / tq * c->cfg.n_kv_heads * lq * B;
+            int32_t n_kv_max = 1;
+            for (int32_t b = 0; b < B; ++b)
+                n_kv_max = std::max<int32_t>(n_kv_max, (cache->n_slots[b] + n_suffix + 127) / 128);
+            if (c->cfg.attn_split >= 1) {
+                n_split = c->cfg.attn_split;
+            } else if (2 * units <= c->sms) {
+                // at most half of the SMs would have work: split toward one wave, keeping at
+                // least 8 key tiles per split (below that the merge costs more than it saves)
+                n_split = (int32_t)std::min<int64_t>(16, c->sms / units);
+                n_split = std::max<int32_t>(1, std::min<int32_t>(n_split, n_kv_max / 8));
+            }
+            if (n_split > 1) {
+                const size_t rows = (size_t)lq * B * n_suffix * c->cfg.n_q_heads;
+                e = pool_alloc(c, reinterpret_cast<void**>(&part),
+                               (size_t)n_split * rows * (c->cfg.head_dim + 1) * sizeof(float));
+                if (e != cudaSuccess) {
+                    pool_free(c, q_rot);
+                    return cuda_fail(c, e, "attend: split scratch allocation");
+                }
+            }
+        }
+        const size_t part_rows = (size_t)lq * B * n_suffix * c->cfg.n_q_heads;
+        c2kv::AttnParams last{};
         for (int32_t b0 = 0; e == cudaSuccess && b0 < B; b0 += c2kv::kMaxReq) {
             const int32_t nb = std::min<int32_t>(c2kv::kMaxReq, B - b0);
             c2kv::SuffixParams s{};
@@ -593,11 +628,20 @@ c2kv_status c2kv_attend(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
             a.hq = c->cfg.n_q_heads;
             a.hkv = c->cfg.n_kv_heads;
             a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)c->cfg.head_dim));
+            a.n_split = n_split;
+            a.part_o = part;
+            a.part_lse = part ? part + (size_t)n_split * part_rows * c->cfg.head_dim : nullptr;
             for (int32_t i = 0; i < nb; ++i) a.req[i] = s.req[i];
             ProfScope prof_attn(c, C2KV_PROF_ATTN);
             e = use_tc ? c2kv::launch_attn_tc(a, c->stream)
                        : c2kv::launch_attn_simt(a, c->cfg.dtype, c->cfg.head_dim, c->stream);
+            last = a;
         }
+        if (e == cudaSuccess && n_split > 1) {   // one merge over every request's rows
+            ProfScope prof_combine(c, C2KV_PROF_COMBINE);
+            e = c2kv::launch_attn_combine(last, c->stream);
+        }
+        pool_free(c, part);
         pool_free(c, q_rot);
         if (e != cudaSuccess) return cuda_fail(c, e, "attend");
         return C2KV_OK;

@@ -117,7 +117,9 @@ struct AttnParams {
     int32_t hq;
     int32_t hkv;
     float scale_log2;        // log2(e) / sqrt(d)
-    int32_t pad;
+    int32_t n_split;         // key-range splits per work unit (1 = write O directly)
+    float* part_o;           // n_split > 1: [n_split][Lq][Btot][Sq][Hq][d] fp32, normalised
+    float* part_lse;         // n_split > 1: [n_split][Lq][Btot][Hq][Sq] fp32, log2 domain
     ReqParam req[kMaxReq];
 };
 
@@ -130,6 +132,10 @@ cudaError_t launch_attn_simt(const AttnParams& p, int dtype, int d, cudaStream_t
 // Tensor-core attention (attn_tc.cu).
 bool attn_tc_supported(int dtype, int d, int hq, int hkv);
 cudaError_t launch_attn_tc(const AttnParams& p, cudaStream_t s);
+// Merge n_split partial (O, lse) over disjoint key ranges into out (bf16) and lse (attn_tc.cu).
+cudaError_t launch_attn_combine(const AttnParams& p, cudaStream_t s);
+// Work units (CTAs per split) the tensor-core kernel launches for these parameters.
+int64_t attn_tc_units(const AttnParams& p);
 
 // Read-only view of a context and one of its caches, for entry points defined outside
 // c2kv_api.cu (c2kv_attend_noalloc).

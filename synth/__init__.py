@@ -15,7 +15,7 @@ Workload shapes
                   ratio 4, offsets 0/128/256/384, 32 suffix tokens.
 ``llama8b``       Llama-3-8B layer: Hq 32 / Hkv 8, d 128, theta 5e5, bf16; 10 chunks x 512
                   tokens, ratio 4 (5120 composed positions), 64 suffix tokens, batch 1;
-                  32 layers when timed as a whole model.
+                  32 layers when timed as a whole model (``llama8b_l1``: one layer).
 ``batched``       pool of 256 chunks x 512 tokens (ratio 4); 16 requests, each 8 distinct
                   chunks drawn Zipf(s=1.1), random order; 128 suffix tokens.
 ``long70b``       Llama-3-70B layer: Hq 64 / Hkv 8, d 128; 32 chunks x 1024 tokens,
@@ -74,6 +74,8 @@ WORKLOADS = {
     "long70b": Workload("long70b", 1, 64, 8, 128, 5.0e5, "bf16", 1024, 16, 256, 2, 32, 64,
                         "distinct"),
 }
+# the same Llama-3-8B workload timed one layer at a time (per-layer TTFT proxy)
+WORKLOADS["llama8b_l1"] = dataclasses.replace(WORKLOADS["llama8b"], name="llama8b_l1", layers=1)
 for _k in SWEEP_RATIOS:
     WORKLOADS[f"sweep_k{_k}"] = Workload(f"sweep_k{_k}", 1, 32, 8, 128, 5.0e5, "bf16", 2048,
                                          _k, 128, 8, 16, 128, "distinct")

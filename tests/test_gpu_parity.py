@@ -183,7 +183,7 @@ def test_compose_empty_request_in_batch():
 
 # ------------------------------------------------------------------ attend
 
-def _attend_case(wl, attn_impl=0, layer=-1, n_suffix=None, requests=None):
+def _attend_case(wl, attn_impl=0, layer=-1, n_suffix=None, requests=None, attn_split=0):
     """End to end: oracle-stored chunks -> GPU compose -> GPU attend, vs oracle compose +
     attend on the same inputs.  Checks O, lse, and the suffix rows written to the cache."""
     c2kv = H.lib()
@@ -193,7 +193,8 @@ def _attend_case(wl, attn_impl=0, layer=-1, n_suffix=None, requests=None):
     all_ids = sorted({c for ids, _ in reqs for c in ids})
     chunks = H.oracle_chunks_meanpool(wl, all_ids)
     ctx = H.make_ctx(wl, pool_slots=sum(orc.n_slots(wl.chunk_tokens, wl.ratio_k)
-                                        for _ in all_ids) + 16, attn_impl=attn_impl)
+                                        for _ in all_ids) + 16, attn_impl=attn_impl,
+                       attn_split=attn_split)
     try:
         dev = H.load_stored(ctx, wl, chunks)
         req_ptr = np.cumsum([0] + [len(ids) for ids, _ in reqs])
@@ -275,3 +276,18 @@ def test_attend_single_chunk_k1_offset0_is_causal_attention():
     wl = _small(L8B_1, chunk_tokens=200, ratio_k=1, chunks_per_request=1, pool_chunks=1,
                 n_suffix=50)
     _attend_case(wl)
+
+
+@pytest.mark.parametrize("split", [1, 3, 7])
+def test_attend_key_range_splits(split):
+    # one short chunk and a long suffix: 3 key tiles, so with 7 splits four are empty, and
+    # the last non-empty split sees no visible key for the early suffix rows
+    wl = _small(L8B_1, chunks_per_request=1, pool_chunks=1, chunk_tokens=64, ratio_k=4,
+                n_suffix=300)
+    _attend_case(wl, attn_split=split)
+
+
+def test_attend_forced_split_batched():
+    wl = _small(synth.workload("batched"), batch=3, chunks_per_request=4, pool_chunks=32,
+                n_suffix=40)
+    _attend_case(wl, attn_split=5)
