@@ -54,6 +54,7 @@ typedef int32_t c2kv_status;
 #define C2KV_MODE_MEANPOOL 0  /* tokens -> slots: block mean of pre-RoPE K/V rows            */
 #define C2KV_MODE_PROVIDED 1  /* slots given pre-RoPE by an external extractor               */
 #define C2KV_MODE_STORED   2  /* slots given already in stored form (load from host storage) */
+#define C2KV_MODE_HOST     3  /* stored-form slots that stay in pinned host memory (no copy)   */
 
 /* c2kv_attend kernel choice */
 #define C2KV_ATTN_AUTO   0    /* tensor-core kernel where it applies, SIMT otherwise */
@@ -143,6 +144,12 @@ c2kv_status c2kv_set_stream(c2kv_ctx* ctx, void* stream);
  *              extractor (the paper's C2 token K/V, Sec. 3.2.2); K is turned to p_j.
  *              STORED: host or device [L][m][Hkv][d] slots already in stored form (K at
  *              p_j), copied verbatim -- the "load from host memory" step of Appendix C.
+ *              HOST: the same stored form in pinned, device-mapped host memory, NOT copied:
+ *              the chunk takes no pool slots and c2kv_compose reads it over the host link
+ *              (load, re-rotation and gather in one pass).  The caller keeps the memory
+ *              valid and unchanged until the chunk is freed.  ERR_ARG if k or v is not
+ *              pinned (cudaHostAlloc / cudaHostRegister) or does not start on a 16-byte
+ *              boundary; the whole L*m*Hkv*d span must lie in the pinned allocation.
  *   n_tokens : original chunk length n >= 1.
  *   ratio_k  : compression ratio k >= 1 (k = 1: uncompressed control).
  *   mode     : C2KV_MODE_*.

@@ -27,7 +27,7 @@ OK = 0
 ERR_ARG, ERR_DTYPE, ERR_NOMEM, ERR_POOL_FULL, ERR_BAD_CHUNK = -1, -2, -3, -4, -5
 ERR_POSITIONS, ERR_CUDA, ERR_DEVICE_BOUNDS, ERR_STATE, ERR_UNSUPPORTED = -6, -7, -8, -9, -10
 DTYPE_BF16, DTYPE_F32 = 0, 1
-MODE_MEANPOOL, MODE_PROVIDED, MODE_STORED = 0, 1, 2
+MODE_MEANPOOL, MODE_PROVIDED, MODE_STORED, MODE_HOST = 0, 1, 2, 3
 ATTN_AUTO, ATTN_SIMT, ATTN_TC = 0, 1, 2
 PROF_COMPOSE, PROF_COMPRESS, PROF_SUFFIX, PROF_ATTN, PROF_COMBINE, PROF_KINDS = 0, 1, 2, 3, 4, 5
 PROF_NAMES = ("compose", "compress", "suffix", "attention", "combine")

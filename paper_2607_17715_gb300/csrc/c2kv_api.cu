@@ -12,6 +12,7 @@
 #include <algorithm>
 #include <cmath>
 #include <cstdarg>
+#include <cstdint>
 #include <cstdio>
 #include <cstring>
 #include <map>
@@ -27,6 +28,9 @@ constexpr int64_t kTileRows = 128;   // composed-cache request regions align to 
 struct Chunk {
     int32_t n = 0, k = 0, m = 0, base = 0;
     bool live = false;
+    bool host = false;                  // registered in host memory (C2KV_MODE_HOST)
+    const void* host_k = nullptr;       // device-accessible addresses of the host slots
+    const void* host_v = nullptr;
 };
 
 thread_local std::string g_create_error;
@@ -303,8 +307,45 @@ c2kv_status c2kv_compress_chunk(c2kv_ctx* c, const void* k, const void* v, int32
         c->err.clear();
         if (!k || !v || !chunk_id_out) return fail(c, C2KV_ERR_ARG, "compress: null pointer");
         if (n_tokens < 1 || ratio_k < 1) return fail(c, C2KV_ERR_ARG, "compress: need n >= 1, k >= 1");
-        if (mode != C2KV_MODE_MEANPOOL && mode != C2KV_MODE_PROVIDED && mode != C2KV_MODE_STORED)
+        if (mode != C2KV_MODE_MEANPOOL && mode != C2KV_MODE_PROVIDED && mode != C2KV_MODE_STORED &&
+            mode != C2KV_MODE_HOST)
             return fail(c, C2KV_ERR_ARG, "compress: bad mode %d", mode);
+        if (mode == C2KV_MODE_HOST) {
+            // no copy: keep the device-accessible addresses of the caller's pinned slots
+            const void* dk = nullptr;
+            const void* dv = nullptr;
+            for (int w = 0; w < 2; ++w) {
+                cudaPointerAttributes at{};
+                const void* p = w ? v : k;
+                if (cudaPointerGetAttributes(&at, p) != cudaSuccess || at.type != cudaMemoryTypeHost ||
+                    at.devicePointer == nullptr) {
+                    (void)cudaGetLastError();
+                    return fail(c, C2KV_ERR_ARG, "compress: HOST mode needs pinned, device-mapped host memory");
+                }
+                if (reinterpret_cast<uintptr_t>(at.devicePointer) % 16 != 0)
+                    return fail(c, C2KV_ERR_ARG, "compress: HOST mode slots must start on a 16-byte boundary");
+                (w ? dv : dk) = at.devicePointer;
+            }
+            int32_t id = -1;
+            for (size_t i = 0; i < c->chunks.size(); ++i)
+                if (!c->chunks[i].live) { id = (int32_t)i; break; }
+            if (id < 0) {
+                c->chunks.emplace_back();
+                id = (int32_t)c->chunks.size() - 1;
+            }
+            Chunk& ch = c->chunks[id];
+            ch = Chunk{};
+            ch.n = n_tokens;
+            ch.k = ratio_k;
+            ch.m = (int32_t)(((int64_t)n_tokens + ratio_k - 1) / ratio_k);
+            ch.base = -1;
+            ch.live = true;
+            ch.host = true;
+            ch.host_k = dk;
+            ch.host_v = dv;
+            *chunk_id_out = id;
+            return C2KV_OK;
+        }
         if (mode != C2KV_MODE_STORED && (!is_device_ptr(k) || !is_device_ptr(v)))
             return fail(c, C2KV_ERR_ARG, "compress: MEANPOOL/PROVIDED inputs must be device memory");
         const int32_t m = (int32_t)(((int64_t)n_tokens + ratio_k - 1) / ratio_k);
@@ -353,6 +394,7 @@ c2kv_status c2kv_compress_chunk(c2kv_ctx* c, const void* k, const void* v, int32
             id = (int32_t)c->chunks.size() - 1;
         }
         Chunk& ch = c->chunks[id];
+        ch = Chunk{};
         ch.n = n_tokens;
         ch.k = ratio_k;
         ch.m = m;
@@ -371,7 +413,7 @@ c2kv_status c2kv_free_chunk(c2kv_ctx* c, int32_t id) {
     if (id < 0 || id >= (int32_t)c->chunks.size() || !c->chunks[id].live)
         return fail(c, C2KV_ERR_BAD_CHUNK, "free_chunk: unknown chunk %d", id);
     Chunk& ch = c->chunks[id];
-    give_range(c, ch.base, ch.m);
+    if (!ch.host) give_range(c, ch.base, ch.m);
     ch.live = false;
     return C2KV_OK;
 }
@@ -385,9 +427,15 @@ c2kv_status c2kv_chunk_info(const c2kv_ctx* c, int32_t id, c2kv_chunk_desc* out)
     out->ratio_k = ch.k;
     out->n_slots = ch.m;
     out->slot_base = ch.base;
-    out->k = static_cast<char*>(c->pool_k) + (size_t)ch.base * rb;
-    out->v = static_cast<char*>(c->pool_v) + (size_t)ch.base * rb;
-    out->layer_stride = (int64_t)c->cfg.pool_slots * row_elems(c);
+    if (ch.host) {
+        out->k = const_cast<void*>(ch.host_k);
+        out->v = const_cast<void*>(ch.host_v);
+        out->layer_stride = (int64_t)ch.m * row_elems(c);
+    } else {
+        out->k = static_cast<char*>(c->pool_k) + (size_t)ch.base * rb;
+        out->v = static_cast<char*>(c->pool_v) + (size_t)ch.base * rb;
+        out->layer_stride = (int64_t)c->cfg.pool_slots * row_elems(c);
+    }
     return C2KV_OK;
 }
 
@@ -447,7 +495,9 @@ c2kv_status c2kv_compose(c2kv_ctx* c, int32_t batch, const int32_t* req_ptr,
                 rec.k = ch.k;
                 rec.m = ch.m;
                 rec.tile_base = 0;
-                rec.pad = 0;
+                rec.host = ch.host ? 1 : 0;
+                rec.host_k = ch.host_k;
+                rec.host_v = ch.host_v;
                 slots += ch.m;
             }
             const int64_t cap = (slots + suffix_capacity + kTileRows - 1) / kTileRows * kTileRows;

@@ -14,7 +14,7 @@ namespace c2kv {
 constexpr int kDtypeBf16 = 0;
 constexpr int kDtypeF32 = 1;
 constexpr int kMaxHalf = 64;        // head_dim / 2 for head_dim <= 128
-constexpr int kMaxOcc = 128;        // chunk occurrences per compose launch
+constexpr int kMaxOcc = 96;         // chunk occurrences per compose launch
 constexpr int kMaxReq = 256;        // requests per suffix / attention launch
 constexpr int kComposeTile = 16;    // composed slots per compose CTA (per layer)
 
@@ -28,14 +28,16 @@ struct RopeTurns {
 
 // One chunk occurrence of a compose launch.
 struct OccParam {
-    int32_t src_base;    // first pool slot of the chunk
+    int32_t src_base;    // first pool slot of the chunk (pool chunks)
     int32_t dest_row;    // first composed row
     int32_t delta;       // positions to turn by (o_i, or 0 under fixed_pos)
     int32_t n;           // original chunk length
     int32_t k;           // ratio
     int32_t m;           // slots
     int32_t tile_base;   // first compose tile of this occurrence (prefix over the launch)
-    int32_t pad;
+    int32_t host;        // 1: the chunk stays in host memory, read through host_k / host_v
+    const void* host_k;  // device-accessible [L][m][Hkv][d] (host-resident chunks)
+    const void* host_v;
 };
 
 struct ComposeParams {

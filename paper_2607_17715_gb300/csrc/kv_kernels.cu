@@ -134,18 +134,28 @@ __global__ void __launch_bounds__(256) compose_kernel(const __grid_constant__ Co
             const int j = j0 + s;
             const int64_t src = (int64_t)o.src_base + j;
             const int64_t dst = (int64_t)o.dest_row + j;
-            if (src < 0 || src >= P.pool_slots || dst < 0 || dst >= P.rows) {
+            if ((!o.host && (src < 0 || src >= P.pool_slots)) || dst < 0 || dst >= P.rows) {
                 atomicOr(P.err, 1);
                 live[u] = false;
                 continue;
             }
-            const int64_t so = ((int64_t)l * P.pool_slots + src) * row_elems + h * D + iv * E;
             dof[u] = ((int64_t)l * P.rows + dst) * row_elems + h * D + iv * E;
             civ[u] = iv * E;
-            kx[u] = ld16(pk + so);
-            ky[u] = ld16(pk + so + HALF);
-            vx[u] = ld16(pv + so);
-            vy[u] = ld16(pv + so + HALF);
+            const T* sk;
+            const T* sv;
+            if (o.host) {       // host-resident chunk: [L][m][Hkv][d] read over the host link
+                const int64_t so = ((int64_t)l * o.m + j) * row_elems + h * D + iv * E;
+                sk = static_cast<const T*>(o.host_k) + so;
+                sv = static_cast<const T*>(o.host_v) + so;
+            } else {
+                const int64_t so = ((int64_t)l * P.pool_slots + src) * row_elems + h * D + iv * E;
+                sk = pk + so;
+                sv = pv + so;
+            }
+            kx[u] = ld16(sk);
+            ky[u] = ld16(sk + HALF);
+            vx[u] = ld16(sv);
+            vy[u] = ld16(sv + HALF);
             if (l == 0 && p == 0) P.pos[dst] = o.delta + min((j + 1) * o.k, o.n) - 1;
         }
 #pragma unroll

@@ -133,11 +133,19 @@ def oracle_chunks_meanpool(wl, ids):
     return out
 
 
-def load_stored(ctx, wl, chunks):
-    """Put stored-form chunks into the device pool (MODE_STORED); returns pool id map."""
+def load_stored(ctx, wl, chunks, host=(), keep=None):
+    """Register stored-form chunks: copied into the device pool (MODE_STORED), or, for the
+    ids in `host`, left in pinned host memory (MODE_HOST; the pinned tensors are appended to
+    `keep`, which must outlive the chunks).  Returns the library id of every chunk."""
     c2kv = lib()
     ids = {}
     for cid, (ks, vs, n, k) in chunks.items():
-        ids[cid] = c2kv.c2kv_compress_chunk(ctx, to_dev(ks, wl), to_dev(vs, wl), n, k,
-                                            c2kv.MODE_STORED)
+        if cid in host:
+            kh, vh = (torch.from_numpy(np.ascontiguousarray(x, np.float32)).to(tdtype(wl))
+                      .pin_memory() for x in (ks, vs))
+            keep.extend((kh, vh))
+            ids[cid] = c2kv.c2kv_compress_chunk(ctx, kh, vh, n, k, c2kv.MODE_HOST)
+        else:
+            ids[cid] = c2kv.c2kv_compress_chunk(ctx, to_dev(ks, wl), to_dev(vs, wl), n, k,
+                                                c2kv.MODE_STORED)
     return ids

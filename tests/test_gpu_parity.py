@@ -104,15 +104,17 @@ def test_compress_stored_roundtrip_from_host():
 
 # ------------------------------------------------------------------ compose
 
-def _compose_case(wl, requests, fixed_pos=False, pool_slots=4096):
+def _compose_case(wl, requests, fixed_pos=False, pool_slots=4096, host=()):
     """Compose `requests` (list of (ids, offsets)) on the GPU from oracle-stored chunks and
-    compare every request with the oracle's compose."""
+    compare every request with the oracle's compose.  Chunks named in `host` stay in pinned
+    host memory (MODE_HOST) and compose reads them there."""
     c2kv = H.lib()
     all_ids = sorted({c for ids, _ in requests for c in ids})
     chunks = H.oracle_chunks_meanpool(wl, all_ids)
     ctx = H.make_ctx(wl, pool_slots=pool_slots, fixed_pos=int(fixed_pos))
+    keep = []
     try:
-        dev = H.load_stored(ctx, wl, chunks)
+        dev = H.load_stored(ctx, wl, chunks, host=host, keep=keep)
         req_ptr = np.cumsum([0] + [len(ids) for ids, _ in requests])
         flat_ids = [dev[c] for ids, _ in requests for c in ids]
         flat_pos = [o for _, offs in requests for o in offs]
@@ -181,11 +183,76 @@ def test_compose_empty_request_in_batch():
     _compose_case(wl, [([0, 1], [0, 64]), ([], []), ([1], [5])])
 
 
+def test_compose_host_chunks():
+    # every chunk stays in pinned host memory: compose reads, re-rotates and gathers it
+    # in one pass; V and positions bit-exact as from the pool
+    _compose_case(L8B_1, synth.requests(L8B_1), host=set(range(L8B_1.pool_chunks)))
+
+
+def test_compose_host_and_pool_chunks_mixed():
+    wl = _small(L8B_1, layers=2, chunk_tokens=203, ratio_k=10, pool_chunks=5)
+    reqs = [([0, 3, 0], [7, 300, 800]),
+            ([4], [0]),
+            ([2, 1, 4, 3], [0, 203, 406, 10000])]
+    _compose_case(wl, reqs, host={0, 2, 4})
+    _compose_case(wl, reqs, host={0, 1, 2, 3, 4}, fixed_pos=True)
+
+
+def test_host_chunks_take_no_pool_slots():
+    # a pool of 8 slots composes host chunks of 103 slots each; freeing them leaves the pool
+    # untouched (a pool chunk of 8 slots still fits afterwards)
+    c2kv = H.lib()
+    wl = _small(L8B_1, layers=2, chunk_tokens=412, ratio_k=4, pool_chunks=3)
+    chunks = H.oracle_chunks_meanpool(wl, [0, 1, 2])
+    ctx = H.make_ctx(wl, pool_slots=8)
+    keep = []
+    try:
+        dev = H.load_stored(ctx, wl, chunks, host={0, 1, 2}, keep=keep)
+        info = c2kv.c2kv_chunk_info(ctx, dev[1])
+        assert info["n_slots"] == 103 and info["layer_stride"] == 103 * wl.n_kv_heads * wl.head_dim
+        cache = c2kv.c2kv_compose(ctx, [0, 3], [dev[2], dev[0], dev[1]], [0, 412, 824], 4)
+        info_c, gk, gv, gpos = H.cache_arrays(cache, wl)
+        ok, ov, opos, l_req = orc.compose(chunks, [2, 0, 1], [0, 412, 824], wl.rope_theta,
+                                          wl.dtype)
+        assert np.array_equal(gpos[:ok.shape[1]], opos) and np.array_equal(gv[:, :ok.shape[1]], ov)
+        c2kv.c2kv_cache_release(ctx, cache)
+        for c in (0, 1, 2):
+            c2kv.c2kv_free_chunk(ctx, dev[c])
+        ks, vs = synth.chunk_slots(wl, 9, 8)
+        c2kv.c2kv_compress_chunk(ctx, H.to_dev(ks, wl), H.to_dev(vs, wl), 32, 4,
+                                 c2kv.MODE_STORED)
+    finally:
+        c2kv.c2kv_destroy(ctx)
+
+
+def test_host_mode_rejects_pageable_and_misaligned():
+    # both refusals are taken on the host before anything is enqueued
+    c2kv = H.lib()
+    wl = _small(L8B_1, layers=1)
+    ctx = H.make_ctx(wl, pool_slots=64)
+    try:
+        ks, vs = synth.chunk_slots(wl, 1, 8)
+        kp = torch.from_numpy(ks).to(torch.bfloat16)                   # pageable
+        vp = torch.from_numpy(vs).to(torch.bfloat16)
+        with pytest.raises(c2kv.C2KVError) as ei:
+            c2kv.c2kv_compress_chunk(ctx, kp, vp, 32, 4, c2kv.MODE_HOST)
+        assert ei.value.status == c2kv.ERR_ARG
+        buf = torch.zeros(2 * ks.size + 8, dtype=torch.bfloat16).pin_memory()
+        with pytest.raises(c2kv.C2KVError) as ei:                      # 2-byte offset
+            c2kv.c2kv_compress_chunk(ctx, buf.data_ptr() + 2, buf.data_ptr() + 2 * ks.size + 2,
+                                     32, 4, c2kv.MODE_HOST)
+        assert ei.value.status == c2kv.ERR_ARG
+    finally:
+        c2kv.c2kv_destroy(ctx)
+
+
 # ------------------------------------------------------------------ attend
 
-def _attend_case(wl, attn_impl=0, layer=-1, n_suffix=None, requests=None, attn_split=0):
+def _attend_case(wl, attn_impl=0, layer=-1, n_suffix=None, requests=None, attn_split=0,
+                 host=()):
     """End to end: oracle-stored chunks -> GPU compose -> GPU attend, vs oracle compose +
-    attend on the same inputs.  Checks O, lse, and the suffix rows written to the cache."""
+    attend on the same inputs.  Checks O, lse, and the suffix rows written to the cache.
+    Chunks named in `host` stay in pinned host memory (MODE_HOST)."""
     c2kv = H.lib()
     sq = wl.n_suffix if n_suffix is None else n_suffix
     wl = synth.scaled(wl, n_suffix=sq)
@@ -195,8 +262,9 @@ def _attend_case(wl, attn_impl=0, layer=-1, n_suffix=None, requests=None, attn_s
     ctx = H.make_ctx(wl, pool_slots=sum(orc.n_slots(wl.chunk_tokens, wl.ratio_k)
                                         for _ in all_ids) + 16, attn_impl=attn_impl,
                        attn_split=attn_split)
+    keep = []
     try:
-        dev = H.load_stored(ctx, wl, chunks)
+        dev = H.load_stored(ctx, wl, chunks, host=host, keep=keep)
         req_ptr = np.cumsum([0] + [len(ids) for ids, _ in reqs])
         cache = c2kv.c2kv_compose(ctx, req_ptr, [dev[c] for ids, _ in reqs for c in ids],
                                   [o for _, offs in reqs for o in offs], suffix_capacity=sq)
@@ -285,6 +353,11 @@ def test_attend_key_range_splits(split):
     wl = _small(L8B_1, chunks_per_request=1, pool_chunks=1, chunk_tokens=64, ratio_k=4,
                 n_suffix=300)
     _attend_case(wl, attn_split=split)
+
+
+def test_attend_from_host_chunks():
+    wl = _small(L8B_1, layers=2)
+    _attend_case(wl, host=set(range(wl.pool_chunks)))
 
 
 def test_attend_forced_split_batched():
