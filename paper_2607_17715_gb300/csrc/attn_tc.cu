@@ -1,26 +1,38 @@
 // Tensor-core attention over [composed cache; suffix] for sm_103a: tcgen05.mma with TMEM
 // accumulators, operands staged by TMA in 128-byte-swizzled shared memory.
 //
-// Work unit (one CTA): 128 packed query rows of one (layer, request, KV head).  Row
-// m = t * G + g is suffix token t0 + t, query head h_kv * G + g (G = Hq / Hkv), so the
-// G query heads that share a KV head form the M dimension of one MMA and every K/V tile
-// is fetched once for all of them.  The CTA walks the request's key tiles of 128 rows
-// (composed slots first, then its own suffix rows); only the tiles past S_r + t0 need
-// the causal mask.
+// Work unit (one CTA): two query tiles A and B of 128 packed rows each, consecutive in the
+// suffix, of one (layer, request, KV head).  Row m = t * G + g of a tile is suffix token
+// t0 + t, query head h_kv * G + g (G = Hq / Hkv), so the G query heads that share a KV
+// head form the M dimension of one MMA.  Every K/V tile brought into shared memory feeds
+// both tiles' MMAs: 128 KB of MMA work per 64 KB of K/V, which keeps the TMA ingress of an
+// SM (about 63 B per clock from L2) below what the tensor core consumes.  The CTA walks
+// the request's key tiles of 128 rows (composed slots first, then its own suffix rows);
+// only the tiles past S_r + t0 need the causal mask.
 //
-// Warp roles (192 threads):
-//   warp 0      TMA producer: Q once, then K tiles into a 3-stage ring and V tiles into a
-//               3-stage ring, each issued as soon as its own stage is free (a K stage is
-//               refilled once S_j = Q K_j^T has read it, a V stage after P_j.V_j), so K
-//               loads never queue behind V releases.
-//   warp 1      MMA issuer (one lane) and TMEM owner:  S_j = Q K_j^T into one of two TMEM
-//               S buffers, then O += P_{j-1} V_{j-1}, P read from TMEM as the A operand.
-//   warps 2..5  softmax / correction / epilogue: thread i owns TMEM lane (row) i.  Reads
-//               S_j, masks, keeps the running max and sum, writes P_j (bf16, two keys per
-//               32-bit column) into one of two TMEM P buffers (so P_{j+1} is written while
-//               P_j.V_j runs), rescales O in TMEM only when its row max grew by more than
-//               2^8 (otherwise the stale reference max is kept: the normaliser uses the
-//               same one, so the result is exact).
+// Tensor memory (512 columns): S_A [0,128), S_B [128,256), O_A [256,384), O_B [384,512).
+// P_x (bf16, two keys per 32-bit column) is written over the first 64 columns of S_x once
+// the softmax has read S_x into registers.
+//
+// The MMA issuer runs, per key tile j,   PV_A(j-1), S_A(j), PV_B(j-1), S_B(j):
+// S_A(j) overwrites P_A(j-1) only after PV_A(j-1) in issue order (tcgen05.mma from one
+// thread execute in order), and while the softmax of tile A works on S_A(j) the tensor
+// core runs PV_B(j-1) and S_B(j), so neither softmax sits on the tensor core's critical
+// path as long as it takes less than half a period.  A tcgen05.commit tracks every earlier
+// MMA of the thread, so when S_x(j) is reported complete, O_x holds every P.V up to j-1
+// and the softmax may rescale it.
+//
+// Warp roles (384 threads):
+//   warp 0      TMA producer: Q_A and Q_B once, then K tiles into a 3-stage ring and V
+//               tiles into a 2-stage ring, each issued as soon as its own stage is free (a
+//               K stage once S_B has read it, a V stage once P_B.V has).
+//   warp 1      MMA issuer (one lane) and TMEM owner.  Warps 2 and 3 only complete
+//               warpgroup 0, which hands most of its registers to the softmax warpgroups.
+//   warps 4..7  softmax / correction / epilogue of tile A: thread i owns TMEM lane (row) i.
+//   warps 8..11 the same for tile B.
+//   A softmax thread reads S_j, masks, keeps the running max and sum, rescales O in TMEM
+//   only when its row max grew by more than 2^8 (otherwise the stale reference max is
+//   kept: the normaliser uses the same one, so the result is exact), and writes P_j.
 //
 // Every mbarrier wait is bounded (kWaitCycles); on expiry the waiting thread sets bit 1
 // of the error word and carries on, so the kernel always terminates and the host reports
@@ -37,31 +49,38 @@
 namespace c2kv {
 namespace {
 
-constexpr int BM = 128;                 // query rows per CTA (MMA M)
+constexpr int BM = 128;                 // query rows per tile (MMA M)
 constexpr int BN = 128;                 // keys per tile (MMA N of S, K of P.V)
 constexpr int HD = 128;                 // head dim
 constexpr int KSTAGES = 3;              // K ring depth
-constexpr int VSTAGES = 3;              // V ring depth
+constexpr int VSTAGES = 2;              // V ring depth
 constexpr int TILE = BN * HD * 2;       // bytes of one 128 x 128 bf16 tile (32 KB)
 constexpr int HALF_TILE = TILE / 2;     // one 128-byte-wide swizzle column block
-constexpr int kThreads = 192;
-constexpr uint32_t kTmemCols = 512;     // S0 [0,128) S1 [128,256) O [256,384) P0, P1 [384,512)
-constexpr uint32_t kColS = 0, kColO = 256, kColP = 384;
-constexpr long long kWaitCycles = 4000000000LL;
+constexpr int kThreads = 384;
+// Register split (setmaxnreg): warpgroup 0 (TMA producer, MMA issuer, two idle warps) gives
+// registers to the two softmax warpgroups.  The kernel is launched with kLaunchRegs per
+// thread (the cap that 384 threads leave, 3 warps per SM sub-partition); the split below
+// hands out exactly that total, which the host checks against the compiled count.
+constexpr int kLaunchRegs = 168;
+constexpr int kRegsLow = 104;
+constexpr int kRegsHigh = 200;
+static_assert(128 * kRegsLow + 256 * kRegsHigh <= kThreads * kLaunchRegs, "register split");
+constexpr uint32_t kTmemCols = 512;     // S_A, S_B, O_A, O_B; P_x over the first half of S_x
+constexpr uint32_t kColS = 0, kColO = 256;
+constexpr long long kWaitCycles = 2000000000LL;   // about 1 s
 
 // barrier slots
-constexpr int B_Q = 0;
+constexpr int B_Q = 0;                   // both Q tiles landed
 constexpr int B_KF = 1;                  // + stage
-constexpr int B_KE = B_KF + KSTAGES;     // + stage: K stage free (both S MMAs finished)
+constexpr int B_KE = B_KF + KSTAGES;     // + stage: K stage free (S_A and S_B finished)
 constexpr int B_VF = B_KE + KSTAGES;     // + stage
-constexpr int B_VE = B_VF + VSTAGES;     // + stage: V stage free (both P.V MMAs finished)
-constexpr int B_SF = B_VE + VSTAGES;     // + buffer: S ready in TMEM
-constexpr int B_SFREE = B_SF + 2;        // + buffer: S read out by the softmax warps
-constexpr int B_PF = B_SFREE + 2;        // + buffer: P_j written (and O corrected)
-constexpr int B_PFREE = B_PF + 2;        // + buffer: P_j.V_j finished (buffer free, O current)
-constexpr int NBAR = B_PFREE + 2;
+constexpr int B_VE = B_VF + VSTAGES;     // + stage: V stage free (both P.V finished)
+constexpr int B_SF = B_VE + VSTAGES;     // + tile: S_x(j) complete (and every MMA before it)
+constexpr int B_PF = B_SF + 2;           // + tile: P_x(j) written (and O_x corrected)
+constexpr int B_OD = B_PF + 2;           // every MMA finished: O_A, O_B final
+constexpr int NBAR = B_OD + 1;
 
-constexpr int kSmemTiles = 1 /*Q*/ + KSTAGES + VSTAGES;
+constexpr int kSmemTiles = 2 /*Q_A, Q_B*/ + KSTAGES + VSTAGES;
 constexpr size_t kSmemBytes = 1024 /*align*/ + (size_t)TILE * kSmemTiles + 8 * NBAR + 16;
 static_assert(kSmemBytes <= 232448, "shared memory budget of one sm_100 CTA");
 
@@ -112,13 +131,18 @@ __device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
     return ok != 0;
 }
 
-// Bounded wait for the phase with the given parity to complete.
-__device__ __forceinline__ void mbar_wait(uint32_t bar, uint32_t parity, int32_t* err) {
+// Bounded wait for the phase with the given parity to complete.  The first wait of a CTA
+// that gives up raises the CTA's abort flag (shared memory), and every later wait returns
+// as soon as it sees it, so a CTA spends at most one time limit in waits.
+__device__ __forceinline__ void mbar_wait(uint32_t bar, uint32_t parity, int32_t* err,
+                                          volatile uint32_t* abort) {
     if (mbar_try(bar, parity)) return;
     const long long t0 = clock64();
     while (!mbar_try(bar, parity)) {
+        if (*abort) return;
         if (clock64() - t0 > kWaitCycles) {
             atomicOr(err, 2);
+            *abort = 1u;
             return;
         }
     }
@@ -210,16 +234,23 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
         : "r"(taddr));
 }
 
-__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&v)[32]) {
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&v)[16]) {
     asm volatile(
-        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], "
-        "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16, "
-        "%17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31, %32};" ::"r"(taddr),
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+        "{%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15}, [%16];"
+        : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]),
+          "=r"(v[7]), "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]),
+          "=r"(v[13]), "=r"(v[14]), "=r"(v[15])
+        : "r"(taddr));
+}
+
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t (&v)[16]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], "
+        "{%1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, %15, %16};" ::"r"(taddr),
         "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
         "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]),
-        "r"(v[15]), "r"(v[16]), "r"(v[17]), "r"(v[18]), "r"(v[19]), "r"(v[20]), "r"(v[21]),
-        "r"(v[22]), "r"(v[23]), "r"(v[24]), "r"(v[25]), "r"(v[26]), "r"(v[27]), "r"(v[28]),
-        "r"(v[29]), "r"(v[30]), "r"(v[31])
+        "r"(v[15])
         : "memory");
 }
 
@@ -243,17 +274,300 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
     return *reinterpret_cast<uint32_t*>(&v);
 }
 
+// Two fp32 lanes per instruction (sm_100 packed f32x2 arithmetic, round to nearest: each
+// lane is bitwise the scalar fmaf / add), and the three-input maximum.
+__device__ __forceinline__ void ffma2(float& d0, float& d1, float a0, float a1, float b, float c) {
+    asm("{\n\t.reg .b64 pa, pb, pc, pd;\n\t"
+        "mov.b64 pa, {%2, %3};\n\t"
+        "mov.b64 pb, {%4, %4};\n\t"
+        "mov.b64 pc, {%5, %5};\n\t"
+        "fma.rn.f32x2 pd, pa, pb, pc;\n\t"
+        "mov.b64 {%0, %1}, pd;\n\t}"
+        : "=f"(d0), "=f"(d1)
+        : "f"(a0), "f"(a1), "f"(b), "f"(c));
+}
+
+__device__ __forceinline__ void fadd2(float& d0, float& d1, float a0, float a1) {
+    asm("{\n\t.reg .b64 pa, pd;\n\t"
+        "mov.b64 pa, {%2, %3};\n\t"
+        "mov.b64 pd, {%0, %1};\n\t"
+        "add.rn.f32x2 pd, pd, pa;\n\t"
+        "mov.b64 {%0, %1}, pd;\n\t}"
+        : "+f"(d0), "+f"(d1)
+        : "f"(a0), "f"(a1));
+}
+
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+    float d;
+    asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+    return d;
+}
+
 // ------------------------------------------------------------------ kernel
+
+// One softmax thread's work on tile x (A or B) for every key tile, then its epilogue.
+// r = TMEM lane (row within the tile), t0 = first suffix token of the tile.
+__device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, uint32_t sBar, int x,
+                                            int quad, int lane, int t0, int l, int bl, int b,
+                                            int hk, int sp, int j_base, int n_kv,
+                                            volatile uint32_t* abort) {
+    auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
+    const int G = P.group;
+    const int s_r = P.req[bl].n_slots;
+    const int r = quad * 32 + lane;                 // row = TMEM lane
+    const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
+    const uint32_t colS = kColS + (uint32_t)x * BN;  // S_x, and P_x over its first 64 columns
+    const uint32_t colO = kColO + (uint32_t)x * HD;
+    const int t_row = min(t0 + r / G, P.sq - 1);    // rows past the suffix mirror its end
+    const int lim = s_r + t_row;                    // last key this row may see
+    const float sc = P.scale_log2;
+    float m_run = -CUDART_INF_F;
+    float l_run = 0.f;
+
+    for (int j = 0; j < n_kv; ++j) {
+        mbar_wait(bar(B_SF + x), (uint32_t)j & 1u, P.err, abort);
+        tc_fence_after();
+        uint32_t sv[4][32];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) tmem_ld32(tmem + lane_addr + colS + c * 32, sv[c]);
+        tmem_ld_wait();
+
+        const int kbase = (j_base + j) * BN;
+        if (kbase + BN - 1 > lim) {
+#pragma unroll
+            for (int c = 0; c < 4; ++c)
+#pragma unroll
+                for (int e = 0; e < 32; ++e)
+                    if (kbase + c * 32 + e > lim) sv[c][e] = __float_as_uint(-CUDART_INF_F);
+        }
+        // row max: three-input maxima, one chain per 32-column chunk
+        float mx4[4];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            float m = fmaxf(__uint_as_float(sv[c][0]), __uint_as_float(sv[c][1]));
+#pragma unroll
+            for (int e = 2; e < 32; e += 2)
+                m = fmax3(m, __uint_as_float(sv[c][e]), __uint_as_float(sv[c][e + 1]));
+            mx4[c] = m;
+        }
+        const float mx = fmaxf(fmaxf(mx4[0], mx4[1]), fmaxf(mx4[2], mx4[3]));
+        const float m_new = fmaxf(m_run, mx * sc);
+        const bool resc = m_new > m_run + 8.0f;       // false while nothing is visible
+        const float m_use = resc ? m_new : m_run;
+        const float alpha = resc ? ex2(m_run - m_new) : 1.0f;
+        const float m_sub = m_use == -CUDART_INF_F ? 0.f : m_use;   // all masked so far
+
+        // S_x(j) complete implies P_x(j-1).V(j-1) complete: O_x is current and may be scaled
+        if (j >= 1 && __any_sync(0xffffffffu, resc)) {
+#pragma unroll 1
+            for (int c = 0; c < 8; ++c) {
+                uint32_t ov[16];
+                tmem_ld16(tmem + lane_addr + colO + c * 16, ov);
+                tmem_ld_wait();
+#pragma unroll
+                for (int e = 0; e < 16; ++e) ov[e] = __float_as_uint(__uint_as_float(ov[e]) * alpha);
+                tmem_st16(tmem + lane_addr + colO + c * 16, ov);
+            }
+        }
+        float ps[4];                                   // two packed accumulators
+#pragma unroll
+        for (int e = 0; e < 4; ++e) ps[e] = 0.f;
+        // P_j (bf16, keys 2c and 2c+1 packed in column c) over the first half of S_x
+        const uint32_t p_addr = tmem + lane_addr + colS;
+        const float neg_m = -m_sub;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            uint32_t pk[16];
+#pragma unroll
+            for (int e = 0; e < 32; e += 2) {
+                float a0, a1;
+                ffma2(a0, a1, __uint_as_float(sv[c][e]), __uint_as_float(sv[c][e + 1]), sc, neg_m);
+                a0 = ex2(a0);
+                a1 = ex2(a1);
+                if (e & 2) fadd2(ps[2], ps[3], a0, a1); else fadd2(ps[0], ps[1], a0, a1);
+                pk[e >> 1] = pack_bf16(a0, a1);
+            }
+            tmem_st16(p_addr + (uint32_t)c * 16u, pk);
+        }
+        tmem_st_wait();
+        const float sum = (ps[0] + ps[1]) + (ps[2] + ps[3]);
+        l_run = l_run * alpha + sum;
+        m_run = m_use;
+        tc_fence_before();
+        mbar_arrive(bar(B_PF + x));
+    }
+
+    // ---------------------------------------------------------------- epilogue
+    if (n_kv > 0) {
+        mbar_wait(bar(B_OD), 0u, P.err, abort);
+        tc_fence_after();
+    }
+    const int t = t0 + r / G;
+    const int g = r - (r / G) * G;
+    const bool any = l_run > 0.f;                 // some key of this split was visible
+    const float inv = any ? 1.0f / l_run : 0.f;
+    const int64_t row_id = (((int64_t)l * P.batch_total + b) * P.sq + t) * P.hq + hk * G + g;
+    const int64_t lse_id = (((int64_t)l * P.batch_total + b) * P.hq + hk * G + g) * P.sq + t;
+    if (P.n_split == 1) {
+        __nv_bfloat16* orow = static_cast<__nv_bfloat16*>(P.out) + row_id * HD;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            uint32_t ov[32];
+            tmem_ld32(tmem + lane_addr + colO + c * 32, ov);
+            tmem_ld_wait();
+            if (t < P.sq) {
+#pragma unroll
+                for (int q8 = 0; q8 < 4; ++q8) {
+                    uint4 w;
+                    w.x = pack_bf16(__uint_as_float(ov[q8 * 8 + 0]) * inv, __uint_as_float(ov[q8 * 8 + 1]) * inv);
+                    w.y = pack_bf16(__uint_as_float(ov[q8 * 8 + 2]) * inv, __uint_as_float(ov[q8 * 8 + 3]) * inv);
+                    w.z = pack_bf16(__uint_as_float(ov[q8 * 8 + 4]) * inv, __uint_as_float(ov[q8 * 8 + 5]) * inv);
+                    w.w = pack_bf16(__uint_as_float(ov[q8 * 8 + 6]) * inv, __uint_as_float(ov[q8 * 8 + 7]) * inv);
+                    *reinterpret_cast<uint4*>(orow + c * 32 + q8 * 8) = w;
+                }
+            }
+        }
+        if (P.lse != nullptr && t < P.sq)
+            P.lse[lse_id] = (m_run + log2f(l_run)) * 0.69314718055994531f;
+    } else {
+        // partial over this split's keys: normalised O (fp32) and its log2-domain lse
+        const int64_t part_rows = (int64_t)P.lq * P.batch_total * P.sq * P.hq;
+        float* orow = P.part_o + ((int64_t)sp * part_rows + row_id) * HD;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            uint32_t ov[32];
+            if (n_kv > 0) {
+                tmem_ld32(tmem + lane_addr + colO + c * 32, ov);
+                tmem_ld_wait();
+            } else {
+#pragma unroll
+                for (int e = 0; e < 32; ++e) ov[e] = 0u;
+            }
+            if (t < P.sq) {
+#pragma unroll
+                for (int q4 = 0; q4 < 8; ++q4) {
+                    float4 w = make_float4(__uint_as_float(ov[q4 * 4 + 0]) * inv, __uint_as_float(ov[q4 * 4 + 1]) * inv,
+                                           __uint_as_float(ov[q4 * 4 + 2]) * inv, __uint_as_float(ov[q4 * 4 + 3]) * inv);
+                    *reinterpret_cast<float4*>(orow + c * 32 + q4 * 4) = w;
+                }
+            }
+        }
+        if (t < P.sq)
+            P.part_lse[(int64_t)sp * part_rows + lse_id] = any ? m_run + log2f(l_run) : -CUDART_INF_F;
+    }
+}
+
+// The MMA issuer (one thread).  The tensor core's queue holds about one MMA, so anything
+// the issuing thread does between two MMAs idles it: descriptors are precomputed and the
+// ring stages advance by counters.  Each block waits for its own inputs only: a wait for a
+// later block's P inside an S block would hold that S back until the other tile's softmax
+// finished, putting the two softmaxes in series.
+__device__ __forceinline__ void mma_issuer(const TcParams& P, uint32_t tmem, uint32_t sQ, uint32_t sK,
+                                           uint32_t sV, uint32_t sBar, bool has_b, int n_kv,
+                                           volatile uint32_t* abort) {
+    auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
+    constexpr uint32_t idS = idesc_bf16(BM, BN, false);
+    constexpr uint32_t idO = idesc_bf16(BM, HD, true);
+    constexpr uint64_t kTileDesc = (uint64_t)(TILE >> 4);     // one tile in descriptor units
+    // descriptors of tile bases; a K step adds its byte offset / 16 to the low field
+    const uint64_t dQa = sw128_desc(sQ, 16, 1024);
+    const uint64_t dQb = sw128_desc(sQ + TILE, 16, 1024);
+    const uint64_t dK0 = sw128_desc(sK, 16, 1024);
+    const uint64_t dV0 = sw128_desc(sV, HALF_TILE, 1024);
+    const uint32_t tS_a = tmem + kColS, tS_b = tmem + kColS + BN;
+    const uint32_t tO_a = tmem + kColO, tO_b = tmem + kColO + HD;
+
+    // S = Q K^T (8 K steps of 16)
+    auto s_block = [&](uint64_t dq, uint64_t dk, uint32_t d) {
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk) {
+            const uint64_t off = (uint64_t)(((kk >> 2) * HALF_TILE + (kk & 3) * 32) >> 4);
+            mma_bf16(d, dq + off, dk + off, idS, kk > 0 ? 1u : 0u);
+        }
+    };
+    // O += P V with P (bf16 pairs) from TMEM: 16 keys (8 columns) per step
+    auto pv_block = [&](uint32_t p, uint64_t dv, uint32_t o, bool first) {
+#pragma unroll
+        for (int kk = 0; kk < BN / 16; ++kk) {
+            mma_bf16_ts(o, p + (uint32_t)kk * 8u, dv + (uint64_t)((kk * 2048) >> 4), idO,
+                        (!first || kk > 0) ? 1u : 0u);
+        }
+    };
+    auto wait = [&](int i, uint32_t parity) {
+        mbar_wait(bar(i), parity, P.err, abort);
+        tc_fence_after();
+    };
+
+    // ring positions: stage index and the phase parity of its current fill
+    int ks = 0, vs = 0;
+    uint32_t kph = 0, vph = 0;
+    uint64_t dk = dK0, dv = dV0;
+    auto next_k = [&] {
+        if (++ks == KSTAGES) { ks = 0; kph ^= 1u; dk = dK0; } else { dk += kTileDesc; }
+    };
+    auto next_v = [&] {
+        if (++vs == VSTAGES) { vs = 0; vph ^= 1u; dv = dV0; } else { dv += kTileDesc; }
+    };
+
+    wait(B_Q, 0u);
+    wait(B_KF + 0, 0u);
+    // key tile 0: S_A(0), S_B(0)
+    s_block(dQa, dk, tS_a);
+    mma_commit(bar(B_SF + 0));
+    if (has_b) {
+        s_block(dQb, dk, tS_b);
+        mma_commit(bar(B_SF + 1));
+    }
+    mma_commit(bar(B_KE + 0));
+    next_k();
+    // key tiles 1 .. n_kv-1:  PV_A(j-1)  S_A(j)  PV_B(j-1)  S_B(j).  While the softmax of tile
+    // A works on S_A(j), the tensor core runs PV_B(j-1) and S_B(j), and the other way round.
+    for (int j = 1; j < n_kv; ++j) {
+        const uint32_t pj = (uint32_t)(j - 1) & 1u;      // parity of P_x(j-1)
+        const bool first = j == 1;
+        wait(B_PF + 0, pj);
+        wait(B_VF + vs, vph);
+        pv_block(tS_a, dv, tO_a, first);
+        wait(B_KF + ks, kph);
+        s_block(dQa, dk, tS_a);
+        mma_commit(bar(B_SF + 0));
+        if (has_b) {
+            wait(B_PF + 1, pj);
+            pv_block(tS_b, dv, tO_b, first);
+        }
+        mma_commit(bar(B_VE + vs));
+        next_v();
+        if (has_b) {
+            s_block(dQb, dk, tS_b);
+            mma_commit(bar(B_SF + 1));
+        }
+        mma_commit(bar(B_KE + ks));
+        next_k();
+    }
+    // last P.V pair
+    const uint32_t pl = (uint32_t)(n_kv - 1) & 1u;
+    const bool first = n_kv == 1;
+    wait(B_PF + 0, pl);
+    wait(B_VF + vs, vph);
+    pv_block(tS_a, dv, tO_a, first);
+    if (has_b) {
+        wait(B_PF + 1, pl);
+        pv_block(tS_b, dv, tO_b, first);
+    }
+    mma_commit(bar(B_VE + vs));
+    mma_commit(bar(B_OD));
+}
 
 __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_constant__ TcParams P) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~uintptr_t(1023));
-    const uint32_t sQ = smem_u32(smem);
-    const uint32_t sK = sQ + TILE;
+    const uint32_t sQ = smem_u32(smem);             // Q_A, then Q_B
+    const uint32_t sK = sQ + 2 * TILE;
     const uint32_t sV = sK + KSTAGES * TILE;
     const uint32_t sBar = sV + VSTAGES * TILE;
     uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(smem + (size_t)TILE * kSmemTiles + 8 * NBAR);
+    volatile uint32_t* abort = tmem_slot + 1;      // set by the first wait that gives up
     auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
 
     const int warp = threadIdx.x >> 5;
@@ -264,10 +578,12 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_const
     const int bl = blockIdx.z - l * P.batch;
     const int b = P.b0 + bl;
     const int s_r = P.req[bl].n_slots;
-    const int mt = blockIdx.x / P.n_split;          // Q tile
-    const int sp = blockIdx.x - mt * P.n_split;     // key-range split
-    const int t0 = mt * P.tq;
-    const int t_last = min(P.sq - 1, t0 + P.tq - 1);
+    const int pr = blockIdx.x / P.n_split;          // pair of Q tiles
+    const int sp = blockIdx.x - pr * P.n_split;     // key-range split
+    const int t0a = 2 * pr * P.tq;
+    const int t0b = t0a + P.tq;
+    const bool has_b = t0b < P.sq;
+    const int t_last = min(P.sq - 1, (has_b ? t0b : t0a) + P.tq - 1);
     const int n_kv_all = (s_r + t_last + 1 + BN - 1) / BN;
     // this CTA's key tiles: [j_base, j_base + n_kv) of the request's n_kv_all
     const int per_split = (n_kv_all + P.n_split - 1) / P.n_split;
@@ -286,10 +602,10 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_const
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(bar(B_SF + i), 1);
-            mbar_init(bar(B_SFREE + i), 128);
             mbar_init(bar(B_PF + i), 128);
-            mbar_init(bar(B_PFREE + i), 1);
         }
+        mbar_init(bar(B_OD), 1);
+        *abort = 0u;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (warp == 1) {
@@ -304,16 +620,21 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_const
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
 
-    if (warp == 0) {
-        // ---------------------------------------------------------------- TMA producer
-        if (lane == 0) {
+    if (warp < 4) {
+        asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsLow));
+        if (warp == 0 && lane == 0 && n_kv > 0) {
+            // ------------------------------------------------------------ TMA producer
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&P.tm_q)) : "memory");
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&P.tm_k)) : "memory");
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&P.tm_v)) : "memory");
             const int qz = l * P.batch_total + b;
-            mbar_expect_tx(bar(B_Q), TILE);
-            tma_load_4d(sQ, &P.tm_q, 0, hk * G, t0, qz, bar(B_Q));
-            tma_load_4d(sQ + HALF_TILE, &P.tm_q, 64, hk * G, t0, qz, bar(B_Q));
+            mbar_expect_tx(bar(B_Q), has_b ? 2 * TILE : TILE);
+            tma_load_4d(sQ, &P.tm_q, 0, hk * G, t0a, qz, bar(B_Q));
+            tma_load_4d(sQ + HALF_TILE, &P.tm_q, 64, hk * G, t0a, qz, bar(B_Q));
+            if (has_b) {
+                tma_load_4d(sQ + TILE, &P.tm_q, 0, hk * G, t0b, qz, bar(B_Q));
+                tma_load_4d(sQ + TILE + HALF_TILE, &P.tm_q, 64, hk * G, t0b, qz, bar(B_Q));
+            }
             const int key0 = (int)((int64_t)(P.layer0 + l) * P.rows + P.req[bl].row_base) + j_base * BN;
             // two independent queues: a K load waits only for its own K stage
             int jk = 0, jv = 0;
@@ -340,209 +661,21 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_const
                 }
                 // nothing issuable: wait (bounded) for the stage the next K load needs
                 if (jk < n_kv)
-                    mbar_wait(bar(B_KE + jk % KSTAGES), (uint32_t)((jk / KSTAGES) - 1) & 1u, P.err);
+                    mbar_wait(bar(B_KE + jk % KSTAGES), (uint32_t)((jk / KSTAGES) - 1) & 1u, P.err, abort);
                 else
-                    mbar_wait(bar(B_VE + jv % VSTAGES), (uint32_t)((jv / VSTAGES) - 1) & 1u, P.err);
+                    mbar_wait(bar(B_VE + jv % VSTAGES), (uint32_t)((jv / VSTAGES) - 1) & 1u, P.err, abort);
             }
-        }
-    } else if (warp == 1) {
-        // ---------------------------------------------------------------- MMA issuer
-        if (lane == 0) {
-            constexpr uint32_t idS = idesc_bf16(BM, BN, false);
-            constexpr uint32_t idO = idesc_bf16(BM, HD, true);
-            mbar_wait(bar(B_Q), 0, P.err);
-            tc_fence_after();
-            for (int j = 0; j <= n_kv; ++j) {
-                if (j < n_kv) {
-                    const int ks = j % KSTAGES;
-                    const int sb = j & 1;
-                    mbar_wait(bar(B_KF + ks), (uint32_t)(j / KSTAGES) & 1u, P.err);
-                    if (j >= 2) mbar_wait(bar(B_SFREE + sb), (uint32_t)((j - 2) >> 1) & 1u, P.err);
-                    tc_fence_after();
-                    const uint32_t kb = sK + ks * TILE;
-#pragma unroll
-                    for (int kk = 0; kk < HD / 16; ++kk) {
-                        const uint32_t off = (uint32_t)(kk >> 2) * HALF_TILE + (uint32_t)(kk & 3) * 32u;
-                        mma_bf16(tmem + kColS + sb * BN, sw128_desc(sQ + off, 16, 1024),
-                                 sw128_desc(kb + off, 16, 1024), idS, kk > 0 ? 1u : 0u);
-                    }
-                    mma_commit(bar(B_SF + sb));
-                    mma_commit(bar(B_KE + ks));
-                }
-                if (j >= 1) {
-                    const int jp = j - 1;
-                    const int vs = jp % VSTAGES;
-                    const int pb = jp & 1;
-                    mbar_wait(bar(B_PF + pb), (uint32_t)(jp >> 1) & 1u, P.err);
-                    mbar_wait(bar(B_VF + vs), (uint32_t)(jp / VSTAGES) & 1u, P.err);
-                    tc_fence_after();
-                    const uint32_t vb = sV + vs * TILE;
-                    const uint32_t pcol = tmem + kColP + (uint32_t)pb * (BN / 2);
-#pragma unroll
-                    for (int kk = 0; kk < BN / 16; ++kk) {
-                        // A = P_j from TMEM: 16 keys (8 packed columns) per instruction
-                        mma_bf16_ts(tmem + kColO, pcol + (uint32_t)kk * 8u,
-                                    sw128_desc(vb + (uint32_t)kk * 2048u, HALF_TILE, 1024), idO,
-                                    (jp > 0 || kk > 0) ? 1u : 0u);
-                    }
-                    mma_commit(bar(B_VE + vs));
-                    mma_commit(bar(B_PFREE + pb));
-                }
-            }
+        } else if (warp == 1 && lane == 0 && n_kv > 0) {
+            // ------------------------------------------------------------ MMA issuer
+            mma_issuer(P, tmem, sQ, sK, sV, sBar, has_b, n_kv, abort);
         }
     } else {
+        asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegsHigh));
         // ---------------------------------------------------------------- softmax warps
-        const int quad = warp & 3;
-        const int r = quad * 32 + lane;                 // row = TMEM lane
-        const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
-        const int t_row = min(t0 + r / G, P.sq - 1);   // rows past the suffix mirror its end
-        const int lim = s_r + t_row;                    // last key this row may see
-        const float sc = P.scale_log2;
-        float m_run = -CUDART_INF_F;
-        float l_run = 0.f;
-
-        for (int j = 0; j < n_kv; ++j) {
-            const int sb = j & 1;
-            mbar_wait(bar(B_SF + sb), (uint32_t)(j >> 1) & 1u, P.err);
-            tc_fence_after();
-            uint32_t sv[4][32];
-#pragma unroll
-            for (int c = 0; c < 4; ++c) tmem_ld32(tmem + lane_addr + kColS + sb * BN + c * 32, sv[c]);
-            tmem_ld_wait();
-            tc_fence_before();
-            mbar_arrive(bar(B_SFREE + sb));
-
-            const int kbase = (j_base + j) * BN;
-            if (kbase + BN - 1 > lim) {
-#pragma unroll
-                for (int c = 0; c < 4; ++c)
-#pragma unroll
-                    for (int e = 0; e < 32; ++e)
-                        if (kbase + c * 32 + e > lim) sv[c][e] = __float_as_uint(-CUDART_INF_F);
-            }
-            // row max with 8 independent chains (no 128-long dependency)
-            float mx8[8];
-#pragma unroll
-            for (int e = 0; e < 8; ++e) mx8[e] = -CUDART_INF_F;
-#pragma unroll
-            for (int c = 0; c < 4; ++c)
-#pragma unroll
-                for (int e = 0; e < 32; ++e)
-                    mx8[e & 7] = fmaxf(mx8[e & 7], __uint_as_float(sv[c][e]));
-            const float mx = fmaxf(fmaxf(fmaxf(mx8[0], mx8[1]), fmaxf(mx8[2], mx8[3])),
-                                   fmaxf(fmaxf(mx8[4], mx8[5]), fmaxf(mx8[6], mx8[7])));
-            const float m_new = fmaxf(m_run, mx * sc);
-            const bool resc = m_new > m_run + 8.0f;       // false while nothing is visible
-            const float m_use = resc ? m_new : m_run;
-            const float alpha = resc ? ex2(m_run - m_new) : 1.0f;
-            const float m_sub = m_use == -CUDART_INF_F ? 0.f : m_use;   // all masked so far
-
-            const int pb = j & 1;
-            // P buffer pb is free once P_{j-2}.V_{j-2} has finished
-            if (j >= 2) mbar_wait(bar(B_PFREE + pb), (uint32_t)((j - 2) >> 1) & 1u, P.err);
-            if (j >= 1 && __any_sync(0xffffffffu, resc)) {
-                // O must hold every P.V up to tile j-1 before it is rescaled
-                mbar_wait(bar(B_PFREE + (pb ^ 1)), (uint32_t)((j - 1) >> 1) & 1u, P.err);
-                tc_fence_after();
-#pragma unroll
-                for (int c = 0; c < 4; ++c) {
-                    uint32_t ov[32];
-                    tmem_ld32(tmem + lane_addr + kColO + c * 32, ov);
-                    tmem_ld_wait();
-#pragma unroll
-                    for (int e = 0; e < 32; ++e) ov[e] = __float_as_uint(__uint_as_float(ov[e]) * alpha);
-                    tmem_st32(tmem + lane_addr + kColO + c * 32, ov);
-                }
-                tmem_st_wait();
-            }
-            float ps[8];
-#pragma unroll
-            for (int e = 0; e < 8; ++e) ps[e] = 0.f;
-            // P_j (bf16, keys 2c and 2c+1 packed in column c) into TMEM buffer pb
-            const uint32_t p_addr = tmem + lane_addr + kColP + (uint32_t)pb * (BN / 2);
-#pragma unroll
-            for (int half = 0; half < 2; ++half) {
-                uint32_t pk[32];
-#pragma unroll
-                for (int cc = 0; cc < 2; ++cc) {
-                    const int c = half * 2 + cc;
-#pragma unroll
-                    for (int e = 0; e < 32; e += 2) {
-                        const float a0 = ex2(fmaf(__uint_as_float(sv[c][e]), sc, -m_sub));
-                        const float a1 = ex2(fmaf(__uint_as_float(sv[c][e + 1]), sc, -m_sub));
-                        ps[e & 7] += a0;
-                        ps[(e + 1) & 7] += a1;
-                        pk[cc * 16 + (e >> 1)] = pack_bf16(a0, a1);
-                    }
-                }
-                tmem_st32(p_addr + (uint32_t)half * 32u, pk);
-            }
-            tmem_st_wait();
-            const float sum = ((ps[0] + ps[1]) + (ps[2] + ps[3])) + ((ps[4] + ps[5]) + (ps[6] + ps[7]));
-            l_run = l_run * alpha + sum;
-            m_run = m_use;
-            tc_fence_before();
-            mbar_arrive(bar(B_PF + pb));
-        }
-
-        // ---------------------------------------------------------------- epilogue
-        if (n_kv > 0) {
-            mbar_wait(bar(B_PFREE + ((n_kv - 1) & 1)), (uint32_t)((n_kv - 1) >> 1) & 1u, P.err);
-            tc_fence_after();
-        }
-        const int t = t0 + r / G;
-        const int g = r - (r / G) * G;
-        const bool any = l_run > 0.f;                 // some key of this split was visible
-        const float inv = any ? 1.0f / l_run : 0.f;
-        const int64_t row_id = (((int64_t)l * P.batch_total + b) * P.sq + t) * P.hq + hk * G + g;
-        const int64_t lse_id = (((int64_t)l * P.batch_total + b) * P.hq + hk * G + g) * P.sq + t;
-        if (P.n_split == 1) {
-            __nv_bfloat16* orow = static_cast<__nv_bfloat16*>(P.out) + row_id * HD;
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                uint32_t ov[32];
-                tmem_ld32(tmem + lane_addr + kColO + c * 32, ov);
-                tmem_ld_wait();
-                if (t < P.sq) {
-#pragma unroll
-                    for (int q8 = 0; q8 < 4; ++q8) {
-                        uint4 w;
-                        w.x = pack_bf16(__uint_as_float(ov[q8 * 8 + 0]) * inv, __uint_as_float(ov[q8 * 8 + 1]) * inv);
-                        w.y = pack_bf16(__uint_as_float(ov[q8 * 8 + 2]) * inv, __uint_as_float(ov[q8 * 8 + 3]) * inv);
-                        w.z = pack_bf16(__uint_as_float(ov[q8 * 8 + 4]) * inv, __uint_as_float(ov[q8 * 8 + 5]) * inv);
-                        w.w = pack_bf16(__uint_as_float(ov[q8 * 8 + 6]) * inv, __uint_as_float(ov[q8 * 8 + 7]) * inv);
-                        *reinterpret_cast<uint4*>(orow + c * 32 + q8 * 8) = w;
-                    }
-                }
-            }
-            if (P.lse != nullptr && t < P.sq)
-                P.lse[lse_id] = (m_run + log2f(l_run)) * 0.69314718055994531f;
-        } else {
-            // partial over this split's keys: normalised O (fp32) and its log2-domain lse
-            const int64_t part_rows = (int64_t)P.lq * P.batch_total * P.sq * P.hq;
-            float* orow = P.part_o + ((int64_t)sp * part_rows + row_id) * HD;
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                uint32_t ov[32];
-                if (n_kv > 0) {
-                    tmem_ld32(tmem + lane_addr + kColO + c * 32, ov);
-                    tmem_ld_wait();
-                } else {
-#pragma unroll
-                    for (int e = 0; e < 32; ++e) ov[e] = 0u;
-                }
-                if (t < P.sq) {
-#pragma unroll
-                    for (int q4 = 0; q4 < 8; ++q4) {
-                        float4 w = make_float4(__uint_as_float(ov[q4 * 4 + 0]) * inv, __uint_as_float(ov[q4 * 4 + 1]) * inv,
-                                               __uint_as_float(ov[q4 * 4 + 2]) * inv, __uint_as_float(ov[q4 * 4 + 3]) * inv);
-                        *reinterpret_cast<float4*>(orow + c * 32 + q4 * 4) = w;
-                    }
-                }
-            }
-            if (t < P.sq)
-                P.part_lse[(int64_t)sp * part_rows + lse_id] = any ? m_run + log2f(l_run) : -CUDART_INF_F;
-        }
+        const int x = warp >= 8 ? 1 : 0;               // tile A (warps 4..7) or B (8..11)
+        if (x == 0 || has_b)
+            softmax_tile(P, tmem, sBar, x, warp & 3, lane, x ? t0b : t0a, l, bl, b, hk, sp, j_base,
+                         n_kv, abort);
     }
 
     tc_fence_before();
@@ -633,9 +766,10 @@ bool encode(CUtensorMap* tm, const void* base, int rank, const cuuint64_t* dims,
 
 }  // namespace
 
-int64_t attn_tc_units(const AttnParams& a) {
-    const int tq = BM / (a.hq / a.hkv);
-    return (int64_t)((a.sq + tq - 1) / tq) * a.hkv * a.lq * a.batch;
+int64_t attn_tc_units(int hq, int hkv, int sq, int lq, int batch) {
+    const int tq = BM / (hq / hkv);
+    const int64_t tiles = (sq + tq - 1) / tq;
+    return (tiles + 1) / 2 * hkv * lq * batch;     // one CTA per pair of query tiles
 }
 
 cudaError_t launch_attn_combine(const AttnParams& a, cudaStream_t s) {
@@ -659,6 +793,16 @@ cudaError_t launch_attn_tc(const AttnParams& a, cudaStream_t s) {
     cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)kSmemBytes);
     if (e != cudaSuccess) return e;
+    {   // the register split must not ask for more than the launch holds
+        static int launch_regs = -1;
+        if (launch_regs < 0) {
+            cudaFuncAttributes fa{};
+            e = cudaFuncGetAttributes(&fa, attn_tc_kernel);
+            if (e != cudaSuccess) return e;
+            launch_regs = fa.numRegs;
+        }
+        if (launch_regs * kThreads < 128 * kRegsLow + 256 * kRegsHigh) return cudaErrorInvalidConfiguration;
+    }
     TcParams p;
     std::memset(&p, 0, sizeof(p));
     const int G = a.hq / a.hkv;
@@ -698,7 +842,8 @@ cudaError_t launch_attn_tc(const AttnParams& a, cudaStream_t s) {
     p.part_o = a.part_o;
     p.part_lse = a.part_lse;
     std::memcpy(p.req, a.req, sizeof(ReqParam) * (size_t)a.batch);
-    const int64_t gx = (int64_t)((a.sq + tq - 1) / tq) * p.n_split;
+    const int64_t pairs = ((a.sq + tq - 1) / tq + 1) / 2;
+    const int64_t gx = pairs * p.n_split;
     if (gx > 0x7fffffffLL) return cudaErrorInvalidValue;
     const dim3 grid((unsigned)gx, a.hkv, a.lq * a.batch);
     if (grid.z > 65535u || grid.y > 65535u) return cudaErrorInvalidValue;

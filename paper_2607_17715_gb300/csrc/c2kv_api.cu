@@ -608,8 +608,8 @@ c2kv_status c2kv_attend(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
         int32_t n_split = 1;
         float* part = nullptr;
         if (use_tc) {
-            const int64_t tq = 128 / (c->cfg.n_q_heads / c->cfg.n_kv_heads);
-            const int64_t units = (n_suffix + tq - 1) / tq * c->cfg.n_kv_heads * lq * B;
+            const int64_t units =
+                c2kv::attn_tc_units(c->cfg.n_q_heads, c->cfg.n_kv_heads, n_suffix, lq, B);
             int32_t n_kv_max = 1;
             for (int32_t b = 0; b < B; ++b)
                 n_kv_max = std::max<int32_t>(n_kv_max, (cache->n_slots[b] + n_suffix + 127) / 128);

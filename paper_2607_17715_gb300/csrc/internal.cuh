@@ -137,7 +137,8 @@ cudaError_t launch_attn_tc(const AttnParams& p, cudaStream_t s);
 // Merge n_split partial (O, lse) over disjoint key ranges into out (bf16) and lse (attn_tc.cu).
 cudaError_t launch_attn_combine(const AttnParams& p, cudaStream_t s);
 // Work units (CTAs per split) the tensor-core kernel launches for these parameters.
-int64_t attn_tc_units(const AttnParams& p);
+// CTAs of one tensor-core attention launch before key-range splitting.
+int64_t attn_tc_units(int hq, int hkv, int sq, int lq, int batch);
 
 // Read-only view of a context and one of its caches, for entry points defined outside
 // c2kv_api.cu (c2kv_attend_noalloc).
