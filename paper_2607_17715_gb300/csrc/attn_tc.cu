@@ -62,8 +62,8 @@ constexpr int kThreads = 384;
 // thread (the cap that 384 threads leave, 3 warps per SM sub-partition); the split below
 // hands out exactly that total, which the host checks against the compiled count.
 constexpr int kLaunchRegs = 168;
-constexpr int kRegsLow = 104;
-constexpr int kRegsHigh = 200;
+constexpr int kRegsLow = 136;
+constexpr int kRegsHigh = 184;
 static_assert(128 * kRegsLow + 256 * kRegsHigh <= kThreads * kLaunchRegs, "register split");
 constexpr uint32_t kTmemCols = 512;     // S_A, S_B, O_A, O_B; P_x over the first half of S_x
 constexpr uint32_t kColS = 0, kColO = 256;
@@ -458,13 +458,18 @@ __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, u
 }
 
 // The MMA issuer (one thread).  The tensor core's queue holds about one MMA, so anything
-// the issuing thread does between two MMAs idles it: descriptors are precomputed and the
-// ring stages advance by counters.  Each block waits for its own inputs only: a wait for a
-// later block's P inside an S block would hold that S back until the other tile's softmax
-// finished, putting the two softmaxes in series.
+// the issuing thread does between two MMAs idles it, and a branch there costs about as much
+// as an MMA.  So the descriptors are precomputed, the issue blocks are straight-line code,
+// and the main loop is unrolled over six key tiles (the least common multiple of the two
+// ring depths): every ring stage and every barrier parity in it is a compile-time constant.
+// Each block waits for its own inputs only: waiting for a later block's P inside an S block
+// would hold that S back until the other tile's softmax finished, putting the two softmaxes
+// in series.
+template <bool kHasB>
 __device__ __forceinline__ void mma_issuer(const TcParams& P, uint32_t tmem, uint32_t sQ, uint32_t sK,
-                                           uint32_t sV, uint32_t sBar, bool has_b, int n_kv,
+                                           uint32_t sV, uint32_t sBar, int n_kv,
                                            volatile uint32_t* abort) {
+    static_assert(KSTAGES == 3 && VSTAGES == 2, "the unrolled schedule assumes 3 K and 2 V stages");
     auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
     constexpr uint32_t idS = idesc_bf16(BM, BN, false);
     constexpr uint32_t idO = idesc_bf16(BM, HD, true);
@@ -485,76 +490,78 @@ __device__ __forceinline__ void mma_issuer(const TcParams& P, uint32_t tmem, uin
             mma_bf16(d, dq + off, dk + off, idS, kk > 0 ? 1u : 0u);
         }
     };
-    // O += P V with P (bf16 pairs) from TMEM: 16 keys (8 columns) per step
-    auto pv_block = [&](uint32_t p, uint64_t dv, uint32_t o, bool first) {
+    // O += P V with P (bf16 pairs) from TMEM: 16 keys (8 columns) per step; the first step
+    // of the first block overwrites O
+    auto pv_block = [&](uint32_t p, uint64_t dv, uint32_t o, uint32_t acc0) {
 #pragma unroll
-        for (int kk = 0; kk < BN / 16; ++kk) {
+        for (int kk = 0; kk < BN / 16; ++kk)
             mma_bf16_ts(o, p + (uint32_t)kk * 8u, dv + (uint64_t)((kk * 2048) >> 4), idO,
-                        (!first || kk > 0) ? 1u : 0u);
-        }
+                        kk > 0 ? 1u : acc0);
     };
     auto wait = [&](int i, uint32_t parity) {
         mbar_wait(bar(i), parity, P.err, abort);
         tc_fence_after();
     };
-
-    // ring positions: stage index and the phase parity of its current fill
-    int ks = 0, vs = 0;
-    uint32_t kph = 0, vph = 0;
-    uint64_t dk = dK0, dv = dV0;
-    auto next_k = [&] {
-        if (++ks == KSTAGES) { ks = 0; kph ^= 1u; dk = dK0; } else { dk += kTileDesc; }
-    };
-    auto next_v = [&] {
-        if (++vs == VSTAGES) { vs = 0; vph ^= 1u; dv = dV0; } else { dv += kTileDesc; }
+    // one key tile j >= 1:  PV_A(j-1)  S_A(j)  PV_B(j-1)  S_B(j)
+    //   ks, kph: K stage and fill parity of tile j;  vs, vph: V stage and parity of tile j-1;
+    //   pp: parity of P_x(j-1);  acc0: 0 only for the first P.V (j == 1)
+    auto tile = [&](int ks, uint32_t kph, int vs, uint32_t vph, uint32_t pp, uint32_t acc0) {
+        const uint64_t dk = dK0 + (uint64_t)ks * kTileDesc;
+        const uint64_t dv = dV0 + (uint64_t)vs * kTileDesc;
+        wait(B_PF + 0, pp);
+        wait(B_VF + vs, vph);
+        pv_block(tS_a, dv, tO_a, acc0);
+        wait(B_KF + ks, kph);
+        s_block(dQa, dk, tS_a);
+        mma_commit(bar(B_SF + 0));
+        if (kHasB) {
+            wait(B_PF + 1, pp);
+            pv_block(tS_b, dv, tO_b, acc0);
+        }
+        mma_commit(bar(B_VE + vs));
+        if (kHasB) {
+            s_block(dQb, dk, tS_b);
+            mma_commit(bar(B_SF + 1));
+        }
+        mma_commit(bar(B_KE + ks));
     };
 
     wait(B_Q, 0u);
     wait(B_KF + 0, 0u);
     // key tile 0: S_A(0), S_B(0)
-    s_block(dQa, dk, tS_a);
+    s_block(dQa, dK0, tS_a);
     mma_commit(bar(B_SF + 0));
-    if (has_b) {
-        s_block(dQb, dk, tS_b);
+    if (kHasB) {
+        s_block(dQb, dK0, tS_b);
         mma_commit(bar(B_SF + 1));
     }
     mma_commit(bar(B_KE + 0));
-    next_k();
-    // key tiles 1 .. n_kv-1:  PV_A(j-1)  S_A(j)  PV_B(j-1)  S_B(j).  While the softmax of tile
-    // A works on S_A(j), the tensor core runs PV_B(j-1) and S_B(j), and the other way round.
+    // tiles 1 .. n_kv-1, ring positions advanced without branches
+    int ks = 1, vs = 0;
+    uint32_t kph = 0u, vph = 0u, acc0 = 0u;
     for (int j = 1; j < n_kv; ++j) {
-        const uint32_t pj = (uint32_t)(j - 1) & 1u;      // parity of P_x(j-1)
-        const bool first = j == 1;
-        wait(B_PF + 0, pj);
-        wait(B_VF + vs, vph);
-        pv_block(tS_a, dv, tO_a, first);
-        wait(B_KF + ks, kph);
-        s_block(dQa, dk, tS_a);
-        mma_commit(bar(B_SF + 0));
-        if (has_b) {
-            wait(B_PF + 1, pj);
-            pv_block(tS_b, dv, tO_b, first);
-        }
-        mma_commit(bar(B_VE + vs));
-        next_v();
-        if (has_b) {
-            s_block(dQb, dk, tS_b);
-            mma_commit(bar(B_SF + 1));
-        }
-        mma_commit(bar(B_KE + ks));
-        next_k();
+        tile(ks, kph, vs, vph, (uint32_t)(j - 1) & 1u, acc0);
+        acc0 = 1u;
+        const bool kw = ks == KSTAGES - 1;
+        ks = kw ? 0 : ks + 1;
+        kph ^= kw ? 1u : 0u;
+        const bool vw = vs == VSTAGES - 1;
+        vs = vw ? 0 : vs + 1;
+        vph ^= vw ? 1u : 0u;
     }
-    // last P.V pair
+    // last P.V pair: P_x(n_kv - 1), V stage (n_kv - 1) % 2
+    const int vl = vs;
+    const uint32_t vphl = vph;
     const uint32_t pl = (uint32_t)(n_kv - 1) & 1u;
-    const bool first = n_kv == 1;
+    const uint64_t dvl = dV0 + (uint64_t)vl * kTileDesc;
     wait(B_PF + 0, pl);
-    wait(B_VF + vs, vph);
-    pv_block(tS_a, dv, tO_a, first);
-    if (has_b) {
+    wait(B_VF + vl, vphl);
+    pv_block(tS_a, dvl, tO_a, acc0);
+    if (kHasB) {
         wait(B_PF + 1, pl);
-        pv_block(tS_b, dv, tO_b, first);
+        pv_block(tS_b, dvl, tO_b, acc0);
     }
-    mma_commit(bar(B_VE + vs));
+    mma_commit(bar(B_VE + vl));
     mma_commit(bar(B_OD));
 }
 
@@ -667,7 +674,10 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_const
             }
         } else if (warp == 1 && lane == 0 && n_kv > 0) {
             // ------------------------------------------------------------ MMA issuer
-            mma_issuer(P, tmem, sQ, sK, sV, sBar, has_b, n_kv, abort);
+            if (has_b)
+                mma_issuer<true>(P, tmem, sQ, sK, sV, sBar, n_kv, abort);
+            else
+                mma_issuer<false>(P, tmem, sQ, sK, sV, sBar, n_kv, abort);
         }
     } else {
         asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegsHigh));
