@@ -109,7 +109,7 @@ typedef struct c2kv_cache_desc {
 } c2kv_cache_desc;
 
 /* ABI version of this header (bumped on any incompatible change). */
-#define C2KV_ABI_VERSION 1
+#define C2KV_ABI_VERSION 2
 int32_t c2kv_abi_version(void);
 
 /*
@@ -250,6 +250,34 @@ c2kv_status c2kv_attend_noalloc(c2kv_ctx* ctx, c2kv_cache* cache, int32_t layer,
                                 const void* q, const void* k_suf, const void* v_suf,
                                 int32_t n_suffix, void* out, float* lse);
 
+/*
+ * c2kv_decode -- one generation step after the suffix (the decode phase that follows the
+ * first token; time between tokens): for each request r the new token, suffix index
+ * steps[r], sits at position L_r + steps[r].  Its Q and K are RoPE'd there, its K/V written
+ * to cache row S_r + steps[r], and
+ *     O[h] = softmax_j( Q_h . K_j,h/G / sqrt(d) ) V_j,h/G      over keys j <= S_r + steps[r]
+ * (every composed slot and suffix rows 0 .. steps[r]; G = Hq / Hkv).  This is the same
+ * operator as c2kv_attend for one query row (Sec. 3.2.2).  Rows S_r .. S_r + steps[r] - 1
+ * must already hold the earlier suffix tokens (written by c2kv_attend or earlier decode
+ * calls); the library does not track which rows were written.  A later c2kv_attend zeroes
+ * the rows after its own suffix up to the next 128-row boundary, decoded rows included.
+ *
+ *   layer : layer index, or -1 for all layers in one launch.
+ *   q     : device [Lq][B][Hq][d] pre-RoPE query of the new token (Lq = L if layer == -1).
+ *   k_new, v_new : device [Lq][B][Hkv][d] pre-RoPE K, V of the new token.
+ *   steps : host int32[B], 0 <= steps[r] < the cache's suffix_capacity.
+ *   out   : device [Lq][B][Hq][d] attention output (context dtype).
+ *   lse   : device [Lq][B][Hq] fp32 natural-log softmax normaliser, or NULL.
+ * The key range of each (layer, request, KV head) is split over several CTAs and merged
+ * exactly (log-sum-exp); the split buffer comes from the context's memory pool.
+ * Errors: ERR_ARG, ERR_STATE (cache from another context), ERR_UNSUPPORTED (head layout the
+ * decode kernel does not take: G = Hq/Hkv in {1,2,4,8,16}, d in {64,128}, G*d <= 1024, and
+ * G <= 8 for bf16), ERR_NOMEM, ERR_CUDA.
+ */
+c2kv_status c2kv_decode(c2kv_ctx* ctx, c2kv_cache* cache, int32_t layer, const void* q,
+                        const void* k_new, const void* v_new, const int32_t* steps, void* out,
+                        float* lse);
+
 /* c2kv_cache_release -- free a composed cache (stream-ordered). */
 c2kv_status c2kv_cache_release(c2kv_ctx* ctx, c2kv_cache* cache);
 
@@ -274,7 +302,8 @@ const char* c2kv_last_error(const c2kv_ctx* ctx);
 #define C2KV_PROF_SUFFIX   2   /* suffix RoPE + append + pad zeroing */
 #define C2KV_PROF_ATTN     3   /* the attention kernel alone */
 #define C2KV_PROF_COMBINE  4   /* merge of key-range splits (when attention was split) */
-#define C2KV_PROF_KINDS    5
+#define C2KV_PROF_DECODE   5   /* decode attention (with the merge of its splits) */
+#define C2KV_PROF_KINDS    6
 c2kv_status c2kv_profile_enable(c2kv_ctx* ctx, int32_t on);
 /* mean_ms[C2KV_PROF_KINDS] receives mean milliseconds (0 where none), launches[] the
  * counts; either may be NULL. */

@@ -18,7 +18,8 @@ What it computes (C2KV, arXiv 2607.17715):
   spans its original token length), then concatenated.  With RoPE this is a rotation of
   the stored K by the chunk's offset; V is copied.
 * Inference (Sec. 2.2, Eq. for F).  The suffix (query) tokens run standard attention over
-  [composed cache; suffix], causal inside the suffix, every composed slot visible.
+  [composed cache; suffix], causal inside the suffix, every composed slot visible.  A
+  decode step is the same operator for one new token over everything cached before it.
 
 RoPE is the rotate-half form used by the Llama / Qwen models the paper evaluates
 (Sec. 4.1): channel i pairs with i + d/2 and turns by pos * theta^(-2i/d).
@@ -267,6 +268,45 @@ def attend(k_c, v_c, l_req: int, q, k_suf, v_suf, theta: float, dtype: str):
             tot = e.sum(axis=1, keepdims=True)
             out[layer, :, h, :] = (e / tot) @ vals[:, g, :]
             lse[layer, h, :] = (mx + np.log(tot))[:, 0]
+    return out, lse
+
+
+def decode_step(k_c, v_c, l_req: int, k_prev, v_prev, q_new, k_new, v_new, step: int,
+                theta: float, dtype: str):
+    """One generation step after the suffix, for one request.
+
+    The new token is suffix token ``step``; suffix tokens 0 .. step-1 (pre-RoPE k_prev,
+    v_prev [L, step, Hkv, d]) are already in the cache at positions L_req + t.  The new
+    token's q_new [L, Hq, d] and k_new, v_new [L, Hkv, d] (pre-RoPE) sit at L_req + step.
+    Its single query row attends to every key: the composed slots k_c, v_c [L, S, Hkv, d]
+    and suffix rows 0 .. step (the same standard attention as ``attend``, Sec. 3.2.2, for
+    one query; nothing is masked because every cached key precedes it).
+    Returns O [L, Hq, d] (float64) and lse [L, Hq] (natural log).
+    """
+    k_c = np.asarray(k_c, np.float64)
+    v_c = np.asarray(v_c, np.float64)
+    n_layers, _, hkv, d = k_c.shape
+    hq = q_new.shape[1]
+    grp = hq // hkv
+    prev_pos = suffix_positions(l_req, step)
+    out = np.zeros((n_layers, hq, d))
+    lse = np.zeros((n_layers, hq))
+    for layer in range(n_layers):
+        q_r = store(rope(q_new[layer][None], [l_req + step], theta), dtype)[0]      # [Hq, d]
+        k_old = store(rope(k_prev[layer], prev_pos, theta), dtype) if step else \
+            np.zeros((0, hkv, d))
+        k_now = store(rope(k_new[layer][None], [l_req + step], theta), dtype)
+        keys = np.concatenate([k_c[layer], k_old, k_now], axis=0)                 # [S+step+1, Hkv, d]
+        vals = np.concatenate([v_c[layer], np.asarray(v_prev[layer], np.float64).reshape(-1, hkv, d),
+                               np.asarray(v_new[layer], np.float64)[None]], axis=0)
+        for h in range(hq):
+            g = h // grp
+            s = keys[:, g, :] @ q_r[h] / math.sqrt(d)                              # [keys]
+            mx = s.max()
+            e = np.exp(s - mx)
+            tot = e.sum()
+            out[layer, h] = (e / tot) @ vals[:, g, :]
+            lse[layer, h] = mx + math.log(tot)
     return out, lse
 
 

@@ -29,8 +29,9 @@ ERR_POSITIONS, ERR_CUDA, ERR_DEVICE_BOUNDS, ERR_STATE, ERR_UNSUPPORTED = -6, -7,
 DTYPE_BF16, DTYPE_F32 = 0, 1
 MODE_MEANPOOL, MODE_PROVIDED, MODE_STORED, MODE_HOST = 0, 1, 2, 3
 ATTN_AUTO, ATTN_SIMT, ATTN_TC = 0, 1, 2
-PROF_COMPOSE, PROF_COMPRESS, PROF_SUFFIX, PROF_ATTN, PROF_COMBINE, PROF_KINDS = 0, 1, 2, 3, 4, 5
-PROF_NAMES = ("compose", "compress", "suffix", "attention", "combine")
+PROF_COMPOSE, PROF_COMPRESS, PROF_SUFFIX, PROF_ATTN, PROF_COMBINE, PROF_DECODE = 0, 1, 2, 3, 4, 5
+PROF_KINDS = 6
+PROF_NAMES = ("compose", "compress", "suffix", "attention", "combine", "decode")
 
 STATUS_NAMES = {
     0: "OK", -1: "ERR_ARG", -2: "ERR_DTYPE", -3: "ERR_NOMEM", -4: "ERR_POOL_FULL",
@@ -77,6 +78,7 @@ _SIGS = {
     "c2kv_cache_info": (_I32, [_VP, ctypes.POINTER(c2kv_cache_desc)]),
     "c2kv_attend": (_I32, [_VP, _VP, _I32, _VP, _VP, _VP, _I32, _VP, _VP]),
     "c2kv_attend_noalloc": (_I32, [_VP, _VP, _I32, _VP, _VP, _VP, _I32, _VP, _VP]),
+    "c2kv_decode": (_I32, [_VP, _VP, _I32, _VP, _VP, _VP, _P32, _VP, _VP]),
     "c2kv_cache_release": (_I32, [_VP, _VP]),
     "c2kv_sync": (_I32, [_VP]),
     "c2kv_last_error": (ctypes.c_char_p, [_VP]),
@@ -206,6 +208,13 @@ def c2kv_attend_noalloc(ctx, cache, layer, q, k_suf, v_suf, n_suffix, out, lse=N
     see include/c2kv.h for the limits)."""
     _check(_lib.c2kv_attend_noalloc(ctx, cache, layer, _ptr(q), _ptr(k_suf), _ptr(v_suf),
                                     n_suffix, _ptr(out), _ptr(lse)), ctx)
+
+
+def c2kv_decode(ctx, cache, layer, q, k_new, v_new, steps, out, lse=None):
+    """One decode step: request r's new token at suffix index steps[r] (host int array)."""
+    st, st_p = _i32(steps)
+    _check(_lib.c2kv_decode(ctx, cache, layer, _ptr(q), _ptr(k_new), _ptr(v_new), st_p,
+                            _ptr(out), _ptr(lse)), ctx)
 
 
 def c2kv_cache_release(ctx, cache):

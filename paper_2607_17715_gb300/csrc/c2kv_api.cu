@@ -652,6 +652,7 @@ c2kv_status c2kv_attend(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
             s.sq = n_suffix;
             s.hq = c->cfg.n_q_heads;
             s.hkv = c->cfg.n_kv_heads;
+            s.pad_rows = 1;
             s.rope = c->turns;
             for (int32_t i = 0; i < nb; ++i)
                 s.req[i] = c2kv::ReqParam{cache->row_base[b0 + i], cache->n_slots[b0 + i],
@@ -697,6 +698,111 @@ c2kv_status c2kv_attend(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
         return C2KV_OK;
     } catch (const std::bad_alloc&) {
         return fail(c, C2KV_ERR_NOMEM, "attend: host allocation failed");
+    }
+}
+
+c2kv_status c2kv_decode(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const void* q,
+                        const void* k_new, const void* v_new, const int32_t* steps, void* out,
+                        float* lse) {
+    if (!c) return C2KV_ERR_ARG;
+    try {
+        c->err.clear();
+        if (!own_cache(c, cache)) return fail(c, C2KV_ERR_STATE, "decode: cache not owned by this context");
+        if (!q || !k_new || !v_new || !steps || !out) return fail(c, C2KV_ERR_ARG, "decode: null pointer");
+        if (layer < -1 || layer >= c->cfg.layers) return fail(c, C2KV_ERR_ARG, "decode: bad layer %d", layer);
+        if (!c2kv::decode_supported(c->cfg.dtype, c->cfg.head_dim, c->cfg.n_q_heads, c->cfg.n_kv_heads))
+            return fail(c, C2KV_ERR_UNSUPPORTED, "decode: head layout not supported");
+        const int32_t B = cache->batch;
+        int32_t n_keys_max = 1;
+        for (int32_t b = 0; b < B; ++b) {
+            if (steps[b] < 0 || steps[b] >= cache->suffix_capacity)
+                return fail(c, C2KV_ERR_ARG, "decode: steps[%d] = %d outside [0, %d)", b, steps[b],
+                            cache->suffix_capacity);
+            n_keys_max = std::max<int32_t>(n_keys_max, cache->n_slots[b] + steps[b] + 1);
+        }
+        if (B == 0) return C2KV_OK;
+        const int32_t lq = layer < 0 ? c->cfg.layers : 1;
+        const int32_t layer0 = layer < 0 ? 0 : layer;
+        const int32_t hq = c->cfg.n_q_heads, hkv = c->cfg.n_kv_heads, d = c->cfg.head_dim;
+        // key-range splits: about two CTAs per SM over all (layer, request, KV head), and at
+        // least 256 keys per split
+        const int64_t units = (int64_t)hkv * lq * std::min<int32_t>(B, c2kv::kMaxReq);
+        int32_t n_split = (int32_t)std::min<int64_t>(64, std::max<int64_t>(1, (2 * c->sms + units - 1) / units));
+        n_split = std::max<int32_t>(1, std::min<int32_t>(n_split, (n_keys_max + 255) / 256));
+        const int32_t keys_per_split = (n_keys_max + n_split - 1) / n_split;
+
+        const size_t q_bytes = (size_t)lq * B * hq * d * c->eb;
+        void* q_rot = nullptr;
+        cudaError_t e = pool_alloc(c, &q_rot, q_bytes);
+        if (e != cudaSuccess) return cuda_fail(c, e, "decode: scratch allocation");
+        float* part = nullptr;
+        const size_t rows_all = (size_t)lq * B * hq;
+        if (n_split > 1) {
+            e = pool_alloc(c, reinterpret_cast<void**>(&part), (size_t)n_split * rows_all * (d + 1) * sizeof(float));
+            if (e != cudaSuccess) {
+                pool_free(c, q_rot);
+                return cuda_fail(c, e, "decode: split scratch allocation");
+            }
+        }
+        for (int32_t b0 = 0; e == cudaSuccess && b0 < B; b0 += c2kv::kMaxReq) {
+            const int32_t nb = std::min<int32_t>(c2kv::kMaxReq, B - b0);
+            c2kv::SuffixParams s{};
+            s.q = q;
+            s.k = k_new;
+            s.v = v_new;
+            s.q_rot = q_rot;
+            s.cache_k = cache->k;
+            s.cache_v = cache->v;
+            s.pos = cache->pos;
+            s.rows = cache->rows;
+            s.layer0 = layer0;
+            s.lq = lq;
+            s.batch = nb;
+            s.batch_total = B;
+            s.b0 = b0;
+            s.sq = 1;
+            s.hq = hq;
+            s.hkv = hkv;
+            s.pad_rows = 0;
+            s.rope = c->turns;
+            for (int32_t i = 0; i < nb; ++i)
+                s.req[i] = c2kv::ReqParam{cache->row_base[b0 + i], cache->n_slots[b0 + i],
+                                          cache->l_req[b0 + i], steps[b0 + i]};
+            {
+                ProfScope prof_suffix(c, C2KV_PROF_SUFFIX);
+                e = c2kv::launch_suffix_prep(s, c->cfg.dtype, d, c->stream);
+            }
+            if (e != cudaSuccess) break;
+            c2kv::DecodeParams p{};
+            p.q_rot = q_rot;
+            p.cache_k = cache->k;
+            p.cache_v = cache->v;
+            p.out = out;
+            p.lse = lse;
+            p.part_o = part;
+            p.part_lse = part ? part + (size_t)n_split * rows_all * d : nullptr;
+            p.rows = cache->rows;
+            p.layer0 = layer0;
+            p.lq = lq;
+            p.batch = nb;
+            p.batch_total = B;
+            p.b0 = b0;
+            p.hq = hq;
+            p.hkv = hkv;
+            p.d = d;
+            p.n_split = n_split;
+            p.keys_per_split = keys_per_split;
+            p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)d));
+            for (int32_t i = 0; i < nb; ++i) p.req[i] = s.req[i];
+            ProfScope prof_decode(c, C2KV_PROF_DECODE);
+            e = c2kv::launch_decode(p, c->cfg.dtype, c->stream);
+        }
+        pool_free(c, part);
+        pool_free(c, q_rot);
+        if (e != cudaSuccess) return cuda_fail(c, e, "decode");
+        return C2KV_OK;
+    } catch (const std::bad_alloc&) {
+        return fail(c, C2KV_ERR_NOMEM, "decode: host allocation failed");
     }
 }
 

@@ -78,7 +78,8 @@ struct ReqParam {
     int32_t row_base;        // first cache row of the request
     int32_t n_slots;         // composed slots S_r
     int32_t l_req;           // composed span L_r (suffix token t sits at L_r + t)
-    int32_t pad;
+    int32_t t0;              // suffix index of this launch's first token (0 for attend; the
+                             // decode step for decode)
 };
 
 struct SuffixParams {
@@ -98,6 +99,7 @@ struct SuffixParams {
     int32_t sq;
     int32_t hq;
     int32_t hkv;
+    int32_t pad_rows;        // 1: zero the rows after the suffix up to the next 128-row boundary
     RopeTurns rope;
     ReqParam req[kMaxReq];
 };
@@ -130,6 +132,33 @@ cudaError_t launch_compose(const ComposeParams& p, int dtype, int d, int layers,
 cudaError_t launch_compress(const CompressParams& p, int dtype, int d, cudaStream_t s);
 cudaError_t launch_suffix_prep(const SuffixParams& p, int dtype, int d, cudaStream_t s);
 cudaError_t launch_attn_simt(const AttnParams& p, int dtype, int d, cudaStream_t s);
+
+// Decode attention (decode.cu): one new token per request (suffix index ReqParam::t0,
+// already rotated into q_rot and appended to the cache) over keys 0 .. S_r + t0.
+struct DecodeParams {
+    const void* q_rot;       // [Lq][Btot][Hq][d]
+    const void* cache_k;     // [L][rows][Hkv][d]
+    const void* cache_v;
+    void* out;               // [Lq][Btot][Hq][d]
+    float* lse;              // [Lq][Btot][Hq] or null
+    float* part_o;           // n_split > 1: [n_split][Lq][Btot][Hq][d] fp32, normalised
+    float* part_lse;         // n_split > 1: [n_split][Lq][Btot][Hq] fp32, log2 domain
+    int64_t rows;
+    int32_t layer0;
+    int32_t lq;
+    int32_t batch;
+    int32_t batch_total;
+    int32_t b0;
+    int32_t hq;
+    int32_t hkv;
+    int32_t d;
+    int32_t n_split;         // key-range splits per (layer, request, KV head)
+    int32_t keys_per_split;
+    float scale_log2;        // log2(e) / sqrt(d)
+    ReqParam req[kMaxReq];
+};
+bool decode_supported(int dtype, int d, int hq, int hkv);
+cudaError_t launch_decode(const DecodeParams& p, int dtype, cudaStream_t s);
 
 // Tensor-core attention (attn_tc.cu).
 bool attn_tc_supported(int dtype, int d, int hq, int hkv);

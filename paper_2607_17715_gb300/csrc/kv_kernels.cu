@@ -9,55 +9,11 @@
 // once to a float in [-1/2, 1/2) turns and handed to sincospif.  The error is about
 // 1e-7 rad at any position, where forming p * inv_freq in fp32 would lose p * 2^-24 rad.
 #include "internal.cuh"
+#include "vec16.cuh"
 
 namespace c2kv {
 namespace {
 
-template <typename T>
-struct Vec16;
-
-template <>
-struct Vec16<__nv_bfloat16> {
-    static constexpr int N = 8;
-    __device__ __forceinline__ static void unpack(const uint4& r, float* f) {
-        const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&r);
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            float2 t = __bfloat1622float2(h[i]);
-            f[2 * i] = t.x;
-            f[2 * i + 1] = t.y;
-        }
-    }
-    __device__ __forceinline__ static uint4 pack(const float* f) {
-        uint4 r;
-        __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&r);
-#pragma unroll
-        for (int i = 0; i < 4; ++i) h[i] = __floats2bfloat162_rn(f[2 * i], f[2 * i + 1]);
-        return r;
-    }
-};
-
-template <>
-struct Vec16<float> {
-    static constexpr int N = 4;
-    __device__ __forceinline__ static void unpack(const uint4& r, float* f) {
-        f[0] = __uint_as_float(r.x);
-        f[1] = __uint_as_float(r.y);
-        f[2] = __uint_as_float(r.z);
-        f[3] = __uint_as_float(r.w);
-    }
-    __device__ __forceinline__ static uint4 pack(const float* f) {
-        return make_uint4(__float_as_uint(f[0]), __float_as_uint(f[1]), __float_as_uint(f[2]),
-                          __float_as_uint(f[3]));
-    }
-};
-
-__device__ __forceinline__ uint4 ld16(const void* p) {
-    return __ldg(reinterpret_cast<const uint4*>(p));
-}
-__device__ __forceinline__ void st16(void* p, const uint4& v) {
-    *reinterpret_cast<uint4*>(p) = v;
-}
 
 // (cos, sin) of pos * theta^(-2i/d) from the 0.64 fixed-point turn of frequency i.
 __device__ __forceinline__ float2 turn_cs(uint64_t turn, int64_t pos) {
@@ -293,10 +249,10 @@ __global__ void __launch_bounds__(256) suffix_kernel(const __grid_constant__ Suf
     const int bl = blockIdx.x / P.sq;
     const int t = blockIdx.x - bl * P.sq;
     const ReqParam& rq = P.req[bl];
-    const int64_t position = (int64_t)rq.l_req + t;
+    const int64_t position = (int64_t)rq.l_req + rq.t0 + t;      // suffix index t0 + t
     if (threadIdx.x < HALF) cs[threadIdx.x] = turn_cs(P.rope.turn[threadIdx.x], position);
     __syncthreads();
-    const int64_t crow = (int64_t)rq.row_base + rq.n_slots + t;
+    const int64_t crow = (int64_t)rq.row_base + rq.n_slots + rq.t0 + t;
     if (threadIdx.x == 0 && l == 0 && crow >= 0 && crow < P.rows) P.pos[crow] = (int32_t)position;
     const int64_t grow = ((int64_t)l * P.batch_total + P.b0 + bl) * P.sq + t;  // tensor row
     const int nq = P.hq * VPH;
@@ -388,7 +344,7 @@ cudaError_t launch_compress(const CompressParams& p, int dtype, int d, cudaStrea
 cudaError_t launch_suffix_prep(const SuffixParams& p, int dtype, int d, cudaStream_t s) {
     (void)cudaGetLastError();   // report this launch's error only, not a stale one
     if (p.batch < 1 || p.sq < 1 || p.lq < 1) return cudaSuccess;
-    const int64_t blocks = (int64_t)p.batch * p.sq + p.batch;
+    const int64_t blocks = (int64_t)p.batch * p.sq + (p.pad_rows ? p.batch : 0);
     if (blocks > 0x7fffffffLL || p.lq > 65535) return cudaErrorInvalidValue;
     const dim3 grid((unsigned)blocks, p.lq);
     C2KV_DISPATCH(suffix_kernel, grid, p, dtype, d, s);

@@ -112,6 +112,7 @@ extern "C" c2kv_status c2kv_attend_noalloc(c2kv_ctx* ctx, c2kv_cache* cache, int
         s.sq = n_suffix;
         s.hq = v.n_q_heads;
         s.hkv = v.n_kv_heads;
+        s.pad_rows = 1;
         s.rope = v.turns;
         for (int32_t i = 0; i < nb; ++i)
             s.req[i] = c2kv::ReqParam{v.row_base[b0 + i], v.n_slots[b0 + i], v.l_req[b0 + i], 0};

@@ -12,6 +12,17 @@ def pytest_configure(config):
     config.addinivalue_line("markers", "gpu: needs a CUDA GPU (sm_103a) and the built library")
 
 
+def pytest_collection_modifyitems(config, items):
+    # A GPU test that stops making progress ends its process (thread method: a blocked CUDA
+    # call never returns to the interpreter) instead of holding the device; needs the
+    # pytest-timeout plugin, skipped without it.
+    if not config.pluginmanager.hasplugin("timeout"):
+        return
+    for item in items:
+        if item.get_closest_marker("gpu") is not None and item.get_closest_marker("timeout") is None:
+            item.add_marker(pytest.mark.timeout(300, method="thread"))
+
+
 @pytest.fixture(scope="session")
 def repo_root():
     return ROOT

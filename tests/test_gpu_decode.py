@@ -1,0 +1,148 @@
+"""Decode attention (one new token per request after the suffix) against the oracle's
+decode step: every composed slot and suffix rows 0 .. step as keys, one query row."""
+import numpy as np
+import pytest
+import torch
+
+import synth
+from oracle import c2kv_oracle as orc
+from tests import _gpu_helpers as H
+
+pytestmark = pytest.mark.gpu
+
+L8B_1 = synth.scaled(synth.workload("llama8b"), layers=1)
+TINY = synth.workload("tiny_f32")
+
+
+def _small(wl, **kw):
+    base = dict(batch=1, chunks_per_request=3, pool_chunks=3, chunk_tokens=256)
+    base.update(kw)
+    return synth.scaled(wl, **base)
+
+
+def _decode_case(wl, steps, prefill=None, layer=-1, extra_steps=0, attn_first=True):
+    """Compose the workload's requests, optionally run c2kv_attend over `prefill` suffix
+    tokens, then decode: request r's new token at suffix index steps[r] (and, with
+    extra_steps, the following steps one call at a time).  Every decode output and lse is
+    compared with the oracle's decode step for that request."""
+    c2kv = H.lib()
+    reqs = synth.requests(wl)
+    B = len(reqs)
+    n_tok = max(steps) + extra_steps + 1
+    wl_s = synth.scaled(wl, n_suffix=n_tok)
+    all_ids = sorted({c for ids, _ in reqs for c in ids})
+    chunks = H.oracle_chunks_meanpool(wl, all_ids)
+    pool = sum(orc.n_slots(wl.chunk_tokens, wl.ratio_k) for _ in all_ids) + 16
+    ctx = H.make_ctx(wl, pool_slots=pool)
+    try:
+        dev = H.load_stored(ctx, wl, chunks)
+        req_ptr = np.cumsum([0] + [len(ids) for ids, _ in reqs])
+        cache = c2kv.c2kv_compose(ctx, req_ptr, [dev[c] for ids, _ in reqs for c in ids],
+                                  [o for _, offs in reqs for o in offs], suffix_capacity=n_tok)
+        q, ks, vs = synth.suffix(wl_s, layers=wl.layers)          # [L, B, n_tok, H, d]
+        q, ks, vs = q[:, :B], ks[:, :B], vs[:, :B]
+        lsel = slice(None) if layer == -1 else slice(layer, layer + 1)
+        if prefill:
+            # write suffix tokens 0 .. prefill-1 with the suffix attention
+            qd, kd, vd = (H.to_dev(x[lsel, :, :prefill], wl) for x in (q, ks, vs))
+            out = torch.empty_like(qd)
+            c2kv.c2kv_attend(ctx, cache, layer, qd, kd, vd, prefill, out)
+        oracle = [orc.compose(chunks, ids, offs, wl.rope_theta, wl.dtype) for ids, offs in reqs]
+        st = np.asarray(steps)
+        for extra in range(extra_steps + 1):
+            cur = st + extra
+            pick = lambda x: np.stack([x[:, b, cur[b]] for b in range(B)], axis=1)  # [L, B, H, d]
+            qd, kd, vd = (H.to_dev(pick(x)[lsel], wl) for x in (q, ks, vs))
+            out = torch.full_like(qd, float("nan"))
+            lse = torch.full(qd.shape[:-1], float("nan"), device="cuda")
+            c2kv.c2kv_decode(ctx, cache, layer, qd, kd, vd, cur, out, lse)
+            c2kv.c2kv_sync(ctx)
+            got = out.double().cpu().numpy()
+            got_lse = lse.double().cpu().numpy()
+            for b in range(B):
+                k_c, v_c, _, l_req = oracle[b]
+                t = int(cur[b])
+                o, l_ = orc.decode_step(k_c[lsel], v_c[lsel], l_req, ks[lsel, b, :t], vs[lsel, b, :t],
+                                        q[lsel, b, t], ks[lsel, b, t], vs[lsel, b, t], t,
+                                        wl.rope_theta, wl.dtype)
+                H.check_attention(got[:, b], o, wl, f"decode O req {b} step {t}")
+                assert np.allclose(got_lse[:, b], l_, atol=1e-3, rtol=1e-4), f"lse req {b} step {t}"
+        # the decode token's position was recorded with its row
+        info, gk, gv, gpos = H.cache_arrays(cache, wl)
+        for b in range(B):
+            base, s = info["row_base"][b], info["n_slots"][b]
+            last = int(st[b]) + extra_steps
+            assert gpos[base + s + last] == oracle[b][3] + last
+        c2kv.c2kv_cache_release(ctx, cache)
+    finally:
+        c2kv.c2kv_destroy(ctx)
+
+
+def test_decode_after_suffix_attention():
+    # the suffix of 16 tokens written by attend, then the 17th token decoded
+    _decode_case(_small(L8B_1, layers=2), steps=[16], prefill=16)
+
+
+def test_decode_sequence_from_step0():
+    # straight after compose: steps 0, 1, 2, 3 one call at a time
+    _decode_case(_small(L8B_1, layers=2), steps=[0], extra_steps=3)
+
+
+def test_decode_batched_ragged_steps():
+    wl = _small(synth.workload("batched"), batch=3, chunks_per_request=4, pool_chunks=32)
+    _decode_case(wl, steps=[5, 0, 11], prefill=12)
+
+
+def test_decode_single_layer_of_many():
+    _decode_case(_small(L8B_1, layers=3), steps=[7], prefill=8, layer=1)
+
+
+def test_decode_f32_tiny():
+    _decode_case(TINY, steps=[4], prefill=5)
+
+
+def test_decode_long_context_splits():
+    # 32 chunks x 1024 tokens at k=4: 8192 slots, so the key range is split over many CTAs
+    # and merged
+    wl = _small(L8B_1, chunk_tokens=1024, ratio_k=4, chunks_per_request=32, pool_chunks=32)
+    _decode_case(wl, steps=[3], prefill=3)
+
+
+def test_decode_gqa8_and_mha():
+    _decode_case(_small(synth.workload("long70b"), batch=1, chunks_per_request=4,
+                        pool_chunks=4), steps=[2], prefill=2)
+    _decode_case(_small(L8B_1, n_q_heads=8, n_kv_heads=8), steps=[1], prefill=1)
+
+
+def test_decode_rejects_bad_steps_and_layouts():
+    c2kv = H.lib()
+    wl = _small(L8B_1)
+    ctx = H.make_ctx(wl, pool_slots=1024)
+    try:
+        chunks = H.oracle_chunks_meanpool(wl, [0])
+        dev = H.load_stored(ctx, wl, chunks)
+        cache = c2kv.c2kv_compose(ctx, [0, 1], [dev[0]], [0], suffix_capacity=4)
+        q = torch.zeros((1, 1, wl.n_q_heads, wl.head_dim), dtype=torch.bfloat16, device="cuda")
+        kv = torch.zeros((1, 1, wl.n_kv_heads, wl.head_dim), dtype=torch.bfloat16, device="cuda")
+        for bad in ([4], [-1]):                      # outside [0, suffix_capacity)
+            with pytest.raises(c2kv.C2KVError) as ei:
+                c2kv.c2kv_decode(ctx, cache, -1, q, kv, kv, bad, torch.empty_like(q))
+            assert ei.value.status == c2kv.ERR_ARG
+        with pytest.raises(c2kv.C2KVError) as ei:
+            c2kv.c2kv_decode(ctx, cache, 5, q, kv, kv, [0], torch.empty_like(q))
+        assert ei.value.status == c2kv.ERR_ARG
+    finally:
+        c2kv.c2kv_destroy(ctx)
+    wl3 = _small(L8B_1, n_q_heads=6, n_kv_heads=2)   # G = 3
+    ctx = H.make_ctx(wl3, pool_slots=1024)
+    try:
+        chunks = H.oracle_chunks_meanpool(wl3, [0])
+        dev = H.load_stored(ctx, wl3, chunks)
+        cache = c2kv.c2kv_compose(ctx, [0, 1], [dev[0]], [0], suffix_capacity=4)
+        q = torch.zeros((1, 1, 6, wl3.head_dim), dtype=torch.bfloat16, device="cuda")
+        kv = torch.zeros((1, 1, 2, wl3.head_dim), dtype=torch.bfloat16, device="cuda")
+        with pytest.raises(c2kv.C2KVError) as ei:
+            c2kv.c2kv_decode(ctx, cache, -1, q, kv, kv, [0], torch.empty_like(q))
+        assert ei.value.status == c2kv.ERR_UNSUPPORTED
+    finally:
+        c2kv.c2kv_destroy(ctx)

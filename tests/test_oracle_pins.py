@@ -383,6 +383,51 @@ def test_attend_slot_permutation_invariance():
     assert np.allclose(a, b, atol=1e-13) and np.allclose(la, lb, atol=1e-13)
 
 
+def _decode_case(s_len, step, hq=4, hkv=2, d=8, l_req=70):
+    k_c = RNG.standard_normal((2, s_len, hkv, d))
+    v_c = RNG.standard_normal((2, s_len, hkv, d))
+    q = RNG.standard_normal((2, step + 1, hq, d))
+    k_s = RNG.standard_normal((2, step + 1, hkv, d))
+    v_s = RNG.standard_normal((2, step + 1, hkv, d))
+    return k_c, v_c, q, k_s, v_s, l_req
+
+
+@pytest.mark.parametrize("s_len,step", [(20, 0), (20, 4), (0, 3), (33, 9)])
+def test_decode_step_equals_last_row_of_attend(s_len, step):
+    # one query over every key vs the masked matrix form: row `step` of a suffix of
+    # step + 1 tokens sees exactly the keys the decode step sees
+    k_c, v_c, q, k_s, v_s, l_req = _decode_case(s_len, step)
+    out, lse = orc.decode_step(k_c, v_c, l_req, k_s[:, :step], v_s[:, :step], q[:, step],
+                               k_s[:, step], v_s[:, step], step, 1e4, "f64")
+    full, lse_full = orc.attend(k_c, v_c, l_req, q, k_s, v_s, 1e4, "f64")
+    assert np.allclose(out, full[:, step], atol=1e-13)
+    assert np.allclose(lse, lse_full[:, :, step], atol=1e-13)
+
+
+def test_decode_step_closed_forms():
+    d = 8
+    empty = np.zeros((1, 0, 1, d))
+    # a single key: the output is its value and the lse is the scaled score
+    q = RNG.standard_normal((1, 2, d))
+    k = RNG.standard_normal((1, 1, d))
+    v = RNG.standard_normal((1, 1, d))
+    out, lse = orc.decode_step(empty, empty, 5, empty, empty, q, k, v, 0, 1e4, "f64")
+    assert np.allclose(out[0, 0], v[0, 0], atol=1e-15) and np.allclose(out[0, 1], v[0, 0], atol=1e-15)
+    qr = rope_complex(q[0][None], [5], 1e4)[0]                 # [Hq, d]
+    kr = rope_complex(k[0][None], [5], 1e4)[0, 0]              # [d]
+    assert abs(lse[0, 0] - qr[0] @ kr / math.sqrt(d)) < 1e-12
+    assert abs(lse[0, 1] - qr[1] @ kr / math.sqrt(d)) < 1e-12
+    # all keys zero (a rotated zero stays zero): every score is 0, the weights are uniform
+    # over the 6 composed slots and the new token, and lse = log 7
+    vals = RNG.standard_normal((1, 6, 1, d))
+    v_new = RNG.standard_normal((1, 1, d))
+    out, lse = orc.decode_step(np.zeros((1, 6, 1, d)), vals, 9, empty, empty, q[:, :1],
+                               np.zeros((1, 1, d)), v_new, 0, 1e4, "f64")
+    mean = (vals[0, :, 0].sum(axis=0) + v_new[0, 0]) / 7.0
+    assert np.allclose(out[0, 0], mean, atol=1e-14)
+    assert abs(lse[0, 0] - math.log(7.0)) < 1e-13
+
+
 def test_lse_combine_equals_unsplit():
     s_len, sq, d, hq, hkv = 50, 7, 8, 4, 2
     keys = RNG.standard_normal((s_len + sq, hkv, d))
