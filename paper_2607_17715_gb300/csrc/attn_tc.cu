@@ -45,6 +45,7 @@
 #include <cstring>
 
 #include "internal.cuh"
+#include "ptx.cuh"
 
 namespace c2kv {
 namespace {
@@ -67,7 +68,6 @@ constexpr int kRegsHigh = 184;
 static_assert(128 * kRegsLow + 256 * kRegsHigh <= kThreads * kLaunchRegs, "register split");
 constexpr uint32_t kTmemCols = 512;     // S_A, S_B, O_A, O_B; P_x over the first half of S_x
 constexpr uint32_t kColS = 0, kColO = 256;
-constexpr long long kWaitCycles = 2000000000LL;   // about 1 s
 
 // barrier slots
 constexpr int B_Q = 0;                   // both Q tiles landed
@@ -100,71 +100,7 @@ struct TcParams {                // CUtensorMap members carry their own alignmen
     ReqParam req[kMaxReq];
 };
 
-// ------------------------------------------------------------------ PTX wrappers
-
-__device__ __forceinline__ uint32_t smem_u32(const void* p) {
-    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
-}
-
-__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
-}
-
-__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
-                 : "memory");
-}
-
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
-
-__device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(bar), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-
-// Bounded wait for the phase with the given parity to complete.  The first wait of a CTA
-// that gives up raises the CTA's abort flag (shared memory), and every later wait returns
-// as soon as it sees it, so a CTA spends at most one time limit in waits.
-__device__ __forceinline__ void mbar_wait(uint32_t bar, uint32_t parity, int32_t* err,
-                                          volatile uint32_t* abort) {
-    if (mbar_try(bar, parity)) return;
-    const long long t0 = clock64();
-    while (!mbar_try(bar, parity)) {
-        if (*abort) return;
-        if (clock64() - t0 > kWaitCycles) {
-            atomicOr(err, 2);
-            *abort = 1u;
-            return;
-        }
-    }
-}
-
-__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap* tm, int c0, int c1,
-                                            int c2, uint32_t bar) {
-    asm volatile(
-        "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-        " [%0], [%1, {%2, %3, %4}], [%5];" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(c2), "r"(bar)
-        : "memory");
-}
-
-__device__ __forceinline__ void tma_load_4d(uint32_t dst, const CUtensorMap* tm, int c0, int c1,
-                                            int c2, int c3, uint32_t bar) {
-    asm volatile(
-        "cp.async.bulk.tensor.4d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
-        " [%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(dst),
-        "l"(reinterpret_cast<uint64_t>(tm)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(bar)
-        : "memory");
-}
+// ------------------------------------------------------------------ tcgen05 wrappers
 
 __device__ __forceinline__ void tc_fence_before() {
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -749,7 +685,17 @@ __global__ void __launch_bounds__(256) attn_combine_kernel(const __grid_constant
 
 // ------------------------------------------------------------------ host side
 
-PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+bool encode(CUtensorMap* tm, const void* base, int rank, const cuuint64_t* dims,
+            const cuuint64_t* strides_bytes, const cuuint32_t* box) {
+    return encode_tensor_map(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, rank, base, dims, strides_bytes,
+                             box, CU_TENSOR_MAP_SWIZZLE_128B);
+}
+
+}  // namespace
+
+bool encode_tensor_map(CUtensorMap* tm, CUtensorMapDataType type, int rank, const void* base,
+                       const cuuint64_t* dims, const cuuint64_t* strides_bytes, const cuuint32_t* box,
+                       CUtensorMapSwizzle swizzle) {
     static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
     if (!fn) {
         void* p = nullptr;
@@ -759,22 +705,13 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
             q == cudaDriverEntryPointSuccess)
             fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
     }
-    return fn;
-}
-
-bool encode(CUtensorMap* tm, const void* base, int rank, const cuuint64_t* dims,
-            const cuuint64_t* strides_bytes, const cuuint32_t* box) {
-    auto fn = encode_fn();
     if (!fn) return false;
     cuuint32_t estr[5] = {1, 1, 1, 1, 1};
-    const CUresult r = fn(tm, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, (cuuint32_t)rank,
-                          const_cast<void*>(base), dims, strides_bytes, box, estr,
-                          CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+    const CUresult r = fn(tm, type, (cuuint32_t)rank, const_cast<void*>(base), dims, strides_bytes, box,
+                          estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle,
                           CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     return r == CUDA_SUCCESS;
 }
-
-}  // namespace
 
 int64_t attn_tc_units(int hq, int hkv, int sq, int lq, int batch) {
     const int tq = BM / (hq / hkv);
@@ -798,11 +735,16 @@ bool attn_tc_supported(int dtype, int d, int hq, int hkv) {
     return g == 1 || g == 2 || g == 4 || g == 8 || g == 16;
 }
 
-cudaError_t launch_attn_tc(const AttnParams& a, cudaStream_t s) {
+cudaError_t launch_attn_tc(const AttnParams& a, cudaStream_t s, Hook before) {
     (void)cudaGetLastError();   // report this launch's error only, not a stale one
-    cudaError_t e = cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)kSmemBytes);
-    if (e != cudaSuccess) return e;
+    cudaError_t e = cudaSuccess;
+    static bool smem_set = false;           // once per process (one device per context)
+    if (!smem_set) {
+        e = cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)kSmemBytes);
+        if (e != cudaSuccess) return e;
+        smem_set = true;
+    }
     {   // the register split must not ask for more than the launch holds
         static int launch_regs = -1;
         if (launch_regs < 0) {
@@ -857,6 +799,7 @@ cudaError_t launch_attn_tc(const AttnParams& a, cudaStream_t s) {
     if (gx > 0x7fffffffLL) return cudaErrorInvalidValue;
     const dim3 grid((unsigned)gx, a.hkv, a.lq * a.batch);
     if (grid.z > 65535u || grid.y > 65535u) return cudaErrorInvalidValue;
+    before();
     attn_tc_kernel<<<grid, kThreads, kSmemBytes, s>>>(p);
     return cudaGetLastError();
 }

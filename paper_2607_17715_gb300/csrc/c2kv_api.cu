@@ -186,8 +186,16 @@ struct ProfScope {
     c2kv_ctx* c;
     int kind;
     cudaEvent_t a = nullptr;
-    ProfScope(c2kv_ctx* ctx, int k) : c(ctx), kind(k) {
-        if (c->prof && (a = prof_event(c)) != nullptr) cudaEventRecord(a, c->stream);
+    // deferred: the start event is recorded by start(), which a launcher calls through its
+    // Hook once its host-side preparation is done
+    ProfScope(c2kv_ctx* ctx, int k, bool deferred = false) : c(ctx), kind(k) {
+        if (!deferred) start();
+    }
+    void start() {
+        if (!a && c->prof && (a = prof_event(c)) != nullptr) cudaEventRecord(a, c->stream);
+    }
+    c2kv::Hook hook() {
+        return c2kv::Hook{[](void* self) { static_cast<ProfScope*>(self)->start(); }, this};
     }
     ~ProfScope() {
         if (!a) return;
@@ -683,8 +691,8 @@ c2kv_status c2kv_attend(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
             a.part_o = part;
             a.part_lse = part ? part + (size_t)n_split * part_rows * c->cfg.head_dim : nullptr;
             for (int32_t i = 0; i < nb; ++i) a.req[i] = s.req[i];
-            ProfScope prof_attn(c, C2KV_PROF_ATTN);
-            e = use_tc ? c2kv::launch_attn_tc(a, c->stream)
+            ProfScope prof_attn(c, C2KV_PROF_ATTN, use_tc);
+            e = use_tc ? c2kv::launch_attn_tc(a, c->stream, prof_attn.hook())
                        : c2kv::launch_attn_simt(a, c->cfg.dtype, c->cfg.head_dim, c->stream);
             last = a;
         }
@@ -724,11 +732,29 @@ c2kv_status c2kv_decode(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
         const int32_t lq = layer < 0 ? c->cfg.layers : 1;
         const int32_t layer0 = layer < 0 ? 0 : layer;
         const int32_t hq = c->cfg.n_q_heads, hkv = c->cfg.n_kv_heads, d = c->cfg.head_dim;
-        // key-range splits: about two CTAs per SM over all (layer, request, KV head), and at
-        // least 256 keys per split
+        // Key-range splits per (layer, request, KV head), from a model of the schedule: the
+        // CTAs run in waves of (resident CTAs per SM) x SMs; a CTA spends a start latency
+        // (about 2 us: its first tiles in flight) plus its keys' K/V bytes at its share of
+        // HBM, at most what one CTA's four consumer warps keep up with (about 25 GB/s,
+        // measured); a split adds the merge (about 3 us).  Splits keep at least 128 keys.
         const int64_t units = (int64_t)hkv * lq * std::min<int32_t>(B, c2kv::kMaxReq);
-        int32_t n_split = (int32_t)std::min<int64_t>(64, std::max<int64_t>(1, (2 * c->sms + units - 1) / units));
-        n_split = std::max<int32_t>(1, std::min<int32_t>(n_split, (n_keys_max + 255) / 256));
+        const int32_t grp = hq / hkv;
+        const int64_t slots = (int64_t)(grp >= 8 ? 1 : 2) * c->sms;
+        const double bytes_per_key = 2.0 * d * (double)c->eb;
+        int32_t n_split = 1;
+        double best = 0.0;
+        for (int32_t n = 1; n <= 64; ++n) {
+            const int32_t kps = (n_keys_max + n - 1) / n;
+            if (n > 1 && kps < 128) break;
+            const int64_t ctas = units * n;
+            const int64_t waves = (ctas + slots - 1) / slots;
+            const double bw = std::min(6.0e12 / (double)std::min(ctas, slots), 25.0e9);
+            const double t = (double)waves * (2e-6 + kps * bytes_per_key / bw) + (n > 1 ? 3e-6 : 0.0);
+            if (n == 1 || t < best) {
+                best = t;
+                n_split = n;
+            }
+        }
         const int32_t keys_per_split = (n_keys_max + n_split - 1) / n_split;
 
         const size_t q_bytes = (size_t)lq * B * hq * d * c->eb;
@@ -781,6 +807,7 @@ c2kv_status c2kv_decode(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
             p.lse = lse;
             p.part_o = part;
             p.part_lse = part ? part + (size_t)n_split * rows_all * d : nullptr;
+            p.err = c->d_err;
             p.rows = cache->rows;
             p.layer0 = layer0;
             p.lq = lq;
@@ -794,8 +821,8 @@ c2kv_status c2kv_decode(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
             p.keys_per_split = keys_per_split;
             p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)d));
             for (int32_t i = 0; i < nb; ++i) p.req[i] = s.req[i];
-            ProfScope prof_decode(c, C2KV_PROF_DECODE);
-            e = c2kv::launch_decode(p, c->cfg.dtype, c->stream);
+            ProfScope prof_decode(c, C2KV_PROF_DECODE, true);
+            e = c2kv::launch_decode(p, c->cfg.dtype, c->stream, prof_decode.hook());
         }
         pool_free(c, part);
         pool_free(c, q_rot);

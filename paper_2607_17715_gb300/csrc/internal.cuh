@@ -5,6 +5,8 @@
 // and no device-side metadata buffer.
 #pragma once
 
+#include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
 #include <stdint.h>
@@ -133,6 +135,17 @@ cudaError_t launch_compress(const CompressParams& p, int dtype, int d, cudaStrea
 cudaError_t launch_suffix_prep(const SuffixParams& p, int dtype, int d, cudaStream_t s);
 cudaError_t launch_attn_simt(const AttnParams& p, int dtype, int d, cudaStream_t s);
 
+// Called by a launcher after its host-side preparation (tensor maps, function attributes)
+// and right before it enqueues its kernels, so that a trace event recorded there brackets
+// device work only.
+struct Hook {
+    void (*fn)(void*) = nullptr;
+    void* arg = nullptr;
+    void operator()() const {
+        if (fn) fn(arg);
+    }
+};
+
 // Decode attention (decode.cu): one new token per request (suffix index ReqParam::t0,
 // already rotated into q_rot and appended to the cache) over keys 0 .. S_r + t0.
 struct DecodeParams {
@@ -143,6 +156,7 @@ struct DecodeParams {
     float* lse;              // [Lq][Btot][Hq] or null
     float* part_o;           // n_split > 1: [n_split][Lq][Btot][Hq][d] fp32, normalised
     float* part_lse;         // n_split > 1: [n_split][Lq][Btot][Hq] fp32, log2 domain
+    int32_t* err;            // device error word: bit 1 = a bounded wait expired
     int64_t rows;
     int32_t layer0;
     int32_t lq;
@@ -158,11 +172,17 @@ struct DecodeParams {
     ReqParam req[kMaxReq];
 };
 bool decode_supported(int dtype, int d, int hq, int hkv);
-cudaError_t launch_decode(const DecodeParams& p, int dtype, cudaStream_t s);
+cudaError_t launch_decode(const DecodeParams& p, int dtype, cudaStream_t s, Hook before = {});
+
+// Tiled tensor map for TMA (cuTensorMapEncodeTiled through the runtime's driver entry point);
+// false when the driver refuses it (attn_tc.cu).
+bool encode_tensor_map(CUtensorMap* tm, CUtensorMapDataType type, int rank, const void* base,
+                       const cuuint64_t* dims, const cuuint64_t* strides_bytes, const cuuint32_t* box,
+                       CUtensorMapSwizzle swizzle);
 
 // Tensor-core attention (attn_tc.cu).
 bool attn_tc_supported(int dtype, int d, int hq, int hkv);
-cudaError_t launch_attn_tc(const AttnParams& p, cudaStream_t s);
+cudaError_t launch_attn_tc(const AttnParams& p, cudaStream_t s, Hook before = {});
 // Merge n_split partial (O, lse) over disjoint key ranges into out (bf16) and lse (attn_tc.cu).
 cudaError_t launch_attn_combine(const AttnParams& p, cudaStream_t s);
 // Work units (CTAs per split) the tensor-core kernel launches for these parameters.
