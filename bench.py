@@ -268,6 +268,46 @@ class Arm:
         for cid in loaded.values():
             c2kv.c2kv_free_chunk(self.ctx, cid)
 
+    def decode_run(self, steps, warmup, events):
+        """Decode after the suffix: compose once, write the suffix with attend, then decode
+        `warmup` untimed and `steps` timed tokens per request (one c2kv_decode call per token,
+        all layers), L2 flushed before each.  Returns (ms per timed step, mean decode kernel
+        ms from the library trace, keys read per timed step summed over requests)."""
+        c2kv, wl, torch = self.c2kv, self.wl, self.torch
+        ids = [self.dev_ids[c] for ids_, _ in self.reqs for c in ids_]
+        cache = c2kv.c2kv_compose(self.ctx, self.req_ptr, ids, self.positions,
+                                  wl.n_suffix + warmup + steps)
+        c2kv.c2kv_attend(self.ctx, cache, -1, *self.q_dev, wl.n_suffix, self.out)
+        B = len(self.reqs)
+        gen = torch.Generator(device="cuda").manual_seed(1)
+        qd = torch.randn((wl.layers, B, wl.n_q_heads, wl.head_dim), device="cuda", generator=gen).to(self.tdt)
+        kd = torch.randn((wl.layers, B, wl.n_kv_heads, wl.head_dim), device="cuda", generator=gen).to(self.tdt)
+        vd = torch.randn_like(kd)
+        od = torch.empty_like(qd)
+        n_slots = c2kv.c2kv_cache_info(cache)["n_slots"]
+        for i in range(warmup):
+            self.flush_l2()
+            c2kv.c2kv_decode(self.ctx, cache, -1, qd, kd, vd, [wl.n_suffix + i] * B, od)
+        c2kv.c2kv_sync(self.ctx)
+        c2kv.c2kv_profile_read(self.ctx)
+        c2kv.c2kv_profile_enable(self.ctx, True)
+        keys = 0
+        total = 0.0
+        for i in range(steps):
+            st = wl.n_suffix + warmup + i
+            self.flush_l2()                                    # untimed
+            events[i][0].record(self.stream)
+            c2kv.c2kv_decode(self.ctx, cache, -1, qd, kd, vd, [st] * B, od)
+            events[i][1].record(self.stream)
+            keys += int(sum(int(n) + st + 1 for n in n_slots))
+        torch.cuda.synchronize()
+        c2kv.c2kv_sync(self.ctx)
+        kern = c2kv.c2kv_profile_read(self.ctx)
+        c2kv.c2kv_profile_enable(self.ctx, False)
+        total = sum(ev[0].elapsed_time(ev[1]) for ev in events[:steps])
+        c2kv.c2kv_cache_release(self.ctx, cache)
+        return total / steps, kern["decode"][0], keys / steps
+
     def e2e_bytes(self, zero_copy=False):
         """Host->device and device->host bytes of one e2e step.  Staged: each distinct
         chunk is copied once.  Zero-copy: compose reads a chunk's slots once per occurrence."""
@@ -282,6 +322,25 @@ class Arm:
 
     def close(self):
         self.c2kv.c2kv_destroy(self.ctx)
+
+
+def decode_line(wl, world, dec_ms, dec_kernel_ms, dec_keys, hbm, src):
+    eb = 4 if wl.dtype == "f32" else 2
+    bytes_step = dec_keys * wl.layers * wl.n_kv_heads * wl.head_dim * eb * 2
+    kernel_gbs = bytes_step / (dec_kernel_ms / 1e3) / 1e9 if dec_kernel_ms else None
+    return {
+        "metric": "decode tokens/s", "unit": "tokens/s",
+        "value": round(wl.batch * world / (dec_ms / 1e3), 1),
+        "ms_per_step": round(dec_ms, 5),
+        "what": "one new token per request after the suffix, all layers per call (c2kv_decode); "
+                "RoPE/append and the split-KV attention; L2 flushed before each step (untimed)",
+        "keys_per_request": round(dec_keys / wl.batch, 1),
+        "kernel_ms": round(dec_kernel_ms, 5),
+        "roofline": {"bound": "hbm", "kernel": "decode_kernel (+ merge)",
+                     "achieved": round(kernel_gbs, 1) if kernel_gbs else None, "peak": hbm,
+                     "unit": "GB/s", "frac": round(kernel_gbs / hbm, 4) if kernel_gbs else None,
+                     "peak_source": f"{src} hbm_gbs", "bytes_per_launch": int(bytes_step)},
+    }
 
 
 def dist_setup():
@@ -358,8 +417,13 @@ def run_ours(args):
     h2d, d2h = arm.e2e_bytes(zero_copy=True)
     h2d_staged, _ = arm.e2e_bytes(zero_copy=False)
 
+    # decode after the suffix (one new token per request per step, all layers)
+    dec_events = [[E(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
+    dec_ms, dec_kernel_ms, dec_keys = arm.decode_run(args.steps, args.warmup, dec_events)
+
     from paper_2607_17715_gb300.shard import max_over_ranks
-    total_ms, e2e_ms, staged_ms = max_over_ranks([total_ms, e2e_ms, staged_ms], device="cuda")
+    total_ms, e2e_ms, staged_ms, dec_ms = max_over_ranks([total_ms, e2e_ms, staged_ms, dec_ms],
+                                                         device="cuda")
     arm.close()
     if rank != 0:
         if world > 1:
@@ -405,6 +469,9 @@ def run_ours(args):
                            "ms_per_step": round(staged_ms / args.steps, 4),
                            "h2d_bytes_per_step": h2d_staged,
                            "path": "chunks copied host->pool (MODE_STORED), then compose"}},
+        # decode after the suffix: tokens generated per second over the whole job, and the
+        # decode kernel against HBM (algorithmic bytes: K and V of every key it attends to)
+        "decode": decode_line(wl, world, dec_ms, dec_kernel_ms, dec_keys, hbm, src),
         # every kernel the library launched in the timed steps (its own trace counts)
         "gpu_launches": sum(v[1] for v in kern.values()),
         "clocks": clk,
