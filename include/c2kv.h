@@ -109,7 +109,7 @@ typedef struct c2kv_cache_desc {
 } c2kv_cache_desc;
 
 /* ABI version of this header (bumped on any incompatible change). */
-#define C2KV_ABI_VERSION 2
+#define C2KV_ABI_VERSION 3
 int32_t c2kv_abi_version(void);
 
 /*
@@ -278,6 +278,32 @@ c2kv_status c2kv_decode(c2kv_ctx* ctx, c2kv_cache* cache, int32_t layer, const v
                         const void* k_new, const void* v_new, const int32_t* steps, void* out,
                         float* lse);
 
+/*
+ * c2kv_extract_attention -- one attention layer of the C2 Extractor's forward over a chunk
+ * under the Structured Information Flow mask (Sec. 3.3).  The sequence is the n document
+ * tokens followed by the m = ceil(n/k) C2 tokens, [x_0 .. x_{n-1}; c_0 .. c_{m-1}]
+ * (Sec. 3.3.1); document token t sits at position t, C2 token c_j at the position of the
+ * last token of its block B(j) = [jk, min((j+1)k, n)).  Q and K are RoPE'd there and
+ *     O[t, h] = softmax_u( Q_t,h . K_u,h/G / sqrt(d) + M[t, u] ) V_u,h/G
+ * with the mask (Sec. 3.3.2):
+ *   - a document token sees document tokens 0..t only (so its output is the frozen model's);
+ *   - c_j sees the document tokens of B(j) and of the sink block, and c_0 .. c_j.
+ * The sink block, B(0) in the paper's 1-based numbering, is read as the first block
+ * [0, min(k, n)).  The trained C2 embeddings and QKV projections that produce q, k, v for
+ * the C2 tokens are the caller's; this is the attention operator they feed.
+ *
+ *   n_layers : layers in the tensors (each processed independently).
+ *   q        : device [n_layers][n + m][Hq][d] pre-RoPE queries.
+ *   k, v     : device [n_layers][n + m][Hkv][d] pre-RoPE keys, values.
+ *   n_tokens : n >= 1;  ratio_k : k >= 1.
+ *   out      : device [n_layers][n + m][Hq][d] (context dtype).
+ *   lse      : device [n_layers][Hq][n + m] fp32 natural-log normaliser, or NULL.
+ * Errors: ERR_ARG, ERR_UNSUPPORTED (d not 64 or 128), ERR_NOMEM, ERR_CUDA.
+ */
+c2kv_status c2kv_extract_attention(c2kv_ctx* ctx, int32_t n_layers, const void* q, const void* k,
+                                   const void* v, int32_t n_tokens, int32_t ratio_k, void* out,
+                                   float* lse);
+
 /* c2kv_cache_release -- free a composed cache (stream-ordered). */
 c2kv_status c2kv_cache_release(c2kv_ctx* ctx, c2kv_cache* cache);
 
@@ -303,7 +329,8 @@ const char* c2kv_last_error(const c2kv_ctx* ctx);
 #define C2KV_PROF_ATTN     3   /* the attention kernel alone */
 #define C2KV_PROF_COMBINE  4   /* merge of key-range splits (when attention was split) */
 #define C2KV_PROF_DECODE   5   /* decode attention (with the merge of its splits) */
-#define C2KV_PROF_KINDS    6
+#define C2KV_PROF_EXTRACT  6   /* SIF-masked extraction attention (RoPE + attention) */
+#define C2KV_PROF_KINDS    7
 c2kv_status c2kv_profile_enable(c2kv_ctx* ctx, int32_t on);
 /* mean_ms[C2KV_PROF_KINDS] receives mean milliseconds (0 where none), launches[] the
  * counts; either may be NULL. */

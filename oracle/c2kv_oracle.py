@@ -20,6 +20,8 @@ What it computes (C2KV, arXiv 2607.17715):
 * Inference (Sec. 2.2, Eq. for F).  The suffix (query) tokens run standard attention over
   [composed cache; suffix], causal inside the suffix, every composed slot visible.  A
   decode step is the same operator for one new token over everything cached before it.
+* Extraction attention (Sec. 3.3).  The extractor's attention layer over a chunk's
+  document tokens and its C2 tokens under the Structured Information Flow mask.
 
 RoPE is the rotate-half form used by the Llama / Qwen models the paper evaluates
 (Sec. 4.1): channel i pairs with i + d/2 and turns by pos * theta^(-2i/d).
@@ -307,6 +309,65 @@ def decode_step(k_c, v_c, l_req: int, k_prev, v_prev, q_new, k_new, v_new, step:
             tot = e.sum()
             out[layer, h] = (e / tot) @ vals[:, g, :]
             lse[layer, h] = mx + math.log(tot)
+    return out, lse
+
+
+def sif_positions(n: int, k: int) -> np.ndarray:
+    """Extraction positions of [x_0 .. x_{n-1}; c_0 .. c_{m-1}] (Sec. 3.3.1): document token
+    t at t, C2 token c_j at the last token of its block B(j) = [jk, min((j+1)k, n))."""
+    return np.concatenate([np.arange(n), slot_local_positions(n, k)]).astype(np.int64)
+
+
+def sif_mask(n: int, k: int) -> np.ndarray:
+    """Visibility of key u to query t under Structured Information Flow (Sec. 3.3.2), as a
+    boolean [n+m, n+m] matrix over [x_0 .. x_{n-1}; c_0 .. c_{m-1}]:
+      * original-token invariance: a document token sees document tokens 0..t, never a C2
+        token;
+      * block-local extraction: c_j sees the document tokens of B(j) and of the sink block;
+      * causal accumulation: c_j sees c_0 .. c_j.
+    The sink block (B(0) in the paper's 1-based numbering, left undefined by its block
+    formula) is read as the first block [0, min(k, n))."""
+    m = n_slots(n, k)
+    vis = np.zeros((n + m, n + m), dtype=bool)
+    for t in range(n):
+        vis[t, :t + 1] = True
+    for j in range(m):
+        lo, hi = block(j, n, k)
+        vis[n + j, lo:hi] = True
+        s_lo, s_hi = block(0, n, k)
+        vis[n + j, s_lo:s_hi] = True
+        vis[n + j, n:n + j + 1] = True
+    return vis
+
+
+def sif_attention(q, k_in, v, n: int, k: int, theta: float, dtype: str):
+    """One attention layer of the extractor over a chunk under the SIF mask.
+
+    q: [L, n+m, Hq, d], k_in, v: [L, n+m, Hkv, d] (pre-RoPE), ordered
+    [document tokens; C2 tokens].  Q and K are turned to ``sif_positions`` and stored
+    (rounded) like any cached activation; scale 1/sqrt(d); exact softmax under ``sif_mask``.
+    Returns O [L, n+m, Hq, d] (float64) and lse [L, Hq, n+m] (natural log)."""
+    n_layers, n_all, hq, d = q.shape
+    hkv = k_in.shape[2]
+    grp = hq // hkv
+    pos = sif_positions(n, k)
+    assert len(pos) == n_all
+    vis = sif_mask(n, k)
+    out = np.zeros((n_layers, n_all, hq, d))
+    lse = np.zeros((n_layers, hq, n_all))
+    for layer in range(n_layers):
+        q_r = store(rope(q[layer], pos, theta), dtype)
+        k_r = store(rope(k_in[layer], pos, theta), dtype)
+        vals = np.asarray(v[layer], np.float64)
+        for h in range(hq):
+            g = h // grp
+            s = q_r[:, h, :] @ k_r[:, g, :].T / math.sqrt(d)            # [n+m, n+m]
+            s = np.where(vis, s, -np.inf)
+            mx = s.max(axis=1, keepdims=True)
+            e = np.exp(s - mx)
+            tot = e.sum(axis=1, keepdims=True)
+            out[layer, :, h, :] = (e / tot) @ vals[:, g, :]
+            lse[layer, h, :] = (mx + np.log(tot))[:, 0]
     return out, lse
 
 

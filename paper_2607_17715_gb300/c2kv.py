@@ -30,8 +30,9 @@ DTYPE_BF16, DTYPE_F32 = 0, 1
 MODE_MEANPOOL, MODE_PROVIDED, MODE_STORED, MODE_HOST = 0, 1, 2, 3
 ATTN_AUTO, ATTN_SIMT, ATTN_TC = 0, 1, 2
 PROF_COMPOSE, PROF_COMPRESS, PROF_SUFFIX, PROF_ATTN, PROF_COMBINE, PROF_DECODE = 0, 1, 2, 3, 4, 5
-PROF_KINDS = 6
-PROF_NAMES = ("compose", "compress", "suffix", "attention", "combine", "decode")
+PROF_EXTRACT = 6
+PROF_KINDS = 7
+PROF_NAMES = ("compose", "compress", "suffix", "attention", "combine", "decode", "extract")
 
 STATUS_NAMES = {
     0: "OK", -1: "ERR_ARG", -2: "ERR_DTYPE", -3: "ERR_NOMEM", -4: "ERR_POOL_FULL",
@@ -79,6 +80,7 @@ _SIGS = {
     "c2kv_attend": (_I32, [_VP, _VP, _I32, _VP, _VP, _VP, _I32, _VP, _VP]),
     "c2kv_attend_noalloc": (_I32, [_VP, _VP, _I32, _VP, _VP, _VP, _I32, _VP, _VP]),
     "c2kv_decode": (_I32, [_VP, _VP, _I32, _VP, _VP, _VP, _P32, _VP, _VP]),
+    "c2kv_extract_attention": (_I32, [_VP, _I32, _VP, _VP, _VP, _I32, _I32, _VP, _VP]),
     "c2kv_cache_release": (_I32, [_VP, _VP]),
     "c2kv_sync": (_I32, [_VP]),
     "c2kv_last_error": (ctypes.c_char_p, [_VP]),
@@ -215,6 +217,12 @@ def c2kv_decode(ctx, cache, layer, q, k_new, v_new, steps, out, lse=None):
     st, st_p = _i32(steps)
     _check(_lib.c2kv_decode(ctx, cache, layer, _ptr(q), _ptr(k_new), _ptr(v_new), st_p,
                             _ptr(out), _ptr(lse)), ctx)
+
+
+def c2kv_extract_attention(ctx, n_layers, q, k, v, n_tokens, ratio_k, out, lse=None):
+    """SIF-masked extraction attention over [document tokens; C2 tokens] of one chunk."""
+    _check(_lib.c2kv_extract_attention(ctx, n_layers, _ptr(q), _ptr(k), _ptr(v), n_tokens,
+                                       ratio_k, _ptr(out), _ptr(lse)), ctx)
 
 
 def c2kv_cache_release(ctx, cache):

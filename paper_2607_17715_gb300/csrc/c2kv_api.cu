@@ -833,6 +833,61 @@ c2kv_status c2kv_decode(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
     }
 }
 
+c2kv_status c2kv_extract_attention(c2kv_ctx* c, int32_t n_layers, const void* q, const void* k,
+                                   const void* v, int32_t n_tokens, int32_t ratio_k, void* out,
+                                   float* lse) {
+    if (!c) return C2KV_ERR_ARG;
+    try {
+        c->err.clear();
+        if (!q || !k || !v || !out) return fail(c, C2KV_ERR_ARG, "extract: null pointer");
+        if (n_layers < 1 || n_tokens < 1 || ratio_k < 1)
+            return fail(c, C2KV_ERR_ARG, "extract: need n_layers, n_tokens, ratio_k >= 1");
+        const int32_t d = c->cfg.head_dim;
+        if (d != 64 && d != 128) return fail(c, C2KV_ERR_UNSUPPORTED, "extract: head_dim %d", d);
+        const int64_t m = ((int64_t)n_tokens + ratio_k - 1) / ratio_k;
+        if ((int64_t)n_tokens + m > 0x7fffffffLL / 128) return fail(c, C2KV_ERR_ARG, "extract: chunk too long");
+        const int32_t n_all = (int32_t)(n_tokens + m);
+        const int32_t hq = c->cfg.n_q_heads, hkv = c->cfg.n_kv_heads;
+        const size_t qb = (size_t)n_layers * n_all * hq * d * c->eb;
+        const size_t kb = (size_t)n_layers * n_all * hkv * d * c->eb;
+        void* q_rot = nullptr;
+        void* k_rot = nullptr;
+        cudaError_t e = pool_alloc(c, &q_rot, qb);
+        if (e != cudaSuccess) return cuda_fail(c, e, "extract: scratch allocation");
+        e = pool_alloc(c, &k_rot, kb);
+        if (e != cudaSuccess) {
+            pool_free(c, q_rot);
+            return cuda_fail(c, e, "extract: scratch allocation");
+        }
+        c2kv::ExtractParams p{};
+        p.q = q;
+        p.k = k;
+        p.v = v;
+        p.q_rot = q_rot;
+        p.k_rot = k_rot;
+        p.out = out;
+        p.lse = lse;
+        p.lq = n_layers;
+        p.n = n_tokens;
+        p.ratio = ratio_k;
+        p.n_all = n_all;
+        p.hq = hq;
+        p.hkv = hkv;
+        p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)d));
+        p.rope = c->turns;
+        {
+            ProfScope prof(c, C2KV_PROF_EXTRACT);
+            e = c2kv::launch_extract(p, c->cfg.dtype, d, c->stream);
+        }
+        pool_free(c, k_rot);
+        pool_free(c, q_rot);
+        if (e != cudaSuccess) return cuda_fail(c, e, "extract");
+        return C2KV_OK;
+    } catch (const std::bad_alloc&) {
+        return fail(c, C2KV_ERR_NOMEM, "extract: host allocation failed");
+    }
+}
+
 c2kv_status c2kv_cache_release(c2kv_ctx* c, c2kv_cache* cache) {
     if (!c) return C2KV_ERR_ARG;
     c->err.clear();

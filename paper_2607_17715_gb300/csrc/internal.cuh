@@ -174,6 +174,27 @@ struct DecodeParams {
 bool decode_supported(int dtype, int d, int hq, int hkv);
 cudaError_t launch_decode(const DecodeParams& p, int dtype, cudaStream_t s, Hook before = {});
 
+// SIF-masked extraction attention (extract.cu): one attention layer of the extractor over
+// a chunk's n document tokens and m = ceil(n/k) C2 tokens, [x_0..x_{n-1}; c_0..c_{m-1}].
+struct ExtractParams {
+    const void* q;           // [Lq][n_all][Hq][d] pre-RoPE
+    const void* k;           // [Lq][n_all][Hkv][d] pre-RoPE
+    const void* v;           // [Lq][n_all][Hkv][d]
+    void* q_rot;             // scratch, shaped like q
+    void* k_rot;             // scratch, shaped like k
+    void* out;               // [Lq][n_all][Hq][d]
+    float* lse;              // [Lq][Hq][n_all] or null
+    int32_t lq;
+    int32_t n;               // document tokens
+    int32_t ratio;           // k, the block size
+    int32_t n_all;           // n + ceil(n / k)
+    int32_t hq;
+    int32_t hkv;
+    float scale_log2;
+    RopeTurns rope;
+};
+cudaError_t launch_extract(const ExtractParams& p, int dtype, int d, cudaStream_t s);
+
 // Tiled tensor map for TMA (cuTensorMapEncodeTiled through the runtime's driver entry point);
 // false when the driver refuses it (attn_tc.cu).
 bool encode_tensor_map(CUtensorMap* tm, CUtensorMapDataType type, int rank, const void* base,

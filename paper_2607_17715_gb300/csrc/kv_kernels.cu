@@ -9,6 +9,7 @@
 // once to a float in [-1/2, 1/2) turns and handed to sincospif.  The error is about
 // 1e-7 rad at any position, where forming p * inv_freq in fp32 would lose p * 2^-24 rad.
 #include "internal.cuh"
+#include "rope.cuh"
 #include "vec16.cuh"
 
 namespace c2kv {
@@ -16,23 +17,6 @@ namespace {
 
 
 // (cos, sin) of pos * theta^(-2i/d) from the 0.64 fixed-point turn of frequency i.
-__device__ __forceinline__ float2 turn_cs(uint64_t turn, int64_t pos) {
-    const uint64_t frac = (uint64_t)pos * turn;                 // turns mod 1, exact
-    const float x = (float)(long long)frac * 0x1p-63f;          // 2 * turns in [-1, 1)
-    float s, c;
-    sincospif(x, &s, &c);
-    return make_float2(c, s);
-}
-
-template <int E>
-__device__ __forceinline__ void rotate(const float* x, const float* y, const float2* cs,
-                                       float* ox, float* oy) {
-#pragma unroll
-    for (int e = 0; e < E; ++e) {
-        ox[e] = x[e] * cs[e].x - y[e] * cs[e].y;
-        oy[e] = x[e] * cs[e].y + y[e] * cs[e].x;
-    }
-}
 
 // ---------------------------------------------------------------------------------------
 // compose.  grid = (tiles, layers); a tile is kComposeTile consecutive slots of one chunk

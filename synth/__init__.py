@@ -107,7 +107,7 @@ def _rng(seed: int, *stream: int) -> np.random.Generator:
     return np.random.Generator(np.random.PCG64(np.random.SeedSequence([seed, *stream])))
 
 
-_TAG_OUTLIER, _TAG_CHUNK, _TAG_SLOTS, _TAG_REQ, _TAG_SUFFIX = 1, 2, 3, 4, 5
+_TAG_OUTLIER, _TAG_CHUNK, _TAG_SLOTS, _TAG_REQ, _TAG_SUFFIX, _TAG_EXTRACT = 1, 2, 3, 4, 5, 6
 
 
 def _outlier_mask(wl: Workload, seed: int) -> np.ndarray:
@@ -196,3 +196,20 @@ def suffix(wl: Workload, seed: int = 0, layers: int | None = None):
     return _finish(q, wl.dtype), _finish(k, wl.dtype), _finish(v, wl.dtype)
 
 
+
+
+def extraction_inputs(wl: Workload, chunk_id: int, n_tokens: int, ratio_k: int, seed: int = 0):
+    """Inputs of one extraction attention layer over a chunk: q [layers, n+m, Hq, d] and
+    k, v [layers, n+m, Hkv, d] (pre-RoPE), ordered [document tokens; m = ceil(n/k) C2
+    tokens].  The document K/V are the chunk's own tokens (``chunk_tokens``); the queries
+    and the C2 tokens' K/V, which trained projections would make, are standard normal."""
+    n = n_tokens
+    m = -(-n // ratio_k)
+    kd, vd = chunk_tokens(wl, chunk_id, seed, n_tokens=n)
+    rng = _rng(seed, _TAG_EXTRACT, chunk_id)
+    q = rng.standard_normal((wl.layers, n + m, wl.n_q_heads, wl.head_dim), dtype=np.float32)
+    kc = rng.standard_normal((wl.layers, m, wl.n_kv_heads, wl.head_dim), dtype=np.float32)
+    vc = rng.standard_normal((wl.layers, m, wl.n_kv_heads, wl.head_dim), dtype=np.float32)
+    k = np.concatenate([kd, _finish(kc, wl.dtype)], axis=1)
+    v = np.concatenate([vd, _finish(vc, wl.dtype)], axis=1)
+    return _finish(q, wl.dtype), k, v

@@ -1,0 +1,71 @@
+"""SIF-masked extraction attention (c2kv_extract_attention) against the oracle."""
+import numpy as np
+import pytest
+import torch
+
+import synth
+from oracle import c2kv_oracle as orc
+from tests import _gpu_helpers as H
+
+pytestmark = pytest.mark.gpu
+
+L8B = synth.workload("llama8b")
+TINY = synth.workload("tiny_f32")
+
+
+def _extract_case(wl, n, k, layers=1, chunk_id=0):
+    c2kv = H.lib()
+    wl = synth.scaled(wl, layers=layers)
+    q, kk, v = synth.extraction_inputs(wl, chunk_id, n, k)
+    ctx = H.make_ctx(wl, pool_slots=64)
+    try:
+        qd, kd, vd = (H.to_dev(x, wl) for x in (q, kk, v))
+        out = torch.full_like(qd, float("nan"))
+        lse = torch.full((layers, wl.n_q_heads, q.shape[1]), float("nan"), device="cuda")
+        c2kv.c2kv_extract_attention(ctx, layers, qd, kd, vd, n, k, out, lse)
+        c2kv.c2kv_sync(ctx)
+        ref, ref_lse = orc.sif_attention(q, kk, v, n, k, wl.rope_theta, wl.dtype)
+        got = out.double().cpu().numpy()
+        H.check_attention(got[:, :n], ref[:, :n], wl, "document rows")
+        H.check_attention(got[:, n:], ref[:, n:], wl, "C2 rows")
+        assert np.allclose(lse.double().cpu().numpy(), ref_lse, atol=1e-3, rtol=1e-4), "lse"
+    finally:
+        c2kv.c2kv_destroy(ctx)
+
+
+@pytest.mark.parametrize("n,k", [(512, 4), (77, 4), (203, 10), (64, 1), (40, 64)])
+def test_extract_bf16(n, k):
+    _extract_case(L8B, n, k)
+
+
+def test_extract_two_layers_gqa8():
+    _extract_case(synth.workload("long70b"), 300, 16, layers=2)
+
+
+def test_extract_f32_tiny():
+    _extract_case(TINY, 128, 4, layers=1)
+
+
+def test_extract_document_rows_equal_suffix_free_prefill():
+    # original-token invariance on the device: perturbing every C2 token leaves the document
+    # rows bit-identical
+    c2kv = H.lib()
+    wl = synth.scaled(L8B, layers=1)
+    n, k = 96, 8
+    q, kk, v = synth.extraction_inputs(wl, 3, n, k)
+    ctx = H.make_ctx(wl, pool_slots=64)
+    try:
+        outs = []
+        for bump in (0.0, 1.0):
+            k2, v2, q2 = kk.copy(), v.copy(), q.copy()
+            k2[:, n:] += bump
+            v2[:, n:] -= bump
+            q2[:, n:] *= 1.0 + bump
+            qd, kd, vd = (H.to_dev(x, wl) for x in (q2, k2, v2))
+            out = torch.empty_like(qd)
+            c2kv.c2kv_extract_attention(ctx, 1, qd, kd, vd, n, k, out)
+            c2kv.c2kv_sync(ctx)
+            outs.append(out[:, :n].clone())
+        assert torch.equal(outs[0], outs[1])
+    finally:
+        c2kv.c2kv_destroy(ctx)

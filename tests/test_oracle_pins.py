@@ -428,6 +428,84 @@ def test_decode_step_closed_forms():
     assert abs(lse[0, 0] - math.log(7.0)) < 1e-13
 
 
+def _sif_case(n, k, hq=4, hkv=2, d=8, layers=1):
+    m = orc.n_slots(n, k)
+    q = RNG.standard_normal((layers, n + m, hq, d))
+    kk = RNG.standard_normal((layers, n + m, hkv, d))
+    v = RNG.standard_normal((layers, n + m, hkv, d))
+    return q, kk, v
+
+
+@pytest.mark.parametrize("n,k", [(13, 4), (8, 8), (9, 1), (20, 30)])
+def test_sif_document_rows_are_causal_attention(n, k):
+    # original-token invariance: the document rows equal plain causal attention over the
+    # document alone (torch SDPA in fp64, its own causal mask and GQA mapping)
+    q, kk, v = _sif_case(n, k)
+    out, _ = orc.sif_attention(q, kk, v, n, k, 1e4, "f64")
+    q_r = rope_complex(q[0, :n], np.arange(n), 1e4)
+    k_r = rope_complex(kk[0, :n], np.arange(n), 1e4)
+    qt = torch.from_numpy(q_r).permute(1, 0, 2)[None]
+    kt = torch.from_numpy(k_r).permute(1, 0, 2)[None]
+    vt = torch.from_numpy(v[0, :n]).permute(1, 0, 2)[None]
+    ref = torch.nn.functional.scaled_dot_product_attention(qt, kt, vt, is_causal=True,
+                                                           enable_gqa=True)
+    assert np.allclose(out[0, :n], ref[0].permute(1, 0, 2).numpy(), atol=1e-12)
+
+
+def test_sif_c2_rows_bruteforce():
+    # C2 token c_j by explicit loops over the key set the paper states: B(j), the first
+    # block (sink), and c_0 .. c_j; positions are block ends
+    n, k, d = 10, 4, 4
+    q, kk, v = _sif_case(n, k, hq=2, hkv=1, d=d)
+    out, lse = orc.sif_attention(q, kk, v, n, k, 1e4, "f64")
+    m = orc.n_slots(n, k)
+    for j in range(m):
+        end = min((j + 1) * k, n)
+        keys = sorted(set(range(j * k, end)) | set(range(0, min(k, n))) |
+                      {n + i for i in range(j + 1)})
+        def posof(t):
+            return t if t < n else min((t - n + 1) * k, n) - 1
+        qr = rope_complex(q[0, n + j][None], [posof(n + j)], 1e4)[0]
+        for h in range(2):
+            sc = []
+            for u in keys:
+                kr = rope_complex(kk[0, u][None], [posof(u)], 1e4)[0, 0]
+                sc.append(sum(qr[h, c] * kr[c] for c in range(d)) / 2.0)
+            mx = max(sc)
+            w = [math.exp(x - mx) for x in sc]
+            o = sum(wi * v[0, u, 0] for wi, u in zip(w, keys)) / sum(w)
+            assert np.allclose(out[0, n + j, h], o, atol=1e-13)
+            assert abs(lse[0, h, n + j] - (mx + math.log(sum(w)))) < 1e-13
+
+
+def test_sif_mask_structure():
+    n, k = 11, 3
+    vis = orc.sif_mask(n, k)
+    m = orc.n_slots(n, k)
+    assert not vis[:n, n:].any()                           # documents never see C2 tokens
+    assert (vis[:n, :n] == np.tril(np.ones((n, n), bool))).all()
+    assert (vis[n:, n:] == np.tril(np.ones((m, m), bool))).all()
+    # c_j sees exactly its block and the first block among the document tokens
+    for j in range(m):
+        want = np.zeros(n, bool)
+        want[j * k:min((j + 1) * k, n)] = True
+        want[:k] = True
+        assert (vis[n + j, :n] == want).all()
+
+
+def test_pins_catch_a_leaky_sif_mask(monkeypatch):
+    # a mask that lets document tokens see the C2 tokens breaks original-token invariance
+    good = orc.sif_mask
+
+    def leaky(n, k):
+        vis = good(n, k)
+        vis[:n, n:] = True
+        return vis
+    monkeypatch.setattr(orc, "sif_mask", leaky)
+    with pytest.raises(AssertionError):
+        test_sif_document_rows_are_causal_attention(13, 4)
+
+
 def test_lse_combine_equals_unsplit():
     s_len, sq, d, hq, hkv = 50, 7, 8, 4, 2
     keys = RNG.standard_normal((s_len + sq, hkv, d))
