@@ -28,9 +28,35 @@ def _extract_case(wl, n, k, layers=1, chunk_id=0):
         got = out.double().cpu().numpy()
         H.check_attention(got[:, :n], ref[:, :n], wl, "document rows")
         H.check_attention(got[:, n:], ref[:, n:], wl, "C2 rows")
-        assert np.allclose(lse.double().cpu().numpy(), ref_lse, atol=1e-3, rtol=1e-4), "lse"
+        gl = lse.double().cpu().numpy()
+        bad = np.abs(gl - ref_lse) > 1e-3 + 1e-4 * np.abs(ref_lse) + _lse_rounding_bound(q, kk, n, k, wl)
+        if bad.any():
+            i = np.unravel_index(np.argmax(np.abs(gl - ref_lse)), gl.shape)
+            raise AssertionError(f"lse: {bad.sum()} off; worst at {i}: got {gl[i]} want {ref_lse[i]}")
     finally:
         c2kv.c2kv_destroy(ctx)
+
+
+def _lse_rounding_bound(q, kk, n, k, wl):
+    """Per (layer, head, row) bound on the lse difference that storage rounding alone can
+    make: both sides store the rotated Q and K in the context dtype but round from different
+    rotations (fp32 here, fp64 in the oracle), so an element may differ by one unit in the
+    last place (relative 2^-8 for bf16, 2^-24 for fp32).  A score then moves by at most
+    rel * sum_c |q_c k_c| / sqrt(d), and lse = log sum exp is 1-Lipschitz in the scores, so
+    its change is at most the largest such move over the row's visible keys."""
+    rel = 2.0 ** -8 if wl.dtype == "bf16" else 2.0 ** -24
+    pos = orc.sif_positions(n, k)
+    vis = orc.sif_mask(n, k)
+    layers, n_all, hq, d = q.shape
+    grp = hq // kk.shape[2]
+    out = np.zeros((layers, hq, n_all))
+    for layer in range(layers):
+        q_r = np.abs(orc.store(orc.rope(q[layer], pos, wl.rope_theta), wl.dtype))
+        k_r = np.abs(orc.store(orc.rope(kk[layer], pos, wl.rope_theta), wl.dtype))
+        for h in range(hq):
+            mag = q_r[:, h, :] @ k_r[:, h // grp, :].T / np.sqrt(d)
+            out[layer, h] = rel * np.where(vis, mag, 0.0).max(axis=1)
+    return out
 
 
 @pytest.mark.parametrize("n,k", [(512, 4), (77, 4), (203, 10), (64, 1), (40, 64)])
