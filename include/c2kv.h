@@ -22,6 +22,8 @@
  *     the context dtype (bf16 or fp32) unless stated.
  *   - The caller owns every buffer it passes in; the library owns the chunk pool and the
  *     composed caches it returns.
+ *   - Tensor pointers passed in must be 16-byte aligned (fp32 lse arrays: 4-byte), since
+ *     the kernels move rows in 16-byte vectors and by TMA; others give ERR_ARG.
  *   - A context is used from one host thread at a time.
  */
 #ifndef C2KV_H

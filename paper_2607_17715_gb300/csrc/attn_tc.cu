@@ -85,14 +85,14 @@ constexpr size_t kSmemBytes = 1024 /*align*/ + (size_t)TILE * kSmemTiles + 8 * N
 static_assert(kSmemBytes <= 232448, "shared memory budget of one sm_100 CTA");
 
 struct TcParams {                // CUtensorMap members carry their own alignment
-    CUtensorMap tm_q;        // q_rot   [Lq*Btot][Sq][Hq][128]  box {64, G, TQ, 1}
+    CUtensorMap tm_q;        // q_rot   [Lq*Btot][Sq'][Hq][128] box {64, G, TQ, 1}; Sq' = sq_pitch
     CUtensorMap tm_k;        // cache K [L*rows][Hkv][128]      box {64, 1, 128}
     CUtensorMap tm_v;        // cache V, same
     void* out;
     float* lse;
     int32_t* err;
     int64_t rows;
-    int32_t layer0, lq, batch, batch_total, b0, sq, hq, hkv, group, tq;
+    int32_t layer0, lq, batch, batch_total, b0, sq, sq_pitch, hq, hkv, group, tq;
     float scale_log2;
     int32_t n_split;
     float* part_o;
@@ -342,8 +342,8 @@ __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, u
     const int g = r - (r / G) * G;
     const bool any = l_run > 0.f;                 // some key of this split was visible
     const float inv = any ? 1.0f / l_run : 0.f;
-    const int64_t row_id = (((int64_t)l * P.batch_total + b) * P.sq + t) * P.hq + hk * G + g;
-    const int64_t lse_id = (((int64_t)l * P.batch_total + b) * P.hq + hk * G + g) * P.sq + t;
+    const int64_t row_id = (((int64_t)l * P.batch_total + b) * P.sq_pitch + t) * P.hq + hk * G + g;
+    const int64_t lse_id = (((int64_t)l * P.batch_total + b) * P.hq + hk * G + g) * P.sq_pitch + t;
     if (P.n_split == 1) {
         __nv_bfloat16* orow = static_cast<__nv_bfloat16*>(P.out) + row_id * HD;
 #pragma unroll
@@ -396,16 +396,15 @@ __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, u
 // The MMA issuer (one thread).  The tensor core's queue holds about one MMA, so anything
 // the issuing thread does between two MMAs idles it, and a branch there costs about as much
 // as an MMA.  So the descriptors are precomputed, the issue blocks are straight-line code,
-// and the main loop is unrolled over six key tiles (the least common multiple of the two
-// ring depths): every ring stage and every barrier parity in it is a compile-time constant.
-// Each block waits for its own inputs only: waiting for a later block's P inside an S block
-// would hold that S back until the other tile's softmax finished, putting the two softmaxes
-// in series.
+// the kernel is specialised on whether the CTA has a tile B, and the ring stages and
+// barrier parities advance by selects rather than branches.  Each block waits for its own
+// inputs only: waiting for a later block's P inside an S block would hold that S back until
+// the other tile's softmax finished, putting the two softmaxes in series.
 template <bool kHasB>
 __device__ __forceinline__ void mma_issuer(const TcParams& P, uint32_t tmem, uint32_t sQ, uint32_t sK,
                                            uint32_t sV, uint32_t sBar, int n_kv,
                                            volatile uint32_t* abort) {
-    static_assert(KSTAGES == 3 && VSTAGES == 2, "the unrolled schedule assumes 3 K and 2 V stages");
+    static_assert(KSTAGES == 3 && VSTAGES == 2, "the issue schedule assumes 3 K and 2 V stages");
     auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
     constexpr uint32_t idS = idesc_bf16(BM, BN, false);
     constexpr uint32_t idO = idesc_bf16(BM, HD, true);
@@ -521,8 +520,10 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_const
     const int bl = blockIdx.z - l * P.batch;
     const int b = P.b0 + bl;
     const int s_r = P.req[bl].n_slots;
-    const int pr = blockIdx.x / P.n_split;          // pair of Q tiles
-    const int sp = blockIdx.x - pr * P.n_split;     // key-range split
+    // pair of Q tiles, the last first: under a causal mask the later pairs see more keys, so
+    // the longest CTAs start in the first wave
+    const int pr = (int)(gridDim.x / P.n_split) - 1 - (int)(blockIdx.x / P.n_split);
+    const int sp = (int)(blockIdx.x % P.n_split);   // key-range split
     const int t0a = 2 * pr * P.tq;
     const int t0b = t0a + P.tq;
     const bool has_b = t0b < P.sq;
@@ -721,7 +722,7 @@ int64_t attn_tc_units(int hq, int hkv, int sq, int lq, int batch) {
 
 cudaError_t launch_attn_combine(const AttnParams& a, cudaStream_t s) {
     (void)cudaGetLastError();
-    if (a.n_split > kMaxSplit) return cudaErrorInvalidValue;
+    if (a.n_split > kMaxSplit || (a.sq_pitch != 0 && a.sq_pitch != a.sq)) return cudaErrorInvalidValue;
     const int64_t rows = (int64_t)a.lq * a.batch_total * a.sq * a.hq;
     const int64_t blocks = (rows + 7) / 8;
     if (blocks > 0x7fffffffLL) return cudaErrorInvalidValue;
@@ -755,15 +756,17 @@ cudaError_t launch_attn_tc(const AttnParams& a, cudaStream_t s, Hook before) {
         }
         if (launch_regs * kThreads < 128 * kRegsLow + 256 * kRegsHigh) return cudaErrorInvalidConfiguration;
     }
+    const int pitch = a.sq_pitch > 0 ? a.sq_pitch : a.sq;
+    if (pitch < a.sq || (pitch != a.sq && a.n_split > 1)) return cudaErrorInvalidValue;
     TcParams p;
     std::memset(&p, 0, sizeof(p));
     const int G = a.hq / a.hkv;
     const int tq = BM / G;
-    {   // Q: q_rot [Lq*Btot][Sq][Hq][128] -> dims (d, Hq, Sq, Lq*Btot)
+    {   // Q: q_rot [Lq*Btot][Sq'][Hq][128] -> dims (d, Hq, Sq, Lq*Btot); tokens past Sq read 0
         const cuuint64_t dims[4] = {HD, (cuuint64_t)a.hq, (cuuint64_t)a.sq,
                                     (cuuint64_t)a.lq * a.batch_total};
         const cuuint64_t str[3] = {(cuuint64_t)HD * 2, (cuuint64_t)a.hq * HD * 2,
-                                   (cuuint64_t)a.sq * a.hq * HD * 2};
+                                   (cuuint64_t)pitch * a.hq * HD * 2};
         const cuuint32_t box[4] = {64, (cuuint32_t)G, (cuuint32_t)tq, 1};
         if (!encode(&p.tm_q, a.q_rot, 4, dims, str, box)) return cudaErrorInvalidValue;
     }
@@ -785,6 +788,7 @@ cudaError_t launch_attn_tc(const AttnParams& a, cudaStream_t s, Hook before) {
     p.batch_total = a.batch_total;
     p.b0 = a.b0;
     p.sq = a.sq;
+    p.sq_pitch = pitch;
     p.hq = a.hq;
     p.hkv = a.hkv;
     p.group = G;

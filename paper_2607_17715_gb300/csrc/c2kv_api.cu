@@ -156,6 +156,10 @@ bool is_device_ptr(const void* p) {
     return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
 }
 
+// Every tensor pointer is at least this aligned (16 bytes; lse arrays 4): the kernels move
+// rows in 16-byte vectors and by TMA, and a misaligned vector access would fault.
+bool aligned(const void* p, uintptr_t a = 16) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
+
 bool own_cache(const c2kv_ctx* c, const c2kv_cache* cache) {
     return cache && std::find(c->caches.begin(), c->caches.end(), cache) != c->caches.end();
 }
@@ -314,6 +318,7 @@ c2kv_status c2kv_compress_chunk(c2kv_ctx* c, const void* k, const void* v, int32
     try {
         c->err.clear();
         if (!k || !v || !chunk_id_out) return fail(c, C2KV_ERR_ARG, "compress: null pointer");
+        if (!aligned(k) || !aligned(v)) return fail(c, C2KV_ERR_ARG, "compress: k, v must be 16-byte aligned");
         if (n_tokens < 1 || ratio_k < 1) return fail(c, C2KV_ERR_ARG, "compress: need n >= 1, k >= 1");
         if (mode != C2KV_MODE_MEANPOOL && mode != C2KV_MODE_PROVIDED && mode != C2KV_MODE_STORED &&
             mode != C2KV_MODE_HOST)
@@ -593,6 +598,8 @@ c2kv_status c2kv_attend(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
         c->err.clear();
         if (!own_cache(c, cache)) return fail(c, C2KV_ERR_STATE, "attend: cache not owned by this context");
         if (!q || !k_suf || !v_suf || !out) return fail(c, C2KV_ERR_ARG, "attend: null pointer");
+        if (!aligned(q) || !aligned(k_suf) || !aligned(v_suf) || !aligned(out) || !aligned(lse, 4))
+            return fail(c, C2KV_ERR_ARG, "attend: misaligned tensor pointer");
         if (layer < -1 || layer >= c->cfg.layers) return fail(c, C2KV_ERR_ARG, "attend: bad layer %d", layer);
         if (n_suffix < 1 || n_suffix > cache->suffix_capacity)
             return fail(c, C2KV_ERR_ARG, "attend: n_suffix %d outside [1, %d]", n_suffix,
@@ -717,6 +724,8 @@ c2kv_status c2kv_decode(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
         c->err.clear();
         if (!own_cache(c, cache)) return fail(c, C2KV_ERR_STATE, "decode: cache not owned by this context");
         if (!q || !k_new || !v_new || !steps || !out) return fail(c, C2KV_ERR_ARG, "decode: null pointer");
+        if (!aligned(q) || !aligned(k_new) || !aligned(v_new) || !aligned(out) || !aligned(lse, 4))
+            return fail(c, C2KV_ERR_ARG, "decode: misaligned tensor pointer");
         if (layer < -1 || layer >= c->cfg.layers) return fail(c, C2KV_ERR_ARG, "decode: bad layer %d", layer);
         if (!c2kv::decode_supported(c->cfg.dtype, c->cfg.head_dim, c->cfg.n_q_heads, c->cfg.n_kv_heads))
             return fail(c, C2KV_ERR_UNSUPPORTED, "decode: head layout not supported");
@@ -840,6 +849,8 @@ c2kv_status c2kv_extract_attention(c2kv_ctx* c, int32_t n_layers, const void* q,
     try {
         c->err.clear();
         if (!q || !k || !v || !out) return fail(c, C2KV_ERR_ARG, "extract: null pointer");
+        if (!aligned(q) || !aligned(k) || !aligned(v) || !aligned(out) || !aligned(lse, 4))
+            return fail(c, C2KV_ERR_ARG, "extract: misaligned tensor pointer");
         if (n_layers < 1 || n_tokens < 1 || ratio_k < 1)
             return fail(c, C2KV_ERR_ARG, "extract: need n_layers, n_tokens, ratio_k >= 1");
         const int32_t d = c->cfg.head_dim;
@@ -850,16 +861,23 @@ c2kv_status c2kv_extract_attention(c2kv_ctx* c, int32_t n_layers, const void* q,
         const int32_t hq = c->cfg.n_q_heads, hkv = c->cfg.n_kv_heads;
         const size_t qb = (size_t)n_layers * n_all * hq * d * c->eb;
         const size_t kb = (size_t)n_layers * n_all * hkv * d * c->eb;
+        // the tensor-core route merges two partials for the C2 rows through a normaliser
+        const bool need_lse = lse == nullptr && c2kv::extract_uses_tc(c->cfg.dtype, d, hq, hkv);
+        const size_t lb = need_lse ? (size_t)n_layers * hq * n_all * sizeof(float) : 0;
         void* q_rot = nullptr;
         void* k_rot = nullptr;
+        void* lse_scratch = nullptr;
         cudaError_t e = pool_alloc(c, &q_rot, qb);
-        if (e != cudaSuccess) return cuda_fail(c, e, "extract: scratch allocation");
-        e = pool_alloc(c, &k_rot, kb);
+        if (e == cudaSuccess) e = pool_alloc(c, &k_rot, kb);
+        if (e == cudaSuccess && need_lse) e = pool_alloc(c, &lse_scratch, lb);
         if (e != cudaSuccess) {
-            pool_free(c, q_rot);
+            if (k_rot) pool_free(c, k_rot);
+            if (q_rot) pool_free(c, q_rot);
             return cuda_fail(c, e, "extract: scratch allocation");
         }
         c2kv::ExtractParams p{};
+        p.lse_scratch = static_cast<float*>(lse_scratch);
+        p.err = c->d_err;
         p.q = q;
         p.k = k;
         p.v = v;
@@ -879,6 +897,7 @@ c2kv_status c2kv_extract_attention(c2kv_ctx* c, int32_t n_layers, const void* q,
             ProfScope prof(c, C2KV_PROF_EXTRACT);
             e = c2kv::launch_extract(p, c->cfg.dtype, d, c->stream);
         }
+        if (lse_scratch) pool_free(c, lse_scratch);
         pool_free(c, k_rot);
         pool_free(c, q_rot);
         if (e != cudaSuccess) return cuda_fail(c, e, "extract");

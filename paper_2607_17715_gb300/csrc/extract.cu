@@ -12,10 +12,25 @@
 // it is read as the first block, [0, min(k, n)).
 //
 // extract_rope_kernel turns Q and K to those positions (fp32 arithmetic, stored in the
-// context dtype like every cached activation); extract_attn_kernel runs the masked attention
-// on the CUDA cores with fp32 accumulation: one CTA holds RB packed query rows (row
-// r = t * G + g: token t, query head h_kv * G + g) of one (layer, KV head), stages K/V tiles
-// of KT keys in shared memory, and skips the tiles none of its rows can see.
+// context dtype like every cached activation).  The masked attention then takes one of two
+// routes.
+//
+// Tensor cores (bf16, d = 128, the group sizes attn_tc_kernel takes).  The mask splits into
+// pieces the suffix-attention kernel already computes:
+//   1. document rows: plain causal attention over document keys 0..t, i.e. a "suffix" of n
+//      tokens over an empty prefix;
+//   2. C2 rows, causal part: c_j over c_0 .. c_j, a "suffix" of m tokens over an empty
+//      prefix whose keys start at row n;
+//   3. C2 rows, block-local part: c_j over the at most 2k document keys of the sink block
+//      and B(j), on the CUDA cores (extract_local_kernel), merged with part 2 exactly by
+//      log-sum-exp: the two key sets are disjoint and together are what c_j sees.
+// Parts 1 and 2 are launches of attn_tc_kernel with a token pitch of n + m, so they read
+// and write the extraction layout in place.
+//
+// CUDA cores (fp32, d = 64, other group sizes): extract_attn_kernel runs every row with fp32
+// accumulation: one CTA holds RB packed query rows (row r = t * G + g: token t, query head
+// h_kv * G + g) of one (layer, KV head), stages K/V tiles of KT keys in shared memory, and
+// skips the tiles none of its rows can see.
 #include <math_constants.h>
 
 #include "internal.cuh"
@@ -206,6 +221,170 @@ __global__ void __launch_bounds__(XNW * 32) extract_attn_kernel(const __grid_con
     }
 }
 
+// Part 3 of the tensor-core route: one warp per (layer, C2 token c_j, KV head).  Lane i
+// holds channels 4i .. 4i+3 of the G query heads; each visible document key (the sink block,
+// then B(j) when j > 0) is one coalesced 256-byte row of K and of V, its G scores are
+// butterfly-summed across the warp, and every lane keeps the same online softmax.  The
+// partial (O_b, lse_b) is merged with part 2's (O_a, lse_a), read from out and the
+// normaliser array, by the exact rule O = (2^lse_a O_a + 2^lse_b O_b) / (2^lse_a + 2^lse_b).
+template <int G>
+__global__ void __launch_bounds__(128) extract_local_kernel(const __grid_constant__ ExtractParams P) {
+    constexpr int D = 128;
+    const int lane = threadIdx.x & 31;
+    const int m = P.n_all - P.n;
+    const int64_t w = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
+    if (w >= (int64_t)P.lq * m * P.hkv) return;               // warp-uniform
+    const int hk = (int)(w % P.hkv);
+    const int64_t lj = w / P.hkv;
+    const int j = (int)(lj % m);
+    const int l = (int)(lj / m);
+    const int n = P.n, k = P.ratio;
+    const int tq = n + j;
+    const float sc = P.scale_log2;
+
+    using bf = __nv_bfloat16;
+    auto ld4 = [](const bf* p, float* f) {
+        const uint2 u = *reinterpret_cast<const uint2*>(p);
+        const __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162*>(&u.x);
+        const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162*>(&u.y);
+        f[0] = __low2float(a);
+        f[1] = __high2float(a);
+        f[2] = __low2float(b);
+        f[3] = __high2float(b);
+    };
+    float q[G][4];
+    const bf* qr = static_cast<const bf*>(P.q_rot) + (((int64_t)l * P.n_all + tq) * P.hq + hk * G) * D + lane * 4;
+#pragma unroll
+    for (int g = 0; g < G; ++g) ld4(qr + g * D, q[g]);
+
+    const int sink_end = min(k, n);
+    const int lo = j * k, hi = min((j + 1) * k, n);
+    const int nk = j == 0 ? hi - lo : sink_end + (hi - lo);    // B(0) is the sink block
+    const int64_t kv_stride = (int64_t)P.hkv * D;
+    const bf* kb = static_cast<const bf*>(P.k_rot) + ((int64_t)l * P.n_all * P.hkv + hk) * D + lane * 4;
+    const bf* vb = static_cast<const bf*>(P.v) + ((int64_t)l * P.n_all * P.hkv + hk) * D + lane * 4;
+    float mr[G], lr[G], acc[G][4];
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+        mr[g] = -CUDART_INF_F;
+        lr[g] = 0.f;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) acc[g][c] = 0.f;
+    }
+    for (int i = 0; i < nk; ++i) {
+        const int u = j == 0 ? lo + i : (i < sink_end ? i : lo + i - sink_end);
+        float kk[4], vv[4];
+        ld4(kb + u * kv_stride, kk);
+        ld4(vb + u * kv_stride, vv);
+        float s[G];
+#pragma unroll
+        for (int g = 0; g < G; ++g)
+            s[g] = fmaf(q[g][0], kk[0], fmaf(q[g][1], kk[1], fmaf(q[g][2], kk[2], q[g][3] * kk[3])));
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1)
+#pragma unroll
+            for (int g = 0; g < G; ++g) s[g] += __shfl_xor_sync(0xffffffffu, s[g], o);
+#pragma unroll
+        for (int g = 0; g < G; ++g) {
+            const float sl = s[g] * sc;
+            const float mn = fmaxf(mr[g], sl);
+            const float a = exp2f(mr[g] - mn);                   // 0 on the first key
+            const float pw = exp2f(sl - mn);
+            lr[g] = lr[g] * a + pw;
+#pragma unroll
+            for (int c = 0; c < 4; ++c) acc[g][c] = fmaf(pw, vv[c], acc[g][c] * a);
+            mr[g] = mn;
+        }
+    }
+
+    float* lse_ab = P.lse != nullptr ? P.lse : P.lse_scratch;
+    bf* out = static_cast<bf*>(P.out);
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+        const int h = hk * G + g;
+        const int64_t lse_id = ((int64_t)l * P.hq + h) * P.n_all + tq;
+        const float la = lse_ab[lse_id] * 1.4426950408889634f;   // part 2, natural log -> log2
+        const float lb = mr[g] + log2f(lr[g]);
+        const float mx = fmaxf(la, lb);
+        const float wa = exp2f(la - mx), wb = exp2f(lb - mx);
+        const float inv = 1.f / (wa + wb);
+        const float fb = wb * inv / lr[g];
+        bf* orow = out + (((int64_t)l * P.n_all + tq) * P.hq + h) * D + lane * 4;
+        float oa[4];
+        ld4(orow, oa);
+        __nv_bfloat162 r0 = __floats2bfloat162_rn(fmaf(wa * inv, oa[0], fb * acc[g][0]),
+                                                  fmaf(wa * inv, oa[1], fb * acc[g][1]));
+        __nv_bfloat162 r1 = __floats2bfloat162_rn(fmaf(wa * inv, oa[2], fb * acc[g][2]),
+                                                  fmaf(wa * inv, oa[3], fb * acc[g][3]));
+        uint2 st;
+        st.x = *reinterpret_cast<uint32_t*>(&r0);
+        st.y = *reinterpret_cast<uint32_t*>(&r1);
+        *reinterpret_cast<uint2*>(orow) = st;
+        __syncwarp();                                            // every lane has read lse_a
+        if (P.lse != nullptr && lane == 0) P.lse[lse_id] = (mx + log2f(wa + wb)) * 0.69314718055994531f;
+    }
+}
+
+template <int G>
+cudaError_t launch_local(const ExtractParams& p, cudaStream_t s) {
+    const int64_t warps = (int64_t)p.lq * (p.n_all - p.n) * p.hkv;
+    const int64_t blocks = (warps + 3) / 4;
+    if (blocks > 0x7fffffffLL) return cudaErrorInvalidValue;
+    extract_local_kernel<G><<<(unsigned)blocks, 128, 0, s>>>(p);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_tc(const ExtractParams& p, cudaStream_t s) {
+    constexpr int D = 128;
+    extract_rope_kernel<__nv_bfloat16, D / 2 / Vec16<__nv_bfloat16>::N>
+        <<<dim3((unsigned)p.n_all, (unsigned)p.lq), 256, 0, s>>>(p);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    const int m = p.n_all - p.n;
+    float* lse_ab = p.lse != nullptr ? p.lse : p.lse_scratch;
+    AttnParams a{};
+    a.cache_k = p.k_rot;
+    a.cache_v = p.v;
+    a.err = p.err;
+    a.rows = p.n_all;
+    a.layer0 = 0;
+    a.lq = p.lq;
+    a.batch = 1;
+    a.batch_total = 1;
+    a.b0 = 0;
+    a.sq_pitch = p.n_all;
+    a.hq = p.hq;
+    a.hkv = p.hkv;
+    a.scale_log2 = p.scale_log2;
+    a.n_split = 1;
+    // 1. document rows over document keys 0..t
+    a.q_rot = p.q_rot;
+    a.out = p.out;
+    a.lse = p.lse;
+    a.sq = p.n;
+    a.req[0] = ReqParam{0, 0, 0, 0};
+    e = launch_attn_tc(a, s);
+    if (e != cudaSuccess) return e;
+    // 2. C2 rows over c_0 .. c_j (keys from row n), always with a normaliser for the merge
+    const int64_t c2_off = (int64_t)p.n * p.hq * D;
+    a.q_rot = static_cast<const __nv_bfloat16*>(p.q_rot) + c2_off;
+    a.out = static_cast<__nv_bfloat16*>(p.out) + c2_off;
+    a.lse = lse_ab + p.n;
+    a.sq = m;
+    a.req[0] = ReqParam{p.n, 0, 0, 0};
+    e = launch_attn_tc(a, s);
+    if (e != cudaSuccess) return e;
+    // 3. C2 rows over the sink block and their own block, merged into 2
+    switch (p.hq / p.hkv) {
+        case 1: return launch_local<1>(p, s);
+        case 2: return launch_local<2>(p, s);
+        case 4: return launch_local<4>(p, s);
+        case 8: return launch_local<8>(p, s);
+        case 16: return launch_local<16>(p, s);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
 template <typename T, int D>
 cudaError_t launch_typed(const ExtractParams& p, cudaStream_t s) {
     constexpr int VPH = D / 2 / Vec16<T>::N;
@@ -220,10 +399,16 @@ cudaError_t launch_typed(const ExtractParams& p, cudaStream_t s) {
 
 }  // namespace
 
+bool extract_uses_tc(int dtype, int d, int hq, int hkv) { return attn_tc_supported(dtype, d, hq, hkv); }
+
 cudaError_t launch_extract(const ExtractParams& p, int dtype, int d, cudaStream_t s) {
     (void)cudaGetLastError();   // report this launch's error only, not a stale one
     if (p.n_all < 1 || p.lq < 1) return cudaSuccess;
     if (p.lq > 65535 || p.hkv > 65535) return cudaErrorInvalidValue;
+    if (extract_uses_tc(dtype, d, p.hq, p.hkv)) {
+        if (p.lse == nullptr && p.lse_scratch == nullptr) return cudaErrorInvalidValue;
+        return launch_tc(p, s);
+    }
     if (dtype == kDtypeF32 && d == 64) return launch_typed<float, 64>(p, s);
     if (dtype == kDtypeF32 && d == 128) return launch_typed<float, 128>(p, s);
     if (dtype == kDtypeBf16 && d == 64) return launch_typed<__nv_bfloat16, 64>(p, s);

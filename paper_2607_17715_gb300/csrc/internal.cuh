@@ -107,11 +107,11 @@ struct SuffixParams {
 };
 
 struct AttnParams {
-    const void* q_rot;       // [Lq][Btot][Sq][Hq][d]
+    const void* q_rot;       // [Lq][Btot][Sq'][Hq][d], Sq' = sq_pitch
     const void* cache_k;     // [L][rows][Hkv][d]
     const void* cache_v;
-    void* out;               // [Lq][Btot][Sq][Hq][d]
-    float* lse;              // [Lq][Btot][Hq][Sq] or null
+    void* out;               // [Lq][Btot][Sq'][Hq][d]
+    float* lse;              // [Lq][Btot][Hq][Sq'] or null
     int32_t* err;            // device error word: bit 1 = a bounded wait expired
     int64_t rows;
     int32_t layer0;
@@ -120,6 +120,9 @@ struct AttnParams {
     int32_t batch_total;
     int32_t b0;
     int32_t sq;
+    int32_t sq_pitch;        // tokens allocated per (layer, request) in q_rot, out and lse:
+                             // rows sq .. sq_pitch-1 are neither read nor written; 0 = sq
+                             // (tensor-core kernel only, and only with n_split == 1)
     int32_t hq;
     int32_t hkv;
     float scale_log2;        // log2(e) / sqrt(d)
@@ -184,6 +187,8 @@ struct ExtractParams {
     void* k_rot;             // scratch, shaped like k
     void* out;               // [Lq][n_all][Hq][d]
     float* lse;              // [Lq][Hq][n_all] or null
+    float* lse_scratch;      // shaped like lse: the C2 rows' partial normaliser when lse is null
+    int32_t* err;            // device error word (bounded waits of the tensor-core kernel)
     int32_t lq;
     int32_t n;               // document tokens
     int32_t ratio;           // k, the block size
@@ -194,6 +199,9 @@ struct ExtractParams {
     RopeTurns rope;
 };
 cudaError_t launch_extract(const ExtractParams& p, int dtype, int d, cudaStream_t s);
+// Whether launch_extract takes the tensor-core route (and so needs lse_scratch when lse is
+// null); otherwise every row runs on the CUDA cores.
+bool extract_uses_tc(int dtype, int d, int hq, int hkv);
 
 // Tiled tensor map for TMA (cuTensorMapEncodeTiled through the runtime's driver entry point);
 // false when the driver refuses it (attn_tc.cu).

@@ -70,6 +70,10 @@ extern "C" c2kv_status c2kv_attend_noalloc(c2kv_ctx* ctx, c2kv_cache* cache, int
         return refuse(ctx, C2KV_ERR_STATE, "attend_noalloc: cache not owned by this context");
     if (!q || !k_suf || !v_suf || !out)
         return refuse(ctx, C2KV_ERR_ARG, "attend_noalloc: null pointer");
+    const auto misaligned = [](const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) != 0; };
+    if (misaligned(q, 16) || misaligned(k_suf, 16) || misaligned(v_suf, 16) || misaligned(out, 16) ||
+        misaligned(lse, 4))
+        return refuse(ctx, C2KV_ERR_ARG, "attend_noalloc: misaligned tensor pointer");
     if (layer < -1 || layer >= v.layers)
         return refuse(ctx, C2KV_ERR_ARG, "attend_noalloc: bad layer");
     if (n_suffix < 1 || n_suffix > v.suffix_capacity)

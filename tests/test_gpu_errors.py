@@ -114,6 +114,33 @@ def test_attend_arg_checks(ctx):
     assert _status(c2kv.c2kv_cache_release, ctx, cache) == c2kv.ERR_STATE
 
 
+def test_misaligned_pointers_refused(ctx):
+    # rows move in 16-byte vectors and by TMA: a misaligned tensor is refused on the host
+    c2kv = H.lib()
+    a = _chunk(ctx)
+    cache = c2kv.c2kv_compose(ctx, [0, 1], [a], None, 4)
+    q = torch.zeros((2, 1, 4, WL.n_q_heads, WL.head_dim), device="cuda", dtype=torch.bfloat16)
+    kv = torch.zeros((2, 1, 4, WL.n_kv_heads, WL.head_dim), device="cuda", dtype=torch.bfloat16)
+    out = torch.empty_like(q)
+    lse = torch.empty((2, 1, WL.n_q_heads, 4), device="cuda")
+    odd = q.data_ptr() + 2
+    assert _status(c2kv.c2kv_attend, ctx, cache, -1, odd, kv, kv, 4, out) == c2kv.ERR_ARG
+    assert _status(c2kv.c2kv_attend, ctx, cache, -1, q, kv, kv, 4, out.data_ptr() + 8) == c2kv.ERR_ARG
+    assert _status(c2kv.c2kv_attend, ctx, cache, -1, q, kv, kv, 4, out, lse.data_ptr() + 2) == c2kv.ERR_ARG
+    assert _status(c2kv.c2kv_attend_noalloc, ctx, cache, -1, odd, kv, kv, 4, out) == c2kv.ERR_ARG
+    steps = np.zeros(1, np.int32)
+    assert _status(c2kv.c2kv_decode, ctx, cache, -1, odd, kv, kv, steps, out) == c2kv.ERR_ARG
+    assert _status(c2kv.c2kv_extract_attention, ctx, 1, odd, kv, kv, 3, 1, out) == c2kv.ERR_ARG
+    kt, vt = synth.chunk_tokens(WL, 0, n_tokens=8)
+    kd, vd = H.to_dev(kt, WL), H.to_dev(vt, WL)
+    assert _status(c2kv.c2kv_compress_chunk, ctx, kd.data_ptr() + 2, vd, 8, 4, 0) == c2kv.ERR_ARG
+    # nothing was changed: the aligned call still runs
+    c2kv.c2kv_attend(ctx, cache, -1, q, kv, kv, 4, out, lse)
+    c2kv.c2kv_sync(ctx)
+    assert torch.isfinite(out.float()).all()
+    c2kv.c2kv_cache_release(ctx, cache)
+
+
 def test_device_bounds_check_reports_and_recovers(ctx):
     c2kv = H.lib()
     a = _chunk(ctx)

@@ -59,9 +59,39 @@ def _lse_rounding_bound(q, kk, n, k, wl):
     return out
 
 
-@pytest.mark.parametrize("n,k", [(512, 4), (77, 4), (203, 10), (64, 1), (40, 64)])
+@pytest.mark.parametrize("n,k", [(512, 4), (77, 4), (203, 10), (64, 1), (40, 64), (1030, 4),
+                                 (1999, 16), (1, 1), (5, 3)])
 def test_extract_bf16(n, k):
     _extract_case(L8B, n, k)
+
+
+@pytest.mark.parametrize("hq,hkv", [(8, 8), (16, 8), (32, 2)])
+def test_extract_bf16_group_sizes(hq, hkv):
+    # G = 1, 2 and 16 query heads per KV head (one to sixteen tokens per 128-row tile)
+    _extract_case(synth.scaled(L8B, n_q_heads=hq, n_kv_heads=hkv), 333, 4)
+
+
+def test_extract_without_lse_matches_with_lse():
+    # without an lse array the C2 rows' partial normaliser goes to library scratch; the
+    # outputs are the same bits either way
+    c2kv = H.lib()
+    wl = synth.scaled(L8B, layers=2)
+    n, k = 700, 4
+    q, kk, v = synth.extraction_inputs(wl, 5, n, k)
+    ctx = H.make_ctx(wl, pool_slots=64)
+    try:
+        qd, kd, vd = (H.to_dev(x, wl) for x in (q, kk, v))
+        a = torch.full_like(qd, float("nan"))
+        b = torch.full_like(qd, float("nan"))
+        lse = torch.empty((2, wl.n_q_heads, q.shape[1]), device="cuda")
+        c2kv.c2kv_extract_attention(ctx, 2, qd, kd, vd, n, k, a, lse)
+        c2kv.c2kv_extract_attention(ctx, 2, qd, kd, vd, n, k, b)
+        c2kv.c2kv_sync(ctx)
+        assert torch.equal(a, b)
+        ref, _ = orc.sif_attention(q, kk, v, n, k, wl.rope_theta, wl.dtype)
+        H.check_attention(b.double().cpu().numpy(), ref, wl, "no-lse call")
+    finally:
+        c2kv.c2kv_destroy(ctx)
 
 
 def test_extract_two_layers_gqa8():
