@@ -49,7 +49,7 @@ def workload_facts(wl):
     # attention bytes: every cache row (slots + suffix) read once, Q read, O written
     attn_bytes = wl.layers * wl.batch * ((S + sq) * row_bytes * 2
                                          + 2 * sq * wl.n_q_heads * wl.head_dim * eb)
-    return dict(slots=S, span=span, positions=wl.batch * span, row_bytes=row_bytes,
+    return dict(name=wl.name, slots=S, span=span, positions=wl.batch * span, row_bytes=row_bytes, dtype=wl.dtype,
                 compose_bytes=compose_bytes, attn_flops=attn_flops, attn_bytes=attn_bytes,
                 slots_per_chunk=m)
 
@@ -62,21 +62,28 @@ def describe(wl):
             f"positions/request), {wl.n_suffix} suffix tokens")
 
 
-def captured_traffic(kernel):
-    """DRAM bytes per launch from the committed ncu summary, if the kernel's source is still
-    the one that was captured (else None: the counters no longer describe this kernel)."""
+def source_digest(paths):
+    """First 16 hex digits of the sha256 of the given source files, concatenated in order."""
     import hashlib
+    h = hashlib.sha256()
+    for rel in paths:
+        with open(os.path.join(ROOT, rel), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def captured_traffic(kernel, workload):
+    """DRAM bytes per launch from the committed ncu summary, if it was captured on this
+    workload and every source the kernel is built from is still the one that was captured
+    (else None: the counters do not describe this launch)."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(path):
         return None
     with open(path) as fh:
         rec = json.load(fh).get(kernel)
-    if not rec:
+    if not rec or "sources" not in rec or rec.get("workload") != workload:
         return None
-    src = os.path.join(ROOT, rec["source"])
-    with open(src, "rb") as fh:
-        digest = hashlib.sha256(fh.read()).hexdigest()[:16]
-    return rec["traffic_bytes"] if digest == rec["sha256_16"] else None
+    return rec["traffic_bytes"] if source_digest(rec["sources"]) == rec["sha256_16"] else None
 
 
 def measured_peaks():
@@ -94,7 +101,7 @@ def rooflines(compose_ms, attn_ms, f, hbm, bf16, src):
     comp_gbs = f["compose_bytes"] / (compose_ms / 1e3) / 1e9
     compose = {"bound": "hbm", "kernel": "compose_kernel", "achieved": round(comp_gbs, 1),
                "peak": hbm, "unit": "GB/s", "frac": round(comp_gbs / hbm, 4),
-               "traffic": captured_traffic("compose_kernel"), "peak_source": f"{src} hbm_gbs",
+               "traffic": captured_traffic("compose_kernel", f["name"]), "peak_source": f"{src} hbm_gbs",
                "bytes_per_launch": f["compose_bytes"]}
     intensity = f["attn_flops"] / f["attn_bytes"]
     ridge = bf16 * 1e12 / (hbm * 1e9)
@@ -108,7 +115,16 @@ def rooflines(compose_ms, attn_ms, f, hbm, bf16, src):
         attend = {"bound": "tensor", "achieved": round(attn_tfs, 2), "peak": bf16,
                   "unit": "TFLOP/s", "frac": round(attn_tfs / bf16, 4),
                   "peak_source": f"{src} bf16_tflops (burst)", "flops_per_launch": f["attn_flops"]}
-    attend.update({"kernel": "attn_tc_kernel", "traffic": captured_traffic("attn_tc_kernel"),
+    if f.get("dtype") == "f32":
+        # fp32 attention runs on the CUDA cores (attn_simt_kernel): plain FP32 FMA arithmetic,
+        # against 128 FMA lanes x 2 flop x 152 SMs x 2.07 GHz = 80.5 TFLOP/s
+        alu = 128 * 2 * 152 * 2.07e9 / 1e12
+        return {"roofline": {"bound": "alu", "kernel": "attn_simt_kernel", "achieved": round(attn_tfs, 3),
+                             "peak": round(alu, 1), "unit": "TFLOP/s", "frac": round(attn_tfs / alu, 4),
+                             "peak_source": "derived: FP32 FMA lanes x clock", "traffic": None,
+                             "flops_per_launch": f["attn_flops"]},
+                "roofline_compose": compose}
+    attend.update({"kernel": "attn_tc_kernel", "traffic": captured_traffic("attn_tc_kernel", f["name"]),
                    "intensity_flop_per_byte": round(intensity, 1), "ridge": round(ridge, 1),
                    "tensor_frac": round(attn_tfs / bf16, 4), "hbm_frac": round(attn_gbs / hbm, 4)})
     if attn_ms >= compose_ms:
@@ -271,12 +287,13 @@ class Arm:
     def decode_run(self, steps, warmup, events):
         """Decode after the suffix: compose once, write the suffix with attend, then decode
         `warmup` untimed and `steps` timed tokens per request (one c2kv_decode call per token,
-        all layers), L2 flushed before each.  Returns (ms per timed step, mean decode kernel
-        ms from the library trace, keys read per timed step summed over requests)."""
+        all layers), L2 flushed before each; then `steps` more tokens with the library's trace
+        on, for the decode kernel's own time.  Returns (ms per timed step, mean decode kernel
+        ms from the trace, keys read per timed step summed over requests)."""
         c2kv, wl, torch = self.c2kv, self.wl, self.torch
         ids = [self.dev_ids[c] for ids_, _ in self.reqs for c in ids_]
         cache = c2kv.c2kv_compose(self.ctx, self.req_ptr, ids, self.positions,
-                                  wl.n_suffix + warmup + steps)
+                                  wl.n_suffix + warmup + 2 * steps)
         c2kv.c2kv_attend(self.ctx, cache, -1, *self.q_dev, wl.n_suffix, self.out)
         B = len(self.reqs)
         gen = torch.Generator(device="cuda").manual_seed(1)
@@ -289,10 +306,7 @@ class Arm:
             self.flush_l2()
             c2kv.c2kv_decode(self.ctx, cache, -1, qd, kd, vd, [wl.n_suffix + i] * B, od)
         c2kv.c2kv_sync(self.ctx)
-        c2kv.c2kv_profile_read(self.ctx)
-        c2kv.c2kv_profile_enable(self.ctx, True)
         keys = 0
-        total = 0.0
         for i in range(steps):
             st = wl.n_suffix + warmup + i
             self.flush_l2()                                    # untimed
@@ -302,11 +316,51 @@ class Arm:
             keys += int(sum(int(n) + st + 1 for n in n_slots))
         torch.cuda.synchronize()
         c2kv.c2kv_sync(self.ctx)
+        total = sum(ev[0].elapsed_time(ev[1]) for ev in events[:steps])
+        c2kv.c2kv_profile_read(self.ctx)
+        c2kv.c2kv_profile_enable(self.ctx, True)
+        for i in range(steps):
+            self.flush_l2()
+            c2kv.c2kv_decode(self.ctx, cache, -1, qd, kd, vd, [wl.n_suffix + warmup + steps + i] * B, od)
         kern = c2kv.c2kv_profile_read(self.ctx)
         c2kv.c2kv_profile_enable(self.ctx, False)
-        total = sum(ev[0].elapsed_time(ev[1]) for ev in events[:steps])
+        c2kv.c2kv_sync(self.ctx)
         c2kv.c2kv_cache_release(self.ctx, cache)
         return total / steps, kern["decode"][0], keys / steps
+
+    def extract_run(self, steps, warmup, events):
+        """Extraction attention over one chunk of the workload's size (n tokens, ratio k, all
+        layers in one call), L2 flushed before each call (untimed).  The inputs are drawn on
+        the device: the timing does not depend on their values.  Returns (mean ms per call,
+        mean ms of the library's trace of the call)."""
+        c2kv, wl, torch = self.c2kv, self.wl, self.torch
+        n, k = wl.chunk_tokens, wl.ratio_k
+        n_all = n + -(-n // k)
+        gen = torch.Generator(device="cuda").manual_seed(2)
+        q = torch.randn((wl.layers, n_all, wl.n_q_heads, wl.head_dim), device="cuda", generator=gen).to(self.tdt)
+        kk = torch.randn((wl.layers, n_all, wl.n_kv_heads, wl.head_dim), device="cuda", generator=gen).to(self.tdt)
+        v = torch.randn_like(kk)
+        out = torch.empty_like(q)
+        for _ in range(warmup):
+            self.flush_l2()
+            c2kv.c2kv_extract_attention(self.ctx, wl.layers, q, kk, v, n, k, out)
+        c2kv.c2kv_sync(self.ctx)
+        for i in range(steps):
+            self.flush_l2()                                    # untimed
+            events[i][0].record(self.stream)
+            c2kv.c2kv_extract_attention(self.ctx, wl.layers, q, kk, v, n, k, out)
+            events[i][1].record(self.stream)
+        torch.cuda.synchronize()
+        c2kv.c2kv_sync(self.ctx)
+        ms = sum(ev[0].elapsed_time(ev[1]) for ev in events[:steps]) / steps
+        c2kv.c2kv_profile_read(self.ctx)
+        c2kv.c2kv_profile_enable(self.ctx, True)
+        for i in range(steps):
+            self.flush_l2()
+            c2kv.c2kv_extract_attention(self.ctx, wl.layers, q, kk, v, n, k, out)
+        kern = c2kv.c2kv_profile_read(self.ctx)
+        c2kv.c2kv_profile_enable(self.ctx, False)
+        return ms, kern["extract"][0]
 
     def e2e_bytes(self, zero_copy=False):
         """Host->device and device->host bytes of one e2e step.  Staged: each distinct
@@ -324,6 +378,51 @@ class Arm:
         self.c2kv.c2kv_destroy(self.ctx)
 
 
+def sif_visible_pairs(n, k):
+    """(query, key) pairs the Structured Information Flow mask lets through over
+    [n document tokens; m = ceil(n/k) C2 tokens]: document token t sees t + 1 keys; C2
+    token c_j sees its block, the first (sink) block when j > 0, and c_0 .. c_j."""
+    m = -(-n // k)
+    sink = min(k, n)
+    pairs = n * (n + 1) // 2
+    for j in range(m):
+        blk = min((j + 1) * k, n) - j * k
+        pairs += blk + (sink if j > 0 else 0) + j + 1
+    return pairs
+
+
+def extract_line(wl, world, ms, kernel_ms, hbm, bf16, src):
+    """Extraction attention over one chunk per rank: document tokens/s over the job, and the
+    call against the tensor and HBM rooflines (algorithmic flops: 4 d per visible (query
+    head, key) pair; bytes: Q, K, V read and O written once)."""
+    eb = 4 if wl.dtype == "f32" else 2
+    n, k = wl.chunk_tokens, wl.ratio_k
+    n_all = n + -(-n // k)
+    flops = 4.0 * wl.head_dim * wl.n_q_heads * sif_visible_pairs(n, k) * wl.layers
+    nbytes = n_all * (2 * wl.n_q_heads + 2 * wl.n_kv_heads) * wl.head_dim * eb * wl.layers
+    t = (kernel_ms or ms) / 1e3
+    tfs, gbs = flops / t / 1e12, nbytes / t / 1e9
+    ridge = bf16 * 1e12 / (hbm * 1e9)
+    tensor = flops / nbytes >= ridge
+    return {
+        "metric": "extracted document tokens/s", "unit": "tokens/s",
+        "value": round(n * world / (ms / 1e3), 1), "ms_per_call": round(ms, 5),
+        "what": f"c2kv_extract_attention over one {n}-token chunk at k={k}, all {wl.layers} "
+                "layers per call (RoPE at the extraction positions, SIF-masked attention); "
+                "L2 flushed before each call (untimed)",
+        "kernel_ms": round(kernel_ms, 5) if kernel_ms else None,
+        "roofline": {"bound": "tensor" if tensor else "hbm",
+                     "kernel": "extraction call (extract_rope_kernel, attn_tc_kernel x2, extract_local_kernel)",
+                     "achieved": round(tfs, 2) if tensor else round(gbs, 1),
+                     "peak": bf16 if tensor else hbm, "unit": "TFLOP/s" if tensor else "GB/s",
+                     "frac": round(tfs / bf16 if tensor else gbs / hbm, 4),
+                     "peak_source": f"{src} " + ("bf16_tflops (burst)" if tensor else "hbm_gbs"),
+                     "flops_per_launch": flops, "bytes_per_launch": nbytes,
+                     "traffic": captured_traffic("extract_call", wl.name),
+                     "tensor_frac": round(tfs / bf16, 4), "hbm_frac": round(gbs / hbm, 4)},
+    }
+
+
 def decode_line(wl, world, dec_ms, dec_kernel_ms, dec_keys, hbm, src):
     eb = 4 if wl.dtype == "f32" else 2
     bytes_step = dec_keys * wl.layers * wl.n_kv_heads * wl.head_dim * eb * 2
@@ -339,7 +438,8 @@ def decode_line(wl, world, dec_ms, dec_kernel_ms, dec_keys, hbm, src):
         "roofline": {"bound": "hbm", "kernel": "decode_kernel (+ merge)",
                      "achieved": round(kernel_gbs, 1) if kernel_gbs else None, "peak": hbm,
                      "unit": "GB/s", "frac": round(kernel_gbs / hbm, 4) if kernel_gbs else None,
-                     "peak_source": f"{src} hbm_gbs", "bytes_per_launch": int(bytes_step)},
+                     "peak_source": f"{src} hbm_gbs", "bytes_per_launch": int(bytes_step),
+                     "traffic": captured_traffic("decode_kernel", wl.name)},
     }
 
 
@@ -378,8 +478,6 @@ def run_ours(args):
     c2kv.c2kv_sync(arm.ctx)
 
     events = [[E(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
-    c2kv.c2kv_profile_read(arm.ctx)            # drop anything recorded before the timed region
-    c2kv.c2kv_profile_enable(arm.ctx, True)     # per-kernel events on the library's stream
     barrier()
     with ClockSampler(local) as clocks:
         t0 = time.perf_counter()
@@ -390,7 +488,18 @@ def run_ours(args):
         wall = time.perf_counter() - t0
     barrier()
     c2kv.c2kv_sync(arm.ctx)
-    kern = c2kv.c2kv_profile_read(arm.ctx)      # mean device ms per kernel kind, timed steps
+    # Per-kernel device times: the same steps again with the library's trace on (events on
+    # its stream around every launch).  An event recorded between two kernels holds the
+    # second back by a few us, so the steps that give the headline run without the trace.
+    c2kv.c2kv_profile_read(arm.ctx)            # drop anything recorded before
+    c2kv.c2kv_profile_enable(arm.ctx, True)
+    trace_events = [[E(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    for i in range(args.steps):
+        arm.flush_l2()
+        arm.step_device(trace_events[i])
+    torch.cuda.synchronize()
+    c2kv.c2kv_sync(arm.ctx)
+    kern = c2kv.c2kv_profile_read(arm.ctx)      # mean device ms per kernel kind
     c2kv.c2kv_profile_enable(arm.ctx, False)
     step_ms = [ev[0].elapsed_time(ev[3]) for ev in events]
     compose_ms = [ev[0].elapsed_time(ev[1]) for ev in events]
@@ -421,9 +530,13 @@ def run_ours(args):
     dec_events = [[E(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
     dec_ms, dec_kernel_ms, dec_keys = arm.decode_run(args.steps, args.warmup, dec_events)
 
+    # extraction attention over one chunk (the encoding side, Sec. 3.3)
+    ext_events = [[E(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
+    ext_ms, ext_kernel_ms = arm.extract_run(args.steps, args.warmup, ext_events)
+
     from paper_2607_17715_gb300.shard import max_over_ranks
-    total_ms, e2e_ms, staged_ms, dec_ms = max_over_ranks([total_ms, e2e_ms, staged_ms, dec_ms],
-                                                         device="cuda")
+    total_ms, e2e_ms, staged_ms, dec_ms, ext_ms = max_over_ranks(
+        [total_ms, e2e_ms, staged_ms, dec_ms, ext_ms], device="cuda")
     arm.close()
     if rank != 0:
         if world > 1:
@@ -472,7 +585,10 @@ def run_ours(args):
         # decode after the suffix: tokens generated per second over the whole job, and the
         # decode kernel against HBM (algorithmic bytes: K and V of every key it attends to)
         "decode": decode_line(wl, world, dec_ms, dec_kernel_ms, dec_keys, hbm, src),
-        # every kernel the library launched in the timed steps (its own trace counts)
+        # extraction attention (the C2 Extractor's masked attention) over one chunk
+        "extract": extract_line(wl, world, ext_ms, ext_kernel_ms, hbm, bf16, src),
+        # every kernel the library launched in the timed steps (counted by its trace of the
+        # identical traced pass)
         "gpu_launches": sum(v[1] for v in kern.values()),
         "clocks": clk,
     }

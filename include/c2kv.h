@@ -320,10 +320,11 @@ const char* c2kv_last_error(const c2kv_ctx* ctx);
 
 /*
  * Tracing: per-kernel device time.  While enabled, each kernel launch the library makes
- * (compose, compress, suffix RoPE/append, attention) is bracketed by CUDA events on the
- * context's stream.  c2kv_profile_read synchronizes the stream and returns, per kind, the
- * mean device time of the launches recorded since the previous read (or since enabling),
- * then forgets them.  Kinds index the arrays:
+ * (compose, compress, suffix RoPE/append, attention, decode, extraction) is bracketed by
+ * CUDA events on the context's stream.  Enabling creates a stock of events up front, so a
+ * traced call only records them.  c2kv_profile_read synchronizes the stream and returns,
+ * per kind, the mean device time of the launches recorded since the previous read (or
+ * since enabling), then forgets them.  Kinds index the arrays:
  */
 #define C2KV_PROF_COMPOSE  0
 #define C2KV_PROF_COMPRESS 1

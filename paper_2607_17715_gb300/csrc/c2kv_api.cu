@@ -171,6 +171,8 @@ void destroy_cache(c2kv_ctx* c, c2kv_cache* cache) {
     delete cache;
 }
 
+constexpr size_t kProfEvents = 1024;   // events made ready when tracing is enabled
+
 cudaEvent_t prof_event(c2kv_ctx* c) {
     if (!c->prof_free.empty()) {
         cudaEvent_t e = c->prof_free.back();
@@ -934,6 +936,20 @@ c2kv_status c2kv_sync(c2kv_ctx* c) {
 c2kv_status c2kv_profile_enable(c2kv_ctx* c, int32_t on) {
     if (!c) return C2KV_ERR_ARG;
     c->prof = on != 0;
+    // create the trace's events now, so that a traced call only records them: creating
+    // events inside the calls would slow the host enough to delay the launches it traces
+    try {
+        const size_t have = c->prof_free.size() + 2 * c->prof_recs.size();
+        for (size_t i = have; c->prof && i < kProfEvents; ++i) {
+            cudaEvent_t e = nullptr;
+            if (cudaEventCreate(&e) != cudaSuccess) {
+                (void)cudaGetLastError();
+                break;
+            }
+            c->prof_free.push_back(e);
+        }
+    } catch (const std::bad_alloc&) {
+    }
     return C2KV_OK;
 }
 

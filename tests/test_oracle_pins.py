@@ -506,6 +506,38 @@ def test_pins_catch_a_leaky_sif_mask(monkeypatch):
         test_sif_document_rows_are_causal_attention(13, 4)
 
 
+def test_pins_catch_a_sif_mask_that_sees_ahead(monkeypatch):
+    # c_j also seeing c_{j+1} (a causal accumulation shifted by one) fails the brute force
+    good = orc.sif_mask
+
+    def ahead(n, k):
+        vis = good(n, k)
+        m = vis.shape[0] - n
+        for j in range(m - 1):
+            vis[n + j, n + j + 1] = True
+        return vis
+    monkeypatch.setattr(orc, "sif_mask", ahead)
+    with pytest.raises(AssertionError):
+        test_sif_c2_rows_bruteforce()
+
+
+def test_pins_catch_a_sif_sink_taken_as_the_last_block(monkeypatch):
+    # reading the sink block as the chunk's last block instead of its first fails the pins
+    good = orc.sif_mask
+
+    def last_sink(n, k):
+        vis = good(n, k)
+        m = vis.shape[0] - n
+        for j in range(m):
+            vis[n + j, :n] = False
+            vis[n + j, j * k:min((j + 1) * k, n)] = True
+            vis[n + j, (m - 1) * k:n] = True
+        return vis
+    monkeypatch.setattr(orc, "sif_mask", last_sink)
+    with pytest.raises(AssertionError):
+        test_sif_c2_rows_bruteforce()
+
+
 def test_lse_combine_equals_unsplit():
     s_len, sq, d, hq, hkv = 50, 7, 8, 4, 2
     keys = RNG.standard_normal((s_len + sq, hkv, d))
