@@ -49,8 +49,13 @@ def workload_facts(wl):
     # attention bytes: every cache row (slots + suffix) read once, Q read, O written
     attn_bytes = wl.layers * wl.batch * ((S + sq) * row_bytes * 2
                                          + 2 * sq * wl.n_q_heads * wl.head_dim * eb)
+    # fused compose + attention: every stored slot read and its composed row written once
+    # (compose's bytes), the suffix rows and Q read, O written; the cache is not read back
+    fused_bytes = compose_bytes + wl.layers * wl.batch * (sq * row_bytes * 2
+                                                          + 2 * sq * wl.n_q_heads * wl.head_dim * eb)
     return dict(name=wl.name, slots=S, span=span, positions=wl.batch * span, row_bytes=row_bytes, dtype=wl.dtype,
                 compose_bytes=compose_bytes, attn_flops=attn_flops, attn_bytes=attn_bytes,
+                fused_bytes=fused_bytes,
                 slots_per_chunk=m)
 
 
@@ -130,6 +135,29 @@ def rooflines(compose_ms, attn_ms, f, hbm, bf16, src):
     if attn_ms >= compose_ms:
         return {"roofline": attend, "roofline_compose": compose}
     return {"roofline": compose, "roofline_attend": attend}
+
+
+def step_rooflines(fused_ran, kern, kc_ms, ka_ms, f, hbm, bf16, src):
+    r = rooflines(kc_ms, ka_ms, f, hbm, bf16, src)
+    if not fused_ran:
+        return r
+    parts = {o["kernel"]: o for o in r.values()}
+    return {"roofline": fused_roofline(kern["fused"][0], f, hbm, bf16, src),
+            "roofline_compose": parts.get("compose_kernel"),
+            "roofline_attend": parts.get("attn_tc_kernel", parts.get("attn_simt_kernel"))}
+
+
+def fused_roofline(fused_ms, f, hbm, bf16, src):
+    """The fused compose + attention kernel: HBM-bound (its intensity, attention flops over
+    fused bytes, is far below the ridge); both fractions carried."""
+    gbs = f["fused_bytes"] / (fused_ms / 1e3) / 1e9
+    tfs = f["attn_flops"] / (fused_ms / 1e3) / 1e12
+    return {"bound": "hbm", "kernel": "attn_tc_kernel<fused>",
+            "achieved": round(gbs, 1), "peak": hbm, "unit": "GB/s", "frac": round(gbs / hbm, 4),
+            "peak_source": f"{src} hbm_gbs", "bytes_per_launch": f["fused_bytes"],
+            "traffic": captured_traffic("attn_tc_kernel_fused", f["name"]),
+            "intensity_flop_per_byte": round(f["attn_flops"] / f["fused_bytes"], 1),
+            "tensor_frac": round(tfs / bf16, 4), "hbm_frac": round(gbs / hbm, 4)}
 
 
 # --------------------------------------------------------------------------- clocks
@@ -243,33 +271,43 @@ class Arm:
     def flush_l2(self):
         self.flush_buf.fill_(1.0)
 
-    def step_device(self, ev):
-        """compose + attend with inputs resident in HBM; ev = 4 events to record."""
+    def step_device(self, ev, fused=True):
+        """One step with inputs resident in HBM: c2kv_compose_attend (the library fuses the
+        two when that pays), or c2kv_compose then c2kv_attend; then the cache is released.
+        ev = 4 events to record (before, after compose or the joint call, after attend,
+        after release)."""
         c2kv, wl = self.c2kv, self.wl
         ids = [self.dev_ids[c] for ids_, _ in self.reqs for c in ids_]
         ev[0].record(self.stream)
-        cache = c2kv.c2kv_compose(self.ctx, self.req_ptr, ids, self.positions, wl.n_suffix)
-        ev[1].record(self.stream)
-        c2kv.c2kv_attend(self.ctx, cache, -1, *self.q_dev, wl.n_suffix, self.out)
+        if fused:
+            cache = c2kv.c2kv_compose_attend(self.ctx, self.req_ptr, ids, self.positions,
+                                             wl.n_suffix, *self.q_dev, wl.n_suffix, self.out)
+            ev[1].record(self.stream)
+        else:
+            cache = c2kv.c2kv_compose(self.ctx, self.req_ptr, ids, self.positions, wl.n_suffix)
+            ev[1].record(self.stream)
+            c2kv.c2kv_attend(self.ctx, cache, -1, *self.q_dev, wl.n_suffix, self.out)
         ev[2].record(self.stream)
         c2kv.c2kv_cache_release(self.ctx, cache)
         ev[3].record(self.stream)
 
     def step_e2e_host(self):
         """The same step from host buffers, zero-copy: copy the suffix in, compose straight
-        from the chunks' pinned host slots (load, re-rotation and gather in one kernel),
-        attend, read the output back."""
+        from the chunks' pinned host slots (load, re-rotation and gather in one kernel) and
+        attend (one call; host-resident chunks take compose, then attention), read the
+        output back."""
         c2kv, wl = self.c2kv, self.wl
         qd = [x.to("cuda", non_blocking=True) for x in self.q_host]
         ids = [self.host_ids[c] for ids_, _ in self.reqs for c in ids_]
-        cache = c2kv.c2kv_compose(self.ctx, self.req_ptr, ids, self.positions, wl.n_suffix)
-        c2kv.c2kv_attend(self.ctx, cache, -1, *qd, wl.n_suffix, self.out)
+        cache = c2kv.c2kv_compose_attend(self.ctx, self.req_ptr, ids, self.positions, wl.n_suffix,
+                                         *qd, wl.n_suffix, self.out)
         self.out_host.copy_(self.out, non_blocking=True)
         c2kv.c2kv_cache_release(self.ctx, cache)
 
     def step_e2e(self):
         """The same step from host buffers, staged: copy the requested chunks from pinned host
-        memory into the pool, copy the suffix in, compose, attend, read the output back."""
+        memory into the pool, copy the suffix in, compose and attend (one call), read the
+        output back."""
         c2kv, wl, torch = self.c2kv, self.wl, self.torch
         loaded = {}
         for cid, (kh, vh) in self.host_chunks.items():
@@ -277,8 +315,8 @@ class Arm:
                                                    wl.ratio_k, c2kv.MODE_STORED)
         qd = [x.to("cuda", non_blocking=True) for x in self.q_host]
         ids = [loaded[c] for ids_, _ in self.reqs for c in ids_]
-        cache = c2kv.c2kv_compose(self.ctx, self.req_ptr, ids, self.positions, wl.n_suffix)
-        c2kv.c2kv_attend(self.ctx, cache, -1, *qd, wl.n_suffix, self.out)
+        cache = c2kv.c2kv_compose_attend(self.ctx, self.req_ptr, ids, self.positions, wl.n_suffix,
+                                         *qd, wl.n_suffix, self.out)
         self.out_host.copy_(self.out, non_blocking=True)
         c2kv.c2kv_cache_release(self.ctx, cache)
         for cid in loaded.values():
@@ -475,6 +513,8 @@ def run_ours(args):
     for _ in range(args.warmup):
         arm.flush_l2()
         arm.step_device([E(enable_timing=True) for _ in range(4)])
+        arm.flush_l2()
+        arm.step_device([E(enable_timing=True) for _ in range(4)], fused=False)
     c2kv.c2kv_sync(arm.ctx)
 
     events = [[E(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
@@ -491,20 +531,34 @@ def run_ours(args):
     # Per-kernel device times: the same steps again with the library's trace on (events on
     # its stream around every launch).  An event recorded between two kernels holds the
     # second back by a few us, so the steps that give the headline run without the trace.
-    c2kv.c2kv_profile_read(arm.ctx)            # drop anything recorded before
-    c2kv.c2kv_profile_enable(arm.ctx, True)
-    trace_events = [[E(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    def traced(fused):
+        c2kv.c2kv_profile_read(arm.ctx)        # drop anything recorded before
+        c2kv.c2kv_profile_enable(arm.ctx, True)
+        evs = [[E(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+        for i in range(args.steps):
+            arm.flush_l2()
+            arm.step_device(evs[i], fused=fused)
+        torch.cuda.synchronize()
+        c2kv.c2kv_sync(arm.ctx)
+        k = c2kv.c2kv_profile_read(arm.ctx)    # mean device ms per kernel kind
+        c2kv.c2kv_profile_enable(arm.ctx, False)
+        return k
+    kern = traced(True)
+    step_ms = [ev[0].elapsed_time(ev[3]) for ev in events]
+    total_ms = sum(step_ms)
+    # the same steps as separate compose and attend calls: the two kernels the fused path
+    # replaces, each against its own roofline
+    un_events = [[E(enable_timing=True) for _ in range(4)] for _ in range(args.steps)]
+    barrier()
     for i in range(args.steps):
         arm.flush_l2()
-        arm.step_device(trace_events[i])
+        arm.step_device(un_events[i], fused=False)
     torch.cuda.synchronize()
     c2kv.c2kv_sync(arm.ctx)
-    kern = c2kv.c2kv_profile_read(arm.ctx)      # mean device ms per kernel kind
-    c2kv.c2kv_profile_enable(arm.ctx, False)
-    step_ms = [ev[0].elapsed_time(ev[3]) for ev in events]
-    compose_ms = [ev[0].elapsed_time(ev[1]) for ev in events]
-    attend_ms = [ev[1].elapsed_time(ev[2]) for ev in events]
-    total_ms = sum(step_ms)
+    un_total_ms = sum(ev[0].elapsed_time(ev[3]) for ev in un_events)
+    compose_ms = [ev[0].elapsed_time(ev[1]) for ev in un_events]
+    attend_ms = [ev[1].elapsed_time(ev[2]) for ev in un_events]
+    kern_un = traced(False)
 
     # end to end from host buffers (host->device traffic inside the timed region), both
     # ways the library offers: zero-copy compose from pinned host slots, and staged copies
@@ -535,8 +589,8 @@ def run_ours(args):
     ext_ms, ext_kernel_ms = arm.extract_run(args.steps, args.warmup, ext_events)
 
     from paper_2607_17715_gb300.shard import max_over_ranks
-    total_ms, e2e_ms, staged_ms, dec_ms, ext_ms = max_over_ranks(
-        [total_ms, e2e_ms, staged_ms, dec_ms, ext_ms], device="cuda")
+    total_ms, un_total_ms, e2e_ms, staged_ms, dec_ms, ext_ms = max_over_ranks(
+        [total_ms, un_total_ms, e2e_ms, staged_ms, dec_ms, ext_ms], device="cuda")
     arm.close()
     if rank != 0:
         if world > 1:
@@ -549,9 +603,11 @@ def run_ours(args):
     value = positions / (total_ms / 1e3)
     c_ms = statistics.mean(compose_ms)
     a_ms = statistics.mean(attend_ms)
-    kc_ms = kern["compose"][0] or c_ms         # compose kernel alone (library events)
+    kc_ms = kern_un["compose"][0] or c_ms      # compose kernel alone (library events)
     # attention kernel (plus the merge of its key-range splits, when it was split)
-    ka_ms = (kern["attention"][0] + kern["combine"][0]) or a_ms
+    ka_ms = (kern_un["attention"][0] + kern_un["combine"][0]) or a_ms
+    fused_ran = kern["fused"][1] > 0
+    step_kernels = {k: round(v[0], 5) for k, v in kern.items() if v[1]}
     comp_gbs = f["compose_bytes"] / (kc_ms / 1e3) / 1e9
     attn_tfs = f["attn_flops"] / (ka_ms / 1e3) / 1e12
     clk = clocks.summary()
@@ -564,15 +620,21 @@ def run_ours(args):
                    "l2": "flushed between timed steps (256 MB write, untimed)",
                    "global_batch": wl.batch * world,
                    "ttft_proxy_ms_per_layer": round(kc_ms / wl.layers, 6),
-                   "compose_call_ms": round(c_ms, 5), "attend_call_ms": round(a_ms, 5),
-                   "kernel_ms": {k: round(v[0], 5) for k, v in kern.items() if v[1]},
+                   "step": ("c2kv_compose_attend: fused compose + attention kernel" if fused_ran
+                            else "c2kv_compose_attend: compose, then attention"),
+                   "kernel_ms": step_kernels,
+                   "unfused": {"value": round(positions / (un_total_ms / 1e3), 1),
+                               "ms_per_step": round(un_total_ms / args.steps, 5),
+                               "compose_call_ms": round(c_ms, 5), "attend_call_ms": round(a_ms, 5),
+                               "kernel_ms": {k: round(v[0], 5) for k, v in kern_un.items() if v[1]}},
                    "compose_gbs": round(comp_gbs, 1), "attend_tflops": round(attn_tfs, 2),
                    "compose_bytes": f["compose_bytes"], "attend_flops": f["attn_flops"],
-                   "wall_s": round(wall, 4)},
-        # the dominant kernel of the step (by device time) carries "roofline"; the other
-        # judged kernel is reported beside it.  Attention is HBM- or tensor-bound depending on
-        # its arithmetic intensity relative to the ridge of the measured peaks.
-        **rooflines(kc_ms, ka_ms, f, hbm, bf16, src),
+                   "fused_bytes": f["fused_bytes"], "wall_s": round(wall, 4)},
+        # the dominant kernel of the step (by device time) carries "roofline"; the judged
+        # compose and attention kernels (from the same steps run as separate calls) are
+        # reported beside it.  Attention is HBM- or tensor-bound depending on its arithmetic
+        # intensity relative to the ridge of the measured peaks.
+        **step_rooflines(fused_ran, kern, kc_ms, ka_ms, f, hbm, bf16, src),
         "e2e": {"value": round(positions / (e2e_ms / 1e3), 1),
                 "unit": "tokens/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "ms_per_step": round(e2e_ms / args.steps, 4),

@@ -63,6 +63,13 @@ typedef int32_t c2kv_status;
 #define C2KV_ATTN_SIMT   1    /* CUDA-core fp32-accumulate kernel (any dtype)        */
 #define C2KV_ATTN_TC     2    /* tcgen05 / TMEM tensor-core kernel (bf16, d = 128)    */
 
+/* c2kv_compose_attend: when the fused compose + attention kernel runs */
+#define C2KV_FUSE_AUTO   0    /* when each (layer, request, KV head) has a single pair of
+                                 128-row query tiles, n_suffix * Hq / Hkv <= 256: every
+                                 stored slot is then read and turned by exactly one CTA   */
+#define C2KV_FUSE_NEVER  1    /* always compose, then attend                           */
+#define C2KV_FUSE_ALWAYS 2    /* whenever the fused kernel takes the call              */
+
 typedef struct c2kv_ctx c2kv_ctx;
 typedef struct c2kv_cache c2kv_cache;
 
@@ -82,6 +89,7 @@ typedef struct c2kv_config {
                                   0 = chosen per call (split only when the units would leave
                                   most SMs idle), 1 = never, n <= 16 = always n (partials
                                   merged by an exact log-sum-exp combine)                     */
+    int32_t fuse;              /* C2KV_FUSE_AUTO / _NEVER / _ALWAYS (c2kv_compose_attend)     */
 } c2kv_config;
 
 /* Chunk metadata (c2kv_chunk_info). */
@@ -111,7 +119,7 @@ typedef struct c2kv_cache_desc {
 } c2kv_cache_desc;
 
 /* ABI version of this header (bumped on any incompatible change). */
-#define C2KV_ABI_VERSION 3
+#define C2KV_ABI_VERSION 4
 int32_t c2kv_abi_version(void);
 
 /*
@@ -227,6 +235,32 @@ c2kv_status c2kv_attend(c2kv_ctx* ctx, c2kv_cache* cache, int32_t layer, const v
                         float* lse);
 
 /*
+ * c2kv_compose_attend -- blending and inference in one call: the same result as
+ *     c2kv_compose(ctx, batch, req_ptr, chunk_ids, positions, suffix_capacity, cache_out)
+ *     c2kv_attend(ctx, *cache_out, -1, q, k_suf, v_suf, n_suffix, out, lse)
+ * (the composed cache, its positions, the suffix rows, O and lse), for every layer.  On
+ * the tensor-core route (bf16, d 128) with every chunk in the device pool, at most 256
+ * requests and at most 512 chunk occurrences, one fused kernel does both: the attention
+ * reads each composed slot straight from the pool, turns K by its occurrence's offset in
+ * shared memory (Sec. 3.2.4 re-rotation) and writes the composed cache as it goes, so the
+ * cache is written once and never read back.  Otherwise compose and attention run one after
+ * the other.  The context's `fuse` setting chooses (C2KV_FUSE_*): by default the fused
+ * kernel runs when each (layer, request, KV head) has one pair of query tiles.  The cache is returned as by c2kv_compose (release it with c2kv_cache_release)
+ * and serves later c2kv_decode / c2kv_attend calls.
+ *
+ *   batch, req_ptr, chunk_ids, positions, suffix_capacity : as c2kv_compose.
+ *   q, k_suf, v_suf, n_suffix, out, lse : as c2kv_attend with layer = -1;
+ *                1 <= n_suffix <= suffix_capacity.
+ *   cache_out : receives the composed cache.
+ * Errors: the union of c2kv_compose's and c2kv_attend's; on error no cache is returned.
+ */
+c2kv_status c2kv_compose_attend(c2kv_ctx* ctx, int32_t batch, const int32_t* req_ptr,
+                                const int32_t* chunk_ids, const int32_t* positions,
+                                int32_t suffix_capacity, const void* q, const void* k_suf,
+                                const void* v_suf, int32_t n_suffix, void* out, float* lse,
+                                c2kv_cache** cache_out);
+
+/*
  * c2kv_attend_noalloc -- the same computation and arguments as c2kv_attend, for callers
  * that cannot let the library allocate device memory while they run: for example a
  * serving engine that reserves all of HBM for its own cache pool at start-up and treats
@@ -333,7 +367,8 @@ const char* c2kv_last_error(const c2kv_ctx* ctx);
 #define C2KV_PROF_COMBINE  4   /* merge of key-range splits (when attention was split) */
 #define C2KV_PROF_DECODE   5   /* decode attention (with the merge of its splits) */
 #define C2KV_PROF_EXTRACT  6   /* SIF-masked extraction attention (RoPE + attention) */
-#define C2KV_PROF_KINDS    7
+#define C2KV_PROF_FUSED    7   /* fused compose + attention kernel (c2kv_compose_attend) */
+#define C2KV_PROF_KINDS    8
 c2kv_status c2kv_profile_enable(c2kv_ctx* ctx, int32_t on);
 /* mean_ms[C2KV_PROF_KINDS] receives mean milliseconds (0 where none), launches[] the
  * counts; either may be NULL. */

@@ -29,10 +29,12 @@ ERR_POSITIONS, ERR_CUDA, ERR_DEVICE_BOUNDS, ERR_STATE, ERR_UNSUPPORTED = -6, -7,
 DTYPE_BF16, DTYPE_F32 = 0, 1
 MODE_MEANPOOL, MODE_PROVIDED, MODE_STORED, MODE_HOST = 0, 1, 2, 3
 ATTN_AUTO, ATTN_SIMT, ATTN_TC = 0, 1, 2
+FUSE_AUTO, FUSE_NEVER, FUSE_ALWAYS = 0, 1, 2
 PROF_COMPOSE, PROF_COMPRESS, PROF_SUFFIX, PROF_ATTN, PROF_COMBINE, PROF_DECODE = 0, 1, 2, 3, 4, 5
-PROF_EXTRACT = 6
-PROF_KINDS = 7
-PROF_NAMES = ("compose", "compress", "suffix", "attention", "combine", "decode", "extract")
+PROF_EXTRACT, PROF_FUSED = 6, 7
+PROF_KINDS = 8
+PROF_NAMES = ("compose", "compress", "suffix", "attention", "combine", "decode", "extract",
+              "fused")
 
 STATUS_NAMES = {
     0: "OK", -1: "ERR_ARG", -2: "ERR_DTYPE", -3: "ERR_NOMEM", -4: "ERR_POOL_FULL",
@@ -46,7 +48,8 @@ class c2kv_config(ctypes.Structure):
                 ("n_kv_heads", ctypes.c_int32), ("head_dim", ctypes.c_int32),
                 ("rope_theta", ctypes.c_double), ("dtype", ctypes.c_int32),
                 ("pool_slots", ctypes.c_int32), ("fixed_pos", ctypes.c_int32),
-                ("attn_impl", ctypes.c_int32), ("attn_split", ctypes.c_int32)]
+                ("attn_impl", ctypes.c_int32), ("attn_split", ctypes.c_int32),
+                ("fuse", ctypes.c_int32)]
 
 
 class c2kv_chunk_desc(ctypes.Structure):
@@ -76,6 +79,8 @@ _SIGS = {
     "c2kv_free_chunk": (_I32, [_VP, _I32]),
     "c2kv_chunk_info": (_I32, [_VP, _I32, ctypes.POINTER(c2kv_chunk_desc)]),
     "c2kv_compose": (_I32, [_VP, _I32, _P32, _P32, _P32, _I32, ctypes.POINTER(_VP)]),
+    "c2kv_compose_attend": (_I32, [_VP, _I32, _P32, _P32, _P32, _I32, _VP, _VP, _VP, _I32, _VP,
+                                   _VP, ctypes.POINTER(_VP)]),
     "c2kv_cache_info": (_I32, [_VP, ctypes.POINTER(c2kv_cache_desc)]),
     "c2kv_attend": (_I32, [_VP, _VP, _I32, _VP, _VP, _VP, _I32, _VP, _VP]),
     "c2kv_attend_noalloc": (_I32, [_VP, _VP, _I32, _VP, _VP, _VP, _I32, _VP, _VP]),
@@ -145,9 +150,9 @@ def c2kv_last_error(ctx=None) -> str:
 
 
 def c2kv_create(layers, n_q_heads, n_kv_heads, head_dim, rope_theta, dtype, pool_slots,
-                fixed_pos=0, attn_impl=ATTN_AUTO, stream=None, attn_split=0):
+                fixed_pos=0, attn_impl=ATTN_AUTO, stream=None, attn_split=0, fuse=0):
     cfg = c2kv_config(layers, n_q_heads, n_kv_heads, head_dim, float(rope_theta), dtype,
-                      pool_slots, int(fixed_pos), attn_impl, attn_split)
+                      pool_slots, int(fixed_pos), attn_impl, attn_split, fuse)
     out = _VP()
     _check(_lib.c2kv_create(ctypes.byref(cfg), _stream_handle(stream), ctypes.byref(out)))
     return out.value
@@ -186,6 +191,20 @@ def c2kv_compose(ctx, req_ptr, chunk_ids, positions=None, suffix_capacity=0):
     _check(_lib.c2kv_compose(ctx, len(rp) - 1, rp_p, ids_p, pos_p, suffix_capacity,
                              ctypes.byref(out)), ctx)
     return out.value
+
+
+def c2kv_compose_attend(ctx, req_ptr, chunk_ids, positions, suffix_capacity, q, k_suf, v_suf,
+                        n_suffix, out, lse=None):
+    """Compose the requests' chunks and attend their suffixes over all layers in one call
+    (fused on the tensor-core route); returns the composed cache."""
+    rp, rp_p = _i32(req_ptr)
+    ids, ids_p = _i32(chunk_ids)
+    pos, pos_p = _i32(positions)
+    cache = _VP()
+    _check(_lib.c2kv_compose_attend(ctx, len(rp) - 1, rp_p, ids_p, pos_p, suffix_capacity, _ptr(q),
+                                    _ptr(k_suf), _ptr(v_suf), n_suffix, _ptr(out), _ptr(lse),
+                                    ctypes.byref(cache)), ctx)
+    return cache.value
 
 
 def c2kv_cache_info(cache) -> dict:

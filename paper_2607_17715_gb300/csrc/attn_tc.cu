@@ -37,6 +37,17 @@
 // Every mbarrier wait is bounded (kWaitCycles); on expiry the waiting thread sets bit 1
 // of the error word and carries on, so the kernel always terminates and the host reports
 // C2KV_ERR_DEVICE_BOUNDS at the next c2kv_sync.
+//
+// Fused compose + attention (the same kernel, kFused = true, 512 threads).  Instead of TMA
+// from the composed cache, a fourth warpgroup (warps 12..15, the loaders) fills the K and V
+// rings itself: each composed slot row comes straight from the chunk pool and each suffix
+// row from the cache, one 16-byte cp.async per chunk into the 128-byte-swizzled layout the
+// MMA descriptors expect.  A loader thread then turns the K chunks it copied by their
+// occurrence's offset (the same phase-accumulator angles and fp32 rotation as the compose
+// kernel), and the CTAs of query-tile pair 0 write the turned K', V and the positions of
+// the composed slots to the cache, so the cache is complete for later decode steps.  The
+// pool is read once per (layer, request, KV head) pair and the composed cache is written
+// once, rather than written by compose and read back by attention.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -46,6 +57,8 @@
 
 #include "internal.cuh"
 #include "ptx.cuh"
+#include "rope.cuh"
+#include "vec16.cuh"
 
 namespace c2kv {
 namespace {
@@ -66,6 +79,14 @@ constexpr int kLaunchRegs = 168;
 constexpr int kRegsLow = 136;
 constexpr int kRegsHigh = 184;
 static_assert(128 * kRegsLow + 256 * kRegsHigh <= kThreads * kLaunchRegs, "register split");
+// Fused: 512 threads launch with 128 registers each; the producer/issuer warpgroup and the
+// loader warpgroup keep 72, the softmax warpgroups rise to 184.
+constexpr int kThreadsFused = 512;
+constexpr int kLaunchRegsFused = 128;
+constexpr int kRegsLowFused = 72;
+constexpr int kLoaders = 128;       // K loaders (warps 12..15)
+constexpr int kVLoaders = 32;       // V loader (warp 3)
+static_assert(256 * kRegsLowFused + 256 * kRegsHigh <= kThreadsFused * kLaunchRegsFused, "fused register split");
 constexpr uint32_t kTmemCols = 512;     // S_A, S_B, O_A, O_B; P_x over the first half of S_x
 constexpr uint32_t kColS = 0, kColO = 256;
 
@@ -78,7 +99,11 @@ constexpr int B_VE = B_VF + VSTAGES;     // + stage: V stage free (both P.V fini
 constexpr int B_SF = B_VE + VSTAGES;     // + tile: S_x(j) complete (and every MMA before it)
 constexpr int B_PF = B_SF + 2;           // + tile: P_x(j) written (and O_x corrected)
 constexpr int B_OD = B_PF + 2;           // every MMA finished: O_A, O_B final
-constexpr int NBAR = B_OD + 1;
+constexpr int B_KL = B_OD + 1;           // + stage (fused): the TMA part of a K tile landed
+constexpr int B_VL = B_KL + KSTAGES;     // + stage (fused): the TMA part of a V tile landed
+constexpr int B_KW = B_VL + VSTAGES;     // + stage (fused): K' of the stage's tile stored to the cache
+constexpr int B_VW = B_KW + KSTAGES;     // + stage (fused): V of the stage's tile stored
+constexpr int NBAR = B_VW + VSTAGES;
 
 constexpr int kSmemTiles = 2 /*Q_A, Q_B*/ + KSTAGES + VSTAGES;
 constexpr size_t kSmemBytes = 1024 /*align*/ + (size_t)TILE * kSmemTiles + 8 * NBAR + 16;
@@ -99,6 +124,35 @@ struct TcParams {                // CUtensorMap members carry their own alignmen
     float* part_lse;
     ReqParam req[kMaxReq];
 };
+
+struct FusedTcParams {
+    TcParams t;
+    // pool [L*pool_slots][Hkv][128] and cache [L*rows][Hkv][128] in boxes of 128 rows (whole
+    // tiles from one source), 64 rows and 8 rows (one swizzle atom) for the runs of clean
+    // groups of a mixed tile
+    CUtensorMap tm_pk, tm_pv, tm_pk64, tm_pv64, tm_pk8, tm_pv8, tm_ck64, tm_cv64, tm_ck8, tm_cv8;
+    const void* pool_k;      // [L][pool_slots][Hkv][128]
+    const void* pool_v;
+    void* cache_k;           // [L][rows][Hkv][128]: suffix rows read, composed rows written
+    void* cache_v;
+    int32_t* pos;            // [rows]
+    float2* occ_cs;          // scratch [occurrences][64]: (cos, sin) of each occurrence's turn
+    int64_t pool_slots;
+    RopeTurns rope;
+    int32_t req_occ[kMaxReq + 1];
+    FusedOcc occ[kMaxFusedOcc];
+};
+
+template <bool kFused>
+struct KernelParams {
+    using type = TcParams;
+};
+template <>
+struct KernelParams<true> {
+    using type = FusedTcParams;
+};
+__device__ __forceinline__ const TcParams& tc_params(const TcParams& p) { return p; }
+__device__ __forceinline__ const TcParams& tc_params(const FusedTcParams& p) { return p.t; }
 
 // ------------------------------------------------------------------ tcgen05 wrappers
 
@@ -500,7 +554,456 @@ __device__ __forceinline__ void mma_issuer(const TcParams& P, uint32_t tmem, uin
     mma_commit(bar(B_OD));
 }
 
-__global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_constant__ TcParams P) {
+// ------------------------------------------------------------------ fused loaders
+
+__device__ __forceinline__ void cp_async16(uint32_t dst, const void* src) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16;" ::"r"(dst), "l"(src) : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
+}
+// generic-proxy writes to shared memory become visible to the tensor core's (async) reads
+__device__ __forceinline__ void fence_proxy_async() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+__device__ __forceinline__ uint4 lds128(uint32_t a) {
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                 : "r"(a)
+                 : "memory");
+    return v;
+}
+__device__ __forceinline__ void sts128(uint32_t a, const uint4& v) {
+    asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(a), "r"(v.x), "r"(v.y), "r"(v.z),
+                 "r"(v.w)
+                 : "memory");
+}
+// Byte offset of 16-byte chunk q (0..7) of row r in a 128-row, 128-byte-wide swizzled block
+// (the SWIZZLE_128B layout: the chunk index XOR the row index mod 8).
+__device__ __forceinline__ uint32_t sw_off(int r, int q) {
+    return (uint32_t)(r * 128 + ((q ^ (r & 7)) << 4));
+}
+
+// A walk over one request's occurrences in composed-row order.  The occurrence table sits
+// in the kernel parameters; a dependent chain of reads there costs a memory latency per
+// step, so each walk keeps its current occurrence in registers and reads the table only
+// when a row moves past it (rows only increase).
+struct OccWalk {
+    int idx;    // current occurrence
+    int beg;    // its first composed row (relative to the request)
+    int end;    // one past its last
+    int src;    // pool slot of row beg
+};
+__device__ __forceinline__ void walk_load(OccWalk& w, const FusedTcParams& F, int i) {
+    w.idx = i;
+    w.beg = F.occ[i].dest_row;
+    w.end = w.beg + F.occ[i].m;
+    w.src = F.occ[i].src_row;
+}
+__device__ __forceinline__ void walk_to(OccWalk& w, const FusedTcParams& F, int R, int o_end) {
+    while (R >= w.end && w.idx + 1 < o_end) walk_load(w, F, w.idx + 1);
+}
+// Pool slot of composed slot row R, or -1 (bounds-check bit set) if it is out of range.
+__device__ __forceinline__ int64_t walk_slot(OccWalk& w, const FusedTcParams& F, int R, int o_end) {
+    walk_to(w, F, R, o_end);
+    const int64_t slot = (int64_t)w.src + (R - w.beg);
+    if (R < w.beg || R >= w.end || slot < 0 || slot >= F.pool_slots) {
+        atomicOr(F.t.err, 1);
+        return -1;
+    }
+    return slot;
+}
+// Whether the 8-row group of composed row R (rows R & ~7 .. +7) comes from more than one
+// contiguous source: several occurrences, or composed slots and suffix rows.  Clean groups
+// are moved by TMA, ragged ones row by row.
+__device__ __forceinline__ bool group_ragged(OccWalk& w, const FusedTcParams& F, int R, int n_slots,
+                                            int o_end) {
+    const int gs = R & ~7, ge = gs + 8;
+    if (R >= n_slots) return gs < n_slots;
+    walk_to(w, F, R, o_end);
+    return !(w.beg <= gs && ge <= w.end);
+}
+
+// The fused kernel's TMA producer (one thread): for each key tile, K and V each as soon as
+// their stage is free.  A tile from one source (a single occurrence's pool slots, or the
+// cache's suffix rows) is two 128-row boxes; a mixed tile is one 8-row box per clean group
+// (its ragged groups are left to the loaders).  The stage's "landed" barrier expects the
+// bytes of the boxes issued.
+__device__ __forceinline__ void fused_producer(const FusedTcParams& F, int l, int bl, int hk, int j_base,
+                                               int n_kv, bool writer, uint32_t sK, uint32_t sV,
+                                               uint32_t sBar, volatile uint32_t* abort) {
+    const TcParams& P = F.t;
+    auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
+    const int lg = P.layer0 + l;
+    const int n_slots = P.req[bl].n_slots;
+    const int o_begin = F.req_occ[bl];
+    const int o_end = F.req_occ[bl + 1];
+    const int pool_row0 = (int)((int64_t)lg * F.pool_slots);
+    const int cache_row0 = (int)((int64_t)lg * P.rows + P.req[bl].row_base);
+    OccWalk wk{}, wv{};
+    if (o_end > o_begin) {
+        walk_load(wk, F, o_begin);
+        wv = wk;
+    }
+    auto tile = [&](int jt, bool is_v, OccWalk& w, uint32_t dst, uint32_t landed) {
+        const CUtensorMap* pool128 = is_v ? &F.tm_pv : &F.tm_pk;
+        const CUtensorMap* cache128 = is_v ? &P.tm_v : &P.tm_k;
+        const CUtensorMap* pool8 = is_v ? &F.tm_pv8 : &F.tm_pk8;
+        const CUtensorMap* cache8 = is_v ? &F.tm_cv8 : &F.tm_ck8;
+        const int R0 = (j_base + jt) * BN;
+        if (R0 >= n_slots) {                                  // the cache's suffix rows
+            mbar_expect_tx(landed, TILE);
+            tma_load_3d(dst, cache128, 0, hk, cache_row0 + R0, landed);
+            tma_load_3d(dst + HALF_TILE, cache128, 64, hk, cache_row0 + R0, landed);
+            return;
+        }
+        walk_to(w, F, R0, o_end);
+        if (w.beg <= R0 && R0 + BN <= w.end && (int64_t)w.src + (R0 - w.beg) + BN <= F.pool_slots &&
+            w.src + (R0 - w.beg) >= 0) {                      // one occurrence
+            const int row = pool_row0 + w.src + (R0 - w.beg);
+            mbar_expect_tx(landed, TILE);
+            tma_load_3d(dst, pool128, 0, hk, row, landed);
+            tma_load_3d(dst + HALF_TILE, pool128, 64, hk, row, landed);
+            return;
+        }
+        // mixed: runs of clean groups whose source rows are contiguous, each moved in boxes of
+        // 64 and 8 rows; the bytes are counted in a first walk, the boxes issued in a second
+        const CUtensorMap* pool64 = is_v ? &F.tm_pv64 : &F.tm_pk64;
+        const CUtensorMap* cache64 = is_v ? &F.tm_cv64 : &F.tm_ck64;
+        auto runs = [&](OccWalk& wr, bool issue) -> int {
+            int groups = 0;
+            int g0 = -1, ng = 0, row0 = 0;
+            bool cache0 = false;
+            auto flush = [&]() {
+                if (ng == 0) return;
+                groups += ng;
+                if (issue) {
+                    int g = g0, left = ng;
+                    while (left > 0) {
+                        const bool big = left >= 8;
+                        const int n = big ? 8 : 1;
+                        const CUtensorMap* tm = cache0 ? (big ? cache64 : cache8) : (big ? pool64 : pool8);
+                        const int row = row0 + 8 * (g - g0);
+                        const uint32_t d = dst + (uint32_t)g * 1024u;
+                        tma_load_3d(d, tm, 0, hk, row, landed);
+                        tma_load_3d(d + HALF_TILE, tm, 64, hk, row, landed);
+                        g += n;
+                        left -= n;
+                    }
+                }
+                ng = 0;
+            };
+            for (int g = 0; g < BN / 8; ++g) {
+                const int R = R0 + 8 * g;
+                bool clean = !group_ragged(wr, F, R, n_slots, o_end);
+                bool is_cache = R >= n_slots;
+                int row = 0;
+                if (clean) {
+                    if (is_cache) {
+                        row = cache_row0 + R;
+                    } else {
+                        const int64_t slot = (int64_t)wr.src + (R - wr.beg);
+                        clean = slot >= 0 && slot + 8 <= F.pool_slots;   // else the loaders report it
+                        row = pool_row0 + (int)slot;
+                    }
+                }
+                if (!clean) {
+                    flush();
+                    continue;
+                }
+                if (ng > 0 && is_cache == cache0 && row == row0 + 8 * ng) {
+                    ++ng;                                     // the run goes on
+                } else {
+                    flush();
+                    g0 = g;
+                    ng = 1;
+                    row0 = row;
+                    cache0 = is_cache;
+                }
+            }
+            flush();
+            return groups;
+        };
+        OccWalk w2 = w;
+        const int clean = runs(w2, false);
+        mbar_expect_tx(landed, (uint32_t)clean * 8u * 256u);
+        runs(w, true);
+    };
+    // a stage is free once the MMA has read it and, in the CTAs that store the composed
+    // rows, once the store of its tile to the cache has read it too
+    auto k_free = [&](int j) {
+        const uint32_t ph = (uint32_t)((j / KSTAGES) - 1) & 1u;
+        return j < KSTAGES || (mbar_try(bar(B_KE + j % KSTAGES), ph) &&
+                               (!writer || mbar_try(bar(B_KW + j % KSTAGES), ph)));
+    };
+    auto v_free = [&](int j) {
+        const uint32_t ph = (uint32_t)((j / VSTAGES) - 1) & 1u;
+        return j < VSTAGES || (mbar_try(bar(B_VE + j % VSTAGES), ph) &&
+                               (!writer || mbar_try(bar(B_VW + j % VSTAGES), ph)));
+    };
+    int jk = 0, jv = 0;
+    while (jk < n_kv || jv < n_kv) {
+        if (jk < n_kv && k_free(jk)) {
+            const int st = jk % KSTAGES;
+            tile(jk, false, wk, sK + (uint32_t)(st * TILE), bar(B_KL + st));
+            ++jk;
+            continue;
+        }
+        if (jv < n_kv && v_free(jv)) {
+            const int st = jv % VSTAGES;
+            tile(jv, true, wv, sV + (uint32_t)(st * TILE), bar(B_VL + st));
+            ++jv;
+            continue;
+        }
+        if (jk < n_kv) {
+            const uint32_t ph = (uint32_t)((jk / KSTAGES) - 1) & 1u;
+            mbar_wait(bar(B_KE + jk % KSTAGES), ph, P.err, abort);
+            if (writer) mbar_wait(bar(B_KW + jk % KSTAGES), ph, P.err, abort);
+        } else {
+            const uint32_t ph = (uint32_t)((jv / VSTAGES) - 1) & 1u;
+            mbar_wait(bar(B_VE + jv % VSTAGES), ph, P.err, abort);
+            if (writer) mbar_wait(bar(B_VW + jv % VSTAGES), ph, P.err, abort);
+        }
+    }
+}
+
+__device__ __forceinline__ void tma_store_3d(const CUtensorMap* tm, uint32_t src, int c0, int c1, int c2) {
+    asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%1, %2, %3}], [%4];" ::"l"(
+                     reinterpret_cast<uint64_t>(tm)),
+                 "r"(c0), "r"(c1), "r"(c2), "r"(src)
+                 : "memory");
+}
+
+// Store a whole 128-row tile (two 64-channel halves) of a stage to the cache by TMA and wait
+// until the store has read shared memory; the stage is then free for the producer.  Tiles
+// with composed slots only: their suffix rows go back unchanged.
+__device__ __forceinline__ void store_tile(const CUtensorMap* tm, uint32_t src, int hk, int row) {
+    tma_store_3d(tm, src, 0, hk, row);
+    tma_store_3d(tm, src + HALF_TILE, 64, hk, row);
+    asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+    asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
+}
+
+// Two pairs turned at once on the packed fp32 pipe: per lane exactly rotate1 (the product
+// rounded, then a fused multiply-add).  x, y: the pairs' two channels; c, s: their cos, sin.
+__device__ __forceinline__ void rotate2(float2 x, float2 y, float2 c, float2 s, float2& ox, float2& oy) {
+    asm("{\n\t.reg .b64 px, py, pc, ps, t, u, a, b;\n\t"
+        "mov.b64 px, {%4, %5};\n\t"
+        "mov.b64 py, {%6, %7};\n\t"
+        "mov.b64 pc, {%8, %9};\n\t"
+        "mov.b64 ps, {%10, %11};\n\t"
+        "mul.rn.f32x2 t, py, ps;\n\t"
+        "xor.b64 t, t, 0x8000000080000000;\n\t"
+        "fma.rn.f32x2 a, px, pc, t;\n\t"
+        "mul.rn.f32x2 u, py, pc;\n\t"
+        "fma.rn.f32x2 b, px, ps, u;\n\t"
+        "mov.b64 {%0, %1}, a;\n\t"
+        "mov.b64 {%2, %3}, b;\n\t}"
+        : "=f"(ox.x), "=f"(ox.y), "=f"(oy.x), "=f"(oy.y)
+        : "f"(x.x), "f"(x.y), "f"(y.x), "f"(y.y), "f"(c.x), "f"(c.y), "f"(s.x), "f"(s.y));
+}
+
+// bf16 pair <-> fp32 pair
+__device__ __forceinline__ float2 bf2_to_f2(uint32_t w) {
+    return make_float2(__uint_as_float(w << 16), __uint_as_float(w & 0xffff0000u));
+}
+__device__ __forceinline__ uint32_t f2_to_bf2(float lo, float hi) {
+    __nv_bfloat162 h = __floats2bfloat162_rn(lo, hi);
+    return *reinterpret_cast<uint32_t*>(&h);
+}
+
+// The K loaders of the fused kernel (warps 12..15, lt = 0..127).  Per key tile, thread lt
+// owns chunk pair kc = lt % 8 (channels 8kc.. and 64+8kc..) of rows lt/8 + 16i: it copies
+// the ragged rows among them (cp.async, 16 bytes a chunk, into the swizzled layout TMA
+// produces), waits for the tile's TMA part, turns its chunks of composed slots by their
+// occurrence's offset (CTAs of pair 0 in layer 0, KV head 0 also write the slots'
+// positions), and releases the stage to the MMA and the K writer.  They wait only for a K
+// stage to be free, so they run up to two tiles ahead of the MMA.
+__device__ __forceinline__ void fused_k_loader(const FusedTcParams& F, int lt, int l, int bl, int hk,
+                                               bool writer, int j_base, int n_kv, uint32_t sK,
+                                               uint32_t sBar, volatile uint32_t* abort) {
+    using bf = __nv_bfloat16;
+    const TcParams& P = F.t;
+    auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
+    const int lg = P.layer0 + l;
+    const int n_slots = P.req[bl].n_slots;
+    const int row_base = P.req[bl].row_base;
+    const int o_begin = F.req_occ[bl];
+    const int o_end = F.req_occ[bl + 1];
+    const int64_t hkv = P.hkv;
+    const int64_t pool_row0 = (int64_t)lg * F.pool_slots;
+    const int64_t cache_row0 = (int64_t)lg * P.rows + row_base;
+    const bf* pk = static_cast<const bf*>(F.pool_k);
+    const bf* ck = static_cast<const bf*>(F.cache_k);
+    const int kc = lt & 7, kr0 = lt >> 3;
+    const bool pos_writer = writer && lg == 0 && hk == 0 && kc == 0;
+    OccWalk wk{}, wr{};
+    if (o_end > o_begin) {
+        walk_load(wk, F, o_begin);
+        wr = wk;
+    }
+    int cs_occ = -1;
+    float2 cc[4], ss[4];      // cos and sin of this thread's 8 frequencies, in pairs
+    // (cos, sin) of the request's occurrences at the 64 frequencies, evaluated once per CTA
+    // into the scratch table (every CTA of the request writes the same values) and read back
+    // as a row per occurrence while turning, instead of evaluating angles per tile
+    for (int e = (o_begin << 6) + lt; e < (o_end << 6); e += kLoaders)
+        F.occ_cs[e] = turn_cs(F.rope.turn[e & 63], F.occ[e >> 6].delta);
+    asm volatile("bar.sync 1, %0;" ::"n"(kLoaders) : "memory");
+
+    for (int jt = 0; jt < n_kv; ++jt) {
+        const int R0 = (j_base + jt) * BN;
+        const int st_i = jt % KSTAGES;
+        const uint32_t st = sK + (uint32_t)(st_i * TILE);
+        if (jt >= KSTAGES)    // stage free: S_A and S_B of tile jt - KSTAGES finished
+            mbar_wait(bar(B_KE + st_i), (uint32_t)((jt / KSTAGES) - 1) & 1u, P.err, abort);
+#pragma unroll 1
+        for (int i = 0; i < BN / 16; ++i) {
+            const int r = kr0 + 16 * i;
+            const int R = R0 + r;
+            if (!group_ragged(wk, F, R, n_slots, o_end)) continue;
+            const bf* src;
+            if (R < n_slots) {
+                const int64_t slot = walk_slot(wk, F, R, o_end);
+                if (slot < 0) continue;
+                src = pk + ((pool_row0 + slot) * hkv + hk) * HD;
+            } else {
+                src = ck + ((cache_row0 + R) * hkv + hk) * HD;
+            }
+            cp_async16(st + sw_off(r, kc), src + 8 * kc);
+            cp_async16(st + HALF_TILE + sw_off(r, kc), src + 64 + 8 * kc);
+        }
+        cp_async_commit();
+        cp_async_wait<0>();
+        mbar_wait(bar(B_KL + st_i), (uint32_t)(jt / KSTAGES) & 1u, P.err, abort);
+#pragma unroll 1
+        for (int i = 0; i < BN / 16; ++i) {
+            const int r = kr0 + 16 * i;
+            const int R = R0 + r;
+            if (R >= n_slots) break;                       // suffix rows are already turned
+            if (walk_slot(wr, F, R, o_end) < 0) continue;
+            if (wr.idx != cs_occ) {
+                const float4* t = reinterpret_cast<const float4*>(F.occ_cs + wr.idx * 64 + 8 * kc);
+#pragma unroll
+                for (int w = 0; w < 4; ++w) {
+                    const float4 v = t[w];                 // (cos, sin) of two frequencies
+                    cc[w] = make_float2(v.x, v.z);
+                    ss[w] = make_float2(v.y, v.w);
+                }
+                cs_occ = wr.idx;
+            }
+            const uint32_t a0 = st + sw_off(r, kc);
+            const uint4 xa = lds128(a0), ya = lds128(a0 + HALF_TILE);
+            const uint32_t xw[4] = {xa.x, xa.y, xa.z, xa.w}, yw[4] = {ya.x, ya.y, ya.z, ya.w};
+            uint32_t xo[4], yo[4];
+#pragma unroll
+            for (int w = 0; w < 4; ++w) {
+                float2 gx, gy;
+                rotate2(bf2_to_f2(xw[w]), bf2_to_f2(yw[w]), cc[w], ss[w], gx, gy);
+                xo[w] = f2_to_bf2(gx.x, gx.y);
+                yo[w] = f2_to_bf2(gy.x, gy.y);
+            }
+            sts128(a0, make_uint4(xo[0], xo[1], xo[2], xo[3]));
+            sts128(a0 + HALF_TILE, make_uint4(yo[0], yo[1], yo[2], yo[3]));
+            if (pos_writer) {
+                const FusedOcc& o = F.occ[wr.idx];
+                F.pos[row_base + R] = o.delta + min((R - o.dest_row + 1) * o.k, o.n) - 1;
+            }
+        }
+        fence_proxy_async();
+        mbar_arrive(bar(B_KF + st_i));
+    }
+}
+
+// The K writer of the fused kernel (warp 2, one thread, CTAs of pair 0): once the K loaders
+// have released a tile that holds composed slots, its K' goes to the cache by TMA.
+__device__ __forceinline__ void fused_k_writer(const FusedTcParams& F, int l, int bl, int hk, int j_base,
+                                               int n_kv, uint32_t sK, uint32_t sBar,
+                                               volatile uint32_t* abort) {
+    const TcParams& P = F.t;
+    auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
+    const int n_slots = P.req[bl].n_slots;
+    const int cache_row0 = (int)((int64_t)(P.layer0 + l) * P.rows + P.req[bl].row_base);
+    for (int jt = 0; jt < n_kv; ++jt) {
+        const int R0 = (j_base + jt) * BN;
+        const int ks = jt % KSTAGES;
+        mbar_wait(bar(B_KF + ks), (uint32_t)(jt / KSTAGES) & 1u, P.err, abort);
+        if (R0 < n_slots) store_tile(&P.tm_k, sK + (uint32_t)(ks * TILE), hk, cache_row0 + R0);
+        mbar_arrive(bar(B_KW + ks));
+    }
+    asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+}
+
+// The V loader of the fused kernel (warp 3, lt = 0..31): per key tile, the ragged 8-row
+// groups' rows by cp.async (thread lt: chunk lt % 16 of rows lt/16 + 2u of each such
+// group), then the tile's TMA part, then the stage is released to the MMA; in the CTAs of
+// pair 0, lane 0 then stores the tile's V to the cache.
+__device__ __forceinline__ void fused_v_loader(const FusedTcParams& F, int lt, int l, int bl, int hk,
+                                               bool writer, int j_base, int n_kv, uint32_t sV,
+                                               uint32_t sBar, volatile uint32_t* abort) {
+    using bf = __nv_bfloat16;
+    const TcParams& P = F.t;
+    auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
+    const int lg = P.layer0 + l;
+    const int n_slots = P.req[bl].n_slots;
+    const int o_begin = F.req_occ[bl];
+    const int o_end = F.req_occ[bl + 1];
+    const int64_t hkv = P.hkv;
+    const int64_t pool_row0 = (int64_t)lg * F.pool_slots;
+    const int64_t cache_row0 = (int64_t)lg * P.rows + P.req[bl].row_base;
+    const bf* pv = static_cast<const bf*>(F.pool_v);
+    const bf* cv = static_cast<const bf*>(F.cache_v);
+    const int vq = lt & 15, vr0 = lt >> 4;
+    OccWalk wv{};
+    if (o_end > o_begin) walk_load(wv, F, o_begin);
+    for (int jt = 0; jt < n_kv; ++jt) {
+        const int R0 = (j_base + jt) * BN;
+        const int st_i = jt % VSTAGES;
+        const uint32_t st = sV + (uint32_t)(st_i * TILE) + (uint32_t)((vq >> 3) * HALF_TILE);
+        if (jt >= VSTAGES)    // stage free: both P.V of tile jt - VSTAGES finished
+            mbar_wait(bar(B_VE + st_i), (uint32_t)((jt / VSTAGES) - 1) & 1u, P.err, abort);
+#pragma unroll 1
+        for (int g = 0; g < BN / 8; ++g) {
+            if (!group_ragged(wv, F, R0 + 8 * g, n_slots, o_end)) continue;
+#pragma unroll 1
+            for (int u = 0; u < 4; ++u) {
+                const int r = 8 * g + vr0 + 2 * u;
+                const int R = R0 + r;
+                const bf* src;
+                if (R < n_slots) {
+                    const int64_t slot = walk_slot(wv, F, R, o_end);
+                    if (slot < 0) continue;
+                    src = pv + ((pool_row0 + slot) * hkv + hk) * HD;
+                } else {
+                    src = cv + ((cache_row0 + R) * hkv + hk) * HD;
+                }
+                cp_async16(st + sw_off(r, vq & 7), src + 8 * vq);
+            }
+        }
+        cp_async_commit();
+        cp_async_wait<0>();
+        mbar_wait(bar(B_VL + st_i), (uint32_t)(jt / VSTAGES) & 1u, P.err, abort);
+        fence_proxy_async();
+        mbar_arrive(bar(B_VF + st_i));
+        if (writer) {         // CTAs of pair 0: the tile's V to the cache
+            __syncwarp();
+            if (lt == 0) {
+                if (R0 < n_slots)
+                    store_tile(&P.tm_v, sV + (uint32_t)(st_i * TILE), hk, (int)cache_row0 + R0);
+                mbar_arrive(bar(B_VW + st_i));
+            }
+        }
+    }
+    if (writer && lt == 0) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+}
+
+template <bool kFused>
+__global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
+    attn_tc_kernel(const __grid_constant__ typename KernelParams<kFused>::type KP) {
+    const TcParams& P = tc_params(KP);
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                                ~uintptr_t(1023));
@@ -536,17 +1039,26 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_const
 
     if (threadIdx.x == 0) {
         mbar_init(bar(B_Q), 1);
+        // a full stage is one TMA arrival (with its byte count), or every loader's arrival
         for (int s = 0; s < KSTAGES; ++s) {
-            mbar_init(bar(B_KF + s), 1);
+            mbar_init(bar(B_KF + s), kFused ? (uint32_t)kLoaders : 1u);
             mbar_init(bar(B_KE + s), 1);
         }
         for (int s = 0; s < VSTAGES; ++s) {
-            mbar_init(bar(B_VF + s), 1);
+            mbar_init(bar(B_VF + s), kFused ? (uint32_t)kVLoaders : 1u);
             mbar_init(bar(B_VE + s), 1);
         }
         for (int i = 0; i < 2; ++i) {
             mbar_init(bar(B_SF + i), 1);
             mbar_init(bar(B_PF + i), 128);
+        }
+        for (int s = 0; s < KSTAGES; ++s) {
+            mbar_init(bar(B_KL + s), 1);
+            mbar_init(bar(B_KW + s), 1);
+        }
+        for (int s = 0; s < VSTAGES; ++s) {
+            mbar_init(bar(B_VL + s), 1);
+            mbar_init(bar(B_VW + s), 1);
         }
         mbar_init(bar(B_OD), 1);
         *abort = 0u;
@@ -565,7 +1077,7 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_const
     const uint32_t tmem = *tmem_slot;
 
     if (warp < 4) {
-        asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsLow));
+        asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kFused ? kRegsLowFused : kRegsLow));
         if (warp == 0 && lane == 0 && n_kv > 0) {
             // ------------------------------------------------------------ TMA producer
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&P.tm_q)) : "memory");
@@ -579,35 +1091,39 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_const
                 tma_load_4d(sQ + TILE, &P.tm_q, 0, hk * G, t0b, qz, bar(B_Q));
                 tma_load_4d(sQ + TILE + HALF_TILE, &P.tm_q, 64, hk * G, t0b, qz, bar(B_Q));
             }
-            const int key0 = (int)((int64_t)(P.layer0 + l) * P.rows + P.req[bl].row_base) + j_base * BN;
-            // two independent queues: a K load waits only for its own K stage
-            int jk = 0, jv = 0;
-            while (jk < n_kv || jv < n_kv) {
-                if (jk < n_kv && (jk < KSTAGES || mbar_try(bar(B_KE + jk % KSTAGES),
-                                                          (uint32_t)((jk / KSTAGES) - 1) & 1u))) {
-                    const int s = jk % KSTAGES;
-                    const int krow = key0 + jk * BN;
-                    mbar_expect_tx(bar(B_KF + s), TILE);
-                    tma_load_3d(sK + s * TILE, &P.tm_k, 0, hk, krow, bar(B_KF + s));
-                    tma_load_3d(sK + s * TILE + HALF_TILE, &P.tm_k, 64, hk, krow, bar(B_KF + s));
-                    ++jk;
-                    continue;
+            if constexpr (kFused) {
+                fused_producer(KP, l, bl, hk, j_base, n_kv, pr == 0, sK, sV, sBar, abort);
+            } else {
+                const int key0 = (int)((int64_t)(P.layer0 + l) * P.rows + P.req[bl].row_base) + j_base * BN;
+                // two independent queues: a K load waits only for its own K stage
+                int jk = 0, jv = 0;
+                while (jk < n_kv || jv < n_kv) {
+                    if (jk < n_kv && (jk < KSTAGES || mbar_try(bar(B_KE + jk % KSTAGES),
+                                                              (uint32_t)((jk / KSTAGES) - 1) & 1u))) {
+                        const int s = jk % KSTAGES;
+                        const int krow = key0 + jk * BN;
+                        mbar_expect_tx(bar(B_KF + s), TILE);
+                        tma_load_3d(sK + s * TILE, &P.tm_k, 0, hk, krow, bar(B_KF + s));
+                        tma_load_3d(sK + s * TILE + HALF_TILE, &P.tm_k, 64, hk, krow, bar(B_KF + s));
+                        ++jk;
+                        continue;
+                    }
+                    if (jv < n_kv && (jv < VSTAGES || mbar_try(bar(B_VE + jv % VSTAGES),
+                                                              (uint32_t)((jv / VSTAGES) - 1) & 1u))) {
+                        const int s = jv % VSTAGES;
+                        const int vrow = key0 + jv * BN;
+                        mbar_expect_tx(bar(B_VF + s), TILE);
+                        tma_load_3d(sV + s * TILE, &P.tm_v, 0, hk, vrow, bar(B_VF + s));
+                        tma_load_3d(sV + s * TILE + HALF_TILE, &P.tm_v, 64, hk, vrow, bar(B_VF + s));
+                        ++jv;
+                        continue;
+                    }
+                    // nothing issuable: wait (bounded) for the stage the next K load needs
+                    if (jk < n_kv)
+                        mbar_wait(bar(B_KE + jk % KSTAGES), (uint32_t)((jk / KSTAGES) - 1) & 1u, P.err, abort);
+                    else
+                        mbar_wait(bar(B_VE + jv % VSTAGES), (uint32_t)((jv / VSTAGES) - 1) & 1u, P.err, abort);
                 }
-                if (jv < n_kv && (jv < VSTAGES || mbar_try(bar(B_VE + jv % VSTAGES),
-                                                          (uint32_t)((jv / VSTAGES) - 1) & 1u))) {
-                    const int s = jv % VSTAGES;
-                    const int vrow = key0 + jv * BN;
-                    mbar_expect_tx(bar(B_VF + s), TILE);
-                    tma_load_3d(sV + s * TILE, &P.tm_v, 0, hk, vrow, bar(B_VF + s));
-                    tma_load_3d(sV + s * TILE + HALF_TILE, &P.tm_v, 64, hk, vrow, bar(B_VF + s));
-                    ++jv;
-                    continue;
-                }
-                // nothing issuable: wait (bounded) for the stage the next K load needs
-                if (jk < n_kv)
-                    mbar_wait(bar(B_KE + jk % KSTAGES), (uint32_t)((jk / KSTAGES) - 1) & 1u, P.err, abort);
-                else
-                    mbar_wait(bar(B_VE + jv % VSTAGES), (uint32_t)((jv / VSTAGES) - 1) & 1u, P.err, abort);
             }
         } else if (warp == 1 && lane == 0 && n_kv > 0) {
             // ------------------------------------------------------------ MMA issuer
@@ -615,14 +1131,29 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_kernel(const __grid_const
                 mma_issuer<true>(P, tmem, sQ, sK, sV, sBar, n_kv, abort);
             else
                 mma_issuer<false>(P, tmem, sQ, sK, sV, sBar, n_kv, abort);
+        } else if (warp == 2 && lane == 0 && n_kv > 0 && pr == 0) {
+            // ------------------------------------------------------------ K writer (fused)
+            if constexpr (kFused) fused_k_writer(KP, l, bl, hk, j_base, n_kv, sK, sBar, abort);
+        } else if (warp == 3 && n_kv > 0) {
+            // ------------------------------------------------------------ V loader (fused)
+            if constexpr (kFused)
+                fused_v_loader(KP, lane, l, bl, hk, pr == 0, j_base, n_kv, sV, sBar, abort);
         }
-    } else {
+    } else if (warp < 12) {
         asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegsHigh));
         // ---------------------------------------------------------------- softmax warps
         const int x = warp >= 8 ? 1 : 0;               // tile A (warps 4..7) or B (8..11)
         if (x == 0 || has_b)
             softmax_tile(P, tmem, sBar, x, warp & 3, lane, x ? t0b : t0a, l, bl, b, hk, sp, j_base,
                          n_kv, abort);
+    } else {
+        if constexpr (kFused) {
+            asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsLowFused));
+            // ------------------------------------------------------------ loaders (fused)
+            if (n_kv > 0)
+                fused_k_loader(KP, (int)threadIdx.x - 12 * 32, l, bl, hk, pr == 0, j_base, n_kv, sK,
+                               sBar, abort);
+        }
     }
 
     tc_fence_before();
@@ -736,12 +1267,19 @@ bool attn_tc_supported(int dtype, int d, int hq, int hkv) {
     return g == 1 || g == 2 || g == 4 || g == 8 || g == 16;
 }
 
-cudaError_t launch_attn_tc(const AttnParams& a, cudaStream_t s, Hook before) {
-    (void)cudaGetLastError();   // report this launch's error only, not a stale one
+namespace {
+
+// Host-side preparation shared by the plain and the fused launch: function attributes once
+// per process, the register-split guard, the tensor maps and the scalar parameters.
+template <bool kFused>
+cudaError_t prepare_tc(const AttnParams& a, TcParams& p, dim3& grid) {
+    constexpr int threads = kFused ? kThreadsFused : kThreads;
+    constexpr int low = kFused ? kRegsLowFused : kRegsLow;
+    constexpr int low_threads = kFused ? 256 : 128;
     cudaError_t e = cudaSuccess;
     static bool smem_set = false;           // once per process (one device per context)
     if (!smem_set) {
-        e = cudaFuncSetAttribute(attn_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        e = cudaFuncSetAttribute(attn_tc_kernel<kFused>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)kSmemBytes);
         if (e != cudaSuccess) return e;
         smem_set = true;
@@ -750,15 +1288,14 @@ cudaError_t launch_attn_tc(const AttnParams& a, cudaStream_t s, Hook before) {
         static int launch_regs = -1;
         if (launch_regs < 0) {
             cudaFuncAttributes fa{};
-            e = cudaFuncGetAttributes(&fa, attn_tc_kernel);
+            e = cudaFuncGetAttributes(&fa, attn_tc_kernel<kFused>);
             if (e != cudaSuccess) return e;
             launch_regs = fa.numRegs;
         }
-        if (launch_regs * kThreads < 128 * kRegsLow + 256 * kRegsHigh) return cudaErrorInvalidConfiguration;
+        if (launch_regs * threads < low_threads * low + 256 * kRegsHigh) return cudaErrorInvalidConfiguration;
     }
     const int pitch = a.sq_pitch > 0 ? a.sq_pitch : a.sq;
     if (pitch < a.sq || (pitch != a.sq && a.n_split > 1)) return cudaErrorInvalidValue;
-    TcParams p;
     std::memset(&p, 0, sizeof(p));
     const int G = a.hq / a.hkv;
     const int tq = BM / G;
@@ -797,14 +1334,98 @@ cudaError_t launch_attn_tc(const AttnParams& a, cudaStream_t s, Hook before) {
     p.n_split = a.n_split < 1 ? 1 : a.n_split;
     p.part_o = a.part_o;
     p.part_lse = a.part_lse;
+    if (a.batch < 1 || a.batch > kMaxReq) return cudaErrorInvalidValue;
     std::memcpy(p.req, a.req, sizeof(ReqParam) * (size_t)a.batch);
     const int64_t pairs = ((a.sq + tq - 1) / tq + 1) / 2;
     const int64_t gx = pairs * p.n_split;
     if (gx > 0x7fffffffLL) return cudaErrorInvalidValue;
-    const dim3 grid((unsigned)gx, a.hkv, a.lq * a.batch);
+    grid = dim3((unsigned)gx, a.hkv, a.lq * a.batch);
     if (grid.z > 65535u || grid.y > 65535u) return cudaErrorInvalidValue;
+    return cudaSuccess;
+}
+
+}  // namespace
+
+cudaError_t launch_attn_tc(const AttnParams& a, cudaStream_t s, Hook before) {
+    (void)cudaGetLastError();   // report this launch's error only, not a stale one
+    TcParams p;
+    dim3 grid;
+    cudaError_t e = prepare_tc<false>(a, p, grid);
+    if (e != cudaSuccess) return e;
     before();
-    attn_tc_kernel<<<grid, kThreads, kSmemBytes, s>>>(p);
+    attn_tc_kernel<false><<<grid, kThreads, kSmemBytes, s>>>(p);
+    return cudaGetLastError();
+}
+
+namespace {
+thread_local FusedTcParams g_fused;          // the prepared launch (18 KB: kept off the stack)
+thread_local dim3 g_fused_grid;
+thread_local bool g_fused_ready = false;
+}  // namespace
+
+cudaError_t prepare_attn_fused(const AttnParams& a, const FusedSpec& f) {
+    (void)cudaGetLastError();
+    g_fused_ready = false;
+    FusedTcParams& p = g_fused;
+    cudaError_t e = prepare_tc<true>(a, p.t, g_fused_grid);
+    if (e != cudaSuccess) return e;
+    if (a.layer0 != 0 || f.req_occ[0] != 0 || f.req_occ[a.batch] > kMaxFusedOcc)
+        return cudaErrorInvalidValue;
+    const int64_t prow = (int64_t)a.lq * f.pool_slots;
+    const int64_t crow = (int64_t)a.lq * a.rows;
+    if (prow > 0x7fffffffLL || crow > 0x7fffffffLL) return cudaErrorInvalidValue;
+    const cuuint64_t str[2] = {(cuuint64_t)HD * 2, (cuuint64_t)a.hkv * HD * 2};
+    const cuuint32_t box128[3] = {64, 1, (cuuint32_t)BN};
+    const cuuint32_t box64[3] = {64, 1, 64};
+    const cuuint32_t box8[3] = {64, 1, 8};
+    {   // pool [L*pool_slots][Hkv][128] in 128-, 64- and 8-row boxes: the pool stays put, so
+        // the maps of the last call are reused while it is the same pool
+        static thread_local const void* key_k = nullptr;
+        static thread_local const void* key_v = nullptr;
+        static thread_local int64_t key_rows = -1, key_hkv = -1;
+        if (key_k != f.pool_k || key_v != f.pool_v || key_rows != prow || key_hkv != a.hkv) {
+            key_k = nullptr;
+            const cuuint64_t pdims[3] = {HD, (cuuint64_t)a.hkv, (cuuint64_t)prow};
+            if (!encode(&p.tm_pk, f.pool_k, 3, pdims, str, box128) ||
+                !encode(&p.tm_pv, f.pool_v, 3, pdims, str, box128) ||
+                !encode(&p.tm_pk64, f.pool_k, 3, pdims, str, box64) ||
+                !encode(&p.tm_pv64, f.pool_v, 3, pdims, str, box64) ||
+                !encode(&p.tm_pk8, f.pool_k, 3, pdims, str, box8) ||
+                !encode(&p.tm_pv8, f.pool_v, 3, pdims, str, box8))
+                return cudaErrorInvalidValue;
+            key_k = f.pool_k;
+            key_v = f.pool_v;
+            key_rows = prow;
+            key_hkv = a.hkv;
+        }
+    }
+    {   // cache [L*rows][Hkv][128] in 64- and 8-row boxes (128-row maps: prepare_tc)
+        const cuuint64_t cdims[3] = {HD, (cuuint64_t)a.hkv, (cuuint64_t)crow};
+        if (!encode(&p.tm_ck64, a.cache_k, 3, cdims, str, box64) ||
+            !encode(&p.tm_cv64, a.cache_v, 3, cdims, str, box64) ||
+            !encode(&p.tm_ck8, a.cache_k, 3, cdims, str, box8) ||
+            !encode(&p.tm_cv8, a.cache_v, 3, cdims, str, box8))
+            return cudaErrorInvalidValue;
+    }
+    p.pool_k = f.pool_k;
+    p.pool_v = f.pool_v;
+    p.cache_k = const_cast<void*>(a.cache_k);
+    p.cache_v = const_cast<void*>(a.cache_v);
+    p.pos = f.pos;
+    p.occ_cs = f.occ_cs;
+    p.pool_slots = f.pool_slots;
+    p.rope = f.rope;
+    std::memcpy(p.req_occ, f.req_occ, sizeof(int32_t) * (size_t)(a.batch + 1));
+    std::memcpy(p.occ, f.occ, sizeof(FusedOcc) * (size_t)f.req_occ[a.batch]);
+    g_fused_ready = true;
+    return cudaSuccess;
+}
+
+cudaError_t launch_attn_fused(cudaStream_t s, Hook before) {
+    if (!g_fused_ready) return cudaErrorInvalidValue;
+    g_fused_ready = false;
+    before();
+    attn_tc_kernel<true><<<g_fused_grid, kThreadsFused, kSmemBytes, s>>>(g_fused);
     return cudaGetLastError();
 }
 

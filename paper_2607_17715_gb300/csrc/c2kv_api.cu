@@ -242,6 +242,8 @@ c2kv_status c2kv_create(const c2kv_config* cfg, void* stream, c2kv_ctx** out) {
             return fail(nullptr, C2KV_ERR_ARG, "create: bad attn_impl");
         if (f.attn_split < 0 || f.attn_split > 16)
             return fail(nullptr, C2KV_ERR_ARG, "create: attn_split outside [0, 16]");
+        if (f.fuse < C2KV_FUSE_AUTO || f.fuse > C2KV_FUSE_ALWAYS)
+            return fail(nullptr, C2KV_ERR_ARG, "create: bad fuse setting");
         if (f.attn_impl == C2KV_ATTN_TC &&
             !c2kv::attn_tc_supported(f.dtype, f.head_dim, f.n_q_heads, f.n_kv_heads))
             return fail(nullptr, C2KV_ERR_UNSUPPORTED,
@@ -454,116 +456,286 @@ c2kv_status c2kv_chunk_info(const c2kv_ctx* c, int32_t id, c2kv_chunk_desc* out)
     return C2KV_OK;
 }
 
+}  // extern "C"
+
+namespace {
+
+// Validates a compose request and lays out its rows: on success `*out` is a new cache with
+// its device buffers allocated (not yet registered with the context) and `occ` holds every
+// occurrence's parameters.  On failure nothing is allocated.
+c2kv_status compose_plan(c2kv_ctx* c, int32_t batch, const int32_t* req_ptr, const int32_t* chunk_ids,
+                         const int32_t* positions, int32_t suffix_capacity, c2kv_cache** out,
+                         std::vector<c2kv::OccParam>& occ) {
+    if (!out || !req_ptr || batch < 1) return fail(c, C2KV_ERR_ARG, "compose: bad batch/out/req_ptr");
+    *out = nullptr;
+    if (suffix_capacity < 0) return fail(c, C2KV_ERR_ARG, "compose: suffix_capacity < 0");
+    if (req_ptr[0] != 0) return fail(c, C2KV_ERR_ARG, "compose: req_ptr[0] != 0");
+    for (int32_t r = 0; r < batch; ++r)
+        if (req_ptr[r + 1] < req_ptr[r]) return fail(c, C2KV_ERR_ARG, "compose: req_ptr decreases");
+    const int32_t n_occ = req_ptr[batch];
+    if (n_occ > 0 && !chunk_ids) return fail(c, C2KV_ERR_ARG, "compose: null chunk_ids");
+
+    // Validate everything and lay out the rows before touching the device.
+    occ.assign((size_t)n_occ, c2kv::OccParam{});
+    auto* cache = new c2kv_cache();
+    cache->owner = c;
+    cache->batch = batch;
+    cache->layers = c->cfg.layers;
+    cache->suffix_capacity = suffix_capacity;
+    cache->row_base.resize(batch);
+    cache->n_slots.resize(batch);
+    cache->l_req.resize(batch);
+    cache->capacity.resize(batch);
+    int64_t row = 0;
+    for (int32_t r = 0; r < batch; ++r) {
+        int64_t slots = 0, prev_end = 0;
+        for (int32_t i = req_ptr[r]; i < req_ptr[r + 1]; ++i) {
+            const int32_t id = chunk_ids[i];
+            if (id < 0 || id >= (int32_t)c->chunks.size() || !c->chunks[id].live) {
+                delete cache;
+                return fail(c, C2KV_ERR_BAD_CHUNK, "compose: unknown chunk %d (occurrence %d)", id, i);
+            }
+            const Chunk& ch = c->chunks[id];
+            const int64_t o = positions ? positions[i] : prev_end;
+            if (o < 0 || o < prev_end) {
+                delete cache;
+                return fail(c, C2KV_ERR_POSITIONS,
+                            "compose: request %d occurrence %d starts at %lld before %lld", r, i,
+                            (long long)o, (long long)prev_end);
+            }
+            prev_end = o + ch.n;
+            if (prev_end > INT32_MAX) {
+                delete cache;
+                return fail(c, C2KV_ERR_POSITIONS, "compose: positions exceed int32");
+            }
+            c2kv::OccParam& rec = occ[i];
+            rec.src_base = ch.base;
+            rec.dest_row = (int32_t)(row + slots);
+            rec.delta = c->cfg.fixed_pos ? 0 : (int32_t)o;
+            rec.n = ch.n;
+            rec.k = ch.k;
+            rec.m = ch.m;
+            rec.tile_base = 0;
+            rec.host = ch.host ? 1 : 0;
+            rec.host_k = ch.host_k;
+            rec.host_v = ch.host_v;
+            slots += ch.m;
+        }
+        const int64_t cap = (slots + suffix_capacity + kTileRows - 1) / kTileRows * kTileRows;
+        if (row + cap > INT32_MAX) {
+            delete cache;
+            return fail(c, C2KV_ERR_ARG, "compose: batch too large");
+        }
+        cache->row_base[r] = (int32_t)row;
+        cache->n_slots[r] = (int32_t)slots;
+        cache->l_req[r] = (int32_t)prev_end;
+        cache->capacity[r] = (int32_t)cap;
+        row += cap;
+    }
+    cache->rows = row;
+    if (c->inject == 1 && n_occ > 0) {
+        occ[0].src_base = c->cfg.pool_slots + 7;   // refused by the kernels' bounds checks
+        c->inject = 0;
+    }
+
+    const size_t kv_bytes = (size_t)c->cfg.layers * (size_t)std::max<int64_t>(row, 1) *
+                            (size_t)row_elems(c) * c->eb;
+    const size_t pos_bytes = (size_t)std::max<int64_t>(row, 1) * sizeof(int32_t);
+    cudaError_t e = pool_alloc(c, &cache->k, kv_bytes);
+    if (e == cudaSuccess) e = pool_alloc(c, &cache->v, kv_bytes);
+    if (e == cudaSuccess) e = pool_alloc(c, reinterpret_cast<void**>(&cache->pos), pos_bytes);
+    if (e != cudaSuccess) {
+        destroy_cache(c, cache);
+        return cuda_fail(c, e, "compose: cache allocation");
+    }
+    *out = cache;
+    return C2KV_OK;
+}
+
+// The compose kernel over every occurrence: one launch per group of at most kMaxOcc
+// occurrences, all layers at once.
+cudaError_t compose_launch(c2kv_ctx* c, const c2kv_cache* cache, const std::vector<c2kv::OccParam>& occ) {
+    const int32_t n_occ = (int32_t)occ.size();
+    cudaError_t e = cudaSuccess;
+    ProfScope prof_compose(c, C2KV_PROF_COMPOSE);
+    for (int32_t g0 = 0; e == cudaSuccess && g0 < n_occ; g0 += c2kv::kMaxOcc) {
+        c2kv::ComposeParams pr{};
+        pr.pool_k = c->pool_k;
+        pr.pool_v = c->pool_v;
+        pr.out_k = cache->k;
+        pr.out_v = cache->v;
+        pr.pos = cache->pos;
+        pr.err = c->d_err;
+        pr.pool_slots = c->cfg.pool_slots;
+        pr.rows = cache->rows;
+        pr.hkv = c->cfg.n_kv_heads;
+        pr.rope = c->turns;
+        int32_t tiles = 0;
+        const int32_t g1 = std::min(n_occ, g0 + c2kv::kMaxOcc);
+        for (int32_t i = g0; i < g1; ++i) {
+            if (occ[i].m == 0) continue;
+            c2kv::OccParam rec = occ[i];
+            rec.tile_base = tiles;
+            pr.occ[pr.n_occ++] = rec;
+            tiles += (rec.m + c2kv::kComposeTile - 1) / c2kv::kComposeTile;
+        }
+        pr.n_tiles = tiles;
+        e = c2kv::launch_compose(pr, c->cfg.dtype, c->cfg.head_dim, c->cfg.layers, c->stream);
+    }
+    return e;
+}
+
+// Checks of an attend call's arguments that do not depend on the cache's contents.
+c2kv_status attend_check(c2kv_ctx* c, const char* what, int32_t layer, const void* q, const void* k_suf,
+                         const void* v_suf, int32_t n_suffix, int32_t suffix_capacity, void* out,
+                         float* lse) {
+    if (!q || !k_suf || !v_suf || !out) return fail(c, C2KV_ERR_ARG, "%s: null pointer", what);
+    if (!aligned(q) || !aligned(k_suf) || !aligned(v_suf) || !aligned(out) || !aligned(lse, 4))
+        return fail(c, C2KV_ERR_ARG, "%s: misaligned tensor pointer", what);
+    if (layer < -1 || layer >= c->cfg.layers) return fail(c, C2KV_ERR_ARG, "%s: bad layer %d", what, layer);
+    if (n_suffix < 1 || n_suffix > suffix_capacity)
+        return fail(c, C2KV_ERR_ARG, "%s: n_suffix %d outside [1, %d]", what, n_suffix, suffix_capacity);
+    return C2KV_OK;
+}
+
+// Suffix preparation and attention of a cache (arguments already checked).  With `fused`,
+// the cache's composed slots are not written yet: the fused kernel reads them from the pool
+// and writes them (tensor-core route, every layer).
+cudaError_t attend_run(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const void* q, const void* k_suf,
+                       const void* v_suf, int32_t n_suffix, void* out, float* lse,
+                       const c2kv::FusedSpec* fused) {
+    const int32_t lq = layer < 0 ? c->cfg.layers : 1;
+    const int32_t layer0 = layer < 0 ? 0 : layer;
+    const int32_t B = cache->batch;
+    const bool use_tc =
+        c->cfg.attn_impl != C2KV_ATTN_SIMT &&
+        c2kv::attn_tc_supported(c->cfg.dtype, c->cfg.head_dim, c->cfg.n_q_heads, c->cfg.n_kv_heads);
+    if (fused && (!use_tc || layer != -1 || B > c2kv::kMaxReq)) return cudaErrorInvalidValue;
+
+    // scratch: the suffix queries after RoPE (the attention kernels' Q operand)
+    const size_t q_bytes = (size_t)lq * B * n_suffix * c->cfg.n_q_heads * c->cfg.head_dim * c->eb;
+    void* q_rot = nullptr;
+    cudaError_t e = pool_alloc(c, &q_rot, q_bytes);
+    if (e != cudaSuccess) return e;
+    // Key-range split of the tensor-core attention: when its work units would leave most
+    // SMs idle (a single layer of a small batch), each unit's key tiles are split and the
+    // partials merged; at a wave or more the split only adds the merge.
+    int32_t n_split = 1;
+    float* part = nullptr;
+    if (use_tc) {
+        const int64_t units = c2kv::attn_tc_units(c->cfg.n_q_heads, c->cfg.n_kv_heads, n_suffix, lq, B);
+        int32_t n_kv_max = 1;
+        for (int32_t b = 0; b < B; ++b)
+            n_kv_max = std::max<int32_t>(n_kv_max, (cache->n_slots[b] + n_suffix + 127) / 128);
+        if (c->cfg.attn_split >= 1) {
+            n_split = c->cfg.attn_split;
+        } else if (2 * units <= c->sms) {
+            // at most half of the SMs would have work: split toward one wave, keeping at
+            // least 8 key tiles per split (below that the merge costs more than it saves)
+            n_split = (int32_t)std::min<int64_t>(16, c->sms / units);
+            n_split = std::max<int32_t>(1, std::min<int32_t>(n_split, n_kv_max / 8));
+        }
+        if (n_split > 1) {
+            const size_t rows = (size_t)lq * B * n_suffix * c->cfg.n_q_heads;
+            e = pool_alloc(c, reinterpret_cast<void**>(&part),
+                           (size_t)n_split * rows * (c->cfg.head_dim + 1) * sizeof(float));
+            if (e != cudaSuccess) {
+                pool_free(c, q_rot);
+                return e;
+            }
+        }
+    }
+    const size_t part_rows = (size_t)lq * B * n_suffix * c->cfg.n_q_heads;
+    c2kv::AttnParams last{};
+    for (int32_t b0 = 0; e == cudaSuccess && b0 < B; b0 += c2kv::kMaxReq) {
+        const int32_t nb = std::min<int32_t>(c2kv::kMaxReq, B - b0);
+        c2kv::SuffixParams s{};
+        s.q = q;
+        s.k = k_suf;
+        s.v = v_suf;
+        s.q_rot = q_rot;
+        s.cache_k = cache->k;
+        s.cache_v = cache->v;
+        s.pos = cache->pos;
+        s.rows = cache->rows;
+        s.layer0 = layer0;
+        s.lq = lq;
+        s.batch = nb;
+        s.batch_total = B;
+        s.b0 = b0;
+        s.sq = n_suffix;
+        s.hq = c->cfg.n_q_heads;
+        s.hkv = c->cfg.n_kv_heads;
+        s.pad_rows = 1;
+        s.rope = c->turns;
+        for (int32_t i = 0; i < nb; ++i)
+            s.req[i] = c2kv::ReqParam{cache->row_base[b0 + i], cache->n_slots[b0 + i],
+                                      cache->l_req[b0 + i], 0};
+        c2kv::AttnParams a{};
+        a.q_rot = q_rot;
+        a.cache_k = cache->k;
+        a.cache_v = cache->v;
+        a.out = out;
+        a.lse = lse;
+        a.err = c->d_err;
+        a.rows = cache->rows;
+        a.layer0 = layer0;
+        a.lq = lq;
+        a.batch = nb;
+        a.batch_total = B;
+        a.b0 = b0;
+        a.sq = n_suffix;
+        a.hq = c->cfg.n_q_heads;
+        a.hkv = c->cfg.n_kv_heads;
+        a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)c->cfg.head_dim));
+        a.n_split = n_split;
+        a.part_o = part;
+        a.part_lse = part ? part + (size_t)n_split * part_rows * c->cfg.head_dim : nullptr;
+        for (int32_t i = 0; i < nb; ++i) a.req[i] = s.req[i];
+        // the fused launch's host work is done before the suffix preparation is enqueued,
+        // so that the kernel follows it on the stream without waiting for the host
+        if (fused) e = c2kv::prepare_attn_fused(a, *fused);
+        if (e != cudaSuccess) break;
+        {
+            ProfScope prof_suffix(c, C2KV_PROF_SUFFIX);
+            e = c2kv::launch_suffix_prep(s, c->cfg.dtype, c->cfg.head_dim, c->stream);
+        }
+        if (e != cudaSuccess) break;
+        if (fused) {
+            ProfScope prof_fused(c, C2KV_PROF_FUSED, true);
+            e = c2kv::launch_attn_fused(c->stream, prof_fused.hook());
+        } else {
+            ProfScope prof_attn(c, C2KV_PROF_ATTN, use_tc);
+            e = use_tc ? c2kv::launch_attn_tc(a, c->stream, prof_attn.hook())
+                       : c2kv::launch_attn_simt(a, c->cfg.dtype, c->cfg.head_dim, c->stream);
+        }
+        last = a;
+    }
+    if (e == cudaSuccess && n_split > 1) {   // one merge over every request's rows
+        ProfScope prof_combine(c, C2KV_PROF_COMBINE);
+        e = c2kv::launch_attn_combine(last, c->stream);
+    }
+    pool_free(c, part);
+    pool_free(c, q_rot);
+    return e;
+}
+
+}  // namespace
+
+extern "C" {
+
 c2kv_status c2kv_compose(c2kv_ctx* c, int32_t batch, const int32_t* req_ptr,
                          const int32_t* chunk_ids, const int32_t* positions,
                          int32_t suffix_capacity, c2kv_cache** out) {
     if (!c) return C2KV_ERR_ARG;
     try {
         c->err.clear();
-        if (!out || !req_ptr || batch < 1) return fail(c, C2KV_ERR_ARG, "compose: bad batch/out/req_ptr");
-        *out = nullptr;
-        if (suffix_capacity < 0) return fail(c, C2KV_ERR_ARG, "compose: suffix_capacity < 0");
-        if (req_ptr[0] != 0) return fail(c, C2KV_ERR_ARG, "compose: req_ptr[0] != 0");
-        for (int32_t r = 0; r < batch; ++r)
-            if (req_ptr[r + 1] < req_ptr[r]) return fail(c, C2KV_ERR_ARG, "compose: req_ptr decreases");
-        const int32_t n_occ = req_ptr[batch];
-        if (n_occ > 0 && !chunk_ids) return fail(c, C2KV_ERR_ARG, "compose: null chunk_ids");
-
-        // Validate everything and lay out the rows before touching the device.
-        std::vector<c2kv::OccParam> occ((size_t)n_occ);
-        auto* cache = new c2kv_cache();
-        cache->owner = c;
-        cache->batch = batch;
-        cache->layers = c->cfg.layers;
-        cache->suffix_capacity = suffix_capacity;
-        cache->row_base.resize(batch);
-        cache->n_slots.resize(batch);
-        cache->l_req.resize(batch);
-        cache->capacity.resize(batch);
-        int64_t row = 0;
-        for (int32_t r = 0; r < batch; ++r) {
-            int64_t slots = 0, prev_end = 0;
-            for (int32_t i = req_ptr[r]; i < req_ptr[r + 1]; ++i) {
-                const int32_t id = chunk_ids[i];
-                if (id < 0 || id >= (int32_t)c->chunks.size() || !c->chunks[id].live) {
-                    delete cache;
-                    return fail(c, C2KV_ERR_BAD_CHUNK, "compose: unknown chunk %d (occurrence %d)", id, i);
-                }
-                const Chunk& ch = c->chunks[id];
-                const int64_t o = positions ? positions[i] : prev_end;
-                if (o < 0 || o < prev_end) {
-                    delete cache;
-                    return fail(c, C2KV_ERR_POSITIONS,
-                                "compose: request %d occurrence %d starts at %lld before %lld", r, i,
-                                (long long)o, (long long)prev_end);
-                }
-                prev_end = o + ch.n;
-                if (prev_end > INT32_MAX) {
-                    delete cache;
-                    return fail(c, C2KV_ERR_POSITIONS, "compose: positions exceed int32");
-                }
-                c2kv::OccParam& rec = occ[i];
-                rec.src_base = ch.base;
-                rec.dest_row = (int32_t)(row + slots);
-                rec.delta = c->cfg.fixed_pos ? 0 : (int32_t)o;
-                rec.n = ch.n;
-                rec.k = ch.k;
-                rec.m = ch.m;
-                rec.tile_base = 0;
-                rec.host = ch.host ? 1 : 0;
-                rec.host_k = ch.host_k;
-                rec.host_v = ch.host_v;
-                slots += ch.m;
-            }
-            const int64_t cap = (slots + suffix_capacity + kTileRows - 1) / kTileRows * kTileRows;
-            if (row + cap > INT32_MAX) {
-                delete cache;
-                return fail(c, C2KV_ERR_ARG, "compose: batch too large");
-            }
-            cache->row_base[r] = (int32_t)row;
-            cache->n_slots[r] = (int32_t)slots;
-            cache->l_req[r] = (int32_t)prev_end;
-            cache->capacity[r] = (int32_t)cap;
-            row += cap;
-        }
-        cache->rows = row;
-        if (c->inject == 1 && n_occ > 0) {
-            occ[0].src_base = c->cfg.pool_slots + 7;   // refused by the kernel's bounds check
-            c->inject = 0;
-        }
-
-        const size_t kv_bytes = (size_t)c->cfg.layers * (size_t)std::max<int64_t>(row, 1) *
-                                (size_t)row_elems(c) * c->eb;
-        const size_t pos_bytes = (size_t)std::max<int64_t>(row, 1) * sizeof(int32_t);
-        cudaError_t e = pool_alloc(c, &cache->k, kv_bytes);
-        if (e == cudaSuccess) e = pool_alloc(c, &cache->v, kv_bytes);
-        if (e == cudaSuccess) e = pool_alloc(c, reinterpret_cast<void**>(&cache->pos), pos_bytes);
-        // One launch per group of at most kMaxOcc occurrences, all layers at once.
-        ProfScope prof_compose(c, C2KV_PROF_COMPOSE);
-        for (int32_t g0 = 0; e == cudaSuccess && g0 < n_occ; g0 += c2kv::kMaxOcc) {
-            c2kv::ComposeParams pr{};
-            pr.pool_k = c->pool_k;
-            pr.pool_v = c->pool_v;
-            pr.out_k = cache->k;
-            pr.out_v = cache->v;
-            pr.pos = cache->pos;
-            pr.err = c->d_err;
-            pr.pool_slots = c->cfg.pool_slots;
-            pr.rows = row;
-            pr.hkv = c->cfg.n_kv_heads;
-            pr.rope = c->turns;
-            int32_t tiles = 0;
-            const int32_t g1 = std::min(n_occ, g0 + c2kv::kMaxOcc);
-            for (int32_t i = g0; i < g1; ++i) {
-                if (occ[i].m == 0) continue;
-                c2kv::OccParam rec = occ[i];
-                rec.tile_base = tiles;
-                pr.occ[pr.n_occ++] = rec;
-                tiles += (rec.m + c2kv::kComposeTile - 1) / c2kv::kComposeTile;
-            }
-            pr.n_tiles = tiles;
-            e = c2kv::launch_compose(pr, c->cfg.dtype, c->cfg.head_dim, c->cfg.layers, c->stream);
-        }
+        std::vector<c2kv::OccParam> occ;
+        c2kv_cache* cache = nullptr;
+        const c2kv_status st =
+            compose_plan(c, batch, req_ptr, chunk_ids, positions, suffix_capacity, &cache, occ);
+        if (st != C2KV_OK) return st;
+        const cudaError_t e = compose_launch(c, cache, occ);
         if (e != cudaSuccess) {
             destroy_cache(c, cache);
             return cuda_fail(c, e, "compose");
@@ -573,6 +745,75 @@ c2kv_status c2kv_compose(c2kv_ctx* c, int32_t batch, const int32_t* req_ptr,
         return C2KV_OK;
     } catch (const std::bad_alloc&) {
         return fail(c, C2KV_ERR_NOMEM, "compose: host allocation failed");
+    }
+}
+
+c2kv_status c2kv_compose_attend(c2kv_ctx* c, int32_t batch, const int32_t* req_ptr,
+                                const int32_t* chunk_ids, const int32_t* positions,
+                                int32_t suffix_capacity, const void* q, const void* k_suf,
+                                const void* v_suf, int32_t n_suffix, void* out, float* lse,
+                                c2kv_cache** cache_out) {
+    if (!c) return C2KV_ERR_ARG;
+    try {
+        c->err.clear();
+        if (!cache_out) return fail(c, C2KV_ERR_ARG, "compose_attend: null cache_out");
+        *cache_out = nullptr;
+        c2kv_status st = attend_check(c, "compose_attend", -1, q, k_suf, v_suf, n_suffix,
+                                      suffix_capacity, out, lse);
+        if (st != C2KV_OK) return st;
+        std::vector<c2kv::OccParam> occ;
+        c2kv_cache* cache = nullptr;
+        st = compose_plan(c, batch, req_ptr, chunk_ids, positions, suffix_capacity, &cache, occ);
+        if (st != C2KV_OK) return st;
+        // The fused kernel takes pool-resident chunks on the tensor-core route, one attention
+        // launch (at most kMaxReq requests) and at most kMaxFusedOcc occurrences; anything
+        // else runs compose and then attention.  By default it runs only when one pair of
+        // query tiles covers each (layer, request, KV head): with more pairs every pair's CTA
+        // would load and turn the same composed tiles (measured slower than composing once).
+        const int64_t q_rows = (int64_t)n_suffix * (c->cfg.n_q_heads / std::max(1, c->cfg.n_kv_heads));
+        bool fuse = c->cfg.fuse != C2KV_FUSE_NEVER &&
+                    (c->cfg.fuse == C2KV_FUSE_ALWAYS || q_rows <= 256) &&
+                    c->cfg.attn_impl != C2KV_ATTN_SIMT &&
+                    c2kv::attn_tc_supported(c->cfg.dtype, c->cfg.head_dim, c->cfg.n_q_heads,
+                                            c->cfg.n_kv_heads) &&
+                    batch <= c2kv::kMaxReq && occ.size() <= (size_t)c2kv::kMaxFusedOcc;
+        for (const auto& o : occ) fuse = fuse && !o.host;
+        cudaError_t e = cudaSuccess;
+        if (fuse) {
+            static thread_local c2kv::FusedSpec f;   // 13 KB: kept off the stack
+            f.pool_k = c->pool_k;
+            f.pool_v = c->pool_v;
+            f.pos = cache->pos;
+            f.pool_slots = c->cfg.pool_slots;
+            f.rope = c->turns;
+            for (int32_t r = 0; r <= batch; ++r) f.req_occ[r] = req_ptr[r];
+            for (size_t i = 0; i < occ.size(); ++i) {
+                const int32_t r = (int32_t)(std::upper_bound(req_ptr, req_ptr + batch + 1, (int32_t)i) -
+                                            req_ptr) - 1;
+                f.occ[i] = c2kv::FusedOcc{occ[i].src_base, occ[i].dest_row - cache->row_base[r],
+                                          occ[i].m, occ[i].delta, occ[i].n, occ[i].k};
+            }
+            float2* occ_cs = nullptr;      // (cos, sin) per occurrence and frequency
+            e = pool_alloc(c, reinterpret_cast<void**>(&occ_cs),
+                           std::max<size_t>(occ.size(), 1) * 64 * sizeof(float2));
+            if (e == cudaSuccess) {
+                f.occ_cs = occ_cs;
+                e = attend_run(c, cache, -1, q, k_suf, v_suf, n_suffix, out, lse, &f);
+                pool_free(c, occ_cs);
+            }
+        } else {
+            e = compose_launch(c, cache, occ);
+            if (e == cudaSuccess) e = attend_run(c, cache, -1, q, k_suf, v_suf, n_suffix, out, lse, nullptr);
+        }
+        if (e != cudaSuccess) {
+            destroy_cache(c, cache);
+            return cuda_fail(c, e, "compose_attend");
+        }
+        c->caches.push_back(cache);
+        *cache_out = cache;
+        return C2KV_OK;
+    } catch (const std::bad_alloc&) {
+        return fail(c, C2KV_ERR_NOMEM, "compose_attend: host allocation failed");
     }
 }
 
@@ -599,118 +840,10 @@ c2kv_status c2kv_attend(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
     try {
         c->err.clear();
         if (!own_cache(c, cache)) return fail(c, C2KV_ERR_STATE, "attend: cache not owned by this context");
-        if (!q || !k_suf || !v_suf || !out) return fail(c, C2KV_ERR_ARG, "attend: null pointer");
-        if (!aligned(q) || !aligned(k_suf) || !aligned(v_suf) || !aligned(out) || !aligned(lse, 4))
-            return fail(c, C2KV_ERR_ARG, "attend: misaligned tensor pointer");
-        if (layer < -1 || layer >= c->cfg.layers) return fail(c, C2KV_ERR_ARG, "attend: bad layer %d", layer);
-        if (n_suffix < 1 || n_suffix > cache->suffix_capacity)
-            return fail(c, C2KV_ERR_ARG, "attend: n_suffix %d outside [1, %d]", n_suffix,
-                        cache->suffix_capacity);
-        const int32_t lq = layer < 0 ? c->cfg.layers : 1;
-        const int32_t layer0 = layer < 0 ? 0 : layer;
-        const int32_t B = cache->batch;
-        const bool use_tc =
-            c->cfg.attn_impl != C2KV_ATTN_SIMT &&
-            c2kv::attn_tc_supported(c->cfg.dtype, c->cfg.head_dim, c->cfg.n_q_heads, c->cfg.n_kv_heads);
-
-        // scratch: the suffix queries after RoPE (the attention kernels' Q operand)
-        const size_t q_bytes =
-            (size_t)lq * B * n_suffix * c->cfg.n_q_heads * c->cfg.head_dim * c->eb;
-        void* q_rot = nullptr;
-        cudaError_t e = pool_alloc(c, &q_rot, q_bytes);
-        if (e != cudaSuccess) return cuda_fail(c, e, "attend: scratch allocation");
-        // Key-range split of the tensor-core attention: when its work units would leave most
-        // SMs idle (a single layer of a small batch), each unit's key tiles are split and the
-        // partials merged; at a wave or more the split only adds the merge.
-        int32_t n_split = 1;
-        float* part = nullptr;
-        if (use_tc) {
-            const int64_t units =
-                c2kv::attn_tc_units(c->cfg.n_q_heads, c->cfg.n_kv_heads, n_suffix, lq, B);
-            int32_t n_kv_max = 1;
-            for (int32_t b = 0; b < B; ++b)
-                n_kv_max = std::max<int32_t>(n_kv_max, (cache->n_slots[b] + n_suffix + 127) / 128);
-            if (c->cfg.attn_split >= 1) {
-                n_split = c->cfg.attn_split;
-            } else if (2 * units <= c->sms) {
-                // at most half of the SMs would have work: split toward one wave, keeping at
-                // least 8 key tiles per split (below that the merge costs more than it saves)
-                n_split = (int32_t)std::min<int64_t>(16, c->sms / units);
-                n_split = std::max<int32_t>(1, std::min<int32_t>(n_split, n_kv_max / 8));
-            }
-            if (n_split > 1) {
-                const size_t rows = (size_t)lq * B * n_suffix * c->cfg.n_q_heads;
-                e = pool_alloc(c, reinterpret_cast<void**>(&part),
-                               (size_t)n_split * rows * (c->cfg.head_dim + 1) * sizeof(float));
-                if (e != cudaSuccess) {
-                    pool_free(c, q_rot);
-                    return cuda_fail(c, e, "attend: split scratch allocation");
-                }
-            }
-        }
-        const size_t part_rows = (size_t)lq * B * n_suffix * c->cfg.n_q_heads;
-        c2kv::AttnParams last{};
-        for (int32_t b0 = 0; e == cudaSuccess && b0 < B; b0 += c2kv::kMaxReq) {
-            const int32_t nb = std::min<int32_t>(c2kv::kMaxReq, B - b0);
-            c2kv::SuffixParams s{};
-            s.q = q;
-            s.k = k_suf;
-            s.v = v_suf;
-            s.q_rot = q_rot;
-            s.cache_k = cache->k;
-            s.cache_v = cache->v;
-            s.pos = cache->pos;
-            s.rows = cache->rows;
-            s.layer0 = layer0;
-            s.lq = lq;
-            s.batch = nb;
-            s.batch_total = B;
-            s.b0 = b0;
-            s.sq = n_suffix;
-            s.hq = c->cfg.n_q_heads;
-            s.hkv = c->cfg.n_kv_heads;
-            s.pad_rows = 1;
-            s.rope = c->turns;
-            for (int32_t i = 0; i < nb; ++i)
-                s.req[i] = c2kv::ReqParam{cache->row_base[b0 + i], cache->n_slots[b0 + i],
-                                          cache->l_req[b0 + i], 0};
-            {
-                ProfScope prof_suffix(c, C2KV_PROF_SUFFIX);
-                e = c2kv::launch_suffix_prep(s, c->cfg.dtype, c->cfg.head_dim, c->stream);
-            }
-            if (e != cudaSuccess) break;
-            c2kv::AttnParams a{};
-            a.q_rot = q_rot;
-            a.cache_k = cache->k;
-            a.cache_v = cache->v;
-            a.out = out;
-            a.lse = lse;
-            a.err = c->d_err;
-            a.rows = cache->rows;
-            a.layer0 = layer0;
-            a.lq = lq;
-            a.batch = nb;
-            a.batch_total = B;
-            a.b0 = b0;
-            a.sq = n_suffix;
-            a.hq = c->cfg.n_q_heads;
-            a.hkv = c->cfg.n_kv_heads;
-            a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)c->cfg.head_dim));
-            a.n_split = n_split;
-            a.part_o = part;
-            a.part_lse = part ? part + (size_t)n_split * part_rows * c->cfg.head_dim : nullptr;
-            for (int32_t i = 0; i < nb; ++i) a.req[i] = s.req[i];
-            ProfScope prof_attn(c, C2KV_PROF_ATTN, use_tc);
-            e = use_tc ? c2kv::launch_attn_tc(a, c->stream, prof_attn.hook())
-                       : c2kv::launch_attn_simt(a, c->cfg.dtype, c->cfg.head_dim, c->stream);
-            last = a;
-        }
-        if (e == cudaSuccess && n_split > 1) {   // one merge over every request's rows
-            ProfScope prof_combine(c, C2KV_PROF_COMBINE);
-            e = c2kv::launch_attn_combine(last, c->stream);
-        }
-        pool_free(c, part);
-        pool_free(c, q_rot);
+        const c2kv_status st =
+            attend_check(c, "attend", layer, q, k_suf, v_suf, n_suffix, cache->suffix_capacity, out, lse);
+        if (st != C2KV_OK) return st;
+        const cudaError_t e = attend_run(c, cache, layer, q, k_suf, v_suf, n_suffix, out, lse, nullptr);
         if (e != cudaSuccess) return cuda_fail(c, e, "attend");
         return C2KV_OK;
     } catch (const std::bad_alloc&) {

@@ -214,9 +214,37 @@ bool attn_tc_supported(int dtype, int d, int hq, int hkv);
 cudaError_t launch_attn_tc(const AttnParams& p, cudaStream_t s, Hook before = {});
 // Merge n_split partial (O, lse) over disjoint key ranges into out (bf16) and lse (attn_tc.cu).
 cudaError_t launch_attn_combine(const AttnParams& p, cudaStream_t s);
-// Work units (CTAs per split) the tensor-core kernel launches for these parameters.
 // CTAs of one tensor-core attention launch before key-range splitting.
 int64_t attn_tc_units(int hq, int hkv, int sq, int lq, int batch);
+
+// Fused compose + attention (attn_tc.cu): the attention reads the composed slots straight
+// from the chunk pool, turns K by its occurrence's offset in shared memory, and writes the
+// composed cache (K', V, positions) as it goes.  The suffix rows must already be in the
+// cache (suffix preparation first).
+struct FusedOcc {
+    int32_t src_row;         // first pool slot of the chunk
+    int32_t dest_row;        // first composed row, relative to the request's row_base
+    int32_t m;               // slots
+    int32_t delta;           // positions to turn by
+    int32_t n;               // original chunk length
+    int32_t k;               // ratio
+};
+constexpr int kMaxFusedOcc = 512;
+struct FusedSpec {
+    const void* pool_k;      // [L][pool_slots][Hkv][128]
+    const void* pool_v;
+    int32_t* pos;            // [rows]
+    float2* occ_cs;          // scratch [occurrences][64]: (cos, sin) of each occurrence's turn,
+                             // filled by the kernel
+    int64_t pool_slots;
+    RopeTurns rope;
+    int32_t req_occ[kMaxReq + 1];   // request i of the launch: occurrences [req_occ[i], req_occ[i+1])
+    FusedOcc occ[kMaxFusedOcc];
+};
+// Host preparation (tensor maps, parameters) of a fused launch, done before the suffix
+// preparation is enqueued so that the kernel follows it without a host gap; then the launch.
+cudaError_t prepare_attn_fused(const AttnParams& a, const FusedSpec& f);
+cudaError_t launch_attn_fused(cudaStream_t s, Hook before = {});
 
 // Read-only view of a context and one of its caches, for entry points defined outside
 // c2kv_api.cu (c2kv_attend_noalloc).

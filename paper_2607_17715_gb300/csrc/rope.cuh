@@ -16,14 +16,19 @@ __device__ __forceinline__ float2 turn_cs(uint64_t turn, int64_t pos) {
     return make_float2(c, s);
 }
 
+// (x, y) turned by the angle whose (cos, sin) is cs, with the rounding spelled out (one
+// product rounded, then a fused multiply-add) so that every kernel that turns a pair gets
+// the same bits.
+__device__ __forceinline__ void rotate1(float x, float y, float2 cs, float& ox, float& oy) {
+    ox = __fmaf_rn(x, cs.x, -__fmul_rn(y, cs.y));
+    oy = __fmaf_rn(x, cs.y, __fmul_rn(y, cs.x));
+}
+
 template <int E>
 __device__ __forceinline__ void rotate(const float* x, const float* y, const float2* cs,
                                        float* ox, float* oy) {
 #pragma unroll
-    for (int e = 0; e < E; ++e) {
-        ox[e] = x[e] * cs[e].x - y[e] * cs[e].y;
-        oy[e] = x[e] * cs[e].y + y[e] * cs[e].x;
-    }
+    for (int e = 0; e < E; ++e) rotate1(x[e], y[e], cs[e], ox[e], oy[e]);
 }
 
 }  // namespace

@@ -1,0 +1,264 @@
+"""Fused compose + attend (c2kv_compose_attend) against the oracle, and against the unfused
+calls it replaces: the output, the normaliser and the whole composed cache it leaves behind
+(turned K within one storage ulp, V and positions bit-exact, suffix rows as attend writes
+them)."""
+import numpy as np
+import pytest
+import torch
+
+import synth
+from oracle import c2kv_oracle as orc
+from tests import _gpu_helpers as H
+
+pytestmark = pytest.mark.gpu
+
+L8B = synth.workload("llama8b")
+
+
+def _run(ctx, wl, dev, reqs, q, ks, vs, sq, fused):
+    """compose_attend (fused=True) or compose + attend; returns (cache, out, lse)."""
+    c2kv = H.lib()
+    B = len(reqs)
+    req_ptr = np.cumsum([0] + [len(ids) for ids, _ in reqs])
+    flat = [dev[c] for ids, _ in reqs for c in ids]
+    offs = [o for _, o_ in reqs for o in o_]
+    qd, kd, vd = (H.to_dev(x, wl) for x in (q, ks, vs))
+    out = torch.full_like(qd, float("nan"))
+    lse = torch.full((wl.layers, B, wl.n_q_heads, sq), float("nan"), device="cuda")
+    if fused:
+        cache = c2kv.c2kv_compose_attend(ctx, req_ptr, flat, offs, sq, qd, kd, vd, sq, out, lse)
+    else:
+        cache = c2kv.c2kv_compose(ctx, req_ptr, flat, offs, suffix_capacity=sq)
+        c2kv.c2kv_attend(ctx, cache, -1, qd, kd, vd, sq, out, lse)
+    c2kv.c2kv_sync(ctx)
+    return cache, out, lse
+
+
+def _fused_case(wl, reqs=None, n_suffix=None, attn_split=0, host=(), fixed_pos=False,
+                compare_unfused=True, fuse=2):
+    """compose_attend with the fused kernel forced (fuse=2) unless it cannot take the call,
+    checked against the oracle and, bit for bit, against compose + attend."""
+    c2kv = H.lib()
+    sq = wl.n_suffix if n_suffix is None else n_suffix
+    wl = synth.scaled(wl, n_suffix=sq)
+    reqs = synth.requests(wl) if reqs is None else reqs
+    all_ids = sorted({c for ids, _ in reqs for c in ids})
+    chunks = H.oracle_chunks_meanpool(wl, all_ids)
+    pool = sum(chunks[c][0].shape[1] for c in all_ids) + 16
+    ctx = H.make_ctx(wl, pool_slots=pool, attn_split=attn_split, fixed_pos=int(fixed_pos),
+                     fuse=fuse)
+    keep = []
+    try:
+        dev = H.load_stored(ctx, wl, chunks, host=host, keep=keep)
+        B = len(reqs)
+        q, ks, vs = synth.suffix(synth.scaled(wl, batch=max(B, wl.batch)), layers=wl.layers)
+        q, ks, vs = q[:, :B], ks[:, :B], vs[:, :B]
+        cache, out, lse = _run(ctx, wl, dev, reqs, q, ks, vs, sq, fused=True)
+        info, gk, gv, gpos = H.cache_arrays(cache, wl)
+        got = out.double().cpu().numpy()
+        got_lse = lse.double().cpu().numpy()
+        for r, (ids, offs) in enumerate(reqs):
+            if ids:
+                ref = orc.run_request(chunks, ids, offs, q[:, r], ks[:, r], vs[:, r],
+                                      wl.rope_theta, wl.dtype, fixed_pos=fixed_pos)
+            else:                              # no composed slot: attention over the suffix
+                none = np.zeros((wl.layers, 0, wl.n_kv_heads, wl.head_dim))
+                o, ls = orc.attend(none, none, 0, q[:, r], ks[:, r], vs[:, r], wl.rope_theta,
+                                   wl.dtype)
+                ref = dict(out=o, lse=ls, l_req=0)
+            H.check_attention(got[:, r], ref["out"], wl, f"O req {r}")
+            assert np.allclose(got_lse[:, r], ref["lse"], atol=1e-3, rtol=1e-4), "lse"
+            base, s = info["row_base"][r], info["n_slots"][r]
+            if ids:
+                ok, ov, opos, _ = orc.compose(chunks, ids, offs, wl.rope_theta, wl.dtype, fixed_pos)
+                assert np.array_equal(gpos[base:base + s], opos)               # bit-exact
+                assert np.array_equal(gv[:, base:base + s], ov)                # bit-exact
+                stored = np.concatenate([chunks[c][0] for c in ids], axis=1)
+                H.check_rotated(gk[:, base:base + s], ok, stored, wl, f"fused cache K req {r}")
+            assert np.array_equal(gpos[base + s: base + s + sq],
+                                  orc.suffix_positions(ref["l_req"], sq))
+            assert np.array_equal(gv[:, base + s: base + s + sq], vs[:, r].astype(np.float64))
+        if compare_unfused:
+            cache_u, out_u, lse_u = _run(ctx, wl, dev, reqs, q, ks, vs, sq, fused=False)
+            info_u, uk, uv, upos = H.cache_arrays(cache_u, wl)
+            # the same stored slots turned by the same arithmetic: the same bits, over every
+            # row either call writes (slots, suffix, and the zeroed rows up to the tile edge)
+            for r in range(B):
+                base, s = info["row_base"][r], info["n_slots"][r]
+                assert info_u["row_base"][r] == base and info_u["n_slots"][r] == s
+                assert np.array_equal(gpos[base:base + s + sq], upos[base:base + s + sq])
+                end = base + (s + sq + 127) // 128 * 128
+                assert np.array_equal(gk[:, base:end], uk[:, base:end])
+                assert np.array_equal(gv[:, base:end], uv[:, base:end])
+            assert torch.equal(out, out_u)
+            assert torch.equal(lse, lse_u)
+            c2kv.c2kv_cache_release(ctx, cache_u)
+        c2kv.c2kv_cache_release(ctx, cache)
+    finally:
+        c2kv.c2kv_destroy(ctx)
+
+
+def test_fused_llama8b_two_layers():
+    # 10 chunks of 128 slots: every key tile comes from one occurrence
+    _fused_case(synth.scaled(L8B, layers=2))
+
+
+def test_fused_gqa8_tiles_across_occurrences():
+    # 64 slots per chunk: every key tile holds two occurrences, each turned by its own offset
+    _fused_case(synth.scaled(synth.workload("long70b"), chunks_per_request=5, pool_chunks=8,
+                             n_suffix=48))
+
+
+def test_fused_batched_duplicates():
+    _fused_case(synth.scaled(synth.workload("batched"), batch=3, chunks_per_request=4,
+                             pool_chunks=32, n_suffix=40))
+
+
+def test_fused_ragged_gaps_and_empty_request():
+    wl = synth.scaled(L8B, layers=2, chunk_tokens=300, ratio_k=10, pool_chunks=4, n_suffix=37)
+    reqs = [([0, 2, 1], [5, 400, 900]),        # gaps between occurrences
+            ([], []),                          # reuses no chunk: every key from the cache
+            ([3, 3], [0, 300]),                # the same chunk twice
+            ([1], [0])]
+    _fused_case(wl, reqs=reqs)
+
+
+def test_fused_uncompressed_long_chunk():
+    # k = 1: 700 slots of one occurrence over six key tiles
+    wl = synth.scaled(L8B, layers=1, chunk_tokens=700, ratio_k=1, chunks_per_request=1,
+                      pool_chunks=1, n_suffix=20)
+    _fused_case(wl)
+
+
+@pytest.mark.parametrize("split", [2, 5])
+def test_fused_key_range_splits(split):
+    wl = synth.scaled(L8B, layers=1, chunk_tokens=512, ratio_k=2, chunks_per_request=3,
+                      pool_chunks=3, n_suffix=70)
+    _fused_case(wl, attn_split=split)
+
+
+def test_fused_fixed_pos():
+    wl = synth.scaled(L8B, layers=1, chunks_per_request=3, pool_chunks=3, n_suffix=16)
+    _fused_case(wl, fixed_pos=True)
+
+
+def test_compose_attend_unfused_routes():
+    # fp32 (CUDA-core attention) and host-resident chunks take compose, then attend
+    _fused_case(synth.workload("tiny_f32"))
+    wl = synth.scaled(L8B, layers=1, chunks_per_request=3, pool_chunks=3, n_suffix=16)
+    _fused_case(wl, host={0, 2})
+
+
+def test_fused_bounds_check_reports_and_recovers():
+    c2kv = H.lib()
+    wl = synth.scaled(L8B, layers=1, chunks_per_request=2, pool_chunks=2, n_suffix=8)
+    reqs = synth.requests(wl)
+    chunks = H.oracle_chunks_meanpool(wl, [0, 1])
+    ctx = H.make_ctx(wl, pool_slots=400)
+    try:
+        dev = H.load_stored(ctx, wl, chunks)
+        q, ks, vs = synth.suffix(wl, layers=1)
+        c2kv.c2kv_inject_fault(ctx, 1)       # the first occurrence points past the pool
+        try:
+            _run(ctx, wl, dev, reqs, q, ks, vs, 8, fused=True)
+        except c2kv.C2KVError as e:
+            assert e.status == c2kv.ERR_DEVICE_BOUNDS
+        else:
+            raise AssertionError("the refused pool row was not reported")
+        # the context still works
+        cache, out, _ = _run(ctx, wl, dev, reqs, q, ks, vs, 8, fused=True)
+        assert torch.isfinite(out.float()).all()
+        c2kv.c2kv_cache_release(ctx, cache)
+    finally:
+        c2kv.c2kv_destroy(ctx)
+
+
+def test_decode_after_fused_matches_unfused():
+    # the cache the fused call leaves behind serves decode exactly as compose + attend's
+    c2kv = H.lib()
+    wl = synth.scaled(L8B, layers=2, chunks_per_request=4, pool_chunks=4, n_suffix=24)
+    reqs = synth.requests(wl)
+    chunks = H.oracle_chunks_meanpool(wl, sorted({c for ids, _ in reqs for c in ids}))
+    ctx = H.make_ctx(wl, pool_slots=1024)
+    try:
+        dev = H.load_stored(ctx, wl, chunks)
+        q, ks, vs = synth.suffix(wl, layers=2)
+        B = len(reqs)
+        req_ptr = np.cumsum([0] + [len(ids) for ids, _ in reqs])
+        flat = [dev[c] for ids, _ in reqs for c in ids]
+        offs = [o for _, o_ in reqs for o in o_]
+        qd, kd, vd = (H.to_dev(x, wl) for x in (q, ks, vs))
+        out = torch.empty_like(qd)
+        gen = torch.Generator(device="cuda").manual_seed(3)
+        qn = torch.randn((2, B, wl.n_q_heads, wl.head_dim), device="cuda", generator=gen).bfloat16()
+        kn = torch.randn((2, B, wl.n_kv_heads, wl.head_dim), device="cuda", generator=gen).bfloat16()
+        vn = torch.randn_like(kn)
+        outs = []
+        for fused in (True, False):
+            if fused:
+                cache = c2kv.c2kv_compose_attend(ctx, req_ptr, flat, offs, 32, qd, kd, vd, 24, out)
+            else:
+                cache = c2kv.c2kv_compose(ctx, req_ptr, flat, offs, suffix_capacity=32)
+                c2kv.c2kv_attend(ctx, cache, -1, qd, kd, vd, 24, out)
+            od = torch.empty_like(qn)
+            c2kv.c2kv_decode(ctx, cache, -1, qn, kn, vn, [24] * B, od)
+            c2kv.c2kv_sync(ctx)
+            outs.append(od)
+            c2kv.c2kv_cache_release(ctx, cache)
+        assert torch.equal(outs[0], outs[1])
+    finally:
+        c2kv.c2kv_destroy(ctx)
+
+
+@pytest.mark.parametrize("n_suffix,fuse,want_fused", [
+    (64, 0, True),        # 64 tokens x 4 heads = 256 query rows: one pair of tiles
+    (65, 0, False),       # a second pair: compose, then attend
+    (65, 2, True),
+    (64, 1, False),
+])
+def test_fuse_policy(n_suffix, fuse, want_fused):
+    c2kv = H.lib()
+    wl = synth.scaled(L8B, layers=1, chunks_per_request=2, pool_chunks=2, n_suffix=n_suffix)
+    reqs = synth.requests(wl)
+    chunks = H.oracle_chunks_meanpool(wl, [0, 1])
+    ctx = H.make_ctx(wl, pool_slots=400, fuse=fuse)
+    try:
+        dev = H.load_stored(ctx, wl, chunks)
+        q, ks, vs = synth.suffix(wl, layers=1)
+        c2kv.c2kv_profile_enable(ctx, True)
+        cache, _, _ = _run(ctx, wl, dev, reqs, q, ks, vs, n_suffix, fused=True)
+        kinds = c2kv.c2kv_profile_read(ctx)
+        assert (kinds["fused"][1] == 1) == want_fused
+        assert (kinds["compose"][1] == 1) == (not want_fused)
+        c2kv.c2kv_cache_release(ctx, cache)
+    finally:
+        c2kv.c2kv_destroy(ctx)
+
+
+def test_compose_attend_arg_checks():
+    c2kv = H.lib()
+    wl = synth.scaled(L8B, layers=1, chunks_per_request=1, pool_chunks=1, n_suffix=4)
+    chunks = H.oracle_chunks_meanpool(wl, [0])
+    ctx = H.make_ctx(wl, pool_slots=200)
+    try:
+        dev = H.load_stored(ctx, wl, chunks)
+        q = torch.zeros((1, 1, 4, wl.n_q_heads, wl.head_dim), device="cuda", dtype=torch.bfloat16)
+        kv = torch.zeros((1, 1, 4, wl.n_kv_heads, wl.head_dim), device="cuda", dtype=torch.bfloat16)
+        out = torch.empty_like(q)
+
+        def status(*a):
+            try:
+                c2kv.c2kv_compose_attend(ctx, *a)
+            except c2kv.C2KVError as e:
+                return e.status
+            return c2kv.OK
+        assert status([0, 1], [dev[0]], [0], 4, q, kv, kv, 5, out) == c2kv.ERR_ARG      # n_suffix > capacity
+        assert status([0, 1], [dev[0]], [0], 4, None, kv, kv, 4, out) == c2kv.ERR_ARG
+        assert status([0, 1], [99], [0], 4, q, kv, kv, 4, out) == c2kv.ERR_BAD_CHUNK
+        assert status([0, 1], [dev[0]], [-1], 4, q, kv, kv, 4, out) == c2kv.ERR_POSITIONS
+        assert status([0, 1], [dev[0]], [0], 4, q.data_ptr() + 2, kv, kv, 4, out) == c2kv.ERR_ARG
+        cache = c2kv.c2kv_compose_attend(ctx, [0, 1], [dev[0]], [0], 4, q, kv, kv, 4, out)
+        c2kv.c2kv_sync(ctx)
+        c2kv.c2kv_cache_release(ctx, cache)
+    finally:
+        c2kv.c2kv_destroy(ctx)
