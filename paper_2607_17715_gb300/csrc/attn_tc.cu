@@ -84,9 +84,11 @@ static_assert(128 * kRegsLow + 256 * kRegsHigh <= kThreads * kLaunchRegs, "regis
 constexpr int kThreadsFused = 512;
 constexpr int kLaunchRegsFused = 128;
 constexpr int kRegsLowFused = 72;
+constexpr int kRegsHighFused = 184;
 constexpr int kLoaders = 128;       // K loaders (warps 12..15)
 constexpr int kVLoaders = 32;       // V loader (warp 3)
-static_assert(256 * kRegsLowFused + 256 * kRegsHigh <= kThreadsFused * kLaunchRegsFused, "fused register split");
+static_assert(256 * kRegsLowFused + 256 * kRegsHighFused <= kThreadsFused * kLaunchRegsFused,
+              "fused register split");
 constexpr uint32_t kTmemCols = 512;     // S_A, S_B, O_A, O_B; P_x over the first half of S_x
 constexpr uint32_t kColS = 0, kColO = 256;
 
@@ -1140,7 +1142,7 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
                 fused_v_loader(KP, lane, l, bl, hk, pr == 0, j_base, n_kv, sV, sBar, abort);
         }
     } else if (warp < 12) {
-        asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kRegsHigh));
+        asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kFused ? kRegsHighFused : kRegsHigh));
         // ---------------------------------------------------------------- softmax warps
         const int x = warp >= 8 ? 1 : 0;               // tile A (warps 4..7) or B (8..11)
         if (x == 0 || has_b)
@@ -1275,6 +1277,7 @@ template <bool kFused>
 cudaError_t prepare_tc(const AttnParams& a, TcParams& p, dim3& grid) {
     constexpr int threads = kFused ? kThreadsFused : kThreads;
     constexpr int low = kFused ? kRegsLowFused : kRegsLow;
+    constexpr int high = kFused ? kRegsHighFused : kRegsHigh;
     constexpr int low_threads = kFused ? 256 : 128;
     cudaError_t e = cudaSuccess;
     static bool smem_set = false;           // once per process (one device per context)
@@ -1292,7 +1295,7 @@ cudaError_t prepare_tc(const AttnParams& a, TcParams& p, dim3& grid) {
             if (e != cudaSuccess) return e;
             launch_regs = fa.numRegs;
         }
-        if (launch_regs * threads < low_threads * low + 256 * kRegsHigh) return cudaErrorInvalidConfiguration;
+        if (launch_regs * threads < low_threads * low + 256 * high) return cudaErrorInvalidConfiguration;
     }
     const int pitch = a.sq_pitch > 0 ? a.sq_pitch : a.sq;
     if (pitch < a.sq || (pitch != a.sq && a.n_split > 1)) return cudaErrorInvalidValue;
