@@ -194,30 +194,25 @@ __global__ void __launch_bounds__(256) compress_kernel(const __grid_constant__ C
 }
 
 // ---------------------------------------------------------------------------------------
-// suffix preparation.  grid = (row blocks of kSuffixRows suffix rows + batch pad blocks,
-// layers).  A row block forms its rows' d/2 (cos, sin) at L_b + t in shared memory, then
-// streams the rows' items (row, head, vector pair): the Hq query heads turned into q_rot,
-// the Hkv key heads turned into the cache row row_base + S_b + t and V copied alongside,
-// IPT items per thread loaded before any is stored.  A pad block zeroes its request's cache
-// rows from the end of the suffix to the next 128-row boundary, so a key tile that straddles
-// the end reads finite zeros (masked keys must not carry NaN/Inf garbage into P.V).
+// suffix preparation.  grid = (batch * Sq suffix rows + batch pad blocks, layers).  A row
+// block forms the row's d/2 (cos, sin) at L_b + t once in shared memory, then turns the
+// Hq query heads into q_rot and the Hkv key heads into the cache row row_base + S_b + t
+// (V copied alongside) for its layer.  A pad block zeroes its request's cache rows from
+// the end of the suffix to the next 128-row boundary, so a key tile that straddles the end
+// reads finite zeros (masked keys must not carry NaN/Inf garbage into P.V).
 // ---------------------------------------------------------------------------------------
-constexpr int kSuffixRows = 8;
-
 template <typename T, int VPH>
 __global__ void __launch_bounds__(256) suffix_kernel(const __grid_constant__ SuffixParams P) {
     using V = Vec16<T>;
     constexpr int E = V::N;
     constexpr int HALF = VPH * E;
     constexpr int D = 2 * HALF;
-    constexpr int IPT = 4;
-    __shared__ float2 cs[kSuffixRows][HALF];
+    __shared__ float2 cs[HALF];
     const int l = blockIdx.y;
     const int n_rows = P.batch * P.sq;
-    const int n_blocks = (n_rows + kSuffixRows - 1) / kSuffixRows;
     const int64_t row_elems = (int64_t)P.hkv * D;
-    if ((int)blockIdx.x >= n_blocks) {
-        const int bl = blockIdx.x - n_blocks;
+    if ((int)blockIdx.x >= n_rows) {
+        const int bl = blockIdx.x - n_rows;
         const int used = P.req[bl].n_slots + P.sq;
         const int end = (used + 127) / 128 * 128;
         constexpr int VPR_ELEMS = 16 / (int)sizeof(T);
@@ -235,83 +230,53 @@ __global__ void __launch_bounds__(256) suffix_kernel(const __grid_constant__ Suf
         }
         return;
     }
-    const int r0 = blockIdx.x * kSuffixRows;
-    const int nr = min(kSuffixRows, n_rows - r0);
-    for (int i = threadIdx.x; i < nr * HALF; i += blockDim.x) {
-        const int rr = i / HALF, f = i - (i / HALF) * HALF;
-        const int bl = (r0 + rr) / P.sq, t = (r0 + rr) - bl * P.sq;
-        const ReqParam& rq = P.req[bl];
-        const int64_t position = (int64_t)rq.l_req + rq.t0 + t;      // suffix index t0 + t
-        cs[rr][f] = turn_cs(P.rope.turn[f], position);
-        if (f == 0 && l == 0) {
-            const int64_t crow = (int64_t)rq.row_base + rq.n_slots + rq.t0 + t;
-            if (crow >= 0 && crow < P.rows) P.pos[crow] = (int32_t)position;
-        }
-    }
+    const int bl = blockIdx.x / P.sq;
+    const int t = blockIdx.x - bl * P.sq;
+    const ReqParam& rq = P.req[bl];
+    const int64_t position = (int64_t)rq.l_req + rq.t0 + t;      // suffix index t0 + t
+    if (threadIdx.x < HALF) cs[threadIdx.x] = turn_cs(P.rope.turn[threadIdx.x], position);
     __syncthreads();
+    const int64_t crow = (int64_t)rq.row_base + rq.n_slots + rq.t0 + t;
+    if (threadIdx.x == 0 && l == 0 && crow >= 0 && crow < P.rows) P.pos[crow] = (int32_t)position;
+    const int64_t grow = ((int64_t)l * P.batch_total + P.b0 + bl) * P.sq + t;  // tensor row
     const int nq = P.hq * VPH;
-    const int per_row = (P.hq + P.hkv) * VPH;
-    const int items = nr * per_row;
-    for (int base = 0; base < items; base += 256 * IPT) {
-        uint4 a[IPT], b[IPT], c[IPT], d[IPT];
-        T* dst[IPT];
-        T* dstv[IPT];
-        int rrs[IPT], ivs[IPT];
-        bool live[IPT], isq[IPT];
-#pragma unroll
-        for (int u = 0; u < IPT; ++u) {
-            const int it = base + u * 256 + (int)threadIdx.x;
-            live[u] = it < items;
-            if (!live[u]) continue;
-            const int rr = it / per_row;
-            const int p = it - rr * per_row;
-            const int row = r0 + rr;
-            const int bl = row / P.sq, t = row - bl * P.sq;
-            const ReqParam& rq = P.req[bl];
-            const int64_t grow = ((int64_t)l * P.batch_total + P.b0 + bl) * P.sq + t;  // tensor row
-            isq[u] = p < nq;
-            const int pp = isq[u] ? p : p - nq;
-            const int h = pp / VPH;
-            const int iv = pp - h * VPH;
-            rrs[u] = rr;
-            ivs[u] = iv;
-            if (isq[u]) {
-                const int64_t off = (grow * P.hq + h) * D + iv * E;
-                const T* src = static_cast<const T*>(P.q) + off;
-                a[u] = ld16(src);
-                b[u] = ld16(src + HALF);
-                dst[u] = static_cast<T*>(P.q_rot) + off;
-            } else {
-                const int64_t crow = (int64_t)rq.row_base + rq.n_slots + rq.t0 + t;
-                if (crow < 0 || crow >= P.rows) {
-                    live[u] = false;
-                    continue;
-                }
-                const int64_t off = (grow * P.hkv + h) * D + iv * E;
-                const int64_t coff = ((int64_t)(P.layer0 + l) * P.rows + crow) * row_elems + h * D + iv * E;
-                const T* ks = static_cast<const T*>(P.k) + off;
-                const T* vs = static_cast<const T*>(P.v) + off;
-                a[u] = ld16(ks);
-                b[u] = ld16(ks + HALF);
-                c[u] = ld16(vs);
-                d[u] = ld16(vs + HALF);
-                dst[u] = static_cast<T*>(P.cache_k) + coff;
-                dstv[u] = static_cast<T*>(P.cache_v) + coff;
-            }
-        }
-#pragma unroll
-        for (int u = 0; u < IPT; ++u) {
-            if (!live[u]) continue;
-            float x[E], y[E], gx[E], gy[E];
-            V::unpack(a[u], x);
-            V::unpack(b[u], y);
-            rotate<E>(x, y, &cs[rrs[u]][ivs[u] * E], gx, gy);
-            st16(dst[u], V::pack(gx));
-            st16(dst[u] + HALF, V::pack(gy));
-            if (!isq[u]) {
-                st16(dstv[u], c[u]);
-                st16(dstv[u] + HALF, d[u]);
-            }
+    const int items = (P.hq + P.hkv) * VPH;
+    for (int p = threadIdx.x; p < items; p += blockDim.x) {
+        const bool is_q = p < nq;
+        const int pp = is_q ? p : p - nq;
+        const int h = pp / VPH;
+        const int iv = pp - h * VPH;
+        float x[E], y[E], gx[E], gy[E];
+        if (is_q) {
+            const int64_t off = (grow * P.hq + h) * D + iv * E;
+            const T* src = static_cast<const T*>(P.q) + off;
+            const uint4 a = ld16(src);
+            const uint4 b = ld16(src + HALF);
+            V::unpack(a, x);
+            V::unpack(b, y);
+            rotate<E>(x, y, cs + iv * E, gx, gy);
+            T* dst = static_cast<T*>(P.q_rot) + off;
+            st16(dst, V::pack(gx));
+            st16(dst + HALF, V::pack(gy));
+        } else {
+            if (crow < 0 || crow >= P.rows) continue;
+            const int64_t off = (grow * P.hkv + h) * D + iv * E;
+            const int64_t coff = ((int64_t)(P.layer0 + l) * P.rows + crow) * row_elems + h * D + iv * E;
+            const T* ks = static_cast<const T*>(P.k) + off;
+            const T* vs = static_cast<const T*>(P.v) + off;
+            const uint4 ka = ld16(ks);
+            const uint4 kb = ld16(ks + HALF);
+            const uint4 va = ld16(vs);
+            const uint4 vb = ld16(vs + HALF);
+            V::unpack(ka, x);
+            V::unpack(kb, y);
+            rotate<E>(x, y, cs + iv * E, gx, gy);
+            T* kd = static_cast<T*>(P.cache_k) + coff;
+            T* vd = static_cast<T*>(P.cache_v) + coff;
+            st16(kd, V::pack(gx));
+            st16(kd + HALF, V::pack(gy));
+            st16(vd, va);
+            st16(vd + HALF, vb);
         }
     }
 }
@@ -363,7 +328,7 @@ cudaError_t launch_compress(const CompressParams& p, int dtype, int d, cudaStrea
 cudaError_t launch_suffix_prep(const SuffixParams& p, int dtype, int d, cudaStream_t s) {
     (void)cudaGetLastError();   // report this launch's error only, not a stale one
     if (p.batch < 1 || p.sq < 1 || p.lq < 1) return cudaSuccess;
-    const int64_t blocks = ((int64_t)p.batch * p.sq + kSuffixRows - 1) / kSuffixRows + (p.pad_rows ? p.batch : 0);
+    const int64_t blocks = (int64_t)p.batch * p.sq + (p.pad_rows ? p.batch : 0);
     if (blocks > 0x7fffffffLL || p.lq > 65535) return cudaErrorInvalidValue;
     const dim3 grid((unsigned)blocks, p.lq);
     C2KV_DISPATCH(suffix_kernel, grid, p, dtype, d, s);
