@@ -221,116 +221,132 @@ __global__ void __launch_bounds__(XNW * 32) extract_attn_kernel(const __grid_con
     }
 }
 
-// Part 3 of the tensor-core route: one warp per (layer, C2 token c_j, KV head).  Lane i
-// holds channels 4i .. 4i+3 of the G query heads; each visible document key (the sink block,
-// then B(j) when j > 0) is one coalesced 256-byte row of K and of V, its G scores are
-// butterfly-summed across the warp, and every lane keeps the same online softmax.  The
-// partial (O_b, lse_b) is merged with part 2's (O_a, lse_a), read from out and the
-// normaliser array, by the exact rule O = (2^lse_a O_a + 2^lse_b O_b) / (2^lse_a + 2^lse_b).
+// Part 3 of the tensor-core route, on the CUDA cores: four threads per (C2 token c_j, query
+// head) pair, each holding 32 of the 128 channels of its query and of its output; a CTA takes
+// 32 pairs (32/G tokens) of one (layer, KV head).  Per visible document key (the sink block,
+// then B(j) when j > 0) the four threads read their 64-byte slices of the K and V rows, the
+// score is summed over the four with two shuffles within the group, and each keeps the same
+// online softmax.  The loads of KB keys are issued before any is used.  The partial
+// (O_b, lse_b) is merged with part 2's (O_a, lse_a), read from out and the normaliser array,
+// by the exact rule O = (2^lse_a O_a + 2^lse_b O_b) / (2^lse_a + 2^lse_b).
 template <int G>
 __global__ void __launch_bounds__(128) extract_local_kernel(const __grid_constant__ ExtractParams P) {
-    constexpr int D = 128;
+    constexpr int D = 128, CH = 32, TPC = 32 / G, KB = 2;
+    using bf = __nv_bfloat16;
     const int lane = threadIdx.x & 31;
+    const int cg = threadIdx.x & 3;                        // channel group: 32cg .. 32cg+31
+    const int pi = threadIdx.x >> 2;                       // pair
+    const int jj = pi / G, g = pi - (pi / G) * G;
     const int m = P.n_all - P.n;
-    const int64_t w = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
-    if (w >= (int64_t)P.lq * m * P.hkv) return;               // warp-uniform
-    const int hk = (int)(w % P.hkv);
-    const int64_t lj = w / P.hkv;
-    const int j = (int)(lj % m);
-    const int l = (int)(lj / m);
+    const int j = blockIdx.x * TPC + jj;
+    const int hk = blockIdx.y, l = blockIdx.z;
+    if (j >= m) return;                                    // the pair's four lanes leave together
+    const unsigned grp = 0xfu << (lane & 28);              // the pair's four lanes
     const int n = P.n, k = P.ratio;
     const int tq = n + j;
+    const int h = hk * G + g;
     const float sc = P.scale_log2;
-
-    using bf = __nv_bfloat16;
-    auto ld4 = [](const bf* p, float* f) {
-        const uint2 u = *reinterpret_cast<const uint2*>(p);
-        const __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162*>(&u.x);
-        const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162*>(&u.y);
-        f[0] = __low2float(a);
-        f[1] = __high2float(a);
-        f[2] = __low2float(b);
-        f[3] = __high2float(b);
-    };
-    float q[G][4];
-    const bf* qr = static_cast<const bf*>(P.q_rot) + (((int64_t)l * P.n_all + tq) * P.hq + hk * G) * D + lane * 4;
+    auto unpack8 = [](const uint4& u, float* f) {
+        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
 #pragma unroll
-    for (int g = 0; g < G; ++g) ld4(qr + g * D, q[g]);
-
+        for (int i = 0; i < 4; ++i) {
+            f[2 * i] = __uint_as_float(w[i] << 16);
+            f[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
+        }
+    };
+    float q[CH];
+    {
+        const uint4* qr = reinterpret_cast<const uint4*>(
+            static_cast<const bf*>(P.q_rot) + (((int64_t)l * P.n_all + tq) * P.hq + h) * D + cg * CH);
+#pragma unroll
+        for (int c = 0; c < 4; ++c) unpack8(qr[c], q + 8 * c);
+    }
     const int sink_end = min(k, n);
     const int lo = j * k, hi = min((j + 1) * k, n);
-    const int nk = j == 0 ? hi - lo : sink_end + (hi - lo);    // B(0) is the sink block
+    const int nk = j == 0 ? hi - lo : sink_end + (hi - lo);     // B(0) is the sink block
     const int64_t kv_stride = (int64_t)P.hkv * D;
-    const bf* kb = static_cast<const bf*>(P.k_rot) + ((int64_t)l * P.n_all * P.hkv + hk) * D + lane * 4;
-    const bf* vb = static_cast<const bf*>(P.v) + ((int64_t)l * P.n_all * P.hkv + hk) * D + lane * 4;
-    float mr[G], lr[G], acc[G][4];
+    const bf* kb = static_cast<const bf*>(P.k_rot) + ((int64_t)l * P.n_all * P.hkv + hk) * D + cg * CH;
+    const bf* vb = static_cast<const bf*>(P.v) + ((int64_t)l * P.n_all * P.hkv + hk) * D + cg * CH;
+    float mr = -CUDART_INF_F, lr = 0.f, acc[CH];
 #pragma unroll
-    for (int g = 0; g < G; ++g) {
-        mr[g] = -CUDART_INF_F;
-        lr[g] = 0.f;
+    for (int c = 0; c < CH; ++c) acc[c] = 0.f;
+    for (int i0 = 0; i0 < nk; i0 += KB) {
+        uint4 kx[KB][4], vx[KB][4];
 #pragma unroll
-        for (int c = 0; c < 4; ++c) acc[g][c] = 0.f;
-    }
-    for (int i = 0; i < nk; ++i) {
-        const int u = j == 0 ? lo + i : (i < sink_end ? i : lo + i - sink_end);
-        float kk[4], vv[4];
-        ld4(kb + u * kv_stride, kk);
-        ld4(vb + u * kv_stride, vv);
-        float s[G];
+        for (int b = 0; b < KB; ++b) {
+            const int i = i0 + b;
+            if (i >= nk) break;
+            const int u = j == 0 ? lo + i : (i < sink_end ? i : lo + i - sink_end);
+            const uint4* kr = reinterpret_cast<const uint4*>(kb + u * kv_stride);
+            const uint4* vr = reinterpret_cast<const uint4*>(vb + u * kv_stride);
 #pragma unroll
-        for (int g = 0; g < G; ++g)
-            s[g] = fmaf(q[g][0], kk[0], fmaf(q[g][1], kk[1], fmaf(q[g][2], kk[2], q[g][3] * kk[3])));
+            for (int c = 0; c < 4; ++c) {
+                kx[b][c] = kr[c];
+                vx[b][c] = vr[c];
+            }
+        }
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1)
+        for (int b = 0; b < KB; ++b) {
+            if (i0 + b >= nk) break;                       // the same for the pair's four lanes
+            float sp[4] = {0.f, 0.f, 0.f, 0.f};            // four independent chains
 #pragma unroll
-            for (int g = 0; g < G; ++g) s[g] += __shfl_xor_sync(0xffffffffu, s[g], o);
+            for (int c = 0; c < 4; ++c) {
+                float kf[8];
+                unpack8(kx[b][c], kf);
 #pragma unroll
-        for (int g = 0; g < G; ++g) {
-            const float sl = s[g] * sc;
-            const float mn = fmaxf(mr[g], sl);
-            const float a = exp2f(mr[g] - mn);                   // 0 on the first key
+                for (int e = 0; e < 8; ++e) sp[c] = fmaf(q[8 * c + e], kf[e], sp[c]);
+            }
+            float s = (sp[0] + sp[1]) + (sp[2] + sp[3]);
+            s += __shfl_xor_sync(grp, s, 1);
+            s += __shfl_xor_sync(grp, s, 2);
+            const float sl = s * sc;
+            const float mn = fmaxf(mr, sl);
+            const float a = exp2f(mr - mn);                // 0 on the first key
             const float pw = exp2f(sl - mn);
-            lr[g] = lr[g] * a + pw;
+            lr = lr * a + pw;
 #pragma unroll
-            for (int c = 0; c < 4; ++c) acc[g][c] = fmaf(pw, vv[c], acc[g][c] * a);
-            mr[g] = mn;
+            for (int c = 0; c < 4; ++c) {
+                float vf[8];
+                unpack8(vx[b][c], vf);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) acc[8 * c + e] = fmaf(pw, vf[e], acc[8 * c + e] * a);
+            }
+            mr = mn;
         }
     }
 
     float* lse_ab = P.lse != nullptr ? P.lse : P.lse_scratch;
-    bf* out = static_cast<bf*>(P.out);
+    const int64_t lse_id = ((int64_t)l * P.hq + h) * P.n_all + tq;
+    const float la = lse_ab[lse_id] * 1.4426950408889634f;   // part 2, natural log -> log2
+    const float lb = mr + log2f(lr);
+    const float mx = fmaxf(la, lb);
+    const float wa = exp2f(la - mx), wb = exp2f(lb - mx);
+    const float inv = 1.f / (wa + wb);
+    const float fa = wa * inv, fb = wb * inv / lr;
+    uint4* orow = reinterpret_cast<uint4*>(static_cast<bf*>(P.out) + (((int64_t)l * P.n_all + tq) * P.hq + h) * D + cg * CH);
 #pragma unroll
-    for (int g = 0; g < G; ++g) {
-        const int h = hk * G + g;
-        const int64_t lse_id = ((int64_t)l * P.hq + h) * P.n_all + tq;
-        const float la = lse_ab[lse_id] * 1.4426950408889634f;   // part 2, natural log -> log2
-        const float lb = mr[g] + log2f(lr[g]);
-        const float mx = fmaxf(la, lb);
-        const float wa = exp2f(la - mx), wb = exp2f(lb - mx);
-        const float inv = 1.f / (wa + wb);
-        const float fb = wb * inv / lr[g];
-        bf* orow = out + (((int64_t)l * P.n_all + tq) * P.hq + h) * D + lane * 4;
-        float oa[4];
-        ld4(orow, oa);
-        __nv_bfloat162 r0 = __floats2bfloat162_rn(fmaf(wa * inv, oa[0], fb * acc[g][0]),
-                                                  fmaf(wa * inv, oa[1], fb * acc[g][1]));
-        __nv_bfloat162 r1 = __floats2bfloat162_rn(fmaf(wa * inv, oa[2], fb * acc[g][2]),
-                                                  fmaf(wa * inv, oa[3], fb * acc[g][3]));
-        uint2 st;
-        st.x = *reinterpret_cast<uint32_t*>(&r0);
-        st.y = *reinterpret_cast<uint32_t*>(&r1);
-        *reinterpret_cast<uint2*>(orow) = st;
-        __syncwarp();                                            // every lane has read lse_a
-        if (P.lse != nullptr && lane == 0) P.lse[lse_id] = (mx + log2f(wa + wb)) * 0.69314718055994531f;
+    for (int c = 0; c < 4; ++c) {
+        float oa[8];
+        unpack8(orow[c], oa);
+        uint32_t w[4];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            __nv_bfloat162 r = __floats2bfloat162_rn(fmaf(fa, oa[2 * e], fb * acc[8 * c + 2 * e]),
+                                                     fmaf(fa, oa[2 * e + 1], fb * acc[8 * c + 2 * e + 1]));
+            w[e] = *reinterpret_cast<uint32_t*>(&r);
+        }
+        orow[c] = make_uint4(w[0], w[1], w[2], w[3]);
     }
+    __syncwarp(grp);                                       // every lane of the pair has read lse_a
+    if (P.lse != nullptr && cg == 0) P.lse[lse_id] = (mx + log2f(wa + wb)) * 0.69314718055994531f;
 }
 
 template <int G>
 cudaError_t launch_local(const ExtractParams& p, cudaStream_t s) {
-    const int64_t warps = (int64_t)p.lq * (p.n_all - p.n) * p.hkv;
-    const int64_t blocks = (warps + 3) / 4;
-    if (blocks > 0x7fffffffLL) return cudaErrorInvalidValue;
-    extract_local_kernel<G><<<(unsigned)blocks, 128, 0, s>>>(p);
+    constexpr int TPC = 32 / G;
+    const dim3 grid((unsigned)((p.n_all - p.n + TPC - 1) / TPC), (unsigned)p.hkv, (unsigned)p.lq);
+    if (grid.x > 0x7fffffffu) return cudaErrorInvalidValue;
+    extract_local_kernel<G><<<grid, 128, 0, s>>>(p);
     return cudaGetLastError();
 }
 
