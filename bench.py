@@ -68,12 +68,19 @@ def describe(wl):
 
 
 def source_digest(paths):
-    """First 16 hex digits of the sha256 of the given source files, concatenated in order."""
+    """First 16 hex digits of the sha256 of the given C++/CUDA source files, concatenated in
+    order, with comments and blank lines removed (so that a comment edit does not count as a
+    change of the kernel)."""
     import hashlib
+    import re
     h = hashlib.sha256()
     for rel in paths:
-        with open(os.path.join(ROOT, rel), "rb") as fh:
-            h.update(fh.read())
+        with open(os.path.join(ROOT, rel), encoding="utf-8") as fh:
+            text = fh.read()
+        text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+        text = re.sub(r"//[^\n]*", "", text)
+        code = "\n".join(line.rstrip() for line in text.splitlines() if line.strip())
+        h.update(code.encode("utf-8"))
     return h.hexdigest()[:16]
 
 

@@ -38,16 +38,18 @@
 // of the error word and carries on, so the kernel always terminates and the host reports
 // C2KV_ERR_DEVICE_BOUNDS at the next c2kv_sync.
 //
-// Fused compose + attention (the same kernel, kFused = true, 512 threads).  Instead of TMA
-// from the composed cache, a fourth warpgroup (warps 12..15, the loaders) fills the K and V
-// rings itself: each composed slot row comes straight from the chunk pool and each suffix
-// row from the cache, one 16-byte cp.async per chunk into the 128-byte-swizzled layout the
-// MMA descriptors expect.  A loader thread then turns the K chunks it copied by their
-// occurrence's offset (the same phase-accumulator angles and fp32 rotation as the compose
-// kernel), and the CTAs of query-tile pair 0 write the turned K', V and the positions of
-// the composed slots to the cache, so the cache is complete for later decode steps.  The
-// pool is read once per (layer, request, KV head) pair and the composed cache is written
-// once, rather than written by compose and read back by attention.
+// Fused compose + attention (the same kernel, kFused = true, 512 threads).  The key tiles
+// come straight from their sources instead of the composed cache: the composed slots from the
+// chunk pool, the suffix rows from the cache.  The TMA producer moves whole tiles of one
+// source, and runs of 8-row groups of one contiguous source in mixed tiles; the rows of
+// groups that straddle a boundary are copied by 16-byte cp.async into the same swizzled
+// layout.  A fourth warpgroup (warps 12..15, the K loaders) turns each composed slot's K in
+// shared memory by its occurrence's offset (the compose kernel's angles and rounding), warp
+// 3 releases the V tiles, and in the CTAs of query-tile pair 0 the turned K' and V go to the
+// cache by TMA stores (warp 2 and warp 3) with the slots' positions, so the cache is
+// complete for later decode steps.  The pool is read once per (layer, request, KV head)
+// pair and the composed cache written once, rather than written by compose and read back by
+// attention.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
