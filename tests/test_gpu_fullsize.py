@@ -1,5 +1,6 @@
 """Full-size parity: every workload at its real size, run the way bench.py runs it (one
-compose launch for all layers and requests, one attend call with layer = -1), checked
+c2kv_compose_attend call for all layers and requests: on llama8b the fused compose +
+attention kernel, elsewhere one compose launch and one attend with layer = -1), checked
 against the oracle on sampled outputs (chosen layers / requests, all of their rows).
 
 llama8b and tiny_f32 run the whole chain from tokens (GPU mean-pool compress -> compose
@@ -17,12 +18,12 @@ from tests import _gpu_helpers as H
 pytestmark = pytest.mark.gpu
 
 
-def _run_full(wl, from_tokens, sample_layers, sample_reqs, seed=0):
+def _run_full(wl, from_tokens, sample_layers, sample_reqs, seed=0, fuse=0):
     c2kv = H.lib()
     reqs = synth.requests(wl, seed)
     pool_ids = sorted({c for ids, _ in reqs for c in ids})
     m = orc.n_slots(wl.chunk_tokens, wl.ratio_k)
-    ctx = H.make_ctx(wl, pool_slots=len(pool_ids) * m + 8)
+    ctx = H.make_ctx(wl, pool_slots=len(pool_ids) * m + 8, fuse=fuse)
     needed = {c for r in sample_reqs for c in reqs[r][0]}
     oracle_chunks = {}
     v_scale = {}        # block mean of |v|: the operand scale of the fp32 mean
@@ -52,12 +53,12 @@ def _run_full(wl, from_tokens, sample_layers, sample_reqs, seed=0):
                                           wl.chunk_tokens, wl.ratio_k)
             torch.cuda.current_stream().synchronize()
         req_ptr = np.cumsum([0] + [len(ids) for ids, _ in reqs])
-        cache = c2kv.c2kv_compose(ctx, req_ptr, [dev[c] for ids, _ in reqs for c in ids],
-                                  [o for _, offs in reqs for o in offs], wl.n_suffix)
         q, ks_, vs_ = synth.suffix(wl, seed)
         qd, kd, vd = (H.to_dev(x, wl) for x in (q, ks_, vs_))
         out = torch.full_like(qd, float("nan"))
-        c2kv.c2kv_attend(ctx, cache, -1, qd, kd, vd, wl.n_suffix, out)
+        cache = c2kv.c2kv_compose_attend(ctx, req_ptr, [dev[c] for ids, _ in reqs for c in ids],
+                                         [o for _, offs in reqs for o in offs], wl.n_suffix,
+                                         qd, kd, vd, wl.n_suffix, out)
         c2kv.c2kv_sync(ctx)
         info = c2kv.c2kv_cache_info(cache)
         shp = (info["layers"], info["rows"], wl.n_kv_heads, wl.head_dim)
@@ -95,11 +96,25 @@ def test_full_tiny_f32():
 
 
 def test_full_llama8b_32_layers():
-    _run_full(synth.workload("llama8b"), True, [0, 13, 31], [0])
+    _run_full(synth.workload("llama8b"), True, [0, 13, 31], [0])            # fused
+
+
+def test_full_llama8b_32_layers_unfused():
+    _run_full(synth.workload("llama8b"), True, [0, 13, 31], [0], fuse=1)   # compose, attend
 
 
 def test_full_batched_zipf():
     _run_full(synth.workload("batched"), False, [0], [0, 7, 15])
+
+
+def test_full_batched_zipf_fused():
+    # the fused kernel forced on 16 requests with two query-tile pairs each
+    _run_full(synth.workload("batched"), False, [0], [0, 7, 15], fuse=2)
+
+
+def test_full_long70b_fused():
+    # the fused kernel forced where every key tile holds two occurrences (64 slots each)
+    _run_full(synth.workload("long70b"), False, [0], [0, 1], fuse=2)
 
 
 def test_full_long70b():
