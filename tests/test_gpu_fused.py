@@ -235,6 +235,35 @@ def test_fuse_policy(n_suffix, fuse, want_fused):
         c2kv.c2kv_destroy(ctx)
 
 
+@pytest.mark.parametrize("n_req,per_req", [(300, 1), (130, 4)])
+def test_compose_attend_many_requests_or_occurrences(n_req, per_req):
+    # more than 256 requests, or more than 512 occurrences: the call composes, then attends
+    # in groups of 256 requests; sampled requests against the oracle
+    c2kv = H.lib()
+    wl = synth.scaled(L8B, layers=1, chunk_tokens=64, ratio_k=4, pool_chunks=5, n_suffix=3,
+                      batch=n_req)
+    chunks = H.oracle_chunks_meanpool(wl, list(range(5)))
+    ctx = H.make_ctx(wl, pool_slots=200, fuse=2)
+    try:
+        dev = H.load_stored(ctx, wl, chunks)
+        rng = np.random.default_rng(5)
+        reqs = []
+        for _ in range(n_req):
+            ids = [int(x) for x in rng.integers(0, 5, per_req)]
+            reqs.append((ids, [64 * i for i in range(per_req)]))
+        q, ks, vs = synth.suffix(wl, layers=1)
+        cache, out, lse = _run(ctx, wl, dev, reqs, q, ks, vs, 3, fused=True)
+        got = out.double().cpu().numpy()
+        for r in (0, 1, n_req // 2, n_req - 1):
+            ids, offs = reqs[r]
+            ref = orc.run_request(chunks, ids, offs, q[:, r], ks[:, r], vs[:, r], wl.rope_theta,
+                                  wl.dtype)
+            H.check_attention(got[:, r], ref["out"], wl, f"O req {r}")
+        c2kv.c2kv_cache_release(ctx, cache)
+    finally:
+        c2kv.c2kv_destroy(ctx)
+
+
 def test_compose_attend_arg_checks():
     c2kv = H.lib()
     wl = synth.scaled(L8B, layers=1, chunks_per_request=1, pool_chunks=1, n_suffix=4)
