@@ -574,7 +574,9 @@ def run_ours(args):
     # end to end from host buffers (host->device traffic inside the timed region), both
     # ways the library offers: zero-copy compose from pinned host slots, and staged copies
     def timed_e2e(step):
-        for _ in range(max(1, args.warmup // 2)):
+        # the first passes over pinned host memory are slower (page walks over the link):
+        # as many warm-up steps as the device step gets
+        for _ in range(max(3, args.warmup)):
             step()
         barrier()
         e0, e1 = E(enable_timing=True), E(enable_timing=True)

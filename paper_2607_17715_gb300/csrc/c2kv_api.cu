@@ -64,6 +64,9 @@ struct c2kv_ctx {
     int32_t inject = 0;
     int sms = 148;
     c2kv::RopeTurns turns{};
+    // second stream and events of the pipelined compose + attend (host-resident chunks)
+    cudaStream_t aux = nullptr;
+    std::vector<cudaEvent_t> aux_ev;
     // tracing (c2kv_profile_enable): event pairs around launches, by kind
     bool prof = false;
     struct ProfRec { int kind; cudaEvent_t a, b; };
@@ -298,6 +301,11 @@ c2kv_status c2kv_destroy(c2kv_ctx* c) {
             cudaEventDestroy(r.b);
         }
         for (cudaEvent_t e : c->prof_free) cudaEventDestroy(e);
+        if (c->aux) {
+            cudaStreamSynchronize(c->aux);
+            cudaStreamDestroy(c->aux);
+        }
+        for (cudaEvent_t e : c->aux_ev) cudaEventDestroy(e);
         if (c->mempool) cudaMemPoolDestroy(c->mempool);
         if (c->pool_k) cudaFree(c->pool_k);
         if (c->pool_v) cudaFree(c->pool_v);
@@ -554,8 +562,10 @@ c2kv_status compose_plan(c2kv_ctx* c, int32_t batch, const int32_t* req_ptr, con
 
 // The compose kernel over every occurrence: one launch per group of at most kMaxOcc
 // occurrences, all layers at once.
-cudaError_t compose_launch(c2kv_ctx* c, const c2kv_cache* cache, const std::vector<c2kv::OccParam>& occ) {
+cudaError_t compose_launch(c2kv_ctx* c, const c2kv_cache* cache, const std::vector<c2kv::OccParam>& occ,
+                           int32_t layer0 = 0, int32_t n_layers = -1, int max_ctas = 0) {
     const int32_t n_occ = (int32_t)occ.size();
+    if (n_layers < 0) n_layers = c->cfg.layers;
     cudaError_t e = cudaSuccess;
     ProfScope prof_compose(c, C2KV_PROF_COMPOSE);
     for (int32_t g0 = 0; e == cudaSuccess && g0 < n_occ; g0 += c2kv::kMaxOcc) {
@@ -569,6 +579,7 @@ cudaError_t compose_launch(c2kv_ctx* c, const c2kv_cache* cache, const std::vect
         pr.pool_slots = c->cfg.pool_slots;
         pr.rows = cache->rows;
         pr.hkv = c->cfg.n_kv_heads;
+        pr.layer0 = layer0;
         pr.rope = c->turns;
         int32_t tiles = 0;
         const int32_t g1 = std::min(n_occ, g0 + c2kv::kMaxOcc);
@@ -580,7 +591,7 @@ cudaError_t compose_launch(c2kv_ctx* c, const c2kv_cache* cache, const std::vect
             tiles += (rec.m + c2kv::kComposeTile - 1) / c2kv::kComposeTile;
         }
         pr.n_tiles = tiles;
-        e = c2kv::launch_compose(pr, c->cfg.dtype, c->cfg.head_dim, c->cfg.layers, c->stream);
+        e = c2kv::launch_compose(pr, c->cfg.dtype, c->cfg.head_dim, n_layers, c->stream, max_ctas);
     }
     return e;
 }
@@ -601,16 +612,15 @@ c2kv_status attend_check(c2kv_ctx* c, const char* what, int32_t layer, const voi
 // Suffix preparation and attention of a cache (arguments already checked).  With `fused`,
 // the cache's composed slots are not written yet: the fused kernel reads them from the pool
 // and writes them (tensor-core route, every layer).
-cudaError_t attend_run(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const void* q, const void* k_suf,
-                       const void* v_suf, int32_t n_suffix, void* out, float* lse,
+cudaError_t attend_run(c2kv_ctx* c, c2kv_cache* cache, int32_t layer0, int32_t lq, const void* q,
+                       const void* k_suf, const void* v_suf, int32_t n_suffix, void* out, float* lse,
                        const c2kv::FusedSpec* fused) {
-    const int32_t lq = layer < 0 ? c->cfg.layers : 1;
-    const int32_t layer0 = layer < 0 ? 0 : layer;
     const int32_t B = cache->batch;
     const bool use_tc =
         c->cfg.attn_impl != C2KV_ATTN_SIMT &&
         c2kv::attn_tc_supported(c->cfg.dtype, c->cfg.head_dim, c->cfg.n_q_heads, c->cfg.n_kv_heads);
-    if (fused && (!use_tc || layer != -1 || B > c2kv::kMaxReq)) return cudaErrorInvalidValue;
+    if (fused && (!use_tc || layer0 != 0 || lq != c->cfg.layers || B > c2kv::kMaxReq))
+        return cudaErrorInvalidValue;
 
     // scratch: the suffix queries after RoPE (the attention kernels' Q operand)
     const size_t q_bytes = (size_t)lq * B * n_suffix * c->cfg.n_q_heads * c->cfg.head_dim * c->eb;
@@ -720,6 +730,70 @@ cudaError_t attend_run(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const void
     return e;
 }
 
+// Makes `c->stream` another stream while it lives (a context is used from one host thread
+// at a time), so that allocations, launches and the trace of a call land on that stream.
+struct StreamSwap {
+    c2kv_ctx* c;
+    cudaStream_t saved;
+    StreamSwap(c2kv_ctx* ctx, cudaStream_t s) : c(ctx), saved(ctx->stream) { c->stream = s; }
+    ~StreamSwap() { c->stream = saved; }
+};
+
+// Compose + attend when chunks are read from host memory: compose is bound by the host link,
+// so the layers go in groups.  The context's stream composes group g with a few CTAs (the
+// link is the limit, and the other SMs stay free), and a second stream runs group g's suffix
+// preparation and attention as soon as its composed rows are in, while group g + 1 is read.
+// The call's work ends on the context's stream, and the second stream first waits for the
+// work enqueued there before the call.
+cudaError_t compose_attend_pipelined(c2kv_ctx* c, c2kv_cache* cache, const std::vector<c2kv::OccParam>& occ,
+                                     const void* q, const void* k_suf, const void* v_suf,
+                                     int32_t n_suffix, void* out, float* lse) {
+    const int32_t L = c->cfg.layers;
+    const int32_t groups = std::min<int32_t>(4, L);
+    const int32_t per = (L + groups - 1) / groups;
+    cudaError_t e = cudaSuccess;
+    if (!c->aux) {
+        e = cudaStreamCreateWithFlags(&c->aux, cudaStreamNonBlocking);
+        if (e != cudaSuccess) {
+            c->aux = nullptr;
+            return e;
+        }
+    }
+    while (c->aux_ev.size() < (size_t)groups + 2) {
+        cudaEvent_t ev = nullptr;
+        e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
+        if (e != cudaSuccess) return e;
+        c->aux_ev.push_back(ev);
+    }
+    const size_t eb = (size_t)c->eb, d = (size_t)c->cfg.head_dim, B = (size_t)cache->batch;
+    const size_t q_layer = B * n_suffix * c->cfg.n_q_heads * d * eb;       // bytes per layer
+    const size_t kv_layer = B * n_suffix * c->cfg.n_kv_heads * d * eb;
+    const size_t lse_layer = B * c->cfg.n_q_heads * n_suffix;              // floats per layer
+    e = cudaEventRecord(c->aux_ev[0], c->stream);                          // the caller's work
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(c->aux, c->aux_ev[0], 0);
+    for (int32_t g = 0; e == cudaSuccess && g < groups; ++g) {
+        const int32_t l0 = g * per;
+        const int32_t nl = std::min(per, L - l0);
+        if (nl <= 0) break;
+        const int max_ctas = std::max(1, c->sms / (4 * nl));                // about a quarter of the SMs
+        e = compose_launch(c, cache, occ, l0, nl, max_ctas);
+        if (e == cudaSuccess) e = cudaEventRecord(c->aux_ev[1 + g], c->stream);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(c->aux, c->aux_ev[1 + g], 0);
+        if (e != cudaSuccess) break;
+        StreamSwap on_aux(c, c->aux);
+        e = attend_run(c, cache, l0, nl, static_cast<const char*>(q) + l0 * q_layer,
+                       static_cast<const char*>(k_suf) + l0 * kv_layer,
+                       static_cast<const char*>(v_suf) + l0 * kv_layer, n_suffix,
+                       static_cast<char*>(out) + l0 * q_layer, lse ? lse + l0 * lse_layer : nullptr,
+                       nullptr);
+    }
+    // the call ends on the context's stream, after everything on the second stream
+    const cudaError_t e2 = cudaEventRecord(c->aux_ev[groups + 1], c->aux);
+    if (e2 == cudaSuccess) cudaStreamWaitEvent(c->stream, c->aux_ev[groups + 1], 0);
+    if (e != cudaSuccess || e2 != cudaSuccess) cudaStreamSynchronize(c->aux);
+    return e != cudaSuccess ? e : e2;
+}
+
 }  // namespace
 
 extern "C" {
@@ -777,7 +851,9 @@ c2kv_status c2kv_compose_attend(c2kv_ctx* c, int32_t batch, const int32_t* req_p
                     c2kv::attn_tc_supported(c->cfg.dtype, c->cfg.head_dim, c->cfg.n_q_heads,
                                             c->cfg.n_kv_heads) &&
                     batch <= c2kv::kMaxReq && occ.size() <= (size_t)c2kv::kMaxFusedOcc;
-        for (const auto& o : occ) fuse = fuse && !o.host;
+        bool host_chunks = false;
+        for (const auto& o : occ) host_chunks = host_chunks || o.host;
+        fuse = fuse && !host_chunks;
         cudaError_t e = cudaSuccess;
         if (fuse) {
             static thread_local c2kv::FusedSpec f;   // 13 KB: kept off the stack
@@ -798,12 +874,15 @@ c2kv_status c2kv_compose_attend(c2kv_ctx* c, int32_t batch, const int32_t* req_p
                            std::max<size_t>(occ.size(), 1) * 64 * sizeof(float2));
             if (e == cudaSuccess) {
                 f.occ_cs = occ_cs;
-                e = attend_run(c, cache, -1, q, k_suf, v_suf, n_suffix, out, lse, &f);
+                e = attend_run(c, cache, 0, c->cfg.layers, q, k_suf, v_suf, n_suffix, out, lse, &f);
                 pool_free(c, occ_cs);
             }
+        } else if (host_chunks && c->cfg.layers >= 2) {
+            e = compose_attend_pipelined(c, cache, occ, q, k_suf, v_suf, n_suffix, out, lse);
         } else {
             e = compose_launch(c, cache, occ);
-            if (e == cudaSuccess) e = attend_run(c, cache, -1, q, k_suf, v_suf, n_suffix, out, lse, nullptr);
+            if (e == cudaSuccess)
+                e = attend_run(c, cache, 0, c->cfg.layers, q, k_suf, v_suf, n_suffix, out, lse, nullptr);
         }
         if (e != cudaSuccess) {
             destroy_cache(c, cache);
@@ -843,7 +922,8 @@ c2kv_status c2kv_attend(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
         const c2kv_status st =
             attend_check(c, "attend", layer, q, k_suf, v_suf, n_suffix, cache->suffix_capacity, out, lse);
         if (st != C2KV_OK) return st;
-        const cudaError_t e = attend_run(c, cache, layer, q, k_suf, v_suf, n_suffix, out, lse, nullptr);
+        const cudaError_t e = attend_run(c, cache, layer < 0 ? 0 : layer, layer < 0 ? c->cfg.layers : 1, q,
+                                         k_suf, v_suf, n_suffix, out, lse, nullptr);
         if (e != cudaSuccess) return cuda_fail(c, e, "attend");
         return C2KV_OK;
     } catch (const std::bad_alloc&) {

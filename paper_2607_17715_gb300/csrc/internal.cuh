@@ -54,7 +54,7 @@ struct ComposeParams {
     int32_t n_occ;
     int32_t n_tiles;
     int32_t hkv;
-    int32_t pad;
+    int32_t layer0;          // layer of grid row 0 (a launch covers layers layer0 .. + gridDim.y)
     RopeTurns rope;
     OccParam occ[kMaxOcc];
 };
@@ -133,7 +133,10 @@ struct AttnParams {
 };
 
 // Launchers: return the launch error, never throw.  `d` is head_dim.
-cudaError_t launch_compose(const ComposeParams& p, int dtype, int d, int layers, cudaStream_t s);
+// max_ctas > 0 caps the CTAs per layer; each then walks several tiles (a compose that reads
+// host-resident chunks is bound by the host link, and leaves the other SMs to attention).
+cudaError_t launch_compose(const ComposeParams& p, int dtype, int d, int layers, cudaStream_t s,
+                           int max_ctas = 0);
 cudaError_t launch_compress(const CompressParams& p, int dtype, int d, cudaStream_t s);
 cudaError_t launch_suffix_prep(const SuffixParams& p, int dtype, int d, cudaStream_t s);
 cudaError_t launch_attn_simt(const AttnParams& p, int dtype, int d, cudaStream_t s);

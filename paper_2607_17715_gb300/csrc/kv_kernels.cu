@@ -19,8 +19,9 @@ namespace {
 // (cos, sin) of pos * theta^(-2i/d) from the 0.64 fixed-point turn of frequency i.
 
 // ---------------------------------------------------------------------------------------
-// compose.  grid = (tiles, layers); a tile is kComposeTile consecutive slots of one chunk
-// occurrence.  The CTA forms the occurrence's d/2 (cos, sin) of delta once in shared
+// compose.  grid = (CTAs per layer, layers); a tile is kComposeTile consecutive slots of one
+// chunk occurrence, and CTA x takes tiles x, x + gridDim.x, ... (one each unless the launch
+// caps its CTAs).  Per tile the CTA forms the occurrence's d/2 (cos, sin) of delta in shared
 // memory, then streams the tile: per item (slot, head, vector pair) four 16-byte loads of
 // stored K/V, K turned, four 16-byte stores into the composed cache.  IPT items per
 // thread are loaded before any is stored, so 16 loads per thread are in flight.
@@ -33,82 +34,83 @@ __global__ void __launch_bounds__(256) compose_kernel(const __grid_constant__ Co
     constexpr int D = 2 * HALF;
     constexpr int IPT = 4;
     __shared__ float2 cs[HALF];
-
-    const int tile = blockIdx.x;
-    const int l = blockIdx.y;
-    int lo = 0, hi = P.n_occ - 1;
-    while (lo < hi) {                       // last occurrence whose tile_base <= tile
-        const int mid = (lo + hi + 1) >> 1;
-        if (P.occ[mid].tile_base <= tile) lo = mid;
-        else hi = mid - 1;
-    }
-    const OccParam& o = P.occ[lo];
-    const int j0 = (tile - o.tile_base) * kComposeTile;
-    const int ns = min(kComposeTile, o.m - j0);
-    if (threadIdx.x < HALF) cs[threadIdx.x] = turn_cs(P.rope.turn[threadIdx.x], o.delta);
-    __syncthreads();
-    if (ns <= 0) return;
-
-    const T* __restrict__ pk = static_cast<const T*>(P.pool_k);
-    const T* __restrict__ pv = static_cast<const T*>(P.pool_v);
-    T* __restrict__ ok = static_cast<T*>(P.out_k);
-    T* __restrict__ ov = static_cast<T*>(P.out_v);
-    const int pairs = P.hkv * VPH;
-    const int items = ns * pairs;
-    const int64_t row_elems = (int64_t)P.hkv * D;
-
-    for (int base = 0; base < items; base += 256 * IPT) {
-        uint4 kx[IPT], ky[IPT], vx[IPT], vy[IPT];
-        int64_t dof[IPT];
-        int civ[IPT];
-        bool live[IPT];
-#pragma unroll
-        for (int u = 0; u < IPT; ++u) {
-            const int it = base + u * 256 + (int)threadIdx.x;
-            live[u] = it < items;
-            if (!live[u]) continue;
-            const int s = it / pairs;
-            const int p = it - s * pairs;
-            const int h = p / VPH;
-            const int iv = p - h * VPH;
-            const int j = j0 + s;
-            const int64_t src = (int64_t)o.src_base + j;
-            const int64_t dst = (int64_t)o.dest_row + j;
-            if ((!o.host && (src < 0 || src >= P.pool_slots)) || dst < 0 || dst >= P.rows) {
-                atomicOr(P.err, 1);
-                live[u] = false;
-                continue;
-            }
-            dof[u] = ((int64_t)l * P.rows + dst) * row_elems + h * D + iv * E;
-            civ[u] = iv * E;
-            const T* sk;
-            const T* sv;
-            if (o.host) {       // host-resident chunk: [L][m][Hkv][d] read over the host link
-                const int64_t so = ((int64_t)l * o.m + j) * row_elems + h * D + iv * E;
-                sk = static_cast<const T*>(o.host_k) + so;
-                sv = static_cast<const T*>(o.host_v) + so;
-            } else {
-                const int64_t so = ((int64_t)l * P.pool_slots + src) * row_elems + h * D + iv * E;
-                sk = pk + so;
-                sv = pv + so;
-            }
-            kx[u] = ld16(sk);
-            ky[u] = ld16(sk + HALF);
-            vx[u] = ld16(sv);
-            vy[u] = ld16(sv + HALF);
-            if (l == 0 && p == 0) P.pos[dst] = o.delta + min((j + 1) * o.k, o.n) - 1;
+    const int l = P.layer0 + (int)blockIdx.y;
+    for (int tile = blockIdx.x; tile < P.n_tiles; tile += gridDim.x) {
+        int lo = 0, hi = P.n_occ - 1;
+        while (lo < hi) {                       // last occurrence whose tile_base <= tile
+            const int mid = (lo + hi + 1) >> 1;
+            if (P.occ[mid].tile_base <= tile) lo = mid;
+            else hi = mid - 1;
         }
-#pragma unroll
-        for (int u = 0; u < IPT; ++u) {
-            if (!live[u]) continue;
-            float fx[E], fy[E], gx[E], gy[E];
-            V::unpack(kx[u], fx);
-            V::unpack(ky[u], fy);
-            rotate<E>(fx, fy, cs + civ[u], gx, gy);
-            st16(ok + dof[u], V::pack(gx));
-            st16(ok + dof[u] + HALF, V::pack(gy));
-            st16(ov + dof[u], vx[u]);
-            st16(ov + dof[u] + HALF, vy[u]);
+        const OccParam& o = P.occ[lo];
+        const int j0 = (tile - o.tile_base) * kComposeTile;
+        const int ns = min(kComposeTile, o.m - j0);
+        __syncthreads();                        // the previous tile is done with cs
+        if (threadIdx.x < HALF) cs[threadIdx.x] = turn_cs(P.rope.turn[threadIdx.x], o.delta);
+        __syncthreads();
+        if (ns <= 0) continue;                  // the same for the whole CTA
+
+        const T* __restrict__ pk = static_cast<const T*>(P.pool_k);
+        const T* __restrict__ pv = static_cast<const T*>(P.pool_v);
+        T* __restrict__ ok = static_cast<T*>(P.out_k);
+        T* __restrict__ ov = static_cast<T*>(P.out_v);
+        const int pairs = P.hkv * VPH;
+        const int items = ns * pairs;
+        const int64_t row_elems = (int64_t)P.hkv * D;
+
+        for (int base = 0; base < items; base += 256 * IPT) {
+            uint4 kx[IPT], ky[IPT], vx[IPT], vy[IPT];
+            int64_t dof[IPT];
+            int civ[IPT];
+            bool live[IPT];
+    #pragma unroll
+            for (int u = 0; u < IPT; ++u) {
+                const int it = base + u * 256 + (int)threadIdx.x;
+                live[u] = it < items;
+                if (!live[u]) continue;
+                const int s = it / pairs;
+                const int p = it - s * pairs;
+                const int h = p / VPH;
+                const int iv = p - h * VPH;
+                const int j = j0 + s;
+                const int64_t src = (int64_t)o.src_base + j;
+                const int64_t dst = (int64_t)o.dest_row + j;
+                if ((!o.host && (src < 0 || src >= P.pool_slots)) || dst < 0 || dst >= P.rows) {
+                    atomicOr(P.err, 1);
+                    live[u] = false;
+                    continue;
+                }
+                dof[u] = ((int64_t)l * P.rows + dst) * row_elems + h * D + iv * E;
+                civ[u] = iv * E;
+                const T* sk;
+                const T* sv;
+                if (o.host) {       // host-resident chunk: [L][m][Hkv][d] read over the host link
+                    const int64_t so = ((int64_t)l * o.m + j) * row_elems + h * D + iv * E;
+                    sk = static_cast<const T*>(o.host_k) + so;
+                    sv = static_cast<const T*>(o.host_v) + so;
+                } else {
+                    const int64_t so = ((int64_t)l * P.pool_slots + src) * row_elems + h * D + iv * E;
+                    sk = pk + so;
+                    sv = pv + so;
+                }
+                kx[u] = ld16(sk);
+                ky[u] = ld16(sk + HALF);
+                vx[u] = ld16(sv);
+                vy[u] = ld16(sv + HALF);
+                if (l == 0 && p == 0) P.pos[dst] = o.delta + min((j + 1) * o.k, o.n) - 1;
+            }
+    #pragma unroll
+            for (int u = 0; u < IPT; ++u) {
+                if (!live[u]) continue;
+                float fx[E], fy[E], gx[E], gy[E];
+                V::unpack(kx[u], fx);
+                V::unpack(ky[u], fy);
+                rotate<E>(fx, fy, cs + civ[u], gx, gy);
+                st16(ok + dof[u], V::pack(gx));
+                st16(ok + dof[u] + HALF, V::pack(gy));
+                st16(ov + dof[u], vx[u]);
+                st16(ov + dof[u] + HALF, vy[u]);
+            }
         }
     }
 }
@@ -307,11 +309,12 @@ int vph_of(int dtype, int d) { return d / 2 / (dtype == kDtypeBf16 ? 8 : 4); }
         else return cudaErrorInvalidValue;                                                     \
     } while (0)
 
-cudaError_t launch_compose(const ComposeParams& p, int dtype, int d, int layers, cudaStream_t s) {
+cudaError_t launch_compose(const ComposeParams& p, int dtype, int d, int layers, cudaStream_t s,
+                           int max_ctas) {
     if (p.n_tiles == 0 || p.n_occ == 0) return cudaSuccess;
     (void)cudaGetLastError();   // report this launch's error only, not a stale one
     if (layers > 65535) return cudaErrorInvalidValue;
-    const dim3 grid(p.n_tiles, layers);
+    const dim3 grid(max_ctas > 0 && max_ctas < p.n_tiles ? max_ctas : p.n_tiles, layers);
     C2KV_DISPATCH(compose_kernel, grid, p, dtype, d, s);
     return cudaGetLastError();
 }

@@ -149,6 +149,15 @@ def test_compose_attend_unfused_routes():
     _fused_case(wl, host={0, 2})
 
 
+@pytest.mark.parametrize("layers", [2, 5])
+def test_compose_attend_host_chunks_pipelined(layers):
+    # host-resident chunks over several layers: composed in layer groups while the previous
+    # group attends on a second stream; the same bits as compose + attend
+    wl = synth.scaled(L8B, layers=layers, chunks_per_request=3, pool_chunks=3, n_suffix=20)
+    _fused_case(wl, host={0, 1, 2})
+    _fused_case(synth.scaled(wl, batch=2, chunks_per_request=2, pool_chunks=4), host={1, 3})
+
+
 def test_fused_bounds_check_reports_and_recovers():
     c2kv = H.lib()
     wl = synth.scaled(L8B, layers=1, chunks_per_request=2, pool_chunks=2, n_suffix=8)
