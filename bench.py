@@ -49,9 +49,10 @@ def workload_facts(wl):
     # attention bytes: every cache row (slots + suffix) read once, Q read, O written
     attn_bytes = wl.layers * wl.batch * ((S + sq) * row_bytes * 2
                                          + 2 * sq * wl.n_q_heads * wl.head_dim * eb)
-    # fused compose + attention: every stored slot read and its composed row written once
-    # (compose's bytes), the suffix rows and Q read, O written; the cache is not read back
-    fused_bytes = compose_bytes + wl.layers * wl.batch * (sq * row_bytes * 2
+    # fused compose + suffix preparation + attention (one kernel): every stored slot read and
+    # its composed row written once (compose's bytes), the suffix rows read and written to the
+    # cache once, Q read, O written; the cache is not read back
+    fused_bytes = compose_bytes + wl.layers * wl.batch * (2 * sq * row_bytes * 2
                                                           + 2 * sq * wl.n_q_heads * wl.head_dim * eb)
     return dict(name=wl.name, slots=S, span=span, positions=wl.batch * span, row_bytes=row_bytes, dtype=wl.dtype,
                 compose_bytes=compose_bytes, attn_flops=attn_flops, attn_bytes=attn_bytes,
@@ -155,8 +156,8 @@ def step_rooflines(fused_ran, kern, kc_ms, ka_ms, f, hbm, bf16, src):
 
 
 def fused_roofline(fused_ms, f, hbm, bf16, src):
-    """The fused compose + attention kernel: HBM-bound (its intensity, attention flops over
-    fused bytes, is far below the ridge); both fractions carried."""
+    """The fused compose + suffix preparation + attention kernel: HBM-bound (its intensity,
+    attention flops over fused bytes, is far below the ridge); both fractions carried."""
     gbs = f["fused_bytes"] / (fused_ms / 1e3) / 1e9
     tfs = f["attn_flops"] / (fused_ms / 1e3) / 1e12
     return {"bound": "hbm", "kernel": "attn_tc_kernel<fused>",
@@ -633,7 +634,8 @@ def run_ours(args):
                    "l2": "flushed between timed steps (256 MB write, untimed)",
                    "global_batch": wl.batch * world,
                    "ttft_proxy_ms_per_layer": round(kc_ms / wl.layers, 6),
-                   "step": ("c2kv_compose_attend: fused compose + attention kernel" if fused_ran
+                   "step": ("c2kv_compose_attend: one kernel (compose, suffix preparation and "
+                            "attention fused)" if fused_ran
                             else "c2kv_compose_attend: compose, then attention"),
                    "kernel_ms": step_kernels,
                    "unfused": {"value": round(positions / (un_total_ms / 1e3), 1),

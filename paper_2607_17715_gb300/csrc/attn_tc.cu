@@ -38,18 +38,21 @@
 // of the error word and carries on, so the kernel always terminates and the host reports
 // C2KV_ERR_DEVICE_BOUNDS at the next c2kv_sync.
 //
-// Fused compose + attention (the same kernel, kFused = true, 512 threads).  The key tiles
-// come straight from their sources instead of the composed cache: the composed slots from the
-// chunk pool, the suffix rows from the cache.  The TMA producer moves whole tiles of one
-// source, and runs of 8-row groups of one contiguous source in mixed tiles; the rows of
-// groups that straddle a boundary are copied by 16-byte cp.async into the same swizzled
-// layout.  A fourth warpgroup (warps 12..15, the K loaders) turns each composed slot's K in
-// shared memory by its occurrence's offset (the compose kernel's angles and rounding), warp
-// 3 releases the V tiles, and in the CTAs of query-tile pair 0 the turned K' and V go to the
-// cache by TMA stores (warp 2 and warp 3) with the slots' positions, so the cache is
-// complete for later decode steps.  The pool is read once per (layer, request, KV head)
-// pair and the composed cache written once, rather than written by compose and read back by
-// attention.
+// Fused compose + suffix preparation + attention (the same kernel, kFused = true, 512
+// threads, the whole step in one launch).  The key tiles come straight from their sources
+// instead of the composed cache: the composed slots from the chunk pool, the suffix rows from
+// the caller's k_suf / v_suf.  The TMA producer moves whole tiles of one source, and runs of
+// 8-row groups of one contiguous source in mixed tiles; the rows of groups that straddle a
+// boundary are copied by 16-byte cp.async into the same swizzled layout, and rows past the
+// suffix are zeroed.  A fourth warpgroup (warps 12..15, the K loaders) turns each composed
+// slot's K in shared memory by its occurrence's offset and each suffix row's K by its
+// token's position (the compose and suffix kernels' angles and rounding), warp 3 releases
+// the V tiles, and the softmax warps, idle until the first S tile, turn the Q tiles in
+// shared memory.  In the CTAs of the last query-tile pair (the one whose causal range covers
+// the whole suffix) the turned K' and V go to the cache by TMA stores (warp 2 and warp 3)
+// with the rows' positions, so the cache is complete for later decode steps.  The pool is
+// read once per (layer, request, KV head) and the composed cache written once, rather than
+// written by compose and read back by attention.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -107,7 +110,8 @@ constexpr int B_KL = B_OD + 1;           // + stage (fused): the TMA part of a K
 constexpr int B_VL = B_KL + KSTAGES;     // + stage (fused): the TMA part of a V tile landed
 constexpr int B_KW = B_VL + VSTAGES;     // + stage (fused): K' of the stage's tile stored to the cache
 constexpr int B_VW = B_KW + KSTAGES;     // + stage (fused): V of the stage's tile stored
-constexpr int NBAR = B_VW + VSTAGES;
+constexpr int B_QR = B_VW + VSTAGES;     // (fused) Q turned in shared memory, suffix K' in the cache
+constexpr int NBAR = B_QR + 1;
 
 constexpr int kSmemTiles = 2 /*Q_A, Q_B*/ + KSTAGES + VSTAGES;
 constexpr size_t kSmemBytes = 1024 /*align*/ + (size_t)TILE * kSmemTiles + 8 * NBAR + 16;
@@ -131,13 +135,17 @@ struct TcParams {                // CUtensorMap members carry their own alignmen
 
 struct FusedTcParams {
     TcParams t;
-    // pool [L*pool_slots][Hkv][128] and cache [L*rows][Hkv][128] in boxes of 128 rows (whole
-    // tiles from one source), 64 rows and 8 rows (one swizzle atom) for the runs of clean
-    // groups of a mixed tile
-    CUtensorMap tm_pk, tm_pv, tm_pk64, tm_pv64, tm_pk8, tm_pv8, tm_ck64, tm_cv64, tm_ck8, tm_cv8;
+    // pool [L*pool_slots][Hkv][128], suffix V [L*Btot*Sq][Hkv][128] and cache K [L*rows][Hkv]
+    // [128] (the suffix rows' K' once turned) in boxes of 128 rows (whole tiles from one
+    // source), 64 rows and 8 rows (one swizzle atom) for the runs of clean groups of a mixed
+    // tile; the cache's 128-row K map is t.tm_k
+    CUtensorMap tm_pk, tm_pv, tm_pk64, tm_pv64, tm_pk8, tm_pv8;
+    CUtensorMap tm_sv, tm_sv64, tm_sv8, tm_ck64, tm_ck8;
     const void* pool_k;      // [L][pool_slots][Hkv][128]
     const void* pool_v;
-    void* cache_k;           // [L][rows][Hkv][128]: suffix rows read, composed rows written
+    const void* k_suf;       // [L][Btot][Sq][Hkv][128], K before RoPE
+    const void* v_suf;
+    void* cache_k;           // [L][rows][Hkv][128]: written (composed slots, suffix, zero rows)
     void* cache_v;
     int32_t* pos;            // [rows]
     float2* occ_cs;          // scratch [occurrences][64]: (cos, sin) of each occurrence's turn
@@ -460,7 +468,7 @@ __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, u
 // the other tile's softmax finished, putting the two softmaxes in series.
 template <bool kHasB>
 __device__ __forceinline__ void mma_issuer(const TcParams& P, uint32_t tmem, uint32_t sQ, uint32_t sK,
-                                           uint32_t sV, uint32_t sBar, int n_kv,
+                                           uint32_t sV, uint32_t sBar, int n_kv, int q_ready,
                                            volatile uint32_t* abort) {
     static_assert(KSTAGES == 3 && VSTAGES == 2, "the issue schedule assumes 3 K and 2 V stages");
     auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
@@ -519,7 +527,7 @@ __device__ __forceinline__ void mma_issuer(const TcParams& P, uint32_t tmem, uin
         mma_commit(bar(B_KE + ks));
     };
 
-    wait(B_Q, 0u);
+    wait(q_ready, 0u);
     wait(B_KF + 0, 0u);
     // key tile 0: S_A(0), S_B(0)
     s_block(dQa, dK0, tS_a);
@@ -620,22 +628,24 @@ __device__ __forceinline__ int64_t walk_slot(OccWalk& w, const FusedTcParams& F,
     }
     return slot;
 }
-// Whether the 8-row group of composed row R (rows R & ~7 .. +7) comes from more than one
-// contiguous source: several occurrences, or composed slots and suffix rows.  Clean groups
-// are moved by TMA, ragged ones row by row.
+// Whether the 8-row group of composed row R (rows R & ~7 .. +7) is not one contiguous run of
+// one source: several occurrences, composed slots and suffix rows, or rows past the suffix
+// (`used` = slots + suffix tokens; those rows are zeros).  Clean groups are moved by TMA,
+// ragged ones row by row.
 __device__ __forceinline__ bool group_ragged(OccWalk& w, const FusedTcParams& F, int R, int n_slots,
-                                            int o_end) {
+                                            int used, int o_end) {
     const int gs = R & ~7, ge = gs + 8;
-    if (R >= n_slots) return gs < n_slots;
+    if (R >= n_slots) return gs < n_slots || ge > used;
     walk_to(w, F, R, o_end);
     return !(w.beg <= gs && ge <= w.end);
 }
 
 // The fused kernel's TMA producer (one thread): for each key tile, K and V each as soon as
-// their stage is free.  A tile from one source (a single occurrence's pool slots, or the
-// cache's suffix rows) is two 128-row boxes; a mixed tile is one 8-row box per clean group
-// (its ragged groups are left to the loaders).  The stage's "landed" barrier expects the
-// bytes of the boxes issued.
+// their stage is free.  A tile from one source (a single occurrence's pool slots, or 128 of
+// the request's suffix rows) is two 128-row boxes; a mixed tile is moved as runs of clean
+// 8-row groups in boxes of 64 and 8 rows (its ragged groups are left to the loaders).  The
+// stage's "landed" barrier expects the bytes of the boxes issued.  Suffix rows come from
+// v_suf for V and, for K, from the cache once the softmax warps have written them turned.
 __device__ __forceinline__ void fused_producer(const FusedTcParams& F, int l, int bl, int hk, int j_base,
                                                int n_kv, bool writer, uint32_t sK, uint32_t sV,
                                                uint32_t sBar, volatile uint32_t* abort) {
@@ -643,10 +653,14 @@ __device__ __forceinline__ void fused_producer(const FusedTcParams& F, int l, in
     auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
     const int lg = P.layer0 + l;
     const int n_slots = P.req[bl].n_slots;
+    const int used = n_slots + P.sq;
     const int o_begin = F.req_occ[bl];
     const int o_end = F.req_occ[bl + 1];
     const int pool_row0 = (int)((int64_t)lg * F.pool_slots);
+    // suffix row R (R >= n_slots): row sfx_row0 + R of v_suf, row cache_row0 + R of the cache
+    const int sfx_row0 = (l * P.batch_total + P.b0 + bl) * P.sq - n_slots;
     const int cache_row0 = (int)((int64_t)lg * P.rows + P.req[bl].row_base);
+    bool k_turned = false;     // the suffix rows' K' are in the cache
     OccWalk wk{}, wv{};
     if (o_end > o_begin) {
         walk_load(wk, F, o_begin);
@@ -654,33 +668,40 @@ __device__ __forceinline__ void fused_producer(const FusedTcParams& F, int l, in
     }
     auto tile = [&](int jt, bool is_v, OccWalk& w, uint32_t dst, uint32_t landed) {
         const CUtensorMap* pool128 = is_v ? &F.tm_pv : &F.tm_pk;
-        const CUtensorMap* cache128 = is_v ? &P.tm_v : &P.tm_k;
+        const CUtensorMap* sfx128 = is_v ? &F.tm_sv : &P.tm_k;
         const CUtensorMap* pool8 = is_v ? &F.tm_pv8 : &F.tm_pk8;
-        const CUtensorMap* cache8 = is_v ? &F.tm_cv8 : &F.tm_ck8;
+        const CUtensorMap* sfx8 = is_v ? &F.tm_sv8 : &F.tm_ck8;
+        const int sfx_base = is_v ? sfx_row0 : cache_row0;
         const int R0 = (j_base + jt) * BN;
-        if (R0 >= n_slots) {                                  // the cache's suffix rows
+        if (!is_v && !k_turned && R0 + BN > n_slots) {
+            mbar_wait(bar(B_QR), 0u, P.err, abort);
+            k_turned = true;
+        }
+        if (R0 >= n_slots && R0 + BN <= used) {              // 128 suffix rows
             mbar_expect_tx(landed, TILE);
-            tma_load_3d(dst, cache128, 0, hk, cache_row0 + R0, landed);
-            tma_load_3d(dst + HALF_TILE, cache128, 64, hk, cache_row0 + R0, landed);
+            tma_load_3d(dst, sfx128, 0, hk, sfx_base + R0, landed);
+            tma_load_3d(dst + HALF_TILE, sfx128, 64, hk, sfx_base + R0, landed);
             return;
         }
-        walk_to(w, F, R0, o_end);
-        if (w.beg <= R0 && R0 + BN <= w.end && (int64_t)w.src + (R0 - w.beg) + BN <= F.pool_slots &&
-            w.src + (R0 - w.beg) >= 0) {                      // one occurrence
-            const int row = pool_row0 + w.src + (R0 - w.beg);
-            mbar_expect_tx(landed, TILE);
-            tma_load_3d(dst, pool128, 0, hk, row, landed);
-            tma_load_3d(dst + HALF_TILE, pool128, 64, hk, row, landed);
-            return;
+        if (R0 < n_slots) {
+            walk_to(w, F, R0, o_end);
+            if (w.beg <= R0 && R0 + BN <= w.end && (int64_t)w.src + (R0 - w.beg) + BN <= F.pool_slots &&
+                w.src + (R0 - w.beg) >= 0) {                  // one occurrence
+                const int row = pool_row0 + w.src + (R0 - w.beg);
+                mbar_expect_tx(landed, TILE);
+                tma_load_3d(dst, pool128, 0, hk, row, landed);
+                tma_load_3d(dst + HALF_TILE, pool128, 64, hk, row, landed);
+                return;
+            }
         }
         // mixed: runs of clean groups whose source rows are contiguous, each moved in boxes of
         // 64 and 8 rows; the bytes are counted in a first walk, the boxes issued in a second
         const CUtensorMap* pool64 = is_v ? &F.tm_pv64 : &F.tm_pk64;
-        const CUtensorMap* cache64 = is_v ? &F.tm_cv64 : &F.tm_ck64;
+        const CUtensorMap* sfx64 = is_v ? &F.tm_sv64 : &F.tm_ck64;
         auto runs = [&](OccWalk& wr, bool issue) -> int {
             int groups = 0;
             int g0 = -1, ng = 0, row0 = 0;
-            bool cache0 = false;
+            bool sfx0 = false;
             auto flush = [&]() {
                 if (ng == 0) return;
                 groups += ng;
@@ -689,7 +710,7 @@ __device__ __forceinline__ void fused_producer(const FusedTcParams& F, int l, in
                     while (left > 0) {
                         const bool big = left >= 8;
                         const int n = big ? 8 : 1;
-                        const CUtensorMap* tm = cache0 ? (big ? cache64 : cache8) : (big ? pool64 : pool8);
+                        const CUtensorMap* tm = sfx0 ? (big ? sfx64 : sfx8) : (big ? pool64 : pool8);
                         const int row = row0 + 8 * (g - g0);
                         const uint32_t d = dst + (uint32_t)g * 1024u;
                         tma_load_3d(d, tm, 0, hk, row, landed);
@@ -702,12 +723,12 @@ __device__ __forceinline__ void fused_producer(const FusedTcParams& F, int l, in
             };
             for (int g = 0; g < BN / 8; ++g) {
                 const int R = R0 + 8 * g;
-                bool clean = !group_ragged(wr, F, R, n_slots, o_end);
-                bool is_cache = R >= n_slots;
+                bool clean = !group_ragged(wr, F, R, n_slots, used, o_end);
+                const bool is_sfx = R >= n_slots;
                 int row = 0;
                 if (clean) {
-                    if (is_cache) {
-                        row = cache_row0 + R;
+                    if (is_sfx) {
+                        row = sfx_base + R;
                     } else {
                         const int64_t slot = (int64_t)wr.src + (R - wr.beg);
                         clean = slot >= 0 && slot + 8 <= F.pool_slots;   // else the loaders report it
@@ -718,14 +739,14 @@ __device__ __forceinline__ void fused_producer(const FusedTcParams& F, int l, in
                     flush();
                     continue;
                 }
-                if (ng > 0 && is_cache == cache0 && row == row0 + 8 * ng) {
+                if (ng > 0 && is_sfx == sfx0 && row == row0 + 8 * ng) {
                     ++ng;                                     // the run goes on
                 } else {
                     flush();
                     g0 = g;
                     ng = 1;
                     row0 = row;
-                    cache0 = is_cache;
+                    sfx0 = is_sfx;
                 }
             }
             flush();
@@ -782,8 +803,7 @@ __device__ __forceinline__ void tma_store_3d(const CUtensorMap* tm, uint32_t src
 }
 
 // Store a whole 128-row tile (two 64-channel halves) of a stage to the cache by TMA and wait
-// until the store has read shared memory; the stage is then free for the producer.  Tiles
-// with composed slots only: their suffix rows go back unchanged.
+// until the store has read shared memory; the stage is then free for the producer.
 __device__ __forceinline__ void store_tile(const CUtensorMap* tm, uint32_t src, int hk, int row) {
     tma_store_3d(tm, src, 0, hk, row);
     tma_store_3d(tm, src + HALF_TILE, 64, hk, row);
@@ -822,8 +842,9 @@ __device__ __forceinline__ uint32_t f2_to_bf2(float lo, float hi) {
 // The K loaders of the fused kernel (warps 12..15, lt = 0..127).  Per key tile, thread lt
 // owns chunk pair kc = lt % 8 (channels 8kc.. and 64+8kc..) of rows lt/8 + 16i: it copies
 // the ragged rows among them (cp.async, 16 bytes a chunk, into the swizzled layout TMA
-// produces), waits for the tile's TMA part, turns its chunks of composed slots by their
-// occurrence's offset (CTAs of pair 0 in layer 0, KV head 0 also write the slots'
+// produces; suffix rows from the cache, once the softmax warps have turned them) and zeroes
+// those past the suffix, waits for the tile's TMA part, turns its chunks of composed slots
+// by their occurrence's offset (the writer CTAs in layer 0, KV head 0 also write the slots'
 // positions), and releases the stage to the MMA and the K writer.  They wait only for a K
 // stage to be free, so they run up to two tiles ahead of the MMA.
 __device__ __forceinline__ void fused_k_loader(const FusedTcParams& F, int lt, int l, int bl, int hk,
@@ -833,8 +854,10 @@ __device__ __forceinline__ void fused_k_loader(const FusedTcParams& F, int lt, i
     const TcParams& P = F.t;
     auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
     const int lg = P.layer0 + l;
-    const int n_slots = P.req[bl].n_slots;
-    const int row_base = P.req[bl].row_base;
+    const ReqParam& rq = P.req[bl];
+    const int n_slots = rq.n_slots;
+    const int used = n_slots + P.sq;
+    const int row_base = rq.row_base;
     const int o_begin = F.req_occ[bl];
     const int o_end = F.req_occ[bl + 1];
     const int64_t hkv = P.hkv;
@@ -849,13 +872,17 @@ __device__ __forceinline__ void fused_k_loader(const FusedTcParams& F, int lt, i
         walk_load(wk, F, o_begin);
         wr = wk;
     }
-    int cs_occ = -1;
+    int cs_occ = -1;          // occurrence whose angles cc, ss hold
+    bool k_turned = false;    // the suffix rows' K' are in the cache
     float2 cc[4], ss[4];      // cos and sin of this thread's 8 frequencies, in pairs
     // (cos, sin) of the request's occurrences at the 64 frequencies, evaluated once per CTA
     // into the scratch table (every CTA of the request writes the same values) and read back
     // as a row per occurrence while turning, instead of evaluating angles per tile
-    for (int e = (o_begin << 6) + lt; e < (o_end << 6); e += kLoaders)
-        F.occ_cs[e] = turn_cs(F.rope.turn[e & 63], F.occ[e >> 6].delta);
+    {
+        const uint64_t turn = F.rope.turn[lt & 63];     // entry e has frequency e % 64 = lt % 64
+        for (int e = (o_begin << 6) + lt; e < (o_end << 6); e += kLoaders)
+            F.occ_cs[e] = turn_cs(turn, F.occ[e >> 6].delta);
+    }
     asm volatile("bar.sync 1, %0;" ::"n"(kLoaders) : "memory");
 
     for (int jt = 0; jt < n_kv; ++jt) {
@@ -868,13 +895,22 @@ __device__ __forceinline__ void fused_k_loader(const FusedTcParams& F, int lt, i
         for (int i = 0; i < BN / 16; ++i) {
             const int r = kr0 + 16 * i;
             const int R = R0 + r;
-            if (!group_ragged(wk, F, R, n_slots, o_end)) continue;
+            if (!group_ragged(wk, F, R, n_slots, used, o_end)) continue;
+            if (R >= used) {                              // past the suffix: zeros
+                sts128(st + sw_off(r, kc), make_uint4(0u, 0u, 0u, 0u));
+                sts128(st + HALF_TILE + sw_off(r, kc), make_uint4(0u, 0u, 0u, 0u));
+                continue;
+            }
             const bf* src;
             if (R < n_slots) {
                 const int64_t slot = walk_slot(wk, F, R, o_end);
                 if (slot < 0) continue;
                 src = pk + ((pool_row0 + slot) * hkv + hk) * HD;
             } else {
+                if (!k_turned) {
+                    mbar_wait(bar(B_QR), 0u, P.err, abort);
+                    k_turned = true;
+                }
                 src = ck + ((cache_row0 + R) * hkv + hk) * HD;
             }
             cp_async16(st + sw_off(r, kc), src + 8 * kc);
@@ -922,29 +958,29 @@ __device__ __forceinline__ void fused_k_loader(const FusedTcParams& F, int lt, i
     }
 }
 
-// The K writer of the fused kernel (warp 2, one thread, CTAs of pair 0): once the K loaders
-// have released a tile that holds composed slots, its K' goes to the cache by TMA.
+// The K writer of the fused kernel (warp 2, one thread, writer CTAs): once the K loaders have
+// released a tile, its K' (composed slots and suffix rows turned, zero rows past the suffix)
+// goes to the cache by TMA.
 __device__ __forceinline__ void fused_k_writer(const FusedTcParams& F, int l, int bl, int hk, int j_base,
                                                int n_kv, uint32_t sK, uint32_t sBar,
                                                volatile uint32_t* abort) {
     const TcParams& P = F.t;
     auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
-    const int n_slots = P.req[bl].n_slots;
     const int cache_row0 = (int)((int64_t)(P.layer0 + l) * P.rows + P.req[bl].row_base);
     for (int jt = 0; jt < n_kv; ++jt) {
         const int R0 = (j_base + jt) * BN;
         const int ks = jt % KSTAGES;
         mbar_wait(bar(B_KF + ks), (uint32_t)(jt / KSTAGES) & 1u, P.err, abort);
-        if (R0 < n_slots) store_tile(&P.tm_k, sK + (uint32_t)(ks * TILE), hk, cache_row0 + R0);
+        store_tile(&P.tm_k, sK + (uint32_t)(ks * TILE), hk, cache_row0 + R0);
         mbar_arrive(bar(B_KW + ks));
     }
     asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
 }
 
 // The V loader of the fused kernel (warp 3, lt = 0..31): per key tile, the ragged 8-row
-// groups' rows by cp.async (thread lt: chunk lt % 16 of rows lt/16 + 2u of each such
-// group), then the tile's TMA part, then the stage is released to the MMA; in the CTAs of
-// pair 0, lane 0 then stores the tile's V to the cache.
+// groups' rows by cp.async, or zeros past the suffix (thread lt: chunk lt % 16 of rows
+// lt/16 + 2u of each such group), then the tile's TMA part, then the stage is released to
+// the MMA; in the writer CTAs, lane 0 then stores the tile's V to the cache.
 __device__ __forceinline__ void fused_v_loader(const FusedTcParams& F, int lt, int l, int bl, int hk,
                                                bool writer, int j_base, int n_kv, uint32_t sV,
                                                uint32_t sBar, volatile uint32_t* abort) {
@@ -953,13 +989,15 @@ __device__ __forceinline__ void fused_v_loader(const FusedTcParams& F, int lt, i
     auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
     const int lg = P.layer0 + l;
     const int n_slots = P.req[bl].n_slots;
+    const int used = n_slots + P.sq;
     const int o_begin = F.req_occ[bl];
     const int o_end = F.req_occ[bl + 1];
     const int64_t hkv = P.hkv;
     const int64_t pool_row0 = (int64_t)lg * F.pool_slots;
     const int64_t cache_row0 = (int64_t)lg * P.rows + P.req[bl].row_base;
+    const int64_t sfx_row0 = ((int64_t)l * P.batch_total + P.b0 + bl) * P.sq - n_slots;
     const bf* pv = static_cast<const bf*>(F.pool_v);
-    const bf* cv = static_cast<const bf*>(F.cache_v);
+    const bf* sv = static_cast<const bf*>(F.v_suf);
     const int vq = lt & 15, vr0 = lt >> 4;
     OccWalk wv{};
     if (o_end > o_begin) walk_load(wv, F, o_begin);
@@ -971,18 +1009,22 @@ __device__ __forceinline__ void fused_v_loader(const FusedTcParams& F, int lt, i
             mbar_wait(bar(B_VE + st_i), (uint32_t)((jt / VSTAGES) - 1) & 1u, P.err, abort);
 #pragma unroll 1
         for (int g = 0; g < BN / 8; ++g) {
-            if (!group_ragged(wv, F, R0 + 8 * g, n_slots, o_end)) continue;
+            if (!group_ragged(wv, F, R0 + 8 * g, n_slots, used, o_end)) continue;
 #pragma unroll 1
             for (int u = 0; u < 4; ++u) {
                 const int r = 8 * g + vr0 + 2 * u;
                 const int R = R0 + r;
+                if (R >= used) {                          // past the suffix: zeros
+                    sts128(st + sw_off(r, vq & 7), make_uint4(0u, 0u, 0u, 0u));
+                    continue;
+                }
                 const bf* src;
                 if (R < n_slots) {
                     const int64_t slot = walk_slot(wv, F, R, o_end);
                     if (slot < 0) continue;
                     src = pv + ((pool_row0 + slot) * hkv + hk) * HD;
                 } else {
-                    src = cv + ((cache_row0 + R) * hkv + hk) * HD;
+                    src = sv + ((sfx_row0 + R) * hkv + hk) * HD;
                 }
                 cp_async16(st + sw_off(r, vq & 7), src + 8 * vq);
             }
@@ -992,16 +1034,117 @@ __device__ __forceinline__ void fused_v_loader(const FusedTcParams& F, int lt, i
         mbar_wait(bar(B_VL + st_i), (uint32_t)(jt / VSTAGES) & 1u, P.err, abort);
         fence_proxy_async();
         mbar_arrive(bar(B_VF + st_i));
-        if (writer) {         // CTAs of pair 0: the tile's V to the cache
+        if (writer) {         // writer CTAs: the tile's V to the cache
             __syncwarp();
             if (lt == 0) {
-                if (R0 < n_slots)
-                    store_tile(&P.tm_v, sV + (uint32_t)(st_i * TILE), hk, (int)cache_row0 + R0);
+                store_tile(&P.tm_v, sV + (uint32_t)(st_i * TILE), hk, (int)cache_row0 + R0);
                 mbar_arrive(bar(B_VW + st_i));
             }
         }
     }
     if (writer && lt == 0) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+}
+
+// generic-proxy writes to global and shared memory become visible to the async proxy (TMA
+// loads of the cache, tensor-core reads of shared memory)
+__device__ __forceinline__ void fence_proxy_async_all() { asm volatile("fence.proxy.async;" ::: "memory"); }
+
+// The suffix preparation of the fused kernel, done by the softmax warps (ts = 0..255) while
+// they wait for their first S tile.  Item (token tt, chunk pair q = ts % 8) evaluates the
+// angles of position L_r + tt at the 8 frequencies of chunk pair q once and turns with them
+//   - chunk pair q of suffix row tt's K, from k_suf into the cache, for tt in [k_lo, k_hi)
+//     (the suffix rows among this CTA's key tiles; the CTAs of a request write the same
+//     bits), with the row's position in the CTAs that own the positions;
+//   - chunk pair q of the G query rows of token tt in shared memory, for tt in [q_lo, q_hi)
+//     (this CTA's query tokens), once Q has landed.
+// The angles and the rounding are the suffix kernel's.  Then the writes are made visible to
+// the async proxy and the MMA issuer, the producer and the K loaders are told (B_QR).
+__device__ __forceinline__ void fused_suffix_prep(const FusedTcParams& F, int ts, int l, int bl, int hk,
+                                                  int k_lo, int k_hi, int q_lo, int q_hi, bool pos_rows,
+                                                  uint32_t sQ, uint32_t sBar, volatile uint32_t* abort) {
+    using bf = __nv_bfloat16;
+    const TcParams& P = F.t;
+    auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
+    const ReqParam& rq = P.req[bl];
+    const int64_t pos0 = (int64_t)rq.l_req + rq.t0;
+    const int G = P.group, tq = P.tq;
+    const int q = ts & 7;                  // every item of this thread has chunk pair q
+    uint64_t turn[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) turn[j] = F.rope.turn[8 * q + j];
+    const int64_t row_elems = (int64_t)P.hkv * HD;
+    const bf* ksrc = static_cast<const bf*>(F.k_suf) +
+                     ((int64_t)l * P.batch_total + P.b0 + bl) * P.sq * row_elems + hk * HD + 8 * q;
+    bf* kdst = static_cast<bf*>(F.cache_k) +
+               ((int64_t)(P.layer0 + l) * P.rows + rq.row_base + rq.n_slots) * row_elems + hk * HD + 8 * q;
+    int lo = 0, hi = 0;
+    if (k_hi > k_lo) {
+        lo = k_lo;
+        hi = k_hi;
+    }
+    if (q_hi > q_lo) {
+        lo = hi > lo ? min(lo, q_lo) : q_lo;
+        hi = max(hi, q_hi);
+    }
+    bool q_landed = false;
+#pragma unroll 1
+    for (int i = ts; i < (hi - lo) * 8; i += 256) {
+        const int tt = lo + (i >> 3);
+        const bool do_k = tt >= k_lo && tt < k_hi;
+        const bool do_q = tt >= q_lo && tt < q_hi;
+        uint4 xa = make_uint4(0u, 0u, 0u, 0u), ya = xa;
+        if (do_k) {
+            xa = ld16(ksrc + tt * row_elems);
+            ya = ld16(ksrc + tt * row_elems + 64);
+        }
+        float2 cc[4], ss[4];
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+            const float2 c0 = turn_cs(turn[2 * w], pos0 + tt);
+            const float2 c1 = turn_cs(turn[2 * w + 1], pos0 + tt);
+            cc[w] = make_float2(c0.x, c1.x);
+            ss[w] = make_float2(c0.y, c1.y);
+        }
+        auto turn_chunks = [&](const uint4& xv, const uint4& yv, uint4& xo, uint4& yo) {
+            const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w}, yw[4] = {yv.x, yv.y, yv.z, yv.w};
+            uint32_t a[4], b[4];
+#pragma unroll
+            for (int w = 0; w < 4; ++w) {
+                float2 gx, gy;
+                rotate2(bf2_to_f2(xw[w]), bf2_to_f2(yw[w]), cc[w], ss[w], gx, gy);
+                a[w] = f2_to_bf2(gx.x, gx.y);
+                b[w] = f2_to_bf2(gy.x, gy.y);
+            }
+            xo = make_uint4(a[0], a[1], a[2], a[3]);
+            yo = make_uint4(b[0], b[1], b[2], b[3]);
+        };
+        if (do_k) {
+            uint4 xo, yo;
+            turn_chunks(xa, ya, xo, yo);
+            st16(kdst + tt * row_elems, xo);
+            st16(kdst + tt * row_elems + 64, yo);
+            if (pos_rows && q == 0) F.pos[rq.row_base + rq.n_slots + tt] = (int32_t)(pos0 + tt);
+        }
+        if (do_q) {
+            if (!q_landed) {
+                mbar_wait(bar(B_Q), 0u, P.err, abort);
+                q_landed = true;
+            }
+            const int x = (tt - q_lo) / tq;           // tile A or B
+            const int u = tt - q_lo - x * tq;         // token within the tile
+            const uint32_t base = sQ + (uint32_t)x * TILE;
+#pragma unroll 1
+            for (int g = 0; g < G; ++g) {
+                const uint32_t a0 = base + sw_off(u * G + g, q);
+                uint4 xo, yo;
+                turn_chunks(lds128(a0), lds128(a0 + HALF_TILE), xo, yo);
+                sts128(a0, xo);
+                sts128(a0 + HALF_TILE, yo);
+            }
+        }
+    }
+    fence_proxy_async_all();
+    mbar_arrive(bar(B_QR));
 }
 
 template <bool kFused>
@@ -1029,8 +1172,12 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
     const int s_r = P.req[bl].n_slots;
     // pair of Q tiles, the last first: under a causal mask the later pairs see more keys, so
     // the longest CTAs start in the first wave
-    const int pr = (int)(gridDim.x / P.n_split) - 1 - (int)(blockIdx.x / P.n_split);
+    const int n_pairs = (int)(gridDim.x / P.n_split);
+    const int pr = n_pairs - 1 - (int)(blockIdx.x / P.n_split);
     const int sp = (int)(blockIdx.x % P.n_split);   // key-range split
+    // fused: the CTAs of the last pair see every key row of the request (all of the suffix),
+    // so they write the composed cache
+    const bool writer = pr == n_pairs - 1;
     const int t0a = 2 * pr * P.tq;
     const int t0b = t0a + P.tq;
     const bool has_b = t0b < P.sq;
@@ -1064,6 +1211,7 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
             mbar_init(bar(B_VL + s), 1);
             mbar_init(bar(B_VW + s), 1);
         }
+        mbar_init(bar(B_QR), 256u);
         mbar_init(bar(B_OD), 1);
         *abort = 0u;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -1096,7 +1244,7 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
                 tma_load_4d(sQ + TILE + HALF_TILE, &P.tm_q, 64, hk * G, t0b, qz, bar(B_Q));
             }
             if constexpr (kFused) {
-                fused_producer(KP, l, bl, hk, j_base, n_kv, pr == 0, sK, sV, sBar, abort);
+                fused_producer(KP, l, bl, hk, j_base, n_kv, writer, sK, sV, sBar, abort);
             } else {
                 const int key0 = (int)((int64_t)(P.layer0 + l) * P.rows + P.req[bl].row_base) + j_base * BN;
                 // two independent queues: a K load waits only for its own K stage
@@ -1132,21 +1280,29 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
         } else if (warp == 1 && lane == 0 && n_kv > 0) {
             // ------------------------------------------------------------ MMA issuer
             if (has_b)
-                mma_issuer<true>(P, tmem, sQ, sK, sV, sBar, n_kv, abort);
+                mma_issuer<true>(P, tmem, sQ, sK, sV, sBar, n_kv, kFused ? B_QR : B_Q, abort);
             else
-                mma_issuer<false>(P, tmem, sQ, sK, sV, sBar, n_kv, abort);
-        } else if (warp == 2 && lane == 0 && n_kv > 0 && pr == 0) {
+                mma_issuer<false>(P, tmem, sQ, sK, sV, sBar, n_kv, kFused ? B_QR : B_Q, abort);
+        } else if (warp == 2 && lane == 0 && n_kv > 0 && writer) {
             // ------------------------------------------------------------ K writer (fused)
             if constexpr (kFused) fused_k_writer(KP, l, bl, hk, j_base, n_kv, sK, sBar, abort);
         } else if (warp == 3 && n_kv > 0) {
             // ------------------------------------------------------------ V loader (fused)
             if constexpr (kFused)
-                fused_v_loader(KP, lane, l, bl, hk, pr == 0, j_base, n_kv, sV, sBar, abort);
+                fused_v_loader(KP, lane, l, bl, hk, writer, j_base, n_kv, sV, sBar, abort);
         }
     } else if (warp < 12) {
         asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kFused ? kRegsHighFused : kRegsHigh));
         // ---------------------------------------------------------------- softmax warps
         const int x = warp >= 8 ? 1 : 0;               // tile A (warps 4..7) or B (8..11)
+        if constexpr (kFused) {
+            // the suffix rows among this CTA's key tiles, and its query tokens
+            const int k_lo = max(0, j_base * BN - s_r);
+            const int k_hi = min(P.sq, (j_base + n_kv) * BN - s_r);
+            const int q_hi = n_kv > 0 ? t_last + 1 : t0a;
+            fused_suffix_prep(KP, (int)threadIdx.x - 128, l, bl, hk, k_lo, k_hi, t0a, q_hi,
+                              writer && P.layer0 + l == 0 && hk == 0, sQ, sBar, abort);
+        }
         if (x == 0 || has_b)
             softmax_tile(P, tmem, sBar, x, warp & 3, lane, x ? t0b : t0a, l, bl, b, hk, sp, j_base,
                          n_kv, abort);
@@ -1155,7 +1311,7 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
             asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsLowFused));
             // ------------------------------------------------------------ loaders (fused)
             if (n_kv > 0)
-                fused_k_loader(KP, (int)threadIdx.x - 12 * 32, l, bl, hk, pr == 0, j_base, n_kv, sK,
+                fused_k_loader(KP, (int)threadIdx.x - 12 * 32, l, bl, hk, writer, j_base, n_kv, sK,
                                sBar, abort);
         }
     }
@@ -1374,11 +1530,13 @@ cudaError_t prepare_attn_fused(const AttnParams& a, const FusedSpec& f) {
     FusedTcParams& p = g_fused;
     cudaError_t e = prepare_tc<true>(a, p.t, g_fused_grid);
     if (e != cudaSuccess) return e;
-    if (a.layer0 != 0 || f.req_occ[0] != 0 || f.req_occ[a.batch] > kMaxFusedOcc)
+    if (a.layer0 != 0 || p.t.sq_pitch != a.sq || f.req_occ[0] != 0 || f.req_occ[a.batch] > kMaxFusedOcc)
         return cudaErrorInvalidValue;
     const int64_t prow = (int64_t)a.lq * f.pool_slots;
     const int64_t crow = (int64_t)a.lq * a.rows;
-    if (prow > 0x7fffffffLL || crow > 0x7fffffffLL) return cudaErrorInvalidValue;
+    const int64_t srow = (int64_t)a.lq * a.batch_total * a.sq;
+    if (prow > 0x7fffffffLL || crow > 0x7fffffffLL || srow > 0x7fffffffLL) return cudaErrorInvalidValue;
+    if (!f.k_suf || !f.v_suf || !f.occ_cs) return cudaErrorInvalidValue;
     const cuuint64_t str[2] = {(cuuint64_t)HD * 2, (cuuint64_t)a.hkv * HD * 2};
     const cuuint32_t box128[3] = {64, 1, (cuuint32_t)BN};
     const cuuint32_t box64[3] = {64, 1, 64};
@@ -1404,16 +1562,21 @@ cudaError_t prepare_attn_fused(const AttnParams& a, const FusedSpec& f) {
             key_hkv = a.hkv;
         }
     }
-    {   // cache [L*rows][Hkv][128] in 64- and 8-row boxes (128-row maps: prepare_tc)
+    {   // suffix V [Lq*Btot*Sq][Hkv][128] in 128-, 64- and 8-row boxes, cache K [L*rows][Hkv]
+        // [128] in 64- and 8-row boxes (its 128-row map: prepare_tc)
+        const cuuint64_t sdims[3] = {HD, (cuuint64_t)a.hkv, (cuuint64_t)srow};
         const cuuint64_t cdims[3] = {HD, (cuuint64_t)a.hkv, (cuuint64_t)crow};
-        if (!encode(&p.tm_ck64, a.cache_k, 3, cdims, str, box64) ||
-            !encode(&p.tm_cv64, a.cache_v, 3, cdims, str, box64) ||
-            !encode(&p.tm_ck8, a.cache_k, 3, cdims, str, box8) ||
-            !encode(&p.tm_cv8, a.cache_v, 3, cdims, str, box8))
+        if (!encode(&p.tm_sv, f.v_suf, 3, sdims, str, box128) ||
+            !encode(&p.tm_sv64, f.v_suf, 3, sdims, str, box64) ||
+            !encode(&p.tm_sv8, f.v_suf, 3, sdims, str, box8) ||
+            !encode(&p.tm_ck64, a.cache_k, 3, cdims, str, box64) ||
+            !encode(&p.tm_ck8, a.cache_k, 3, cdims, str, box8))
             return cudaErrorInvalidValue;
     }
     p.pool_k = f.pool_k;
     p.pool_v = f.pool_v;
+    p.k_suf = f.k_suf;
+    p.v_suf = f.v_suf;
     p.cache_k = const_cast<void*>(a.cache_k);
     p.cache_v = const_cast<void*>(a.cache_v);
     p.pos = f.pos;

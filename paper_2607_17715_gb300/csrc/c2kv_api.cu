@@ -610,8 +610,9 @@ c2kv_status attend_check(c2kv_ctx* c, const char* what, int32_t layer, const voi
 }
 
 // Suffix preparation and attention of a cache (arguments already checked).  With `fused`,
-// the cache's composed slots are not written yet: the fused kernel reads them from the pool
-// and writes them (tensor-core route, every layer).
+// the cache is not written yet: the fused kernel reads the composed slots from the pool and
+// the suffix from k_suf / v_suf, turns the queries itself, and writes the whole cache
+// (tensor-core route, every layer, one launch).
 cudaError_t attend_run(c2kv_ctx* c, c2kv_cache* cache, int32_t layer0, int32_t lq, const void* q,
                        const void* k_suf, const void* v_suf, int32_t n_suffix, void* out, float* lse,
                        const c2kv::FusedSpec* fused) {
@@ -622,10 +623,11 @@ cudaError_t attend_run(c2kv_ctx* c, c2kv_cache* cache, int32_t layer0, int32_t l
     if (fused && (!use_tc || layer0 != 0 || lq != c->cfg.layers || B > c2kv::kMaxReq))
         return cudaErrorInvalidValue;
 
-    // scratch: the suffix queries after RoPE (the attention kernels' Q operand)
+    // scratch: the suffix queries after RoPE (the attention kernels' Q operand); the fused
+    // kernel turns them in shared memory
     const size_t q_bytes = (size_t)lq * B * n_suffix * c->cfg.n_q_heads * c->cfg.head_dim * c->eb;
     void* q_rot = nullptr;
-    cudaError_t e = pool_alloc(c, &q_rot, q_bytes);
+    cudaError_t e = fused ? cudaSuccess : pool_alloc(c, &q_rot, q_bytes);
     if (e != cudaSuccess) return e;
     // Key-range split of the tensor-core attention: when its work units would leave most
     // SMs idle (a single layer of a small batch), each unit's key tiles are split and the
@@ -682,7 +684,7 @@ cudaError_t attend_run(c2kv_ctx* c, c2kv_cache* cache, int32_t layer0, int32_t l
             s.req[i] = c2kv::ReqParam{cache->row_base[b0 + i], cache->n_slots[b0 + i],
                                       cache->l_req[b0 + i], 0};
         c2kv::AttnParams a{};
-        a.q_rot = q_rot;
+        a.q_rot = fused ? q : q_rot;
         a.cache_k = cache->k;
         a.cache_v = cache->v;
         a.out = out;
@@ -702,19 +704,17 @@ cudaError_t attend_run(c2kv_ctx* c, c2kv_cache* cache, int32_t layer0, int32_t l
         a.part_o = part;
         a.part_lse = part ? part + (size_t)n_split * part_rows * c->cfg.head_dim : nullptr;
         for (int32_t i = 0; i < nb; ++i) a.req[i] = s.req[i];
-        // the fused launch's host work is done before the suffix preparation is enqueued,
-        // so that the kernel follows it on the stream without waiting for the host
-        if (fused) e = c2kv::prepare_attn_fused(a, *fused);
-        if (e != cudaSuccess) break;
-        {
-            ProfScope prof_suffix(c, C2KV_PROF_SUFFIX);
-            e = c2kv::launch_suffix_prep(s, c->cfg.dtype, c->cfg.head_dim, c->stream);
-        }
-        if (e != cudaSuccess) break;
         if (fused) {
+            e = c2kv::prepare_attn_fused(a, *fused);
+            if (e != cudaSuccess) break;
             ProfScope prof_fused(c, C2KV_PROF_FUSED, true);
             e = c2kv::launch_attn_fused(c->stream, prof_fused.hook());
         } else {
+            {
+                ProfScope prof_suffix(c, C2KV_PROF_SUFFIX);
+                e = c2kv::launch_suffix_prep(s, c->cfg.dtype, c->cfg.head_dim, c->stream);
+            }
+            if (e != cudaSuccess) break;
             ProfScope prof_attn(c, C2KV_PROF_ATTN, use_tc);
             e = use_tc ? c2kv::launch_attn_tc(a, c->stream, prof_attn.hook())
                        : c2kv::launch_attn_simt(a, c->cfg.dtype, c->cfg.head_dim, c->stream);
@@ -874,6 +874,8 @@ c2kv_status c2kv_compose_attend(c2kv_ctx* c, int32_t batch, const int32_t* req_p
                            std::max<size_t>(occ.size(), 1) * 64 * sizeof(float2));
             if (e == cudaSuccess) {
                 f.occ_cs = occ_cs;
+                f.k_suf = k_suf;
+                f.v_suf = v_suf;
                 e = attend_run(c, cache, 0, c->cfg.layers, q, k_suf, v_suf, n_suffix, out, lse, &f);
                 pool_free(c, occ_cs);
             }

@@ -236,6 +236,8 @@ constexpr int kMaxFusedOcc = 512;
 struct FusedSpec {
     const void* pool_k;      // [L][pool_slots][Hkv][128]
     const void* pool_v;
+    const void* k_suf;       // [L][B][Sq][Hkv][128]: the suffix rows before RoPE (K) and V
+    const void* v_suf;
     int32_t* pos;            // [rows]
     float2* occ_cs;          // scratch [occurrences][64]: (cos, sin) of each occurrence's turn,
                              // filled by the kernel
@@ -244,8 +246,10 @@ struct FusedSpec {
     int32_t req_occ[kMaxReq + 1];   // request i of the launch: occurrences [req_occ[i], req_occ[i+1])
     FusedOcc occ[kMaxFusedOcc];
 };
-// Host preparation (tensor maps, parameters) of a fused launch, done before the suffix
-// preparation is enqueued so that the kernel follows it without a host gap; then the launch.
+// Host preparation (tensor maps, parameters) of a fused launch, then the launch.  The fused
+// kernel also does the suffix preparation (the queries and the suffix keys turned in shared
+// memory, the suffix rows and the zero rows up to the next 128-row boundary written to the
+// cache): the AttnParams' q_rot is the queries before RoPE.
 cudaError_t prepare_attn_fused(const AttnParams& a, const FusedSpec& f);
 cudaError_t launch_attn_fused(cudaStream_t s, Hook before = {});
 

@@ -130,6 +130,15 @@ def test_fused_uncompressed_long_chunk():
     _fused_case(wl)
 
 
+def test_fused_long_suffix_across_tiles():
+    # 225 composed slots, 300 suffix tokens: the suffix starts inside tile 1, fills tiles 2
+    # and 3 (whole tiles from the suffix tensors) and ends inside tile 4, whose rows past it
+    # are zeros; five pairs of query tiles, the last of which writes the cache
+    wl = synth.scaled(L8B, layers=2, chunk_tokens=300, ratio_k=4, chunks_per_request=3,
+                      pool_chunks=3, n_suffix=300)
+    _fused_case(wl)
+
+
 @pytest.mark.parametrize("split", [2, 5])
 def test_fused_key_range_splits(split):
     wl = synth.scaled(L8B, layers=1, chunk_tokens=512, ratio_k=2, chunks_per_request=3,
