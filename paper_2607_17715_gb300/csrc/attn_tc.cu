@@ -43,8 +43,8 @@
 // instead of the composed cache: the composed slots from the chunk pool, the suffix rows from
 // the caller's k_suf / v_suf.  The TMA producer moves whole tiles of one source, and runs of
 // 8-row groups of one contiguous source in mixed tiles; the rows of groups that straddle a
-// boundary are copied by 16-byte cp.async into the same swizzled layout, and rows past the
-// suffix are zeroed.  A fourth warpgroup (warps 12..15, the K loaders) turns each composed
+// boundary, and the suffix rows of K, are copied by 16-byte cp.async into the same swizzled
+// layout, and rows past the suffix are zeroed.  A fourth warpgroup (warps 12..15, the K loaders) turns each composed
 // slot's K in shared memory by its occurrence's offset and each suffix row's K by its
 // token's position (the compose and suffix kernels' angles and rounding), warp 3 releases
 // the V tiles, and the softmax warps, idle until the first S tile, turn the Q tiles in
@@ -58,6 +58,7 @@
 
 #include <math_constants.h>
 
+#include <algorithm>
 #include <cstring>
 
 #include "internal.cuh"
@@ -85,11 +86,12 @@ constexpr int kRegsLow = 136;
 constexpr int kRegsHigh = 184;
 static_assert(128 * kRegsLow + 256 * kRegsHigh <= kThreads * kLaunchRegs, "register split");
 // Fused: 512 threads launch with 128 registers each; the producer/issuer warpgroup and the
-// loader warpgroup keep 72, the softmax warpgroups rise to 184.
+// loader warpgroup keep 88 (fewer spills there measured faster than more registers for the
+// softmax), the softmax warpgroups rise to 168.
 constexpr int kThreadsFused = 512;
 constexpr int kLaunchRegsFused = 128;
-constexpr int kRegsLowFused = 72;
-constexpr int kRegsHighFused = 184;
+constexpr int kRegsLowFused = 88;
+constexpr int kRegsHighFused = 168;
 constexpr int kLoaders = 128;       // K loaders (warps 12..15)
 constexpr int kVLoaders = 32;       // V loader (warp 3)
 static_assert(256 * kRegsLowFused + 256 * kRegsHighFused <= kThreadsFused * kLaunchRegsFused,
@@ -110,8 +112,9 @@ constexpr int B_KL = B_OD + 1;           // + stage (fused): the TMA part of a K
 constexpr int B_VL = B_KL + KSTAGES;     // + stage (fused): the TMA part of a V tile landed
 constexpr int B_KW = B_VL + VSTAGES;     // + stage (fused): K' of the stage's tile stored to the cache
 constexpr int B_VW = B_KW + KSTAGES;     // + stage (fused): V of the stage's tile stored
-constexpr int B_QR = B_VW + VSTAGES;     // (fused) Q turned in shared memory, suffix K' in the cache
-constexpr int NBAR = B_QR + 1;
+constexpr int B_QR = B_VW + VSTAGES;     // (fused) Q turned in shared memory
+constexpr int B_SK = B_QR + 1;           // (fused) the suffix rows' K' turned into the cache
+constexpr int NBAR = B_SK + 1;
 
 constexpr int kSmemTiles = 2 /*Q_A, Q_B*/ + KSTAGES + VSTAGES;
 constexpr size_t kSmemBytes = 1024 /*align*/ + (size_t)TILE * kSmemTiles + 8 * NBAR + 16;
@@ -135,12 +138,11 @@ struct TcParams {                // CUtensorMap members carry their own alignmen
 
 struct FusedTcParams {
     TcParams t;
-    // pool [L*pool_slots][Hkv][128], suffix V [L*Btot*Sq][Hkv][128] and cache K [L*rows][Hkv]
-    // [128] (the suffix rows' K' once turned) in boxes of 128 rows (whole tiles from one
-    // source), 64 rows and 8 rows (one swizzle atom) for the runs of clean groups of a mixed
-    // tile; the cache's 128-row K map is t.tm_k
+    // pool [L*pool_slots][Hkv][128] and suffix V [L*Btot*Sq][Hkv][128] in boxes of 128 rows
+    // (whole tiles from one source), 64 rows and 8 rows (one swizzle atom) for the runs of
+    // clean groups of a mixed tile
     CUtensorMap tm_pk, tm_pv, tm_pk64, tm_pv64, tm_pk8, tm_pv8;
-    CUtensorMap tm_sv, tm_sv64, tm_sv8, tm_ck64, tm_ck8;
+    CUtensorMap tm_sv, tm_sv64, tm_sv8;
     const void* pool_k;      // [L][pool_slots][Hkv][128]
     const void* pool_v;
     const void* k_suf;       // [L][Btot][Sq][Hkv][128], K before RoPE
@@ -148,7 +150,10 @@ struct FusedTcParams {
     void* cache_k;           // [L][rows][Hkv][128]: written (composed slots, suffix, zero rows)
     void* cache_v;
     int32_t* pos;            // [rows]
-    float2* occ_cs;          // scratch [occurrences][64]: (cos, sin) of each occurrence's turn
+    float2* occ_cs;          // scratch [L][occurrences][64]: (cos, sin) of each occurrence's turn
+    const float2* sfx_cs;    // [B][Sq][64]: (cos, sin) of each suffix token's position, written
+                             // by suffix_angles_kernel (the prerequisite grid)
+    int32_t n_occ;           // occurrences of the launch
     int64_t pool_slots;
     RopeTurns rope;
     int32_t req_occ[kMaxReq + 1];
@@ -644,8 +649,9 @@ __device__ __forceinline__ bool group_ragged(OccWalk& w, const FusedTcParams& F,
 // their stage is free.  A tile from one source (a single occurrence's pool slots, or 128 of
 // the request's suffix rows) is two 128-row boxes; a mixed tile is moved as runs of clean
 // 8-row groups in boxes of 64 and 8 rows (its ragged groups are left to the loaders).  The
-// stage's "landed" barrier expects the bytes of the boxes issued.  Suffix rows come from
-// v_suf for V and, for K, from the cache once the softmax warps have written them turned.
+// stage's "landed" barrier expects the bytes of the boxes issued.  Suffix rows of V come from
+// v_suf; those of K are copied by the K loaders from the cache, where the softmax warps
+// write them turned (generic-proxy stores, which TMA would need a proxy fence to see).
 __device__ __forceinline__ void fused_producer(const FusedTcParams& F, int l, int bl, int hk, int j_base,
                                                int n_kv, bool writer, uint32_t sK, uint32_t sV,
                                                uint32_t sBar, volatile uint32_t* abort) {
@@ -657,10 +663,8 @@ __device__ __forceinline__ void fused_producer(const FusedTcParams& F, int l, in
     const int o_begin = F.req_occ[bl];
     const int o_end = F.req_occ[bl + 1];
     const int pool_row0 = (int)((int64_t)lg * F.pool_slots);
-    // suffix row R (R >= n_slots): row sfx_row0 + R of v_suf, row cache_row0 + R of the cache
+    // suffix row R (R >= n_slots) of V: row sfx_row0 + R of v_suf
     const int sfx_row0 = (l * P.batch_total + P.b0 + bl) * P.sq - n_slots;
-    const int cache_row0 = (int)((int64_t)lg * P.rows + P.req[bl].row_base);
-    bool k_turned = false;     // the suffix rows' K' are in the cache
     OccWalk wk{}, wv{};
     if (o_end > o_begin) {
         walk_load(wk, F, o_begin);
@@ -668,19 +672,12 @@ __device__ __forceinline__ void fused_producer(const FusedTcParams& F, int l, in
     }
     auto tile = [&](int jt, bool is_v, OccWalk& w, uint32_t dst, uint32_t landed) {
         const CUtensorMap* pool128 = is_v ? &F.tm_pv : &F.tm_pk;
-        const CUtensorMap* sfx128 = is_v ? &F.tm_sv : &P.tm_k;
         const CUtensorMap* pool8 = is_v ? &F.tm_pv8 : &F.tm_pk8;
-        const CUtensorMap* sfx8 = is_v ? &F.tm_sv8 : &F.tm_ck8;
-        const int sfx_base = is_v ? sfx_row0 : cache_row0;
         const int R0 = (j_base + jt) * BN;
-        if (!is_v && !k_turned && R0 + BN > n_slots) {
-            mbar_wait(bar(B_QR), 0u, P.err, abort);
-            k_turned = true;
-        }
-        if (R0 >= n_slots && R0 + BN <= used) {              // 128 suffix rows
+        if (is_v && R0 >= n_slots && R0 + BN <= used) {      // 128 suffix rows of V
             mbar_expect_tx(landed, TILE);
-            tma_load_3d(dst, sfx128, 0, hk, sfx_base + R0, landed);
-            tma_load_3d(dst + HALF_TILE, sfx128, 64, hk, sfx_base + R0, landed);
+            tma_load_3d(dst, &F.tm_sv, 0, hk, sfx_row0 + R0, landed);
+            tma_load_3d(dst + HALF_TILE, &F.tm_sv, 64, hk, sfx_row0 + R0, landed);
             return;
         }
         if (R0 < n_slots) {
@@ -697,7 +694,6 @@ __device__ __forceinline__ void fused_producer(const FusedTcParams& F, int l, in
         // mixed: runs of clean groups whose source rows are contiguous, each moved in boxes of
         // 64 and 8 rows; the bytes are counted in a first walk, the boxes issued in a second
         const CUtensorMap* pool64 = is_v ? &F.tm_pv64 : &F.tm_pk64;
-        const CUtensorMap* sfx64 = is_v ? &F.tm_sv64 : &F.tm_ck64;
         auto runs = [&](OccWalk& wr, bool issue) -> int {
             int groups = 0;
             int g0 = -1, ng = 0, row0 = 0;
@@ -710,7 +706,7 @@ __device__ __forceinline__ void fused_producer(const FusedTcParams& F, int l, in
                     while (left > 0) {
                         const bool big = left >= 8;
                         const int n = big ? 8 : 1;
-                        const CUtensorMap* tm = sfx0 ? (big ? sfx64 : sfx8) : (big ? pool64 : pool8);
+                        const CUtensorMap* tm = sfx0 ? (big ? &F.tm_sv64 : &F.tm_sv8) : (big ? pool64 : pool8);
                         const int row = row0 + 8 * (g - g0);
                         const uint32_t d = dst + (uint32_t)g * 1024u;
                         tma_load_3d(d, tm, 0, hk, row, landed);
@@ -723,12 +719,12 @@ __device__ __forceinline__ void fused_producer(const FusedTcParams& F, int l, in
             };
             for (int g = 0; g < BN / 8; ++g) {
                 const int R = R0 + 8 * g;
-                bool clean = !group_ragged(wr, F, R, n_slots, used, o_end);
                 const bool is_sfx = R >= n_slots;
+                bool clean = !group_ragged(wr, F, R, n_slots, used, o_end) && (is_v || !is_sfx);
                 int row = 0;
                 if (clean) {
                     if (is_sfx) {
-                        row = sfx_base + R;
+                        row = sfx_row0 + R;
                     } else {
                         const int64_t slot = (int64_t)wr.src + (R - wr.beg);
                         clean = slot >= 0 && slot + 8 <= F.pool_slots;   // else the loaders report it
@@ -758,39 +754,44 @@ __device__ __forceinline__ void fused_producer(const FusedTcParams& F, int l, in
         runs(w, true);
     };
     // a stage is free once the MMA has read it and, in the CTAs that store the composed
-    // rows, once the store of its tile to the cache has read it too
+    // rows, once the store of its tile to the cache has read it too (non-blocking tests: the
+    // producer serves whichever ring frees a stage first)
     auto k_free = [&](int j) {
         const uint32_t ph = (uint32_t)((j / KSTAGES) - 1) & 1u;
-        return j < KSTAGES || (mbar_try(bar(B_KE + j % KSTAGES), ph) &&
-                               (!writer || mbar_try(bar(B_KW + j % KSTAGES), ph)));
+        return j < KSTAGES || (mbar_test(bar(B_KE + j % KSTAGES), ph) &&
+                               (!writer || mbar_test(bar(B_KW + j % KSTAGES), ph)));
     };
     auto v_free = [&](int j) {
         const uint32_t ph = (uint32_t)((j / VSTAGES) - 1) & 1u;
-        return j < VSTAGES || (mbar_try(bar(B_VE + j % VSTAGES), ph) &&
-                               (!writer || mbar_try(bar(B_VW + j % VSTAGES), ph)));
+        return j < VSTAGES || (mbar_test(bar(B_VE + j % VSTAGES), ph) &&
+                               (!writer || mbar_test(bar(B_VW + j % VSTAGES), ph)));
     };
     int jk = 0, jv = 0;
+    long long idle0 = -1;      // start of the current wait for a free stage
     while (jk < n_kv || jv < n_kv) {
         if (jk < n_kv && k_free(jk)) {
             const int st = jk % KSTAGES;
             tile(jk, false, wk, sK + (uint32_t)(st * TILE), bar(B_KL + st));
             ++jk;
+            idle0 = -1;
             continue;
         }
         if (jv < n_kv && v_free(jv)) {
             const int st = jv % VSTAGES;
             tile(jv, true, wv, sV + (uint32_t)(st * TILE), bar(B_VL + st));
             ++jv;
+            idle0 = -1;
             continue;
         }
-        if (jk < n_kv) {
-            const uint32_t ph = (uint32_t)((jk / KSTAGES) - 1) & 1u;
-            mbar_wait(bar(B_KE + jk % KSTAGES), ph, P.err, abort);
-            if (writer) mbar_wait(bar(B_KW + jk % KSTAGES), ph, P.err, abort);
-        } else {
-            const uint32_t ph = (uint32_t)((jv / VSTAGES) - 1) & 1u;
-            mbar_wait(bar(B_VE + jv % VSTAGES), ph, P.err, abort);
-            if (writer) mbar_wait(bar(B_VW + jv % VSTAGES), ph, P.err, abort);
+        // nothing issuable: poll both rings again, within the wait limit
+        if (*abort) return;
+        const long long now = clock64();
+        if (idle0 < 0) {
+            idle0 = now;
+        } else if (now - idle0 > kWaitCycles) {
+            atomicOr(P.err, 2);
+            *abort = 1u;
+            return;
         }
     }
 }
@@ -802,13 +803,12 @@ __device__ __forceinline__ void tma_store_3d(const CUtensorMap* tm, uint32_t src
                  : "memory");
 }
 
-// Store a whole 128-row tile (two 64-channel halves) of a stage to the cache by TMA and wait
-// until the store has read shared memory; the stage is then free for the producer.
-__device__ __forceinline__ void store_tile(const CUtensorMap* tm, uint32_t src, int hk, int row) {
+// Store a whole 128-row tile (two 64-channel halves) of a stage to the cache by TMA, as one
+// bulk async-group (the caller waits for its read of shared memory before freeing the stage).
+__device__ __forceinline__ void issue_store(const CUtensorMap* tm, uint32_t src, int hk, int row) {
     tma_store_3d(tm, src, 0, hk, row);
     tma_store_3d(tm, src + HALF_TILE, 64, hk, row);
     asm volatile("cp.async.bulk.commit_group;" ::: "memory");
-    asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
 }
 
 // Two pairs turned at once on the packed fp32 pipe: per lane exactly rotate1 (the product
@@ -849,7 +849,7 @@ __device__ __forceinline__ uint32_t f2_to_bf2(float lo, float hi) {
 // stage to be free, so they run up to two tiles ahead of the MMA.
 __device__ __forceinline__ void fused_k_loader(const FusedTcParams& F, int lt, int l, int bl, int hk,
                                                bool writer, int j_base, int n_kv, uint32_t sK,
-                                               uint32_t sBar, volatile uint32_t* abort) {
+                                               uint8_t* gK, uint32_t sBar, volatile uint32_t* abort) {
     using bf = __nv_bfloat16;
     const TcParams& P = F.t;
     auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
@@ -872,16 +872,42 @@ __device__ __forceinline__ void fused_k_loader(const FusedTcParams& F, int lt, i
         walk_load(wk, F, o_begin);
         wr = wk;
     }
+    float2* occ_cs = F.occ_cs + (int64_t)l * F.n_occ * 64;    // this layer's table
     int cs_occ = -1;          // occurrence whose angles cc, ss hold
     bool k_turned = false;    // the suffix rows' K' are in the cache
     float2 cc[4], ss[4];      // cos and sin of this thread's 8 frequencies, in pairs
-    // (cos, sin) of the request's occurrences at the 64 frequencies, evaluated once per CTA
-    // into the scratch table (every CTA of the request writes the same values) and read back
-    // as a row per occurrence while turning, instead of evaluating angles per tile
+    auto load_cs = [&](int idx) {
+        const float4* t = reinterpret_cast<const float4*>(occ_cs + idx * 64 + 8 * kc);
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+            const float4 v = t[w];                     // (cos, sin) of two frequencies
+            cc[w] = make_float2(v.x, v.z);
+            ss[w] = make_float2(v.y, v.w);
+        }
+        cs_occ = idx;
+    };
+    // chunk pair (x, y) of a row turned by cc, ss
+    auto turn_pair = [&](const uint4& xa, const uint4& ya, uint4& xo, uint4& yo) {
+        const uint32_t xw[4] = {xa.x, xa.y, xa.z, xa.w}, yw[4] = {ya.x, ya.y, ya.z, ya.w};
+        uint32_t a[4], b[4];
+#pragma unroll
+        for (int w = 0; w < 4; ++w) {
+            float2 gx, gy;
+            rotate2(bf2_to_f2(xw[w]), bf2_to_f2(yw[w]), cc[w], ss[w], gx, gy);
+            a[w] = f2_to_bf2(gx.x, gx.y);
+            b[w] = f2_to_bf2(gy.x, gy.y);
+        }
+        xo = make_uint4(a[0], a[1], a[2], a[3]);
+        yo = make_uint4(b[0], b[1], b[2], b[3]);
+    };
+    // (cos, sin) of the request's occurrences at the 64 frequencies, evaluated while the
+    // first tiles are on their way into this layer's rows of the scratch table (the CTAs of
+    // the layer and request write the same values; a table per layer keeps the CTAs that
+    // write one line few) and read back as a row per occurrence while turning
     {
         const uint64_t turn = F.rope.turn[lt & 63];     // entry e has frequency e % 64 = lt % 64
         for (int e = (o_begin << 6) + lt; e < (o_end << 6); e += kLoaders)
-            F.occ_cs[e] = turn_cs(turn, F.occ[e >> 6].delta);
+            occ_cs[e] = turn_cs(turn, F.occ[e >> 6].delta);
     }
     asm volatile("bar.sync 1, %0;" ::"n"(kLoaders) : "memory");
 
@@ -891,11 +917,19 @@ __device__ __forceinline__ void fused_k_loader(const FusedTcParams& F, int lt, i
         const uint32_t st = sK + (uint32_t)(st_i * TILE);
         if (jt >= KSTAGES)    // stage free: S_A and S_B of tile jt - KSTAGES finished
             mbar_wait(bar(B_KE + st_i), (uint32_t)((jt / KSTAGES) - 1) & 1u, P.err, abort);
+        // a tile of one occurrence (the producer moves it whole): no ragged row, one set of
+        // angles, loaded while the tile lands
+        bool whole = false;
+        if (R0 + BN <= n_slots && o_end > o_begin) {
+            walk_to(wk, F, R0, o_end);
+            const int64_t s0 = (int64_t)wk.src + (R0 - wk.beg);
+            whole = wk.beg <= R0 && R0 + BN <= wk.end && s0 >= 0 && s0 + BN <= F.pool_slots;
+        }
 #pragma unroll 1
-        for (int i = 0; i < BN / 16; ++i) {
+        for (int i = 0; i < (whole ? 0 : BN / 16); ++i) {
             const int r = kr0 + 16 * i;
             const int R = R0 + r;
-            if (!group_ragged(wk, F, R, n_slots, used, o_end)) continue;
+            if (R < n_slots && !group_ragged(wk, F, R, n_slots, used, o_end)) continue;
             if (R >= used) {                              // past the suffix: zeros
                 sts128(st + sw_off(r, kc), make_uint4(0u, 0u, 0u, 0u));
                 sts128(st + HALF_TILE + sw_off(r, kc), make_uint4(0u, 0u, 0u, 0u));
@@ -908,7 +942,7 @@ __device__ __forceinline__ void fused_k_loader(const FusedTcParams& F, int lt, i
                 src = pk + ((pool_row0 + slot) * hkv + hk) * HD;
             } else {
                 if (!k_turned) {
-                    mbar_wait(bar(B_QR), 0u, P.err, abort);
+                    mbar_wait(bar(B_SK), 0u, P.err, abort);
                     k_turned = true;
                 }
                 src = ck + ((cache_row0 + R) * hkv + hk) * HD;
@@ -917,40 +951,55 @@ __device__ __forceinline__ void fused_k_loader(const FusedTcParams& F, int lt, i
             cp_async16(st + HALF_TILE + sw_off(r, kc), src + 64 + 8 * kc);
         }
         cp_async_commit();
+        if (whole) {
+            wr = wk;
+            if (wr.idx != cs_occ) load_cs(wr.idx);
+        }
         cp_async_wait<0>();
         mbar_wait(bar(B_KL + st_i), (uint32_t)(jt / KSTAGES) & 1u, P.err, abort);
+        if (whole) {
+            // two rows at a time, plain shared-memory accesses, so that the loads of both
+            // rows are in flight together
+            uint8_t* g = gK + st_i * TILE;
 #pragma unroll 1
-        for (int i = 0; i < BN / 16; ++i) {
-            const int r = kr0 + 16 * i;
-            const int R = R0 + r;
-            if (R >= n_slots) break;                       // suffix rows are already turned
-            if (walk_slot(wr, F, R, o_end) < 0) continue;
-            if (wr.idx != cs_occ) {
-                const float4* t = reinterpret_cast<const float4*>(F.occ_cs + wr.idx * 64 + 8 * kc);
-#pragma unroll
-                for (int w = 0; w < 4; ++w) {
-                    const float4 v = t[w];                 // (cos, sin) of two frequencies
-                    cc[w] = make_float2(v.x, v.z);
-                    ss[w] = make_float2(v.y, v.w);
-                }
-                cs_occ = wr.idx;
+            for (int i = 0; i < BN / 16; i += 2) {
+                uint4* p0 = reinterpret_cast<uint4*>(g + sw_off(kr0 + 16 * i, kc));
+                uint4* p1 = reinterpret_cast<uint4*>(g + sw_off(kr0 + 16 * i + 16, kc));
+                constexpr int kY = HALF_TILE / 16;             // the partner channels' block
+                const uint4 x0 = p0[0], y0 = p0[kY], x1 = p1[0], y1 = p1[kY];
+                uint4 a0, b0, a1, b1;
+                turn_pair(x0, y0, a0, b0);
+                turn_pair(x1, y1, a1, b1);
+                p0[0] = a0;
+                p0[kY] = b0;
+                p1[0] = a1;
+                p1[kY] = b1;
             }
-            const uint32_t a0 = st + sw_off(r, kc);
-            const uint4 xa = lds128(a0), ya = lds128(a0 + HALF_TILE);
-            const uint32_t xw[4] = {xa.x, xa.y, xa.z, xa.w}, yw[4] = {ya.x, ya.y, ya.z, ya.w};
-            uint32_t xo[4], yo[4];
-#pragma unroll
-            for (int w = 0; w < 4; ++w) {
-                float2 gx, gy;
-                rotate2(bf2_to_f2(xw[w]), bf2_to_f2(yw[w]), cc[w], ss[w], gx, gy);
-                xo[w] = f2_to_bf2(gx.x, gx.y);
-                yo[w] = f2_to_bf2(gy.x, gy.y);
-            }
-            sts128(a0, make_uint4(xo[0], xo[1], xo[2], xo[3]));
-            sts128(a0 + HALF_TILE, make_uint4(yo[0], yo[1], yo[2], yo[3]));
             if (pos_writer) {
                 const FusedOcc& o = F.occ[wr.idx];
-                F.pos[row_base + R] = o.delta + min((R - o.dest_row + 1) * o.k, o.n) - 1;
+#pragma unroll 1
+                for (int i = 0; i < BN / 16; ++i) {
+                    const int R = R0 + kr0 + 16 * i;
+                    F.pos[row_base + R] = o.delta + min((R - o.dest_row + 1) * o.k, o.n) - 1;
+                }
+            }
+        } else {
+#pragma unroll 1
+            for (int i = 0; i < BN / 16; ++i) {
+                const int r = kr0 + 16 * i;
+                const int R = R0 + r;
+                if (R >= n_slots) break;                       // suffix rows are already turned
+                if (walk_slot(wr, F, R, o_end) < 0) continue;
+                if (wr.idx != cs_occ) load_cs(wr.idx);
+                const uint32_t a0 = st + sw_off(r, kc);
+                uint4 xo, yo;
+                turn_pair(lds128(a0), lds128(a0 + HALF_TILE), xo, yo);
+                sts128(a0, xo);
+                sts128(a0 + HALF_TILE, yo);
+                if (pos_writer) {
+                    const FusedOcc& o = F.occ[wr.idx];
+                    F.pos[row_base + R] = o.delta + min((R - o.dest_row + 1) * o.k, o.n) - 1;
+                }
             }
         }
         fence_proxy_async();
@@ -958,21 +1007,27 @@ __device__ __forceinline__ void fused_k_loader(const FusedTcParams& F, int lt, i
     }
 }
 
-// The K writer of the fused kernel (warp 2, one thread, writer CTAs): once the K loaders have
+// The writer of the fused kernel (warp 2, one thread, writer CTAs): once the loaders have
 // released a tile, its K' (composed slots and suffix rows turned, zero rows past the suffix)
-// goes to the cache by TMA.
-__device__ __forceinline__ void fused_k_writer(const FusedTcParams& F, int l, int bl, int hk, int j_base,
-                                               int n_kv, uint32_t sK, uint32_t sBar,
-                                               volatile uint32_t* abort) {
+// and its V go to the cache by TMA; both stores are in flight together, and each stage is
+// handed back to the producer as soon as its store has read it.
+__device__ __forceinline__ void fused_writer(const FusedTcParams& F, int l, int bl, int hk, int j_base,
+                                             int n_kv, uint32_t sK, uint32_t sV, uint32_t sBar,
+                                             volatile uint32_t* abort) {
     const TcParams& P = F.t;
     auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
     const int cache_row0 = (int)((int64_t)(P.layer0 + l) * P.rows + P.req[bl].row_base);
     for (int jt = 0; jt < n_kv; ++jt) {
         const int R0 = (j_base + jt) * BN;
-        const int ks = jt % KSTAGES;
+        const int ks = jt % KSTAGES, vs = jt % VSTAGES;
         mbar_wait(bar(B_KF + ks), (uint32_t)(jt / KSTAGES) & 1u, P.err, abort);
-        store_tile(&P.tm_k, sK + (uint32_t)(ks * TILE), hk, cache_row0 + R0);
+        issue_store(&P.tm_k, sK + (uint32_t)(ks * TILE), hk, cache_row0 + R0);
+        mbar_wait(bar(B_VF + vs), (uint32_t)(jt / VSTAGES) & 1u, P.err, abort);
+        issue_store(&P.tm_v, sV + (uint32_t)(vs * TILE), hk, cache_row0 + R0);
+        asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");    // K's store read
         mbar_arrive(bar(B_KW + ks));
+        asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");    // V's
+        mbar_arrive(bar(B_VW + vs));
     }
     asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
 }
@@ -980,10 +1035,10 @@ __device__ __forceinline__ void fused_k_writer(const FusedTcParams& F, int l, in
 // The V loader of the fused kernel (warp 3, lt = 0..31): per key tile, the ragged 8-row
 // groups' rows by cp.async, or zeros past the suffix (thread lt: chunk lt % 16 of rows
 // lt/16 + 2u of each such group), then the tile's TMA part, then the stage is released to
-// the MMA; in the writer CTAs, lane 0 then stores the tile's V to the cache.
+// the MMA and the writer.
 __device__ __forceinline__ void fused_v_loader(const FusedTcParams& F, int lt, int l, int bl, int hk,
-                                               bool writer, int j_base, int n_kv, uint32_t sV,
-                                               uint32_t sBar, volatile uint32_t* abort) {
+                                               int j_base, int n_kv, uint32_t sV, uint32_t sBar,
+                                               volatile uint32_t* abort) {
     using bf = __nv_bfloat16;
     const TcParams& P = F.t;
     auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
@@ -994,7 +1049,6 @@ __device__ __forceinline__ void fused_v_loader(const FusedTcParams& F, int lt, i
     const int o_end = F.req_occ[bl + 1];
     const int64_t hkv = P.hkv;
     const int64_t pool_row0 = (int64_t)lg * F.pool_slots;
-    const int64_t cache_row0 = (int64_t)lg * P.rows + P.req[bl].row_base;
     const int64_t sfx_row0 = ((int64_t)l * P.batch_total + P.b0 + bl) * P.sq - n_slots;
     const bf* pv = static_cast<const bf*>(F.pool_v);
     const bf* sv = static_cast<const bf*>(F.v_suf);
@@ -1034,31 +1088,22 @@ __device__ __forceinline__ void fused_v_loader(const FusedTcParams& F, int lt, i
         mbar_wait(bar(B_VL + st_i), (uint32_t)(jt / VSTAGES) & 1u, P.err, abort);
         fence_proxy_async();
         mbar_arrive(bar(B_VF + st_i));
-        if (writer) {         // writer CTAs: the tile's V to the cache
-            __syncwarp();
-            if (lt == 0) {
-                store_tile(&P.tm_v, sV + (uint32_t)(st_i * TILE), hk, (int)cache_row0 + R0);
-                mbar_arrive(bar(B_VW + st_i));
-            }
-        }
     }
-    if (writer && lt == 0) asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
 }
 
-// generic-proxy writes to global and shared memory become visible to the async proxy (TMA
-// loads of the cache, tensor-core reads of shared memory)
-__device__ __forceinline__ void fence_proxy_async_all() { asm volatile("fence.proxy.async;" ::: "memory"); }
-
 // The suffix preparation of the fused kernel, done by the softmax warps (ts = 0..255) while
-// they wait for their first S tile.  Item (token tt, chunk pair q = ts % 8) evaluates the
-// angles of position L_r + tt at the 8 frequencies of chunk pair q once and turns with them
+// they wait for their first S tile.  Item (token tt, chunk pair q = ts % 8) takes the angles
+// of position L_r + tt at the 8 frequencies of chunk pair q (from the table that
+// suffix_angles_kernel evaluates once per launch) and turns with them
+//   - chunk pair q of the G query rows of token tt in shared memory, for tt in [q_lo, q_hi)
+//     (this CTA's query tokens), once Q has landed; then the MMA issuer is told (B_QR);
 //   - chunk pair q of suffix row tt's K, from k_suf into the cache, for tt in [k_lo, k_hi)
 //     (the suffix rows among this CTA's key tiles; the CTAs of a request write the same
-//     bits), with the row's position in the CTAs that own the positions;
-//   - chunk pair q of the G query rows of token tt in shared memory, for tt in [q_lo, q_hi)
-//     (this CTA's query tokens), once Q has landed.
-// The angles and the rounding are the suffix kernel's.  Then the writes are made visible to
-// the async proxy and the MMA issuer, the producer and the K loaders are told (B_QR).
+//     bits), with the row's position in the CTAs that own the positions; then the K loaders,
+//     which copy these rows into the K tiles, are told (B_SK).
+// The K rows of a thread's first two items are loaded before anything else and their angles
+// kept from the query pass, so the query rows, which the first MMA waits for, go first.  The
+// angles (turn_cs) and the rounding are the suffix kernel's.
 __device__ __forceinline__ void fused_suffix_prep(const FusedTcParams& F, int ts, int l, int bl, int hk,
                                                   int k_lo, int k_hi, int q_lo, int q_hi, bool pos_rows,
                                                   uint32_t sQ, uint32_t sBar, volatile uint32_t* abort) {
@@ -1069,9 +1114,7 @@ __device__ __forceinline__ void fused_suffix_prep(const FusedTcParams& F, int ts
     const int64_t pos0 = (int64_t)rq.l_req + rq.t0;
     const int G = P.group, tq = P.tq;
     const int q = ts & 7;                  // every item of this thread has chunk pair q
-    uint64_t turn[8];
-#pragma unroll
-    for (int j = 0; j < 8; ++j) turn[j] = F.rope.turn[8 * q + j];
+    const float2* tab = F.sfx_cs + (int64_t)bl * P.sq * 64 + 8 * q;
     const int64_t row_elems = (int64_t)P.hkv * HD;
     const bf* ksrc = static_cast<const bf*>(F.k_suf) +
                      ((int64_t)l * P.batch_total + P.b0 + bl) * P.sq * row_elems + hk * HD + 8 * q;
@@ -1086,65 +1129,130 @@ __device__ __forceinline__ void fused_suffix_prep(const FusedTcParams& F, int ts
         lo = hi > lo ? min(lo, q_lo) : q_lo;
         hi = max(hi, q_hi);
     }
-    bool q_landed = false;
-#pragma unroll 1
-    for (int i = ts; i < (hi - lo) * 8; i += 256) {
-        const int tt = lo + (i >> 3);
-        const bool do_k = tt >= k_lo && tt < k_hi;
-        const bool do_q = tt >= q_lo && tt < q_hi;
-        uint4 xa = make_uint4(0u, 0u, 0u, 0u), ya = xa;
-        if (do_k) {
-            xa = ld16(ksrc + tt * row_elems);
-            ya = ld16(ksrc + tt * row_elems + 64);
-        }
-        float2 cc[4], ss[4];
+    const int n_items = (hi - lo) * 8;     // item i: token lo + i / 8, chunk pair i % 8
+    // (cos, sin) of token tt at chunk pair q's 8 frequencies, from the table of the grid
+    // launched before this one (read from L2)
+    auto angles = [&](int tt, float2 (&cc)[4], float2 (&ss)[4]) {
+        const float4* t = reinterpret_cast<const float4*>(tab + (int64_t)tt * 64);
 #pragma unroll
         for (int w = 0; w < 4; ++w) {
-            const float2 c0 = turn_cs(turn[2 * w], pos0 + tt);
-            const float2 c1 = turn_cs(turn[2 * w + 1], pos0 + tt);
-            cc[w] = make_float2(c0.x, c1.x);
-            ss[w] = make_float2(c0.y, c1.y);
+            const float4 v = __ldcg(t + w);
+            cc[w] = make_float2(v.x, v.z);
+            ss[w] = make_float2(v.y, v.w);
         }
-        auto turn_chunks = [&](const uint4& xv, const uint4& yv, uint4& xo, uint4& yo) {
-            const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w}, yw[4] = {yv.x, yv.y, yv.z, yv.w};
-            uint32_t a[4], b[4];
+    };
+    auto turn_chunks = [&](const uint4& xv, const uint4& yv, const float2 (&cc)[4], const float2 (&ss)[4],
+                           uint4& xo, uint4& yo) {
+        const uint32_t xw[4] = {xv.x, xv.y, xv.z, xv.w}, yw[4] = {yv.x, yv.y, yv.z, yv.w};
+        uint32_t a[4], b[4];
 #pragma unroll
-            for (int w = 0; w < 4; ++w) {
-                float2 gx, gy;
-                rotate2(bf2_to_f2(xw[w]), bf2_to_f2(yw[w]), cc[w], ss[w], gx, gy);
-                a[w] = f2_to_bf2(gx.x, gx.y);
-                b[w] = f2_to_bf2(gy.x, gy.y);
-            }
-            xo = make_uint4(a[0], a[1], a[2], a[3]);
-            yo = make_uint4(b[0], b[1], b[2], b[3]);
-        };
-        if (do_k) {
-            uint4 xo, yo;
-            turn_chunks(xa, ya, xo, yo);
-            st16(kdst + tt * row_elems, xo);
-            st16(kdst + tt * row_elems + 64, yo);
-            if (pos_rows && q == 0) F.pos[rq.row_base + rq.n_slots + tt] = (int32_t)(pos0 + tt);
+        for (int w = 0; w < 4; ++w) {
+            float2 gx, gy;
+            rotate2(bf2_to_f2(xw[w]), bf2_to_f2(yw[w]), cc[w], ss[w], gx, gy);
+            a[w] = f2_to_bf2(gx.x, gx.y);
+            b[w] = f2_to_bf2(gy.x, gy.y);
         }
-        if (do_q) {
-            if (!q_landed) {
-                mbar_wait(bar(B_Q), 0u, P.err, abort);
-                q_landed = true;
-            }
-            const int x = (tt - q_lo) / tq;           // tile A or B
-            const int u = tt - q_lo - x * tq;         // token within the tile
-            const uint32_t base = sQ + (uint32_t)x * TILE;
+        xo = make_uint4(a[0], a[1], a[2], a[3]);
+        yo = make_uint4(b[0], b[1], b[2], b[3]);
+    };
+    auto is_k = [&](int tt) { return tt >= k_lo && tt < k_hi; };
+    auto is_q = [&](int tt) { return tt >= q_lo && tt < q_hi; };
+    bool q_landed = false;
+    auto q_item = [&](int tt, const float2 (&cc)[4], const float2 (&ss)[4]) {
+        if (!q_landed) {
+            mbar_wait(bar(B_Q), 0u, P.err, abort);
+            q_landed = true;
+        }
+        const int x = (tt - q_lo) / tq;           // tile A or B
+        const int t = tt - q_lo - x * tq;         // token within the tile
+        const uint32_t base = sQ + (uint32_t)x * TILE;
 #pragma unroll 1
-            for (int g = 0; g < G; ++g) {
-                const uint32_t a0 = base + sw_off(u * G + g, q);
-                uint4 xo, yo;
-                turn_chunks(lds128(a0), lds128(a0 + HALF_TILE), xo, yo);
-                sts128(a0, xo);
-                sts128(a0 + HALF_TILE, yo);
-            }
+        for (int g = 0; g < G; ++g) {
+            const uint32_t a0 = base + sw_off(t * G + g, q);
+            uint4 xo, yo;
+            turn_chunks(lds128(a0), lds128(a0 + HALF_TILE), cc, ss, xo, yo);
+            sts128(a0, xo);
+            sts128(a0 + HALF_TILE, yo);
         }
+    };
+    auto k_item = [&](int tt, const uint4& xa, const uint4& ya, const float2 (&cc)[4],
+                      const float2 (&ss)[4]) {
+        uint4 xo, yo;
+        turn_chunks(xa, ya, cc, ss, xo, yo);
+        st16(kdst + tt * row_elems, xo);
+        st16(kdst + tt * row_elems + 64, yo);
+        if (pos_rows && q == 0) F.pos[rq.row_base + rq.n_slots + tt] = (int32_t)(pos0 + tt);
+    };
+    // the first two items: their K rows are loaded first and stay in flight while the query
+    // rows are turned, and their angles are kept for the K pass
+    const int t_0 = lo + (ts >> 3), t_1 = t_0 + 32;
+    const bool v0 = ts < n_items, v1 = ts + 256 < n_items;
+    const bool k0 = v0 && is_k(t_0), k1 = v1 && is_k(t_1);
+    uint4 x0 = make_uint4(0u, 0u, 0u, 0u), y0 = x0, x1 = x0, y1 = x0;
+    if (k0) {
+        x0 = ld16(ksrc + t_0 * row_elems);
+        y0 = ld16(ksrc + t_0 * row_elems + 64);
     }
-    fence_proxy_async_all();
+    if (k1) {
+        x1 = ld16(ksrc + t_1 * row_elems);
+        y1 = ld16(ksrc + t_1 * row_elems + 64);
+    }
+    float2 c0[4], s0[4], c1[4], s1[4];
+    // the table's grid has finished and its writes are visible (returns at once when this
+    // grid was launched after it completed)
+    if (n_items > 0) asm volatile("griddepcontrol.wait;" ::: "memory");
+    if (v0) {
+        angles(t_0, c0, s0);
+        if (is_q(t_0)) q_item(t_0, c0, s0);
+    }
+    if (v1) {
+        angles(t_1, c1, s1);
+        if (is_q(t_1)) q_item(t_1, c1, s1);
+    }
+#pragma unroll 1
+    for (int i = ts + 512; i < n_items; i += 256) {
+        const int tt = lo + (i >> 3);
+        if (!is_q(tt)) continue;
+        float2 cc[4], ss[4];
+        angles(tt, cc, ss);
+        q_item(tt, cc, ss);
+    }
+    fence_proxy_async();
     mbar_arrive(bar(B_QR));
+    if (k0) k_item(t_0, x0, y0, c0, s0);
+    if (k1) k_item(t_1, x1, y1, c1, s1);
+#pragma unroll 1
+    for (int i = ts + 512; i < n_items; i += 256) {
+        const int tt = lo + (i >> 3);
+        if (!is_k(tt)) continue;
+        const uint4 xa = ld16(ksrc + tt * row_elems), ya = ld16(ksrc + tt * row_elems + 64);
+        float2 cc[4], ss[4];
+        angles(tt, cc, ss);
+        k_item(tt, xa, ya, cc, ss);
+    }
+    mbar_arrive(bar(B_SK));    // the K loaders read these rows with cp.async (generic proxy)
+}
+
+// The table of the suffix tokens' (cos, sin) at the 64 frequencies, [B][Sq][64], evaluated once
+// per fused launch (turn_cs, as the suffix kernel evaluates them) rather than by each of the
+// request's CTAs.  It lets the dependent fused grid start at once (programmatic dependent
+// launch): only the fused kernel's softmax warps wait for it, the pool loads and the K
+// rotation do not.
+struct SfxAngles {
+    float2* tab;
+    int32_t sq, batch;
+    RopeTurns rope;
+    ReqParam req[kMaxReq];
+};
+__global__ void __launch_bounds__(256) suffix_angles_kernel(const __grid_constant__ SfxAngles A) {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    const int64_t n = (int64_t)A.batch * A.sq * 64;
+    for (int64_t e = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; e < n; e += (int64_t)gridDim.x * blockDim.x) {
+        const int64_t bt = e >> 6;                       // request * Sq + token
+        const int b = (int)(bt / A.sq);
+        const int tt = (int)(bt - (int64_t)b * A.sq);
+        A.tab[e] = turn_cs(A.rope.turn[e & 63], (int64_t)A.req[b].l_req + A.req[b].t0 + tt);
+    }
 }
 
 template <bool kFused>
@@ -1212,6 +1320,7 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
             mbar_init(bar(B_VW + s), 1);
         }
         mbar_init(bar(B_QR), 256u);
+        mbar_init(bar(B_SK), 256u);
         mbar_init(bar(B_OD), 1);
         *abort = 0u;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -1247,34 +1356,43 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
                 fused_producer(KP, l, bl, hk, j_base, n_kv, writer, sK, sV, sBar, abort);
             } else {
                 const int key0 = (int)((int64_t)(P.layer0 + l) * P.rows + P.req[bl].row_base) + j_base * BN;
-                // two independent queues: a K load waits only for its own K stage
+                // two independent queues: a K load waits only for its own K stage, and the
+                // thread serves whichever ring frees a stage first
                 int jk = 0, jv = 0;
+                long long idle0 = -1;
                 while (jk < n_kv || jv < n_kv) {
-                    if (jk < n_kv && (jk < KSTAGES || mbar_try(bar(B_KE + jk % KSTAGES),
-                                                              (uint32_t)((jk / KSTAGES) - 1) & 1u))) {
+                    if (jk < n_kv && (jk < KSTAGES || mbar_test(bar(B_KE + jk % KSTAGES),
+                                                               (uint32_t)((jk / KSTAGES) - 1) & 1u))) {
                         const int s = jk % KSTAGES;
                         const int krow = key0 + jk * BN;
                         mbar_expect_tx(bar(B_KF + s), TILE);
                         tma_load_3d(sK + s * TILE, &P.tm_k, 0, hk, krow, bar(B_KF + s));
                         tma_load_3d(sK + s * TILE + HALF_TILE, &P.tm_k, 64, hk, krow, bar(B_KF + s));
                         ++jk;
+                        idle0 = -1;
                         continue;
                     }
-                    if (jv < n_kv && (jv < VSTAGES || mbar_try(bar(B_VE + jv % VSTAGES),
-                                                              (uint32_t)((jv / VSTAGES) - 1) & 1u))) {
+                    if (jv < n_kv && (jv < VSTAGES || mbar_test(bar(B_VE + jv % VSTAGES),
+                                                               (uint32_t)((jv / VSTAGES) - 1) & 1u))) {
                         const int s = jv % VSTAGES;
                         const int vrow = key0 + jv * BN;
                         mbar_expect_tx(bar(B_VF + s), TILE);
                         tma_load_3d(sV + s * TILE, &P.tm_v, 0, hk, vrow, bar(B_VF + s));
                         tma_load_3d(sV + s * TILE + HALF_TILE, &P.tm_v, 64, hk, vrow, bar(B_VF + s));
                         ++jv;
+                        idle0 = -1;
                         continue;
                     }
-                    // nothing issuable: wait (bounded) for the stage the next K load needs
-                    if (jk < n_kv)
-                        mbar_wait(bar(B_KE + jk % KSTAGES), (uint32_t)((jk / KSTAGES) - 1) & 1u, P.err, abort);
-                    else
-                        mbar_wait(bar(B_VE + jv % VSTAGES), (uint32_t)((jv / VSTAGES) - 1) & 1u, P.err, abort);
+                    // nothing issuable: poll both rings again, within the wait limit
+                    if (*abort) break;
+                    const long long now = clock64();
+                    if (idle0 < 0) {
+                        idle0 = now;
+                    } else if (now - idle0 > kWaitCycles) {
+                        atomicOr(P.err, 2);
+                        *abort = 1u;
+                        break;
+                    }
                 }
             }
         } else if (warp == 1 && lane == 0 && n_kv > 0) {
@@ -1284,12 +1402,12 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
             else
                 mma_issuer<false>(P, tmem, sQ, sK, sV, sBar, n_kv, kFused ? B_QR : B_Q, abort);
         } else if (warp == 2 && lane == 0 && n_kv > 0 && writer) {
-            // ------------------------------------------------------------ K writer (fused)
-            if constexpr (kFused) fused_k_writer(KP, l, bl, hk, j_base, n_kv, sK, sBar, abort);
+            // ------------------------------------------------------------ writer (fused)
+            if constexpr (kFused) fused_writer(KP, l, bl, hk, j_base, n_kv, sK, sV, sBar, abort);
         } else if (warp == 3 && n_kv > 0) {
             // ------------------------------------------------------------ V loader (fused)
             if constexpr (kFused)
-                fused_v_loader(KP, lane, l, bl, hk, writer, j_base, n_kv, sV, sBar, abort);
+                fused_v_loader(KP, lane, l, bl, hk, j_base, n_kv, sV, sBar, abort);
         }
     } else if (warp < 12) {
         asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kFused ? kRegsHighFused : kRegsHigh));
@@ -1299,7 +1417,7 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
             // the suffix rows among this CTA's key tiles, and its query tokens
             const int k_lo = max(0, j_base * BN - s_r);
             const int k_hi = min(P.sq, (j_base + n_kv) * BN - s_r);
-            const int q_hi = n_kv > 0 ? t_last + 1 : t0a;
+            const int q_hi = n_kv > 0 ? t_last + 1 : t0a;   // (the loaders run iff n_kv > 0)
             fused_suffix_prep(KP, (int)threadIdx.x - 128, l, bl, hk, k_lo, k_hi, t0a, q_hi,
                               writer && P.layer0 + l == 0 && hk == 0, sQ, sBar, abort);
         }
@@ -1312,7 +1430,7 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
             // ------------------------------------------------------------ loaders (fused)
             if (n_kv > 0)
                 fused_k_loader(KP, (int)threadIdx.x - 12 * 32, l, bl, hk, writer, j_base, n_kv, sK,
-                               sBar, abort);
+                               smem + 2 * TILE, sBar, abort);
         }
     }
 
@@ -1520,6 +1638,7 @@ cudaError_t launch_attn_tc(const AttnParams& a, cudaStream_t s, Hook before) {
 
 namespace {
 thread_local FusedTcParams g_fused;          // the prepared launch (18 KB: kept off the stack)
+thread_local SfxAngles g_angles;
 thread_local dim3 g_fused_grid;
 thread_local bool g_fused_ready = false;
 }  // namespace
@@ -1536,7 +1655,7 @@ cudaError_t prepare_attn_fused(const AttnParams& a, const FusedSpec& f) {
     const int64_t crow = (int64_t)a.lq * a.rows;
     const int64_t srow = (int64_t)a.lq * a.batch_total * a.sq;
     if (prow > 0x7fffffffLL || crow > 0x7fffffffLL || srow > 0x7fffffffLL) return cudaErrorInvalidValue;
-    if (!f.k_suf || !f.v_suf || !f.occ_cs) return cudaErrorInvalidValue;
+    if (!f.k_suf || !f.v_suf || !f.occ_cs || !f.sfx_cs) return cudaErrorInvalidValue;
     const cuuint64_t str[2] = {(cuuint64_t)HD * 2, (cuuint64_t)a.hkv * HD * 2};
     const cuuint32_t box128[3] = {64, 1, (cuuint32_t)BN};
     const cuuint32_t box64[3] = {64, 1, 64};
@@ -1562,15 +1681,11 @@ cudaError_t prepare_attn_fused(const AttnParams& a, const FusedSpec& f) {
             key_hkv = a.hkv;
         }
     }
-    {   // suffix V [Lq*Btot*Sq][Hkv][128] in 128-, 64- and 8-row boxes, cache K [L*rows][Hkv]
-        // [128] in 64- and 8-row boxes (its 128-row map: prepare_tc)
+    {   // suffix V [Lq*Btot*Sq][Hkv][128] in 128-, 64- and 8-row boxes
         const cuuint64_t sdims[3] = {HD, (cuuint64_t)a.hkv, (cuuint64_t)srow};
-        const cuuint64_t cdims[3] = {HD, (cuuint64_t)a.hkv, (cuuint64_t)crow};
         if (!encode(&p.tm_sv, f.v_suf, 3, sdims, str, box128) ||
             !encode(&p.tm_sv64, f.v_suf, 3, sdims, str, box64) ||
-            !encode(&p.tm_sv8, f.v_suf, 3, sdims, str, box8) ||
-            !encode(&p.tm_ck64, a.cache_k, 3, cdims, str, box64) ||
-            !encode(&p.tm_ck8, a.cache_k, 3, cdims, str, box8))
+            !encode(&p.tm_sv8, f.v_suf, 3, sdims, str, box8))
             return cudaErrorInvalidValue;
     }
     p.pool_k = f.pool_k;
@@ -1581,6 +1696,13 @@ cudaError_t prepare_attn_fused(const AttnParams& a, const FusedSpec& f) {
     p.cache_v = const_cast<void*>(a.cache_v);
     p.pos = f.pos;
     p.occ_cs = f.occ_cs;
+    p.sfx_cs = f.sfx_cs;
+    p.n_occ = f.req_occ[a.batch];
+    g_angles.tab = f.sfx_cs;
+    g_angles.sq = a.sq;
+    g_angles.batch = a.batch;
+    g_angles.rope = f.rope;
+    std::memcpy(g_angles.req, a.req, sizeof(ReqParam) * (size_t)a.batch);
     p.pool_slots = f.pool_slots;
     p.rope = f.rope;
     std::memcpy(p.req_occ, f.req_occ, sizeof(int32_t) * (size_t)(a.batch + 1));
@@ -1593,7 +1715,24 @@ cudaError_t launch_attn_fused(cudaStream_t s, Hook before) {
     if (!g_fused_ready) return cudaErrorInvalidValue;
     g_fused_ready = false;
     before();
-    attn_tc_kernel<true><<<g_fused_grid, kThreadsFused, kSmemBytes, s>>>(g_fused);
+    // the suffix angles on a few CTAs, then the fused kernel as its programmatic dependent
+    const int64_t n = (int64_t)g_angles.batch * g_angles.sq * 64;
+    const unsigned blocks = (unsigned)std::min<int64_t>(32, (n + 255) / 256);
+    suffix_angles_kernel<<<blocks, 256, 0, s>>>(g_angles);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    cudaLaunchConfig_t cfg{};
+    cfg.gridDim = g_fused_grid;
+    cfg.blockDim = dim3(kThreadsFused);
+    cfg.dynamicSmemBytes = kSmemBytes;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, attn_tc_kernel<true>, g_fused);
+    if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }
 

@@ -869,11 +869,14 @@ c2kv_status c2kv_compose_attend(c2kv_ctx* c, int32_t batch, const int32_t* req_p
                 f.occ[i] = c2kv::FusedOcc{occ[i].src_base, occ[i].dest_row - cache->row_base[r],
                                           occ[i].m, occ[i].delta, occ[i].n, occ[i].k};
             }
-            float2* occ_cs = nullptr;      // (cos, sin) per occurrence and frequency
+            // (cos, sin) per layer, occurrence and frequency, then per suffix token and frequency
+            float2* occ_cs = nullptr;
+            const size_t n_occ_cs = (size_t)c->cfg.layers * std::max<size_t>(occ.size(), 1) * 64;
             e = pool_alloc(c, reinterpret_cast<void**>(&occ_cs),
-                           std::max<size_t>(occ.size(), 1) * 64 * sizeof(float2));
+                           (n_occ_cs + (size_t)batch * n_suffix * 64) * sizeof(float2));
             if (e == cudaSuccess) {
                 f.occ_cs = occ_cs;
+                f.sfx_cs = occ_cs + n_occ_cs;
                 f.k_suf = k_suf;
                 f.v_suf = v_suf;
                 e = attend_run(c, cache, 0, c->cfg.layers, q, k_suf, v_suf, n_suffix, out, lse, &f);

@@ -239,8 +239,10 @@ struct FusedSpec {
     const void* k_suf;       // [L][B][Sq][Hkv][128]: the suffix rows before RoPE (K) and V
     const void* v_suf;
     int32_t* pos;            // [rows]
-    float2* occ_cs;          // scratch [occurrences][64]: (cos, sin) of each occurrence's turn,
-                             // filled by the kernel
+    float2* occ_cs;          // scratch [L][occurrences][64]: (cos, sin) of each occurrence's
+                             // turn, filled by the kernel
+    float2* sfx_cs;          // scratch [B][Sq][64]: (cos, sin) of each suffix token's position,
+                             // filled by a small kernel launched just before
     int64_t pool_slots;
     RopeTurns rope;
     int32_t req_occ[kMaxReq + 1];   // request i of the launch: occurrences [req_occ[i], req_occ[i+1])
