@@ -240,13 +240,18 @@ c2kv_status c2kv_attend(c2kv_ctx* ctx, c2kv_cache* cache, int32_t layer, const v
  *     c2kv_attend(ctx, *cache_out, -1, q, k_suf, v_suf, n_suffix, out, lse)
  * (the composed cache, its positions, the suffix rows, O and lse), for every layer.  On
  * the tensor-core route (bf16, d 128) with every chunk in the device pool, at most 256
- * requests and at most 512 chunk occurrences, one fused kernel does both: the attention
- * reads each composed slot straight from the pool, turns K by its occurrence's offset in
- * shared memory (Sec. 3.2.4 re-rotation) and writes the composed cache as it goes, so the
- * cache is written once and never read back.  Otherwise compose and attention run one after
- * the other.  The context's `fuse` setting chooses (C2KV_FUSE_*): by default the fused
- * kernel runs when each (layer, request, KV head) has one pair of query tiles.  The cache is returned as by c2kv_compose (release it with c2kv_cache_release)
- * and serves later c2kv_decode / c2kv_attend calls.
+ * requests and at most 512 chunk occurrences, one fused kernel does all of it: the
+ * attention reads each composed slot straight from the pool, turns K by its occurrence's
+ * offset in shared memory (Sec. 3.2.4 re-rotation), turns the queries and the suffix keys by
+ * their positions, and writes the composed cache as it goes, so the cache is written once
+ * and never read back (a small kernel before it evaluates the suffix positions' angles).
+ * Otherwise compose and attention run one after the other; with chunks in host memory and
+ * two or more layers, the layers go in groups so that reading one group over the host link
+ * overlaps the attention of the previous one (on a second stream; the call's work still
+ * ends on the context's stream).  The context's `fuse` setting chooses (C2KV_FUSE_*): by
+ * default the fused kernel runs when each (layer, request, KV head) has one pair of query
+ * tiles.  The cache is returned as by c2kv_compose (release it with c2kv_cache_release) and
+ * serves later c2kv_decode / c2kv_attend calls.
  *
  *   batch, req_ptr, chunk_ids, positions, suffix_capacity : as c2kv_compose.
  *   q, k_suf, v_suf, n_suffix, out, lse : as c2kv_attend with layer = -1;
