@@ -196,13 +196,17 @@ __global__ void __launch_bounds__(256) compress_kernel(const __grid_constant__ C
 }
 
 // ---------------------------------------------------------------------------------------
-// suffix preparation.  grid = (batch * Sq suffix rows + batch pad blocks, layers).  A row
-// block forms the row's d/2 (cos, sin) at L_b + t once in shared memory, then turns the
-// Hq query heads into q_rot and the Hkv key heads into the cache row row_base + S_b + t
-// (V copied alongside) for its layer.  A pad block zeroes its request's cache rows from
-// the end of the suffix to the next 128-row boundary, so a key tile that straddles the end
-// reads finite zeros (masked keys must not carry NaN/Inf garbage into P.V).
+// suffix preparation.  grid = (batch * kPadParts pad blocks + batch * Sq suffix rows,
+// layers).  A pad block zeroes every kPadParts-th cache row of its request from the end of
+// the suffix to the next 128-row boundary, so a key tile that straddles the end reads finite
+// zeros (masked keys must not carry NaN/Inf garbage into P.V); the pad blocks come first in
+// the grid and share the work, so that none trails the launch.  A row block issues its
+// loads of the row's Hq query heads and Hkv key/value heads first, forms the row's d/2
+// (cos, sin) at L_b + t in shared memory while they are in flight, then turns the queries
+// into q_rot and the keys into the cache row row_base + S_b + t (V copied alongside).
 // ---------------------------------------------------------------------------------------
+constexpr int kPadParts = 4;
+
 template <typename T, int VPH>
 __global__ void __launch_bounds__(256) suffix_kernel(const __grid_constant__ SuffixParams P) {
     using V = Vec16<T>;
@@ -211,20 +215,22 @@ __global__ void __launch_bounds__(256) suffix_kernel(const __grid_constant__ Suf
     constexpr int D = 2 * HALF;
     __shared__ float2 cs[HALF];
     const int l = blockIdx.y;
-    const int n_rows = P.batch * P.sq;
+    const int n_pad = P.pad_rows ? P.batch * kPadParts : 0;
     const int64_t row_elems = (int64_t)P.hkv * D;
-    if ((int)blockIdx.x >= n_rows) {
-        const int bl = blockIdx.x - n_rows;
+    if ((int)blockIdx.x < n_pad) {
+        const int bl = (int)blockIdx.x / kPadParts;
+        const int part = (int)blockIdx.x - bl * kPadParts;
         const int used = P.req[bl].n_slots + P.sq;
         const int end = (used + 127) / 128 * 128;
         constexpr int VPR_ELEMS = 16 / (int)sizeof(T);
         const int vec_per_row = (int)(row_elems / VPR_ELEMS);
-        const int items = (end - used) * vec_per_row;
+        const int rows = end - used > part ? (end - used - part + kPadParts - 1) / kPadParts : 0;
+        const int items = rows * vec_per_row;
         const uint4 z = make_uint4(0, 0, 0, 0);
         for (int it = threadIdx.x; it < items; it += blockDim.x) {
             const int rr = it / vec_per_row;
             const int vi = it - rr * vec_per_row;
-            const int64_t crow = (int64_t)P.req[bl].row_base + used + rr;
+            const int64_t crow = (int64_t)P.req[bl].row_base + used + part + (int64_t)rr * kPadParts;
             if (crow >= P.rows) continue;
             const int64_t off = ((int64_t)(P.layer0 + l) * P.rows + crow) * row_elems + (int64_t)vi * VPR_ELEMS;
             st16(static_cast<T*>(P.cache_k) + off, z);
@@ -232,54 +238,78 @@ __global__ void __launch_bounds__(256) suffix_kernel(const __grid_constant__ Suf
         }
         return;
     }
-    const int bl = blockIdx.x / P.sq;
-    const int t = blockIdx.x - bl * P.sq;
+    const int rb = (int)blockIdx.x - n_pad;
+    const int bl = rb / P.sq;
+    const int t = rb - bl * P.sq;
     const ReqParam& rq = P.req[bl];
     const int64_t position = (int64_t)rq.l_req + rq.t0 + t;      // suffix index t0 + t
-    if (threadIdx.x < HALF) cs[threadIdx.x] = turn_cs(P.rope.turn[threadIdx.x], position);
-    __syncthreads();
     const int64_t crow = (int64_t)rq.row_base + rq.n_slots + rq.t0 + t;
     if (threadIdx.x == 0 && l == 0 && crow >= 0 && crow < P.rows) P.pos[crow] = (int32_t)position;
     const int64_t grow = ((int64_t)l * P.batch_total + P.b0 + bl) * P.sq + t;  // tensor row
     const int nq = P.hq * VPH;
     const int items = (P.hq + P.hkv) * VPH;
-    for (int p = threadIdx.x; p < items; p += blockDim.x) {
+    const bool row_ok = crow >= 0 && crow < P.rows;
+    // item p: query head p / VPH (p < nq) or key/value head (p - nq) / VPH, vector p % VPH
+    struct Item {
+        uint4 a, b, va, vb;   // the two halves of Q or K, and of V
+    };
+    auto load = [&](int p, Item& it) {
         const bool is_q = p < nq;
         const int pp = is_q ? p : p - nq;
         const int h = pp / VPH;
         const int iv = pp - h * VPH;
-        float x[E], y[E], gx[E], gy[E];
         if (is_q) {
-            const int64_t off = (grow * P.hq + h) * D + iv * E;
-            const T* src = static_cast<const T*>(P.q) + off;
-            const uint4 a = ld16(src);
-            const uint4 b = ld16(src + HALF);
-            V::unpack(a, x);
-            V::unpack(b, y);
-            rotate<E>(x, y, cs + iv * E, gx, gy);
-            T* dst = static_cast<T*>(P.q_rot) + off;
+            const T* src = static_cast<const T*>(P.q) + (grow * P.hq + h) * D + iv * E;
+            it.a = ld16(src);
+            it.b = ld16(src + HALF);
+        } else if (row_ok) {
+            const int64_t off = (grow * P.hkv + h) * D + iv * E;
+            const T* ks = static_cast<const T*>(P.k) + off;
+            const T* vs = static_cast<const T*>(P.v) + off;
+            it.a = ld16(ks);
+            it.b = ld16(ks + HALF);
+            it.va = ld16(vs);
+            it.vb = ld16(vs + HALF);
+        }
+    };
+    auto store = [&](int p, const Item& it) {
+        const bool is_q = p < nq;
+        const int pp = is_q ? p : p - nq;
+        const int h = pp / VPH;
+        const int iv = pp - h * VPH;
+        if (!is_q && !row_ok) return;
+        float x[E], y[E], gx[E], gy[E];
+        V::unpack(it.a, x);
+        V::unpack(it.b, y);
+        rotate<E>(x, y, cs + iv * E, gx, gy);
+        if (is_q) {
+            T* dst = static_cast<T*>(P.q_rot) + (grow * P.hq + h) * D + iv * E;
             st16(dst, V::pack(gx));
             st16(dst + HALF, V::pack(gy));
         } else {
-            if (crow < 0 || crow >= P.rows) continue;
-            const int64_t off = (grow * P.hkv + h) * D + iv * E;
             const int64_t coff = ((int64_t)(P.layer0 + l) * P.rows + crow) * row_elems + h * D + iv * E;
-            const T* ks = static_cast<const T*>(P.k) + off;
-            const T* vs = static_cast<const T*>(P.v) + off;
-            const uint4 ka = ld16(ks);
-            const uint4 kb = ld16(ks + HALF);
-            const uint4 va = ld16(vs);
-            const uint4 vb = ld16(vs + HALF);
-            V::unpack(ka, x);
-            V::unpack(kb, y);
-            rotate<E>(x, y, cs + iv * E, gx, gy);
             T* kd = static_cast<T*>(P.cache_k) + coff;
             T* vd = static_cast<T*>(P.cache_v) + coff;
             st16(kd, V::pack(gx));
             st16(kd + HALF, V::pack(gy));
-            st16(vd, va);
-            st16(vd + HALF, vb);
+            st16(vd, it.va);
+            st16(vd + HALF, it.vb);
         }
+    };
+    // two items per thread per pass, loaded before anything waits on them; the first pass
+    // forms the angles in shared memory while its loads are in flight
+    const int stride = (int)blockDim.x;
+    for (int p0 = 0; p0 < items; p0 += 2 * stride) {
+        const int p1 = p0 + (int)threadIdx.x, p2 = p1 + stride;
+        Item i1{}, i2{};
+        if (p1 < items) load(p1, i1);
+        if (p2 < items) load(p2, i2);
+        if (p0 == 0) {
+            if ((int)threadIdx.x < HALF) cs[threadIdx.x] = turn_cs(P.rope.turn[threadIdx.x], position);
+            __syncthreads();
+        }
+        if (p1 < items) store(p1, i1);
+        if (p2 < items) store(p2, i2);
     }
 }
 
@@ -331,7 +361,7 @@ cudaError_t launch_compress(const CompressParams& p, int dtype, int d, cudaStrea
 cudaError_t launch_suffix_prep(const SuffixParams& p, int dtype, int d, cudaStream_t s) {
     (void)cudaGetLastError();   // report this launch's error only, not a stale one
     if (p.batch < 1 || p.sq < 1 || p.lq < 1) return cudaSuccess;
-    const int64_t blocks = (int64_t)p.batch * p.sq + (p.pad_rows ? p.batch : 0);
+    const int64_t blocks = (int64_t)p.batch * p.sq + (p.pad_rows ? (int64_t)p.batch * kPadParts : 0);
     if (blocks > 0x7fffffffLL || p.lq > 65535) return cudaErrorInvalidValue;
     const dim3 grid((unsigned)blocks, p.lq);
     C2KV_DISPATCH(suffix_kernel, grid, p, dtype, d, s);
