@@ -139,6 +139,25 @@ def test_fused_long_suffix_across_tiles():
     _fused_case(wl)
 
 
+@pytest.mark.parametrize("group", [1, 2, 16])
+def test_fused_query_head_groups(group):
+    # G query heads per KV head: a Q tile packs 128 / G tokens, so the suffix preparation's
+    # items (token, chunk pair) turn G rows each; 2 KV heads keep the case small
+    wl = synth.scaled(L8B, layers=2, n_q_heads=2 * group, n_kv_heads=2, chunk_tokens=300,
+                      ratio_k=4, chunks_per_request=3, pool_chunks=3, n_suffix=50)
+    _fused_case(wl)
+
+
+@pytest.mark.parametrize("n_suffix", [1, 128, 129])
+def test_fused_suffix_at_tile_edges(n_suffix):
+    # 256 composed slots (two whole tiles): a suffix of 128 is one whole suffix tile (V by a
+    # 128-row box, K' by cp.async), 129 adds a tile of one suffix row and 127 zero rows, 1 is
+    # a tile of one row
+    wl = synth.scaled(L8B, layers=2, chunk_tokens=512, ratio_k=4, chunks_per_request=2,
+                      pool_chunks=2, n_suffix=n_suffix)
+    _fused_case(wl)
+
+
 @pytest.mark.parametrize("split", [2, 5])
 def test_fused_key_range_splits(split):
     wl = synth.scaled(L8B, layers=1, chunk_tokens=512, ratio_k=2, chunks_per_request=3,
