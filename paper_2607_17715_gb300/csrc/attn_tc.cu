@@ -845,7 +845,7 @@ __device__ __forceinline__ uint32_t f2_to_bf2(float lo, float hi) {
 // produces; suffix rows from the cache, once the softmax warps have turned them) and zeroes
 // those past the suffix, waits for the tile's TMA part, turns its chunks of composed slots
 // by their occurrence's offset (the writer CTAs in layer 0, KV head 0 also write the slots'
-// positions), and releases the stage to the MMA and the K writer.  They wait only for a K
+// positions), and releases the stage to the MMA and the writer.  They wait only for a K
 // stage to be free, so they run up to two tiles ahead of the MMA.
 __device__ __forceinline__ void fused_k_loader(const FusedTcParams& F, int lt, int l, int bl, int hk,
                                                bool writer, int j_base, int n_kv, uint32_t sK,
