@@ -272,6 +272,46 @@ def test_fuse_policy(n_suffix, fuse, want_fused):
         c2kv.c2kv_destroy(ctx)
 
 
+def test_fused_traced_and_on_a_side_stream_give_the_same_bits():
+    # the fused kernel is launched as the dependent of the suffix-angles kernel: with the
+    # library's trace on, events sit between the two, and on another stream the whole call
+    # runs there; the cache, O and lse must not change
+    c2kv = H.lib()
+    wl = synth.scaled(L8B, layers=2, chunks_per_request=3, pool_chunks=3)
+    reqs = synth.requests(wl)
+    chunks = H.oracle_chunks_meanpool(wl, [0, 1, 2])
+    ctx = H.make_ctx(wl, pool_slots=600, fuse=2)
+    try:
+        dev = H.load_stored(ctx, wl, chunks)
+        q, ks, vs = synth.suffix(wl, layers=2)
+        runs = [_run(ctx, wl, dev, reqs, q, ks, vs, wl.n_suffix, fused=True)]
+        c2kv.c2kv_profile_enable(ctx, True)
+        runs.append(_run(ctx, wl, dev, reqs, q, ks, vs, wl.n_suffix, fused=True))
+        assert c2kv.c2kv_profile_read(ctx)["fused"][1] == 1
+        c2kv.c2kv_profile_enable(ctx, False)
+        side = torch.cuda.Stream()
+        with torch.cuda.stream(side):
+            c2kv.c2kv_set_stream(ctx, side)
+            runs.append(_run(ctx, wl, dev, reqs, q, ks, vs, wl.n_suffix, fused=True))
+        torch.cuda.synchronize()
+        c2kv.c2kv_set_stream(ctx, torch.cuda.current_stream())
+        ref = H.cache_arrays(runs[0][0], wl)
+        for cache, out, lse in runs[1:]:
+            got = H.cache_arrays(cache, wl)
+            for r in range(len(reqs)):
+                base, s = ref[0]["row_base"][r], ref[0]["n_slots"][r]
+                end = base + (s + wl.n_suffix + 127) // 128 * 128
+                assert np.array_equal(got[3][base:s + base + wl.n_suffix], ref[3][base:s + base + wl.n_suffix])
+                assert np.array_equal(got[1][:, base:end], ref[1][:, base:end])
+                assert np.array_equal(got[2][:, base:end], ref[2][:, base:end])
+            assert torch.equal(out, runs[0][1])
+            assert torch.equal(lse, runs[0][2])
+        for cache, _, _ in runs:
+            c2kv.c2kv_cache_release(ctx, cache)
+    finally:
+        c2kv.c2kv_destroy(ctx)
+
+
 @pytest.mark.parametrize("n_req,per_req", [(300, 1), (130, 4)])
 def test_compose_attend_many_requests_or_occurrences(n_req, per_req):
     # more than 256 requests, or more than 512 occurrences: the call composes, then attends
