@@ -221,14 +221,17 @@ c2kv_status c2kv_cache_info(const c2kv_cache* cache, c2kv_cache_desc* out);
  * KV head h / G).
  *
  *   layer    : layer index, or -1 for all layers in one launch.
- *   q        : device [Lq][B][n_suffix][Hq][d] pre-RoPE queries (Lq = L if layer == -1,
- *              else 1).
- *   k_suf, v_suf : device [Lq][B][n_suffix][Hkv][d] pre-RoPE suffix K, V.
+ *   q        : [Lq][B][n_suffix][Hq][d] pre-RoPE queries (Lq = L if layer == -1, else 1).
+ *   k_suf, v_suf : [Lq][B][n_suffix][Hkv][d] pre-RoPE suffix K, V.
  *   n_suffix : suffix tokens per request, 1 <= n_suffix <= the cache's suffix_capacity.
- *   out      : device [Lq][B][n_suffix][Hq][d] attention output (context dtype).
- *   lse      : device [Lq][B][Hq][n_suffix] fp32 natural-log softmax normaliser, or NULL.
- * The call is idempotent: it always writes the suffix at rows S_r .. S_r + n_suffix - 1.
- * Errors: ERR_ARG, ERR_STATE (cache from another context), ERR_NOMEM, ERR_CUDA.
+ *   out      : [Lq][B][n_suffix][Hq][d] attention output (context dtype).
+ *   lse      : [Lq][B][Hq][n_suffix] fp32 natural-log softmax normaliser, or NULL.
+ * q, k_suf, v_suf, out and lse are device memory or pinned host memory (page-locked and
+ * mapped, e.g. cudaHostAlloc); host tensors are copied through device scratch on the
+ * context's stream, in and out of the call.  The call is idempotent: it always writes the
+ * suffix at rows S_r .. S_r + n_suffix - 1.
+ * Errors: ERR_ARG (also for a tensor the GPU cannot address), ERR_STATE (cache from another
+ * context), ERR_NOMEM, ERR_CUDA.
  */
 c2kv_status c2kv_attend(c2kv_ctx* ctx, c2kv_cache* cache, int32_t layer, const void* q,
                         const void* k_suf, const void* v_suf, int32_t n_suffix, void* out,
@@ -254,8 +257,10 @@ c2kv_status c2kv_attend(c2kv_ctx* ctx, c2kv_cache* cache, int32_t layer, const v
  * serves later c2kv_decode / c2kv_attend calls.
  *
  *   batch, req_ptr, chunk_ids, positions, suffix_capacity : as c2kv_compose.
- *   q, k_suf, v_suf, n_suffix, out, lse : as c2kv_attend with layer = -1;
- *                1 <= n_suffix <= suffix_capacity.
+ *   q, k_suf, v_suf, n_suffix, out, lse : as c2kv_attend with layer = -1 (device or pinned
+ *                host memory; with chunks in host memory the host tensors move per layer
+ *                group, each group's suffix in while it is composed and its output out while
+ *                the next group is read); 1 <= n_suffix <= suffix_capacity.
  *   cache_out : receives the composed cache.
  * Errors: the union of c2kv_compose's and c2kv_attend's; on error no cache is returned.
  */

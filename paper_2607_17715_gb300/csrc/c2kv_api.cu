@@ -163,6 +163,22 @@ bool is_device_ptr(const void* p) {
 // rows in 16-byte vectors and by TMA, and a misaligned vector access would fault.
 bool aligned(const void* p, uintptr_t a = 16) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
 
+// Where a caller's tensor lives: device (or managed) memory, pinned host memory the GPU
+// reads and writes over the CPU-GPU link, or memory the CUDA runtime does not know
+// (refused: the kernels would dereference it).
+enum class Where { kDevice, kHost, kUnknown };
+Where where(const void* p) {
+    if (!p) return Where::kDevice;
+    cudaPointerAttributes a{};
+    if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+        (void)cudaGetLastError();
+        return Where::kUnknown;
+    }
+    if (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) return Where::kDevice;
+    if (a.type == cudaMemoryTypeHost && a.devicePointer == p) return Where::kHost;
+    return Where::kUnknown;
+}
+
 bool own_cache(const c2kv_ctx* c, const c2kv_cache* cache) {
     return cache && std::find(c->caches.begin(), c->caches.end(), cache) != c->caches.end();
 }
@@ -603,6 +619,10 @@ c2kv_status attend_check(c2kv_ctx* c, const char* what, int32_t layer, const voi
     if (!q || !k_suf || !v_suf || !out) return fail(c, C2KV_ERR_ARG, "%s: null pointer", what);
     if (!aligned(q) || !aligned(k_suf) || !aligned(v_suf) || !aligned(out) || !aligned(lse, 4))
         return fail(c, C2KV_ERR_ARG, "%s: misaligned tensor pointer", what);
+    for (const void* p : {q, k_suf, v_suf, static_cast<const void*>(out), static_cast<const void*>(lse)})
+        if (where(p) == Where::kUnknown)
+            return fail(c, C2KV_ERR_ARG, "%s: tensor in memory the GPU cannot address (neither device "
+                                         "nor pinned, mapped host memory)", what);
     if (layer < -1 || layer >= c->cfg.layers) return fail(c, C2KV_ERR_ARG, "%s: bad layer %d", what, layer);
     if (n_suffix < 1 || n_suffix > suffix_capacity)
         return fail(c, C2KV_ERR_ARG, "%s: n_suffix %d outside [1, %d]", what, n_suffix, suffix_capacity);
@@ -745,6 +765,84 @@ struct StreamSwap {
 // preparation and attention as soon as its composed rows are in, while group g + 1 is read.
 // The call's work ends on the context's stream, and the second stream first waits for the
 // work enqueued there before the call.
+// Suffix tensors and outputs of a call, and where the kernels read and write them: the
+// caller's buffers, or device scratch that copies fill and drain when the caller's are in
+// pinned host memory (the kernels then touch device memory only, and each copy moves in one
+// bulk transfer rather than as the kernels' small accesses across the link).
+struct SuffixIO {
+    const void* q;
+    const void* k;
+    const void* v;
+    void* out;
+    float* lse;
+    bool staged = false;
+    void* scratch = nullptr;
+    size_t q_layer = 0, kv_layer = 0, lse_layer = 0;   // bytes per layer
+};
+
+cudaError_t suffix_io_open(c2kv_ctx* c, int32_t layers, int32_t B, int32_t n_suffix, const void* q,
+                           const void* k_suf, const void* v_suf, void* out, float* lse, SuffixIO* io) {
+    const size_t eb = (size_t)c->eb, d = (size_t)c->cfg.head_dim, L = (size_t)layers;
+    io->q = q;
+    io->k = k_suf;
+    io->v = v_suf;
+    io->out = out;
+    io->lse = lse;
+    io->q_layer = (size_t)B * n_suffix * c->cfg.n_q_heads * d * eb;
+    io->kv_layer = (size_t)B * n_suffix * c->cfg.n_kv_heads * d * eb;
+    io->lse_layer = (size_t)B * c->cfg.n_q_heads * n_suffix * sizeof(float);
+    bool host = false;
+    for (const void* p : {q, k_suf, v_suf, static_cast<const void*>(out), static_cast<const void*>(lse)})
+        host = host || where(p) == Where::kHost;
+    if (!host) return cudaSuccess;
+    // q, out: q_layer each; k, v: kv_layer each; lse: lse_layer (16-byte aligned pieces)
+    auto up = [](size_t x) { return (x + 255) / 256 * 256; };
+    const size_t bytes = L * (2 * up(io->q_layer) + 2 * up(io->kv_layer) + (lse ? up(io->lse_layer) : 0));
+    cudaError_t e = pool_alloc(c, &io->scratch, bytes);
+    if (e != cudaSuccess) return e;
+    char* p = static_cast<char*>(io->scratch);
+    io->q = p;
+    p += L * up(io->q_layer);
+    io->k = p;
+    p += L * up(io->kv_layer);
+    io->v = p;
+    p += L * up(io->kv_layer);
+    io->out = p;
+    p += L * up(io->q_layer);
+    io->lse = lse ? reinterpret_cast<float*>(p) : nullptr;
+    io->staged = true;    // each region holds its L layers at the caller's stride, then padding
+    return cudaSuccess;
+}
+
+// Copy layers [l0, l0 + n) of the staged inputs in (on the context's current stream).
+cudaError_t suffix_io_in(c2kv_ctx* c, const SuffixIO& io, const void* q, const void* k_suf,
+                         const void* v_suf, int32_t l0, int32_t n) {
+    if (!io.staged) return cudaSuccess;
+    cudaError_t e = cudaSuccess;
+    const size_t ql = io.q_layer, kl = io.kv_layer;
+    auto cp = [&](const void* dst, const void* src, size_t bytes) {
+        if (e == cudaSuccess)
+            e = cudaMemcpyAsync(const_cast<void*>(dst), src, bytes, cudaMemcpyDefault, c->stream);
+    };
+    cp(static_cast<const char*>(io.q) + l0 * ql, static_cast<const char*>(q) + l0 * ql, n * ql);
+    cp(static_cast<const char*>(io.k) + l0 * kl, static_cast<const char*>(k_suf) + l0 * kl, n * kl);
+    cp(static_cast<const char*>(io.v) + l0 * kl, static_cast<const char*>(v_suf) + l0 * kl, n * kl);
+    return e;
+}
+
+// Copy layers [l0, l0 + n) of the staged outputs back (on the context's current stream).
+cudaError_t suffix_io_out(c2kv_ctx* c, const SuffixIO& io, void* out, float* lse, int32_t l0, int32_t n) {
+    if (!io.staged) return cudaSuccess;
+    cudaError_t e = cudaMemcpyAsync(static_cast<char*>(out) + l0 * io.q_layer,
+                                    static_cast<const char*>(io.out) + l0 * io.q_layer, n * io.q_layer,
+                                    cudaMemcpyDefault, c->stream);
+    if (e == cudaSuccess && lse)
+        e = cudaMemcpyAsync(reinterpret_cast<char*>(lse) + l0 * io.lse_layer,
+                            reinterpret_cast<const char*>(io.lse) + l0 * io.lse_layer, n * io.lse_layer,
+                            cudaMemcpyDefault, c->stream);
+    return e;
+}
+
 cudaError_t compose_attend_pipelined(c2kv_ctx* c, c2kv_cache* cache, const std::vector<c2kv::OccParam>& occ,
                                      const void* q, const void* k_suf, const void* v_suf,
                                      int32_t n_suffix, void* out, float* lse) {
@@ -765,32 +863,40 @@ cudaError_t compose_attend_pipelined(c2kv_ctx* c, c2kv_cache* cache, const std::
         if (e != cudaSuccess) return e;
         c->aux_ev.push_back(ev);
     }
-    const size_t eb = (size_t)c->eb, d = (size_t)c->cfg.head_dim, B = (size_t)cache->batch;
-    const size_t q_layer = B * n_suffix * c->cfg.n_q_heads * d * eb;       // bytes per layer
-    const size_t kv_layer = B * n_suffix * c->cfg.n_kv_heads * d * eb;
-    const size_t lse_layer = B * c->cfg.n_q_heads * n_suffix;              // floats per layer
+    SuffixIO io;
+    e = suffix_io_open(c, L, cache->batch, n_suffix, q, k_suf, v_suf, out, lse, &io);
+    if (e != cudaSuccess) return e;
+    const size_t lse_floats = io.lse_layer / sizeof(float);               // per layer
     e = cudaEventRecord(c->aux_ev[0], c->stream);                          // the caller's work
     if (e == cudaSuccess) e = cudaStreamWaitEvent(c->aux, c->aux_ev[0], 0);
     for (int32_t g = 0; e == cudaSuccess && g < groups; ++g) {
         const int32_t l0 = g * per;
         const int32_t nl = std::min(per, L - l0);
         if (nl <= 0) break;
+        {   // the group's suffix slices in, on the second stream, while the group is composed
+            StreamSwap on_aux(c, c->aux);
+            e = suffix_io_in(c, io, q, k_suf, v_suf, l0, nl);
+        }
+        if (e != cudaSuccess) break;
         const int max_ctas = std::max(1, c->sms / (4 * nl));                // about a quarter of the SMs
         e = compose_launch(c, cache, occ, l0, nl, max_ctas);
         if (e == cudaSuccess) e = cudaEventRecord(c->aux_ev[1 + g], c->stream);
         if (e == cudaSuccess) e = cudaStreamWaitEvent(c->aux, c->aux_ev[1 + g], 0);
         if (e != cudaSuccess) break;
         StreamSwap on_aux(c, c->aux);
-        e = attend_run(c, cache, l0, nl, static_cast<const char*>(q) + l0 * q_layer,
-                       static_cast<const char*>(k_suf) + l0 * kv_layer,
-                       static_cast<const char*>(v_suf) + l0 * kv_layer, n_suffix,
-                       static_cast<char*>(out) + l0 * q_layer, lse ? lse + l0 * lse_layer : nullptr,
+        e = attend_run(c, cache, l0, nl, static_cast<const char*>(io.q) + l0 * io.q_layer,
+                       static_cast<const char*>(io.k) + l0 * io.kv_layer,
+                       static_cast<const char*>(io.v) + l0 * io.kv_layer, n_suffix,
+                       static_cast<char*>(io.out) + l0 * io.q_layer, io.lse ? io.lse + l0 * lse_floats : nullptr,
                        nullptr);
+        // the group's outputs back while the next group is read
+        if (e == cudaSuccess) e = suffix_io_out(c, io, out, lse, l0, nl);
     }
     // the call ends on the context's stream, after everything on the second stream
     const cudaError_t e2 = cudaEventRecord(c->aux_ev[groups + 1], c->aux);
     if (e2 == cudaSuccess) cudaStreamWaitEvent(c->stream, c->aux_ev[groups + 1], 0);
     if (e != cudaSuccess || e2 != cudaSuccess) cudaStreamSynchronize(c->aux);
+    pool_free(c, io.scratch);
     return e != cudaSuccess ? e : e2;
 }
 
@@ -855,6 +961,24 @@ c2kv_status c2kv_compose_attend(c2kv_ctx* c, int32_t batch, const int32_t* req_p
         for (const auto& o : occ) host_chunks = host_chunks || o.host;
         fuse = fuse && !host_chunks;
         cudaError_t e = cudaSuccess;
+        // suffix tensors and outputs in pinned host memory: copied through device scratch (the
+        // pipelined route does this per layer group itself)
+        SuffixIO io;
+        const bool pipelined = !fuse && host_chunks && c->cfg.layers >= 2;
+        if (!pipelined) {
+            e = suffix_io_open(c, c->cfg.layers, batch, n_suffix, q, k_suf, v_suf, out, lse, &io);
+            if (e == cudaSuccess) e = suffix_io_in(c, io, q, k_suf, v_suf, 0, c->cfg.layers);
+            if (e != cudaSuccess) {
+                pool_free(c, io.scratch);
+                destroy_cache(c, cache);
+                return cuda_fail(c, e, "compose_attend: staging the suffix");
+            }
+        }
+        const void* q_d = pipelined ? q : io.q;
+        const void* k_d = pipelined ? k_suf : io.k;
+        const void* v_d = pipelined ? v_suf : io.v;
+        void* out_d = pipelined ? out : io.out;
+        float* lse_d = pipelined ? lse : io.lse;
         if (fuse) {
             static thread_local c2kv::FusedSpec f;   // 13 KB: kept off the stack
             f.pool_k = c->pool_k;
@@ -877,18 +1001,20 @@ c2kv_status c2kv_compose_attend(c2kv_ctx* c, int32_t batch, const int32_t* req_p
             if (e == cudaSuccess) {
                 f.occ_cs = occ_cs;
                 f.sfx_cs = occ_cs + n_occ_cs;
-                f.k_suf = k_suf;
-                f.v_suf = v_suf;
-                e = attend_run(c, cache, 0, c->cfg.layers, q, k_suf, v_suf, n_suffix, out, lse, &f);
+                f.k_suf = k_d;
+                f.v_suf = v_d;
+                e = attend_run(c, cache, 0, c->cfg.layers, q_d, k_d, v_d, n_suffix, out_d, lse_d, &f);
                 pool_free(c, occ_cs);
             }
-        } else if (host_chunks && c->cfg.layers >= 2) {
+        } else if (pipelined) {
             e = compose_attend_pipelined(c, cache, occ, q, k_suf, v_suf, n_suffix, out, lse);
         } else {
             e = compose_launch(c, cache, occ);
             if (e == cudaSuccess)
-                e = attend_run(c, cache, 0, c->cfg.layers, q, k_suf, v_suf, n_suffix, out, lse, nullptr);
+                e = attend_run(c, cache, 0, c->cfg.layers, q_d, k_d, v_d, n_suffix, out_d, lse_d, nullptr);
         }
+        if (e == cudaSuccess && !pipelined) e = suffix_io_out(c, io, out, lse, 0, c->cfg.layers);
+        if (!pipelined) pool_free(c, io.scratch);
         if (e != cudaSuccess) {
             destroy_cache(c, cache);
             return cuda_fail(c, e, "compose_attend");
@@ -927,8 +1053,15 @@ c2kv_status c2kv_attend(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
         const c2kv_status st =
             attend_check(c, "attend", layer, q, k_suf, v_suf, n_suffix, cache->suffix_capacity, out, lse);
         if (st != C2KV_OK) return st;
-        const cudaError_t e = attend_run(c, cache, layer < 0 ? 0 : layer, layer < 0 ? c->cfg.layers : 1, q,
-                                         k_suf, v_suf, n_suffix, out, lse, nullptr);
+        const int32_t lq = layer < 0 ? c->cfg.layers : 1;
+        SuffixIO io;    // suffix tensors and outputs in pinned host memory: staged through scratch
+        cudaError_t e = suffix_io_open(c, lq, cache->batch, n_suffix, q, k_suf, v_suf, out, lse, &io);
+        if (e == cudaSuccess) e = suffix_io_in(c, io, q, k_suf, v_suf, 0, lq);
+        if (e == cudaSuccess)
+            e = attend_run(c, cache, layer < 0 ? 0 : layer, lq, io.q, io.k, io.v, n_suffix, io.out, io.lse,
+                           nullptr);
+        if (e == cudaSuccess) e = suffix_io_out(c, io, out, lse, 0, lq);
+        pool_free(c, io.scratch);
         if (e != cudaSuccess) return cuda_fail(c, e, "attend");
         return C2KV_OK;
     } catch (const std::bad_alloc&) {

@@ -15,27 +15,35 @@ pytestmark = pytest.mark.gpu
 L8B = synth.workload("llama8b")
 
 
-def _run(ctx, wl, dev, reqs, q, ks, vs, sq, fused):
-    """compose_attend (fused=True) or compose + attend; returns (cache, out, lse)."""
+def _run(ctx, wl, dev, reqs, q, ks, vs, sq, fused, host_io=False):
+    """compose_attend (fused=True) or compose + attend; returns (cache, out, lse) on the
+    device.  host_io: the suffix tensors, O and lse live in pinned host memory."""
     c2kv = H.lib()
     B = len(reqs)
     req_ptr = np.cumsum([0] + [len(ids) for ids, _ in reqs])
     flat = [dev[c] for ids, _ in reqs for c in ids]
     offs = [o for _, o_ in reqs for o in o_]
     qd, kd, vd = (H.to_dev(x, wl) for x in (q, ks, vs))
-    out = torch.full_like(qd, float("nan"))
-    lse = torch.full((wl.layers, B, wl.n_q_heads, sq), float("nan"), device="cuda")
+    if host_io:
+        qd, kd, vd = (x.cpu().pin_memory() for x in (qd, kd, vd))
+        out = torch.empty(qd.shape, dtype=qd.dtype, pin_memory=True).fill_(float("nan"))
+        lse = torch.empty((wl.layers, B, wl.n_q_heads, sq), pin_memory=True).fill_(float("nan"))
+    else:
+        out = torch.full_like(qd, float("nan"))
+        lse = torch.full((wl.layers, B, wl.n_q_heads, sq), float("nan"), device="cuda")
     if fused:
         cache = c2kv.c2kv_compose_attend(ctx, req_ptr, flat, offs, sq, qd, kd, vd, sq, out, lse)
     else:
         cache = c2kv.c2kv_compose(ctx, req_ptr, flat, offs, suffix_capacity=sq)
         c2kv.c2kv_attend(ctx, cache, -1, qd, kd, vd, sq, out, lse)
     c2kv.c2kv_sync(ctx)
+    if host_io:
+        out, lse = out.cuda(), lse.cuda()
     return cache, out, lse
 
 
 def _fused_case(wl, reqs=None, n_suffix=None, attn_split=0, host=(), fixed_pos=False,
-                compare_unfused=True, fuse=2):
+                compare_unfused=True, fuse=2, host_io=False):
     """compose_attend with the fused kernel forced (fuse=2) unless it cannot take the call,
     checked against the oracle and, bit for bit, against compose + attend."""
     c2kv = H.lib()
@@ -53,7 +61,7 @@ def _fused_case(wl, reqs=None, n_suffix=None, attn_split=0, host=(), fixed_pos=F
         B = len(reqs)
         q, ks, vs = synth.suffix(synth.scaled(wl, batch=max(B, wl.batch)), layers=wl.layers)
         q, ks, vs = q[:, :B], ks[:, :B], vs[:, :B]
-        cache, out, lse = _run(ctx, wl, dev, reqs, q, ks, vs, sq, fused=True)
+        cache, out, lse = _run(ctx, wl, dev, reqs, q, ks, vs, sq, fused=True, host_io=host_io)
         info, gk, gv, gpos = H.cache_arrays(cache, wl)
         got = out.double().cpu().numpy()
         got_lse = lse.double().cpu().numpy()
@@ -184,6 +192,41 @@ def test_compose_attend_host_chunks_pipelined(layers):
     wl = synth.scaled(L8B, layers=layers, chunks_per_request=3, pool_chunks=3, n_suffix=20)
     _fused_case(wl, host={0, 1, 2})
     _fused_case(synth.scaled(wl, batch=2, chunks_per_request=2, pool_chunks=4), host={1, 3})
+
+
+@pytest.mark.parametrize("host_chunks", [True, False])
+def test_compose_attend_suffix_and_output_in_host_memory(host_chunks):
+    # Q, K, V of the suffix, O and lse in pinned host memory: the call copies them through
+    # device scratch (per layer group on the pipelined route, around the fused kernel
+    # otherwise) and gives the same bits as compose + attend on device buffers
+    wl = synth.scaled(L8B, layers=5, chunks_per_request=3, pool_chunks=3, n_suffix=20)
+    _fused_case(wl, host={0, 1, 2} if host_chunks else (), host_io=True)
+
+
+def test_compose_attend_refuses_unpinned_host_memory():
+    # a CPU tensor the CUDA runtime does not know is refused before anything is launched
+    c2kv = H.lib()
+    wl = synth.scaled(L8B, layers=1, chunks_per_request=2, pool_chunks=2, n_suffix=8)
+    reqs = synth.requests(wl)
+    chunks = H.oracle_chunks_meanpool(wl, [0, 1])
+    ctx = H.make_ctx(wl, pool_slots=400)
+    try:
+        dev = H.load_stored(ctx, wl, chunks)
+        q, ks, vs = synth.suffix(wl, layers=1)
+        qd, kd, vd = (H.to_dev(x, wl) for x in (q, ks, vs))
+        out_unpinned = torch.empty(qd.shape, dtype=qd.dtype)          # pageable
+        req_ptr = np.cumsum([0] + [len(ids) for ids, _ in reqs])
+        flat = [dev[c] for ids, _ in reqs for c in ids]
+        offs = [o for _, o_ in reqs for o in o_]
+        with pytest.raises(c2kv.C2KVError) as ei:
+            c2kv.c2kv_compose_attend(ctx, req_ptr, flat, offs, 8, qd, kd, vd, 8, out_unpinned)
+        assert ei.value.status == c2kv.ERR_ARG
+        # the context still works
+        cache, out, _ = _run(ctx, wl, dev, reqs, q, ks, vs, 8, fused=True)
+        assert torch.isfinite(out.float()).all()
+        c2kv.c2kv_cache_release(ctx, cache)
+    finally:
+        c2kv.c2kv_destroy(ctx)
 
 
 def test_fused_bounds_check_reports_and_recovers():
