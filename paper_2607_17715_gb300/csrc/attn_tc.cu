@@ -59,6 +59,7 @@
 #include <math_constants.h>
 
 #include <algorithm>
+#include <cstdlib>
 #include <cstring>
 
 #include "internal.cuh"
@@ -114,7 +115,9 @@ constexpr int B_KW = B_VL + VSTAGES;     // + stage (fused): K' of the stage's t
 constexpr int B_VW = B_KW + KSTAGES;     // + stage (fused): V of the stage's tile stored
 constexpr int B_QR = B_VW + VSTAGES;     // (fused) Q turned in shared memory
 constexpr int B_SK = B_QR + 1;           // (fused) the suffix rows' K' turned into the cache
-constexpr int NBAR = B_SK + 1;
+constexpr int B_QF = B_SK + 1;           // every MMA of a pair has read its Q tiles
+constexpr int B_OE = B_QF + 1;           // a pair's epilogue has read O (pairs run in turn)
+constexpr int NBAR = B_OE + 1;
 
 constexpr int kSmemTiles = 2 /*Q_A, Q_B*/ + KSTAGES + VSTAGES;
 constexpr size_t kSmemBytes = 1024 /*align*/ + (size_t)TILE * kSmemTiles + 8 * NBAR + 16;
@@ -131,6 +134,8 @@ struct TcParams {                // CUtensorMap members carry their own alignmen
     int32_t layer0, lq, batch, batch_total, b0, sq, sq_pitch, hq, hkv, group, tq;
     float scale_log2;
     int32_t n_split;
+    int32_t pairs;           // pairs of query tiles per (layer, request, KV head)
+    int32_t pair_group;      // pairs a CTA runs in turn (1 with key-range splits or fused)
     float* part_o;
     float* part_lse;
     ReqParam req[kMaxReq];
@@ -312,11 +317,15 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
 
 // ------------------------------------------------------------------ kernel
 
-// One softmax thread's work on tile x (A or B) for every key tile, then its epilogue.
-// r = TMEM lane (row within the tile), t0 = first suffix token of the tile.
+// One softmax thread's work on tile x (A or B) for every key tile of a pair, then its
+// epilogue.  r = TMEM lane (row within the tile), t0 = first suffix token of the tile.
+// sf_base: S_x tiles completed in earlier pairs (phase count); od_par: the phase of B_OD that
+// closes this pair; arrive_oe: tell the issuer (B_OE) once O has been read, when the CTA
+// runs further pairs.
 __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, uint32_t sBar, int x,
                                             int quad, int lane, int t0, int l, int bl, int b,
-                                            int hk, int sp, int j_base, int n_kv,
+                                            int hk, int sp, int j_base, int n_kv, uint32_t sf_base,
+                                            uint32_t od_par, bool arrive_oe,
                                             volatile uint32_t* abort) {
     auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
     const int G = P.group;
@@ -332,7 +341,7 @@ __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, u
     float l_run = 0.f;
 
     for (int j = 0; j < n_kv; ++j) {
-        mbar_wait(bar(B_SF + x), (uint32_t)j & 1u, P.err, abort);
+        mbar_wait(bar(B_SF + x), (sf_base + (uint32_t)j) & 1u, P.err, abort);
         tc_fence_after();
         uint32_t sv[4][32];
 #pragma unroll
@@ -406,7 +415,7 @@ __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, u
 
     // ---------------------------------------------------------------- epilogue
     if (n_kv > 0) {
-        mbar_wait(bar(B_OD), 0u, P.err, abort);
+        mbar_wait(bar(B_OD), od_par, P.err, abort);
         tc_fence_after();
     }
     const int t = t0 + r / G;
@@ -462,6 +471,10 @@ __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, u
         if (t < P.sq)
             P.part_lse[(int64_t)sp * part_rows + lse_id] = any ? m_run + log2f(l_run) : -CUDART_INF_F;
     }
+    if (arrive_oe) {          // O has been read out of TMEM: the next pair may overwrite it
+        tc_fence_before();
+        mbar_arrive(bar(B_OE));
+    }
 }
 
 // The MMA issuer (one thread).  The tensor core's queue holds about one MMA, so anything
@@ -471,9 +484,24 @@ __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, u
 // barrier parities advance by selects rather than branches.  Each block waits for its own
 // inputs only: waiting for a later block's P inside an S block would hold that S back until
 // the other tile's softmax finished, putting the two softmaxes in series.
+// Ring positions and phase counts that carry over from one pair of query tiles to the next
+// when a CTA runs several pairs of one (layer, request, KV head) in turn.
+struct RingState {
+    int ks = 0;               // K stage of the next K tile, and its fill parity
+    uint32_t kph = 0u;
+    int vs = 0;               // V stage of the next V tile, and its fill parity
+    uint32_t vph = 0u;
+    uint32_t pa = 0u, pb = 0u;    // P_A, P_B tiles completed in earlier pairs
+};
+
+// The MMA issuer for one pair of query tiles (n_kv >= 1 key tiles).  q_ready / q_par: the
+// barrier phase that says Q is in shared memory.  wait_oe: a previous pair's epilogue must
+// have read O (phase oe_par of B_OE) before this pair's first P.V overwrites it.  B_QF says
+// that every S of the pair has read Q, and B_OD at the end that O is final.
 template <bool kHasB>
 __device__ __forceinline__ void mma_issuer(const TcParams& P, uint32_t tmem, uint32_t sQ, uint32_t sK,
                                            uint32_t sV, uint32_t sBar, int n_kv, int q_ready,
+                                           uint32_t q_par, RingState& st, bool wait_oe, uint32_t oe_par,
                                            volatile uint32_t* abort) {
     static_assert(KSTAGES == 3 && VSTAGES == 2, "the issue schedule assumes 3 K and 2 V stages");
     auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
@@ -508,67 +536,78 @@ __device__ __forceinline__ void mma_issuer(const TcParams& P, uint32_t tmem, uin
         mbar_wait(bar(i), parity, P.err, abort);
         tc_fence_after();
     };
+    auto next_k = [&]() {
+        const bool w = st.ks == KSTAGES - 1;
+        st.ks = w ? 0 : st.ks + 1;
+        st.kph ^= w ? 1u : 0u;
+    };
+    auto next_v = [&]() {
+        const bool w = st.vs == VSTAGES - 1;
+        st.vs = w ? 0 : st.vs + 1;
+        st.vph ^= w ? 1u : 0u;
+    };
     // one key tile j >= 1:  PV_A(j-1)  S_A(j)  PV_B(j-1)  S_B(j)
-    //   ks, kph: K stage and fill parity of tile j;  vs, vph: V stage and parity of tile j-1;
-    //   pp: parity of P_x(j-1);  acc0: 0 only for the first P.V (j == 1)
-    auto tile = [&](int ks, uint32_t kph, int vs, uint32_t vph, uint32_t pp, uint32_t acc0) {
-        const uint64_t dk = dK0 + (uint64_t)ks * kTileDesc;
-        const uint64_t dv = dV0 + (uint64_t)vs * kTileDesc;
-        wait(B_PF + 0, pp);
-        wait(B_VF + vs, vph);
+    //   st.ks, st.kph: K stage and fill parity of tile j;  st.vs, st.vph: V stage and parity
+    //   of tile j-1;  ppa, ppb: parities of P_A(j-1), P_B(j-1);  acc0: 0 only for the first
+    //   P.V of the pair (j == 1), which also waits for the previous epilogue when asked
+    auto tile = [&](uint32_t ppa, uint32_t ppb, uint32_t acc0, bool oe) {
+        const uint64_t dk = dK0 + (uint64_t)st.ks * kTileDesc;
+        const uint64_t dv = dV0 + (uint64_t)st.vs * kTileDesc;
+        wait(B_PF + 0, ppa);
+        wait(B_VF + st.vs, st.vph);
+        if (oe) wait(B_OE, oe_par);
         pv_block(tS_a, dv, tO_a, acc0);
-        wait(B_KF + ks, kph);
+        wait(B_KF + st.ks, st.kph);
         s_block(dQa, dk, tS_a);
         mma_commit(bar(B_SF + 0));
         if (kHasB) {
-            wait(B_PF + 1, pp);
+            wait(B_PF + 1, ppb);
             pv_block(tS_b, dv, tO_b, acc0);
         }
-        mma_commit(bar(B_VE + vs));
+        mma_commit(bar(B_VE + st.vs));
         if (kHasB) {
             s_block(dQb, dk, tS_b);
             mma_commit(bar(B_SF + 1));
         }
-        mma_commit(bar(B_KE + ks));
+        mma_commit(bar(B_KE + st.ks));
     };
 
-    wait(q_ready, 0u);
-    wait(B_KF + 0, 0u);
+    wait(q_ready, q_par);
+    wait(B_KF + st.ks, st.kph);
     // key tile 0: S_A(0), S_B(0)
-    s_block(dQa, dK0, tS_a);
+    const uint64_t dk0 = dK0 + (uint64_t)st.ks * kTileDesc;
+    s_block(dQa, dk0, tS_a);
     mma_commit(bar(B_SF + 0));
     if (kHasB) {
-        s_block(dQb, dK0, tS_b);
+        s_block(dQb, dk0, tS_b);
         mma_commit(bar(B_SF + 1));
     }
-    mma_commit(bar(B_KE + 0));
-    // tiles 1 .. n_kv-1, ring positions advanced without branches
-    int ks = 1, vs = 0;
-    uint32_t kph = 0u, vph = 0u, acc0 = 0u;
+    mma_commit(bar(B_KE + st.ks));
+    next_k();
+    // tiles 1 .. n_kv-1
+    uint32_t acc0 = 0u;
     for (int j = 1; j < n_kv; ++j) {
-        tile(ks, kph, vs, vph, (uint32_t)(j - 1) & 1u, acc0);
+        tile((st.pa + (uint32_t)j - 1u) & 1u, (st.pb + (uint32_t)j - 1u) & 1u, acc0, wait_oe && j == 1);
         acc0 = 1u;
-        const bool kw = ks == KSTAGES - 1;
-        ks = kw ? 0 : ks + 1;
-        kph ^= kw ? 1u : 0u;
-        const bool vw = vs == VSTAGES - 1;
-        vs = vw ? 0 : vs + 1;
-        vph ^= vw ? 1u : 0u;
+        next_k();
+        next_v();
     }
-    // last P.V pair: P_x(n_kv - 1), V stage (n_kv - 1) % 2
-    const int vl = vs;
-    const uint32_t vphl = vph;
-    const uint32_t pl = (uint32_t)(n_kv - 1) & 1u;
-    const uint64_t dvl = dV0 + (uint64_t)vl * kTileDesc;
-    wait(B_PF + 0, pl);
-    wait(B_VF + vl, vphl);
+    mma_commit(bar(B_QF));    // every S of the pair issued: Q is free once they complete
+    // last P.V pair: P_x(n_kv - 1) with V tile n_kv - 1
+    const uint64_t dvl = dV0 + (uint64_t)st.vs * kTileDesc;
+    wait(B_PF + 0, (st.pa + (uint32_t)n_kv - 1u) & 1u);
+    wait(B_VF + st.vs, st.vph);
+    if (wait_oe && n_kv == 1) wait(B_OE, oe_par);
     pv_block(tS_a, dvl, tO_a, acc0);
     if (kHasB) {
-        wait(B_PF + 1, pl);
+        wait(B_PF + 1, (st.pb + (uint32_t)n_kv - 1u) & 1u);
         pv_block(tS_b, dvl, tO_b, acc0);
     }
-    mma_commit(bar(B_VE + vl));
+    mma_commit(bar(B_VE + st.vs));
+    next_v();
     mma_commit(bar(B_OD));
+    st.pa += (uint32_t)n_kv;
+    if (kHasB) st.pb += (uint32_t)n_kv;
 }
 
 // ------------------------------------------------------------------ fused loaders
@@ -1233,6 +1272,100 @@ __device__ __forceinline__ void fused_suffix_prep(const FusedTcParams& F, int ts
     mbar_arrive(bar(B_SK));    // the K loaders read these rows with cp.async (generic proxy)
 }
 
+// The query tokens and key tiles of pair pr of query tiles (split sp of its key range).
+struct PairSpan {
+    int t0a, t0b;       // first suffix token of tile A, of tile B
+    bool has_b;
+    int t_last;         // last suffix token of the pair
+    int j_base, n_kv;   // this split's key tiles: [j_base, j_base + n_kv)
+};
+__device__ __forceinline__ PairSpan pair_span(const TcParams& P, int pr, int sp, int s_r) {
+    PairSpan o;
+    o.t0a = 2 * pr * P.tq;
+    o.t0b = o.t0a + P.tq;
+    o.has_b = o.t0b < P.sq;
+    o.t_last = min(P.sq - 1, (o.has_b ? o.t0b : o.t0a) + P.tq - 1);
+    const int n_kv_all = (s_r + o.t_last + 1 + BN - 1) / BN;
+    const int per_split = (n_kv_all + P.n_split - 1) / P.n_split;
+    o.j_base = sp * per_split;
+    o.n_kv = max(0, min(n_kv_all, o.j_base + per_split) - o.j_base);
+    return o;
+}
+
+// The plain kernel's TMA producer (one thread) for the pairs [p_first, p_first + p_count)
+// that its CTA runs in turn: a pair's Q tiles once the MMAs of the previous pair have read
+// the last ones (B_QF), and the pairs' K and V tiles in order, each as soon as its ring stage
+// is free; whichever of the three can go first goes.
+__device__ __forceinline__ void plain_producer(const TcParams& P, int l, int bl, int b, int hk,
+                                               int p_first, int p_count, int sp, int s_r, uint32_t sQ,
+                                               uint32_t sK, uint32_t sV, uint32_t sBar,
+                                               volatile uint32_t* abort) {
+    auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
+    const int G = P.group;
+    const int qz = l * P.batch_total + b;
+    const int key0 = (int)((int64_t)(P.layer0 + l) * P.rows + P.req[bl].row_base);
+    int qi = 0;                             // next pair whose Q tiles to load
+    int pk = 0, jk = 0, gk = 0;             // K: pair, tile within it, tiles issued in all
+    int pv = 0, jv = 0, gv = 0;             // V: the same
+    PairSpan sk = pair_span(P, p_first, sp, s_r), sv = sk;
+    long long idle0 = -1;                   // start of the current wait for a free stage
+    while (qi < p_count || pk < p_count || pv < p_count) {
+        if (qi < p_count && (qi == 0 || mbar_test(bar(B_QF), (uint32_t)(qi - 1) & 1u))) {
+            const PairSpan sq = pair_span(P, p_first + qi, sp, s_r);
+            mbar_expect_tx(bar(B_Q), sq.has_b ? 2 * TILE : TILE);
+            tma_load_4d(sQ, &P.tm_q, 0, hk * G, sq.t0a, qz, bar(B_Q));
+            tma_load_4d(sQ + HALF_TILE, &P.tm_q, 64, hk * G, sq.t0a, qz, bar(B_Q));
+            if (sq.has_b) {
+                tma_load_4d(sQ + TILE, &P.tm_q, 0, hk * G, sq.t0b, qz, bar(B_Q));
+                tma_load_4d(sQ + TILE + HALF_TILE, &P.tm_q, 64, hk * G, sq.t0b, qz, bar(B_Q));
+            }
+            ++qi;
+            idle0 = -1;
+            continue;
+        }
+        if (pk < p_count && (gk < KSTAGES || mbar_test(bar(B_KE + gk % KSTAGES),
+                                                       (uint32_t)((gk / KSTAGES) - 1) & 1u))) {
+            const int s = gk % KSTAGES;
+            const int krow = key0 + (sk.j_base + jk) * BN;
+            mbar_expect_tx(bar(B_KF + s), TILE);
+            tma_load_3d(sK + s * TILE, &P.tm_k, 0, hk, krow, bar(B_KF + s));
+            tma_load_3d(sK + s * TILE + HALF_TILE, &P.tm_k, 64, hk, krow, bar(B_KF + s));
+            ++gk;
+            if (++jk == sk.n_kv) {
+                jk = 0;
+                if (++pk < p_count) sk = pair_span(P, p_first + pk, sp, s_r);
+            }
+            idle0 = -1;
+            continue;
+        }
+        if (pv < p_count && (gv < VSTAGES || mbar_test(bar(B_VE + gv % VSTAGES),
+                                                       (uint32_t)((gv / VSTAGES) - 1) & 1u))) {
+            const int s = gv % VSTAGES;
+            const int vrow = key0 + (sv.j_base + jv) * BN;
+            mbar_expect_tx(bar(B_VF + s), TILE);
+            tma_load_3d(sV + s * TILE, &P.tm_v, 0, hk, vrow, bar(B_VF + s));
+            tma_load_3d(sV + s * TILE + HALF_TILE, &P.tm_v, 64, hk, vrow, bar(B_VF + s));
+            ++gv;
+            if (++jv == sv.n_kv) {
+                jv = 0;
+                if (++pv < p_count) sv = pair_span(P, p_first + pv, sp, s_r);
+            }
+            idle0 = -1;
+            continue;
+        }
+        // nothing issuable: poll again, within the wait limit
+        if (*abort) return;
+        const long long now = clock64();
+        if (idle0 < 0) {
+            idle0 = now;
+        } else if (now - idle0 > kWaitCycles) {
+            atomicOr(P.err, 2);
+            *abort = 1u;
+            return;
+        }
+    }
+}
+
 // The table of the suffix tokens' (cos, sin) at the 64 frequencies, [B][Sq][64], evaluated once
 // per fused launch (turn_cs, as the suffix kernel evaluates them) rather than by each of the
 // request's CTAs.  It lets the dependent fused grid start at once (programmatic dependent
@@ -1278,23 +1411,24 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
     const int bl = blockIdx.z - l * P.batch;
     const int b = P.b0 + bl;
     const int s_r = P.req[bl].n_slots;
-    // pair of Q tiles, the last first: under a causal mask the later pairs see more keys, so
-    // the longest CTAs start in the first wave
-    const int n_pairs = (int)(gridDim.x / P.n_split);
-    const int pr = n_pairs - 1 - (int)(blockIdx.x / P.n_split);
+    // pairs of Q tiles: the CTA runs pairs [p_first, p_first + p_count) in turn (one pair
+    // unless the plain kernel groups short pairs); the groups go last first: under a causal
+    // mask the later pairs see more keys, so the longest CTAs start in the first wave
+    const int n_groups = (int)(gridDim.x / P.n_split);
+    const int p_first = (n_groups - 1 - (int)(blockIdx.x / P.n_split)) * P.pair_group;
+    const int p_count = min(P.pairs, p_first + P.pair_group) - p_first;
     const int sp = (int)(blockIdx.x % P.n_split);   // key-range split
     // fused: the CTAs of the last pair see every key row of the request (all of the suffix),
     // so they write the composed cache
-    const bool writer = pr == n_pairs - 1;
-    const int t0a = 2 * pr * P.tq;
-    const int t0b = t0a + P.tq;
-    const bool has_b = t0b < P.sq;
-    const int t_last = min(P.sq - 1, (has_b ? t0b : t0a) + P.tq - 1);
-    const int n_kv_all = (s_r + t_last + 1 + BN - 1) / BN;
-    // this CTA's key tiles: [j_base, j_base + n_kv) of the request's n_kv_all
-    const int per_split = (n_kv_all + P.n_split - 1) / P.n_split;
-    const int j_base = sp * per_split;
-    const int n_kv = max(0, min(n_kv_all, j_base + per_split) - j_base);
+    const bool writer = p_first == P.pairs - 1;
+    // the first pair (the fused kernel's only one)
+    const PairSpan ps0 = pair_span(P, p_first, sp, s_r);
+    const int t0a = ps0.t0a;
+    const int t0b = ps0.t0b;
+    const bool has_b = ps0.has_b;
+    const int t_last = ps0.t_last;
+    const int j_base = ps0.j_base;
+    const int n_kv = ps0.n_kv;
 
     if (threadIdx.x == 0) {
         mbar_init(bar(B_Q), 1);
@@ -1321,6 +1455,8 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
         }
         mbar_init(bar(B_QR), 256u);
         mbar_init(bar(B_SK), 256u);
+        mbar_init(bar(B_QF), 1u);
+        mbar_init(bar(B_OE), 256u);
         mbar_init(bar(B_OD), 1);
         *abort = 0u;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -1344,63 +1480,37 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&P.tm_q)) : "memory");
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&P.tm_k)) : "memory");
             asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(&P.tm_v)) : "memory");
-            const int qz = l * P.batch_total + b;
-            mbar_expect_tx(bar(B_Q), has_b ? 2 * TILE : TILE);
-            tma_load_4d(sQ, &P.tm_q, 0, hk * G, t0a, qz, bar(B_Q));
-            tma_load_4d(sQ + HALF_TILE, &P.tm_q, 64, hk * G, t0a, qz, bar(B_Q));
-            if (has_b) {
-                tma_load_4d(sQ + TILE, &P.tm_q, 0, hk * G, t0b, qz, bar(B_Q));
-                tma_load_4d(sQ + TILE + HALF_TILE, &P.tm_q, 64, hk * G, t0b, qz, bar(B_Q));
-            }
             if constexpr (kFused) {
+                const int qz = l * P.batch_total + b;
+                mbar_expect_tx(bar(B_Q), has_b ? 2 * TILE : TILE);
+                tma_load_4d(sQ, &P.tm_q, 0, hk * G, t0a, qz, bar(B_Q));
+                tma_load_4d(sQ + HALF_TILE, &P.tm_q, 64, hk * G, t0a, qz, bar(B_Q));
+                if (has_b) {
+                    tma_load_4d(sQ + TILE, &P.tm_q, 0, hk * G, t0b, qz, bar(B_Q));
+                    tma_load_4d(sQ + TILE + HALF_TILE, &P.tm_q, 64, hk * G, t0b, qz, bar(B_Q));
+                }
                 fused_producer(KP, l, bl, hk, j_base, n_kv, writer, sK, sV, sBar, abort);
             } else {
-                const int key0 = (int)((int64_t)(P.layer0 + l) * P.rows + P.req[bl].row_base) + j_base * BN;
-                // two independent queues: a K load waits only for its own K stage, and the
-                // thread serves whichever ring frees a stage first
-                int jk = 0, jv = 0;
-                long long idle0 = -1;
-                while (jk < n_kv || jv < n_kv) {
-                    if (jk < n_kv && (jk < KSTAGES || mbar_test(bar(B_KE + jk % KSTAGES),
-                                                               (uint32_t)((jk / KSTAGES) - 1) & 1u))) {
-                        const int s = jk % KSTAGES;
-                        const int krow = key0 + jk * BN;
-                        mbar_expect_tx(bar(B_KF + s), TILE);
-                        tma_load_3d(sK + s * TILE, &P.tm_k, 0, hk, krow, bar(B_KF + s));
-                        tma_load_3d(sK + s * TILE + HALF_TILE, &P.tm_k, 64, hk, krow, bar(B_KF + s));
-                        ++jk;
-                        idle0 = -1;
-                        continue;
-                    }
-                    if (jv < n_kv && (jv < VSTAGES || mbar_test(bar(B_VE + jv % VSTAGES),
-                                                               (uint32_t)((jv / VSTAGES) - 1) & 1u))) {
-                        const int s = jv % VSTAGES;
-                        const int vrow = key0 + jv * BN;
-                        mbar_expect_tx(bar(B_VF + s), TILE);
-                        tma_load_3d(sV + s * TILE, &P.tm_v, 0, hk, vrow, bar(B_VF + s));
-                        tma_load_3d(sV + s * TILE + HALF_TILE, &P.tm_v, 64, hk, vrow, bar(B_VF + s));
-                        ++jv;
-                        idle0 = -1;
-                        continue;
-                    }
-                    // nothing issuable: poll both rings again, within the wait limit
-                    if (*abort) break;
-                    const long long now = clock64();
-                    if (idle0 < 0) {
-                        idle0 = now;
-                    } else if (now - idle0 > kWaitCycles) {
-                        atomicOr(P.err, 2);
-                        *abort = 1u;
-                        break;
-                    }
-                }
+                plain_producer(P, l, bl, b, hk, p_first, p_count, sp, s_r, sQ, sK, sV, sBar, abort);
             }
         } else if (warp == 1 && lane == 0 && n_kv > 0) {
             // ------------------------------------------------------------ MMA issuer
-            if (has_b)
-                mma_issuer<true>(P, tmem, sQ, sK, sV, sBar, n_kv, kFused ? B_QR : B_Q, abort);
-            else
-                mma_issuer<false>(P, tmem, sQ, sK, sV, sBar, n_kv, kFused ? B_QR : B_Q, abort);
+            RingState st;
+            if constexpr (kFused) {          // one pair
+                if (has_b)
+                    mma_issuer<true>(P, tmem, sQ, sK, sV, sBar, n_kv, B_QR, 0u, st, false, 0u, abort);
+                else
+                    mma_issuer<false>(P, tmem, sQ, sK, sV, sBar, n_kv, B_QR, 0u, st, false, 0u, abort);
+            } else {
+                for (int pi = 0; pi < p_count; ++pi) {
+                    const PairSpan ps = pi == 0 ? ps0 : pair_span(P, p_first + pi, sp, s_r);
+                    const uint32_t q_par = (uint32_t)pi & 1u, oe_par = (uint32_t)(pi - 1) & 1u;
+                    if (ps.has_b)
+                        mma_issuer<true>(P, tmem, sQ, sK, sV, sBar, ps.n_kv, B_Q, q_par, st, pi > 0, oe_par, abort);
+                    else
+                        mma_issuer<false>(P, tmem, sQ, sK, sV, sBar, ps.n_kv, B_Q, q_par, st, pi > 0, oe_par, abort);
+                }
+            }
         } else if (warp == 2 && lane == 0 && n_kv > 0 && writer) {
             // ------------------------------------------------------------ writer (fused)
             if constexpr (kFused) fused_writer(KP, l, bl, hk, j_base, n_kv, sK, sV, sBar, abort);
@@ -1421,9 +1531,23 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
             fused_suffix_prep(KP, (int)threadIdx.x - 128, l, bl, hk, k_lo, k_hi, t0a, q_hi,
                               writer && P.layer0 + l == 0 && hk == 0, sQ, sBar, abort);
         }
-        if (x == 0 || has_b)
-            softmax_tile(P, tmem, sBar, x, warp & 3, lane, x ? t0b : t0a, l, bl, b, hk, sp, j_base,
-                         n_kv, abort);
+        if constexpr (kFused) {              // one pair
+            if (x == 0 || has_b)
+                softmax_tile(P, tmem, sBar, x, warp & 3, lane, x ? t0b : t0a, l, bl, b, hk, sp, j_base,
+                             n_kv, 0u, 0u, false, abort);
+        } else {
+            uint32_t done = 0u;     // S_x tiles of the earlier pairs
+            for (int pi = 0; pi < p_count; ++pi) {
+                const PairSpan ps = pi == 0 ? ps0 : pair_span(P, p_first + pi, sp, s_r);
+                if (x == 0 || ps.has_b) {
+                    softmax_tile(P, tmem, sBar, x, warp & 3, lane, x ? ps.t0b : ps.t0a, l, bl, b, hk, sp,
+                                 ps.j_base, ps.n_kv, done, (uint32_t)pi & 1u, p_count > 1, abort);
+                    done += (uint32_t)ps.n_kv;
+                } else if (p_count > 1) {    // no tile B in this pair: nothing of O to read
+                    mbar_arrive(bar(B_OE));
+                }
+            }
+        }
     } else {
         if constexpr (kFused) {
             asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsLowFused));
@@ -1616,7 +1740,29 @@ cudaError_t prepare_tc(const AttnParams& a, TcParams& p, dim3& grid) {
     if (a.batch < 1 || a.batch > kMaxReq) return cudaErrorInvalidValue;
     std::memcpy(p.req, a.req, sizeof(ReqParam) * (size_t)a.batch);
     const int64_t pairs = ((a.sq + tq - 1) / tq + 1) / 2;
-    const int64_t gx = pairs * p.n_split;
+    // The plain kernel runs several pairs of one (layer, request, KV head) per CTA when the
+    // launch is many waves of CTAs: each CTA's fixed cost (TMEM, barriers, the first tiles
+    // from HBM, the epilogue) is then paid once for several short pairs (causal extraction
+    // rows: 1 to 4 key tiles a pair).  C2KV_ATTN_PAIRS_PER_CTA overrides the choice (tests).
+    int64_t pg = 1;
+    if (!kFused && p.n_split == 1) {
+        static int sms = 0;
+        if (sms == 0) {
+            int dev = 0;
+            if (cudaGetDevice(&dev) != cudaSuccess ||
+                cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1)
+                sms = 1;
+        }
+        const int64_t ctas = pairs * a.hkv * a.lq * a.batch;
+        pg = std::max<int64_t>(1, std::min<int64_t>(pairs, ctas / sms));
+        if (const char* env = std::getenv("C2KV_ATTN_PAIRS_PER_CTA")) {
+            const long v = std::strtol(env, nullptr, 10);
+            if (v >= 1) pg = std::min<int64_t>(pairs, v);
+        }
+    }
+    p.pairs = (int32_t)pairs;
+    p.pair_group = (int32_t)pg;
+    const int64_t gx = (pairs + pg - 1) / pg * p.n_split;
     if (gx > 0x7fffffffLL) return cudaErrorInvalidValue;
     grid = dim3((unsigned)gx, a.hkv, a.lq * a.batch);
     if (grid.z > 65535u || grid.y > 65535u) return cudaErrorInvalidValue;

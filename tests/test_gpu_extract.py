@@ -94,6 +94,14 @@ def test_extract_without_lse_matches_with_lse():
         c2kv.c2kv_destroy(ctx)
 
 
+@pytest.mark.parametrize("per_cta", [2, 3, 8])
+def test_extract_pairs_run_in_turn(per_cta, monkeypatch):
+    # the attention launches of the call with several pairs of query tiles per CTA (the
+    # document rows have 8 pairs of 1 to 4 key tiles at n = 512): 3 leaves a group of two
+    monkeypatch.setenv("C2KV_ATTN_PAIRS_PER_CTA", str(per_cta))
+    _extract_case(L8B, 512, 4, layers=1)
+
+
 def test_extract_two_layers_gqa8():
     _extract_case(synth.workload("long70b"), 300, 16, layers=2)
 

@@ -166,6 +166,16 @@ def test_fused_suffix_at_tile_edges(n_suffix):
     _fused_case(wl)
 
 
+@pytest.mark.parametrize("per_cta", [2, 3])
+def test_attend_pairs_run_in_turn(per_cta, monkeypatch):
+    # compose, then attention with several pairs of query tiles per CTA: 200 suffix tokens
+    # are 7 query tiles, i.e. 4 pairs, the last without a tile B
+    monkeypatch.setenv("C2KV_ATTN_PAIRS_PER_CTA", str(per_cta))
+    wl = synth.scaled(L8B, layers=2, chunk_tokens=300, ratio_k=4, chunks_per_request=3,
+                      pool_chunks=3, n_suffix=200)
+    _fused_case(wl, fuse=1)
+
+
 @pytest.mark.parametrize("split", [2, 5])
 def test_fused_key_range_splits(split):
     wl = synth.scaled(L8B, layers=1, chunk_tokens=512, ratio_k=2, chunks_per_request=3,
