@@ -1630,15 +1630,16 @@ bool encode(CUtensorMap* tm, const void* base, int rank, const cuuint64_t* dims,
 bool encode_tensor_map(CUtensorMap* tm, CUtensorMapDataType type, int rank, const void* base,
                        const cuuint64_t* dims, const cuuint64_t* strides_bytes, const cuuint32_t* box,
                        CUtensorMapSwizzle swizzle) {
-    static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
-    if (!fn) {
+    // the driver entry point, looked up once (a function-local static: thread-safe)
+    static const PFN_cuTensorMapEncodeTiled_v12000 fn = []() -> PFN_cuTensorMapEncodeTiled_v12000 {
         void* p = nullptr;
         cudaDriverEntryPointQueryResult q{};
         if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
                                              &q) == cudaSuccess &&
             q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
-    }
+            return reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+        return nullptr;
+    }();
     if (!fn) return false;
     cuuint32_t estr[5] = {1, 1, 1, 1, 1};
     const CUresult r = fn(tm, type, (cuuint32_t)rank, const_cast<void*>(base), dims, strides_bytes, box,
@@ -1679,22 +1680,16 @@ cudaError_t prepare_tc(const AttnParams& a, TcParams& p, dim3& grid) {
     constexpr int low = kFused ? kRegsLowFused : kRegsLow;
     constexpr int high = kFused ? kRegsHighFused : kRegsHigh;
     constexpr int low_threads = kFused ? 256 : 128;
-    cudaError_t e = cudaSuccess;
-    static bool smem_set = false;           // once per process (one device per context)
-    if (!smem_set) {
-        e = cudaFuncSetAttribute(attn_tc_kernel<kFused>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)kSmemBytes);
-        if (e != cudaSuccess) return e;
-        smem_set = true;
-    }
+    // once per process (one device per context; function-local statics: thread-safe)
+    static const cudaError_t smem_err = cudaFuncSetAttribute(
+        attn_tc_kernel<kFused>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+    if (smem_err != cudaSuccess) return smem_err;
     {   // the register split must not ask for more than the launch holds
-        static int launch_regs = -1;
-        if (launch_regs < 0) {
+        static const int launch_regs = []() {
             cudaFuncAttributes fa{};
-            e = cudaFuncGetAttributes(&fa, attn_tc_kernel<kFused>);
-            if (e != cudaSuccess) return e;
-            launch_regs = fa.numRegs;
-        }
+            return cudaFuncGetAttributes(&fa, attn_tc_kernel<kFused>) == cudaSuccess ? fa.numRegs : -1;
+        }();
+        if (launch_regs < 0) return cudaErrorInvalidDeviceFunction;
         if (launch_regs * threads < low_threads * low + 256 * high) return cudaErrorInvalidConfiguration;
     }
     const int pitch = a.sq_pitch > 0 ? a.sq_pitch : a.sq;
@@ -1746,13 +1741,13 @@ cudaError_t prepare_tc(const AttnParams& a, TcParams& p, dim3& grid) {
     // rows: 1 to 4 key tiles a pair).  C2KV_ATTN_PAIRS_PER_CTA overrides the choice (tests).
     int64_t pg = 1;
     if (!kFused && p.n_split == 1) {
-        static int sms = 0;
-        if (sms == 0) {
-            int dev = 0;
+        static const int sms = []() {
+            int dev = 0, n = 0;
             if (cudaGetDevice(&dev) != cudaSuccess ||
-                cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1)
-                sms = 1;
-        }
+                cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n < 1)
+                return 1;
+            return n;
+        }();
         const int64_t ctas = pairs * a.hkv * a.lq * a.batch;
         pg = std::max<int64_t>(1, std::min<int64_t>(pairs, ctas / sms));
         if (const char* env = std::getenv("C2KV_ATTN_PAIRS_PER_CTA")) {

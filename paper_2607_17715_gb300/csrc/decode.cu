@@ -398,14 +398,11 @@ cudaError_t launch_g(const DecodeParams& p, cudaStream_t s, Hook before) {
         if (!encode_tensor_map(&x.tm_v, ty, 3, p.cache_v, dims, str, box, CU_TENSOR_MAP_SWIZZLE_NONE))
             return cudaErrorInvalidValue;
     }
+    // once per instantiation (a function-local static: thread-safe)
+    static const cudaError_t smem_err = cudaFuncSetAttribute(
+        decode_kernel<T, D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kDecSmem);
+    if (smem_err != cudaSuccess) return smem_err;
     cudaError_t e = cudaSuccess;
-    static bool smem_set = false;           // once per instantiation
-    if (!smem_set) {
-        e = cudaFuncSetAttribute(decode_kernel<T, D, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)kDecSmem);
-        if (e != cudaSuccess) return e;
-        smem_set = true;
-    }
     const dim3 grid((unsigned)p.n_split, (unsigned)p.hkv, (unsigned)(p.lq * p.batch));
     before();
     decode_kernel<T, D, G><<<grid, kDecThreadsAll, kDecSmem, s>>>(x);
