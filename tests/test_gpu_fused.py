@@ -213,6 +213,43 @@ def test_compose_attend_suffix_and_output_in_host_memory(host_chunks):
     _fused_case(wl, host={0, 1, 2} if host_chunks else (), host_io=True)
 
 
+def test_attend_one_layer_and_no_lse_with_host_tensors():
+    # c2kv_attend of one layer with its Q, K, V and O in pinned host memory, and
+    # c2kv_compose_attend with host tensors and no lse: the same bits as on device buffers
+    c2kv = H.lib()
+    wl = synth.scaled(L8B, layers=3, chunks_per_request=2, pool_chunks=2, n_suffix=24)
+    reqs = synth.requests(wl)
+    chunks = H.oracle_chunks_meanpool(wl, [0, 1])
+    ctx = H.make_ctx(wl, pool_slots=600, fuse=1)
+    try:
+        dev = H.load_stored(ctx, wl, chunks)
+        q, ks, vs = synth.suffix(wl, layers=3)
+        req_ptr = np.cumsum([0] + [len(ids) for ids, _ in reqs])
+        flat = [dev[c] for ids, _ in reqs for c in ids]
+        offs = [o for _, o_ in reqs for o in o_]
+        qd, kd, vd = (H.to_dev(x, wl) for x in (q, ks, vs))
+        # reference: all layers on device buffers
+        cache = c2kv.c2kv_compose(ctx, req_ptr, flat, offs, suffix_capacity=24)
+        ref = torch.empty_like(qd)
+        c2kv.c2kv_attend(ctx, cache, -1, qd, kd, vd, 24, ref)
+        # layer 1 alone, host buffers
+        qh, kh, vh = (x[1:2].cpu().pin_memory() for x in (qd, kd, vd))
+        oh = torch.empty(qh.shape, dtype=qh.dtype, pin_memory=True)
+        c2kv.c2kv_attend(ctx, cache, 1, qh, kh, vh, 24, oh)
+        c2kv.c2kv_sync(ctx)
+        assert torch.equal(oh.cuda(), ref[1:2])
+        c2kv.c2kv_cache_release(ctx, cache)
+        # compose_attend, host buffers, no lse
+        qh, kh, vh = (x.cpu().pin_memory() for x in (qd, kd, vd))
+        oh = torch.empty(qh.shape, dtype=qh.dtype, pin_memory=True)
+        cache = c2kv.c2kv_compose_attend(ctx, req_ptr, flat, offs, 24, qh, kh, vh, 24, oh)
+        c2kv.c2kv_sync(ctx)
+        assert torch.equal(oh.cuda(), ref)
+        c2kv.c2kv_cache_release(ctx, cache)
+    finally:
+        c2kv.c2kv_destroy(ctx)
+
+
 def test_compose_attend_refuses_unpinned_host_memory():
     # a CPU tensor the CUDA runtime does not know is refused before anything is launched
     c2kv = H.lib()
