@@ -68,7 +68,9 @@ typedef int32_t c2kv_status;
                                  128-row query tiles, n_suffix * Hq / Hkv <= 256: every
                                  stored slot is then read and turned by exactly one CTA   */
 #define C2KV_FUSE_NEVER  1    /* always compose, then attend                           */
-#define C2KV_FUSE_ALWAYS 2    /* whenever the fused kernel takes the call              */
+#define C2KV_FUSE_ALWAYS 2    /* whenever the fused kernel takes the call; with several
+                                 pairs of query tiles one CTA runs them in turn, the last
+                                 pair composing the cache and the others reading it      */
 
 typedef struct c2kv_ctx c2kv_ctx;
 typedef struct c2kv_cache c2kv_cache;

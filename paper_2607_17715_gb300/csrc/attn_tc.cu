@@ -117,7 +117,8 @@ constexpr int B_QR = B_VW + VSTAGES;     // (fused) Q turned in shared memory
 constexpr int B_SK = B_QR + 1;           // (fused) the suffix rows' K' turned into the cache
 constexpr int B_QF = B_SK + 1;           // every MMA of a pair has read its Q tiles
 constexpr int B_OE = B_QF + 1;           // a pair's epilogue has read O (pairs run in turn)
-constexpr int NBAR = B_OE + 1;
+constexpr int B_WD = B_OE + 1;           // (fused, pairs in turn) the first pair's cache stores done
+constexpr int NBAR = B_WD + 1;
 
 constexpr int kSmemTiles = 2 /*Q_A, Q_B*/ + KSTAGES + VSTAGES;
 constexpr size_t kSmemBytes = 1024 /*align*/ + (size_t)TILE * kSmemTiles + 8 * NBAR + 16;
@@ -313,6 +314,26 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
     float d;
     asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
     return d;
+}
+
+// The query tokens and key tiles of pair pr of query tiles (split sp of its key range).
+struct PairSpan {
+    int t0a, t0b;       // first suffix token of tile A, of tile B
+    bool has_b;
+    int t_last;         // last suffix token of the pair
+    int j_base, n_kv;   // this split's key tiles: [j_base, j_base + n_kv)
+};
+__device__ __forceinline__ PairSpan pair_span(const TcParams& P, int pr, int sp, int s_r) {
+    PairSpan o;
+    o.t0a = 2 * pr * P.tq;
+    o.t0b = o.t0a + P.tq;
+    o.has_b = o.t0b < P.sq;
+    o.t_last = min(P.sq - 1, (o.has_b ? o.t0b : o.t0a) + P.tq - 1);
+    const int n_kv_all = (s_r + o.t_last + 1 + BN - 1) / BN;
+    const int per_split = (n_kv_all + P.n_split - 1) / P.n_split;
+    o.j_base = sp * per_split;
+    o.n_kv = max(0, min(n_kv_all, o.j_base + per_split) - o.j_base);
+    return o;
 }
 
 // ------------------------------------------------------------------ kernel
@@ -835,6 +856,93 @@ __device__ __forceinline__ void fused_producer(const FusedTcParams& F, int l, in
     }
 }
 
+// The fused kernel's producer after the CTA's first pair, when the CTA runs the pairs of its
+// (layer, request, KV head) in turn: the first was the last pair, which composed the whole
+// cache; pairs 0 .. pairs - 2 follow and read it.  Each pair's Q tiles (before RoPE) once the
+// previous pair's S MMAs have read the last ones; the K and V tiles whole from the cache once
+// the writer's stores are complete (B_WD), each as its stage frees (a stage last used by a
+// first-pair tile is free once its store has read it too).  n_first: the first pair's tiles.
+__device__ __noinline__ void fused_rest_producer(const FusedTcParams& F, int l, int bl, int b, int hk,
+                                                    int p_count, int s_r, int n_first, uint32_t sQ,
+                                                    uint32_t sK, uint32_t sV, uint32_t sBar,
+                                                    volatile uint32_t* abort) {
+    const TcParams& P = F.t;
+    auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
+    const int G = P.group;
+    const int qz = l * P.batch_total + b;
+    const int key0 = (int)((int64_t)(P.layer0 + l) * P.rows + P.req[bl].row_base);
+    // the CTA's pair pi >= 1 is pair pi - 1 of the request
+    int qi = 1;
+    int pk = 1, jk = 0, gk = n_first;
+    int pv = 1, jv = 0, gv = n_first;
+    PairSpan sk = pair_span(P, 0, 0, s_r), sv = sk;
+    bool stored = false;
+    auto k_free = [&](int g) {
+        const uint32_t ph = (uint32_t)((g / KSTAGES) - 1) & 1u;
+        return g < KSTAGES || (mbar_test(bar(B_KE + g % KSTAGES), ph) &&
+                               (g - KSTAGES >= n_first || mbar_test(bar(B_KW + g % KSTAGES), ph)));
+    };
+    auto v_free = [&](int g) {
+        const uint32_t ph = (uint32_t)((g / VSTAGES) - 1) & 1u;
+        return g < VSTAGES || (mbar_test(bar(B_VE + g % VSTAGES), ph) &&
+                               (g - VSTAGES >= n_first || mbar_test(bar(B_VW + g % VSTAGES), ph)));
+    };
+    long long idle0 = -1;
+    while (qi < p_count || pk < p_count || pv < p_count) {
+        if (!stored) stored = mbar_test(bar(B_WD), 0u);
+        if (qi < p_count && mbar_test(bar(B_QF), (uint32_t)(qi - 1) & 1u)) {
+            const PairSpan sq = pair_span(P, qi - 1, 0, s_r);
+            mbar_expect_tx(bar(B_Q), sq.has_b ? 2 * TILE : TILE);
+            tma_load_4d(sQ, &P.tm_q, 0, hk * G, sq.t0a, qz, bar(B_Q));
+            tma_load_4d(sQ + HALF_TILE, &P.tm_q, 64, hk * G, sq.t0a, qz, bar(B_Q));
+            if (sq.has_b) {
+                tma_load_4d(sQ + TILE, &P.tm_q, 0, hk * G, sq.t0b, qz, bar(B_Q));
+                tma_load_4d(sQ + TILE + HALF_TILE, &P.tm_q, 64, hk * G, sq.t0b, qz, bar(B_Q));
+            }
+            ++qi;
+            idle0 = -1;
+            continue;
+        }
+        if (stored && pk < p_count && k_free(gk)) {
+            const int st = gk % KSTAGES;
+            const int row = key0 + (sk.j_base + jk) * BN;
+            mbar_expect_tx(bar(B_KL + st), TILE);
+            tma_load_3d(sK + (uint32_t)(st * TILE), &P.tm_k, 0, hk, row, bar(B_KL + st));
+            tma_load_3d(sK + (uint32_t)(st * TILE) + HALF_TILE, &P.tm_k, 64, hk, row, bar(B_KL + st));
+            ++gk;
+            if (++jk == sk.n_kv) {
+                jk = 0;
+                if (++pk < p_count) sk = pair_span(P, pk - 1, 0, s_r);
+            }
+            idle0 = -1;
+            continue;
+        }
+        if (stored && pv < p_count && v_free(gv)) {
+            const int st = gv % VSTAGES;
+            const int row = key0 + (sv.j_base + jv) * BN;
+            mbar_expect_tx(bar(B_VL + st), TILE);
+            tma_load_3d(sV + (uint32_t)(st * TILE), &P.tm_v, 0, hk, row, bar(B_VL + st));
+            tma_load_3d(sV + (uint32_t)(st * TILE) + HALF_TILE, &P.tm_v, 64, hk, row, bar(B_VL + st));
+            ++gv;
+            if (++jv == sv.n_kv) {
+                jv = 0;
+                if (++pv < p_count) sv = pair_span(P, pv - 1, 0, s_r);
+            }
+            idle0 = -1;
+            continue;
+        }
+        if (*abort) return;
+        const long long now = clock64();
+        if (idle0 < 0) {
+            idle0 = now;
+        } else if (now - idle0 > kWaitCycles) {
+            atomicOr(P.err, 2);
+            *abort = 1u;
+            return;
+        }
+    }
+}
+
 __device__ __forceinline__ void tma_store_3d(const CUtensorMap* tm, uint32_t src, int c0, int c1, int c2) {
     asm volatile("cp.async.bulk.tensor.3d.global.shared::cta.bulk_group [%0, {%1, %2, %3}], [%4];" ::"l"(
                      reinterpret_cast<uint64_t>(tm)),
@@ -887,7 +995,7 @@ __device__ __forceinline__ uint32_t f2_to_bf2(float lo, float hi) {
 // positions), and releases the stage to the MMA and the writer.  They wait only for a K
 // stage to be free, so they run up to two tiles ahead of the MMA.
 __device__ __forceinline__ void fused_k_loader(const FusedTcParams& F, int lt, int l, int bl, int hk,
-                                               bool writer, int j_base, int n_kv, uint32_t sK,
+                                               bool writer, int j_base, int n_kv, int n_all, uint32_t sK,
                                                uint8_t* gK, uint32_t sBar, volatile uint32_t* abort) {
     using bf = __nv_bfloat16;
     const TcParams& P = F.t;
@@ -1044,6 +1152,13 @@ __device__ __forceinline__ void fused_k_loader(const FusedTcParams& F, int lt, i
         fence_proxy_async();
         mbar_arrive(bar(B_KF + st_i));
     }
+    // the key tiles of the CTA's later pairs (pairs run in turn) come whole from the composed
+    // cache: passed on to the MMA as they land
+    for (int g = n_kv; g < n_all; ++g) {
+        const int st_i = g % KSTAGES;
+        mbar_wait(bar(B_KL + st_i), (uint32_t)(g / KSTAGES) & 1u, P.err, abort);
+        mbar_arrive(bar(B_KF + st_i));
+    }
 }
 
 // The writer of the fused kernel (warp 2, one thread, writer CTAs): once the loaders have
@@ -1069,6 +1184,7 @@ __device__ __forceinline__ void fused_writer(const FusedTcParams& F, int l, int 
         mbar_arrive(bar(B_VW + vs));
     }
     asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+    mbar_arrive(bar(B_WD));     // the composed cache is written: later pairs may read it
 }
 
 // The V loader of the fused kernel (warp 3, lt = 0..31): per key tile, the ragged 8-row
@@ -1076,7 +1192,7 @@ __device__ __forceinline__ void fused_writer(const FusedTcParams& F, int l, int 
 // lt/16 + 2u of each such group), then the tile's TMA part, then the stage is released to
 // the MMA and the writer.
 __device__ __forceinline__ void fused_v_loader(const FusedTcParams& F, int lt, int l, int bl, int hk,
-                                               int j_base, int n_kv, uint32_t sV, uint32_t sBar,
+                                               int j_base, int n_kv, int n_all, uint32_t sV, uint32_t sBar,
                                                volatile uint32_t* abort) {
     using bf = __nv_bfloat16;
     const TcParams& P = F.t;
@@ -1128,6 +1244,11 @@ __device__ __forceinline__ void fused_v_loader(const FusedTcParams& F, int lt, i
         fence_proxy_async();
         mbar_arrive(bar(B_VF + st_i));
     }
+    for (int g = n_kv; g < n_all; ++g) {     // the later pairs' tiles, whole from the cache
+        const int st_i = g % VSTAGES;
+        mbar_wait(bar(B_VL + st_i), (uint32_t)(g / VSTAGES) & 1u, P.err, abort);
+        mbar_arrive(bar(B_VF + st_i));
+    }
 }
 
 // The suffix preparation of the fused kernel, done by the softmax warps (ts = 0..255) while
@@ -1145,7 +1266,8 @@ __device__ __forceinline__ void fused_v_loader(const FusedTcParams& F, int lt, i
 // angles (turn_cs) and the rounding are the suffix kernel's.
 __device__ __forceinline__ void fused_suffix_prep(const FusedTcParams& F, int ts, int l, int bl, int hk,
                                                   int k_lo, int k_hi, int q_lo, int q_hi, bool pos_rows,
-                                                  uint32_t sQ, uint32_t sBar, volatile uint32_t* abort) {
+                                                  uint32_t q_par, bool first, uint32_t sQ, uint32_t sBar,
+                                                  volatile uint32_t* abort) {
     using bf = __nv_bfloat16;
     const TcParams& P = F.t;
     auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
@@ -1199,7 +1321,7 @@ __device__ __forceinline__ void fused_suffix_prep(const FusedTcParams& F, int ts
     bool q_landed = false;
     auto q_item = [&](int tt, const float2 (&cc)[4], const float2 (&ss)[4]) {
         if (!q_landed) {
-            mbar_wait(bar(B_Q), 0u, P.err, abort);
+            mbar_wait(bar(B_Q), q_par, P.err, abort);
             q_landed = true;
         }
         const int x = (tt - q_lo) / tq;           // tile A or B
@@ -1269,27 +1391,7 @@ __device__ __forceinline__ void fused_suffix_prep(const FusedTcParams& F, int ts
         angles(tt, cc, ss);
         k_item(tt, xa, ya, cc, ss);
     }
-    mbar_arrive(bar(B_SK));    // the K loaders read these rows with cp.async (generic proxy)
-}
-
-// The query tokens and key tiles of pair pr of query tiles (split sp of its key range).
-struct PairSpan {
-    int t0a, t0b;       // first suffix token of tile A, of tile B
-    bool has_b;
-    int t_last;         // last suffix token of the pair
-    int j_base, n_kv;   // this split's key tiles: [j_base, j_base + n_kv)
-};
-__device__ __forceinline__ PairSpan pair_span(const TcParams& P, int pr, int sp, int s_r) {
-    PairSpan o;
-    o.t0a = 2 * pr * P.tq;
-    o.t0b = o.t0a + P.tq;
-    o.has_b = o.t0b < P.sq;
-    o.t_last = min(P.sq - 1, (o.has_b ? o.t0b : o.t0a) + P.tq - 1);
-    const int n_kv_all = (s_r + o.t_last + 1 + BN - 1) / BN;
-    const int per_split = (n_kv_all + P.n_split - 1) / P.n_split;
-    o.j_base = sp * per_split;
-    o.n_kv = max(0, min(n_kv_all, o.j_base + per_split) - o.j_base);
-    return o;
+    if (first) mbar_arrive(bar(B_SK));    // the K loaders read these rows with cp.async
 }
 
 // The plain kernel's TMA producer (one thread) for the pairs [p_first, p_first + p_count)
@@ -1388,7 +1490,11 @@ __global__ void __launch_bounds__(256) suffix_angles_kernel(const __grid_constan
     }
 }
 
-template <bool kFused>
+// kFused: compose + suffix preparation + attention; kMulti (fused only): the CTA runs every
+// pair of query tiles of its (layer, request, KV head), the last pair first (it composes the
+// cache), the others from the cache.  A separate instantiation, so that the one-pair fused
+// kernel keeps its register allocation.
+template <bool kFused, bool kMulti = false>
 __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
     attn_tc_kernel(const __grid_constant__ typename KernelParams<kFused>::type KP) {
     const TcParams& P = tc_params(KP);
@@ -1418,15 +1524,20 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
     const int p_first = (n_groups - 1 - (int)(blockIdx.x / P.n_split)) * P.pair_group;
     const int p_count = min(P.pairs, p_first + P.pair_group) - p_first;
     const int sp = (int)(blockIdx.x % P.n_split);   // key-range split
+    // the pair the CTA runs first: its first one, except in a fused CTA that runs every pair of
+    // its (layer, request, KV head), where the last pair leads (see fused_rest_producer)
+    const int p_lead = (kMulti && p_count > 1) ? P.pairs - 1 : p_first;
     // fused: the CTAs of the last pair see every key row of the request (all of the suffix),
     // so they write the composed cache
-    const bool writer = p_first == P.pairs - 1;
-    // the first pair (the fused kernel's only one)
-    const PairSpan ps0 = pair_span(P, p_first, sp, s_r);
+    const bool writer = p_lead == P.pairs - 1;
+    const PairSpan ps0 = pair_span(P, p_lead, sp, s_r);
+    // key tiles of all the CTA's pairs (the fused loaders pass the later pairs' tiles on)
+    int n_all = ps0.n_kv;
+    if (kMulti && p_count > 1)
+        for (int pr = 0; pr < P.pairs - 1; ++pr) n_all += pair_span(P, pr, sp, s_r).n_kv;
     const int t0a = ps0.t0a;
     const int t0b = ps0.t0b;
     const bool has_b = ps0.has_b;
-    const int t_last = ps0.t_last;
     const int j_base = ps0.j_base;
     const int n_kv = ps0.n_kv;
 
@@ -1457,6 +1568,7 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
         mbar_init(bar(B_SK), 256u);
         mbar_init(bar(B_QF), 1u);
         mbar_init(bar(B_OE), 256u);
+        mbar_init(bar(B_WD), 1u);
         mbar_init(bar(B_OD), 1);
         *abort = 0u;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
@@ -1490,17 +1602,29 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
                     tma_load_4d(sQ + TILE + HALF_TILE, &P.tm_q, 64, hk * G, t0b, qz, bar(B_Q));
                 }
                 fused_producer(KP, l, bl, hk, j_base, n_kv, writer, sK, sV, sBar, abort);
+                if constexpr (kMulti)
+                    if (p_count > 1)
+                        fused_rest_producer(KP, l, bl, b, hk, p_count, s_r, n_kv, sQ, sK, sV, sBar, abort);
             } else {
                 plain_producer(P, l, bl, b, hk, p_first, p_count, sp, s_r, sQ, sK, sV, sBar, abort);
             }
         } else if (warp == 1 && lane == 0 && n_kv > 0) {
             // ------------------------------------------------------------ MMA issuer
             RingState st;
-            if constexpr (kFused) {          // one pair
+            if constexpr (kFused && !kMulti) {   // one pair
                 if (has_b)
                     mma_issuer<true>(P, tmem, sQ, sK, sV, sBar, n_kv, B_QR, 0u, st, false, 0u, abort);
                 else
                     mma_issuer<false>(P, tmem, sQ, sK, sV, sBar, n_kv, B_QR, 0u, st, false, 0u, abort);
+            } else if constexpr (kFused) {       // the lead pair, then pairs 0 .. pairs - 2
+                for (int pi = 0; pi < p_count; ++pi) {
+                    const PairSpan ps = pi == 0 ? ps0 : pair_span(P, pi - 1, sp, s_r);
+                    const uint32_t q_par = (uint32_t)pi & 1u, oe_par = (uint32_t)(pi - 1) & 1u;
+                    if (ps.has_b)
+                        mma_issuer<true>(P, tmem, sQ, sK, sV, sBar, ps.n_kv, B_QR, q_par, st, pi > 0, oe_par, abort);
+                    else
+                        mma_issuer<false>(P, tmem, sQ, sK, sV, sBar, ps.n_kv, B_QR, q_par, st, pi > 0, oe_par, abort);
+                }
             } else {
                 for (int pi = 0; pi < p_count; ++pi) {
                     const PairSpan ps = pi == 0 ? ps0 : pair_span(P, p_first + pi, sp, s_r);
@@ -1517,24 +1641,42 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
         } else if (warp == 3 && n_kv > 0) {
             // ------------------------------------------------------------ V loader (fused)
             if constexpr (kFused)
-                fused_v_loader(KP, lane, l, bl, hk, j_base, n_kv, sV, sBar, abort);
+                fused_v_loader(KP, lane, l, bl, hk, j_base, n_kv, kMulti ? n_all : n_kv, sV, sBar, abort);
         }
     } else if (warp < 12) {
         asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(kFused ? kRegsHighFused : kRegsHigh));
         // ---------------------------------------------------------------- softmax warps
         const int x = warp >= 8 ? 1 : 0;               // tile A (warps 4..7) or B (8..11)
-        if constexpr (kFused) {
+        if constexpr (kFused && !kMulti) {
             // the suffix rows among this CTA's key tiles, and its query tokens
             const int k_lo = max(0, j_base * BN - s_r);
             const int k_hi = min(P.sq, (j_base + n_kv) * BN - s_r);
-            const int q_hi = n_kv > 0 ? t_last + 1 : t0a;   // (the loaders run iff n_kv > 0)
+            const int q_hi = n_kv > 0 ? ps0.t_last + 1 : t0a;   // (the loaders run iff n_kv > 0)
             fused_suffix_prep(KP, (int)threadIdx.x - 128, l, bl, hk, k_lo, k_hi, t0a, q_hi,
-                              writer && P.layer0 + l == 0 && hk == 0, sQ, sBar, abort);
-        }
-        if constexpr (kFused) {              // one pair
+                              writer && P.layer0 + l == 0 && hk == 0, 0u, true, sQ, sBar, abort);
             if (x == 0 || has_b)
                 softmax_tile(P, tmem, sBar, x, warp & 3, lane, x ? t0b : t0a, l, bl, b, hk, sp, j_base,
                              n_kv, 0u, 0u, false, abort);
+        } else if constexpr (kFused) {
+            // per pair: the suffix preparation (the lead pair's also turns the suffix rows
+            // among its key tiles into the cache), then the softmax over its key tiles
+            uint32_t done = 0u;
+            for (int pi = 0; pi < p_count; ++pi) {
+                const PairSpan ps = pi == 0 ? ps0 : pair_span(P, pi - 1, sp, s_r);
+                const int k_lo = pi == 0 ? max(0, ps.j_base * BN - s_r) : 0;
+                const int k_hi = pi == 0 ? min(P.sq, (ps.j_base + ps.n_kv) * BN - s_r) : 0;
+                const int q_hi = ps.n_kv > 0 ? ps.t_last + 1 : ps.t0a;   // (the loaders run iff n_kv > 0)
+                fused_suffix_prep(KP, (int)threadIdx.x - 128, l, bl, hk, k_lo, k_hi, ps.t0a, q_hi,
+                                  pi == 0 && writer && P.layer0 + l == 0 && hk == 0, (uint32_t)pi & 1u,
+                                  pi == 0, sQ, sBar, abort);
+                if (x == 0 || ps.has_b) {
+                    softmax_tile(P, tmem, sBar, x, warp & 3, lane, x ? ps.t0b : ps.t0a, l, bl, b, hk, sp,
+                                 ps.j_base, ps.n_kv, done, (uint32_t)pi & 1u, p_count > 1, abort);
+                    done += (uint32_t)ps.n_kv;
+                } else if (p_count > 1) {
+                    mbar_arrive(bar(B_OE));
+                }
+            }
         } else {
             uint32_t done = 0u;     // S_x tiles of the earlier pairs
             for (int pi = 0; pi < p_count; ++pi) {
@@ -1553,8 +1695,8 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
             asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsLowFused));
             // ------------------------------------------------------------ loaders (fused)
             if (n_kv > 0)
-                fused_k_loader(KP, (int)threadIdx.x - 12 * 32, l, bl, hk, writer, j_base, n_kv, sK,
-                               smem + 2 * TILE, sBar, abort);
+                fused_k_loader(KP, (int)threadIdx.x - 12 * 32, l, bl, hk, writer, j_base, n_kv,
+                               kMulti ? n_all : n_kv, sK, smem + 2 * TILE, sBar, abort);
         }
     }
 
@@ -1674,7 +1816,7 @@ namespace {
 
 // Host-side preparation shared by the plain and the fused launch: function attributes once
 // per process, the register-split guard, the tensor maps and the scalar parameters.
-template <bool kFused>
+template <bool kFused, bool kMulti = false>
 cudaError_t prepare_tc(const AttnParams& a, TcParams& p, dim3& grid) {
     constexpr int threads = kFused ? kThreadsFused : kThreads;
     constexpr int low = kFused ? kRegsLowFused : kRegsLow;
@@ -1682,12 +1824,12 @@ cudaError_t prepare_tc(const AttnParams& a, TcParams& p, dim3& grid) {
     constexpr int low_threads = kFused ? 256 : 128;
     // once per process (one device per context; function-local statics: thread-safe)
     static const cudaError_t smem_err = cudaFuncSetAttribute(
-        attn_tc_kernel<kFused>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+        attn_tc_kernel<kFused, kMulti>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
     if (smem_err != cudaSuccess) return smem_err;
     {   // the register split must not ask for more than the launch holds
         static const int launch_regs = []() {
             cudaFuncAttributes fa{};
-            return cudaFuncGetAttributes(&fa, attn_tc_kernel<kFused>) == cudaSuccess ? fa.numRegs : -1;
+            return cudaFuncGetAttributes(&fa, attn_tc_kernel<kFused, kMulti>) == cudaSuccess ? fa.numRegs : -1;
         }();
         if (launch_regs < 0) return cudaErrorInvalidDeviceFunction;
         if (launch_regs * threads < low_threads * low + 256 * high) return cudaErrorInvalidConfiguration;
@@ -1740,7 +1882,10 @@ cudaError_t prepare_tc(const AttnParams& a, TcParams& p, dim3& grid) {
     // from HBM, the epilogue) is then paid once for several short pairs (causal extraction
     // rows: 1 to 4 key tiles a pair).  C2KV_ATTN_PAIRS_PER_CTA overrides the choice (tests).
     int64_t pg = 1;
-    if (!kFused && p.n_split == 1) {
+    if (kMulti) {                // every pair of a (layer, request, KV head) in one CTA
+        if (p.n_split != 1) return cudaErrorInvalidValue;
+        pg = pairs;
+    } else if (!kFused && p.n_split == 1) {
         static const int sms = []() {
             int dev = 0, n = 0;
             if (cudaGetDevice(&dev) != cudaSuccess ||
@@ -1782,13 +1927,16 @@ thread_local FusedTcParams g_fused;          // the prepared launch (18 KB: kept
 thread_local SfxAngles g_angles;
 thread_local dim3 g_fused_grid;
 thread_local bool g_fused_ready = false;
+thread_local bool g_fused_multi = false;      // the prepared launch runs the pairs in turn
 }  // namespace
 
 cudaError_t prepare_attn_fused(const AttnParams& a, const FusedSpec& f) {
     (void)cudaGetLastError();
     g_fused_ready = false;
     FusedTcParams& p = g_fused;
-    cudaError_t e = prepare_tc<true>(a, p.t, g_fused_grid);
+    g_fused_multi = f.pairs_in_turn != 0;
+    cudaError_t e = g_fused_multi ? prepare_tc<true, true>(a, p.t, g_fused_grid)
+                                  : prepare_tc<true, false>(a, p.t, g_fused_grid);
     if (e != cudaSuccess) return e;
     if (a.layer0 != 0 || p.t.sq_pitch != a.sq || f.req_occ[0] != 0 || f.req_occ[a.batch] > kMaxFusedOcc)
         return cudaErrorInvalidValue;
@@ -1872,7 +2020,8 @@ cudaError_t launch_attn_fused(cudaStream_t s, Hook before) {
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    e = cudaLaunchKernelEx(&cfg, attn_tc_kernel<true>, g_fused);
+    e = g_fused_multi ? cudaLaunchKernelEx(&cfg, attn_tc_kernel<true, true>, g_fused)
+                      : cudaLaunchKernelEx(&cfg, attn_tc_kernel<true, false>, g_fused);
     if (e != cudaSuccess) return e;
     return cudaGetLastError();
 }

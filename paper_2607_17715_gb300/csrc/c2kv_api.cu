@@ -659,7 +659,9 @@ cudaError_t attend_run(c2kv_ctx* c, c2kv_cache* cache, int32_t layer0, int32_t l
         int32_t n_kv_max = 1;
         for (int32_t b = 0; b < B; ++b)
             n_kv_max = std::max<int32_t>(n_kv_max, (cache->n_slots[b] + n_suffix + 127) / 128);
-        if (c->cfg.attn_split >= 1) {
+        if (fused && fused->pairs_in_turn) {
+            n_split = 1;             // one CTA runs every pair of its (layer, request, KV head)
+        } else if (c->cfg.attn_split >= 1) {
             n_split = c->cfg.attn_split;
         } else if (2 * units <= c->sms) {
             // at most half of the SMs would have work: split toward one wave, keeping at
@@ -948,15 +950,22 @@ c2kv_status c2kv_compose_attend(c2kv_ctx* c, int32_t batch, const int32_t* req_p
         // The fused kernel takes pool-resident chunks on the tensor-core route, one attention
         // launch (at most kMaxReq requests) and at most kMaxFusedOcc occurrences; anything
         // else runs compose and then attention.  By default it runs only when one pair of
-        // query tiles covers each (layer, request, KV head): with more pairs every pair's CTA
-        // would load and turn the same composed tiles (measured slower than composing once).
-        const int64_t q_rows = (int64_t)n_suffix * (c->cfg.n_q_heads / std::max(1, c->cfg.n_kv_heads));
-        bool fuse = c->cfg.fuse != C2KV_FUSE_NEVER &&
-                    (c->cfg.fuse == C2KV_FUSE_ALWAYS || q_rows <= 256) &&
+        // query tiles covers each (layer, request, KV head).  With more pairs, forcing it
+        // (C2KV_FUSE_ALWAYS) runs them in turn in one CTA per (layer, request, KV head), the
+        // last pair first (it composes the cache), the others over the cache; with forced
+        // key-range splits each pair's CTA composes its own tiles instead.  Neither beat
+        // composing once, then attending (batched: 106 us against 100 us of kernels).
+        const int32_t grp = c->cfg.n_q_heads / std::max(1, c->cfg.n_kv_heads);
+        const int64_t q_rows = (int64_t)n_suffix * grp;
+        const int64_t tq = 128 / std::max(1, grp);
+        const int64_t pairs = ((n_suffix + tq - 1) / tq + 1) / 2;
+        const bool forced = c->cfg.fuse == C2KV_FUSE_ALWAYS;
+        bool fuse = c->cfg.fuse != C2KV_FUSE_NEVER && (forced || q_rows <= 256) &&
                     c->cfg.attn_impl != C2KV_ATTN_SIMT &&
                     c2kv::attn_tc_supported(c->cfg.dtype, c->cfg.head_dim, c->cfg.n_q_heads,
                                             c->cfg.n_kv_heads) &&
                     batch <= c2kv::kMaxReq && occ.size() <= (size_t)c2kv::kMaxFusedOcc;
+        const bool pairs_in_turn = pairs > 1 && c->cfg.attn_split <= 1;
         bool host_chunks = false;
         for (const auto& o : occ) host_chunks = host_chunks || o.host;
         fuse = fuse && !host_chunks;
@@ -1001,6 +1010,7 @@ c2kv_status c2kv_compose_attend(c2kv_ctx* c, int32_t batch, const int32_t* req_p
             if (e == cudaSuccess) {
                 f.occ_cs = occ_cs;
                 f.sfx_cs = occ_cs + n_occ_cs;
+                f.pairs_in_turn = pairs_in_turn ? 1 : 0;
                 f.k_suf = k_d;
                 f.v_suf = v_d;
                 e = attend_run(c, cache, 0, c->cfg.layers, q_d, k_d, v_d, n_suffix, out_d, lse_d, &f);

@@ -243,6 +243,8 @@ struct FusedSpec {
                              // turn, filled by the kernel
     float2* sfx_cs;          // scratch [B][Sq][64]: (cos, sin) of each suffix token's position,
                              // filled by a small kernel launched just before
+    int32_t pairs_in_turn;   // 1: a CTA runs every pair of query tiles of its (layer, request,
+                             // KV head), the last pair first, which composes the cache
     int64_t pool_slots;
     RopeTurns rope;
     int32_t req_occ[kMaxReq + 1];   // request i of the launch: occurrences [req_occ[i], req_occ[i+1])
