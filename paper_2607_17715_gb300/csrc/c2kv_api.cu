@@ -1192,6 +1192,7 @@ c2kv_status c2kv_decode(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
             p.n_split = n_split;
             p.keys_per_split = keys_per_split;
             p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)d));
+            p.dependent = c->prof ? 0 : 1;    // a trace records events between the two kernels
             for (int32_t i = 0; i < nb; ++i) p.req[i] = s.req[i];
             ProfScope prof_decode(c, C2KV_PROF_DECODE, true);
             e = c2kv::launch_decode(p, c->cfg.dtype, c->stream, prof_decode.hook());

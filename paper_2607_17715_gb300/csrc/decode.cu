@@ -124,6 +124,9 @@ __global__ void __launch_bounds__(kDecThreadsAll, G >= 8 ? 1 : 2) decode_kernel(
             for (int t = 0; t < n_tiles; ++t) {
                 const int st = t % kDecStages;
                 if (t >= kDecStages) mbar_wait(empty(st), (uint32_t)((t / kDecStages) - 1) & 1u, P.err, abort);
+                // the step's own key row (the last key) is the suffix kernel's: every tile
+                // before it is loaded while that kernel may still run
+                if (t == n_tiles - 1 && k_end == n_keys) asm volatile("griddepcontrol.wait;" ::: "memory");
                 mbar_expect_tx(full(st), 2 * kDecTileBytes);
                 tma_load_3d(sK + st * kDecTileBytes, &X.tm_k, 0, hk, row0 + t * KT, full(st));
                 tma_load_3d(sV + st * kDecTileBytes, &X.tm_v, 0, hk, row0 + t * KT, full(st));
@@ -136,6 +139,7 @@ __global__ void __launch_bounds__(kDecThreadsAll, G >= 8 ? 1 : 2) decode_kernel(
     const int grp = lane / LPK;                           // key row slot within a pass
     const int c = lane - grp * LPK;                       // this lane's channels [cE, cE+E)
     const int64_t qrow = ((int64_t)l * P.batch_total + b) * P.hq + (int64_t)hk * G;
+    asm volatile("griddepcontrol.wait;" ::: "memory");   // the rotated query is the suffix kernel's
     float q[G][E];
 #pragma unroll
     for (int g = 0; g < G; ++g) {
@@ -405,7 +409,22 @@ cudaError_t launch_g(const DecodeParams& p, cudaStream_t s, Hook before) {
     cudaError_t e = cudaSuccess;
     const dim3 grid((unsigned)p.n_split, (unsigned)p.hkv, (unsigned)(p.lq * p.batch));
     before();
-    decode_kernel<T, D, G><<<grid, kDecThreadsAll, kDecSmem, s>>>(x);
+    if (p.dependent) {    // starts while the suffix kernel before it runs (see the waits above)
+        cudaLaunchConfig_t cfg{};
+        cfg.gridDim = grid;
+        cfg.blockDim = dim3(kDecThreadsAll);
+        cfg.dynamicSmemBytes = kDecSmem;
+        cfg.stream = s;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        e = cudaLaunchKernelEx(&cfg, decode_kernel<T, D, G>, x);
+        if (e != cudaSuccess) return e;
+    } else {
+        decode_kernel<T, D, G><<<grid, kDecThreadsAll, kDecSmem, s>>>(x);
+    }
     e = cudaGetLastError();
     if (e != cudaSuccess || p.n_split == 1) return e;
     const int64_t rows_all = (int64_t)p.lq * p.batch_total * p.hq;

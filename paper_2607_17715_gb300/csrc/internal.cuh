@@ -175,6 +175,8 @@ struct DecodeParams {
     int32_t n_split;         // key-range splits per (layer, request, KV head)
     int32_t keys_per_split;
     float scale_log2;        // log2(e) / sqrt(d)
+    int32_t dependent;       // launched as the programmatic dependent of the suffix kernel that
+                             // writes this step's query and key row (nothing between them)
     ReqParam req[kMaxReq];
 };
 bool decode_supported(int dtype, int d, int hq, int hkv);

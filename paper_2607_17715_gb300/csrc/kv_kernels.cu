@@ -213,6 +213,9 @@ __global__ void __launch_bounds__(256) suffix_kernel(const __grid_constant__ Suf
     constexpr int E = V::N;
     constexpr int HALF = VPH * E;
     constexpr int D = 2 * HALF;
+    // a programmatic dependent (the decode kernel) may start now: it waits
+    // (griddepcontrol.wait) before it reads what this kernel writes
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     __shared__ float2 cs[HALF];
     const int l = blockIdx.y;
     const int n_pad = P.pad_rows ? P.batch * kPadParts : 0;
