@@ -629,13 +629,56 @@ c2kv_status attend_check(c2kv_ctx* c, const char* what, int32_t layer, const voi
     return C2KV_OK;
 }
 
+// The suffix kernel's parameters for requests b0 .. b0 + nb - 1 of a cache.
+c2kv::SuffixParams suffix_params(const c2kv_ctx* c, const c2kv_cache* cache, int32_t layer0, int32_t lq,
+                                 const void* q, const void* k_suf, const void* v_suf, int32_t n_suffix,
+                                 void* q_rot, int32_t b0, int32_t nb) {
+    c2kv::SuffixParams s{};
+    s.q = q;
+    s.k = k_suf;
+    s.v = v_suf;
+    s.q_rot = q_rot;
+    s.cache_k = cache->k;
+    s.cache_v = cache->v;
+    s.pos = cache->pos;
+    s.rows = cache->rows;
+    s.layer0 = layer0;
+    s.lq = lq;
+    s.batch = nb;
+    s.batch_total = cache->batch;
+    s.b0 = b0;
+    s.sq = n_suffix;
+    s.hq = c->cfg.n_q_heads;
+    s.hkv = c->cfg.n_kv_heads;
+    s.pad_rows = 1;
+    s.rope = c->turns;
+    for (int32_t i = 0; i < nb; ++i)
+        s.req[i] = c2kv::ReqParam{cache->row_base[b0 + i], cache->n_slots[b0 + i], cache->l_req[b0 + i], 0};
+    return s;
+}
+
+// The suffix preparation of every request alone (suffix RoPE into q_rot, the suffix rows and
+// the zero rows up to the tile edge into the cache), on the context's stream.
+cudaError_t suffix_run(c2kv_ctx* c, const c2kv_cache* cache, int32_t layer0, int32_t lq, const void* q,
+                       const void* k_suf, const void* v_suf, int32_t n_suffix, void* q_rot) {
+    cudaError_t e = cudaSuccess;
+    for (int32_t b0 = 0; e == cudaSuccess && b0 < cache->batch; b0 += c2kv::kMaxReq) {
+        const int32_t nb = std::min<int32_t>(c2kv::kMaxReq, cache->batch - b0);
+        const c2kv::SuffixParams s = suffix_params(c, cache, layer0, lq, q, k_suf, v_suf, n_suffix, q_rot, b0, nb);
+        ProfScope prof_suffix(c, C2KV_PROF_SUFFIX);
+        e = c2kv::launch_suffix_prep(s, c->cfg.dtype, c->cfg.head_dim, c->stream);
+    }
+    return e;
+}
+
 // Suffix preparation and attention of a cache (arguments already checked).  With `fused`,
 // the cache is not written yet: the fused kernel reads the composed slots from the pool and
 // the suffix from k_suf / v_suf, turns the queries itself, and writes the whole cache
-// (tensor-core route, every layer, one launch).
+// (tensor-core route, every layer, one launch).  With `q_rot_ready`, the suffix preparation
+// has already run (suffix_run) into that buffer: only attention is launched.
 cudaError_t attend_run(c2kv_ctx* c, c2kv_cache* cache, int32_t layer0, int32_t lq, const void* q,
                        const void* k_suf, const void* v_suf, int32_t n_suffix, void* out, float* lse,
-                       const c2kv::FusedSpec* fused) {
+                       const c2kv::FusedSpec* fused, void* q_rot_ready = nullptr) {
     const int32_t B = cache->batch;
     const bool use_tc =
         c->cfg.attn_impl != C2KV_ATTN_SIMT &&
@@ -646,9 +689,10 @@ cudaError_t attend_run(c2kv_ctx* c, c2kv_cache* cache, int32_t layer0, int32_t l
     // scratch: the suffix queries after RoPE (the attention kernels' Q operand); the fused
     // kernel turns them in shared memory
     const size_t q_bytes = (size_t)lq * B * n_suffix * c->cfg.n_q_heads * c->cfg.head_dim * c->eb;
-    void* q_rot = nullptr;
-    cudaError_t e = fused ? cudaSuccess : pool_alloc(c, &q_rot, q_bytes);
+    void* q_rot = q_rot_ready;
+    cudaError_t e = fused || q_rot_ready ? cudaSuccess : pool_alloc(c, &q_rot, q_bytes);
     if (e != cudaSuccess) return e;
+    void* const q_rot_own = q_rot_ready ? nullptr : q_rot;    // freed here
     // Key-range split of the tensor-core attention: when its work units would leave most
     // SMs idle (a single layer of a small batch), each unit's key tiles are split and the
     // partials merged; at a wave or more the split only adds the merge.
@@ -674,7 +718,7 @@ cudaError_t attend_run(c2kv_ctx* c, c2kv_cache* cache, int32_t layer0, int32_t l
             e = pool_alloc(c, reinterpret_cast<void**>(&part),
                            (size_t)n_split * rows * (c->cfg.head_dim + 1) * sizeof(float));
             if (e != cudaSuccess) {
-                pool_free(c, q_rot);
+                pool_free(c, q_rot_own);
                 return e;
             }
         }
@@ -683,28 +727,7 @@ cudaError_t attend_run(c2kv_ctx* c, c2kv_cache* cache, int32_t layer0, int32_t l
     c2kv::AttnParams last{};
     for (int32_t b0 = 0; e == cudaSuccess && b0 < B; b0 += c2kv::kMaxReq) {
         const int32_t nb = std::min<int32_t>(c2kv::kMaxReq, B - b0);
-        c2kv::SuffixParams s{};
-        s.q = q;
-        s.k = k_suf;
-        s.v = v_suf;
-        s.q_rot = q_rot;
-        s.cache_k = cache->k;
-        s.cache_v = cache->v;
-        s.pos = cache->pos;
-        s.rows = cache->rows;
-        s.layer0 = layer0;
-        s.lq = lq;
-        s.batch = nb;
-        s.batch_total = B;
-        s.b0 = b0;
-        s.sq = n_suffix;
-        s.hq = c->cfg.n_q_heads;
-        s.hkv = c->cfg.n_kv_heads;
-        s.pad_rows = 1;
-        s.rope = c->turns;
-        for (int32_t i = 0; i < nb; ++i)
-            s.req[i] = c2kv::ReqParam{cache->row_base[b0 + i], cache->n_slots[b0 + i],
-                                      cache->l_req[b0 + i], 0};
+        const c2kv::SuffixParams s = suffix_params(c, cache, layer0, lq, q, k_suf, v_suf, n_suffix, q_rot, b0, nb);
         c2kv::AttnParams a{};
         a.q_rot = fused ? q : q_rot;
         a.cache_k = cache->k;
@@ -732,7 +755,7 @@ cudaError_t attend_run(c2kv_ctx* c, c2kv_cache* cache, int32_t layer0, int32_t l
             ProfScope prof_fused(c, C2KV_PROF_FUSED, true);
             e = c2kv::launch_attn_fused(c->stream, prof_fused.hook());
         } else {
-            {
+            if (!q_rot_ready) {
                 ProfScope prof_suffix(c, C2KV_PROF_SUFFIX);
                 e = c2kv::launch_suffix_prep(s, c->cfg.dtype, c->cfg.head_dim, c->stream);
             }
@@ -748,7 +771,7 @@ cudaError_t attend_run(c2kv_ctx* c, c2kv_cache* cache, int32_t layer0, int32_t l
         e = c2kv::launch_attn_combine(last, c->stream);
     }
     pool_free(c, part);
-    pool_free(c, q_rot);
+    pool_free(c, q_rot_own);
     return e;
 }
 
@@ -760,6 +783,24 @@ struct StreamSwap {
     StreamSwap(c2kv_ctx* ctx, cudaStream_t s) : c(ctx), saved(ctx->stream) { c->stream = s; }
     ~StreamSwap() { c->stream = saved; }
 };
+
+// The context's second stream, and at least n events for forks to it and joins from it.
+cudaError_t aux_ready(c2kv_ctx* c, size_t n) {
+    if (!c->aux) {
+        const cudaError_t e = cudaStreamCreateWithFlags(&c->aux, cudaStreamNonBlocking);
+        if (e != cudaSuccess) {
+            c->aux = nullptr;
+            return e;
+        }
+    }
+    while (c->aux_ev.size() < n) {
+        cudaEvent_t ev = nullptr;
+        const cudaError_t e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
+        if (e != cudaSuccess) return e;
+        c->aux_ev.push_back(ev);
+    }
+    return cudaSuccess;
+}
 
 // Compose + attend when chunks are read from host memory: compose is bound by the host link,
 // so the layers go in groups.  The context's stream composes group g with a few CTAs (the
@@ -851,20 +892,8 @@ cudaError_t compose_attend_pipelined(c2kv_ctx* c, c2kv_cache* cache, const std::
     const int32_t L = c->cfg.layers;
     const int32_t groups = std::min<int32_t>(4, L);
     const int32_t per = (L + groups - 1) / groups;
-    cudaError_t e = cudaSuccess;
-    if (!c->aux) {
-        e = cudaStreamCreateWithFlags(&c->aux, cudaStreamNonBlocking);
-        if (e != cudaSuccess) {
-            c->aux = nullptr;
-            return e;
-        }
-    }
-    while (c->aux_ev.size() < (size_t)groups + 2) {
-        cudaEvent_t ev = nullptr;
-        e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
-        if (e != cudaSuccess) return e;
-        c->aux_ev.push_back(ev);
-    }
+    cudaError_t e = aux_ready(c, (size_t)groups + 2);
+    if (e != cudaSuccess) return e;
     SuffixIO io;
     e = suffix_io_open(c, L, cache->batch, n_suffix, q, k_suf, v_suf, out, lse, &io);
     if (e != cudaSuccess) return e;
@@ -899,6 +928,35 @@ cudaError_t compose_attend_pipelined(c2kv_ctx* c, c2kv_cache* cache, const std::
     if (e2 == cudaSuccess) cudaStreamWaitEvent(c->stream, c->aux_ev[groups + 1], 0);
     if (e != cudaSuccess || e2 != cudaSuccess) cudaStreamSynchronize(c->aux);
     pool_free(c, io.scratch);
+    return e != cudaSuccess ? e : e2;
+}
+
+// Compose + attend from chunks in the pool when the step is not fused.  The suffix
+// preparation writes only what compose does not (the turned queries, the suffix rows and the
+// zero rows after them, their positions), so it runs on the second stream while compose runs
+// on the context's stream, and attention follows both.
+cudaError_t compose_attend_overlapped(c2kv_ctx* c, c2kv_cache* cache, const std::vector<c2kv::OccParam>& occ,
+                                      const void* q, const void* k_suf, const void* v_suf, int32_t n_suffix,
+                                      void* out, float* lse) {
+    const int32_t L = c->cfg.layers;
+    const size_t q_bytes = (size_t)L * cache->batch * n_suffix * c->cfg.n_q_heads * c->cfg.head_dim * c->eb;
+    void* q_rot = nullptr;
+    cudaError_t e = aux_ready(c, 2);
+    if (e == cudaSuccess) e = pool_alloc(c, &q_rot, q_bytes);
+    if (e != cudaSuccess) return e;
+    e = cudaEventRecord(c->aux_ev[0], c->stream);       // the caller's work and q_rot's allocation
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(c->aux, c->aux_ev[0], 0);
+    if (e == cudaSuccess) {
+        StreamSwap on_aux(c, c->aux);
+        e = suffix_run(c, cache, 0, L, q, k_suf, v_suf, n_suffix, q_rot);
+    }
+    cudaError_t e2 = cudaEventRecord(c->aux_ev[1], c->aux);
+    if (e == cudaSuccess) e = compose_launch(c, cache, occ);
+    if (e2 == cudaSuccess) e2 = cudaStreamWaitEvent(c->stream, c->aux_ev[1], 0);
+    if (e == cudaSuccess && e2 == cudaSuccess)
+        e = attend_run(c, cache, 0, L, q, k_suf, v_suf, n_suffix, out, lse, nullptr, q_rot);
+    if (e != cudaSuccess || e2 != cudaSuccess) cudaStreamSynchronize(c->aux);
+    pool_free(c, q_rot);
     return e != cudaSuccess ? e : e2;
 }
 
@@ -1018,7 +1076,9 @@ c2kv_status c2kv_compose_attend(c2kv_ctx* c, int32_t batch, const int32_t* req_p
             }
         } else if (pipelined) {
             e = compose_attend_pipelined(c, cache, occ, q, k_suf, v_suf, n_suffix, out, lse);
-        } else {
+        } else if (!c->prof) {
+            e = compose_attend_overlapped(c, cache, occ, q_d, k_d, v_d, n_suffix, out_d, lse_d);
+        } else {    // traced: one kernel at a time, so that each recorded time is its kernel's own
             e = compose_launch(c, cache, occ);
             if (e == cudaSuccess)
                 e = attend_run(c, cache, 0, c->cfg.layers, q_d, k_d, v_d, n_suffix, out_d, lse_d, nullptr);
