@@ -458,3 +458,49 @@ def test_compose_attend_arg_checks():
         c2kv.c2kv_cache_release(ctx, cache)
     finally:
         c2kv.c2kv_destroy(ctx)
+
+
+def test_unfused_route_suffix_beside_compose():
+    # fuse NEVER, no trace: compose on the context's stream while the suffix kernel runs on
+    # its second stream, then attention; against the oracle and compose + attend
+    _fused_case(synth.scaled(synth.workload("batched"), batch=3, chunks_per_request=4,
+                             pool_chunks=32, n_suffix=40), fuse=1)
+
+
+def test_unfused_route_traced_equals_untraced():
+    # with the trace on, the unfused route runs compose, suffix and attention in turn on one
+    # stream; without it the suffix kernel runs beside compose: the same bits either way
+    c2kv = H.lib()
+    wl = synth.scaled(synth.workload("batched"), batch=4, chunks_per_request=3, pool_chunks=8,
+                      n_suffix=72, layers=2)
+    reqs = synth.requests(wl)
+    all_ids = sorted({c for ids, _ in reqs for c in ids})
+    chunks = H.oracle_chunks_meanpool(wl, all_ids)
+    pool = sum(chunks[c][0].shape[1] for c in all_ids) + 16
+    ctx = H.make_ctx(wl, pool_slots=pool, fuse=1)
+    try:
+        dev = H.load_stored(ctx, wl, chunks)
+        q, ks, vs = synth.suffix(wl, layers=wl.layers)
+        sq = wl.n_suffix
+        runs = []
+        for traced in (False, True):
+            c2kv.c2kv_profile_enable(ctx, traced)
+            cache, out, lse = _run(ctx, wl, dev, reqs, q, ks, vs, sq, fused=True)
+            runs.append((H.cache_arrays(cache, wl), out, lse))
+            c2kv.c2kv_cache_release(ctx, cache)
+        c2kv.c2kv_profile_enable(ctx, False)
+        kinds = c2kv.c2kv_profile_read(ctx)
+        assert kinds.get("suffix", (0, 0))[1] >= 1 and kinds.get("compose", (0, 0))[1] >= 1
+        (info_a, ka, va, pa), out_a, lse_a = runs[0]
+        (info_b, kb, vb, pb), out_b, lse_b = runs[1]
+        for r in range(len(reqs)):
+            base, s = info_a["row_base"][r], info_a["n_slots"][r]
+            assert info_b["row_base"][r] == base and info_b["n_slots"][r] == s
+            end = base + (s + sq + 127) // 128 * 128
+            assert np.array_equal(pa[base:base + s + sq], pb[base:base + s + sq])
+            assert np.array_equal(ka[:, base:end], kb[:, base:end])
+            assert np.array_equal(va[:, base:end], vb[:, base:end])
+        assert torch.equal(out_a, out_b)
+        assert torch.equal(lse_a, lse_b)
+    finally:
+        c2kv.c2kv_destroy(ctx)
