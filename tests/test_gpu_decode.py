@@ -108,6 +108,62 @@ def test_decode_long_context_splits():
     _decode_case(wl, steps=[3], prefill=3)
 
 
+@pytest.mark.parametrize("long", [False, True])
+def test_decode_traced_equals_untraced(long):
+    # untraced, the decode kernel is the suffix kernel's programmatic dependent and loads the
+    # tiles before the new row while that kernel runs; traced, the two run one after the
+    # other.  The same step decoded both ways (the new row rewritten with the same bits):
+    # the same output and lse, bit for bit; long: key-range splits and their merge
+    c2kv = H.lib()
+    if long:
+        wl = _small(L8B_1, chunk_tokens=1024, ratio_k=4, chunks_per_request=32, pool_chunks=32)
+    else:
+        wl = _small(synth.workload("batched"), batch=3, chunks_per_request=4, pool_chunks=32,
+                    layers=2)
+    reqs = synth.requests(wl)
+    B = len(reqs)
+    steps = [4 + 3 * b for b in range(B)]
+    n_tok = max(steps) + 1
+    all_ids = sorted({c for ids, _ in reqs for c in ids})
+    chunks = H.oracle_chunks_meanpool(wl, all_ids)
+    pool = sum(orc.n_slots(wl.chunk_tokens, wl.ratio_k) for _ in all_ids) + 16
+    ctx = H.make_ctx(wl, pool_slots=pool)
+    try:
+        dev = H.load_stored(ctx, wl, chunks)
+        req_ptr = np.cumsum([0] + [len(ids) for ids, _ in reqs])
+        cache = c2kv.c2kv_compose(ctx, req_ptr, [dev[c] for ids, _ in reqs for c in ids],
+                                  [o for _, offs in reqs for o in offs], suffix_capacity=n_tok)
+        q, ks, vs = synth.suffix(synth.scaled(wl, n_suffix=n_tok), layers=wl.layers)
+        q, ks, vs = q[:, :B], ks[:, :B], vs[:, :B]
+        pre = min(steps)
+        qd, kd, vd = (H.to_dev(x[:, :, :pre], wl) for x in (q, ks, vs))
+        c2kv.c2kv_attend(ctx, cache, -1, qd, kd, vd, pre, torch.empty_like(qd))
+        for b in range(B):        # suffix rows pre .. steps[b]-1 of each request, one at a time
+            for t in range(pre, steps[b]):
+                cur = [t if r == b else steps[r] for r in range(B)]
+                pick = [np.stack([x[:, r, cur[r]] for r in range(B)], axis=1) for x in (q, ks, vs)]
+                qd, kd, vd = (H.to_dev(x, wl) for x in pick)
+                c2kv.c2kv_decode(ctx, cache, -1, qd, kd, vd, cur, torch.empty_like(qd))
+        pick = [np.stack([x[:, r, steps[r]] for r in range(B)], axis=1) for x in (q, ks, vs)]
+        qd, kd, vd = (H.to_dev(x, wl) for x in pick)
+        res = []
+        for traced in (False, True):
+            c2kv.c2kv_profile_enable(ctx, traced)
+            out = torch.full_like(qd, float("nan"))
+            lse = torch.full(qd.shape[:-1], float("nan"), device="cuda")
+            c2kv.c2kv_decode(ctx, cache, -1, qd, kd, vd, steps, out, lse)
+            c2kv.c2kv_sync(ctx)
+            res.append((out, lse))
+        c2kv.c2kv_profile_enable(ctx, False)
+        assert c2kv.c2kv_profile_read(ctx)["decode"][1] >= 1
+        assert torch.equal(res[0][0], res[1][0])
+        assert torch.equal(res[0][1], res[1][1])
+        assert not torch.isnan(res[0][0]).any()
+        c2kv.c2kv_cache_release(ctx, cache)
+    finally:
+        c2kv.c2kv_destroy(ctx)
+
+
 def test_decode_gqa8_and_mha():
     _decode_case(_small(synth.workload("long70b"), batch=1, chunks_per_request=4,
                         pool_chunks=4), steps=[2], prefill=2)
