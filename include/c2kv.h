@@ -250,10 +250,11 @@ c2kv_status c2kv_attend(c2kv_ctx* ctx, c2kv_cache* cache, int32_t layer, const v
  * offset in shared memory (Sec. 3.2.4 re-rotation), turns the queries and the suffix keys by
  * their positions, and writes the composed cache as it goes, so the cache is written once
  * and never read back (a small kernel before it evaluates the suffix positions' angles).
- * Otherwise compose and attention run one after the other; with chunks in host memory and
- * two or more layers, the layers go in groups so that reading one group over the host link
- * overlaps the attention of the previous one (on a second stream; the call's work still
- * ends on the context's stream).  The context's `fuse` setting chooses (C2KV_FUSE_*): by
+ * Otherwise compose and attention run one after the other, the suffix preparation beside
+ * compose on a second stream (it writes only rows compose does not; in turn while a trace
+ * is on); with chunks in host memory and two or more layers, the layers go in groups so
+ * that reading one group over the host link overlaps the attention of the previous one (on
+ * a second stream).  Either way the call's work ends on the context's stream.  The context's `fuse` setting chooses (C2KV_FUSE_*): by
  * default the fused kernel runs when each (layer, request, KV head) has one pair of query
  * tiles.  The cache is returned as by c2kv_compose (release it with c2kv_cache_release) and
  * serves later c2kv_decode / c2kv_attend calls.
