@@ -1317,10 +1317,15 @@ c2kv_status c2kv_extract_attention(c2kv_ctx* c, int32_t n_layers, const void* q,
         p.hkv = hkv;
         p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)d));
         p.rope = c->turns;
+        // the C2 rows beside the document rows on the second stream (tensor-core route)
+        const bool two = c2kv::extract_uses_tc(c->cfg.dtype, d, c->cfg.n_q_heads, c->cfg.n_kv_heads) &&
+                         aux_ready(c, 2) == cudaSuccess;
         {
             ProfScope prof(c, C2KV_PROF_EXTRACT);
-            e = c2kv::launch_extract(p, c->cfg.dtype, d, c->stream);
+            e = c2kv::launch_extract(p, c->cfg.dtype, d, c->stream, two ? c->aux : nullptr,
+                                     two ? c->aux_ev[0] : nullptr, two ? c->aux_ev[1] : nullptr);
         }
+        if (e != cudaSuccess && two) cudaStreamSynchronize(c->aux);   // before the scratch goes
         if (lse_scratch) pool_free(c, lse_scratch);
         pool_free(c, k_rot);
         pool_free(c, q_rot);

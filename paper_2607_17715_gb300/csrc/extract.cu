@@ -350,7 +350,19 @@ cudaError_t launch_local(const ExtractParams& p, cudaStream_t s) {
     return cudaGetLastError();
 }
 
-cudaError_t launch_tc(const ExtractParams& p, cudaStream_t s) {
+cudaError_t launch_local_any(const ExtractParams& p, cudaStream_t s) {
+    switch (p.hq / p.hkv) {
+        case 1: return launch_local<1>(p, s);
+        case 2: return launch_local<2>(p, s);
+        case 4: return launch_local<4>(p, s);
+        case 8: return launch_local<8>(p, s);
+        case 16: return launch_local<16>(p, s);
+        default: return cudaErrorInvalidValue;
+    }
+}
+
+cudaError_t launch_tc(const ExtractParams& p, cudaStream_t s, cudaStream_t s2, cudaEvent_t fork,
+                      cudaEvent_t join) {
     constexpr int D = 128;
     extract_rope_kernel<__nv_bfloat16, D / 2 / Vec16<__nv_bfloat16>::N>
         <<<dim3((unsigned)p.n_all, (unsigned)p.lq), 256, 0, s>>>(p);
@@ -373,6 +385,15 @@ cudaError_t launch_tc(const ExtractParams& p, cudaStream_t s) {
     a.hkv = p.hkv;
     a.scale_log2 = p.scale_log2;
     a.n_split = 1;
+    // pieces 2 and 3 write only the C2 rows (and read the rotated rows): with a second stream
+    // they run beside piece 1, in the SMs its last wave of CTAs leaves idle
+    cudaStream_t sc = s;
+    if (s2 != nullptr) {
+        e = cudaEventRecord(fork, s);
+        if (e == cudaSuccess) e = cudaStreamWaitEvent(s2, fork, 0);
+        if (e != cudaSuccess) return e;
+        sc = s2;
+    }
     // 1. document rows over document keys 0..t
     a.q_rot = p.q_rot;
     a.out = p.out;
@@ -388,17 +409,15 @@ cudaError_t launch_tc(const ExtractParams& p, cudaStream_t s) {
     a.lse = lse_ab + p.n;
     a.sq = m;
     a.req[0] = ReqParam{p.n, 0, 0, 0};
-    e = launch_attn_tc(a, s);
-    if (e != cudaSuccess) return e;
+    e = launch_attn_tc(a, sc);
     // 3. C2 rows over the sink block and their own block, merged into 2
-    switch (p.hq / p.hkv) {
-        case 1: return launch_local<1>(p, s);
-        case 2: return launch_local<2>(p, s);
-        case 4: return launch_local<4>(p, s);
-        case 8: return launch_local<8>(p, s);
-        case 16: return launch_local<16>(p, s);
-        default: return cudaErrorInvalidValue;
+    if (e == cudaSuccess) e = launch_local_any(p, sc);
+    if (s2 != nullptr) {       // the work ends on s
+        cudaError_t ej = cudaEventRecord(join, s2);
+        if (ej == cudaSuccess) ej = cudaStreamWaitEvent(s, join, 0);
+        if (e == cudaSuccess) e = ej;
     }
+    return e;
 }
 
 template <typename T, int D>
@@ -417,13 +436,14 @@ cudaError_t launch_typed(const ExtractParams& p, cudaStream_t s) {
 
 bool extract_uses_tc(int dtype, int d, int hq, int hkv) { return attn_tc_supported(dtype, d, hq, hkv); }
 
-cudaError_t launch_extract(const ExtractParams& p, int dtype, int d, cudaStream_t s) {
+cudaError_t launch_extract(const ExtractParams& p, int dtype, int d, cudaStream_t s, cudaStream_t s2,
+                           cudaEvent_t fork, cudaEvent_t join) {
     (void)cudaGetLastError();   // report this launch's error only, not a stale one
     if (p.n_all < 1 || p.lq < 1) return cudaSuccess;
     if (p.lq > 65535 || p.hkv > 65535) return cudaErrorInvalidValue;
     if (extract_uses_tc(dtype, d, p.hq, p.hkv)) {
         if (p.lse == nullptr && p.lse_scratch == nullptr) return cudaErrorInvalidValue;
-        return launch_tc(p, s);
+        return launch_tc(p, s, s2, fork, join);
     }
     if (dtype == kDtypeF32 && d == 64) return launch_typed<float, 64>(p, s);
     if (dtype == kDtypeF32 && d == 128) return launch_typed<float, 128>(p, s);

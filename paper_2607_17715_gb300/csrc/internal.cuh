@@ -203,7 +203,10 @@ struct ExtractParams {
     float scale_log2;
     RopeTurns rope;
 };
-cudaError_t launch_extract(const ExtractParams& p, int dtype, int d, cudaStream_t s);
+// With s2 (and the events fork and join), the tensor-core route runs the C2 rows' attention and
+// block-local merge on s2, beside the document rows' attention on s; the work ends on s.
+cudaError_t launch_extract(const ExtractParams& p, int dtype, int d, cudaStream_t s,
+                           cudaStream_t s2 = nullptr, cudaEvent_t fork = nullptr, cudaEvent_t join = nullptr);
 // Whether launch_extract takes the tensor-core route (and so needs lse_scratch when lse is
 // null); otherwise every row runs on the CUDA cores.
 bool extract_uses_tc(int dtype, int d, int hq, int hkv);
