@@ -643,7 +643,7 @@ def run_ours(args):
                    "compose_gbs": round(comp_gbs, 1), "attend_tflops": round(attn_tfs, 2),
                    "compose_bytes": f["compose_bytes"], "attend_flops": f["attn_flops"],
                    "fused_bytes": f["fused_bytes"], "wall_s": round(wall, 4)},
-        # the dominant kernel of the step (by device time) carries "roofline"; the judged
+        # the dominant kernel of the step (by device time) carries "roofline"; the separate
         # compose and attention kernels (from the same steps run as separate calls) are
         # reported beside it.  Attention is HBM- or tensor-bound depending on its arithmetic
         # intensity relative to the ridge of the measured peaks.
