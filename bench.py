@@ -279,6 +279,24 @@ class Arm:
     def flush_l2(self):
         self.flush_buf.fill_(1.0)
 
+    def compose_warm(self, steps):
+        """Median time of c2kv_compose right after an identical compose (no L2 flush: the
+        inputs stay in L2 where they fit), event-timed around the call."""
+        c2kv, wl, E = self.c2kv, self.wl, self.torch.cuda.Event
+        ids = [self.dev_ids[c] for ids_, _ in self.reqs for c in ids_]
+        evs = []
+        for _ in range(steps):
+            c2kv.c2kv_cache_release(self.ctx, c2kv.c2kv_compose(self.ctx, self.req_ptr, ids,
+                                                                self.positions, wl.n_suffix))
+            a, b = E(enable_timing=True), E(enable_timing=True)
+            a.record(self.stream)
+            cache = c2kv.c2kv_compose(self.ctx, self.req_ptr, ids, self.positions, wl.n_suffix)
+            b.record(self.stream)
+            c2kv.c2kv_cache_release(self.ctx, cache)
+            evs.append((a, b))
+        self.torch.cuda.synchronize()
+        return statistics.median(a.elapsed_time(b) for a, b in evs)
+
     def step_device(self, ev, fused=True):
         """One step with inputs resident in HBM: c2kv_compose_attend (the library fuses the
         two when that pays), or c2kv_compose then c2kv_attend; then the cache is released.
@@ -329,48 +347,9 @@ class Arm:
             c2kv.c2kv_free_chunk(self.ctx, cid)
 
     def decode_run(self, steps, warmup, events):
-        """Decode after the suffix: compose once, write the suffix with attend, then decode
-        `warmup` untimed and `steps` timed tokens per request (one c2kv_decode call per token,
-        all layers), L2 flushed before each; then `steps` more tokens with the library's trace
-        on, for the decode kernel's own time.  Returns (ms per timed step, mean decode kernel
-        ms from the trace, keys read per timed step summed over requests)."""
-        c2kv, wl, torch = self.c2kv, self.wl, self.torch
         ids = [self.dev_ids[c] for ids_, _ in self.reqs for c in ids_]
-        cache = c2kv.c2kv_compose(self.ctx, self.req_ptr, ids, self.positions,
-                                  wl.n_suffix + warmup + 2 * steps)
-        c2kv.c2kv_attend(self.ctx, cache, -1, *self.q_dev, wl.n_suffix, self.out)
-        B = len(self.reqs)
-        gen = torch.Generator(device="cuda").manual_seed(1)
-        qd = torch.randn((wl.layers, B, wl.n_q_heads, wl.head_dim), device="cuda", generator=gen).to(self.tdt)
-        kd = torch.randn((wl.layers, B, wl.n_kv_heads, wl.head_dim), device="cuda", generator=gen).to(self.tdt)
-        vd = torch.randn_like(kd)
-        od = torch.empty_like(qd)
-        n_slots = c2kv.c2kv_cache_info(cache)["n_slots"]
-        for i in range(warmup):
-            self.flush_l2()
-            c2kv.c2kv_decode(self.ctx, cache, -1, qd, kd, vd, [wl.n_suffix + i] * B, od)
-        c2kv.c2kv_sync(self.ctx)
-        keys = 0
-        for i in range(steps):
-            st = wl.n_suffix + warmup + i
-            self.flush_l2()                                    # untimed
-            events[i][0].record(self.stream)
-            c2kv.c2kv_decode(self.ctx, cache, -1, qd, kd, vd, [st] * B, od)
-            events[i][1].record(self.stream)
-            keys += int(sum(int(n) + st + 1 for n in n_slots))
-        torch.cuda.synchronize()
-        c2kv.c2kv_sync(self.ctx)
-        total = sum(ev[0].elapsed_time(ev[1]) for ev in events[:steps])
-        c2kv.c2kv_profile_read(self.ctx)
-        c2kv.c2kv_profile_enable(self.ctx, True)
-        for i in range(steps):
-            self.flush_l2()
-            c2kv.c2kv_decode(self.ctx, cache, -1, qd, kd, vd, [wl.n_suffix + warmup + steps + i] * B, od)
-        kern = c2kv.c2kv_profile_read(self.ctx)
-        c2kv.c2kv_profile_enable(self.ctx, False)
-        c2kv.c2kv_sync(self.ctx)
-        c2kv.c2kv_cache_release(self.ctx, cache)
-        return total / steps, kern["decode"][0], keys / steps
+        return decode_measure(self.c2kv, self.torch, self.ctx, self.wl, self.stream, self.req_ptr, ids,
+                              self.positions, self.q_dev, self.out, steps, warmup, events, self.flush_l2)
 
     def extract_run(self, steps, warmup, events):
         """Extraction attention over one chunk of the workload's size (n tokens, ratio k, all
@@ -420,6 +399,50 @@ class Arm:
 
     def close(self):
         self.c2kv.c2kv_destroy(self.ctx)
+
+
+def decode_measure(c2kv, torch, ctx, wl, stream, req_ptr, ids, positions, q_dev, out, steps, warmup,
+                   events, flush):
+    """Decode after the suffix: compose once, write the suffix with attend, then decode
+    `warmup` untimed and `steps` timed tokens per request (one c2kv_decode call per token,
+    all layers), L2 flushed before each; then `steps` more tokens with the library's trace
+    on, for the decode kernel's own time.  Returns (ms per timed step, mean decode kernel ms
+    from the trace, keys read per timed step summed over requests, list of step ms)."""
+    tdt = torch.float32 if wl.dtype == "f32" else torch.bfloat16
+    cache = c2kv.c2kv_compose(ctx, req_ptr, ids, positions, wl.n_suffix + warmup + 2 * steps)
+    c2kv.c2kv_attend(ctx, cache, -1, *q_dev, wl.n_suffix, out)
+    B = len(req_ptr) - 1
+    gen = torch.Generator(device="cuda").manual_seed(1)
+    qd = torch.randn((wl.layers, B, wl.n_q_heads, wl.head_dim), device="cuda", generator=gen).to(tdt)
+    kd = torch.randn((wl.layers, B, wl.n_kv_heads, wl.head_dim), device="cuda", generator=gen).to(tdt)
+    vd = torch.randn_like(kd)
+    od = torch.empty_like(qd)
+    n_slots = c2kv.c2kv_cache_info(cache)["n_slots"]
+    for i in range(warmup):
+        flush()
+        c2kv.c2kv_decode(ctx, cache, -1, qd, kd, vd, [wl.n_suffix + i] * B, od)
+    c2kv.c2kv_sync(ctx)
+    keys = 0
+    for i in range(steps):
+        st = wl.n_suffix + warmup + i
+        flush()                                            # untimed
+        events[i][0].record(stream)
+        c2kv.c2kv_decode(ctx, cache, -1, qd, kd, vd, [st] * B, od)
+        events[i][1].record(stream)
+        keys += int(sum(int(n) + st + 1 for n in n_slots))
+    torch.cuda.synchronize()
+    c2kv.c2kv_sync(ctx)
+    per = [ev[0].elapsed_time(ev[1]) for ev in events[:steps]]
+    c2kv.c2kv_profile_read(ctx)
+    c2kv.c2kv_profile_enable(ctx, True)
+    for i in range(steps):
+        flush()
+        c2kv.c2kv_decode(ctx, cache, -1, qd, kd, vd, [wl.n_suffix + warmup + steps + i] * B, od)
+    kern = c2kv.c2kv_profile_read(ctx)
+    c2kv.c2kv_profile_enable(ctx, False)
+    c2kv.c2kv_sync(ctx)
+    c2kv.c2kv_cache_release(ctx, cache)
+    return sum(per) / steps, kern["decode"][0], keys / steps, per
 
 
 def sif_visible_pairs(n, k):
@@ -485,6 +508,172 @@ def decode_line(wl, world, dec_ms, dec_kernel_ms, dec_keys, hbm, src):
                      "peak_source": f"{src} hbm_gbs", "bytes_per_launch": int(bytes_step),
                      "traffic": captured_traffic("decode_kernel", wl.name)},
     }
+
+
+# --------------------------------------------------------------------------- other workloads
+
+SIDE_WORKLOADS = ("batched", "long70b", "sweep_k1", "sweep_k4", "sweep_k8", "sweep_k10", "sweep_k16")
+
+
+def error_vs_oracle(got, ref, tol):
+    """max |gpu - oracle|, the largest relative error over elements whose oracle magnitude
+    is at least the tolerance (below it the absolute term of the bound governs), and the
+    largest ratio of the error to the element's bound tol + tol * |oracle| (parity: <= 1)."""
+    diff = np.abs(got - ref)
+    big = np.abs(ref) >= tol
+    return {"max_abs": float(diff.max()),
+            "max_rel": float((diff[big] / np.abs(ref[big])).max()) if big.any() else 0.0,
+            "tol_ratio": round(float((diff / (tol + tol * np.abs(ref))).max()), 4),
+            "tol": tol}
+
+
+def side_workload(name, steps, warmup, torch, c2kv, hbm, bf16, src, flush, with_oracle=True):
+    """One of the other workloads at full size on one GPU, through c2kv_compose_attend as the
+    headline step: the step time (median of `steps`, L2 flushed before each), the compose
+    kernel against HBM (cold, and warm: right after an identical compose, inputs in L2 where
+    they fit), the attention kernel against the bf16 tensor peak, a decode step after the
+    suffix, and the output error against the oracle on one sampled (layer, request).
+
+    The chunks of the sampled request (request 0) are synth's, so that the oracle sees the
+    same bits; the pool's other chunks are drawn on the device with the same shape and
+    outlier channels (their values do not change the timing)."""
+    wl = synth.workload(name)
+    f = workload_facts(wl)
+    tdt = torch.float32 if wl.dtype == "f32" else torch.bfloat16
+    E = torch.cuda.Event
+    stream = torch.cuda.current_stream()
+    reqs = synth.requests(wl, 0)
+    m = f["slots_per_chunk"]
+    pool_ids = sorted({c for ids, _ in reqs for c in ids})
+    t_setup = time.perf_counter()
+    ctx = c2kv.c2kv_create(wl.layers, wl.n_q_heads, wl.n_kv_heads, wl.head_dim, wl.rope_theta,
+                           c2kv.DTYPE_F32 if wl.dtype == "f32" else c2kv.DTYPE_BF16,
+                           pool_slots=len(pool_ids) * m + 64, stream=stream)
+    try:
+        sample = reqs[0]
+        mult = torch.from_numpy(synth.outlier_mask(wl, 0)).to("cuda")
+        gen = torch.Generator(device="cuda").manual_seed(3)
+        shape = (wl.layers, m, wl.n_kv_heads, wl.head_dim)
+        dev, oracle_chunks = {}, {}
+        for cid in pool_ids:
+            if cid in sample[0]:
+                ks, vs = synth.chunk_slots(wl, cid, m, 0)
+                kd, vd = (torch.from_numpy(x).to("cuda", tdt) for x in (ks, vs))
+                oracle_chunks[cid] = (ks[:1].astype(np.float64), vs[:1].astype(np.float64),
+                                      wl.chunk_tokens, wl.ratio_k)
+            else:
+                kd = (torch.randn(shape, device="cuda", generator=gen) * mult).to(tdt)
+                vd = (torch.randn(shape, device="cuda", generator=gen) * mult).to(tdt)
+            dev[cid] = c2kv.c2kv_compress_chunk(ctx, kd, vd, wl.chunk_tokens, wl.ratio_k,
+                                                c2kv.MODE_STORED)
+        req_ptr = np.cumsum([0] + [len(ids) for ids, _ in reqs]).astype(np.int32)
+        ids = [dev[c] for ids_, _ in reqs for c in ids_]
+        positions = [o for _, offs in reqs for o in offs]
+        qn, kn, vn = synth.suffix(wl, 0)
+        q_dev = [torch.from_numpy(x).to("cuda", tdt) for x in (qn, kn, vn)]
+        out = torch.empty_like(q_dev[0])
+        c2kv.c2kv_sync(ctx)
+        setup_s = time.perf_counter() - t_setup
+
+        def step():
+            cache = c2kv.c2kv_compose_attend(ctx, req_ptr, ids, positions, wl.n_suffix, *q_dev,
+                                             wl.n_suffix, out)
+            c2kv.c2kv_cache_release(ctx, cache)
+
+        def timed(fn, cold):
+            evs = [(E(enable_timing=True), E(enable_timing=True)) for _ in range(steps)]
+            for a, b in evs:
+                if cold:
+                    flush()
+                else:
+                    fn()                       # the identical call just before: inputs in L2
+                a.record(stream)
+                fn()
+                b.record(stream)
+            torch.cuda.synchronize()
+            return statistics.median(x.elapsed_time(y) for x, y in evs)
+
+        def compose_only():
+            c2kv.c2kv_cache_release(ctx, c2kv.c2kv_compose(ctx, req_ptr, ids, positions, wl.n_suffix))
+
+        for _ in range(warmup):
+            flush()
+            step()
+            compose_only()
+        c2kv.c2kv_sync(ctx)
+        step_ms = timed(step, cold=True)
+        compose_cold_ms = timed(compose_only, cold=True)
+        compose_warm_ms = timed(compose_only, cold=False)
+        c2kv.c2kv_profile_read(ctx)
+        c2kv.c2kv_profile_enable(ctx, True)
+        for _ in range(steps):
+            flush()
+            step()
+        kern = c2kv.c2kv_profile_read(ctx)
+        c2kv.c2kv_profile_enable(ctx, False)
+        c2kv.c2kv_sync(ctx)
+        fused = kern["fused"][1] > 0
+        kc = kern["compose"][0]
+        ka = kern["attention"][0] + kern["combine"][0]
+        entry = {
+            "workload": describe(wl),
+            "step_ms": round(step_ms, 5),
+            "composed_tokens_per_s": round(f["positions"] / (step_ms / 1e3), 1),
+            "route": "fused compose + attention kernel" if fused else
+                     "compose, then attention (suffix kernel beside compose)",
+        }
+        if fused:
+            entry["fused"] = fused_roofline(kern["fused"][0], f, hbm, bf16, src)
+        else:
+            comp_gbs = f["compose_bytes"] / (kc / 1e3) / 1e9
+            warm_gbs = f["compose_bytes"] / (compose_warm_ms / 1e3) / 1e9
+            attn_tfs = f["attn_flops"] / (ka / 1e3) / 1e12
+            attn_gbs = f["attn_bytes"] / (ka / 1e3) / 1e9
+            entry["compose"] = {
+                "kernel_ms": round(kc, 5), "achieved_gbs": round(comp_gbs, 1),
+                "frac": round(comp_gbs / hbm, 4), "peak": hbm, "peak_source": f"{src} hbm_gbs",
+                "bytes_per_launch": f["compose_bytes"],
+                "cold_call_ms": round(compose_cold_ms, 5), "warm_call_ms": round(compose_warm_ms, 5),
+                "warm_gbs": round(warm_gbs, 1),
+                "traffic": captured_traffic("compose_kernel", name)}
+            entry["suffix_kernel_ms"] = round(kern["suffix"][0], 5)
+            entry["attention"] = {
+                "kernel_ms": round(ka, 5), "achieved_tflops": round(attn_tfs, 2),
+                "frac": round(attn_tfs / bf16, 4), "peak": bf16,
+                "peak_source": f"{src} bf16_tflops (burst)", "flops_per_launch": f["attn_flops"],
+                "hbm_frac": round(attn_gbs / hbm, 4),
+                "split_merge_ms": round(kern["combine"][0], 5),
+                "traffic": captured_traffic("attn_tc_kernel", name)}
+        # decode after the suffix, at this workload's context length
+        dec_events = [[E(enable_timing=True) for _ in range(2)] for _ in range(steps)]
+        d_ms, d_kern, d_keys, d_per = decode_measure(c2kv, torch, ctx, wl, stream, req_ptr, ids,
+                                                      positions, q_dev, out, steps, warmup,
+                                                      dec_events, flush)
+        dline = decode_line(wl, 1, statistics.median(d_per), d_kern, d_keys, hbm, src)
+        entry["decode"] = {k: dline[k] for k in ("value", "unit", "ms_per_step", "keys_per_request",
+                                                 "kernel_ms")}
+        entry["decode"]["roofline"] = {k: dline["roofline"][k] for k in ("achieved", "frac", "unit",
+                                                                         "bytes_per_launch", "traffic")}
+        # output error against the oracle: layer 0 of request 0, every suffix row and head
+        if with_oracle:
+            cache = c2kv.c2kv_compose_attend(ctx, req_ptr, ids, positions, wl.n_suffix, *q_dev,
+                                             wl.n_suffix, out)
+            c2kv.c2kv_sync(ctx)
+            got = out[0, 0].double().cpu().numpy()
+            c2kv.c2kv_cache_release(ctx, cache)
+            from oracle import c2kv_oracle as orc
+            t0 = time.perf_counter()
+            ref = orc.run_request(oracle_chunks, sample[0], sample[1], qn[:1, 0], kn[:1, 0],
+                                  vn[:1, 0], wl.rope_theta, wl.dtype)
+            tol = 1e-5 if wl.dtype == "f32" else 2e-2
+            entry["error_vs_oracle"] = dict(error_vs_oracle(got, ref["out"][0], tol),
+                                            sample=f"layer 0 of request 0: {wl.n_suffix} suffix "
+                                                   f"tokens x {wl.n_q_heads} heads x {wl.head_dim}",
+                                            oracle_s=round(time.perf_counter() - t0, 2))
+        entry["setup_s"] = round(setup_s, 2)
+        return entry
+    finally:
+        c2kv.c2kv_destroy(ctx)
 
 
 def dist_setup():
@@ -569,6 +758,7 @@ def run_ours(args):
     compose_ms = [ev[0].elapsed_time(ev[1]) for ev in un_events]
     attend_ms = [ev[1].elapsed_time(ev[2]) for ev in un_events]
     kern_un = traced(False)
+    compose_warm_ms = arm.compose_warm(args.steps)
 
     # end to end from host buffers (host->device traffic inside the timed region), both
     # ways the library offers: zero-copy compose from pinned host slots, and staged copies
@@ -594,7 +784,7 @@ def run_ours(args):
 
     # decode after the suffix (one new token per request per step, all layers)
     dec_events = [[E(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
-    dec_ms, dec_kernel_ms, dec_keys = arm.decode_run(args.steps, args.warmup, dec_events)
+    dec_ms, dec_kernel_ms, dec_keys, _ = arm.decode_run(args.steps, args.warmup, dec_events)
 
     # extraction attention over one chunk (the encoding side, Sec. 3.3)
     ext_events = [[E(enable_timing=True) for _ in range(2)] for _ in range(args.steps)]
@@ -604,12 +794,19 @@ def run_ours(args):
     total_ms, un_total_ms, e2e_ms, staged_ms, dec_ms, ext_ms = max_over_ranks(
         [total_ms, un_total_ms, e2e_ms, staged_ms, dec_ms, ext_ms], device="cuda")
     arm.close()
+    hbm, bf16, bf16_sus, src = measured_peaks()
+    # the other workloads at full size, each on this rank's GPU (requests sharded like the
+    # headline would take a global batch; here every rank runs its own replica)
+    workloads = {}
+    if args.workloads and rank == 0:
+        for name in args.workloads.split(","):
+            workloads[name] = side_workload(name, args.side_steps, args.warmup, torch, c2kv, hbm, bf16,
+                                            src, arm.flush_l2, with_oracle=not args.no_cpu_baseline)
     if rank != 0:
         if world > 1:
             torch.distributed.destroy_process_group()
         return
 
-    hbm, bf16, bf16_sus, src = measured_peaks()
     gf = workload_facts(synth.scaled(wl, batch=wl.batch * world))   # whole job
     positions = gf["positions"] * args.steps
     value = positions / (total_ms / 1e3)
@@ -626,12 +823,13 @@ def run_ours(args):
     line = {
         "metric": METRIC, "value": round(value, 1), "unit": "tokens/s", "n_gpus": world,
         "steps": args.steps, "warmup": args.warmup,
-        "ms_per_step": round(total_ms / args.steps, 5), "higher_is_better": True,
+        "ms_per_step": round(total_ms / args.steps, 5),
+        "ms_per_step_median": round(statistics.median(step_ms), 5), "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": wl.dtype, "data": "synthetic",
-        "config": {"workload": describe(wl), "parallelism": f"dp{world}: requests sharded over ranks, no data-path collective",
-                   "l2": "flushed between timed steps (256 MB write, untimed)",
-                   "global_batch": wl.batch * world,
-                   "ttft_proxy_ms_per_layer": round(kc_ms / wl.layers, 6),
+        "config": job_config(wl, world),
+        "parallelism": f"dp{world}: requests sharded over ranks, no data-path collective",
+        "l2": "flushed between timed steps (256 MB write, untimed)",
+        "detail": {"ttft_proxy_ms_per_layer": round(kc_ms / wl.layers, 6),
                    "step": ("c2kv_compose_attend: one kernel (compose, suffix preparation and "
                             "attention fused)" if fused_ran
                             else "c2kv_compose_attend: compose, then attention"),
@@ -639,6 +837,9 @@ def run_ours(args):
                    "unfused": {"value": round(positions / (un_total_ms / 1e3), 1),
                                "ms_per_step": round(un_total_ms / args.steps, 5),
                                "compose_call_ms": round(c_ms, 5), "attend_call_ms": round(a_ms, 5),
+                               "compose_call_ms_median": round(statistics.median(compose_ms), 5),
+                               "compose_warm_call_ms": round(compose_warm_ms, 5),
+                               "compose_warm_gbs": round(f["compose_bytes"] / (compose_warm_ms / 1e3) / 1e9, 1),
                                "kernel_ms": {k: round(v[0], 5) for k, v in kern_un.items() if v[1]}},
                    "compose_gbs": round(comp_gbs, 1), "attend_tflops": round(attn_tfs, 2),
                    "compose_bytes": f["compose_bytes"], "attend_flops": f["attn_flops"],
@@ -669,6 +870,10 @@ def run_ours(args):
         "gpu_launches": sum(v[1] for v in kern.values()),
         "clocks": clk,
     }
+    if workloads:
+        # configs 3-5 (batched reuse, long context, the compression-ratio sweep with its
+        # uncompressed control), each run once at full size in the same process
+        line["workloads"] = workloads
     if not args.no_cpu_baseline:
         line["cpu_baseline"] = cpu_baseline(wl, budget_s=args.cpu_budget)
     print(json.dumps(line), flush=True)
@@ -708,43 +913,86 @@ def oracle_sample(wl, layers, seed=0):
     return time.perf_counter() - t0
 
 
-def cpu_baseline(wl, budget_s=15.0):
+def oracle_sample_one_core(wl, layers):
+    """oracle_sample in a child process confined to one core with single-threaded BLAS
+    (the thread pools are sized when numpy loads, so it takes a fresh interpreter)."""
+    code = (f"import os, sys\n"
+            f"os.sched_setaffinity(0, {{sorted(os.sched_getaffinity(0))[0]}})\n"
+            f"sys.path.insert(0, {ROOT!r})\n"
+            f"import bench, synth\n"
+            f"print('SECONDS', bench.oracle_sample(synth.workload({wl.name!r}), {layers}))\n")
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1")
+    res = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True,
+                         timeout=600)
+    for line in res.stdout.splitlines():
+        if line.startswith("SECONDS"):
+            return float(line.split()[1])
+    return None
+
+
+def cpu_baseline(wl, budget_s=15.0, one_core_budget_s=8.0):
     """The oracle as it stands on this host's cores, on a bounded sample: as many layers of
-    request 0 as fit in about `budget_s` seconds, scaled to the whole batch."""
+    request 0 as fit in about `budget_s` seconds, scaled to the whole batch; and the same on
+    one core."""
     f = workload_facts(wl)
     t1 = oracle_sample(wl, 1)
     n = int(max(1, min(wl.layers * wl.batch, budget_s // max(t1, 1e-3))))
     t = oracle_sample(wl, n)
     per_layer_req = t / n
     step_s = per_layer_req * wl.layers * wl.batch
-    return {"value": round(f["positions"] / step_s, 1), "unit": "tokens/s",
-            "cores": cpu_threads(), "kind": "oracle",
-            "sample": f"{n} (layer, request) compose+attend passes of the oracle (fp64 numpy), "
-                      f"{t:.1f} s, scaled to {wl.layers} layers x {wl.batch} requests"}
+    out = {"value": round(f["positions"] / step_s, 1), "unit": "tokens/s",
+           "cores": cpu_threads(), "kind": "oracle",
+           "sample": f"{n} (layer, request) compose+attend passes of the oracle (fp64 numpy), "
+                     f"{t:.1f} s, scaled to {wl.layers} layers x {wl.batch} requests"}
+    # one core: as many passes as fit in about one_core_budget_s at the all-core rate x 4
+    n1 = int(max(1, min(wl.layers * wl.batch, one_core_budget_s // max(4 * per_layer_req, 1e-3))))
+    t1c = oracle_sample_one_core(wl, n1)
+    if t1c:
+        out["one_core"] = {"value": round(f["positions"] / (t1c / n1 * wl.layers * wl.batch), 1),
+                           "cores": 1,
+                           "sample": f"{n1} (layer, request) passes, {t1c:.1f} s, in a child "
+                                     "process pinned to one core with single-threaded BLAS"}
+    return out
+
+
+def job_config(wl, world):
+    """The workload a line describes: the same object in both arms' lines."""
+    return {"workload": describe(wl), "global_batch": wl.batch * world}
 
 
 def run_reference(args):
+    """The oracle arm.  Each step is one bounded sample of the workload: compose + attend of
+    one layer of request 0, i.e. 1 / (layers * requests) of the whole step; ms_per_step is
+    that sample's measured time, and value is the same metric (composed positions of the
+    whole job per second) at the sample's rate."""
     world, rank, _ = dist_setup()
     if rank != 0:
         return
     wl = synth.workload(args.workload)
-    f = workload_facts(wl)
+    f = workload_facts(synth.scaled(wl, batch=wl.batch * world))
     for _ in range(args.warmup):
         oracle_sample(wl, 1)
     times = [oracle_sample(wl, 1) for _ in range(args.steps)]
-    step_s = statistics.mean(times) * wl.layers * wl.batch
-    value = f["positions"] / step_s
+    share = wl.layers * wl.batch * world                 # samples in one whole step
+    sample_s = statistics.mean(times)
+    value = f["positions"] / share / sample_s
     cores = cpu_threads()
     line = {
         "impl": "reference", "metric": METRIC, "value": round(value, 1), "unit": "tokens/s",
         "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
-        "ms_per_step": round(step_s * 1e3, 3), "higher_is_better": True, "scaling": "weak",
+        "ms_per_step": round(sample_s * 1e3, 3),
+        "ms_per_step_median": round(statistics.median(times) * 1e3, 3),
+        "step": f"one sample: compose + attend of 1 layer of request 0 (1/{share} of a whole "
+                f"step of the workload)",
+        "ms_per_whole_step_extrapolated": round(sample_s * share * 1e3, 3),
+        "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-        "config": {"workload": describe(wl), "parallelism": "cpu oracle"},
+        "config": job_config(wl, world),
+        "parallelism": "cpu oracle (rank 0 only)",
         "cpu_baseline": {"value": round(value, 1), "unit": "tokens/s", "cores": cores,
                          "kind": "oracle",
-                         "sample": f"each step: compose+attend of 1 layer of request 0, "
-                                   f"scaled x{wl.layers * wl.batch}"},
+                         "sample": f"each step: compose+attend of 1 layer of request 0 "
+                                   f"(1/{share} of the workload's step)"},
         "e2e": {"value": round(value, 1), "unit": "tokens/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
@@ -762,6 +1010,10 @@ def main():
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--attn-split", type=int, default=0,
                     help="key-range splits of the attention (0 = library's choice)")
+    ap.add_argument("--workloads", default=",".join(SIDE_WORKLOADS),
+                    help="other workloads measured after the headline ('' = none)")
+    ap.add_argument("--side-steps", type=int, default=10,
+                    help="timed steps of each other workload (median reported)")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")

@@ -63,6 +63,12 @@ typedef int32_t c2kv_status;
 #define C2KV_ATTN_SIMT   1    /* CUDA-core fp32-accumulate kernel (any dtype)        */
 #define C2KV_ATTN_TC     2    /* tcgen05 / TMEM tensor-core kernel (bf16, d = 128)    */
 
+/* c2kv_config.storage: the form stored chunk K takes in the pool */
+#define C2KV_STORAGE_LOCAL_ROPE 0   /* K carries RoPE at its chunk-local slot position p_j;
+                                       compose turns it by the occurrence offset o_i      */
+#define C2KV_STORAGE_PRE_ROPE   1   /* K kept before any positional embedding, as Sec. 3.3.1
+                                       stores it; compose applies RoPE at o_i + p_j once   */
+
 /* c2kv_compose_attend: when the fused compose + attention kernel runs */
 #define C2KV_FUSE_AUTO   0    /* when each (layer, request, KV head) has a single pair of
                                  128-row query tiles, n_suffix * Hq / Hkv <= 256: every
@@ -92,6 +98,11 @@ typedef struct c2kv_config {
                                   most SMs idle), 1 = never, n <= 16 = always n (partials
                                   merged by an exact log-sum-exp combine)                     */
     int32_t fuse;              /* C2KV_FUSE_AUTO / _NEVER / _ALWAYS (c2kv_compose_attend)     */
+    int32_t storage;           /* C2KV_STORAGE_LOCAL_ROPE (0) or C2KV_STORAGE_PRE_ROPE          */
+    int32_t attn_pairs;        /* pairs of 128-row query tiles one tensor-core attention CTA
+                                  runs in turn: 0 = chosen per launch (several only when the
+                                  launch is many waves of CTAs), n >= 1 = n (fewer where a
+                                  (layer, request, KV head) has fewer pairs)                  */
 } c2kv_config;
 
 /* Chunk metadata (c2kv_chunk_info). */
@@ -121,7 +132,7 @@ typedef struct c2kv_cache_desc {
 } c2kv_cache_desc;
 
 /* ABI version of this header (bumped on any incompatible change). */
-#define C2KV_ABI_VERSION 4
+#define C2KV_ABI_VERSION 5
 int32_t c2kv_abi_version(void);
 
 /*
@@ -145,17 +156,20 @@ c2kv_status c2kv_set_stream(c2kv_ctx* ctx, void* stream);
  * c2kv_compress_chunk -- the encoding step M: store one chunk (document) as compressed
  * slots in the device pool.  Sec. 3.2.1: a chunk of n tokens gets m = ceil(n/k) slots, one
  * per block of k consecutive tokens; Sec. 3.3.1: slot j takes the position of the last
- * token of its block, p_j = min((j+1)k, n) - 1.  The pool keeps K with RoPE applied at
- * p_j (chunk-local positions) and V as is.
+ * token of its block, p_j = min((j+1)k, n) - 1.  With cfg.storage LOCAL_ROPE (default) the
+ * pool keeps K with RoPE applied at p_j (chunk-local positions); with PRE_ROPE it keeps K
+ * before any positional embedding, as Sec. 3.3.1 stores the C2 tokens' KV.  V as is.
  *
  *   k, v     : MEANPOOL: device [L][n][Hkv][d] pre-RoPE per-token K/V.  Slot j is the mean
  *              of block j's rows divided by the block's true size (a stand-in for the
  *              trained extractor, adapted from the residual mean-pooling variant of
  *              Sec. 3.2.3).
  *              PROVIDED: device [L][m][Hkv][d] pre-RoPE slot K/V from an external
- *              extractor (the paper's C2 token K/V, Sec. 3.2.2); K is turned to p_j.
+ *              extractor (the paper's C2 token K/V, Sec. 3.2.2); K is turned to p_j
+ *              (LOCAL_ROPE) or kept as given (PRE_ROPE).
  *              STORED: host or device [L][m][Hkv][d] slots already in stored form (K at
- *              p_j), copied verbatim -- the "load from host memory" step of Appendix C.
+ *              p_j under LOCAL_ROPE, K before RoPE under PRE_ROPE), copied verbatim -- the
+ *              "load from host memory" step of Appendix C.
  *              HOST: the same stored form in pinned, device-mapped host memory, NOT copied:
  *              the chunk takes no pool slots and c2kv_compose reads it over the host link
  *              (load, re-rotation and gather in one pass).  The caller keeps the memory
@@ -189,8 +203,10 @@ c2kv_status c2kv_chunk_info(const c2kv_ctx* ctx, int32_t chunk_id, c2kv_chunk_de
  * Occurrence i of request r (chunk c_i, n_i tokens, m_i slots, offset o_i) fills rows
  * row_base[r] + D_i + j, j < m_i, D_i = sum of earlier m, for every layer:
  *     K' = R(o_i) K_stored   (turn from p_j to o_i + p_j),   V' = V_stored,
- *     pos = o_i + p_j.
- * With cfg.fixed_pos, K' = K_stored and pos = p_j.
+ *     pos = o_i + p_j
+ * under LOCAL_ROPE storage, and K' = RoPE(K_stored, o_i + p_j) under PRE_ROPE (the same
+ * cache in exact arithmetic; each rounds K' to the storage dtype once per stored form).
+ * With cfg.fixed_pos, pos = p_j and K' = K_stored (LOCAL_ROPE) or RoPE(K_stored, p_j).
  *
  *   batch           : number of requests B >= 1.
  *   req_ptr         : host [B + 1], CSR offsets into chunk_ids (req_ptr[0] = 0,
@@ -245,7 +261,7 @@ c2kv_status c2kv_attend(c2kv_ctx* ctx, c2kv_cache* cache, int32_t layer, const v
  *     c2kv_attend(ctx, *cache_out, -1, q, k_suf, v_suf, n_suffix, out, lse)
  * (the composed cache, its positions, the suffix rows, O and lse), for every layer.  On
  * the tensor-core route (bf16, d 128) with every chunk in the device pool, at most 256
- * requests and at most 512 chunk occurrences, one fused kernel does all of it: the
+ * requests, at most 512 chunk occurrences and LOCAL_ROPE storage, one fused kernel does all of it: the
  * attention reads each composed slot straight from the pool, turns K by its occurrence's
  * offset in shared memory (Sec. 3.2.4 re-rotation), turns the queries and the suffix keys by
  * their positions, and writes the composed cache as it goes, so the cache is written once
@@ -286,13 +302,22 @@ c2kv_status c2kv_compose_attend(c2kv_ctx* ctx, int32_t batch, const int32_t* req
  *   - Refused with C2KV_ERR_ARG (before anything is enqueued) when the rotated queries,
  *     Lq * batch * n_suffix * Hq * head_dim * element size bytes, exceed 16 MiB; split
  *     such a call by layer or by requests.
- *   - Every GPU on which the library's device code is loaded holds the 16 MiB until the
- *     process exits.
- *   - The first call on a device looks up the array's device address (with that device
- *     current) and keeps it; make that first call before any stream capture.
+ *   - c2kv_create looks up the array's device address on the context's device and loads
+ *     every kernel this call can launch there, so the array (and the kernels' code) is
+ *     reserved when the context is made, not at the first call: under CUDA's lazy module
+ *     loading that first call would otherwise be the moment device memory is taken.  Every
+ *     GPU on which a context is created holds the 16 MiB until the process exits.
+ *   - The current device must be the context's device (ERR_STATE otherwise).
  *   - All calls on a device share the array: calls whose GPU work overlaps (other
  *     streams, other contexts on the same device) race on it.  It keeps the last call's
  *     contents; nothing in it needs to start at zero.
+ *   - q, k_suf, v_suf, out and lse may be device memory or pinned, mapped host memory, as
+ *     for c2kv_attend; host tensors are read and written in place over the CPU-GPU link
+ *     (c2kv_attend copies them through scratch instead).  Memory the GPU cannot address is
+ *     refused with ERR_ARG.
+ *   - Unlike c2kv_attend, it never splits a work unit's key range over several CTAs (the
+ *     split partials would need scratch), so a single layer of a small batch leaves most
+ *     SMs idle; and its launches are not recorded by the trace (c2kv_profile_*).
  * Errors: as c2kv_attend, plus ERR_ARG for the size limit.
  */
 c2kv_status c2kv_attend_noalloc(c2kv_ctx* ctx, c2kv_cache* cache, int32_t layer,
@@ -317,6 +342,8 @@ c2kv_status c2kv_attend_noalloc(c2kv_ctx* ctx, c2kv_cache* cache, int32_t layer,
  *   steps : host int32[B], 0 <= steps[r] < the cache's suffix_capacity.
  *   out   : device [Lq][B][Hq][d] attention output (context dtype).
  *   lse   : device [Lq][B][Hq] fp32 natural-log softmax normaliser, or NULL.
+ * q, k_new, v_new, out and lse must be device (or managed) memory: anything else is
+ * refused with ERR_ARG before anything is enqueued.
  * The key range of each (layer, request, KV head) is split over several CTAs and merged
  * exactly (log-sum-exp); the split buffer comes from the context's memory pool.
  * Errors: ERR_ARG, ERR_STATE (cache from another context), ERR_UNSUPPORTED (head layout the
@@ -349,6 +376,8 @@ c2kv_status c2kv_decode(c2kv_ctx* ctx, c2kv_cache* cache, int32_t layer, const v
  *   n_tokens : n >= 1;  ratio_k : k >= 1.
  *   out      : device [n_layers][n + m][Hq][d] (context dtype).
  *   lse      : device [n_layers][Hq][n + m] fp32 natural-log normaliser, or NULL.
+ * q, k, v, out and lse must be device (or managed) memory: anything else is refused with
+ * ERR_ARG before anything is enqueued.
  * Errors: ERR_ARG, ERR_UNSUPPORTED (d not 64 or 128), ERR_NOMEM, ERR_CUDA.
  */
 c2kv_status c2kv_extract_attention(c2kv_ctx* ctx, int32_t n_layers, const void* q, const void* k,

@@ -30,6 +30,7 @@ DTYPE_BF16, DTYPE_F32 = 0, 1
 MODE_MEANPOOL, MODE_PROVIDED, MODE_STORED, MODE_HOST = 0, 1, 2, 3
 ATTN_AUTO, ATTN_SIMT, ATTN_TC = 0, 1, 2
 FUSE_AUTO, FUSE_NEVER, FUSE_ALWAYS = 0, 1, 2
+STORAGE_LOCAL_ROPE, STORAGE_PRE_ROPE = 0, 1
 PROF_COMPOSE, PROF_COMPRESS, PROF_SUFFIX, PROF_ATTN, PROF_COMBINE, PROF_DECODE = 0, 1, 2, 3, 4, 5
 PROF_EXTRACT, PROF_FUSED = 6, 7
 PROF_KINDS = 8
@@ -49,7 +50,8 @@ class c2kv_config(ctypes.Structure):
                 ("rope_theta", ctypes.c_double), ("dtype", ctypes.c_int32),
                 ("pool_slots", ctypes.c_int32), ("fixed_pos", ctypes.c_int32),
                 ("attn_impl", ctypes.c_int32), ("attn_split", ctypes.c_int32),
-                ("fuse", ctypes.c_int32)]
+                ("fuse", ctypes.c_int32), ("storage", ctypes.c_int32),
+                ("attn_pairs", ctypes.c_int32)]
 
 
 class c2kv_chunk_desc(ctypes.Structure):
@@ -150,9 +152,10 @@ def c2kv_last_error(ctx=None) -> str:
 
 
 def c2kv_create(layers, n_q_heads, n_kv_heads, head_dim, rope_theta, dtype, pool_slots,
-                fixed_pos=0, attn_impl=ATTN_AUTO, stream=None, attn_split=0, fuse=0):
+                fixed_pos=0, attn_impl=ATTN_AUTO, stream=None, attn_split=0, fuse=0,
+                storage=STORAGE_LOCAL_ROPE, attn_pairs=0):
     cfg = c2kv_config(layers, n_q_heads, n_kv_heads, head_dim, float(rope_theta), dtype,
-                      pool_slots, int(fixed_pos), attn_impl, attn_split, fuse)
+                      pool_slots, int(fixed_pos), attn_impl, attn_split, fuse, storage, attn_pairs)
     out = _VP()
     _check(_lib.c2kv_create(ctypes.byref(cfg), _stream_handle(stream), ctypes.byref(out)))
     return out.value

@@ -148,6 +148,15 @@ __global__ void __launch_bounds__(NW * 32) attn_simt_kernel(const __grid_constan
 
 }  // namespace
 
+cudaError_t preload_attn_simt_kernels(int dtype, int d) {
+    cudaFuncAttributes fa{};
+    if (dtype == kDtypeF32 && d == 64) return cudaFuncGetAttributes(&fa, attn_simt_kernel<float, 64>);
+    if (dtype == kDtypeF32 && d == 128) return cudaFuncGetAttributes(&fa, attn_simt_kernel<float, 128>);
+    if (dtype == kDtypeBf16 && d == 64) return cudaFuncGetAttributes(&fa, attn_simt_kernel<__nv_bfloat16, 64>);
+    if (dtype == kDtypeBf16 && d == 128) return cudaFuncGetAttributes(&fa, attn_simt_kernel<__nv_bfloat16, 128>);
+    return cudaErrorInvalidValue;
+}
+
 cudaError_t launch_attn_simt(const AttnParams& a, int dtype, int d, cudaStream_t s) {
     (void)cudaGetLastError();   // report this launch's error only, not a stale one
     const int G = a.hq / a.hkv;

@@ -1880,7 +1880,7 @@ cudaError_t prepare_tc(const AttnParams& a, TcParams& p, dim3& grid) {
     // The plain kernel runs several pairs of one (layer, request, KV head) per CTA when the
     // launch is many waves of CTAs: each CTA's fixed cost (TMEM, barriers, the first tiles
     // from HBM, the epilogue) is then paid once for several short pairs (causal extraction
-    // rows: 1 to 4 key tiles a pair).  C2KV_ATTN_PAIRS_PER_CTA overrides the choice (tests).
+    // rows: 1 to 4 key tiles a pair).  The context's attn_pairs setting caps the choice.
     int64_t pg = 1;
     if (kMulti) {                // every pair of a (layer, request, KV head) in one CTA
         if (p.n_split != 1) return cudaErrorInvalidValue;
@@ -1895,10 +1895,7 @@ cudaError_t prepare_tc(const AttnParams& a, TcParams& p, dim3& grid) {
         }();
         const int64_t ctas = pairs * a.hkv * a.lq * a.batch;
         pg = std::max<int64_t>(1, std::min<int64_t>(pairs, ctas / sms));
-        if (const char* env = std::getenv("C2KV_ATTN_PAIRS_PER_CTA")) {
-            const long v = std::strtol(env, nullptr, 10);
-            if (v >= 1) pg = std::min<int64_t>(pairs, v);
-        }
+        if (a.pairs_per_cta >= 1) pg = std::min<int64_t>(pairs, a.pairs_per_cta);
     }
     p.pairs = (int32_t)pairs;
     p.pair_group = (int32_t)pg;
@@ -1910,6 +1907,11 @@ cudaError_t prepare_tc(const AttnParams& a, TcParams& p, dim3& grid) {
 }
 
 }  // namespace
+
+cudaError_t preload_attn_tc_kernels() {
+    cudaFuncAttributes fa{};
+    return cudaFuncGetAttributes(&fa, attn_tc_kernel<false>);
+}
 
 cudaError_t launch_attn_tc(const AttnParams& a, cudaStream_t s, Hook before) {
     (void)cudaGetLastError();   // report this launch's error only, not a stale one

@@ -15,6 +15,7 @@
 #include <cstdint>
 #include <cstdio>
 #include <cstring>
+#include <initializer_list>
 #include <map>
 #include <new>
 #include <string>
@@ -63,6 +64,7 @@ struct c2kv_ctx {
     std::vector<c2kv_cache*> caches;
     int32_t inject = 0;
     int sms = 148;
+    void* noalloc_scratch = nullptr;   // c2kv_attend_noalloc's fixed array on this device
     c2kv::RopeTurns turns{};
     // second stream and events of the pipelined compose + attend (host-resident chunks)
     cudaStream_t aux = nullptr;
@@ -163,20 +165,17 @@ bool is_device_ptr(const void* p) {
 // rows in 16-byte vectors and by TMA, and a misaligned vector access would fault.
 bool aligned(const void* p, uintptr_t a = 16) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
 
-// Where a caller's tensor lives: device (or managed) memory, pinned host memory the GPU
-// reads and writes over the CPU-GPU link, or memory the CUDA runtime does not know
-// (refused: the kernels would dereference it).
-enum class Where { kDevice, kHost, kUnknown };
-Where where(const void* p) {
-    if (!p) return Where::kDevice;
-    cudaPointerAttributes a{};
-    if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
-        (void)cudaGetLastError();
-        return Where::kUnknown;
-    }
-    if (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) return Where::kDevice;
-    if (a.type == cudaMemoryTypeHost && a.devicePointer == p) return Where::kHost;
-    return Where::kUnknown;
+using c2kv::MemKind;
+using c2kv::mem_kind;
+
+// Refuses (ERR_ARG) any of the tensors that is not device or managed memory: the calls whose
+// kernels take only device tensors (decode, extraction).
+c2kv_status require_device(c2kv_ctx* c, const char* what, std::initializer_list<const void*> ps) {
+    for (const void* p : ps)
+        if (mem_kind(p) != MemKind::kDevice)
+            return fail(c, C2KV_ERR_ARG, "%s: tensors must be device memory (a pointer is host "
+                                         "memory or memory the GPU cannot address)", what);
+    return C2KV_OK;
 }
 
 bool own_cache(const c2kv_ctx* c, const c2kv_cache* cache) {
@@ -263,6 +262,9 @@ c2kv_status c2kv_create(const c2kv_config* cfg, void* stream, c2kv_ctx** out) {
             return fail(nullptr, C2KV_ERR_ARG, "create: attn_split outside [0, 16]");
         if (f.fuse < C2KV_FUSE_AUTO || f.fuse > C2KV_FUSE_ALWAYS)
             return fail(nullptr, C2KV_ERR_ARG, "create: bad fuse setting");
+        if (f.storage != C2KV_STORAGE_LOCAL_ROPE && f.storage != C2KV_STORAGE_PRE_ROPE)
+            return fail(nullptr, C2KV_ERR_ARG, "create: bad storage setting");
+        if (f.attn_pairs < 0) return fail(nullptr, C2KV_ERR_ARG, "create: attn_pairs < 0");
         if (f.attn_impl == C2KV_ATTN_TC &&
             !c2kv::attn_tc_supported(f.dtype, f.head_dim, f.n_q_heads, f.n_kv_heads))
             return fail(nullptr, C2KV_ERR_UNSUPPORTED,
@@ -278,6 +280,13 @@ c2kv_status c2kv_create(const c2kv_config* cfg, void* stream, c2kv_ctx** out) {
         if (e == cudaSuccess) e = cudaMalloc(&c->pool_v, pool_bytes);
         if (e == cudaSuccess) e = cudaMalloc(&c->d_err, sizeof(int32_t));
         if (e == cudaSuccess) e = cudaMemset(c->d_err, 0, sizeof(int32_t));
+        if (e == cudaSuccess) {
+            // c2kv_attend_noalloc's scratch array and kernels, reserved now rather than at
+            // its first call (lazy module loading)
+            const bool tc = f.attn_impl != C2KV_ATTN_SIMT &&
+                            c2kv::attn_tc_supported(f.dtype, f.head_dim, f.n_q_heads, f.n_kv_heads);
+            e = c2kv::noalloc_prepare(f.dtype, f.head_dim, tc, &c->noalloc_scratch);
+        }
         if (e == cudaSuccess) {
             cudaMemPoolProps props{};
             props.allocType = cudaMemAllocationTypePinned;
@@ -419,6 +428,7 @@ c2kv_status c2kv_compress_chunk(c2kv_ctx* c, const void* k, const void* v, int32
             a.rows_in = mode == C2KV_MODE_PROVIDED ? m : n_tokens;
             a.layers = c->cfg.layers;
             a.hkv = c->cfg.n_kv_heads;
+            a.turn = c->cfg.storage == C2KV_STORAGE_LOCAL_ROPE ? 1 : 0;
             a.rope = c->turns;
             ProfScope prof_compress(c, C2KV_PROF_COMPRESS);
             e = c2kv::launch_compress(a, c->cfg.dtype, c->cfg.head_dim, c->stream);
@@ -576,6 +586,18 @@ c2kv_status compose_plan(c2kv_ctx* c, int32_t batch, const int32_t* req_ptr, con
     return C2KV_OK;
 }
 
+// Composed slots per compose tile: the largest power of two up to kComposeTile that still
+// gives about six CTAs per SM over the launch's slots and layers, so that a small launch
+// (one layer of a few thousand slots) spreads over every SM instead of leaving a partial
+// wave of large tiles, while a large one keeps the 16-slot tiles that amortise each CTA's
+// angle table.
+int32_t compose_tile_slots(const c2kv_ctx* c, int64_t slots, int32_t n_layers, int max_ctas) {
+    if (max_ctas > 0) return c2kv::kComposeTile;    // a capped grid walks tiles anyway
+    int32_t t = c2kv::kComposeTile;
+    while (t > 2 && (slots + t - 1) / t * n_layers < 6LL * c->sms) t /= 2;
+    return t;
+}
+
 // The compose kernel over every occurrence: one launch per group of at most kMaxOcc
 // occurrences, all layers at once.
 cudaError_t compose_launch(c2kv_ctx* c, const c2kv_cache* cache, const std::vector<c2kv::OccParam>& occ,
@@ -585,6 +607,10 @@ cudaError_t compose_launch(c2kv_ctx* c, const c2kv_cache* cache, const std::vect
     cudaError_t e = cudaSuccess;
     ProfScope prof_compose(c, C2KV_PROF_COMPOSE);
     for (int32_t g0 = 0; e == cudaSuccess && g0 < n_occ; g0 += c2kv::kMaxOcc) {
+        const int32_t g1 = std::min(n_occ, g0 + c2kv::kMaxOcc);
+        int64_t slots = 0;
+        for (int32_t i = g0; i < g1; ++i) slots += occ[i].m;
+        const int32_t ts = compose_tile_slots(c, slots, n_layers, max_ctas);
         c2kv::ComposeParams pr{};
         pr.pool_k = c->pool_k;
         pr.pool_v = c->pool_v;
@@ -596,15 +622,16 @@ cudaError_t compose_launch(c2kv_ctx* c, const c2kv_cache* cache, const std::vect
         pr.rows = cache->rows;
         pr.hkv = c->cfg.n_kv_heads;
         pr.layer0 = layer0;
+        pr.tile_slots = ts;
+        pr.pre_rope = c->cfg.storage == C2KV_STORAGE_PRE_ROPE ? 1 : 0;
         pr.rope = c->turns;
         int32_t tiles = 0;
-        const int32_t g1 = std::min(n_occ, g0 + c2kv::kMaxOcc);
         for (int32_t i = g0; i < g1; ++i) {
             if (occ[i].m == 0) continue;
             c2kv::OccParam rec = occ[i];
             rec.tile_base = tiles;
             pr.occ[pr.n_occ++] = rec;
-            tiles += (rec.m + c2kv::kComposeTile - 1) / c2kv::kComposeTile;
+            tiles += (rec.m + ts - 1) / ts;
         }
         pr.n_tiles = tiles;
         e = c2kv::launch_compose(pr, c->cfg.dtype, c->cfg.head_dim, n_layers, c->stream, max_ctas);
@@ -620,7 +647,7 @@ c2kv_status attend_check(c2kv_ctx* c, const char* what, int32_t layer, const voi
     if (!aligned(q) || !aligned(k_suf) || !aligned(v_suf) || !aligned(out) || !aligned(lse, 4))
         return fail(c, C2KV_ERR_ARG, "%s: misaligned tensor pointer", what);
     for (const void* p : {q, k_suf, v_suf, static_cast<const void*>(out), static_cast<const void*>(lse)})
-        if (where(p) == Where::kUnknown)
+        if (mem_kind(p) == MemKind::kUnknown)
             return fail(c, C2KV_ERR_ARG, "%s: tensor in memory the GPU cannot address (neither device "
                                          "nor pinned, mapped host memory)", what);
     if (layer < -1 || layer >= c->cfg.layers) return fail(c, C2KV_ERR_ARG, "%s: bad layer %d", what, layer);
@@ -746,6 +773,7 @@ cudaError_t attend_run(c2kv_ctx* c, c2kv_cache* cache, int32_t layer0, int32_t l
         a.hkv = c->cfg.n_kv_heads;
         a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)c->cfg.head_dim));
         a.n_split = n_split;
+        a.pairs_per_cta = c->cfg.attn_pairs;
         a.part_o = part;
         a.part_lse = part ? part + (size_t)n_split * part_rows * c->cfg.head_dim : nullptr;
         for (int32_t i = 0; i < nb; ++i) a.req[i] = s.req[i];
@@ -836,7 +864,7 @@ cudaError_t suffix_io_open(c2kv_ctx* c, int32_t layers, int32_t B, int32_t n_suf
     io->lse_layer = (size_t)B * c->cfg.n_q_heads * n_suffix * sizeof(float);
     bool host = false;
     for (const void* p : {q, k_suf, v_suf, static_cast<const void*>(out), static_cast<const void*>(lse)})
-        host = host || where(p) == Where::kHost;
+        host = host || mem_kind(p) == MemKind::kHost;
     if (!host) return cudaSuccess;
     // q, out: q_layer each; k, v: kv_layer each; lse: lse_layer (16-byte aligned pieces)
     auto up = [](size_t x) { return (x + 255) / 256 * 256; };
@@ -1026,7 +1054,9 @@ c2kv_status c2kv_compose_attend(c2kv_ctx* c, int32_t batch, const int32_t* req_p
         const bool pairs_in_turn = pairs > 1 && c->cfg.attn_split <= 1;
         bool host_chunks = false;
         for (const auto& o : occ) host_chunks = host_chunks || o.host;
-        fuse = fuse && !host_chunks;
+        // PRE_ROPE slots turn by a position per slot, which the fused loaders' per-occurrence
+        // angle tables do not hold: compose, then attend
+        fuse = fuse && !host_chunks && c->cfg.storage == C2KV_STORAGE_LOCAL_ROPE;
         cudaError_t e = cudaSuccess;
         // suffix tensors and outputs in pinned host memory: copied through device scratch (the
         // pipelined route does this per layer group itself)
@@ -1149,6 +1179,7 @@ c2kv_status c2kv_decode(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
         if (!q || !k_new || !v_new || !steps || !out) return fail(c, C2KV_ERR_ARG, "decode: null pointer");
         if (!aligned(q) || !aligned(k_new) || !aligned(v_new) || !aligned(out) || !aligned(lse, 4))
             return fail(c, C2KV_ERR_ARG, "decode: misaligned tensor pointer");
+        if (const c2kv_status st = require_device(c, "decode", {q, k_new, v_new, out, lse})) return st;
         if (layer < -1 || layer >= c->cfg.layers) return fail(c, C2KV_ERR_ARG, "decode: bad layer %d", layer);
         if (!c2kv::decode_supported(c->cfg.dtype, c->cfg.head_dim, c->cfg.n_q_heads, c->cfg.n_kv_heads))
             return fail(c, C2KV_ERR_UNSUPPORTED, "decode: head layout not supported");
@@ -1275,6 +1306,7 @@ c2kv_status c2kv_extract_attention(c2kv_ctx* c, int32_t n_layers, const void* q,
         if (!q || !k || !v || !out) return fail(c, C2KV_ERR_ARG, "extract: null pointer");
         if (!aligned(q) || !aligned(k) || !aligned(v) || !aligned(out) || !aligned(lse, 4))
             return fail(c, C2KV_ERR_ARG, "extract: misaligned tensor pointer");
+        if (const c2kv_status st = require_device(c, "extract", {q, k, v, out, lse})) return st;
         if (n_layers < 1 || n_tokens < 1 || ratio_k < 1)
             return fail(c, C2KV_ERR_ARG, "extract: need n_layers, n_tokens, ratio_k >= 1");
         const int32_t d = c->cfg.head_dim;
@@ -1316,6 +1348,7 @@ c2kv_status c2kv_extract_attention(c2kv_ctx* c, int32_t n_layers, const void* q,
         p.hq = hq;
         p.hkv = hkv;
         p.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)d));
+        p.pairs_per_cta = c->cfg.attn_pairs;
         p.rope = c->turns;
         // the C2 rows beside the document rows on the second stream (tensor-core route)
         const bool two = c2kv::extract_uses_tc(c->cfg.dtype, d, c->cfg.n_q_heads, c->cfg.n_kv_heads) &&
@@ -1429,6 +1462,9 @@ bool attend_view(const c2kv_ctx* c, const c2kv_cache* cache, AttendView* v) {
     v->head_dim = c->cfg.head_dim;
     v->dtype = c->cfg.dtype;
     v->attn_impl = c->cfg.attn_impl;
+    v->attn_pairs = c->cfg.attn_pairs;
+    v->device = c->device;
+    v->noalloc_scratch = c->noalloc_scratch;
     v->stream = c->stream;
     v->err = c->d_err;
     v->turns = c->turns;
@@ -1442,6 +1478,18 @@ bool attend_view(const c2kv_ctx* c, const c2kv_cache* cache, AttendView* v) {
     v->n_slots = cache->n_slots.data();
     v->l_req = cache->l_req.data();
     return true;
+}
+
+MemKind mem_kind(const void* p) {
+    if (!p) return MemKind::kDevice;
+    cudaPointerAttributes a{};
+    if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+        (void)cudaGetLastError();
+        return MemKind::kUnknown;
+    }
+    if (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) return MemKind::kDevice;
+    if (a.type == cudaMemoryTypeHost && a.devicePointer == p) return MemKind::kHost;
+    return MemKind::kUnknown;
 }
 
 int32_t set_last_error(c2kv_ctx* c, int32_t code, const char* msg) {

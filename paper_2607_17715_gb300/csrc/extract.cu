@@ -385,6 +385,7 @@ cudaError_t launch_tc(const ExtractParams& p, cudaStream_t s, cudaStream_t s2, c
     a.hkv = p.hkv;
     a.scale_log2 = p.scale_log2;
     a.n_split = 1;
+    a.pairs_per_cta = p.pairs_per_cta;
     // pieces 2 and 3 write only the C2 rows (and read the rotated rows): with a second stream
     // they run beside piece 1, in the SMs its last wave of CTAs leaves idle
     cudaStream_t sc = s;

@@ -16,9 +16,9 @@ namespace c2kv {
 constexpr int kDtypeBf16 = 0;
 constexpr int kDtypeF32 = 1;
 constexpr int kMaxHalf = 64;        // head_dim / 2 for head_dim <= 128
-constexpr int kMaxOcc = 96;         // chunk occurrences per compose launch
+constexpr int kMaxOcc = 512;        // chunk occurrences per compose launch (24 KB of parameters)
 constexpr int kMaxReq = 256;        // requests per suffix / attention launch
-constexpr int kComposeTile = 16;    // composed slots per compose CTA (per layer)
+constexpr int kComposeTile = 16;    // most composed slots per compose tile (per layer)
 
 // RoPE frequency i as a fraction of a full turn in 0.64 fixed point:
 // turn[i] = round(theta^(-2i/d) / (2 pi) * 2^64).  For an integer position p the angle in
@@ -55,6 +55,9 @@ struct ComposeParams {
     int32_t n_tiles;
     int32_t hkv;
     int32_t layer0;          // layer of grid row 0 (a launch covers layers layer0 .. + gridDim.y)
+    int32_t tile_slots;      // composed slots per tile, 1 .. kComposeTile (chosen per launch)
+    int32_t pre_rope;        // 1: stored K is before RoPE; slot j of occurrence o turns by its
+                             // composed position o.delta + p_j (PRE_ROPE storage)
     RopeTurns rope;
     OccParam occ[kMaxOcc];
 };
@@ -73,6 +76,8 @@ struct CompressParams {
     int32_t one_row;         // 1 = provided (slot j is input row j); 0 = block mean
     int32_t layers;
     int32_t hkv;
+    int32_t turn;            // 1: K turned to the slot's local position p_j (LOCAL_ROPE
+                             // storage); 0: kept before RoPE (PRE_ROPE)
     RopeTurns rope;
 };
 
@@ -129,6 +134,8 @@ struct AttnParams {
     int32_t n_split;         // key-range splits per work unit (1 = write O directly)
     float* part_o;           // n_split > 1: [n_split][Lq][Btot][Sq][Hq][d] fp32, normalised
     float* part_lse;         // n_split > 1: [n_split][Lq][Btot][Hq][Sq] fp32, log2 domain
+    int32_t pairs_per_cta;   // tensor-core kernel: at most this many pairs of query tiles per
+                             // CTA (0 = chosen per launch)
     ReqParam req[kMaxReq];
 };
 
@@ -201,6 +208,7 @@ struct ExtractParams {
     int32_t hq;
     int32_t hkv;
     float scale_log2;
+    int32_t pairs_per_cta;   // the tensor-core attention launches' AttnParams::pairs_per_cta
     RopeTurns rope;
 };
 // With s2 (and the events fork and join), the tensor-core route runs the C2 rows' attention and
@@ -262,10 +270,28 @@ struct FusedSpec {
 cudaError_t prepare_attn_fused(const AttnParams& a, const FusedSpec& f);
 cudaError_t launch_attn_fused(cudaStream_t s, Hook before = {});
 
+// Loads (under CUDA's lazy module loading) the kernels of a translation unit that
+// c2kv_attend_noalloc can launch for this dtype and head_dim, so that launching them later
+// takes no device memory.
+cudaError_t preload_suffix_kernels(int dtype, int d);      // kv_kernels.cu
+cudaError_t preload_attn_simt_kernels(int dtype, int d);   // attn_simt.cu
+cudaError_t preload_attn_tc_kernels();                     // attn_tc.cu
+// The device address of c2kv_attend_noalloc's fixed scratch array on the current device, its
+// module loaded, with every kernel that call can launch (noalloc.cu); called by c2kv_create.
+cudaError_t noalloc_prepare(int dtype, int d, bool tc, void** scratch);
+
+// Where a caller's tensor lives: device (or managed) memory, pinned host memory the GPU can
+// address (mapped, same address on both sides), or memory the CUDA runtime does not know
+// (which no kernel may dereference).  NULL counts as device memory.
+enum class MemKind { kDevice, kHost, kUnknown };
+MemKind mem_kind(const void* p);
+
 // Read-only view of a context and one of its caches, for entry points defined outside
 // c2kv_api.cu (c2kv_attend_noalloc).
 struct AttendView {
-    int32_t layers, n_q_heads, n_kv_heads, head_dim, dtype, attn_impl;
+    int32_t layers, n_q_heads, n_kv_heads, head_dim, dtype, attn_impl, attn_pairs;
+    int device;              // the context's device
+    void* noalloc_scratch;   // c2kv_attend_noalloc's fixed array on that device
     cudaStream_t stream;
     int32_t* err;
     RopeTurns turns;

@@ -8,6 +8,8 @@
 // turn fraction is the low 64 bits of p * turn[i], exact integer wrap-around), converted
 // once to a float in [-1/2, 1/2) turns and handed to sincospif.  The error is about
 // 1e-7 rad at any position, where forming p * inv_freq in fp32 would lose p * 2^-24 rad.
+#include <algorithm>
+
 #include "internal.cuh"
 #include "rope.cuh"
 #include "vec16.cuh"
@@ -19,12 +21,16 @@ namespace {
 // (cos, sin) of pos * theta^(-2i/d) from the 0.64 fixed-point turn of frequency i.
 
 // ---------------------------------------------------------------------------------------
-// compose.  grid = (CTAs per layer, layers); a tile is kComposeTile consecutive slots of one
-// chunk occurrence, and CTA x takes tiles x, x + gridDim.x, ... (one each unless the launch
-// caps its CTAs).  Per tile the CTA forms the occurrence's d/2 (cos, sin) of delta in shared
-// memory, then streams the tile: per item (slot, head, vector pair) four 16-byte loads of
-// stored K/V, K turned, four 16-byte stores into the composed cache.  IPT items per
-// thread are loaded before any is stored, so 16 loads per thread are in flight.
+// compose.  grid = (CTAs per layer, layers); a tile is P.tile_slots (<= kComposeTile)
+// consecutive slots of one chunk occurrence, and CTA x takes tiles x, x + gridDim.x, ...
+// (one each unless the launch caps its CTAs).  Per tile the CTA forms the d/2 (cos, sin) of
+// the turn in shared memory -- once for the occurrence's offset delta (LOCAL_ROPE storage),
+// or per slot for its composed position delta + p_j (PRE_ROPE storage, K stored before
+// RoPE) -- then streams the tile: per item (slot, head, vector pair) four 16-byte loads of
+// stored K/V, K turned, four 16-byte stores into the composed cache.  IPT items per thread
+// are loaded before any is stored, so 16 loads per thread are in flight.  The launch sizes
+// the CTA to the tile (tile items / IPT threads, 32 to 256), so a launch of small tiles
+// keeps every thread's loads in flight and spreads evenly over the SMs.
 // ---------------------------------------------------------------------------------------
 template <typename T, int VPH>
 __global__ void __launch_bounds__(256) compose_kernel(const __grid_constant__ ComposeParams P) {
@@ -33,8 +39,9 @@ __global__ void __launch_bounds__(256) compose_kernel(const __grid_constant__ Co
     constexpr int HALF = VPH * E;
     constexpr int D = 2 * HALF;
     constexpr int IPT = 4;
-    __shared__ float2 cs[HALF];
+    __shared__ float2 cs[kComposeTile * HALF];
     const int l = P.layer0 + (int)blockIdx.y;
+    const int ts = P.tile_slots;
     for (int tile = blockIdx.x; tile < P.n_tiles; tile += gridDim.x) {
         int lo = 0, hi = P.n_occ - 1;
         while (lo < hi) {                       // last occurrence whose tile_base <= tile
@@ -43,10 +50,19 @@ __global__ void __launch_bounds__(256) compose_kernel(const __grid_constant__ Co
             else hi = mid - 1;
         }
         const OccParam& o = P.occ[lo];
-        const int j0 = (tile - o.tile_base) * kComposeTile;
-        const int ns = min(kComposeTile, o.m - j0);
+        const int j0 = (tile - o.tile_base) * ts;
+        const int ns = min(ts, o.m - j0);
         __syncthreads();                        // the previous tile is done with cs
-        if (threadIdx.x < HALF) cs[threadIdx.x] = turn_cs(P.rope.turn[threadIdx.x], o.delta);
+        if (!P.pre_rope) {
+            for (int i = threadIdx.x; i < HALF; i += blockDim.x) cs[i] = turn_cs(P.rope.turn[i], o.delta);
+        } else {
+            // row s of the table: slot j0 + s at its composed position delta + p_j
+            for (int e = threadIdx.x; e < ns * HALF; e += blockDim.x) {
+                const int s = e / HALF, i = e - s * HALF;
+                const int64_t pos = (int64_t)o.delta + min((j0 + s + 1) * o.k, o.n) - 1;
+                cs[e] = turn_cs(P.rope.turn[i], pos);
+            }
+        }
         __syncthreads();
         if (ns <= 0) continue;                  // the same for the whole CTA
 
@@ -58,14 +74,15 @@ __global__ void __launch_bounds__(256) compose_kernel(const __grid_constant__ Co
         const int items = ns * pairs;
         const int64_t row_elems = (int64_t)P.hkv * D;
 
-        for (int base = 0; base < items; base += 256 * IPT) {
+        const int nthr = (int)blockDim.x;
+        for (int base = 0; base < items; base += nthr * IPT) {
             uint4 kx[IPT], ky[IPT], vx[IPT], vy[IPT];
             int64_t dof[IPT];
             int civ[IPT];
             bool live[IPT];
     #pragma unroll
             for (int u = 0; u < IPT; ++u) {
-                const int it = base + u * 256 + (int)threadIdx.x;
+                const int it = base + u * nthr + (int)threadIdx.x;
                 live[u] = it < items;
                 if (!live[u]) continue;
                 const int s = it / pairs;
@@ -81,7 +98,7 @@ __global__ void __launch_bounds__(256) compose_kernel(const __grid_constant__ Co
                     continue;
                 }
                 dof[u] = ((int64_t)l * P.rows + dst) * row_elems + h * D + iv * E;
-                civ[u] = iv * E;
+                civ[u] = (P.pre_rope ? s * HALF : 0) + iv * E;
                 const T* sk;
                 const T* sv;
                 if (o.host) {       // host-resident chunk: [L][m][Hkv][d] read over the host link
@@ -117,7 +134,8 @@ __global__ void __launch_bounds__(256) compose_kernel(const __grid_constant__ Co
 
 // ---------------------------------------------------------------------------------------
 // compress: one item = (layer, slot, head, vector pair).  Mean of the block's rows (or the
-// provided slot row), K turned to the slot's local position, both stored in the pool.
+// provided slot row), K turned to the slot's local position (LOCAL_ROPE storage; kept as is
+// under PRE_ROPE), both stored in the pool.
 // ---------------------------------------------------------------------------------------
 template <typename T, int VPH>
 __global__ void __launch_bounds__(256) compress_kernel(const __grid_constant__ CompressParams P) {
@@ -181,11 +199,19 @@ __global__ void __launch_bounds__(256) compress_kernel(const __grid_constant__ C
         }
         // slot j sits at the last token of its block (provided slots: same rule)
         const int64_t p_local = (int64_t)min((j + 1) * P.k, P.n) - 1;
-        float2 cs[E];
-#pragma unroll
-        for (int e = 0; e < E; ++e) cs[e] = turn_cs(P.rope.turn[iv * E + e], p_local);
         float gx[E], gy[E];
-        rotate<E>(sx, sy, cs, gx, gy);
+        if (P.turn) {
+            float2 cs[E];
+#pragma unroll
+            for (int e = 0; e < E; ++e) cs[e] = turn_cs(P.rope.turn[iv * E + e], p_local);
+            rotate<E>(sx, sy, cs, gx, gy);
+        } else {            // PRE_ROPE storage: the slot's K before any positional embedding
+#pragma unroll
+            for (int e = 0; e < E; ++e) {
+                gx[e] = sx[e];
+                gy[e] = sy[e];
+            }
+        }
         const int64_t dof =
             ((int64_t)l * P.pool_slots + P.slot_base + j) * row_elems + h * D + iv * E;
         st16(pk + dof, V::pack(gx));
@@ -342,13 +368,29 @@ int vph_of(int dtype, int d) { return d / 2 / (dtype == kDtypeBf16 ? 8 : 4); }
         else return cudaErrorInvalidValue;                                                     \
     } while (0)
 
+cudaError_t preload_suffix_kernels(int dtype, int d) {
+    cudaFuncAttributes fa{};
+    if (dtype == kDtypeBf16 && d == 128) return cudaFuncGetAttributes(&fa, suffix_kernel<__nv_bfloat16, 8>);
+    if (dtype == kDtypeBf16 && d == 64) return cudaFuncGetAttributes(&fa, suffix_kernel<__nv_bfloat16, 4>);
+    if (dtype == kDtypeF32 && d == 128) return cudaFuncGetAttributes(&fa, suffix_kernel<float, 16>);
+    if (dtype == kDtypeF32 && d == 64) return cudaFuncGetAttributes(&fa, suffix_kernel<float, 8>);
+    return cudaErrorInvalidValue;
+}
+
 cudaError_t launch_compose(const ComposeParams& p, int dtype, int d, int layers, cudaStream_t s,
                            int max_ctas) {
     if (p.n_tiles == 0 || p.n_occ == 0) return cudaSuccess;
     (void)cudaGetLastError();   // report this launch's error only, not a stale one
-    if (layers > 65535) return cudaErrorInvalidValue;
+    if (layers > 65535 || p.tile_slots < 1 || p.tile_slots > kComposeTile) return cudaErrorInvalidValue;
     const dim3 grid(max_ctas > 0 && max_ctas < p.n_tiles ? max_ctas : p.n_tiles, layers);
-    C2KV_DISPATCH(compose_kernel, grid, p, dtype, d, s);
+    // one thread per four items of a tile (item = slot, head, vector pair), in whole warps
+    const int items = p.tile_slots * p.hkv * vph_of(dtype, d);
+    const int threads = std::min(256, std::max(32, (items / 4 + 31) / 32 * 32));
+    if (dtype == kDtypeBf16 && d == 128) compose_kernel<__nv_bfloat16, 8><<<grid, threads, 0, s>>>(p);
+    else if (dtype == kDtypeBf16 && d == 64) compose_kernel<__nv_bfloat16, 4><<<grid, threads, 0, s>>>(p);
+    else if (dtype == kDtypeF32 && d == 128) compose_kernel<float, 16><<<grid, threads, 0, s>>>(p);
+    else if (dtype == kDtypeF32 && d == 64) compose_kernel<float, 8><<<grid, threads, 0, s>>>(p);
+    else return cudaErrorInvalidValue;
     return cudaGetLastError();
 }
 

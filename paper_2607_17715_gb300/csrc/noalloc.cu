@@ -13,16 +13,21 @@
 //   * the array holds kNoAllocScratchBytes (16 MiB); requests whose rotated queries need
 //     more (layers * batch * n_suffix * Hq * head_dim * element size) are refused with
 //     C2KV_ERR_ARG before anything is enqueued;
-//   * every GPU on which the library's device code is loaded holds the array until the
-//     process exits;
-//   * the first call on a device looks the array's device address up (cudaGetSymbolAddress,
-//     with that device current) and caches it; make that first call before any stream
-//     capture;
+//   * c2kv_create looks the array's device address up (cudaGetSymbolAddress, with the
+//     context's device current) and loads every kernel this call can launch: under CUDA's
+//     lazy module loading the first use of a module is when its device memory (static
+//     arrays, code) is taken, and that must not be this call.  Every GPU on which a context
+//     is created holds the array until the process exits;
+//   * the current device must be the context's (the address belongs to that device);
 //   * every call on a device shares the one array: two calls whose work overlaps on the
 //     GPU (different streams, or different contexts on one device) race on it.  The array
 //     keeps the last call's contents; nothing in it needs to start at zero, because each
-//     call writes every rotated query row it later reads.
-#include <mutex>
+//     call writes every rotated query row it later reads;
+//   * suffix tensors in pinned, mapped host memory are read and written in place (there is
+//     no scratch to stage them through); memory the GPU cannot address is refused;
+//   * a work unit's key range is never split over several CTAs (that needs scratch for the
+//     partials), and the launches are not traced.
+#include <initializer_list>
 
 #include "c2kv.h"
 #include "internal.cuh"
@@ -30,36 +35,29 @@
 namespace {
 
 constexpr size_t kNoAllocScratchBytes = size_t(16) << 20;
-constexpr int kMaxDevices = 64;
 
 static __device__ __align__(256) unsigned char g_attend_scratch[kNoAllocScratchBytes];
-
-std::mutex g_scratch_mu;
-void* g_scratch_addr[kMaxDevices] = {};
-
-// Device address of g_attend_scratch on the current device (looked up once per device).
-cudaError_t scratch_address(void** out) {
-    *out = nullptr;
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return e;
-    if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
-    std::lock_guard<std::mutex> lock(g_scratch_mu);
-    if (!g_scratch_addr[dev]) {
-        void* p = nullptr;
-        e = cudaGetSymbolAddress(&p, g_attend_scratch);
-        if (e != cudaSuccess) return e;
-        g_scratch_addr[dev] = p;
-    }
-    *out = g_scratch_addr[dev];
-    return cudaSuccess;
-}
 
 c2kv_status refuse(c2kv_ctx* ctx, c2kv_status code, const char* msg) {
     return c2kv::set_last_error(ctx, code, msg);
 }
 
 }  // namespace
+
+namespace c2kv {
+
+cudaError_t noalloc_prepare(int dtype, int d, bool tc, void** scratch) {
+    *scratch = nullptr;
+    void* p = nullptr;
+    cudaError_t e = cudaGetSymbolAddress(&p, g_attend_scratch);
+    if (e == cudaSuccess) e = preload_suffix_kernels(dtype, d);
+    if (e == cudaSuccess) e = tc ? preload_attn_tc_kernels() : preload_attn_simt_kernels(dtype, d);
+    if (e != cudaSuccess) return e;
+    *scratch = p;
+    return cudaSuccess;
+}
+
+}  // namespace c2kv
 
 extern "C" c2kv_status c2kv_attend_noalloc(c2kv_ctx* ctx, c2kv_cache* cache, int32_t layer,
                                            const void* q, const void* k_suf, const void* v_suf,
@@ -74,6 +72,11 @@ extern "C" c2kv_status c2kv_attend_noalloc(c2kv_ctx* ctx, c2kv_cache* cache, int
     if (misaligned(q, 16) || misaligned(k_suf, 16) || misaligned(v_suf, 16) || misaligned(out, 16) ||
         misaligned(lse, 4))
         return refuse(ctx, C2KV_ERR_ARG, "attend_noalloc: misaligned tensor pointer");
+    for (const void* p : {q, k_suf, v_suf, static_cast<const void*>(out), static_cast<const void*>(lse)})
+        if (c2kv::mem_kind(p) == c2kv::MemKind::kUnknown)
+            return refuse(ctx, C2KV_ERR_ARG,
+                          "attend_noalloc: tensor in memory the GPU cannot address (neither device "
+                          "nor pinned, mapped host memory)");
     if (layer < -1 || layer >= v.layers)
         return refuse(ctx, C2KV_ERR_ARG, "attend_noalloc: bad layer");
     if (n_suffix < 1 || n_suffix > v.suffix_capacity)
@@ -89,12 +92,16 @@ extern "C" c2kv_status c2kv_attend_noalloc(c2kv_ctx* ctx, c2kv_cache* cache, int
                       "16 MiB scratch array (layers * batch * n_suffix * Hq * head_dim * "
                       "element size); split the call by layer or by request batch, or use "
                       "c2kv_attend");
-    void* q_rot = nullptr;
-    cudaError_t e = scratch_address(&q_rot);
-    if (e != cudaSuccess) {
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess) {
         (void)cudaGetLastError();
-        return refuse(ctx, C2KV_ERR_CUDA, "attend_noalloc: cannot resolve the scratch array");
+        return refuse(ctx, C2KV_ERR_CUDA, "attend_noalloc: cannot read the current device");
     }
+    if (dev != v.device || v.noalloc_scratch == nullptr)
+        return refuse(ctx, C2KV_ERR_STATE,
+                      "attend_noalloc: the current device is not the context's device");
+    void* const q_rot = v.noalloc_scratch;
+    cudaError_t e = cudaSuccess;
     const bool use_tc = v.attn_impl != C2KV_ATTN_SIMT &&
                         c2kv::attn_tc_supported(v.dtype, v.head_dim, v.n_q_heads, v.n_kv_heads);
     for (int32_t b0 = 0; e == cudaSuccess && b0 < B; b0 += c2kv::kMaxReq) {
@@ -139,6 +146,7 @@ extern "C" c2kv_status c2kv_attend_noalloc(c2kv_ctx* ctx, c2kv_cache* cache, int
         a.hq = v.n_q_heads;
         a.hkv = v.n_kv_heads;
         a.scale_log2 = (float)(1.4426950408889634 / __builtin_sqrt((double)v.head_dim));
+        a.pairs_per_cta = v.attn_pairs;
         for (int32_t i = 0; i < nb; ++i) a.req[i] = s.req[i];
         e = use_tc ? c2kv::launch_attn_tc(a, v.stream)
                    : c2kv::launch_attn_simt(a, v.dtype, v.head_dim, v.stream);

@@ -31,7 +31,7 @@ import numpy as np
 
 __all__ = [
     "Workload", "WORKLOADS", "workload", "round_f32_to_bf16", "chunk_tokens",
-    "chunk_slots", "requests", "suffix", "scaled",
+    "chunk_slots", "requests", "suffix", "scaled", "outlier_mask",
 ]
 
 SWEEP_RATIOS = (1, 4, 8, 10, 16)
@@ -110,7 +110,7 @@ def _rng(seed: int, *stream: int) -> np.random.Generator:
 _TAG_OUTLIER, _TAG_CHUNK, _TAG_SLOTS, _TAG_REQ, _TAG_SUFFIX, _TAG_EXTRACT = 1, 2, 3, 4, 5, 6
 
 
-def _outlier_mask(wl: Workload, seed: int) -> np.ndarray:
+def outlier_mask(wl: Workload, seed: int = 0) -> np.ndarray:
     """Per-(head, channel) multiplier [Hkv, d]: 1 everywhere except the outlier channels."""
     rng = _rng(seed, _TAG_OUTLIER)
     mult = np.ones((wl.n_kv_heads, wl.head_dim), dtype=np.float32)
@@ -134,7 +134,7 @@ def chunk_tokens(wl: Workload, chunk_id: int, seed: int = 0, n_tokens: int | Non
     n = wl.chunk_tokens if n_tokens is None else n_tokens
     rng = _rng(seed, _TAG_CHUNK, chunk_id)
     shape = (wl.layers, n, wl.n_kv_heads, wl.head_dim)
-    mult = _outlier_mask(wl, seed)
+    mult = outlier_mask(wl, seed)
     k = rng.standard_normal(shape, dtype=np.float32) * mult
     v = rng.standard_normal(shape, dtype=np.float32) * mult
     return _finish(k, wl.dtype), _finish(v, wl.dtype)
@@ -145,7 +145,7 @@ def chunk_slots(wl: Workload, chunk_id: int, n_slots: int, seed: int = 0):
     storage tier would hand back for a chunk (used by the load / STORED path)."""
     rng = _rng(seed, _TAG_SLOTS, chunk_id)
     shape = (wl.layers, n_slots, wl.n_kv_heads, wl.head_dim)
-    mult = _outlier_mask(wl, seed)
+    mult = outlier_mask(wl, seed)
     k = rng.standard_normal(shape, dtype=np.float32) * mult
     v = rng.standard_normal(shape, dtype=np.float32) * mult
     return _finish(k, wl.dtype), _finish(v, wl.dtype)

@@ -31,11 +31,12 @@ def to_dev(x, wl):
     return torch.from_numpy(np.ascontiguousarray(x, dtype=np.float32)).to("cuda", tdtype(wl))
 
 
-def make_ctx(wl, pool_slots, attn_impl=0, fixed_pos=0, attn_split=0, fuse=0):
+def make_ctx(wl, pool_slots, attn_impl=0, fixed_pos=0, attn_split=0, fuse=0, storage=0, attn_pairs=0):
     c2kv = lib()
     return c2kv.c2kv_create(wl.layers, wl.n_q_heads, wl.n_kv_heads, wl.head_dim, wl.rope_theta,
                             dcode(wl), pool_slots, fixed_pos=fixed_pos, attn_impl=attn_impl,
-                            stream=torch.cuda.current_stream(), attn_split=attn_split, fuse=fuse)
+                            stream=torch.cuda.current_stream(), attn_split=attn_split, fuse=fuse,
+                            storage=storage, attn_pairs=attn_pairs)
 
 
 def pool_rows(ctx, wl, chunk_id, pool_slots):

@@ -49,7 +49,7 @@ def test_binding_names_match_header(c2kv, repo_root):
 
 
 def test_abi_version(c2kv):
-    assert c2kv.c2kv_abi_version() == 4
+    assert c2kv.c2kv_abi_version() == 5
 
 
 @pytest.mark.parametrize("args,status", [

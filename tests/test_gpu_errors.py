@@ -165,3 +165,45 @@ def test_destroy_releases_live_caches():
         c2kv.c2kv_compose(c, [0, 1], [a], None, 4)
     c2kv.c2kv_destroy(c)          # must free the three caches without error
     assert np.isfinite(1.0)
+
+
+def test_device_only_calls_refuse_host_memory(ctx):
+    # decode and extraction take device tensors only; attend_noalloc takes device or pinned
+    # host tensors; pageable host memory (which no kernel may dereference) is refused by all
+    # three with ERR_ARG before anything is enqueued
+    c2kv = H.lib()
+    a = _chunk(ctx)
+    cache = c2kv.c2kv_compose(ctx, [0, 1], [a], None, 8)
+    q = torch.zeros((2, 1, 4, WL.n_q_heads, WL.head_dim), device="cuda", dtype=torch.bfloat16)
+    kv = torch.zeros((2, 1, 4, WL.n_kv_heads, WL.head_dim), device="cuda", dtype=torch.bfloat16)
+    out = torch.empty_like(q)
+    pageable = torch.zeros(q.shape, dtype=torch.bfloat16)              # torch CPU tensor
+    numpy_buf = np.zeros((2, 1, 4, WL.n_kv_heads, WL.head_dim), np.float32)  # 16-byte aligned
+    assert numpy_buf.ctypes.data % 16 == 0
+    steps = np.zeros(1, np.int32)
+    qd = q[:, :, 0].contiguous()
+    kd = kv[:, :, 0].contiguous()
+    od = torch.empty_like(qd)
+    for bad in (torch.zeros(qd.shape, dtype=torch.bfloat16),
+                torch.zeros(qd.shape, dtype=torch.bfloat16).pin_memory()):
+        assert _status(c2kv.c2kv_decode, ctx, cache, -1, bad, kd, kd, steps, od) == c2kv.ERR_ARG
+        assert _status(c2kv.c2kv_decode, ctx, cache, -1, qd, kd, kd, steps, bad) == c2kv.ERR_ARG
+    assert _status(c2kv.c2kv_decode, ctx, cache, -1, qd, numpy_buf[:, :, 0].copy(), kd, steps,
+                   od) == c2kv.ERR_ARG
+    n, k = 3, 1
+    xq = torch.zeros((1, 6, WL.n_q_heads, WL.head_dim), device="cuda", dtype=torch.bfloat16)
+    xk = torch.zeros((1, 6, WL.n_kv_heads, WL.head_dim), device="cuda", dtype=torch.bfloat16)
+    xo = torch.empty_like(xq)
+    for bad in (torch.zeros(xq.shape, dtype=torch.bfloat16),
+                torch.zeros(xq.shape, dtype=torch.bfloat16).pin_memory()):
+        assert _status(c2kv.c2kv_extract_attention, ctx, 1, bad, xk, xk, n, k, xo) == c2kv.ERR_ARG
+        assert _status(c2kv.c2kv_extract_attention, ctx, 1, xq, xk, xk, n, k, bad) == c2kv.ERR_ARG
+    assert _status(c2kv.c2kv_attend_noalloc, ctx, cache, -1, q, kv, kv, 4, pageable) == c2kv.ERR_ARG
+    assert _status(c2kv.c2kv_attend_noalloc, ctx, cache, -1, q, numpy_buf, kv, 4, out) == c2kv.ERR_ARG
+    assert "cannot address" in c2kv.c2kv_last_error(ctx)
+    # nothing was enqueued, and the context still works
+    c2kv.c2kv_decode(ctx, cache, -1, qd, kd, kd, steps, od)
+    c2kv.c2kv_extract_attention(ctx, 1, xq, xk, xk, n, k, xo)
+    c2kv.c2kv_sync(ctx)
+    assert torch.isfinite(od.float()).all() and torch.isfinite(xo.float()).all()
+    c2kv.c2kv_cache_release(ctx, cache)

@@ -13,11 +13,11 @@ L8B = synth.workload("llama8b")
 TINY = synth.workload("tiny_f32")
 
 
-def _extract_case(wl, n, k, layers=1, chunk_id=0):
+def _extract_case(wl, n, k, layers=1, chunk_id=0, attn_pairs=0):
     c2kv = H.lib()
     wl = synth.scaled(wl, layers=layers)
     q, kk, v = synth.extraction_inputs(wl, chunk_id, n, k)
-    ctx = H.make_ctx(wl, pool_slots=64)
+    ctx = H.make_ctx(wl, pool_slots=64, attn_pairs=attn_pairs)
     try:
         qd, kd, vd = (H.to_dev(x, wl) for x in (q, kk, v))
         out = torch.full_like(qd, float("nan"))
@@ -95,11 +95,10 @@ def test_extract_without_lse_matches_with_lse():
 
 
 @pytest.mark.parametrize("per_cta", [2, 3, 8])
-def test_extract_pairs_run_in_turn(per_cta, monkeypatch):
+def test_extract_pairs_run_in_turn(per_cta):
     # the attention launches of the call with several pairs of query tiles per CTA (the
     # document rows have 8 pairs of 1 to 4 key tiles at n = 512): 3 leaves a group of two
-    monkeypatch.setenv("C2KV_ATTN_PAIRS_PER_CTA", str(per_cta))
-    _extract_case(L8B, 512, 4, layers=1)
+    _extract_case(L8B, 512, 4, layers=1, attn_pairs=per_cta)
 
 
 def test_extract_two_layers_gqa8():

@@ -79,6 +79,16 @@ def _run_full(wl, from_tokens, sample_layers, sample_reqs, seed=0, fuse=0):
                 # (or fp32 sum error relative to the block's inputs)
                 scale = np.concatenate([v_scale[c] for c in ids], axis=1)
                 H.check_rounded(gv, ref["v"], scale, wl, f"{wl.name} V req {r}")
+                # composed K: the oracle's compose of the slots the GPU stored (the compress
+                # step is checked above through V and below through O) within one ulp
+                pool = len(pool_ids) * m + 8
+                gpu_chunks = {}
+                for c in set(ids):
+                    pk, pv = H.pool_rows(ctx, wl, dev[c], pool)
+                    gpu_chunks[c] = (pk[sample_layers], pv[sample_layers], wl.chunk_tokens, wl.ratio_k)
+                ck, _, _, _ = orc.compose(gpu_chunks, ids, offs, wl.rope_theta, wl.dtype)
+                stored = np.concatenate([gpu_chunks[c][0] for c in ids], axis=1)
+                H.check_rotated(gk, ck, stored, wl, f"{wl.name} K req {r}")
             else:
                 assert np.array_equal(gv, ref["v"])
                 stored = np.concatenate([oracle_chunks[c][0] for c in ids], axis=1)

@@ -43,7 +43,7 @@ def _run(ctx, wl, dev, reqs, q, ks, vs, sq, fused, host_io=False):
 
 
 def _fused_case(wl, reqs=None, n_suffix=None, attn_split=0, host=(), fixed_pos=False,
-                compare_unfused=True, fuse=2, host_io=False):
+                compare_unfused=True, fuse=2, host_io=False, attn_pairs=0):
     """compose_attend with the fused kernel forced (fuse=2) unless it cannot take the call,
     checked against the oracle and, bit for bit, against compose + attend."""
     c2kv = H.lib()
@@ -54,7 +54,7 @@ def _fused_case(wl, reqs=None, n_suffix=None, attn_split=0, host=(), fixed_pos=F
     chunks = H.oracle_chunks_meanpool(wl, all_ids)
     pool = sum(chunks[c][0].shape[1] for c in all_ids) + 16
     ctx = H.make_ctx(wl, pool_slots=pool, attn_split=attn_split, fixed_pos=int(fixed_pos),
-                     fuse=fuse)
+                     fuse=fuse, attn_pairs=attn_pairs)
     keep = []
     try:
         dev = H.load_stored(ctx, wl, chunks, host=host, keep=keep)
@@ -167,13 +167,12 @@ def test_fused_suffix_at_tile_edges(n_suffix):
 
 
 @pytest.mark.parametrize("per_cta", [2, 3])
-def test_attend_pairs_run_in_turn(per_cta, monkeypatch):
+def test_attend_pairs_run_in_turn(per_cta):
     # compose, then attention with several pairs of query tiles per CTA: 200 suffix tokens
     # are 7 query tiles, i.e. 4 pairs, the last without a tile B
-    monkeypatch.setenv("C2KV_ATTN_PAIRS_PER_CTA", str(per_cta))
     wl = synth.scaled(L8B, layers=2, chunk_tokens=300, ratio_k=4, chunks_per_request=3,
                       pool_chunks=3, n_suffix=200)
-    _fused_case(wl, fuse=1)
+    _fused_case(wl, fuse=1, attn_pairs=per_cta)
 
 
 @pytest.mark.parametrize("split", [2, 5])
