@@ -128,6 +128,7 @@ struct TcParams {                // CUtensorMap members carry their own alignmen
     CUtensorMap tm_q;        // q_rot   [Lq*Btot][Sq'][Hq][128] box {64, G, TQ, 1}; Sq' = sq_pitch
     CUtensorMap tm_k;        // cache K [L*rows][Hkv][128]      box {64, 1, 128}
     CUtensorMap tm_v;        // cache V, same
+    CUtensorMap tm_o;        // out, laid out and boxed like tm_q (the epilogue's TMA stores)
     void* out;
     float* lse;
     int32_t* err;
@@ -316,6 +317,18 @@ __device__ __forceinline__ float fmax3(float a, float b, float c) {
     return d;
 }
 
+// A 4-D tile of shared memory to global memory by TMA (bulk async-group of the thread).
+__device__ __forceinline__ void tma_store_4d(const CUtensorMap* tm, uint32_t src, int c0, int c1, int c2, int c3) {
+    asm volatile("cp.async.bulk.tensor.4d.global.shared::cta.bulk_group [%0, {%1, %2, %3, %4}], [%5];" ::"l"(
+                     reinterpret_cast<uint64_t>(tm)),
+                 "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(src)
+                 : "memory");
+}
+__device__ __forceinline__ void sts128_(uint32_t a, const uint4& v) {
+    asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(a), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+                 : "memory");
+}
+
 // The query tokens and key tiles of pair pr of query tiles (split sp of its key range).
 struct PairSpan {
     int t0a, t0b;       // first suffix token of tile A, of tile B
@@ -342,12 +355,15 @@ __device__ __forceinline__ PairSpan pair_span(const TcParams& P, int pr, int sp,
 // epilogue.  r = TMEM lane (row within the tile), t0 = first suffix token of the tile.
 // sf_base: S_x tiles completed in earlier pairs (phase count); od_par: the phase of B_OD that
 // closes this pair; arrive_oe: tell the issuer (B_OE) once O has been read, when the CTA
-// runs further pairs.
+// runs further pairs.  stage: the Q tiles' shared memory when this is the CTA's last pair
+// (no further Q will land there), else 0: O then leaves through it, the tile's rows written
+// in the 128-byte-swizzled layout and stored by TMA, instead of 16-byte stores of a row per
+// thread (which touch a separate cache line per thread).
 __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, uint32_t sBar, int x,
                                             int quad, int lane, int t0, int l, int bl, int b,
                                             int hk, int sp, int j_base, int n_kv, uint32_t sf_base,
                                             uint32_t od_par, bool arrive_oe,
-                                            volatile uint32_t* abort) {
+                                            volatile uint32_t* abort, uint32_t stage = 0u) {
     auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
     const int G = P.group;
     const int s_r = P.req[bl].n_slots;
@@ -445,6 +461,43 @@ __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, u
     const float inv = any ? 1.0f / l_run : 0.f;
     const int64_t row_id = (((int64_t)l * P.batch_total + b) * P.sq_pitch + t) * P.hq + hk * G + g;
     const int64_t lse_id = (((int64_t)l * P.batch_total + b) * P.hq + hk * G + g) * P.sq_pitch + t;
+    if (P.n_split == 1 && stage != 0u && n_kv > 0) {
+        const uint32_t sbase = stage + (uint32_t)x * TILE;
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            uint32_t ov[32];
+            tmem_ld32(tmem + lane_addr + colO + c * 32, ov);
+            tmem_ld_wait();
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+                uint4 w;
+                w.x = pack_bf16(__uint_as_float(ov[k * 8 + 0]) * inv, __uint_as_float(ov[k * 8 + 1]) * inv);
+                w.y = pack_bf16(__uint_as_float(ov[k * 8 + 2]) * inv, __uint_as_float(ov[k * 8 + 3]) * inv);
+                w.z = pack_bf16(__uint_as_float(ov[k * 8 + 4]) * inv, __uint_as_float(ov[k * 8 + 5]) * inv);
+                w.w = pack_bf16(__uint_as_float(ov[k * 8 + 6]) * inv, __uint_as_float(ov[k * 8 + 7]) * inv);
+                const int q = c * 4 + k;                       // 16-byte chunk of the row
+                sts128_(sbase + (uint32_t)((q >> 3) * HALF_TILE + r * 128 + (((q & 7) ^ (r & 7)) << 4)), w);
+            }
+        }
+        if (P.lse != nullptr && t < P.sq)
+            P.lse[lse_id] = (m_run + log2f(l_run)) * 0.69314718055994531f;
+        if (arrive_oe) {
+            tc_fence_before();
+            mbar_arrive(bar(B_OE));
+        }
+        // the rows visible to the TMA engine, every row of the tile written, then one store of
+        // both 64-column halves (tokens past the suffix fall outside the map and are dropped)
+        asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+        asm volatile("bar.sync %0, 128;" ::"r"(2 + x) : "memory");
+        if (r == 0) {
+            const int qz = l * P.batch_total + b;
+            tma_store_4d(&P.tm_o, sbase, 0, hk * G, t0, qz);
+            tma_store_4d(&P.tm_o, sbase + HALF_TILE, 64, hk * G, t0, qz);
+            asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+            asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+        }
+        return;
+    }
     if (P.n_split == 1) {
         __nv_bfloat16* orow = static_cast<__nv_bfloat16*>(P.out) + row_id * HD;
 #pragma unroll
@@ -1362,14 +1415,11 @@ __device__ __forceinline__ void fused_suffix_prep(const FusedTcParams& F, int ts
     // the table's grid has finished and its writes are visible (returns at once when this
     // grid was launched after it completed)
     if (n_items > 0) asm volatile("griddepcontrol.wait;" ::: "memory");
-    if (v0) {
-        angles(t_0, c0, s0);
-        if (is_q(t_0)) q_item(t_0, c0, s0);
-    }
-    if (v1) {
-        angles(t_1, c1, s1);
-        if (is_q(t_1)) q_item(t_1, c1, s1);
-    }
+    // both items' angles in flight before either is used
+    if (v0) angles(t_0, c0, s0);
+    if (v1) angles(t_1, c1, s1);
+    if (v0 && is_q(t_0)) q_item(t_0, c0, s0);
+    if (v1 && is_q(t_1)) q_item(t_1, c1, s1);
 #pragma unroll 1
     for (int i = ts + 512; i < n_items; i += 256) {
         const int tt = lo + (i >> 3);
@@ -1656,7 +1706,7 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
                               writer && P.layer0 + l == 0 && hk == 0, 0u, true, sQ, sBar, abort);
             if (x == 0 || has_b)
                 softmax_tile(P, tmem, sBar, x, warp & 3, lane, x ? t0b : t0a, l, bl, b, hk, sp, j_base,
-                             n_kv, 0u, 0u, false, abort);
+                             n_kv, 0u, 0u, false, abort, sQ);
         } else if constexpr (kFused) {
             // per pair: the suffix preparation (the lead pair's also turns the suffix rows
             // among its key tiles into the cache), then the softmax over its key tiles
@@ -1671,7 +1721,8 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
                                   pi == 0, sQ, sBar, abort);
                 if (x == 0 || ps.has_b) {
                     softmax_tile(P, tmem, sBar, x, warp & 3, lane, x ? ps.t0b : ps.t0a, l, bl, b, hk, sp,
-                                 ps.j_base, ps.n_kv, done, (uint32_t)pi & 1u, p_count > 1, abort);
+                                 ps.j_base, ps.n_kv, done, (uint32_t)pi & 1u, p_count > 1, abort,
+                                 pi == p_count - 1 ? sQ : 0u);
                     done += (uint32_t)ps.n_kv;
                 } else if (p_count > 1) {
                     mbar_arrive(bar(B_OE));
@@ -1683,7 +1734,8 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
                 const PairSpan ps = pi == 0 ? ps0 : pair_span(P, p_first + pi, sp, s_r);
                 if (x == 0 || ps.has_b) {
                     softmax_tile(P, tmem, sBar, x, warp & 3, lane, x ? ps.t0b : ps.t0a, l, bl, b, hk, sp,
-                                 ps.j_base, ps.n_kv, done, (uint32_t)pi & 1u, p_count > 1, abort);
+                                 ps.j_base, ps.n_kv, done, (uint32_t)pi & 1u, p_count > 1, abort,
+                                 pi == p_count - 1 ? sQ : 0u);
                     done += (uint32_t)ps.n_kv;
                 } else if (p_count > 1) {    // no tile B in this pair: nothing of O to read
                     mbar_arrive(bar(B_OE));
@@ -1846,6 +1898,8 @@ cudaError_t prepare_tc(const AttnParams& a, TcParams& p, dim3& grid) {
                                    (cuuint64_t)pitch * a.hq * HD * 2};
         const cuuint32_t box[4] = {64, (cuuint32_t)G, (cuuint32_t)tq, 1};
         if (!encode(&p.tm_q, a.q_rot, 4, dims, str, box)) return cudaErrorInvalidValue;
+        // out has q's layout: its 128-row tiles leave through the same boxes
+        if (!encode(&p.tm_o, a.out, 4, dims, str, box)) return cudaErrorInvalidValue;
     }
     {   // K, V: cache [L*rows][Hkv][128] -> dims (d, Hkv, L*rows); layer0 + lq <= L
         const int64_t lrows = (int64_t)(a.layer0 + a.lq) * a.rows;
