@@ -345,7 +345,13 @@ c2kv_status c2kv_attend_noalloc(c2kv_ctx* ctx, c2kv_cache* cache, int32_t layer,
  * q, k_new, v_new, out and lse must be device (or managed) memory: anything else is
  * refused with ERR_ARG before anything is enqueued.
  * The key range of each (layer, request, KV head) is split over several CTAs and merged
- * exactly (log-sum-exp); the split buffer comes from the context's memory pool.
+ * exactly (log-sum-exp); the split buffer comes from the context's memory pool.  With bf16
+ * and d = 128 the step runs on the tensor-core attention kernel (the new token as a one-row
+ * query tile) when (layers x requests x KV heads) fits one CTA per SM or a request holds
+ * 4096 keys or more, else on a CUDA-core decode kernel (C2KV_ATTN_SIMT forces the latter).
+ * The tensor-core route reads whole 128-row key tiles, so it zeroes the rows after the new
+ * one up to the next 128-row boundary that no earlier call on this cache has written or
+ * zeroed (never rows an earlier c2kv_attend or c2kv_decode wrote).
  * Errors: ERR_ARG, ERR_STATE (cache from another context), ERR_UNSUPPORTED (head layout the
  * decode kernel does not take: G = Hq/Hkv in {1,2,4,8,16}, d in {64,128}, G*d <= 1024, and
  * G <= 8 for bf16), ERR_NOMEM, ERR_CUDA.

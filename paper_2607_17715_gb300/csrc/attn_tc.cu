@@ -366,7 +366,9 @@ __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, u
                                             volatile uint32_t* abort, uint32_t stage = 0u) {
     auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
     const int G = P.group;
-    const int s_r = P.req[bl].n_slots;
+    // keys before the launch's first query token: the composed slots and, for a decode step
+    // (t0 > 0), the suffix rows written before it
+    const int s_r = P.req[bl].n_slots + P.req[bl].t0;
     const int r = quad * 32 + lane;                 // row = TMEM lane
     const uint32_t lane_addr = (uint32_t)(quad * 32) << 16;
     const uint32_t colS = kColS + (uint32_t)x * BN;  // S_x, and P_x over its first 64 columns
@@ -1566,7 +1568,7 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
     const int l = blockIdx.z / P.batch;
     const int bl = blockIdx.z - l * P.batch;
     const int b = P.b0 + bl;
-    const int s_r = P.req[bl].n_slots;
+    const int s_r = P.req[bl].n_slots + P.req[bl].t0;   // keys before the first query token
     // pairs of Q tiles: the CTA runs pairs [p_first, p_first + p_count) in turn (one pair
     // unless the plain kernel groups short pairs); the groups go last first: under a causal
     // mask the later pairs see more keys, so the longest CTAs start in the first wave

@@ -46,6 +46,10 @@ struct c2kv_cache {
     void* v = nullptr;
     int32_t* pos = nullptr;        // device [rows]
     std::vector<int32_t> row_base, n_slots, l_req, capacity;
+    // [layer][request]: rows of the request's region known to hold finite values (written or
+    // zeroed) from its first row on; the tensor-core decode zeroes the rest of the key tile
+    // that holds its new row before it reads it
+    std::vector<int32_t> clean_to;
     int32_t suffix_capacity = 0;
 };
 
@@ -567,6 +571,9 @@ c2kv_status compose_plan(c2kv_ctx* c, int32_t batch, const int32_t* req_ptr, con
         row += cap;
     }
     cache->rows = row;
+    cache->clean_to.assign((size_t)cache->layers * batch, 0);
+    for (int32_t l = 0; l < cache->layers; ++l)
+        for (int32_t r = 0; r < batch; ++r) cache->clean_to[(size_t)l * batch + r] = cache->n_slots[r];
     if (c->inject == 1 && n_occ > 0) {
         occ[0].src_base = c->cfg.pool_slots + 7;   // refused by the kernels' bounds checks
         c->inject = 0;
@@ -639,6 +646,17 @@ cudaError_t compose_launch(c2kv_ctx* c, const c2kv_cache* cache, const std::vect
     return e;
 }
 
+// After a suffix of n_suffix tokens over layers [l0, l0 + n): every request's rows up to the
+// 128-row edge after its suffix hold finite values (the suffix rows, then zeros).
+void mark_suffix_clean(c2kv_cache* cache, int32_t l0, int32_t n, int32_t n_suffix) {
+    for (int32_t l = l0; l < l0 + n; ++l)
+        for (int32_t r = 0; r < cache->batch; ++r) {
+            int32_t& ct = cache->clean_to[(size_t)l * cache->batch + r];
+            const int64_t edge = ((int64_t)cache->n_slots[r] + n_suffix + kTileRows - 1) / kTileRows * kTileRows;
+            ct = std::max<int32_t>(ct, (int32_t)std::min<int64_t>(edge, cache->capacity[r]));
+        }
+}
+
 // Checks of an attend call's arguments that do not depend on the cache's contents.
 c2kv_status attend_check(c2kv_ctx* c, const char* what, int32_t layer, const void* q, const void* k_suf,
                          const void* v_suf, int32_t n_suffix, int32_t suffix_capacity, void* out,
@@ -679,8 +697,10 @@ c2kv::SuffixParams suffix_params(const c2kv_ctx* c, const c2kv_cache* cache, int
     s.hkv = c->cfg.n_kv_heads;
     s.pad_rows = 1;
     s.rope = c->turns;
-    for (int32_t i = 0; i < nb; ++i)
+    for (int32_t i = 0; i < nb; ++i) {
         s.req[i] = c2kv::ReqParam{cache->row_base[b0 + i], cache->n_slots[b0 + i], cache->l_req[b0 + i], 0};
+        s.pad_from[i] = cache->n_slots[b0 + i] + n_suffix;
+    }
     return s;
 }
 
@@ -1119,6 +1139,7 @@ c2kv_status c2kv_compose_attend(c2kv_ctx* c, int32_t batch, const int32_t* req_p
             destroy_cache(c, cache);
             return cuda_fail(c, e, "compose_attend");
         }
+        mark_suffix_clean(cache, 0, c->cfg.layers, n_suffix);
         c->caches.push_back(cache);
         *cache_out = cache;
         return C2KV_OK;
@@ -1163,6 +1184,7 @@ c2kv_status c2kv_attend(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
         if (e == cudaSuccess) e = suffix_io_out(c, io, out, lse, 0, lq);
         pool_free(c, io.scratch);
         if (e != cudaSuccess) return cuda_fail(c, e, "attend");
+        mark_suffix_clean(cache, layer < 0 ? 0 : layer, lq, n_suffix);
         return C2KV_OK;
     } catch (const std::bad_alloc&) {
         return fail(c, C2KV_ERR_NOMEM, "attend: host allocation failed");
@@ -1195,27 +1217,60 @@ c2kv_status c2kv_decode(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
         const int32_t lq = layer < 0 ? c->cfg.layers : 1;
         const int32_t layer0 = layer < 0 ? 0 : layer;
         const int32_t hq = c->cfg.n_q_heads, hkv = c->cfg.n_kv_heads, d = c->cfg.head_dim;
-        // Key-range splits per (layer, request, KV head), from a model of the schedule: the
-        // CTAs run in waves of (resident CTAs per SM) x SMs; a CTA spends a start latency
-        // (about 2 us: its first tiles in flight) plus its keys' K/V bytes at its share of
-        // HBM, at most what one CTA's four consumer warps keep up with (about 25 GB/s,
-        // measured); a split adds the merge (about 3 us).  Splits keep at least 128 keys.
         const int64_t units = (int64_t)hkv * lq * std::min<int32_t>(B, c2kv::kMaxReq);
-        const int32_t grp = hq / hkv;
-        const int64_t slots = (int64_t)(grp >= 8 ? 1 : 2) * c->sms;
-        const double bytes_per_key = 2.0 * d * (double)c->eb;
+        // bf16, d 128: the tensor-core attention kernel with the new token as a one-row
+        // suffix at suffix index steps[r] (its 128-row query tile holds G live rows: the MMA
+        // has time to spare, and its pipeline streams K and V at the rate of HBM) when its
+        // one CTA per SM covers the units in one wave or their key ranges are long; otherwise
+        // (short contexts over more units than SMs: its per-CTA start would be paid twice)
+        // the CUDA-core decode kernel, two CTAs per SM.  Measured on a GB300: Llama-3-8B
+        // layer, 32 layers x 1 request, 1360 keys: 45 us CUDA cores, 52 us tensor cores;
+        // 16 requests x 1160 keys: 31 / 28 us; 2 x 2300 keys, G = 8: 26 / 19 us; 8 x 32900
+        // keys: 212 / 192 us.
+        const int64_t tiles_max = (n_keys_max + 127) / 128;
+        const bool use_tc = c->cfg.attn_impl != C2KV_ATTN_SIMT &&
+                            c2kv::attn_tc_supported(c->cfg.dtype, d, hq, hkv) &&
+                            (units <= c->sms || tiles_max >= 32);
         int32_t n_split = 1;
-        double best = 0.0;
-        for (int32_t n = 1; n <= 64; ++n) {
-            const int32_t kps = (n_keys_max + n - 1) / n;
-            if (n > 1 && kps < 128) break;
-            const int64_t ctas = units * n;
-            const int64_t waves = (ctas + slots - 1) / slots;
-            const double bw = std::min(6.0e12 / (double)std::min(ctas, slots), 25.0e9);
-            const double t = (double)waves * (2e-6 + kps * bytes_per_key / bw) + (n > 1 ? 3e-6 : 0.0);
-            if (n == 1 || t < best) {
-                best = t;
-                n_split = n;
+        if (use_tc) {
+            // splits per (layer, request, KV head): the fewest waves of one-CTA-per-SM work,
+            // each CTA paying about four key tiles' time to start and finish, a split another
+            // two for the merge
+            const int64_t tiles = tiles_max;
+            if (c->cfg.attn_split >= 1) {
+                n_split = (int32_t)std::min<int64_t>(c->cfg.attn_split, tiles);
+            } else {
+                double best = 0.0;
+                for (int32_t n = 1; n <= 16 && n <= tiles; ++n) {
+                    const int64_t waves = (units * n + c->sms - 1) / c->sms;
+                    const double t = (double)waves * ((double)((tiles + n - 1) / n) + 4.0) + (n > 1 ? 2.0 : 0.0);
+                    if (n == 1 || t < best) {
+                        best = t;
+                        n_split = n;
+                    }
+                }
+            }
+        } else {
+            // Key-range splits per (layer, request, KV head), from a model of the schedule: the
+            // CTAs run in waves of (resident CTAs per SM) x SMs; a CTA spends a start latency
+            // (about 2 us: its first tiles in flight) plus its keys' K/V bytes at its share of
+            // HBM, at most what one CTA's consumer warps keep up with (about 25 GB/s,
+            // measured); a split adds the merge (about 3 us).  Splits keep at least 128 keys.
+            const int32_t grp = hq / hkv;
+            const int64_t slots = (int64_t)(grp >= 8 ? 1 : 2) * c->sms;
+            const double bytes_per_key = 2.0 * d * (double)c->eb;
+            double best = 0.0;
+            for (int32_t n = 1; n <= 64; ++n) {
+                const int32_t kps = (n_keys_max + n - 1) / n;
+                if (n > 1 && kps < 128) break;
+                const int64_t ctas = units * n;
+                const int64_t waves = (ctas + slots - 1) / slots;
+                const double bw = std::min(6.0e12 / (double)std::min(ctas, slots), 25.0e9);
+                const double t = (double)waves * (2e-6 + kps * bytes_per_key / bw) + (n > 1 ? 3e-6 : 0.0);
+                if (n == 1 || t < best) {
+                    best = t;
+                    n_split = n;
+                }
             }
         }
         const int32_t keys_per_split = (n_keys_max + n_split - 1) / n_split;
@@ -1233,6 +1288,23 @@ c2kv_status c2kv_decode(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
                 return cuda_fail(c, e, "decode: split scratch allocation");
             }
         }
+        // the tensor-core route reads whole 128-row key tiles: the rows after the new one up to
+        // the next 128-row edge must hold finite values (masked keys weigh zero, but 0 * NaN is
+        // not zero), so each request's are zeroed once, when not written or zeroed before
+        std::vector<int32_t> edge(B), pad_from(B);
+        bool any_pad = false;
+        for (int32_t b = 0; b < B; ++b) {
+            const int64_t next = (int64_t)cache->n_slots[b] + steps[b] + 1;
+            edge[b] = (int32_t)std::min<int64_t>((next + kTileRows - 1) / kTileRows * kTileRows, cache->capacity[b]);
+            bool need = false;
+            for (int32_t l = layer0; use_tc && l < layer0 + lq; ++l)
+                need = need || cache->clean_to[(size_t)l * B + b] < edge[b];
+            pad_from[b] = need ? (int32_t)next : (int32_t)((next + kTileRows - 1) / kTileRows * kTileRows);
+            any_pad = any_pad || need;
+        }
+        std::vector<c2kv::ReqParam> reqs(B);
+        for (int32_t b = 0; b < B; ++b)
+            reqs[b] = c2kv::ReqParam{cache->row_base[b], cache->n_slots[b], cache->l_req[b], steps[b]};
         for (int32_t b0 = 0; e == cudaSuccess && b0 < B; b0 += c2kv::kMaxReq) {
             const int32_t nb = std::min<int32_t>(c2kv::kMaxReq, B - b0);
             c2kv::SuffixParams s{};
@@ -1252,16 +1324,46 @@ c2kv_status c2kv_decode(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
             s.sq = 1;
             s.hq = hq;
             s.hkv = hkv;
-            s.pad_rows = 0;
+            s.pad_rows = any_pad ? 1 : 0;
             s.rope = c->turns;
-            for (int32_t i = 0; i < nb; ++i)
-                s.req[i] = c2kv::ReqParam{cache->row_base[b0 + i], cache->n_slots[b0 + i],
-                                          cache->l_req[b0 + i], steps[b0 + i]};
+            for (int32_t i = 0; i < nb; ++i) {
+                s.req[i] = reqs[b0 + i];
+                s.pad_from[i] = pad_from[b0 + i];
+            }
             {
                 ProfScope prof_suffix(c, C2KV_PROF_SUFFIX);
                 e = c2kv::launch_suffix_prep(s, c->cfg.dtype, d, c->stream);
             }
             if (e != cudaSuccess) break;
+            if (use_tc) {
+                c2kv::AttnParams a{};
+                a.q_rot = q_rot;
+                a.cache_k = cache->k;
+                a.cache_v = cache->v;
+                a.out = out;
+                a.lse = lse;
+                a.err = c->d_err;
+                a.rows = cache->rows;
+                a.layer0 = layer0;
+                a.lq = lq;
+                a.batch = nb;
+                a.batch_total = B;
+                a.b0 = b0;
+                a.sq = 1;
+                a.hq = hq;
+                a.hkv = hkv;
+                a.scale_log2 = (float)(1.4426950408889634 / std::sqrt((double)d));
+                a.n_split = n_split;
+                a.pairs_per_cta = c->cfg.attn_pairs;
+                a.part_o = part;
+                a.part_lse = part ? part + (size_t)n_split * rows_all * d : nullptr;
+                for (int32_t i = 0; i < nb; ++i) a.req[i] = reqs[b0 + i];
+                ProfScope prof_decode(c, C2KV_PROF_DECODE, true);
+                e = c2kv::launch_attn_tc(a, c->stream, prof_decode.hook());
+                // the merge of the splits over every request's rows, after the last group
+                if (e == cudaSuccess && n_split > 1 && b0 + nb >= B) e = c2kv::launch_attn_combine(a, c->stream);
+                continue;
+            }
             c2kv::DecodeParams p{};
             p.q_rot = q_rot;
             p.cache_k = cache->k;
@@ -1291,6 +1393,11 @@ c2kv_status c2kv_decode(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
         pool_free(c, part);
         pool_free(c, q_rot);
         if (e != cudaSuccess) return cuda_fail(c, e, "decode");
+        for (int32_t l = layer0; l < layer0 + lq; ++l)
+            for (int32_t b = 0; b < B; ++b) {
+                int32_t& ct = cache->clean_to[(size_t)l * B + b];
+                ct = std::max(ct, pad_from[b] < edge[b] ? edge[b] : cache->n_slots[b] + steps[b] + 1);
+            }
         return C2KV_OK;
     } catch (const std::bad_alloc&) {
         return fail(c, C2KV_ERR_NOMEM, "decode: host allocation failed");
@@ -1478,6 +1585,10 @@ bool attend_view(const c2kv_ctx* c, const c2kv_cache* cache, AttendView* v) {
     v->n_slots = cache->n_slots.data();
     v->l_req = cache->l_req.data();
     return true;
+}
+
+void note_suffix_written(c2kv_cache* cache, int32_t l0, int32_t n, int32_t n_suffix) {
+    mark_suffix_clean(cache, l0, n, n_suffix);
 }
 
 MemKind mem_kind(const void* p) {

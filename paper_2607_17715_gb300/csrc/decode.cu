@@ -56,16 +56,21 @@ struct DecodeTma {
 
 constexpr size_t kDecSmem = 1024 + (size_t)kDecStages * 2 * kDecTileBytes + 16 * kDecStages + 16;
 
-// Four consumer warps and the producer warp per CTA, two CTAs per SM (one for G >= 8, whose
-// query and output slices need more registers): one CTA's start (the latency of its first
-// tiles) overlaps the other's streaming.
-constexpr int kDecConsumers = 4;
-constexpr int kDecThreadsAll = (kDecConsumers + 1) * 32;
+// Four consumer warps and the producer warp per CTA, two CTAs per SM: one CTA's start (the
+// latency of its first tiles) overlaps the other's streaming.  For G >= 8 the query and
+// output slices of a lane take too many registers for two CTAs, so one CTA runs eight
+// consumer warps instead: two warps per SM sub-partition either way, so that one warp's
+// chain of shuffles and dependent FMAs hides behind the other's.
+template <int G>
+__host__ __device__ constexpr int dec_consumers() { return G >= 8 ? 8 : 4; }
+template <int G>
+__host__ __device__ constexpr int dec_threads() { return (dec_consumers<G>() + 1) * 32; }
 
 // T element type, D head dim, G query heads per KV head.
 template <typename T, int D, int G>
-__global__ void __launch_bounds__(kDecThreadsAll, G >= 8 ? 1 : 2) decode_kernel(const __grid_constant__ DecodeTma X) {
+__global__ void __launch_bounds__(dec_threads<G>(), G >= 8 ? 1 : 2) decode_kernel(const __grid_constant__ DecodeTma X) {
     const DecodeParams& P = X.p;
+    constexpr int kDecConsumers = dec_consumers<G>();
     using V = Vec16<T>;
     constexpr int E = V::N;                            // elements per 16-byte vector
     constexpr int LPK = D / E;                         // lanes per key row
@@ -412,7 +417,7 @@ cudaError_t launch_g(const DecodeParams& p, cudaStream_t s, Hook before) {
     if (p.dependent) {    // starts while the suffix kernel before it runs (see the waits above)
         cudaLaunchConfig_t cfg{};
         cfg.gridDim = grid;
-        cfg.blockDim = dim3(kDecThreadsAll);
+        cfg.blockDim = dim3(dec_threads<G>());
         cfg.dynamicSmemBytes = kDecSmem;
         cfg.stream = s;
         cudaLaunchAttribute attr[1];
@@ -423,7 +428,7 @@ cudaError_t launch_g(const DecodeParams& p, cudaStream_t s, Hook before) {
         e = cudaLaunchKernelEx(&cfg, decode_kernel<T, D, G>, x);
         if (e != cudaSuccess) return e;
     } else {
-        decode_kernel<T, D, G><<<grid, kDecThreadsAll, kDecSmem, s>>>(x);
+        decode_kernel<T, D, G><<<grid, dec_threads<G>(), kDecSmem, s>>>(x);
     }
     e = cudaGetLastError();
     if (e != cudaSuccess || p.n_split == 1) return e;

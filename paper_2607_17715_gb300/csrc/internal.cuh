@@ -106,9 +106,12 @@ struct SuffixParams {
     int32_t sq;
     int32_t hq;
     int32_t hkv;
-    int32_t pad_rows;        // 1: zero the rows after the suffix up to the next 128-row boundary
+    int32_t pad_rows;        // 1: zero each request's rows from pad_from up to the next 128-row
+                             // boundary
     RopeTurns rope;
     ReqParam req[kMaxReq];
+    int32_t pad_from[kMaxReq];   // request-relative row where the zeroing starts (the row after
+                                 // the suffix; at a 128-row boundary for none)
 };
 
 struct AttnParams {
@@ -313,6 +316,9 @@ struct c2kv_cache;
 namespace c2kv {
 // Fills `v` if `cache` belongs to `ctx` (returns false otherwise).
 bool attend_view(const c2kv_ctx* ctx, const c2kv_cache* cache, AttendView* v);
+// Records that a suffix of n_suffix tokens over layers [l0, l0 + n) was written, with the
+// rows after it zeroed up to the 128-row edge (what a later decode step reads as finite).
+void note_suffix_written(c2kv_cache* cache, int32_t l0, int32_t n, int32_t n_suffix);
 // Records `msg` as the context's last error and returns `code`.
 int32_t set_last_error(c2kv_ctx* ctx, int32_t code, const char* msg);
 }  // namespace c2kv

@@ -249,7 +249,7 @@ __global__ void __launch_bounds__(256) suffix_kernel(const __grid_constant__ Suf
     if ((int)blockIdx.x < n_pad) {
         const int bl = (int)blockIdx.x / kPadParts;
         const int part = (int)blockIdx.x - bl * kPadParts;
-        const int used = P.req[bl].n_slots + P.sq;
+        const int used = P.pad_from[bl];
         const int end = (used + 127) / 128 * 128;
         constexpr int VPR_ELEMS = 16 / (int)sizeof(T);
         const int vec_per_row = (int)(row_elems / VPR_ELEMS);

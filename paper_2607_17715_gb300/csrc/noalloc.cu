@@ -125,8 +125,10 @@ extern "C" c2kv_status c2kv_attend_noalloc(c2kv_ctx* ctx, c2kv_cache* cache, int
         s.hkv = v.n_kv_heads;
         s.pad_rows = 1;
         s.rope = v.turns;
-        for (int32_t i = 0; i < nb; ++i)
+        for (int32_t i = 0; i < nb; ++i) {
             s.req[i] = c2kv::ReqParam{v.row_base[b0 + i], v.n_slots[b0 + i], v.l_req[b0 + i], 0};
+            s.pad_from[i] = v.n_slots[b0 + i] + n_suffix;
+        }
         e = c2kv::launch_suffix_prep(s, v.dtype, v.head_dim, v.stream);
         if (e != cudaSuccess) break;
         c2kv::AttnParams a{};
@@ -155,6 +157,7 @@ extern "C" c2kv_status c2kv_attend_noalloc(c2kv_ctx* ctx, c2kv_cache* cache, int
         (void)cudaGetLastError();
         return refuse(ctx, C2KV_ERR_CUDA, "attend_noalloc: kernel launch failed");
     }
+    c2kv::note_suffix_written(cache, layer0, lq, n_suffix);
     c2kv::set_last_error(ctx, C2KV_OK, "");
     return C2KV_OK;
 }

@@ -20,11 +20,13 @@ def _small(wl, **kw):
     return synth.scaled(wl, **base)
 
 
-def _decode_case(wl, steps, prefill=None, layer=-1, extra_steps=0, attn_first=True):
+def _decode_case(wl, steps, prefill=None, layer=-1, extra_steps=0, attn_impl=0):
     """Compose the workload's requests, optionally run c2kv_attend over `prefill` suffix
     tokens, then decode: request r's new token at suffix index steps[r] (and, with
     extra_steps, the following steps one call at a time).  Every decode output and lse is
-    compared with the oracle's decode step for that request."""
+    compared with the oracle's decode step for that request.  attn_impl 0 lets the library
+    pick the route (the tensor-core kernel for these sizes with bf16), C2KV_ATTN_SIMT forces
+    the CUDA-core decode kernel."""
     c2kv = H.lib()
     reqs = synth.requests(wl)
     B = len(reqs)
@@ -33,7 +35,7 @@ def _decode_case(wl, steps, prefill=None, layer=-1, extra_steps=0, attn_first=Tr
     all_ids = sorted({c for ids, _ in reqs for c in ids})
     chunks = H.oracle_chunks_meanpool(wl, all_ids)
     pool = sum(orc.n_slots(wl.chunk_tokens, wl.ratio_k) for _ in all_ids) + 16
-    ctx = H.make_ctx(wl, pool_slots=pool)
+    ctx = H.make_ctx(wl, pool_slots=pool, attn_impl=attn_impl)
     try:
         dev = H.load_stored(ctx, wl, chunks)
         req_ptr = np.cumsum([0] + [len(ids) for ids, _ in reqs])
@@ -78,19 +80,34 @@ def _decode_case(wl, steps, prefill=None, layer=-1, extra_steps=0, attn_first=Tr
         c2kv.c2kv_destroy(ctx)
 
 
-def test_decode_after_suffix_attention():
+IMPLS = pytest.mark.parametrize("impl", [0, 1], ids=["auto", "cuda_core"])   # 1: C2KV_ATTN_SIMT
+
+
+@IMPLS
+def test_decode_after_suffix_attention(impl):
     # the suffix of 16 tokens written by attend, then the 17th token decoded
-    _decode_case(_small(L8B_1, layers=2), steps=[16], prefill=16)
+    _decode_case(_small(L8B_1, layers=2), steps=[16], prefill=16, attn_impl=impl)
 
 
-def test_decode_sequence_from_step0():
+@IMPLS
+def test_decode_sequence_from_step0(impl):
     # straight after compose: steps 0, 1, 2, 3 one call at a time
-    _decode_case(_small(L8B_1, layers=2), steps=[0], extra_steps=3)
+    _decode_case(_small(L8B_1, layers=2), steps=[0], extra_steps=3, attn_impl=impl)
 
 
-def test_decode_batched_ragged_steps():
+@IMPLS
+def test_decode_batched_ragged_steps(impl):
     wl = _small(synth.workload("batched"), batch=3, chunks_per_request=4, pool_chunks=32)
-    _decode_case(wl, steps=[5, 0, 11], prefill=12)
+    _decode_case(wl, steps=[5, 0, 11], prefill=12, attn_impl=impl)
+
+
+def test_decode_at_tile_edges():
+    # new tokens at the last row of a 128-row key tile and at the first two of the next
+    # (slots + step + 1 = 256, 257, 258): the rows after the new token up to the next tile's
+    # edge hold no data until the step zeroes them
+    wl = _small(L8B_1, layers=2, chunk_tokens=256, ratio_k=4, chunks_per_request=3)
+    s = 3 * 64
+    _decode_case(wl, steps=[256 - s - 1], prefill=256 - s - 1, extra_steps=2)
 
 
 def test_decode_single_layer_of_many():
@@ -101,11 +118,49 @@ def test_decode_f32_tiny():
     _decode_case(TINY, steps=[4], prefill=5)
 
 
-def test_decode_long_context_splits():
+@IMPLS
+def test_decode_long_context_splits(impl):
     # 32 chunks x 1024 tokens at k=4: 8192 slots, so the key range is split over many CTAs
     # and merged
     wl = _small(L8B_1, chunk_tokens=1024, ratio_k=4, chunks_per_request=32, pool_chunks=32)
-    _decode_case(wl, steps=[3], prefill=3)
+    _decode_case(wl, steps=[3], prefill=3, attn_impl=impl)
+
+
+@pytest.mark.parametrize("noalloc", [False, True], ids=["attend", "attend_noalloc"])
+def test_decode_keeps_rows_written_by_attend(noalloc):
+    # a suffix of 40 tokens written by attention, then a decode step at suffix index 5 (the
+    # sequence taken back to that point): rows 6 .. 39 keep what the attention wrote, the
+    # zeroing for whole key tiles never reaching rows a call wrote
+    c2kv = H.lib()
+    wl = _small(L8B_1, layers=2)
+    reqs = synth.requests(wl)
+    all_ids = sorted({c for ids, _ in reqs for c in ids})
+    chunks = H.oracle_chunks_meanpool(wl, all_ids)
+    pool = sum(orc.n_slots(wl.chunk_tokens, wl.ratio_k) for _ in all_ids) + 16
+    ctx = H.make_ctx(wl, pool_slots=pool)
+    try:
+        dev = H.load_stored(ctx, wl, chunks)
+        req_ptr = np.cumsum([0] + [len(ids) for ids, _ in reqs])
+        cache = c2kv.c2kv_compose(ctx, req_ptr, [dev[c] for ids, _ in reqs for c in ids],
+                                  [o for _, offs in reqs for o in offs], suffix_capacity=64)
+        q, ks, vs = synth.suffix(synth.scaled(wl, n_suffix=40), layers=wl.layers)
+        qd, kd, vd = (H.to_dev(x, wl) for x in (q, ks, vs))
+        attend = c2kv.c2kv_attend_noalloc if noalloc else c2kv.c2kv_attend
+        attend(ctx, cache, -1, qd, kd, vd, 40, torch.empty_like(qd))
+        c2kv.c2kv_sync(ctx)
+        info, k0, v0, _ = H.cache_arrays(cache, wl)
+        base, s = info["row_base"][0], info["n_slots"][0]
+        pick = [H.to_dev(x[:, :, 5], wl) for x in (q, ks, vs)]
+        out = torch.empty_like(pick[0])
+        c2kv.c2kv_decode(ctx, cache, -1, pick[0], pick[1], pick[2], [5], out)
+        c2kv.c2kv_sync(ctx)
+        _, k1, v1, _ = H.cache_arrays(cache, wl)
+        rows = slice(base + s + 6, base + s + 40)
+        assert np.array_equal(k1[:, rows], k0[:, rows]) and np.array_equal(v1[:, rows], v0[:, rows])
+        assert np.isfinite(out.float().cpu().numpy()).all()
+        c2kv.c2kv_cache_release(ctx, cache)
+    finally:
+        c2kv.c2kv_destroy(ctx)
 
 
 @pytest.mark.parametrize("long", [False, True])
