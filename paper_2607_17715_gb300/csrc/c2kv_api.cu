@@ -605,19 +605,44 @@ int32_t compose_tile_slots(const c2kv_ctx* c, int64_t slots, int32_t n_layers, i
     return t;
 }
 
+// Slots per tile of the bulk-copy compose kernel: at most 16 KB of K rows (the stage then
+// holds 32 KB of K and V, six of them in flight per SM), halved while the launch would give
+// fewer than four tiles per SM, so that a small launch still spreads evenly over the SMs
+// (each tile costs its CTA about a microsecond of fixed work, so smaller tiles than that
+// lose more than they balance).
+int32_t compose_bulk_tile_slots(const c2kv_ctx* c, const std::vector<c2kv::OccParam>& occ, int32_t g0,
+                                int32_t g1, int32_t n_layers) {
+    const int64_t row_bytes = (int64_t)c->cfg.n_kv_heads * c->cfg.head_dim * c->eb;
+    int32_t t = 1;
+    while (t * 2 <= c2kv::kComposeBulkTile && (int64_t)t * 2 * row_bytes <= 16384) t *= 2;
+    auto tiles = [&](int32_t ts) {
+        int64_t n = 0;
+        for (int32_t i = g0; i < g1; ++i) n += (occ[i].m + ts - 1) / ts;
+        return n * n_layers;
+    };
+    while (t > 1 && tiles(t) < 4LL * c->sms) t /= 2;
+    return t;
+}
+
 // The compose kernel over every occurrence: one launch per group of at most kMaxOcc
-// occurrences, all layers at once.
+// occurrences, all layers at once; the bulk-copy kernel when every chunk of the group is in
+// the device pool and the grid is not capped.
 cudaError_t compose_launch(c2kv_ctx* c, const c2kv_cache* cache, const std::vector<c2kv::OccParam>& occ,
                            int32_t layer0 = 0, int32_t n_layers = -1, int max_ctas = 0) {
     const int32_t n_occ = (int32_t)occ.size();
     if (n_layers < 0) n_layers = c->cfg.layers;
     cudaError_t e = cudaSuccess;
-    ProfScope prof_compose(c, C2KV_PROF_COMPOSE);
+    ProfScope prof_compose(c, C2KV_PROF_COMPOSE, true);
     for (int32_t g0 = 0; e == cudaSuccess && g0 < n_occ; g0 += c2kv::kMaxOcc) {
         const int32_t g1 = std::min(n_occ, g0 + c2kv::kMaxOcc);
         int64_t slots = 0;
-        for (int32_t i = g0; i < g1; ++i) slots += occ[i].m;
-        const int32_t ts = compose_tile_slots(c, slots, n_layers, max_ctas);
+        bool bulk = max_ctas == 0;
+        for (int32_t i = g0; i < g1; ++i) {
+            slots += occ[i].m;
+            bulk = bulk && !occ[i].host;
+        }
+        const int32_t ts = bulk ? compose_bulk_tile_slots(c, occ, g0, g1, n_layers)
+                                : compose_tile_slots(c, slots, n_layers, max_ctas);
         c2kv::ComposeParams pr{};
         pr.pool_k = c->pool_k;
         pr.pool_v = c->pool_v;
@@ -630,6 +655,7 @@ cudaError_t compose_launch(c2kv_ctx* c, const c2kv_cache* cache, const std::vect
         pr.hkv = c->cfg.n_kv_heads;
         pr.layer0 = layer0;
         pr.tile_slots = ts;
+        pr.bulk = bulk ? 1 : 0;
         pr.pre_rope = c->cfg.storage == C2KV_STORAGE_PRE_ROPE ? 1 : 0;
         pr.rope = c->turns;
         int32_t tiles = 0;
@@ -641,7 +667,8 @@ cudaError_t compose_launch(c2kv_ctx* c, const c2kv_cache* cache, const std::vect
             tiles += (rec.m + ts - 1) / ts;
         }
         pr.n_tiles = tiles;
-        e = c2kv::launch_compose(pr, c->cfg.dtype, c->cfg.head_dim, n_layers, c->stream, max_ctas);
+        e = c2kv::launch_compose(pr, c->cfg.dtype, c->cfg.head_dim, n_layers, c->stream, max_ctas,
+                                 prof_compose.hook());
     }
     return e;
 }

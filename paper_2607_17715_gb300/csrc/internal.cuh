@@ -19,6 +19,7 @@ constexpr int kMaxHalf = 64;        // head_dim / 2 for head_dim <= 128
 constexpr int kMaxOcc = 512;        // chunk occurrences per compose launch (24 KB of parameters)
 constexpr int kMaxReq = 256;        // requests per suffix / attention launch
 constexpr int kComposeTile = 16;    // most composed slots per compose tile (per layer)
+constexpr int kComposeBulkTile = 32;   // most slots per tile of the bulk-copy compose kernel
 
 // RoPE frequency i as a fraction of a full turn in 0.64 fixed point:
 // turn[i] = round(theta^(-2i/d) / (2 pi) * 2^64).  For an integer position p the angle in
@@ -42,7 +43,8 @@ struct OccParam {
     const void* host_v;
 };
 
-struct ComposeParams {
+// Everything of a compose launch but its occurrence table.
+struct ComposeHead {
     const void* pool_k;      // [L][pool_slots][Hkv][d]
     const void* pool_v;
     void* out_k;             // [L][rows][Hkv][d]
@@ -55,10 +57,15 @@ struct ComposeParams {
     int32_t n_tiles;
     int32_t hkv;
     int32_t layer0;          // layer of grid row 0 (a launch covers layers layer0 .. + gridDim.y)
-    int32_t tile_slots;      // composed slots per tile, 1 .. kComposeTile (chosen per launch)
+    int32_t tile_slots;      // composed slots per tile, 1 .. kComposeTile (1 .. kComposeBulkTile
+                             // with bulk; chosen per launch)
+    int32_t bulk;            // 1: the bulk-copy kernel (every chunk in the device pool)
     int32_t pre_rope;        // 1: stored K is before RoPE; slot j of occurrence o turns by its
                              // composed position o.delta + p_j (PRE_ROPE storage)
     RopeTurns rope;
+};
+
+struct ComposeParams : ComposeHead {
     OccParam occ[kMaxOcc];
 };
 
@@ -142,15 +149,6 @@ struct AttnParams {
     ReqParam req[kMaxReq];
 };
 
-// Launchers: return the launch error, never throw.  `d` is head_dim.
-// max_ctas > 0 caps the CTAs per layer; each then walks several tiles (a compose that reads
-// host-resident chunks is bound by the host link, and leaves the other SMs to attention).
-cudaError_t launch_compose(const ComposeParams& p, int dtype, int d, int layers, cudaStream_t s,
-                           int max_ctas = 0);
-cudaError_t launch_compress(const CompressParams& p, int dtype, int d, cudaStream_t s);
-cudaError_t launch_suffix_prep(const SuffixParams& p, int dtype, int d, cudaStream_t s);
-cudaError_t launch_attn_simt(const AttnParams& p, int dtype, int d, cudaStream_t s);
-
 // Called by a launcher after its host-side preparation (tensor maps, function attributes)
 // and right before it enqueues its kernels, so that a trace event recorded there brackets
 // device work only.
@@ -161,6 +159,16 @@ struct Hook {
         if (fn) fn(arg);
     }
 };
+
+// Launchers: return the launch error, never throw.  `d` is head_dim.
+// max_ctas > 0 caps the CTAs per layer; each then walks several tiles (a compose that reads
+// host-resident chunks is bound by the host link, and leaves the other SMs to attention).
+cudaError_t launch_compose(const ComposeParams& p, int dtype, int d, int layers, cudaStream_t s,
+                           int max_ctas = 0, Hook pre = {});
+cudaError_t launch_compress(const CompressParams& p, int dtype, int d, cudaStream_t s);
+cudaError_t launch_suffix_prep(const SuffixParams& p, int dtype, int d, cudaStream_t s);
+cudaError_t launch_attn_simt(const AttnParams& p, int dtype, int d, cudaStream_t s);
+
 
 // Decode attention (decode.cu): one new token per request (suffix index ReqParam::t0,
 // already rotated into q_rot and appended to the cache) over keys 0 .. S_r + t0.

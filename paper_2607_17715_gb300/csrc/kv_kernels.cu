@@ -9,8 +9,10 @@
 // once to a float in [-1/2, 1/2) turns and handed to sincospif.  The error is about
 // 1e-7 rad at any position, where forming p * inv_freq in fp32 would lose p * 2^-24 rad.
 #include <algorithm>
+#include <atomic>
 
 #include "internal.cuh"
+#include "ptx.cuh"
 #include "rope.cuh"
 #include "vec16.cuh"
 
@@ -129,6 +131,255 @@ __global__ void __launch_bounds__(256) compose_kernel(const __grid_constant__ Co
                 st16(ov + dof[u] + HALF, vy[u]);
             }
         }
+    }
+}
+
+// ---------------------------------------------------------------------------------------
+// compose, bulk-copy form (every chunk of the launch in the device pool).  A tile is up to
+// P.tile_slots consecutive slots of one occurrence in one layer: its K rows and its V rows
+// are each one contiguous run of bytes in the pool and one in the cache, so each moves as
+// one bulk copy (cp.async.bulk) into shared memory and one back out.  The tiles of all
+// layers form one list, layer-major; CTA c (one per SM) takes a contiguous run of it.
+//
+// Warp 0 is the copy warp: its lane 0 fills every stage of the ring, then per tile waits for
+// the turning warps to finish it, stores its K and V, and refills the stage the tile before
+// it used (that store's reads of shared memory complete first: wait_group.read 1).  The
+// other eight warps turn K in shared memory per tile (thread t always takes the same vector
+// of the half-head, so under LOCAL_ROPE storage it forms its E (cos, sin) pairs once per
+// occurrence) and write the positions; V passes through untouched.  The occurrence table
+// sits in the kernel parameters, sized to the launch (N entries), so a launch of few
+// occurrences does not pay for moving a large parameter block.
+// ---------------------------------------------------------------------------------------
+constexpr int kBulkTurnWarps = 8;
+constexpr int kBulkThreads = 32 * (1 + kBulkTurnWarps);
+constexpr int kBulkMaxStages = 8;
+constexpr uint32_t kBulkSmem = 192u * 1024u;
+
+template <int N>
+struct BulkParams : ComposeHead {
+    OccParam occ[N];
+};
+
+struct BulkTile {
+    int32_t layer, src, dst, ns, delta, n, k, j0, ok;
+};
+
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+                 "l"(src), "r"(bytes), "r"(bar)
+                 : "memory");
+}
+__device__ __forceinline__ void bulk_store(void* dst, uint32_t src, uint32_t bytes) {
+    asm volatile("cp.async.bulk.global.shared::cta.bulk_group [%0], [%1], %2;" ::"l"(dst), "r"(src), "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ uint4 lds128(uint32_t a) {
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a));
+    return v;
+}
+__device__ __forceinline__ void sts128(uint32_t a, const uint4& v) {
+    asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(a), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
+                 : "memory");
+}
+
+// A wait that ignores the abort flag (for loads still in flight when the CTA gives up).
+__device__ __forceinline__ void mbar_wait_limit(uint32_t bar, uint32_t parity) {
+    const long long t0 = clock64();
+    while (!mbar_try(bar, parity) && clock64() - t0 < kWaitCycles) {
+    }
+}
+
+template <typename T, int VPH, int N>
+__global__ void __launch_bounds__(kBulkThreads, 1)
+    compose_bulk_kernel(const __grid_constant__ BulkParams<N> P, int n_layers, int nst) {
+    using V = Vec16<T>;
+    constexpr int E = V::N;
+    constexpr int HALF = VPH * E;
+    constexpr int D = 2 * HALF;
+    constexpr int NT = 32 * kBulkTurnWarps;
+    static_assert(NT % VPH == 0, "a thread keeps one vector of the half-head");
+    extern __shared__ __align__(1024) unsigned char bulk_smem[];
+    __shared__ __align__(8) uint64_t full[kBulkMaxStages];
+    __shared__ __align__(8) uint64_t turned[kBulkMaxStages];
+    __shared__ BulkTile desc[kBulkMaxStages];
+    __shared__ uint32_t abort_flag;
+    volatile uint32_t* abort = &abort_flag;
+
+    const int tid = (int)threadIdx.x;
+    const int ts = P.tile_slots;
+    const int64_t row_elems = (int64_t)P.hkv * D;
+    const uint32_t row_bytes = (uint32_t)(row_elems * (int64_t)sizeof(T));
+    const uint32_t half_stage = (uint32_t)ts * row_bytes;          // K, then V
+    const uint32_t sbase = smem_u32(bulk_smem);
+    const int64_t total = (int64_t)P.n_tiles * n_layers;
+    const int64_t it0 = total * blockIdx.x / gridDim.x;
+    const int64_t it1 = total * (blockIdx.x + 1) / gridDim.x;
+    const int count = (int)(it1 - it0);
+    auto full_bar = [&](int st) { return smem_u32(&full[st]); };
+    auto turned_bar = [&](int st) { return smem_u32(&turned[st]); };
+
+    if (tid == 0) {
+        abort_flag = 0u;
+        for (int st = 0; st < nst; ++st) {
+            mbar_init(full_bar(st), 1);
+            mbar_init(turned_bar(st), kBulkTurnWarps);
+        }
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncthreads();
+
+    if (tid < 32) {
+        // ------------------------------------------------------------- copy warp
+        if (tid != 0) return;
+        int occ_i = 0, walk_layer = -1;
+        auto issue = [&](int i) {
+            const int64_t it = it0 + i;
+            const int l = (int)(it / P.n_tiles);
+            const int tile = (int)(it - (int64_t)l * P.n_tiles);
+            if (l != walk_layer) {                // a new layer: find the tile's occurrence
+                int lo = 0, hi = P.n_occ - 1;
+                while (lo < hi) {
+                    const int mid = (lo + hi + 1) >> 1;
+                    if (P.occ[mid].tile_base <= tile) lo = mid;
+                    else hi = mid - 1;
+                }
+                occ_i = lo;
+                walk_layer = l;
+            }
+            while (occ_i + 1 < P.n_occ && P.occ[occ_i + 1].tile_base <= tile) ++occ_i;
+            const OccParam& o = P.occ[occ_i];
+            BulkTile t;
+            t.layer = P.layer0 + l;
+            t.j0 = (tile - o.tile_base) * ts;
+            t.ns = min(ts, o.m - t.j0);
+            t.src = o.src_base + t.j0;
+            t.dst = o.dest_row + t.j0;
+            t.delta = o.delta;
+            t.n = o.n;
+            t.k = o.k;
+            t.ok = t.ns > 0 && t.src >= 0 && (int64_t)t.src + t.ns <= P.pool_slots && t.dst >= 0 &&
+                   (int64_t)t.dst + t.ns <= P.rows;
+            if (!t.ok && t.ns > 0) atomicOr(P.err, 1);
+            const int st = i % nst;
+            desc[st] = t;
+            const uint32_t bytes = t.ok ? (uint32_t)t.ns * row_bytes : 0u;
+            mbar_expect_tx(full_bar(st), 2u * bytes);
+            if (t.ok) {
+                const int64_t so = ((int64_t)t.layer * P.pool_slots + t.src) * row_elems;
+                const uint32_t dk = sbase + (uint32_t)st * 2u * half_stage;
+                bulk_load(dk, static_cast<const T*>(P.pool_k) + so, bytes, full_bar(st));
+                bulk_load(dk + half_stage, static_cast<const T*>(P.pool_v) + so, bytes, full_bar(st));
+            }
+        };
+        int issued = 0;
+        for (; issued < nst && issued < count; ++issued) issue(issued);
+        int stored = 0;
+        for (; stored < count; ++stored) {
+            const int st = stored % nst;
+            mbar_wait(turned_bar(st), (uint32_t)(stored / nst) & 1u, P.err, abort);
+            if (*abort) break;
+            const BulkTile t = desc[st];
+            if (t.ok) {
+                const int64_t co = ((int64_t)t.layer * P.rows + t.dst) * row_elems;
+                const uint32_t bytes = (uint32_t)t.ns * row_bytes;
+                const uint32_t dk = sbase + (uint32_t)st * 2u * half_stage;
+                bulk_store(static_cast<T*>(P.out_k) + co, dk, bytes);
+                bulk_store(static_cast<T*>(P.out_v) + co, dk + half_stage, bytes);
+            }
+            asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+            // the stage of tile `stored - 1` is refilled once that tile's store has read it
+            if (stored >= 1 && issued < count) {
+                asm volatile("cp.async.bulk.wait_group.read 1;" ::: "memory");
+                issue(issued++);
+            }
+        }
+        // after an abort: loads in flight land before the CTA leaves; then every store has
+        // completed
+        for (int i = stored; i < issued; ++i) mbar_wait_limit(full_bar(i % nst), (uint32_t)(i / nst) & 1u);
+        asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+        return;
+    }
+
+    // ----------------------------------------------------------------- turning warps
+    const int ct = tid - 32;
+    const int lane = tid & 31;
+    const int iv = ct % VPH;                  // this thread's vector of the half-head
+    float2 cs[E];
+    int cs_delta = 0;
+    bool cs_valid = false;
+    const int per_slot = P.hkv * VPH;
+    auto turn_item = [](const float2 (&c)[E], uint4& xv, uint4& yv) {
+        float fx[E], fy[E], gx[E], gy[E];
+        V::unpack(xv, fx);
+        V::unpack(yv, fy);
+        rotate<E>(fx, fy, c, gx, gy);
+        xv = V::pack(gx);
+        yv = V::pack(gy);
+    };
+    for (int i = 0; i < count; ++i) {
+        const int st = i % nst;
+        mbar_wait(full_bar(st), (uint32_t)(i / nst) & 1u, P.err, abort);
+        if (*abort) break;                    // the same tile for every turning thread
+        const BulkTile t = desc[st];
+        if (t.ok) {
+            const uint32_t dk = sbase + (uint32_t)st * 2u * half_stage;
+            if (!P.pre_rope && (!cs_valid || cs_delta != t.delta)) {
+#pragma unroll
+                for (int e = 0; e < E; ++e) cs[e] = turn_cs(P.rope.turn[iv * E + e], t.delta);
+                cs_delta = t.delta;
+                cs_valid = true;
+            }
+            const int items = t.ns * per_slot;
+            auto addr = [&](int it) {
+                const int sl = it / per_slot;
+                const int h = (it - sl * per_slot) / VPH;
+                return dk + (uint32_t)sl * row_bytes + (uint32_t)((h * D + iv * E) * (int)sizeof(T));
+            };
+            auto pre_cs = [&](int it, float2 (&c)[E]) {     // slot j at its composed position delta + p_j
+                const int j = t.j0 + it / per_slot;
+                const int64_t pos = (int64_t)t.delta + min((j + 1) * t.k, t.n) - 1;
+#pragma unroll
+                for (int e = 0; e < E; ++e) c[e] = turn_cs(P.rope.turn[iv * E + e], pos);
+            };
+            constexpr uint32_t YO = HALF * (uint32_t)sizeof(T);
+            // two items per pass, both loaded before either is turned
+            for (int a0 = ct; a0 < items; a0 += 2 * NT) {
+                const int a1 = a0 + NT;
+                const bool v1 = a1 < items;
+                const uint32_t p0 = addr(a0), p1 = v1 ? addr(a1) : p0;
+                uint4 x0 = lds128(p0), y0 = lds128(p0 + YO), x1, y1;
+                if (v1) {
+                    x1 = lds128(p1);
+                    y1 = lds128(p1 + YO);
+                }
+                if (P.pre_rope) {
+                    float2 c0[E];
+                    pre_cs(a0, c0);
+                    turn_item(c0, x0, y0);
+                    if (v1) {
+                        float2 c1[E];
+                        pre_cs(a1, c1);
+                        turn_item(c1, x1, y1);
+                    }
+                } else {
+                    turn_item(cs, x0, y0);
+                    if (v1) turn_item(cs, x1, y1);
+                }
+                sts128(p0, x0);
+                sts128(p0 + YO, y0);
+                if (v1) {
+                    sts128(p1, x1);
+                    sts128(p1 + YO, y1);
+                }
+            }
+            if (t.layer == 0)
+                for (int sl = ct; sl < t.ns; sl += NT) P.pos[t.dst + sl] = t.delta + min((t.j0 + sl + 1) * t.k, t.n) - 1;
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");   // turned K visible to the copy engine
+        }
+        __syncwarp();
+        if (lane == 0) mbar_arrive(turned_bar(st));
     }
 }
 
@@ -377,15 +628,61 @@ cudaError_t preload_suffix_kernels(int dtype, int d) {
     return cudaErrorInvalidValue;
 }
 
+template <typename T, int VPH, int N>
+cudaError_t launch_bulk_n(const ComposeParams& p, int layers, cudaStream_t s, Hook pre) {
+    static std::atomic<uint64_t> attr_set{0};     // per instantiation: devices 0..63 done
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    const uint64_t bit = dev < 64 ? (uint64_t)1 << dev : 0;
+    if (!(attr_set.load() & bit)) {
+        e = cudaFuncSetAttribute(compose_bulk_kernel<T, VPH, N>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)kBulkSmem);
+        if (e != cudaSuccess) return e;
+        attr_set.fetch_or(bit);
+    }
+    BulkParams<N> bp;
+    static_cast<ComposeHead&>(bp) = p;
+    for (int i = 0; i < p.n_occ; ++i) bp.occ[i] = p.occ[i];
+    const int64_t row_bytes = (int64_t)p.hkv * VPH * Vec16<T>::N * 2 * (int64_t)sizeof(T);
+    const int64_t stage = 2 * (int64_t)p.tile_slots * row_bytes;
+    const int nst = (int)std::min<int64_t>(kBulkMaxStages, kBulkSmem / stage);
+    if (nst < 2) return cudaErrorInvalidValue;
+    const int64_t items = (int64_t)p.n_tiles * layers;
+    const int grid = (int)std::min<int64_t>(items, sm_count());
+    pre();
+    compose_bulk_kernel<T, VPH, N><<<grid, kBulkThreads, (size_t)(nst * stage), s>>>(bp, layers, nst);
+    return cudaGetLastError();
+}
+
+template <typename T, int VPH>
+cudaError_t launch_bulk(const ComposeParams& p, int layers, cudaStream_t s, Hook pre) {
+    if (p.n_occ <= 16) return launch_bulk_n<T, VPH, 16>(p, layers, s, pre);
+    if (p.n_occ <= 128) return launch_bulk_n<T, VPH, 128>(p, layers, s, pre);
+    static_assert(kMaxOcc == 512, "the largest table size is the launch limit");
+    return launch_bulk_n<T, VPH, 512>(p, layers, s, pre);
+}
+
 cudaError_t launch_compose(const ComposeParams& p, int dtype, int d, int layers, cudaStream_t s,
-                           int max_ctas) {
+                           int max_ctas, Hook pre) {
     if (p.n_tiles == 0 || p.n_occ == 0) return cudaSuccess;
     (void)cudaGetLastError();   // report this launch's error only, not a stale one
+    if (p.bulk) {
+        if (layers < 1 || p.tile_slots < 1 || p.tile_slots > kComposeBulkTile) return cudaErrorInvalidValue;
+        for (int i = 0; i < p.n_occ; ++i)
+            if (p.occ[i].host) return cudaErrorInvalidValue;
+        if (dtype == kDtypeBf16 && d == 128) return launch_bulk<__nv_bfloat16, 8>(p, layers, s, pre);
+        if (dtype == kDtypeBf16 && d == 64) return launch_bulk<__nv_bfloat16, 4>(p, layers, s, pre);
+        if (dtype == kDtypeF32 && d == 128) return launch_bulk<float, 16>(p, layers, s, pre);
+        if (dtype == kDtypeF32 && d == 64) return launch_bulk<float, 8>(p, layers, s, pre);
+        return cudaErrorInvalidValue;
+    }
     if (layers > 65535 || p.tile_slots < 1 || p.tile_slots > kComposeTile) return cudaErrorInvalidValue;
     const dim3 grid(max_ctas > 0 && max_ctas < p.n_tiles ? max_ctas : p.n_tiles, layers);
     // one thread per four items of a tile (item = slot, head, vector pair), in whole warps
     const int items = p.tile_slots * p.hkv * vph_of(dtype, d);
     const int threads = std::min(256, std::max(32, (items / 4 + 31) / 32 * 32));
+    pre();
     if (dtype == kDtypeBf16 && d == 128) compose_kernel<__nv_bfloat16, 8><<<grid, threads, 0, s>>>(p);
     else if (dtype == kDtypeBf16 && d == 64) compose_kernel<__nv_bfloat16, 4><<<grid, threads, 0, s>>>(p);
     else if (dtype == kDtypeF32 && d == 128) compose_kernel<float, 16><<<grid, threads, 0, s>>>(p);
