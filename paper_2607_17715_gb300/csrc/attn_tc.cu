@@ -324,6 +324,12 @@ __device__ __forceinline__ void tma_store_4d(const CUtensorMap* tm, uint32_t src
                  "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(src)
                  : "memory");
 }
+// 32 bytes (one full L2 sector) to global memory in one instruction (sm_100 256-bit stores).
+__device__ __forceinline__ void stg256(void* p, const uint32_t* w) {
+    asm volatile("st.global.v8.b32 [%0], {%1, %2, %3, %4, %5, %6, %7, %8};" ::"l"(p), "r"(w[0]), "r"(w[1]),
+                 "r"(w[2]), "r"(w[3]), "r"(w[4]), "r"(w[5]), "r"(w[6]), "r"(w[7])
+                 : "memory");
+}
 __device__ __forceinline__ void sts128_(uint32_t a, const uint4& v) {
     asm volatile("st.shared.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(a), "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w)
                  : "memory");
@@ -501,7 +507,13 @@ __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, u
         return;
     }
     if (P.n_split == 1) {
+        // each thread writes its own row, a full 32-byte sector per store: the lanes of a
+        // warp hold rows of up to 32 different lines, so a narrower store would leave every
+        // sector it touches half written
+        // (rows are 256 bytes apart, so the output's base alignment decides; the entry points
+        // guarantee 16 bytes only)
         __nv_bfloat16* orow = static_cast<__nv_bfloat16*>(P.out) + row_id * HD;
+        const bool a32 = (reinterpret_cast<uintptr_t>(P.out) & 31u) == 0;
 #pragma unroll
         for (int c = 0; c < 4; ++c) {
             uint32_t ov[32];
@@ -509,13 +521,18 @@ __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, u
             tmem_ld_wait();
             if (t < P.sq) {
 #pragma unroll
-                for (int q8 = 0; q8 < 4; ++q8) {
-                    uint4 w;
-                    w.x = pack_bf16(__uint_as_float(ov[q8 * 8 + 0]) * inv, __uint_as_float(ov[q8 * 8 + 1]) * inv);
-                    w.y = pack_bf16(__uint_as_float(ov[q8 * 8 + 2]) * inv, __uint_as_float(ov[q8 * 8 + 3]) * inv);
-                    w.z = pack_bf16(__uint_as_float(ov[q8 * 8 + 4]) * inv, __uint_as_float(ov[q8 * 8 + 5]) * inv);
-                    w.w = pack_bf16(__uint_as_float(ov[q8 * 8 + 6]) * inv, __uint_as_float(ov[q8 * 8 + 7]) * inv);
-                    *reinterpret_cast<uint4*>(orow + c * 32 + q8 * 8) = w;
+                for (int h = 0; h < 2; ++h) {
+                    uint32_t w[8];
+#pragma unroll
+                    for (int e = 0; e < 8; ++e)
+                        w[e] = pack_bf16(__uint_as_float(ov[h * 16 + 2 * e]) * inv,
+                                         __uint_as_float(ov[h * 16 + 2 * e + 1]) * inv);
+                    if (a32) {
+                        stg256(orow + c * 32 + h * 16, w);
+                    } else {
+                        *reinterpret_cast<uint4*>(orow + c * 32 + h * 16) = make_uint4(w[0], w[1], w[2], w[3]);
+                        *reinterpret_cast<uint4*>(orow + c * 32 + h * 16 + 8) = make_uint4(w[4], w[5], w[6], w[7]);
+                    }
                 }
             }
         }
@@ -537,10 +554,11 @@ __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, u
             }
             if (t < P.sq) {
 #pragma unroll
-                for (int q4 = 0; q4 < 8; ++q4) {
-                    float4 w = make_float4(__uint_as_float(ov[q4 * 4 + 0]) * inv, __uint_as_float(ov[q4 * 4 + 1]) * inv,
-                                           __uint_as_float(ov[q4 * 4 + 2]) * inv, __uint_as_float(ov[q4 * 4 + 3]) * inv);
-                    *reinterpret_cast<float4*>(orow + c * 32 + q4 * 4) = w;
+                for (int q8 = 0; q8 < 4; ++q8) {
+                    uint32_t w[8];
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) w[e] = __float_as_uint(__uint_as_float(ov[q8 * 8 + e]) * inv);
+                    stg256(orow + c * 32 + q8 * 8, w);
                 }
             }
         }

@@ -364,3 +364,37 @@ def test_attend_forced_split_batched():
     wl = _small(synth.workload("batched"), batch=3, chunks_per_request=4, pool_chunks=32,
                 n_suffix=40)
     _attend_case(wl, attn_split=5)
+
+
+def test_attend_output_at_16_byte_offset_matches():
+    # the tensor-core epilogue stores 32 bytes at a time when the output is 32-byte aligned,
+    # 16 otherwise: an output starting 16 bytes into a buffer gives the same bits, through
+    # the per-row stores (CTAs of four pairs of query tiles) and the staged store of the last
+    c2kv = H.lib()
+    wl = synth.scaled(L8B_1, layers=2, chunks_per_request=3, pool_chunks=3, n_suffix=200)
+    reqs = synth.requests(wl)
+    all_ids = sorted({c for ids, _ in reqs for c in ids})
+    chunks = H.oracle_chunks_meanpool(wl, all_ids)
+    ctx = H.make_ctx(wl, pool_slots=sum(orc.n_slots(wl.chunk_tokens, wl.ratio_k) for _ in all_ids) + 16,
+                     attn_pairs=4)
+    try:
+        dev = H.load_stored(ctx, wl, chunks)
+        req_ptr = np.cumsum([0] + [len(ids) for ids, _ in reqs])
+        cache = c2kv.c2kv_compose(ctx, req_ptr, [dev[c] for ids, _ in reqs for c in ids],
+                                  [o for _, offs in reqs for o in offs], suffix_capacity=200)
+        q, ks, vs = synth.suffix(wl, layers=wl.layers)
+        qd, kd, vd = (H.to_dev(x[:, :1], wl) for x in (q, ks, vs))
+        out = torch.full_like(qd, float("nan"))
+        c2kv.c2kv_attend(ctx, cache, -1, qd, kd, vd, 200, out)
+        buf = torch.full((out.numel() + 8,), float("nan"), dtype=out.dtype, device="cuda")
+        off = buf[8:].view(out.shape)                     # 16 bytes past a 256-byte boundary
+        assert off.data_ptr() % 32 == 16
+        c2kv.c2kv_attend(ctx, cache, -1, qd, kd, vd, 200, off)
+        c2kv.c2kv_sync(ctx)
+        assert torch.equal(out, off)
+        ref = orc.run_request(chunks, reqs[0][0], reqs[0][1], q[:, 0], ks[:, 0], vs[:, 0],
+                              wl.rope_theta, wl.dtype)
+        H.check_attention(out.double().cpu().numpy()[:, 0], ref["out"], wl, "O")
+        c2kv.c2kv_cache_release(ctx, cache)
+    finally:
+        c2kv.c2kv_destroy(ctx)
