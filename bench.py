@@ -88,12 +88,14 @@ def source_digest(paths):
 def captured_traffic(kernel, workload):
     """DRAM bytes per launch from the committed ncu summary, if it was captured on this
     workload and every source the kernel is built from is still the one that was captured
-    (else None: the counters do not describe this launch)."""
+    (else None: the counters do not describe this launch).  Records are keyed
+    "kernel@workload" (or "kernel" for the default workload's)."""
     path = os.path.join(ROOT, "profiles", "traffic.json")
     if not os.path.exists(path):
         return None
     with open(path) as fh:
-        rec = json.load(fh).get(kernel)
+        recs = json.load(fh)
+    rec = recs.get(f"{kernel}@{workload}") or recs.get(kernel)
     if not rec or "sources" not in rec or rec.get("workload") != workload:
         return None
     return rec["traffic_bytes"] if source_digest(rec["sources"]) == rec["sha256_16"] else None
@@ -112,7 +114,7 @@ def rooflines(compose_ms, attn_ms, f, hbm, bf16, src):
     """Roofline objects for the compose kernel and the attention kernel (algorithmic work /
     measured kernel time), with the dominant one as "roofline"."""
     comp_gbs = f["compose_bytes"] / (compose_ms / 1e3) / 1e9
-    compose = {"bound": "hbm", "kernel": "compose_kernel", "achieved": round(comp_gbs, 1),
+    compose = {"bound": "hbm", "kernel": "compose_bulk_kernel", "achieved": round(comp_gbs, 1),
                "peak": hbm, "unit": "GB/s", "frac": round(comp_gbs / hbm, 4),
                "traffic": captured_traffic("compose_kernel", f["name"]), "peak_source": f"{src} hbm_gbs",
                "bytes_per_launch": f["compose_bytes"]}
