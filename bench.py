@@ -854,8 +854,8 @@ def run_ours(args):
         "e2e": {"value": round(positions / (e2e_ms / 1e3), 1),
                 "unit": "tokens/s", "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
                 "ms_per_step": round(e2e_ms / args.steps, 4),
-                "path": "chunks (MODE_HOST), suffix Q/K/V and output in pinned host memory, "
-                        "read and written by the kernels across the CPU-GPU link (no copies)",
+                "path": "chunks (MODE_HOST) read by compose across the CPU-GPU link; suffix Q/K/V "
+                        "and output in pinned host memory, copied in and out by the call per layer group",
                 "staged": {"value": round(positions / (staged_ms / 1e3), 1),
                            "ms_per_step": round(staged_ms / args.steps, 4),
                            "h2d_bytes_per_step": h2d_staged,
