@@ -348,7 +348,8 @@ c2kv_status c2kv_attend_noalloc(c2kv_ctx* ctx, c2kv_cache* cache, int32_t layer,
  * exactly (log-sum-exp); the split buffer comes from the context's memory pool.  With bf16
  * and d = 128 the step runs on the tensor-core attention kernel (the new token as a one-row
  * query tile) when (layers x requests x KV heads) fits one CTA per SM or a request holds
- * 4096 keys or more, else on a CUDA-core decode kernel (C2KV_ATTN_SIMT forces the latter).
+ * 4096 keys or more, else on a CUDA-core decode kernel (C2KV_ATTN_TC forces the former,
+ * C2KV_ATTN_SIMT the latter).
  * The tensor-core route reads whole 128-row key tiles, so it zeroes the rows after the new
  * one up to the next 128-row boundary that no earlier call on this cache has written or
  * zeroed (never rows an earlier c2kv_attend or c2kv_decode wrote).

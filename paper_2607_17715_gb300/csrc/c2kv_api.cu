@@ -1257,7 +1257,7 @@ c2kv_status c2kv_decode(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
         const int64_t tiles_max = (n_keys_max + 127) / 128;
         const bool use_tc = c->cfg.attn_impl != C2KV_ATTN_SIMT &&
                             c2kv::attn_tc_supported(c->cfg.dtype, d, hq, hkv) &&
-                            (units <= c->sms || tiles_max >= 32);
+                            (c->cfg.attn_impl == C2KV_ATTN_TC || units <= c->sms || tiles_max >= 32);
         int32_t n_split = 1;
         if (use_tc) {
             // splits per (layer, request, KV head): the fewest waves of one-CTA-per-SM work,

@@ -81,6 +81,7 @@ def _decode_case(wl, steps, prefill=None, layer=-1, extra_steps=0, attn_impl=0):
 
 
 IMPLS = pytest.mark.parametrize("impl", [0, 1], ids=["auto", "cuda_core"])   # 1: C2KV_ATTN_SIMT
+TC = 2                                                                          # C2KV_ATTN_TC
 
 
 @IMPLS
@@ -257,3 +258,13 @@ def test_decode_rejects_bad_steps_and_layouts():
         assert ei.value.status == c2kv.ERR_UNSUPPORTED
     finally:
         c2kv.c2kv_destroy(ctx)
+
+
+@pytest.mark.parametrize("impl", [TC, 1], ids=["tensor_cores", "cuda_core"])
+def test_decode_more_requests_than_one_launch_takes(impl):
+    # 260 requests: the attention kernels take at most 256 requests a launch, so the step runs
+    # as two groups (on the tensor-core route its split partials are merged once, after the
+    # last group); every request's output against the oracle
+    wl = _small(synth.workload("batched"), batch=260, chunks_per_request=1, pool_chunks=260,
+                chunk_tokens=64, layers=1, draw="distinct")
+    _decode_case(wl, steps=[2 + (b % 5) for b in range(260)], prefill=7, attn_impl=impl)
