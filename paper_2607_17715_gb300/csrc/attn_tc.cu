@@ -1476,6 +1476,9 @@ __device__ __forceinline__ void plain_producer(const TcParams& P, int l, int bl,
     const int G = P.group;
     const int qz = l * P.batch_total + b;
     const int key0 = (int)((int64_t)(P.layer0 + l) * P.rows + P.req[bl].row_base);
+    // launched as a programmatic dependent: the grid before it (which wrote Q and the newest
+    // key rows) has completed and its writes are visible (returns at once otherwise)
+    asm volatile("griddepcontrol.wait;" ::: "memory");
     int qi = 0;                             // next pair whose Q tiles to load
     int pk = 0, jk = 0, gk = 0;             // K: pair, tile within it, tiles issued in all
     int pv = 0, jv = 0, gv = 0;             // V: the same
@@ -1654,6 +1657,9 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = *tmem_slot;
+    // a programmatic dependent launched after this grid (the split merge) may start now: it
+    // waits for this grid before it reads what this one writes
+    if (!kFused && threadIdx.x == 0) asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
     if (warp < 4) {
         asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kFused ? kRegsLowFused : kRegsLow));
@@ -1789,6 +1795,7 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
 constexpr int kMaxSplit = 16;
 
 __global__ void __launch_bounds__(256) attn_combine_kernel(const __grid_constant__ AttnParams P) {
+    asm volatile("griddepcontrol.wait;" ::: "memory");   // the partials are complete and visible
     const int64_t rows = (int64_t)P.lq * P.batch_total * P.sq * P.hq;
     const int64_t row = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
     const int lane = threadIdx.x & 31;
@@ -1874,7 +1881,21 @@ cudaError_t launch_attn_combine(const AttnParams& a, cudaStream_t s) {
     const int64_t rows = (int64_t)a.lq * a.batch_total * a.sq * a.hq;
     const int64_t blocks = (rows + 7) / 8;
     if (blocks > 0x7fffffffLL) return cudaErrorInvalidValue;
-    attn_combine_kernel<<<(unsigned)blocks, 256, 0, s>>>(a);
+    if (a.dependent) {          // its launch overlaps the attention's last CTAs
+        cudaLaunchConfig_t cfg{};
+        cfg.gridDim = dim3((unsigned)blocks);
+        cfg.blockDim = dim3(256);
+        cfg.stream = s;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        const cudaError_t e = cudaLaunchKernelEx(&cfg, attn_combine_kernel, a);
+        if (e != cudaSuccess) return e;
+    } else {
+        attn_combine_kernel<<<(unsigned)blocks, 256, 0, s>>>(a);
+    }
     return cudaGetLastError();
 }
 
@@ -1994,7 +2015,22 @@ cudaError_t launch_attn_tc(const AttnParams& a, cudaStream_t s, Hook before) {
     cudaError_t e = prepare_tc<false>(a, p, grid);
     if (e != cudaSuccess) return e;
     before();
-    attn_tc_kernel<false><<<grid, kThreads, kSmemBytes, s>>>(p);
+    if (a.dependent) {          // starts while the kernel before it runs (the producer waits)
+        cudaLaunchConfig_t cfg{};
+        cfg.gridDim = grid;
+        cfg.blockDim = dim3(kThreads);
+        cfg.dynamicSmemBytes = kSmemBytes;
+        cfg.stream = s;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        e = cudaLaunchKernelEx(&cfg, attn_tc_kernel<false>, p);
+        if (e != cudaSuccess) return e;
+    } else {
+        attn_tc_kernel<false><<<grid, kThreads, kSmemBytes, s>>>(p);
+    }
     return cudaGetLastError();
 }
 

@@ -1384,6 +1384,9 @@ c2kv_status c2kv_decode(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
                 a.pairs_per_cta = c->cfg.attn_pairs;
                 a.part_o = part;
                 a.part_lse = part ? part + (size_t)n_split * rows_all * d : nullptr;
+                // the suffix kernel's programmatic dependent, and the merge the attention's,
+                // unless a trace puts events between them
+                a.dependent = c->prof ? 0 : 1;
                 for (int32_t i = 0; i < nb; ++i) a.req[i] = reqs[b0 + i];
                 ProfScope prof_decode(c, C2KV_PROF_DECODE, true);
                 e = c2kv::launch_attn_tc(a, c->stream, prof_decode.hook());

@@ -146,6 +146,9 @@ struct AttnParams {
     float* part_lse;         // n_split > 1: [n_split][Lq][Btot][Hq][Sq] fp32, log2 domain
     int32_t pairs_per_cta;   // tensor-core kernel: at most this many pairs of query tiles per
                              // CTA (0 = chosen per launch)
+    int32_t dependent;       // tensor-core kernel and its merge: launched as the programmatic
+                             // dependent of the kernel before them on the stream (each waits
+                             // for that grid before it reads memory)
     ReqParam req[kMaxReq];
 };
 
