@@ -835,11 +835,15 @@ cudaError_t attend_run(c2kv_ctx* c, c2kv_cache* cache, int32_t layer0, int32_t l
                 e = c2kv::launch_suffix_prep(s, c->cfg.dtype, c->cfg.head_dim, c->stream);
             }
             if (e != cudaSuccess) break;
+            // the suffix kernel's programmatic dependent (its start and set-up overlap that
+            // kernel), unless a trace puts events between them or the suffix ran elsewhere
+            a.dependent = !c->prof && !q_rot_ready ? 1 : 0;
             ProfScope prof_attn(c, C2KV_PROF_ATTN, use_tc);
             e = use_tc ? c2kv::launch_attn_tc(a, c->stream, prof_attn.hook())
                        : c2kv::launch_attn_simt(a, c->cfg.dtype, c->cfg.head_dim, c->stream);
         }
         last = a;
+        last.dependent = !c->prof && !fused && use_tc ? 1 : 0;   // the merge: the attention's dependent
     }
     if (e == cudaSuccess && n_split > 1) {   // one merge over every request's rows
         ProfScope prof_combine(c, C2KV_PROF_COMBINE);

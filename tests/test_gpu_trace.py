@@ -35,3 +35,44 @@ def test_profile_counts_and_times():
         assert np.isfinite(out.float().cpu().numpy()).all()
     finally:
         c2kv.c2kv_destroy(ctx)
+
+
+@pytest.mark.parametrize("split", [False, True], ids=["one_split", "key_range_splits"])
+def test_attend_traced_equals_untraced(split):
+    # untraced, the attention starts as the suffix kernel's programmatic dependent (and the
+    # split merge as the attention's); traced, events sit between them and they run one after
+    # the other: the same O and lse, bit for bit
+    base = synth.workload("llama8b")
+    if split:      # one layer of 3 x 1024 slots: few units, long ranges, so the keys are split
+        wl = synth.scaled(base, layers=1, chunks_per_request=3, pool_chunks=3, chunk_tokens=1024,
+                          ratio_k=1)
+    else:
+        wl = synth.scaled(base, layers=2, chunks_per_request=3, pool_chunks=3)
+    c2kv = H.lib()
+    m = -(-wl.chunk_tokens // wl.ratio_k)
+    ctx = H.make_ctx(wl, pool_slots=3 * m + 16)
+    try:
+        ids = []
+        for cid in range(3):
+            kt, vt = synth.chunk_tokens(wl, cid)
+            ids.append(c2kv.c2kv_compress_chunk(ctx, H.to_dev(kt, wl), H.to_dev(vt, wl),
+                                                wl.chunk_tokens, wl.ratio_k, c2kv.MODE_MEANPOOL))
+        cache = c2kv.c2kv_compose(ctx, [0, 3], ids, None, wl.n_suffix)
+        q, k, v = (H.to_dev(x, wl) for x in synth.suffix(wl))
+        res = []
+        for traced in (False, True, False):
+            c2kv.c2kv_profile_enable(ctx, traced)
+            out = torch.full_like(q, float("nan"))
+            lse = torch.full((wl.layers, 1, wl.n_q_heads, wl.n_suffix), float("nan"), device="cuda")
+            c2kv.c2kv_attend(ctx, cache, -1, q, k, v, wl.n_suffix, out, lse)
+            c2kv.c2kv_sync(ctx)
+            res.append((out, lse))
+        c2kv.c2kv_profile_enable(ctx, False)
+        prof = c2kv.c2kv_profile_read(ctx)
+        assert (prof["combine"][1] >= 1) == split
+        for o, l in res[1:]:
+            assert torch.equal(res[0][0], o) and torch.equal(res[0][1], l)
+        assert not torch.isnan(res[0][0]).any()
+        c2kv.c2kv_cache_release(ctx, cache)
+    finally:
+        c2kv.c2kv_destroy(ctx)
