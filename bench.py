@@ -638,6 +638,14 @@ def side_workload(name, steps, warmup, torch, c2kv, hbm, bf16, src, flush, with_
                 "cold_call_ms": round(compose_cold_ms, 5), "warm_call_ms": round(compose_warm_ms, 5),
                 "warm_gbs": round(warm_gbs, 1),
                 "traffic": captured_traffic("compose_kernel", name)}
+            if len(pool_ids) < len(ids):
+                # repeated chunks (Zipf draws): each distinct chunk's slots read once, every
+                # composed row written; reads of repeats can hit L2, so the algorithmic rate
+                # above may exceed HBM's
+                reads = wl.layers * wl.batch * f["slots"] * f["row_bytes"] * 2
+                uniq = wl.layers * len(pool_ids) * m * f["row_bytes"] * 2 + (f["compose_bytes"] - reads)
+                entry["compose"]["unique_chunk_bytes"] = uniq
+                entry["compose"]["unique_chunk_gbs"] = round(uniq / (kc / 1e3) / 1e9, 1)
             entry["suffix_kernel_ms"] = round(kern["suffix"][0], 5)
             entry["attention"] = {
                 "kernel_ms": round(ka, 5), "achieved_tflops": round(attn_tfs, 2),
@@ -896,6 +904,27 @@ def cpu_threads():
     return len(os.sched_getaffinity(0))
 
 
+def cpu_model():
+    """The host CPU as /proc/cpuinfo names it (x86: model name; Arm: implementer and part)."""
+    import platform
+    try:
+        with open("/proc/cpuinfo") as fh:
+            info = fh.read()
+    except OSError:
+        return platform.machine()
+    for line in info.splitlines():
+        if line.lower().startswith("model name"):
+            return line.split(":", 1)[1].strip()
+    fields = {}
+    for line in info.splitlines():
+        if ":" in line:
+            k, v = (x.strip() for x in line.split(":", 1))
+            fields.setdefault(k, v)
+    if "CPU part" in fields:
+        return f"{platform.machine()}, CPU implementer {fields.get('CPU implementer', '?')}, part {fields['CPU part']}"
+    return platform.machine()
+
+
 def oracle_sample(wl, layers, seed=0):
     """Time the oracle's compose + attend for `layers` layers of request 0's workload."""
     from oracle import c2kv_oracle as orc
@@ -943,7 +972,7 @@ def cpu_baseline(wl, budget_s=15.0, one_core_budget_s=8.0):
     per_layer_req = t / n
     step_s = per_layer_req * wl.layers * wl.batch
     out = {"value": round(f["positions"] / step_s, 1), "unit": "tokens/s",
-           "cores": cpu_threads(), "kind": "oracle",
+           "cores": cpu_threads(), "cpu": cpu_model(), "kind": "oracle",
            "sample": f"{n} (layer, request) compose+attend passes of the oracle (fp64 numpy), "
                      f"{t:.1f} s, scaled to {wl.layers} layers x {wl.batch} requests"}
     # one core: as many passes as fit in about one_core_budget_s at the all-core rate x 4
