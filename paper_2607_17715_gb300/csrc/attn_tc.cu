@@ -140,6 +140,7 @@ struct TcParams {                // CUtensorMap members carry their own alignmen
     int32_t pair_group;      // pairs a CTA runs in turn (1 with key-range splits or fused)
     float* part_o;
     float* part_lse;
+    uint32_t* tickets;       // null, or per-unit counters: the last split merges (plain kernel)
     ReqParam req[kMaxReq];
 };
 
@@ -335,6 +336,80 @@ __device__ __forceinline__ void sts128_(uint32_t a, const uint4& v) {
                  : "memory");
 }
 
+// Splits merged inside the kernel (TcParams::tickets).  Every split CTA of a (layer, request,
+// KV head, pair) unit writes its normalised fp32 partial and log2-domain lse, then both softmax
+// warpgroups meet (named barrier 4); one thread releases the partials (a GPU-scope fence) and
+// takes a ticket.  In the CTA that takes the last one, warpgroup A merges every row of the
+// pair as attn_combine_kernel does: 32 threads a row, 4 channels each, every split's lse and
+// output slice loaded before any is used; lse = log2 sum_s 2^lse_s,
+// O = sum_s 2^(lse_s - lse) O_s.  Then the counter goes back to zero for the next launch.  No
+// thread waits on another CTA.  At most kMaxMergeSplits splits (the host merges by launch
+// beyond that).
+__device__ __forceinline__ void split_merge(const TcParams& P, uint32_t sBar, int x, int r, int t0, int l,
+                                            int b, int hk) {
+    __threadfence();
+    asm volatile("bar.sync 4, 256;" ::: "memory");
+    const uint32_t sFlag = sBar + 8u * (uint32_t)NBAR + 8u;     // spare word after the barriers
+    const int n_groups = (int)(gridDim.x / P.n_split);
+    const int64_t unit = ((int64_t)blockIdx.z * gridDim.y + blockIdx.y) * n_groups + blockIdx.x / P.n_split;
+    if (x == 0 && r == 0) {
+        __threadfence();
+        const uint32_t t = atomicAdd(P.tickets + unit, 1u);
+        asm volatile("st.shared.u32 [%0], %1;" ::"r"(sFlag), "r"(t == (uint32_t)(P.n_split - 1) ? 1u : 0u) : "memory");
+    }
+    asm volatile("bar.sync 4, 256;" ::: "memory");
+    uint32_t last;
+    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(last) : "r"(sFlag) : "memory");
+    if (!last || x != 0) return;
+    __threadfence();                                 // the other splits' partials are visible
+    const int G = P.group, tq = P.tq;
+    const int t0a = t0, t0b = t0 + tq;               // (warpgroup A's tile is tile A)
+    const int rows_a = min(BM, (P.sq - t0a) * G);
+    const int rows_b = t0b < P.sq ? min(BM, (P.sq - t0b) * G) : 0;
+    const int64_t part_rows = (int64_t)P.lq * P.batch_total * P.sq * P.hq;
+    const int ns = P.n_split;
+#pragma unroll 1
+    for (int it = r; it < (rows_a + rows_b) * 32; it += BM) {
+        const int row = it >> 5, c4 = it & 31;
+        const int xr = row < rows_a ? 0 : 1, rr = row - xr * rows_a;
+        const int t = (xr ? t0b : t0a) + rr / G, g = rr - (rr / G) * G;
+        const int64_t row_id = (((int64_t)l * P.batch_total + b) * P.sq_pitch + t) * P.hq + hk * G + g;
+        const int64_t lse_id = (((int64_t)l * P.batch_total + b) * P.hq + hk * G + g) * P.sq_pitch + t;
+        float ls[kMaxMergeSplits];
+        float4 o[kMaxMergeSplits];
+#pragma unroll
+        for (int s = 0; s < kMaxMergeSplits; ++s) {
+            ls[s] = -CUDART_INF_F;
+            o[s] = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (s < ns) {
+                ls[s] = __ldcg(P.part_lse + (int64_t)s * part_rows + lse_id);
+                o[s] = __ldcg(reinterpret_cast<const float4*>(P.part_o + ((int64_t)s * part_rows + row_id) * HD) + c4);
+            }
+        }
+        float mx = -CUDART_INF_F;
+#pragma unroll
+        for (int s = 0; s < kMaxMergeSplits; ++s) mx = fmaxf(mx, ls[s]);
+        float wsum = 0.f;
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int s = 0; s < kMaxMergeSplits; ++s) {
+            const float w = ls[s] == -CUDART_INF_F ? 0.f : ex2(ls[s] - mx);
+            acc.x += w * o[s].x;
+            acc.y += w * o[s].y;
+            acc.z += w * o[s].z;
+            acc.w += w * o[s].w;
+            wsum += w;
+        }
+        const float inv = 1.0f / wsum;
+        uint2 pk;
+        pk.x = pack_bf16(acc.x * inv, acc.y * inv);
+        pk.y = pack_bf16(acc.z * inv, acc.w * inv);
+        *reinterpret_cast<uint2*>(static_cast<__nv_bfloat16*>(P.out) + row_id * HD + c4 * 4) = pk;
+        if (P.lse != nullptr && c4 == 0) P.lse[lse_id] = (mx + log2f(wsum)) * 0.69314718055994531f;
+    }
+    if (r == 0) P.tickets[unit] = 0u;
+}
+
 // The query tokens and key tiles of pair pr of query tiles (split sp of its key range).
 struct PairSpan {
     int t0a, t0b;       // first suffix token of tile A, of tile B
@@ -365,6 +440,8 @@ __device__ __forceinline__ PairSpan pair_span(const TcParams& P, int pr, int sp,
 // (no further Q will land there), else 0: O then leaves through it, the tile's rows written
 // in the 128-byte-swizzled layout and stored by TMA, instead of 16-byte stores of a row per
 // thread (which touch a separate cache line per thread).
+// kMerge: the plain kernel, whose split partials may be merged in the kernel (split_merge).
+template <bool kMerge>
 __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, uint32_t sBar, int x,
                                             int quad, int lane, int t0, int l, int bl, int b,
                                             int hk, int sp, int j_base, int n_kv, uint32_t sf_base,
@@ -564,6 +641,8 @@ __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, u
         }
         if (t < P.sq)
             P.part_lse[(int64_t)sp * part_rows + lse_id] = any ? m_run + log2f(l_run) : -CUDART_INF_F;
+        if constexpr (kMerge)
+            if (P.tickets != nullptr) split_merge(P, sBar, x, r, t0, l, b, hk);
     }
     if (arrive_oe) {          // O has been read out of TMEM: the next pair may overwrite it
         tc_fence_before();
@@ -1731,7 +1810,7 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
             fused_suffix_prep(KP, (int)threadIdx.x - 128, l, bl, hk, k_lo, k_hi, t0a, q_hi,
                               writer && P.layer0 + l == 0 && hk == 0, 0u, true, sQ, sBar, abort);
             if (x == 0 || has_b)
-                softmax_tile(P, tmem, sBar, x, warp & 3, lane, x ? t0b : t0a, l, bl, b, hk, sp, j_base,
+                softmax_tile<false>(P, tmem, sBar, x, warp & 3, lane, x ? t0b : t0a, l, bl, b, hk, sp, j_base,
                              n_kv, 0u, 0u, false, abort, sQ);
         } else if constexpr (kFused) {
             // per pair: the suffix preparation (the lead pair's also turns the suffix rows
@@ -1746,7 +1825,7 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
                                   pi == 0 && writer && P.layer0 + l == 0 && hk == 0, (uint32_t)pi & 1u,
                                   pi == 0, sQ, sBar, abort);
                 if (x == 0 || ps.has_b) {
-                    softmax_tile(P, tmem, sBar, x, warp & 3, lane, x ? ps.t0b : ps.t0a, l, bl, b, hk, sp,
+                    softmax_tile<false>(P, tmem, sBar, x, warp & 3, lane, x ? ps.t0b : ps.t0a, l, bl, b, hk, sp,
                                  ps.j_base, ps.n_kv, done, (uint32_t)pi & 1u, p_count > 1, abort,
                                  pi == p_count - 1 ? sQ : 0u);
                     done += (uint32_t)ps.n_kv;
@@ -1759,12 +1838,15 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
             for (int pi = 0; pi < p_count; ++pi) {
                 const PairSpan ps = pi == 0 ? ps0 : pair_span(P, p_first + pi, sp, s_r);
                 if (x == 0 || ps.has_b) {
-                    softmax_tile(P, tmem, sBar, x, warp & 3, lane, x ? ps.t0b : ps.t0a, l, bl, b, hk, sp,
+                    softmax_tile<true>(P, tmem, sBar, x, warp & 3, lane, x ? ps.t0b : ps.t0a, l, bl, b, hk, sp,
                                  ps.j_base, ps.n_kv, done, (uint32_t)pi & 1u, p_count > 1, abort,
                                  pi == p_count - 1 ? sQ : 0u);
                     done += (uint32_t)ps.n_kv;
                 } else if (p_count > 1) {    // no tile B in this pair: nothing of O to read
                     mbar_arrive(bar(B_OE));
+                } else if (P.tickets != nullptr) {   // a split without tile B: the merge's two
+                    asm volatile("bar.sync 4, 256;" ::: "memory");   // barriers (no rows, no
+                    asm volatile("bar.sync 4, 256;" ::: "memory");   // ticket of its own)
                 }
             }
         }
@@ -1969,6 +2051,7 @@ cudaError_t prepare_tc(const AttnParams& a, TcParams& p, dim3& grid) {
     p.n_split = a.n_split < 1 ? 1 : a.n_split;
     p.part_o = a.part_o;
     p.part_lse = a.part_lse;
+    p.tickets = kFused || p.n_split == 1 || p.n_split > kMaxMergeSplits ? nullptr : a.tickets;
     if (a.batch < 1 || a.batch > kMaxReq) return cudaErrorInvalidValue;
     std::memcpy(p.req, a.req, sizeof(ReqParam) * (size_t)a.batch);
     const int64_t pairs = ((a.sq + tq - 1) / tq + 1) / 2;

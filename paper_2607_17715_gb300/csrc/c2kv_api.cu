@@ -69,6 +69,10 @@ struct c2kv_ctx {
     int32_t inject = 0;
     int sms = 148;
     void* noalloc_scratch = nullptr;   // c2kv_attend_noalloc's fixed array on this device
+    // per-unit counters of the tensor-core attention's in-kernel split merge: zero between
+    // launches (each unit's last split sets its counter back), cleared again after a device error
+    uint32_t* tickets = nullptr;
+    size_t tickets_cap = 0;
     c2kv::RopeTurns turns{};
     // second stream and events of the pipelined compose + attend (host-resident chunks)
     cudaStream_t aux = nullptr;
@@ -109,6 +113,29 @@ cudaError_t pool_alloc(c2kv_ctx* c, void** p, size_t bytes) {
 
 void pool_free(c2kv_ctx* c, void* p) {
     if (p) cudaFreeAsync(p, c->stream);
+}
+
+// At least n zeroed split-merge counters (grown rarely: the old array may still be in use by
+// work on the stream, so the stream drains first).
+cudaError_t tickets_ready(c2kv_ctx* c, size_t n) {
+    if (n <= c->tickets_cap) return cudaSuccess;
+    const size_t cap = std::max<size_t>({n, 2 * c->tickets_cap, 4096});
+    cudaError_t e = cudaStreamSynchronize(c->stream);
+    if (e != cudaSuccess) return e;
+    if (c->tickets) cudaFree(c->tickets);
+    c->tickets = nullptr;
+    c->tickets_cap = 0;
+    void* p = nullptr;
+    e = cudaMalloc(&p, cap * sizeof(uint32_t));
+    // ordered on the context's stream, which need not synchronise with the legacy stream
+    if (e == cudaSuccess) e = cudaMemsetAsync(p, 0, cap * sizeof(uint32_t), c->stream);
+    if (e != cudaSuccess) {
+        if (p) cudaFree(p);
+        return e;
+    }
+    c->tickets = static_cast<uint32_t*>(p);
+    c->tickets_cap = cap;
+    return cudaSuccess;
 }
 
 // RoPE frequency i = theta^(-2i/d) as a fraction of a turn in 0.64 fixed point, from
@@ -339,6 +366,7 @@ c2kv_status c2kv_destroy(c2kv_ctx* c) {
         if (c->pool_k) cudaFree(c->pool_k);
         if (c->pool_v) cudaFree(c->pool_v);
         if (c->d_err) cudaFree(c->d_err);
+        if (c->tickets) cudaFree(c->tickets);
         delete c;
         return C2KV_OK;
     } catch (...) {
@@ -791,12 +819,18 @@ cudaError_t attend_run(c2kv_ctx* c, c2kv_cache* cache, int32_t layer0, int32_t l
             const size_t rows = (size_t)lq * B * n_suffix * c->cfg.n_q_heads;
             e = pool_alloc(c, reinterpret_cast<void**>(&part),
                            (size_t)n_split * rows * (c->cfg.head_dim + 1) * sizeof(float));
+            // the plain kernel merges the splits itself (per-unit counters)
+            if (e == cudaSuccess && !fused && n_split <= c2kv::kMaxMergeSplits)
+                e = tickets_ready(c, (size_t)c2kv::attn_tc_units(c->cfg.n_q_heads, c->cfg.n_kv_heads, n_suffix,
+                                                                 lq, std::min<int32_t>(B, c2kv::kMaxReq)));
             if (e != cudaSuccess) {
+                pool_free(c, part);
                 pool_free(c, q_rot_own);
                 return e;
             }
         }
     }
+    const bool merge_in_kernel = use_tc && !fused && n_split > 1 && n_split <= c2kv::kMaxMergeSplits;
     const size_t part_rows = (size_t)lq * B * n_suffix * c->cfg.n_q_heads;
     c2kv::AttnParams last{};
     for (int32_t b0 = 0; e == cudaSuccess && b0 < B; b0 += c2kv::kMaxReq) {
@@ -823,6 +857,7 @@ cudaError_t attend_run(c2kv_ctx* c, c2kv_cache* cache, int32_t layer0, int32_t l
         a.pairs_per_cta = c->cfg.attn_pairs;
         a.part_o = part;
         a.part_lse = part ? part + (size_t)n_split * part_rows * c->cfg.head_dim : nullptr;
+        a.tickets = merge_in_kernel ? c->tickets : nullptr;
         for (int32_t i = 0; i < nb; ++i) a.req[i] = s.req[i];
         if (fused) {
             e = c2kv::prepare_attn_fused(a, *fused);
@@ -845,7 +880,7 @@ cudaError_t attend_run(c2kv_ctx* c, c2kv_cache* cache, int32_t layer0, int32_t l
         last = a;
         last.dependent = !c->prof && !fused && use_tc ? 1 : 0;   // the merge: the attention's dependent
     }
-    if (e == cudaSuccess && n_split > 1) {   // one merge over every request's rows
+    if (e == cudaSuccess && n_split > 1 && !merge_in_kernel) {   // one merge over every request's rows
         ProfScope prof_combine(c, C2KV_PROF_COMBINE);
         e = c2kv::launch_attn_combine(last, c->stream);
     }
@@ -1314,7 +1349,11 @@ c2kv_status c2kv_decode(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
         const size_t rows_all = (size_t)lq * B * hq;
         if (n_split > 1) {
             e = pool_alloc(c, reinterpret_cast<void**>(&part), (size_t)n_split * rows_all * (d + 1) * sizeof(float));
+            // the tensor-core kernel merges the splits itself (per-unit counters)
+            if (e == cudaSuccess && use_tc && n_split <= c2kv::kMaxMergeSplits)
+                e = tickets_ready(c, (size_t)c2kv::attn_tc_units(hq, hkv, 1, lq, std::min<int32_t>(B, c2kv::kMaxReq)));
             if (e != cudaSuccess) {
+                pool_free(c, part);
                 pool_free(c, q_rot);
                 return cuda_fail(c, e, "decode: split scratch allocation");
             }
@@ -1388,14 +1427,18 @@ c2kv_status c2kv_decode(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
                 a.pairs_per_cta = c->cfg.attn_pairs;
                 a.part_o = part;
                 a.part_lse = part ? part + (size_t)n_split * rows_all * d : nullptr;
-                // the suffix kernel's programmatic dependent, and the merge the attention's,
-                // unless a trace puts events between them
+                // the splits merged in the kernel (beyond kMaxMergeSplits: by a launch after the
+                // last group)
+                const bool in_kernel = n_split > 1 && n_split <= c2kv::kMaxMergeSplits;
+                a.tickets = in_kernel ? c->tickets : nullptr;
+                // the suffix kernel's programmatic dependent, unless a trace puts events
+                // between them
                 a.dependent = c->prof ? 0 : 1;
                 for (int32_t i = 0; i < nb; ++i) a.req[i] = reqs[b0 + i];
                 ProfScope prof_decode(c, C2KV_PROF_DECODE, true);
                 e = c2kv::launch_attn_tc(a, c->stream, prof_decode.hook());
-                // the merge of the splits over every request's rows, after the last group
-                if (e == cudaSuccess && n_split > 1 && b0 + nb >= B) e = c2kv::launch_attn_combine(a, c->stream);
+                if (e == cudaSuccess && n_split > 1 && !in_kernel && b0 + nb >= B)
+                    e = c2kv::launch_attn_combine(a, c->stream);
                 continue;
             }
             c2kv::DecodeParams p{};
@@ -1529,6 +1572,8 @@ c2kv_status c2kv_sync(c2kv_ctx* c) {
     if (e != cudaSuccess) return cuda_fail(c, e, "sync: error word");
     if (word != 0) {
         cudaMemset(c->d_err, 0, sizeof(int32_t));
+        // a launch that gave up may have left split-merge counters part-way
+        if (c->tickets) cudaMemsetAsync(c->tickets, 0, c->tickets_cap * sizeof(uint32_t), c->stream);
         return fail(c, C2KV_ERR_DEVICE_BOUNDS, "sync: a kernel refused an out-of-range index (flags 0x%x)", word);
     }
     return C2KV_OK;

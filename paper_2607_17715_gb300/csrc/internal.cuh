@@ -18,6 +18,7 @@ constexpr int kDtypeF32 = 1;
 constexpr int kMaxHalf = 64;        // head_dim / 2 for head_dim <= 128
 constexpr int kMaxOcc = 512;        // chunk occurrences per compose launch (24 KB of parameters)
 constexpr int kMaxReq = 256;        // requests per suffix / attention launch
+constexpr int kMaxMergeSplits = 16; // key-range splits the tensor-core kernel merges itself
 constexpr int kComposeTile = 16;    // most composed slots per compose tile (per layer)
 constexpr int kComposeBulkTile = 32;   // most slots per tile of the bulk-copy compose kernel
 
@@ -149,6 +150,10 @@ struct AttnParams {
     int32_t dependent;       // tensor-core kernel and its merge: launched as the programmatic
                              // dependent of the kernel before them on the stream (each waits
                              // for that grid before it reads memory)
+    uint32_t* tickets;       // tensor-core kernel with n_split > 1: null (attn_combine_kernel
+                             // merges), or one zeroed counter per (layer, request, KV head,
+                             // pair): the unit's last split merges the partials in the kernel
+                             // and sets it back to zero
     ReqParam req[kMaxReq];
 };
 
