@@ -345,7 +345,8 @@ c2kv_status c2kv_attend_noalloc(c2kv_ctx* ctx, c2kv_cache* cache, int32_t layer,
  * q, k_new, v_new, out and lse must be device (or managed) memory: anything else is
  * refused with ERR_ARG before anything is enqueued.
  * The key range of each (layer, request, KV head) is split over several CTAs and merged
- * exactly (log-sum-exp); the split buffer comes from the context's memory pool.  With bf16
+ * exactly (log-sum-exp; on the tensor-core route by the last split of each unit, inside the
+ * kernel); the split buffer comes from the context's memory pool.  With bf16
  * and d = 128 the step runs on the tensor-core attention kernel (the new token as a one-row
  * query tile) when (layers x requests x KV heads) fits one CTA per SM or a request holds
  * 4096 keys or more, else on a CUDA-core decode kernel (C2KV_ATTN_TC forces the former,
