@@ -512,6 +512,42 @@ def decode_line(wl, world, dec_ms, dec_kernel_ms, dec_keys, hbm, src):
     }
 
 
+def long_decode(torch, c2kv, hbm, src, flush, keys=131072, steps=5, warmup=3):
+    """Decode at the top of the paper's 16k-128k context range: one request whose composed
+    cache holds `keys` slots (64 chunks x 2048 tokens at k = 1, Llama-3-8B layer shape, one
+    layer), its stored slots drawn on the device; `steps` timed decode steps after a short
+    suffix, L2 flushed before each; the kernel from the library's trace against HBM."""
+    base = synth.workload("sweep_k1")
+    chunks = keys // base.chunk_tokens
+    wl = synth.scaled(base, layers=1, batch=1, chunks_per_request=chunks, pool_chunks=chunks,
+                      n_suffix=4)
+    stream = torch.cuda.current_stream()
+    m = wl.chunk_tokens
+    ctx = c2kv.c2kv_create(1, wl.n_q_heads, wl.n_kv_heads, wl.head_dim, wl.rope_theta,
+                           c2kv.DTYPE_BF16, pool_slots=chunks * m + 64, stream=stream)
+    try:
+        gen = torch.Generator(device="cuda").manual_seed(7)
+        shape = (1, m, wl.n_kv_heads, wl.head_dim)
+        ids = []
+        for _ in range(chunks):
+            kd = torch.randn(shape, device="cuda", generator=gen).to(torch.bfloat16)
+            vd = torch.randn(shape, device="cuda", generator=gen).to(torch.bfloat16)
+            ids.append(c2kv.c2kv_compress_chunk(ctx, kd, vd, wl.chunk_tokens, 1, c2kv.MODE_STORED))
+        q_dev = [torch.randn((1, 1, wl.n_suffix, h, wl.head_dim), device="cuda", generator=gen)
+                 .to(torch.bfloat16) for h in (wl.n_q_heads, wl.n_kv_heads, wl.n_kv_heads)]
+        out = torch.empty_like(q_dev[0])
+        events = [[torch.cuda.Event(enable_timing=True) for _ in range(2)] for _ in range(steps)]
+        ms, kern_ms, kv, per = decode_measure(c2kv, torch, ctx, wl, stream, np.array([0, chunks], np.int32),
+                                              ids, None, q_dev, out, steps, warmup, events, flush)
+        line = decode_line(wl, 1, statistics.median(per), kern_ms, kv, hbm, src)
+        line["what"] = (f"one request over a composed cache of {keys} keys (the paper's 16k-128k "
+                        "decode range), Llama-3-8B layer shape, one layer; " + line["what"])
+        line["roofline"]["kernel"] = "attn_tc_kernel (one-row suffix, splits merged in the kernel)"
+        return line
+    finally:
+        c2kv.c2kv_destroy(ctx)
+
+
 # --------------------------------------------------------------------------- other workloads
 
 SIDE_WORKLOADS = ("batched", "long70b", "sweep_k1", "sweep_k4", "sweep_k8", "sweep_k10", "sweep_k16")
@@ -880,6 +916,9 @@ def run_ours(args):
         "gpu_launches": sum(v[1] for v in kern.values()),
         "clocks": clk,
     }
+    if not args.no_long_decode:
+        # decode over a 128k-key composed cache (one layer)
+        line["decode_long"] = long_decode(torch, c2kv, hbm, src, arm.flush_l2)
     if workloads:
         # configs 3-5 (batched reuse, long context, the compression-ratio sweep with its
         # uncompressed control), each run once at full size in the same process
@@ -1038,6 +1077,8 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="llama8b", choices=sorted(synth.WORKLOADS))
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-long-decode", action="store_true",
+                    help="skip the decode leg over a 128k-key cache")
     ap.add_argument("--cpu-budget", type=float, default=15.0)
     ap.add_argument("--attn-split", type=int, default=0,
                     help="key-range splits of the attention (0 = library's choice)")

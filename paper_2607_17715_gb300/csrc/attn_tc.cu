@@ -340,8 +340,8 @@ __device__ __forceinline__ void sts128_(uint32_t a, const uint4& v) {
 // KV head, pair) unit writes its normalised fp32 partial and log2-domain lse, then both softmax
 // warpgroups meet (named barrier 4); one thread releases the partials (a GPU-scope fence) and
 // takes a ticket.  In the CTA that takes the last one, warpgroup A merges every row of the
-// pair as attn_combine_kernel does: 32 threads a row, 4 channels each, every split's lse and
-// output slice loaded before any is used; lse = log2 sum_s 2^lse_s,
+// pair as attn_combine_kernel does: 32 threads a row, 4 channels each, eight splits' lse and
+// output slices loaded before any is used; lse = log2 sum_s 2^lse_s,
 // O = sum_s 2^(lse_s - lse) O_s.  Then the counter goes back to zero for the next launch.  No
 // thread waits on another CTA.  At most kMaxMergeSplits splits (the host merges by launch
 // beyond that).
@@ -375,30 +375,38 @@ __device__ __forceinline__ void split_merge(const TcParams& P, uint32_t sBar, in
         const int t = (xr ? t0b : t0a) + rr / G, g = rr - (rr / G) * G;
         const int64_t row_id = (((int64_t)l * P.batch_total + b) * P.sq_pitch + t) * P.hq + hk * G + g;
         const int64_t lse_id = (((int64_t)l * P.batch_total + b) * P.hq + hk * G + g) * P.sq_pitch + t;
-        float ls[kMaxMergeSplits];
-        float4 o[kMaxMergeSplits];
-#pragma unroll
-        for (int s = 0; s < kMaxMergeSplits; ++s) {
-            ls[s] = -CUDART_INF_F;
-            o[s] = make_float4(0.f, 0.f, 0.f, 0.f);
-            if (s < ns) {
-                ls[s] = __ldcg(P.part_lse + (int64_t)s * part_rows + lse_id);
-                o[s] = __ldcg(reinterpret_cast<const float4*>(P.part_o + ((int64_t)s * part_rows + row_id) * HD) + c4);
-            }
-        }
+        constexpr int SB = 8;                        // splits in flight together
         float mx = -CUDART_INF_F;
+#pragma unroll 1
+        for (int s0 = 0; s0 < ns; s0 += SB) {
 #pragma unroll
-        for (int s = 0; s < kMaxMergeSplits; ++s) mx = fmaxf(mx, ls[s]);
+            for (int s = s0; s < s0 + SB; ++s)
+                if (s < ns) mx = fmaxf(mx, __ldcg(P.part_lse + (int64_t)s * part_rows + lse_id));
+        }
         float wsum = 0.f;
         float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 1
+        for (int s0 = 0; s0 < ns; s0 += SB) {
+            float ls[SB];
+            float4 o[SB];
 #pragma unroll
-        for (int s = 0; s < kMaxMergeSplits; ++s) {
-            const float w = ls[s] == -CUDART_INF_F ? 0.f : ex2(ls[s] - mx);
-            acc.x += w * o[s].x;
-            acc.y += w * o[s].y;
-            acc.z += w * o[s].z;
-            acc.w += w * o[s].w;
-            wsum += w;
+            for (int i = 0; i < SB; ++i) {
+                ls[i] = -CUDART_INF_F;
+                o[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+                if (s0 + i < ns) {
+                    ls[i] = __ldcg(P.part_lse + (int64_t)(s0 + i) * part_rows + lse_id);
+                    o[i] = __ldcg(reinterpret_cast<const float4*>(P.part_o + ((int64_t)(s0 + i) * part_rows + row_id) * HD) + c4);
+                }
+            }
+#pragma unroll
+            for (int i = 0; i < SB; ++i) {
+                const float w = ls[i] == -CUDART_INF_F ? 0.f : ex2(ls[i] - mx);
+                acc.x += w * o[i].x;
+                acc.y += w * o[i].y;
+                acc.z += w * o[i].z;
+                acc.w += w * o[i].w;
+                wsum += w;
+            }
         }
         const float inv = 1.0f / wsum;
         uint2 pk;

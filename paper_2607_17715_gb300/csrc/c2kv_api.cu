@@ -1307,7 +1307,7 @@ c2kv_status c2kv_decode(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
                 n_split = (int32_t)std::min<int64_t>(c->cfg.attn_split, tiles);
             } else {
                 double best = 0.0;
-                for (int32_t n = 1; n <= 16 && n <= tiles; ++n) {
+                for (int32_t n = 1; n <= c2kv::kMaxMergeSplits && n <= tiles; ++n) {
                     const int64_t waves = (units * n + c->sms - 1) / c->sms;
                     const double t = (double)waves * ((double)((tiles + n - 1) / n) + 4.0) + (n > 1 ? 2.0 : 0.0);
                     if (n == 1 || t < best) {

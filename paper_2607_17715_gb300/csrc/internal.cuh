@@ -18,7 +18,7 @@ constexpr int kDtypeF32 = 1;
 constexpr int kMaxHalf = 64;        // head_dim / 2 for head_dim <= 128
 constexpr int kMaxOcc = 512;        // chunk occurrences per compose launch (24 KB of parameters)
 constexpr int kMaxReq = 256;        // requests per suffix / attention launch
-constexpr int kMaxMergeSplits = 16; // key-range splits the tensor-core kernel merges itself
+constexpr int kMaxMergeSplits = 32; // key-range splits the tensor-core kernel merges itself
 constexpr int kComposeTile = 16;    // most composed slots per compose tile (per layer)
 constexpr int kComposeBulkTile = 32;   // most slots per tile of the bulk-copy compose kernel
 
