@@ -87,15 +87,18 @@ constexpr int kRegsLow = 136;
 constexpr int kRegsHigh = 184;
 static_assert(128 * kRegsLow + 256 * kRegsHigh <= kThreads * kLaunchRegs, "register split");
 // Fused: 512 threads launch with 128 registers each; the producer/issuer warpgroup and the
-// loader warpgroup keep 88 (fewer spills there measured faster than more registers for the
-// softmax), the softmax warpgroups rise to 168.
+// K-loader warpgroup keep 96 each, the softmax warpgroups rise to 160.  (88 / 88 / 168 spilled
+// in the first two and measured 7 % slower on the 32-layer step; 88 / 104 / 160 and
+// 104 / 104 / 152 fell between.)
 constexpr int kThreadsFused = 512;
 constexpr int kLaunchRegsFused = 128;
-constexpr int kRegsLowFused = 88;
-constexpr int kRegsHighFused = 168;
+constexpr int kRegsLowFused = 96;       // warps 0..3
+constexpr int kRegsLoadFused = 96;      // warps 12..15
+constexpr int kRegsHighFused = 160;     // warps 4..11
 constexpr int kLoaders = 128;       // K loaders (warps 12..15)
 constexpr int kVLoaders = 32;       // V loader (warp 3)
-static_assert(256 * kRegsLowFused + 256 * kRegsHighFused <= kThreadsFused * kLaunchRegsFused,
+static_assert(128 * kRegsLowFused + 128 * kRegsLoadFused + 256 * kRegsHighFused <=
+                  kThreadsFused * kLaunchRegsFused,
               "fused register split");
 constexpr uint32_t kTmemCols = 512;     // S_A, S_B, O_A, O_B; P_x over the first half of S_x
 constexpr uint32_t kColS = 0, kColO = 256;
@@ -587,7 +590,9 @@ __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, u
             tma_store_4d(&P.tm_o, sbase, 0, hk * G, t0, qz);
             tma_store_4d(&P.tm_o, sbase + HALF_TILE, 64, hk * G, t0, qz);
             asm volatile("cp.async.bulk.commit_group;" ::: "memory");
-            asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+            // the CTA may leave once the store has read shared memory; its writes complete
+            // with the grid
+            asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
         }
         return;
     }
@@ -1327,7 +1332,7 @@ __device__ __forceinline__ void fused_k_loader(const FusedTcParams& F, int lt, i
 // handed back to the producer as soon as its store has read it.
 __device__ __forceinline__ void fused_writer(const FusedTcParams& F, int l, int bl, int hk, int j_base,
                                              int n_kv, uint32_t sK, uint32_t sV, uint32_t sBar,
-                                             volatile uint32_t* abort) {
+                                             bool more_pairs, volatile uint32_t* abort) {
     const TcParams& P = F.t;
     auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
     const int cache_row0 = (int)((int64_t)(P.layer0 + l) * P.rows + P.req[bl].row_base);
@@ -1343,8 +1348,12 @@ __device__ __forceinline__ void fused_writer(const FusedTcParams& F, int l, int 
         asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");    // V's
         mbar_arrive(bar(B_VW + vs));
     }
-    asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
-    mbar_arrive(bar(B_WD));     // the composed cache is written: later pairs may read it
+    if (more_pairs) {
+        asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+        mbar_arrive(bar(B_WD));     // the composed cache is written: later pairs may read it
+    }
+    // otherwise nothing in this CTA reads the cache back: the stores have read shared memory
+    // (above), and their writes complete with the grid
 }
 
 // The V loader of the fused kernel (warp 3, lt = 0..31): per key tile, the ragged 8-row
@@ -1800,7 +1809,8 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
             }
         } else if (warp == 2 && lane == 0 && n_kv > 0 && writer) {
             // ------------------------------------------------------------ writer (fused)
-            if constexpr (kFused) fused_writer(KP, l, bl, hk, j_base, n_kv, sK, sV, sBar, abort);
+            if constexpr (kFused)
+                fused_writer(KP, l, bl, hk, j_base, n_kv, sK, sV, sBar, kMulti && p_count > 1, abort);
         } else if (warp == 3 && n_kv > 0) {
             // ------------------------------------------------------------ V loader (fused)
             if constexpr (kFused)
@@ -1860,7 +1870,7 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
         }
     } else {
         if constexpr (kFused) {
-            asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsLowFused));
+            asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(kRegsLoadFused));
             // ------------------------------------------------------------ loaders (fused)
             if (n_kv > 0)
                 fused_k_loader(KP, (int)threadIdx.x - 12 * 32, l, bl, hk, writer, j_base, n_kv,
@@ -2002,9 +2012,8 @@ namespace {
 template <bool kFused, bool kMulti = false>
 cudaError_t prepare_tc(const AttnParams& a, TcParams& p, dim3& grid) {
     constexpr int threads = kFused ? kThreadsFused : kThreads;
-    constexpr int low = kFused ? kRegsLowFused : kRegsLow;
     constexpr int high = kFused ? kRegsHighFused : kRegsHigh;
-    constexpr int low_threads = kFused ? 256 : 128;
+    constexpr int low_total = kFused ? 128 * (kRegsLowFused + kRegsLoadFused) : 128 * kRegsLow;
     // once per process (one device per context; function-local statics: thread-safe)
     static const cudaError_t smem_err = cudaFuncSetAttribute(
         attn_tc_kernel<kFused, kMulti>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
@@ -2015,7 +2024,7 @@ cudaError_t prepare_tc(const AttnParams& a, TcParams& p, dim3& grid) {
             return cudaFuncGetAttributes(&fa, attn_tc_kernel<kFused, kMulti>) == cudaSuccess ? fa.numRegs : -1;
         }();
         if (launch_regs < 0) return cudaErrorInvalidDeviceFunction;
-        if (launch_regs * threads < low_threads * low + 256 * high) return cudaErrorInvalidConfiguration;
+        if (launch_regs * threads < low_total + 256 * high) return cudaErrorInvalidConfiguration;
     }
     const int pitch = a.sq_pitch > 0 ? a.sq_pitch : a.sq;
     if (pitch < a.sq || (pitch != a.sq && a.n_split > 1)) return cudaErrorInvalidValue;

@@ -296,9 +296,9 @@ __global__ void __launch_bounds__(kBulkThreads, 1)
             }
         }
         // after an abort: loads in flight land before the CTA leaves; then every store has
-        // completed
+        // read shared memory (their writes complete with the grid)
         for (int i = stored; i < issued; ++i) mbar_wait_limit(full_bar(i % nst), (uint32_t)(i / nst) & 1u);
-        asm volatile("cp.async.bulk.wait_group 0;" ::: "memory");
+        asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
         return;
     }
 
