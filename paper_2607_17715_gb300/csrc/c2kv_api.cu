@@ -635,9 +635,10 @@ int32_t compose_tile_slots(const c2kv_ctx* c, int64_t slots, int32_t n_layers, i
 
 // Slots per tile of the bulk-copy compose kernel: at most 16 KB of K rows (the stage then
 // holds 32 KB of K and V, six of them in flight per SM), halved while the launch would give
-// fewer than four tiles per SM, so that a small launch still spreads evenly over the SMs
-// (each tile costs its CTA about a microsecond of fixed work, so smaller tiles than that
-// lose more than they balance).
+// fewer than two tiles per SM, so that a small launch still spreads over the SMs (each tile
+// costs its CTA about a microsecond of fixed work, so smaller tiles than that lose more than
+// they balance: on the one-layer long70b shape, 8-slot tiles took 14.8-15.1 us against
+// 15.7-15.8 us for 4-slot ones, and a threshold of eight tiles per SM 18.7 us).
 int32_t compose_bulk_tile_slots(const c2kv_ctx* c, const std::vector<c2kv::OccParam>& occ, int32_t g0,
                                 int32_t g1, int32_t n_layers) {
     const int64_t row_bytes = (int64_t)c->cfg.n_kv_heads * c->cfg.head_dim * c->eb;
@@ -648,7 +649,7 @@ int32_t compose_bulk_tile_slots(const c2kv_ctx* c, const std::vector<c2kv::OccPa
         for (int32_t i = g0; i < g1; ++i) n += (occ[i].m + ts - 1) / ts;
         return n * n_layers;
     };
-    while (t > 1 && tiles(t) < 4LL * c->sms) t /= 2;
+    while (t > 1 && tiles(t) < 2LL * c->sms) t /= 2;
     return t;
 }
 
