@@ -481,7 +481,7 @@ def extract_line(wl, world, ms, kernel_ms, hbm, bf16, src):
                 "L2 flushed before each call (untimed)",
         "kernel_ms": round(kernel_ms, 5) if kernel_ms else None,
         "roofline": {"bound": "tensor" if tensor else "hbm",
-                     "kernel": "extraction call (extract_rope_kernel, attn_tc_kernel x2, extract_local_kernel)",
+                     "kernel": "extraction call (extract_rope_kernel, attn_tc_kernel x2)",
                      "achieved": round(tfs, 2) if tensor else round(gbs, 1),
                      "peak": bf16 if tensor else hbm, "unit": "TFLOP/s" if tensor else "GB/s",
                      "frac": round(tfs / bf16 if tensor else gbs / hbm, 4),

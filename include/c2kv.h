@@ -375,7 +375,7 @@ c2kv_status c2kv_decode(c2kv_ctx* ctx, c2kv_cache* cache, int32_t layer, const v
  * The sink block, B(0) in the paper's 1-based numbering, is read as the first block
  * [0, min(k, n)).  The trained C2 embeddings and QKV projections that produce q, k, v for
  * the C2 tokens are the caller's; this is the attention operator they feed.  On the
- * tensor-core route (bf16, d 128) the C2 rows' launches run on the context's second stream
+ * tensor-core route (bf16, d 128) the C2 rows' launch runs on the context's second stream
  * beside the document rows' attention; the call's work ends on the context's stream.
  *
  *   n_layers : layers in the tensors (each processed independently).

@@ -144,6 +144,7 @@ struct TcParams {                // CUtensorMap members carry their own alignmen
     float* part_o;
     float* part_lse;
     uint32_t* tickets;       // null, or per-unit counters: the last split merges (plain kernel)
+    int32_t sif_k;           // 0, or extraction C2 rows with ratio k (plain kernel, one split)
     ReqParam req[kMaxReq];
 };
 
@@ -421,23 +422,50 @@ __device__ __forceinline__ void split_merge(const TcParams& P, uint32_t sBar, in
     if (r == 0) P.tickets[unit] = 0u;
 }
 
-// The query tokens and key tiles of pair pr of query tiles (split sp of its key range).
+// The query tokens and key tiles of pair pr of query tiles (split sp of its key range).  The
+// key tiles are, in order: tile 0 if lead0, then n_mid tiles from j_base, then the rest from
+// j_tail; a plain pair's are the n_kv tiles from j_base (lead0 = false, n_mid = n_kv).
 struct PairSpan {
     int t0a, t0b;       // first suffix token of tile A, of tile B
     bool has_b;
     int t_last;         // last suffix token of the pair
-    int j_base, n_kv;   // this split's key tiles: [j_base, j_base + n_kv)
+    int j_base, n_kv;   // this split's key tiles: n_kv of them, the first run from j_base
+    bool lead0;
+    int n_mid, j_tail;
 };
+// Key tile of the pair's i-th key tile.
+__device__ __forceinline__ int span_tile(const PairSpan& o, int i) {
+    const int i1 = i - (o.lead0 ? 1 : 0);
+    return i1 < 0 ? 0 : i1 < o.n_mid ? o.j_base + i1 : o.j_tail + (i1 - o.n_mid);
+}
 __device__ __forceinline__ PairSpan pair_span(const TcParams& P, int pr, int sp, int s_r) {
     PairSpan o;
     o.t0a = 2 * pr * P.tq;
     o.t0b = o.t0a + P.tq;
     o.has_b = o.t0b < P.sq;
     o.t_last = min(P.sq - 1, (o.has_b ? o.t0b : o.t0a) + P.tq - 1);
+    o.lead0 = false;
+    if (P.sif_k > 0) {
+        // extraction C2 rows c_j, j in [t0a, t_last], over a chunk of n = s_r document keys:
+        // the tiles of their blocks' document keys, tile 0 (the sink block) if not among
+        // them, then the tiles of the C2 keys c_0 .. c_{t_last} at rows n .. n + t_last not
+        // already taken (every C2 block holds at least one document token, jk < n)
+        const int k = P.sif_k, n = s_r;
+        const int b0 = (o.t0a * k) / BN, b1 = (min((o.t_last + 1) * k, n) - 1) / BN;
+        const int c0 = max(n / BN, b1 + 1), c1 = (n + o.t_last) / BN;
+        o.lead0 = b0 > 0;
+        o.j_base = b0;
+        o.n_mid = b1 - b0 + 1;
+        o.j_tail = c0;
+        o.n_kv = (o.lead0 ? 1 : 0) + o.n_mid + max(0, c1 - c0 + 1);
+        return o;
+    }
     const int n_kv_all = (s_r + o.t_last + 1 + BN - 1) / BN;
     const int per_split = (n_kv_all + P.n_split - 1) / P.n_split;
     o.j_base = sp * per_split;
     o.n_kv = max(0, min(n_kv_all, o.j_base + per_split) - o.j_base);
+    o.n_mid = o.n_kv;
+    o.j_tail = o.j_base + o.n_kv;
     return o;
 }
 
@@ -455,7 +483,7 @@ __device__ __forceinline__ PairSpan pair_span(const TcParams& P, int pr, int sp,
 template <bool kMerge>
 __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, uint32_t sBar, int x,
                                             int quad, int lane, int t0, int l, int bl, int b,
-                                            int hk, int sp, int j_base, int n_kv, uint32_t sf_base,
+                                            int hk, int sp, const PairSpan& span, uint32_t sf_base,
                                             uint32_t od_par, bool arrive_oe,
                                             volatile uint32_t* abort, uint32_t stage = 0u) {
     auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
@@ -470,6 +498,7 @@ __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, u
     const int t_row = min(t0 + r / G, P.sq - 1);    // rows past the suffix mirror its end
     const int lim = s_r + t_row;                    // last key this row may see
     const float sc = P.scale_log2;
+    const int n_kv = span.n_kv;
     float m_run = -CUDART_INF_F;
     float l_run = 0.f;
 
@@ -481,13 +510,29 @@ __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, u
         for (int c = 0; c < 4; ++c) tmem_ld32(tmem + lane_addr + colS + c * 32, sv[c]);
         tmem_ld_wait();
 
-        const int kbase = (j_base + j) * BN;
+        const int kbase = (kMerge ? span_tile(span, j) : span.j_base + j) * BN;   // (SIF: plain only)
         if (kbase + BN - 1 > lim) {
 #pragma unroll
             for (int c = 0; c < 4; ++c)
 #pragma unroll
                 for (int e = 0; e < 32; ++e)
                     if (kbase + c * 32 + e > lim) sv[c][e] = __float_as_uint(-CUDART_INF_F);
+        }
+        if constexpr (kMerge) {
+            // extraction C2 row c_{t_row}: of the document keys (rows below s_r) it sees the
+            // sink block [0, min(k, n)) and its own block [t_row k, min((t_row + 1) k, n))
+            if (P.sif_k > 0 && kbase < s_r) {
+                const int sink = min(P.sif_k, s_r);
+                const int blo = t_row * P.sif_k, bhi = min(blo + P.sif_k, s_r);
+#pragma unroll
+                for (int c = 0; c < 4; ++c)
+#pragma unroll
+                    for (int e = 0; e < 32; ++e) {
+                        const int key = kbase + c * 32 + e;
+                        if (key < s_r && key >= sink && (key < blo || key >= bhi))
+                            sv[c][e] = __float_as_uint(-CUDART_INF_F);
+                    }
+            }
         }
         // row max: three-input maxima, one chain per 32-column chunk
         float mx4[4];
@@ -1070,7 +1115,7 @@ __device__ __noinline__ void fused_rest_producer(const FusedTcParams& F, int l, 
         }
         if (stored && pk < p_count && k_free(gk)) {
             const int st = gk % KSTAGES;
-            const int row = key0 + (sk.j_base + jk) * BN;
+            const int row = key0 + span_tile(sk, jk) * BN;
             mbar_expect_tx(bar(B_KL + st), TILE);
             tma_load_3d(sK + (uint32_t)(st * TILE), &P.tm_k, 0, hk, row, bar(B_KL + st));
             tma_load_3d(sK + (uint32_t)(st * TILE) + HALF_TILE, &P.tm_k, 64, hk, row, bar(B_KL + st));
@@ -1084,7 +1129,7 @@ __device__ __noinline__ void fused_rest_producer(const FusedTcParams& F, int l, 
         }
         if (stored && pv < p_count && v_free(gv)) {
             const int st = gv % VSTAGES;
-            const int row = key0 + (sv.j_base + jv) * BN;
+            const int row = key0 + span_tile(sv, jv) * BN;
             mbar_expect_tx(bar(B_VL + st), TILE);
             tma_load_3d(sV + (uint32_t)(st * TILE), &P.tm_v, 0, hk, row, bar(B_VL + st));
             tma_load_3d(sV + (uint32_t)(st * TILE) + HALF_TILE, &P.tm_v, 64, hk, row, bar(B_VL + st));
@@ -1597,7 +1642,7 @@ __device__ __forceinline__ void plain_producer(const TcParams& P, int l, int bl,
         if (pk < p_count && (gk < KSTAGES || mbar_test(bar(B_KE + gk % KSTAGES),
                                                        (uint32_t)((gk / KSTAGES) - 1) & 1u))) {
             const int s = gk % KSTAGES;
-            const int krow = key0 + (sk.j_base + jk) * BN;
+            const int krow = key0 + span_tile(sk, jk) * BN;
             mbar_expect_tx(bar(B_KF + s), TILE);
             tma_load_3d(sK + s * TILE, &P.tm_k, 0, hk, krow, bar(B_KF + s));
             tma_load_3d(sK + s * TILE + HALF_TILE, &P.tm_k, 64, hk, krow, bar(B_KF + s));
@@ -1612,7 +1657,7 @@ __device__ __forceinline__ void plain_producer(const TcParams& P, int l, int bl,
         if (pv < p_count && (gv < VSTAGES || mbar_test(bar(B_VE + gv % VSTAGES),
                                                        (uint32_t)((gv / VSTAGES) - 1) & 1u))) {
             const int s = gv % VSTAGES;
-            const int vrow = key0 + (sv.j_base + jv) * BN;
+            const int vrow = key0 + span_tile(sv, jv) * BN;
             mbar_expect_tx(bar(B_VF + s), TILE);
             tma_load_3d(sV + s * TILE, &P.tm_v, 0, hk, vrow, bar(B_VF + s));
             tma_load_3d(sV + s * TILE + HALF_TILE, &P.tm_v, 64, hk, vrow, bar(B_VF + s));
@@ -1828,8 +1873,8 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
             fused_suffix_prep(KP, (int)threadIdx.x - 128, l, bl, hk, k_lo, k_hi, t0a, q_hi,
                               writer && P.layer0 + l == 0 && hk == 0, 0u, true, sQ, sBar, abort);
             if (x == 0 || has_b)
-                softmax_tile<false>(P, tmem, sBar, x, warp & 3, lane, x ? t0b : t0a, l, bl, b, hk, sp, j_base,
-                             n_kv, 0u, 0u, false, abort, sQ);
+                softmax_tile<false>(P, tmem, sBar, x, warp & 3, lane, x ? t0b : t0a, l, bl, b, hk, sp, ps0,
+                             0u, 0u, false, abort, sQ);
         } else if constexpr (kFused) {
             // per pair: the suffix preparation (the lead pair's also turns the suffix rows
             // among its key tiles into the cache), then the softmax over its key tiles
@@ -1844,7 +1889,7 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
                                   pi == 0, sQ, sBar, abort);
                 if (x == 0 || ps.has_b) {
                     softmax_tile<false>(P, tmem, sBar, x, warp & 3, lane, x ? ps.t0b : ps.t0a, l, bl, b, hk, sp,
-                                 ps.j_base, ps.n_kv, done, (uint32_t)pi & 1u, p_count > 1, abort,
+                                 ps, done, (uint32_t)pi & 1u, p_count > 1, abort,
                                  pi == p_count - 1 ? sQ : 0u);
                     done += (uint32_t)ps.n_kv;
                 } else if (p_count > 1) {
@@ -1857,7 +1902,7 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
                 const PairSpan ps = pi == 0 ? ps0 : pair_span(P, p_first + pi, sp, s_r);
                 if (x == 0 || ps.has_b) {
                     softmax_tile<true>(P, tmem, sBar, x, warp & 3, lane, x ? ps.t0b : ps.t0a, l, bl, b, hk, sp,
-                                 ps.j_base, ps.n_kv, done, (uint32_t)pi & 1u, p_count > 1, abort,
+                                 ps, done, (uint32_t)pi & 1u, p_count > 1, abort,
                                  pi == p_count - 1 ? sQ : 0u);
                     done += (uint32_t)ps.n_kv;
                 } else if (p_count > 1) {    // no tile B in this pair: nothing of O to read
@@ -2069,6 +2114,8 @@ cudaError_t prepare_tc(const AttnParams& a, TcParams& p, dim3& grid) {
     p.part_o = a.part_o;
     p.part_lse = a.part_lse;
     p.tickets = kFused || p.n_split == 1 || p.n_split > kMaxMergeSplits ? nullptr : a.tickets;
+    p.sif_k = a.sif_k;
+    if (a.sif_k < 0 || (a.sif_k > 0 && (kFused || p.n_split != 1))) return cudaErrorInvalidValue;
     if (a.batch < 1 || a.batch > kMaxReq) return cudaErrorInvalidValue;
     std::memcpy(p.req, a.req, sizeof(ReqParam) * (size_t)a.batch);
     const int64_t pairs = ((a.sq + tq - 1) / tq + 1) / 2;

@@ -1502,22 +1502,16 @@ c2kv_status c2kv_extract_attention(c2kv_ctx* c, int32_t n_layers, const void* q,
         const int32_t hq = c->cfg.n_q_heads, hkv = c->cfg.n_kv_heads;
         const size_t qb = (size_t)n_layers * n_all * hq * d * c->eb;
         const size_t kb = (size_t)n_layers * n_all * hkv * d * c->eb;
-        // the tensor-core route merges two partials for the C2 rows through a normaliser
-        const bool need_lse = lse == nullptr && c2kv::extract_uses_tc(c->cfg.dtype, d, hq, hkv);
-        const size_t lb = need_lse ? (size_t)n_layers * hq * n_all * sizeof(float) : 0;
         void* q_rot = nullptr;
         void* k_rot = nullptr;
-        void* lse_scratch = nullptr;
         cudaError_t e = pool_alloc(c, &q_rot, qb);
         if (e == cudaSuccess) e = pool_alloc(c, &k_rot, kb);
-        if (e == cudaSuccess && need_lse) e = pool_alloc(c, &lse_scratch, lb);
         if (e != cudaSuccess) {
             if (k_rot) pool_free(c, k_rot);
             if (q_rot) pool_free(c, q_rot);
             return cuda_fail(c, e, "extract: scratch allocation");
         }
         c2kv::ExtractParams p{};
-        p.lse_scratch = static_cast<float*>(lse_scratch);
         p.err = c->d_err;
         p.q = q;
         p.k = k;
@@ -1544,7 +1538,6 @@ c2kv_status c2kv_extract_attention(c2kv_ctx* c, int32_t n_layers, const void* q,
                                      two ? c->aux_ev[0] : nullptr, two ? c->aux_ev[1] : nullptr);
         }
         if (e != cudaSuccess && two) cudaStreamSynchronize(c->aux);   // before the scratch goes
-        if (lse_scratch) pool_free(c, lse_scratch);
         pool_free(c, k_rot);
         pool_free(c, q_rot);
         if (e != cudaSuccess) return cuda_fail(c, e, "extract");

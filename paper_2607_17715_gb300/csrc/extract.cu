@@ -19,13 +19,12 @@
 // pieces the suffix-attention kernel already computes:
 //   1. document rows: plain causal attention over document keys 0..t, i.e. a "suffix" of n
 //      tokens over an empty prefix;
-//   2. C2 rows, causal part: c_j over c_0 .. c_j, a "suffix" of m tokens over an empty
-//      prefix whose keys start at row n;
-//   3. C2 rows, block-local part: c_j over the at most 2k document keys of the sink block
-//      and B(j), on the CUDA cores (extract_local_kernel), merged with part 2 exactly by
-//      log-sum-exp: the two key sets are disjoint and together are what c_j sees.
-// Parts 1 and 2 are launches of attn_tc_kernel with a token pitch of n + m, so they read
-// and write the extraction layout in place.
+//   2. C2 rows: a "suffix" of m tokens after n "slots", the document rows, so that c_j sees
+//      c_0 .. c_j causally; the kernel's SIF mode (sif_k = k) masks every document key but
+//      those of the sink block and B(j), and visits only the key tiles that hold them (for
+//      a pair of 2 x 128 packed rows: its blocks' tiles, tile 0, the C2 tiles).
+// Both are launches of attn_tc_kernel with a token pitch of n + m, so they read and write
+// the extraction layout in place.
 //
 // CUDA cores (fp32, d = 64, other group sizes): extract_attn_kernel runs every row with fp32
 // accumulation: one CTA holds RB packed query rows (row r = t * G + g: token t, query head
@@ -221,146 +220,6 @@ __global__ void __launch_bounds__(XNW * 32) extract_attn_kernel(const __grid_con
     }
 }
 
-// Part 3 of the tensor-core route, on the CUDA cores: four threads per (C2 token c_j, query
-// head) pair, each holding 32 of the 128 channels of its query and of its output; a CTA takes
-// 32 pairs (32/G tokens) of one (layer, KV head).  Per visible document key (the sink block,
-// then B(j) when j > 0) the four threads read their 64-byte slices of the K and V rows, the
-// score is summed over the four with two shuffles within the group, and each keeps the same
-// online softmax.  The loads of KB keys are issued before any is used.  The partial
-// (O_b, lse_b) is merged with part 2's (O_a, lse_a), read from out and the normaliser array,
-// by the exact rule O = (2^lse_a O_a + 2^lse_b O_b) / (2^lse_a + 2^lse_b).
-template <int G>
-__global__ void __launch_bounds__(128) extract_local_kernel(const __grid_constant__ ExtractParams P) {
-    constexpr int D = 128, CH = 32, TPC = 32 / G, KB = 2;
-    using bf = __nv_bfloat16;
-    const int lane = threadIdx.x & 31;
-    const int cg = threadIdx.x & 3;                        // channel group: 32cg .. 32cg+31
-    const int pi = threadIdx.x >> 2;                       // pair
-    const int jj = pi / G, g = pi - (pi / G) * G;
-    const int m = P.n_all - P.n;
-    const int j = blockIdx.x * TPC + jj;
-    const int hk = blockIdx.y, l = blockIdx.z;
-    if (j >= m) return;                                    // the pair's four lanes leave together
-    const unsigned grp = 0xfu << (lane & 28);              // the pair's four lanes
-    const int n = P.n, k = P.ratio;
-    const int tq = n + j;
-    const int h = hk * G + g;
-    const float sc = P.scale_log2;
-    auto unpack8 = [](const uint4& u, float* f) {
-        const uint32_t w[4] = {u.x, u.y, u.z, u.w};
-#pragma unroll
-        for (int i = 0; i < 4; ++i) {
-            f[2 * i] = __uint_as_float(w[i] << 16);
-            f[2 * i + 1] = __uint_as_float(w[i] & 0xffff0000u);
-        }
-    };
-    float q[CH];
-    {
-        const uint4* qr = reinterpret_cast<const uint4*>(
-            static_cast<const bf*>(P.q_rot) + (((int64_t)l * P.n_all + tq) * P.hq + h) * D + cg * CH);
-#pragma unroll
-        for (int c = 0; c < 4; ++c) unpack8(qr[c], q + 8 * c);
-    }
-    const int sink_end = min(k, n);
-    const int lo = j * k, hi = min((j + 1) * k, n);
-    const int nk = j == 0 ? hi - lo : sink_end + (hi - lo);     // B(0) is the sink block
-    const int64_t kv_stride = (int64_t)P.hkv * D;
-    const bf* kb = static_cast<const bf*>(P.k_rot) + ((int64_t)l * P.n_all * P.hkv + hk) * D + cg * CH;
-    const bf* vb = static_cast<const bf*>(P.v) + ((int64_t)l * P.n_all * P.hkv + hk) * D + cg * CH;
-    float mr = -CUDART_INF_F, lr = 0.f, acc[CH];
-#pragma unroll
-    for (int c = 0; c < CH; ++c) acc[c] = 0.f;
-    for (int i0 = 0; i0 < nk; i0 += KB) {
-        uint4 kx[KB][4], vx[KB][4];
-#pragma unroll
-        for (int b = 0; b < KB; ++b) {
-            const int i = i0 + b;
-            if (i >= nk) break;
-            const int u = j == 0 ? lo + i : (i < sink_end ? i : lo + i - sink_end);
-            const uint4* kr = reinterpret_cast<const uint4*>(kb + u * kv_stride);
-            const uint4* vr = reinterpret_cast<const uint4*>(vb + u * kv_stride);
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                kx[b][c] = kr[c];
-                vx[b][c] = vr[c];
-            }
-        }
-#pragma unroll
-        for (int b = 0; b < KB; ++b) {
-            if (i0 + b >= nk) break;                       // the same for the pair's four lanes
-            float sp[4] = {0.f, 0.f, 0.f, 0.f};            // four independent chains
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                float kf[8];
-                unpack8(kx[b][c], kf);
-#pragma unroll
-                for (int e = 0; e < 8; ++e) sp[c] = fmaf(q[8 * c + e], kf[e], sp[c]);
-            }
-            float s = (sp[0] + sp[1]) + (sp[2] + sp[3]);
-            s += __shfl_xor_sync(grp, s, 1);
-            s += __shfl_xor_sync(grp, s, 2);
-            const float sl = s * sc;
-            const float mn = fmaxf(mr, sl);
-            const float a = exp2f(mr - mn);                // 0 on the first key
-            const float pw = exp2f(sl - mn);
-            lr = lr * a + pw;
-#pragma unroll
-            for (int c = 0; c < 4; ++c) {
-                float vf[8];
-                unpack8(vx[b][c], vf);
-#pragma unroll
-                for (int e = 0; e < 8; ++e) acc[8 * c + e] = fmaf(pw, vf[e], acc[8 * c + e] * a);
-            }
-            mr = mn;
-        }
-    }
-
-    float* lse_ab = P.lse != nullptr ? P.lse : P.lse_scratch;
-    const int64_t lse_id = ((int64_t)l * P.hq + h) * P.n_all + tq;
-    const float la = lse_ab[lse_id] * 1.4426950408889634f;   // part 2, natural log -> log2
-    const float lb = mr + log2f(lr);
-    const float mx = fmaxf(la, lb);
-    const float wa = exp2f(la - mx), wb = exp2f(lb - mx);
-    const float inv = 1.f / (wa + wb);
-    const float fa = wa * inv, fb = wb * inv / lr;
-    uint4* orow = reinterpret_cast<uint4*>(static_cast<bf*>(P.out) + (((int64_t)l * P.n_all + tq) * P.hq + h) * D + cg * CH);
-#pragma unroll
-    for (int c = 0; c < 4; ++c) {
-        float oa[8];
-        unpack8(orow[c], oa);
-        uint32_t w[4];
-#pragma unroll
-        for (int e = 0; e < 4; ++e) {
-            __nv_bfloat162 r = __floats2bfloat162_rn(fmaf(fa, oa[2 * e], fb * acc[8 * c + 2 * e]),
-                                                     fmaf(fa, oa[2 * e + 1], fb * acc[8 * c + 2 * e + 1]));
-            w[e] = *reinterpret_cast<uint32_t*>(&r);
-        }
-        orow[c] = make_uint4(w[0], w[1], w[2], w[3]);
-    }
-    __syncwarp(grp);                                       // every lane of the pair has read lse_a
-    if (P.lse != nullptr && cg == 0) P.lse[lse_id] = (mx + log2f(wa + wb)) * 0.69314718055994531f;
-}
-
-template <int G>
-cudaError_t launch_local(const ExtractParams& p, cudaStream_t s) {
-    constexpr int TPC = 32 / G;
-    const dim3 grid((unsigned)((p.n_all - p.n + TPC - 1) / TPC), (unsigned)p.hkv, (unsigned)p.lq);
-    if (grid.x > 0x7fffffffu) return cudaErrorInvalidValue;
-    extract_local_kernel<G><<<grid, 128, 0, s>>>(p);
-    return cudaGetLastError();
-}
-
-cudaError_t launch_local_any(const ExtractParams& p, cudaStream_t s) {
-    switch (p.hq / p.hkv) {
-        case 1: return launch_local<1>(p, s);
-        case 2: return launch_local<2>(p, s);
-        case 4: return launch_local<4>(p, s);
-        case 8: return launch_local<8>(p, s);
-        case 16: return launch_local<16>(p, s);
-        default: return cudaErrorInvalidValue;
-    }
-}
-
 cudaError_t launch_tc(const ExtractParams& p, cudaStream_t s, cudaStream_t s2, cudaEvent_t fork,
                       cudaEvent_t join) {
     constexpr int D = 128;
@@ -369,7 +228,6 @@ cudaError_t launch_tc(const ExtractParams& p, cudaStream_t s, cudaStream_t s2, c
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     const int m = p.n_all - p.n;
-    float* lse_ab = p.lse != nullptr ? p.lse : p.lse_scratch;
     AttnParams a{};
     a.cache_k = p.k_rot;
     a.cache_v = p.v;
@@ -386,8 +244,8 @@ cudaError_t launch_tc(const ExtractParams& p, cudaStream_t s, cudaStream_t s2, c
     a.scale_log2 = p.scale_log2;
     a.n_split = 1;
     a.pairs_per_cta = p.pairs_per_cta;
-    // pieces 2 and 3 write only the C2 rows (and read the rotated rows): with a second stream
-    // they run beside piece 1, in the SMs its last wave of CTAs leaves idle
+    // piece 2 writes only the C2 rows (and reads the rotated rows): with a second stream it
+    // runs beside piece 1, in the SMs its last wave of CTAs leaves idle
     cudaStream_t sc = s;
     if (s2 != nullptr) {
         e = cudaEventRecord(fork, s);
@@ -403,16 +261,17 @@ cudaError_t launch_tc(const ExtractParams& p, cudaStream_t s, cudaStream_t s2, c
     a.req[0] = ReqParam{0, 0, 0, 0};
     e = launch_attn_tc(a, s);
     if (e != cudaSuccess) return e;
-    // 2. C2 rows over c_0 .. c_j (keys from row n), always with a normaliser for the merge
+    // 2. C2 rows: the n document rows as the request's slots, the C2 rows as its suffix, so
+    // that c_j sees c_0 .. c_j causally; the kernel's SIF mode keeps, of the document keys,
+    // the sink block and B(j), and visits only their key tiles
     const int64_t c2_off = (int64_t)p.n * p.hq * D;
     a.q_rot = static_cast<const __nv_bfloat16*>(p.q_rot) + c2_off;
     a.out = static_cast<__nv_bfloat16*>(p.out) + c2_off;
-    a.lse = lse_ab + p.n;
+    a.lse = p.lse != nullptr ? p.lse + p.n : nullptr;
     a.sq = m;
-    a.req[0] = ReqParam{p.n, 0, 0, 0};
+    a.sif_k = p.ratio;
+    a.req[0] = ReqParam{0, p.n, 0, 0};
     e = launch_attn_tc(a, sc);
-    // 3. C2 rows over the sink block and their own block, merged into 2
-    if (e == cudaSuccess) e = launch_local_any(p, sc);
     if (s2 != nullptr) {       // the work ends on s
         cudaError_t ej = cudaEventRecord(join, s2);
         if (ej == cudaSuccess) ej = cudaStreamWaitEvent(s, join, 0);
@@ -442,10 +301,7 @@ cudaError_t launch_extract(const ExtractParams& p, int dtype, int d, cudaStream_
     (void)cudaGetLastError();   // report this launch's error only, not a stale one
     if (p.n_all < 1 || p.lq < 1) return cudaSuccess;
     if (p.lq > 65535 || p.hkv > 65535) return cudaErrorInvalidValue;
-    if (extract_uses_tc(dtype, d, p.hq, p.hkv)) {
-        if (p.lse == nullptr && p.lse_scratch == nullptr) return cudaErrorInvalidValue;
-        return launch_tc(p, s, s2, fork, join);
-    }
+    if (extract_uses_tc(dtype, d, p.hq, p.hkv)) return launch_tc(p, s, s2, fork, join);
     if (dtype == kDtypeF32 && d == 64) return launch_typed<float, 64>(p, s);
     if (dtype == kDtypeF32 && d == 128) return launch_typed<float, 128>(p, s);
     if (dtype == kDtypeBf16 && d == 64) return launch_typed<__nv_bfloat16, 64>(p, s);

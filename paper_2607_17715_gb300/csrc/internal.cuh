@@ -154,6 +154,11 @@ struct AttnParams {
                              // merges), or one zeroed counter per (layer, request, KV head,
                              // pair): the unit's last split merges the partials in the kernel
                              // and sets it back to zero
+    int32_t sif_k;           // tensor-core kernel, extraction C2 rows (Sec. 3.3.1): 0, or the
+                             // ratio k: the request's n_slots key rows are then the chunk's n
+                             // document tokens, suffix token j is C2 token c_j, and of the
+                             // document keys row j sees only the sink block [0, min(k, n)) and
+                             // its own block [jk, min((j+1)k, n)); n_split must be 1
     ReqParam req[kMaxReq];
 };
 
@@ -218,7 +223,6 @@ struct ExtractParams {
     void* k_rot;             // scratch, shaped like k
     void* out;               // [Lq][n_all][Hq][d]
     float* lse;              // [Lq][Hq][n_all] or null
-    float* lse_scratch;      // shaped like lse: the C2 rows' partial normaliser when lse is null
     int32_t* err;            // device error word (bounded waits of the tensor-core kernel)
     int32_t lq;
     int32_t n;               // document tokens
@@ -230,12 +234,12 @@ struct ExtractParams {
     int32_t pairs_per_cta;   // the tensor-core attention launches' AttnParams::pairs_per_cta
     RopeTurns rope;
 };
-// With s2 (and the events fork and join), the tensor-core route runs the C2 rows' attention and
-// block-local merge on s2, beside the document rows' attention on s; the work ends on s.
+// With s2 (and the events fork and join), the tensor-core route runs the C2 rows' attention on
+// s2, beside the document rows' attention on s; the work ends on s.
 cudaError_t launch_extract(const ExtractParams& p, int dtype, int d, cudaStream_t s,
                            cudaStream_t s2 = nullptr, cudaEvent_t fork = nullptr, cudaEvent_t join = nullptr);
-// Whether launch_extract takes the tensor-core route (and so needs lse_scratch when lse is
-// null); otherwise every row runs on the CUDA cores.
+// Whether launch_extract takes the tensor-core route; otherwise every row runs on the CUDA
+// cores.
 bool extract_uses_tc(int dtype, int d, int hq, int hkv);
 
 // Tiled tensor map for TMA (cuTensorMapEncodeTiled through the runtime's driver entry point);
