@@ -433,6 +433,14 @@ struct PairSpan {
     bool lead0;
     int n_mid, j_tail;
 };
+// Bit i set for the keys lo + i (i < 32) that lie in [a, b).
+__device__ __forceinline__ uint32_t range_bits(int lo, int a, int b) {
+    const int x = max(a - lo, 0), y = min(b - lo, 32);
+    if (y <= x) return 0u;                                   // (so x < 32 below)
+    const uint32_t below_y = y >= 32 ? 0xffffffffu : (1u << y) - 1u;
+    return below_y & ~((1u << x) - 1u);
+}
+
 // Key tile of the pair's i-th key tile.
 __device__ __forceinline__ int span_tile(const PairSpan& o, int i) {
     const int i1 = i - (o.lead0 ? 1 : 0);
@@ -480,7 +488,8 @@ __device__ __forceinline__ PairSpan pair_span(const TcParams& P, int pr, int sp,
 // in the 128-byte-swizzled layout and stored by TMA, instead of 16-byte stores of a row per
 // thread (which touch a separate cache line per thread).
 // kMerge: the plain kernel, whose split partials may be merged in the kernel (split_merge).
-template <bool kMerge>
+// kSif: the plain kernel over extraction C2 rows (TcParams::sif_k), its own instantiation.
+template <bool kMerge, bool kSif = false>
 __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, uint32_t sBar, int x,
                                             int quad, int lane, int t0, int l, int bl, int b,
                                             int hk, int sp, const PairSpan& span, uint32_t sf_base,
@@ -510,7 +519,7 @@ __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, u
         for (int c = 0; c < 4; ++c) tmem_ld32(tmem + lane_addr + colS + c * 32, sv[c]);
         tmem_ld_wait();
 
-        const int kbase = (kMerge ? span_tile(span, j) : span.j_base + j) * BN;   // (SIF: plain only)
+        const int kbase = (kSif ? span_tile(span, j) : span.j_base + j) * BN;
         if (kbase + BN - 1 > lim) {
 #pragma unroll
             for (int c = 0; c < 4; ++c)
@@ -518,20 +527,22 @@ __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, u
                 for (int e = 0; e < 32; ++e)
                     if (kbase + c * 32 + e > lim) sv[c][e] = __float_as_uint(-CUDART_INF_F);
         }
-        if constexpr (kMerge) {
+        if constexpr (kSif) {
             // extraction C2 row c_{t_row}: of the document keys (rows below s_r) it sees the
-            // sink block [0, min(k, n)) and its own block [t_row k, min((t_row + 1) k, n))
-            if (P.sif_k > 0 && kbase < s_r) {
+            // sink block [0, min(k, n)) and its own block [t_row k, min((t_row + 1) k, n)); per
+            // 32-key chunk, the bits of the keys that stay (those two blocks and the C2 keys)
+            if (kbase < s_r) {
                 const int sink = min(P.sif_k, s_r);
                 const int blo = t_row * P.sif_k, bhi = min(blo + P.sif_k, s_r);
 #pragma unroll
-                for (int c = 0; c < 4; ++c)
+                for (int c = 0; c < 4; ++c) {
+                    const int lo = kbase + c * 32;
+                    const uint32_t keep = range_bits(lo, 0, sink) | range_bits(lo, blo, bhi) |
+                                          range_bits(lo, s_r, lo + 32);
 #pragma unroll
-                    for (int e = 0; e < 32; ++e) {
-                        const int key = kbase + c * 32 + e;
-                        if (key < s_r && key >= sink && (key < blo || key >= bhi))
-                            sv[c][e] = __float_as_uint(-CUDART_INF_F);
-                    }
+                    for (int e = 0; e < 32; ++e)
+                        if (!(keep & (1u << e))) sv[c][e] = __float_as_uint(-CUDART_INF_F);
+                }
             }
         }
         // row max: three-input maxima, one chain per 32-column chunk
@@ -1115,7 +1126,7 @@ __device__ __noinline__ void fused_rest_producer(const FusedTcParams& F, int l, 
         }
         if (stored && pk < p_count && k_free(gk)) {
             const int st = gk % KSTAGES;
-            const int row = key0 + span_tile(sk, jk) * BN;
+            const int row = key0 + (sk.j_base + jk) * BN;
             mbar_expect_tx(bar(B_KL + st), TILE);
             tma_load_3d(sK + (uint32_t)(st * TILE), &P.tm_k, 0, hk, row, bar(B_KL + st));
             tma_load_3d(sK + (uint32_t)(st * TILE) + HALF_TILE, &P.tm_k, 64, hk, row, bar(B_KL + st));
@@ -1129,7 +1140,7 @@ __device__ __noinline__ void fused_rest_producer(const FusedTcParams& F, int l, 
         }
         if (stored && pv < p_count && v_free(gv)) {
             const int st = gv % VSTAGES;
-            const int row = key0 + span_tile(sv, jv) * BN;
+            const int row = key0 + (sv.j_base + jv) * BN;
             mbar_expect_tx(bar(B_VL + st), TILE);
             tma_load_3d(sV + (uint32_t)(st * TILE), &P.tm_v, 0, hk, row, bar(B_VL + st));
             tma_load_3d(sV + (uint32_t)(st * TILE) + HALF_TILE, &P.tm_v, 64, hk, row, bar(B_VL + st));
@@ -1609,6 +1620,7 @@ __device__ __forceinline__ void fused_suffix_prep(const FusedTcParams& F, int ts
 // that its CTA runs in turn: a pair's Q tiles once the MMAs of the previous pair have read
 // the last ones (B_QF), and the pairs' K and V tiles in order, each as soon as its ring stage
 // is free; whichever of the three can go first goes.
+template <bool kSif>
 __device__ __forceinline__ void plain_producer(const TcParams& P, int l, int bl, int b, int hk,
                                                int p_first, int p_count, int sp, int s_r, uint32_t sQ,
                                                uint32_t sK, uint32_t sV, uint32_t sBar,
@@ -1642,7 +1654,7 @@ __device__ __forceinline__ void plain_producer(const TcParams& P, int l, int bl,
         if (pk < p_count && (gk < KSTAGES || mbar_test(bar(B_KE + gk % KSTAGES),
                                                        (uint32_t)((gk / KSTAGES) - 1) & 1u))) {
             const int s = gk % KSTAGES;
-            const int krow = key0 + span_tile(sk, jk) * BN;
+            const int krow = key0 + (kSif ? span_tile(sk, jk) : sk.j_base + jk) * BN;
             mbar_expect_tx(bar(B_KF + s), TILE);
             tma_load_3d(sK + s * TILE, &P.tm_k, 0, hk, krow, bar(B_KF + s));
             tma_load_3d(sK + s * TILE + HALF_TILE, &P.tm_k, 64, hk, krow, bar(B_KF + s));
@@ -1657,7 +1669,7 @@ __device__ __forceinline__ void plain_producer(const TcParams& P, int l, int bl,
         if (pv < p_count && (gv < VSTAGES || mbar_test(bar(B_VE + gv % VSTAGES),
                                                        (uint32_t)((gv / VSTAGES) - 1) & 1u))) {
             const int s = gv % VSTAGES;
-            const int vrow = key0 + span_tile(sv, jv) * BN;
+            const int vrow = key0 + (kSif ? span_tile(sv, jv) : sv.j_base + jv) * BN;
             mbar_expect_tx(bar(B_VF + s), TILE);
             tma_load_3d(sV + s * TILE, &P.tm_v, 0, hk, vrow, bar(B_VF + s));
             tma_load_3d(sV + s * TILE + HALF_TILE, &P.tm_v, 64, hk, vrow, bar(B_VF + s));
@@ -1707,10 +1719,11 @@ __global__ void __launch_bounds__(256) suffix_angles_kernel(const __grid_constan
 // kFused: compose + suffix preparation + attention; kMulti (fused only): the CTA runs every
 // pair of query tiles of its (layer, request, KV head), the last pair first (it composes the
 // cache), the others from the cache.  A separate instantiation, so that the one-pair fused
-// kernel keeps its register allocation.
-template <bool kFused, bool kMulti = false>
-__global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
-    attn_tc_kernel(const __grid_constant__ typename KernelParams<kFused>::type KP) {
+// kernel keeps its register allocation.  kSif (plain only): extraction C2 rows
+// (TcParams::sif_k), a kernel of its own (attn_tc_sif_kernel) so that the plain kernel's code
+// stays as it is.
+template <bool kFused, bool kMulti, bool kSif>
+__device__ __forceinline__ void attn_tc_body(const typename KernelParams<kFused>::type& KP) {
     const TcParams& P = tc_params(KP);
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
@@ -1823,7 +1836,7 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
                     if (p_count > 1)
                         fused_rest_producer(KP, l, bl, b, hk, p_count, s_r, n_kv, sQ, sK, sV, sBar, abort);
             } else {
-                plain_producer(P, l, bl, b, hk, p_first, p_count, sp, s_r, sQ, sK, sV, sBar, abort);
+                plain_producer<kSif>(P, l, bl, b, hk, p_first, p_count, sp, s_r, sQ, sK, sV, sBar, abort);
             }
         } else if (warp == 1 && lane == 0 && n_kv > 0) {
             // ------------------------------------------------------------ MMA issuer
@@ -1901,7 +1914,7 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
             for (int pi = 0; pi < p_count; ++pi) {
                 const PairSpan ps = pi == 0 ? ps0 : pair_span(P, p_first + pi, sp, s_r);
                 if (x == 0 || ps.has_b) {
-                    softmax_tile<true>(P, tmem, sBar, x, warp & 3, lane, x ? ps.t0b : ps.t0a, l, bl, b, hk, sp,
+                    softmax_tile<true, kSif>(P, tmem, sBar, x, warp & 3, lane, x ? ps.t0b : ps.t0a, l, bl, b, hk, sp,
                                  ps, done, (uint32_t)pi & 1u, p_count > 1, abort,
                                  pi == p_count - 1 ? sQ : 0u);
                     done += (uint32_t)ps.n_kv;
@@ -1931,6 +1944,23 @@ __global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
                      "r"(kTmemCols)
                      : "memory");
     }
+}
+
+template <bool kFused, bool kMulti = false>
+__global__ void __launch_bounds__(kFused ? kThreadsFused : kThreads, 1)
+    attn_tc_kernel(const __grid_constant__ typename KernelParams<kFused>::type KP) {
+    attn_tc_body<kFused, kMulti, false>(KP);
+}
+
+__global__ void __launch_bounds__(kThreads, 1) attn_tc_sif_kernel(const __grid_constant__ TcParams KP) {
+    attn_tc_body<false, false, true>(KP);
+}
+
+// The kernel of an instantiation.
+template <bool kFused, bool kMulti, bool kSif>
+const void* tc_kernel_fn() {
+    if constexpr (kSif) return reinterpret_cast<const void*>(&attn_tc_sif_kernel);
+    else return reinterpret_cast<const void*>(&attn_tc_kernel<kFused, kMulti>);
 }
 
 // Merge the splits: lse = log2 sum_s 2^lse_s, O = sum_s 2^(lse_s - lse) O_s.  One warp per
@@ -2054,19 +2084,19 @@ namespace {
 
 // Host-side preparation shared by the plain and the fused launch: function attributes once
 // per process, the register-split guard, the tensor maps and the scalar parameters.
-template <bool kFused, bool kMulti = false>
+template <bool kFused, bool kMulti = false, bool kSif = false>
 cudaError_t prepare_tc(const AttnParams& a, TcParams& p, dim3& grid) {
     constexpr int threads = kFused ? kThreadsFused : kThreads;
     constexpr int high = kFused ? kRegsHighFused : kRegsHigh;
     constexpr int low_total = kFused ? 128 * (kRegsLowFused + kRegsLoadFused) : 128 * kRegsLow;
     // once per process (one device per context; function-local statics: thread-safe)
     static const cudaError_t smem_err = cudaFuncSetAttribute(
-        attn_tc_kernel<kFused, kMulti>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+        tc_kernel_fn<kFused, kMulti, kSif>(), cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
     if (smem_err != cudaSuccess) return smem_err;
     {   // the register split must not ask for more than the launch holds
         static const int launch_regs = []() {
             cudaFuncAttributes fa{};
-            return cudaFuncGetAttributes(&fa, attn_tc_kernel<kFused, kMulti>) == cudaSuccess ? fa.numRegs : -1;
+            return cudaFuncGetAttributes(&fa, tc_kernel_fn<kFused, kMulti, kSif>()) == cudaSuccess ? fa.numRegs : -1;
         }();
         if (launch_regs < 0) return cudaErrorInvalidDeviceFunction;
         if (launch_regs * threads < low_total + 256 * high) return cudaErrorInvalidConfiguration;
@@ -2115,7 +2145,7 @@ cudaError_t prepare_tc(const AttnParams& a, TcParams& p, dim3& grid) {
     p.part_lse = a.part_lse;
     p.tickets = kFused || p.n_split == 1 || p.n_split > kMaxMergeSplits ? nullptr : a.tickets;
     p.sif_k = a.sif_k;
-    if (a.sif_k < 0 || (a.sif_k > 0 && (kFused || p.n_split != 1))) return cudaErrorInvalidValue;
+    if (kSif != (a.sif_k > 0) || a.sif_k < 0 || (kSif && (kFused || p.n_split != 1))) return cudaErrorInvalidValue;
     if (a.batch < 1 || a.batch > kMaxReq) return cudaErrorInvalidValue;
     std::memcpy(p.req, a.req, sizeof(ReqParam) * (size_t)a.batch);
     const int64_t pairs = ((a.sq + tq - 1) / tq + 1) / 2;
@@ -2159,6 +2189,13 @@ cudaError_t launch_attn_tc(const AttnParams& a, cudaStream_t s, Hook before) {
     (void)cudaGetLastError();   // report this launch's error only, not a stale one
     TcParams p;
     dim3 grid;
+    if (a.sif_k > 0) {          // extraction C2 rows: their own instantiation, launched plainly
+        cudaError_t e = prepare_tc<false, false, true>(a, p, grid);
+        if (e != cudaSuccess) return e;
+        before();
+        attn_tc_sif_kernel<<<grid, kThreads, kSmemBytes, s>>>(p);
+        return cudaGetLastError();
+    }
     cudaError_t e = prepare_tc<false>(a, p, grid);
     if (e != cudaSuccess) return e;
     before();
