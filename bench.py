@@ -153,7 +153,7 @@ def step_rooflines(fused_ran, kern, kc_ms, ka_ms, f, hbm, bf16, src):
         return r
     parts = {o["kernel"]: o for o in r.values()}
     return {"roofline": fused_roofline(kern["fused"][0], f, hbm, bf16, src),
-            "roofline_compose": parts.get("compose_kernel"),
+            "roofline_compose": parts.get("compose_bulk_kernel"),
             "roofline_attend": parts.get("attn_tc_kernel", parts.get("attn_simt_kernel"))}
 
 

@@ -23,3 +23,17 @@ def test_attention_flops_match_the_mask():
     vis[:, s:] = np.tril(np.ones((sq, sq), dtype=bool))
     want = 4.0 * wl.head_dim * wl.n_q_heads * vis.sum() * wl.batch * wl.layers
     assert f["attn_flops"] == pytest.approx(want)
+
+
+def test_fused_step_reports_compose_and_attention_rooflines():
+    # the fused kernel carries "roofline"; the separate compose and attention kernels of the
+    # unfused steps are reported beside it, each against the HBM peak here
+    f = {"compose_bytes": 335544320, "attn_flops": 44040192000, "attn_bytes": 209715200,
+         "name": "llama8b", "fused_bytes": 385881088}
+    r = bench.step_rooflines(True, {"fused": (0.0926, 1)}, 0.0606, 0.0585, f, 6790.3, 1904.5, "measured")
+    assert r["roofline"]["kernel"].startswith("attn_tc_kernel<fused>")
+    assert r["roofline_compose"]["kernel"] == "compose_bulk_kernel"
+    assert abs(r["roofline_compose"]["frac"] - 335544320 / 0.0606e-3 / 6790.3e9) < 1e-3
+    assert r["roofline_attend"]["kernel"] == "attn_tc_kernel"
+    unfused = bench.step_rooflines(False, {}, 0.0606, 0.0585, f, 6790.3, 1904.5, "measured")
+    assert {o["kernel"] for o in unfused.values()} == {"compose_bulk_kernel", "attn_tc_kernel"}
