@@ -145,6 +145,7 @@ struct TcParams {                // CUtensorMap members carry their own alignmen
     float* part_lse;
     uint32_t* tickets;       // null, or per-unit counters: the last split merges (plain kernel)
     int32_t sif_k;           // 0, or extraction C2 rows with ratio k (plain kernel, one split)
+    int32_t key_pingpong;    // a last pair with one query tile splits its key tiles (plain kernel)
     ReqParam req[kMaxReq];
 };
 
@@ -504,7 +505,8 @@ __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, u
                                             int quad, int lane, int t0, int l, int bl, int b,
                                             int hk, int sp, const PairSpan& span, uint32_t sf_base,
                                             uint32_t od_par, bool arrive_oe,
-                                            volatile uint32_t* abort, uint32_t stage = 0u) {
+                                            volatile uint32_t* abort, uint32_t stage = 0u,
+                                            bool kpp = false) {
     auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
     const int G = P.group;
     // keys before the launch's first query token: the composed slots and, for a decode step
@@ -521,8 +523,10 @@ __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, u
     float m_run = -CUDART_INF_F;
     float l_run = 0.f;
 
-    for (int j = 0; j < n_kv; ++j) {
-        mbar_wait(bar(B_SF + x), (sf_base + (uint32_t)j) & 1u, P.err, abort);
+    // kpp: this warpgroup takes every other key tile (x, x + 2, ...) of the pair's one query
+    // tile; i counts the tiles it has taken
+    for (int j = kpp ? x : 0, i = 0; j < n_kv; j += kpp ? 2 : 1, ++i) {
+        mbar_wait(bar(B_SF + x), (sf_base + (uint32_t)i) & 1u, P.err, abort);
         tc_fence_after();
         uint32_t sv[4][32];
 #pragma unroll
@@ -572,8 +576,8 @@ __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, u
         const float alpha = resc ? ex2(m_run - m_new) : 1.0f;
         const float m_sub = m_use == -CUDART_INF_F ? 0.f : m_use;   // all masked so far
 
-        // S_x(j) complete implies P_x(j-1).V(j-1) complete: O_x is current and may be scaled
-        if (j >= 1 && __any_sync(0xffffffffu, resc)) {
+        // S_x(j) complete implies the P_x.V before it complete: O_x is current and may be scaled
+        if (i >= 1 && __any_sync(0xffffffffu, resc)) {
 #pragma unroll 1
             for (int c = 0; c < 8; ++c) {
                 uint32_t ov[16];
@@ -610,6 +614,51 @@ __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, u
         m_run = m_use;
         tc_fence_before();
         mbar_arrive(bar(B_PF + x));
+    }
+
+    if (kpp) {
+        // the two halves meet: B leaves its row's (m, l) in the Q_B tile (unused with one
+        // query tile), and A, once every MMA is done, folds O_B into O_A in TMEM with the
+        // exact rule (log2 domain, each half against its own reference maximum)
+        //     m = max(m_A, m_B),  w_x = 2^(m_x - m),  l = w_A l_A + w_B l_B,  O = w_A O_A + w_B O_B
+        const uint32_t xch = stage + (uint32_t)TILE + (uint32_t)r * 8u;
+        if (x == 1) {
+            asm volatile("st.shared.v2.f32 [%0], {%1, %2};" ::"r"(xch), "f"(m_run), "f"(l_run) : "memory");
+            asm volatile("bar.sync 4, 256;" ::: "memory");
+            if constexpr (kMerge)
+                if (P.n_split > 1 && P.tickets != nullptr) split_merge(P, sBar, x, r, t0, l, b, hk);
+            if (arrive_oe) {
+                tc_fence_before();
+                mbar_arrive(bar(B_OE));
+            }
+            return;
+        }
+        mbar_wait(bar(B_OD), od_par, P.err, abort);
+        tc_fence_after();
+        asm volatile("bar.sync 4, 256;" ::: "memory");
+        float m_b, l_b;
+        asm volatile("ld.shared.v2.f32 {%0, %1}, [%2];" : "=f"(m_b), "=f"(l_b) : "r"(xch) : "memory");
+        const float m = fmaxf(m_run, m_b);
+        const float w_a = l_run > 0.f ? ex2(m_run - m) : 0.f;
+        const float w_b = l_b > 0.f ? ex2(m_b - m) : 0.f;
+        const uint32_t colO_b = kColO + HD;
+#pragma unroll 1
+        for (int c = 0; c < 8; ++c) {
+            uint32_t oa[16], ob[16];
+            tmem_ld16(tmem + lane_addr + colO + c * 16, oa);
+            tmem_ld16(tmem + lane_addr + colO_b + c * 16, ob);
+            tmem_ld_wait();
+#pragma unroll
+            for (int e = 0; e < 16; ++e) {
+                const float va = w_a != 0.f ? w_a * __uint_as_float(oa[e]) : 0.f;   // (an empty half's O
+                const float vb = w_b != 0.f ? w_b * __uint_as_float(ob[e]) : 0.f;   //  is never read)
+                oa[e] = __float_as_uint(va + vb);
+            }
+            tmem_st16(tmem + lane_addr + colO + c * 16, oa);
+        }
+        tmem_st_wait();
+        l_run = w_a * l_run + w_b * l_b;
+        m_run = m;
     }
 
     // ---------------------------------------------------------------- epilogue
@@ -860,6 +909,76 @@ __device__ __forceinline__ void mma_issuer(const TcParams& P, uint32_t tmem, uin
     mma_commit(bar(B_OD));
     st.pa += (uint32_t)n_kv;
     if (kHasB) st.pb += (uint32_t)n_kv;
+}
+
+// The MMA issuer for a pair with one query tile (tile A) and n_kv >= 2 key tiles, the key tiles
+// split between the two halves of TMEM: tiles 0, 2, 4, ... go to (S_A, O_A), tiles 1, 3, 5, ...
+// to (S_B, O_B), and the two softmax warpgroups each run an online softmax over their half, so
+// that one half's softmax overlaps the other's MMAs as two query tiles' do (warpgroup A merges
+// the halves at the end).  Issue order: S(0), S(1), then per key tile j: P(j).V(j), S(j + 2)
+// on the same half (in issue order after the P.V that reads the P it overwrites).
+__device__ __forceinline__ void mma_issuer_kpp(const TcParams& P, uint32_t tmem, uint32_t sQ, uint32_t sK,
+                                               uint32_t sV, uint32_t sBar, int n_kv, int q_ready,
+                                               uint32_t q_par, RingState& st, bool wait_oe, uint32_t oe_par,
+                                               volatile uint32_t* abort) {
+    auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
+    constexpr uint32_t idS = idesc_bf16(BM, BN, false);
+    constexpr uint32_t idO = idesc_bf16(BM, HD, true);
+    constexpr uint64_t kTileDesc = (uint64_t)(TILE >> 4);
+    const uint64_t dQa = sw128_desc(sQ, 16, 1024);
+    const uint64_t dK0 = sw128_desc(sK, 16, 1024);
+    const uint64_t dV0 = sw128_desc(sV, HALF_TILE, 1024);
+    const uint32_t tS_a = tmem + kColS, tS_b = tmem + kColS + BN;
+    const uint32_t tO_a = tmem + kColO, tO_b = tmem + kColO + HD;
+    auto wait = [&](int i, uint32_t parity) {
+        mbar_wait(bar(i), parity, P.err, abort);
+        tc_fence_after();
+    };
+    int ks = st.ks, vs = st.vs;
+    uint32_t kph = st.kph, vph = st.vph;
+    auto s_next = [&](int x) {        // S of the next key tile into half x, its K stage released after
+        wait(B_KF + ks, kph);
+        const uint64_t dk = dK0 + (uint64_t)ks * kTileDesc;
+#pragma unroll
+        for (int kk = 0; kk < HD / 16; ++kk) {
+            const uint64_t off = (uint64_t)(((kk >> 2) * HALF_TILE + (kk & 3) * 32) >> 4);
+            mma_bf16(x ? tS_b : tS_a, dQa + off, dk + off, idS, kk > 0 ? 1u : 0u);
+        }
+        mma_commit(bar(B_SF + x));
+        mma_commit(bar(B_KE + ks));
+        kph ^= ks == KSTAGES - 1 ? 1u : 0u;
+        ks = ks == KSTAGES - 1 ? 0 : ks + 1;
+    };
+    wait(q_ready, q_par);
+    s_next(0);
+    s_next(1);
+    uint32_t pa = st.pa, pb = st.pb;   // P phases of each half completed before this pair
+#pragma unroll 1
+    for (int j = 0; j < n_kv; ++j) {
+        const int x = j & 1;
+        wait(B_PF + x, (x ? pb : pa) & 1u);
+        pa += x ? 0u : 1u;
+        pb += x ? 1u : 0u;
+        wait(B_VF + vs, vph);
+        if (wait_oe && j == 0) wait(B_OE, oe_par);
+        const uint64_t dv = dV0 + (uint64_t)vs * kTileDesc;
+#pragma unroll
+        for (int kk = 0; kk < BN / 16; ++kk)
+            mma_bf16_ts(x ? tO_b : tO_a, (x ? tS_b : tS_a) + (uint32_t)kk * 8u,
+                        dv + (uint64_t)((kk * 2048) >> 4), idO, kk > 0 || j >= 2 ? 1u : 0u);
+        mma_commit(bar(B_VE + vs));
+        vph ^= vs == VSTAGES - 1 ? 1u : 0u;
+        vs = vs == VSTAGES - 1 ? 0 : vs + 1;
+        if (j + 2 < n_kv) s_next(x);
+    }
+    mma_commit(bar(B_QF));
+    mma_commit(bar(B_OD));
+    st.ks = ks;
+    st.kph = kph;
+    st.vs = vs;
+    st.vph = vph;
+    st.pa = pa;
+    st.pb = pb;
 }
 
 // ------------------------------------------------------------------ fused loaders
@@ -1887,6 +2006,8 @@ __device__ __forceinline__ void attn_tc_body(const typename KernelParams<kFused>
                     const uint32_t q_par = (uint32_t)pi & 1u, oe_par = (uint32_t)(pi - 1) & 1u;
                     if (ps.has_b)
                         mma_issuer<true>(P, tmem, sQ, sK, sV, sBar, ps.n_kv, B_Q, q_par, st, pi > 0, oe_par, abort);
+                    else if (P.key_pingpong && ps.n_kv >= 2 && pi == p_count - 1)   // key tiles ping-pong
+                        mma_issuer_kpp(P, tmem, sQ, sK, sV, sBar, ps.n_kv, B_Q, q_par, st, pi > 0, oe_par, abort);
                     else
                         mma_issuer<false>(P, tmem, sQ, sK, sV, sBar, ps.n_kv, B_Q, q_par, st, pi > 0, oe_par, abort);
                 }
@@ -1939,11 +2060,14 @@ __device__ __forceinline__ void attn_tc_body(const typename KernelParams<kFused>
             uint32_t done = 0u;     // S_x tiles of the earlier pairs
             for (int pi = 0; pi < p_count; ++pi) {
                 const PairSpan ps = pi == 0 ? ps0 : pair_span(P, p_first + pi, sp, s_r);
-                if (x == 0 || ps.has_b) {
-                    softmax_tile<true, kSif>(P, tmem, sBar, x, warp & 3, lane, x ? ps.t0b : ps.t0a, l, bl, b, hk, sp,
-                                 ps, done, (uint32_t)pi & 1u, p_count > 1, abort,
-                                 pi == p_count - 1 ? sQ : 0u);
-                    done += (uint32_t)ps.n_kv;
+                // one query tile over two or more key tiles (the CTA's last pair): the two
+                // warpgroups take alternate key tiles (mma_issuer_kpp) and merge at the end
+                const bool kpp = P.key_pingpong && !ps.has_b && ps.n_kv >= 2 && pi == p_count - 1;
+                if (x == 0 || ps.has_b || kpp) {
+                    softmax_tile<true, kSif>(P, tmem, sBar, x, warp & 3, lane, x && !kpp ? ps.t0b : ps.t0a, l, bl,
+                                 b, hk, sp, ps, done, (uint32_t)pi & 1u, p_count > 1, abort,
+                                 pi == p_count - 1 ? sQ : 0u, kpp);
+                    done += kpp ? (uint32_t)((ps.n_kv + 1 - x) / 2) : (uint32_t)ps.n_kv;
                 } else if (p_count > 1) {    // no tile B in this pair: nothing of O to read
                     mbar_arrive(bar(B_OE));
                 } else if (P.tickets != nullptr) {   // a split without tile B: the merge's two
@@ -2171,6 +2295,7 @@ cudaError_t prepare_tc(const AttnParams& a, TcParams& p, dim3& grid) {
     p.part_lse = a.part_lse;
     p.tickets = kFused || p.n_split == 1 || p.n_split > kMaxMergeSplits ? nullptr : a.tickets;
     p.sif_k = a.sif_k;
+    p.key_pingpong = kFused ? 0 : a.key_pingpong;
     if (kSif != (a.sif_k > 0) || a.sif_k < 0 || (kSif && (kFused || p.n_split != 1))) return cudaErrorInvalidValue;
     if (a.batch < 1 || a.batch > kMaxReq) return cudaErrorInvalidValue;
     std::memcpy(p.req, a.req, sizeof(ReqParam) * (size_t)a.batch);

@@ -1432,6 +1432,8 @@ c2kv_status c2kv_decode(c2kv_ctx* c, c2kv_cache* cache, int32_t layer, const voi
                 // last group)
                 const bool in_kernel = n_split > 1 && n_split <= c2kv::kMaxMergeSplits;
                 a.tickets = in_kernel ? c->tickets : nullptr;
+                // the two softmax warpgroups take alternate key tiles of the one query tile
+                a.key_pingpong = 1;
                 // the suffix kernel's programmatic dependent, unless a trace puts events
                 // between them
                 a.dependent = c->prof ? 0 : 1;

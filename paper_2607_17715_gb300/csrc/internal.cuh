@@ -154,6 +154,10 @@ struct AttnParams {
                              // merges), or one zeroed counter per (layer, request, KV head,
                              // pair): the unit's last split merges the partials in the kernel
                              // and sets it back to zero
+    int32_t key_pingpong;    // tensor-core kernel: a pair with one query tile (a decode step's)
+                             // splits its key tiles between the two softmax warpgroups, merged
+                             // at the end (a different rounding order: off where the result must
+                             // equal the fused kernel's bit for bit)
     int32_t sif_k;           // tensor-core kernel, extraction C2 rows (Sec. 3.3.1): 0, or the
                              // ratio k: the request's n_slots key rows are then the chunk's n
                              // document tokens, suffix token j is C2 token c_j, and of the
