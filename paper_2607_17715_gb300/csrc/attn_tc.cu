@@ -145,7 +145,6 @@ struct TcParams {                // CUtensorMap members carry their own alignmen
     float* part_lse;
     uint32_t* tickets;       // null, or per-unit counters: the last split merges (plain kernel)
     int32_t sif_k;           // 0, or extraction C2 rows with ratio k (plain kernel, one split)
-    int32_t key_pingpong;    // a last pair with one query tile splits its key tiles (plain kernel)
     ReqParam req[kMaxReq];
 };
 
@@ -500,13 +499,15 @@ __device__ __forceinline__ PairSpan pair_span(const TcParams& P, int pr, int sp,
 // thread (which touch a separate cache line per thread).
 // kMerge: the plain kernel, whose split partials may be merged in the kernel (split_merge).
 // kSif: the plain kernel over extraction C2 rows (TcParams::sif_k), its own instantiation.
-template <bool kMerge, bool kSif = false>
+// kKpp: the plain kernel's decode instantiation, whose pairs with one query tile split their
+// key tiles between the two warpgroups (kpp: this pair does).
+template <bool kMerge, bool kSif = false, bool kKpp = false>
 __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, uint32_t sBar, int x,
                                             int quad, int lane, int t0, int l, int bl, int b,
                                             int hk, int sp, const PairSpan& span, uint32_t sf_base,
                                             uint32_t od_par, bool arrive_oe,
                                             volatile uint32_t* abort, uint32_t stage = 0u,
-                                            bool kpp = false) {
+                                            bool kpp_pair = false) {
     auto bar = [&](int i) { return sBar + 8u * (uint32_t)i; };
     const int G = P.group;
     // keys before the launch's first query token: the composed slots and, for a decode step
@@ -525,6 +526,7 @@ __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, u
 
     // kpp: this warpgroup takes every other key tile (x, x + 2, ...) of the pair's one query
     // tile; i counts the tiles it has taken
+    const bool kpp = kKpp && kpp_pair;
     for (int j = kpp ? x : 0, i = 0; j < n_kv; j += kpp ? 2 : 1, ++i) {
         mbar_wait(bar(B_SF + x), (sf_base + (uint32_t)i) & 1u, P.err, abort);
         tc_fence_after();
@@ -616,7 +618,7 @@ __device__ __forceinline__ void softmax_tile(const TcParams& P, uint32_t tmem, u
         mbar_arrive(bar(B_PF + x));
     }
 
-    if (kpp) {
+    if (kKpp && kpp) {
         // the two halves meet: B leaves its row's (m, l) in the Q_B tile (unused with one
         // query tile), and A, once every MMA is done, folds O_B into O_A in TMEM with the
         // exact rule (log2 domain, each half against its own reference maximum)
@@ -1851,7 +1853,7 @@ __global__ void __launch_bounds__(256) suffix_angles_kernel(const __grid_constan
 // kernel keeps its register allocation.  kSif (plain only): extraction C2 rows
 // (TcParams::sif_k), a kernel of its own (attn_tc_sif_kernel) so that the plain kernel's code
 // stays as it is.
-template <bool kFused, bool kMulti, bool kSif>
+template <bool kFused, bool kMulti, bool kSif, bool kKpp = false>
 __device__ __forceinline__ void attn_tc_body(const typename KernelParams<kFused>::type& KP) {
     const TcParams& P = tc_params(KP);
     extern __shared__ uint8_t smem_raw[];
@@ -2006,7 +2008,7 @@ __device__ __forceinline__ void attn_tc_body(const typename KernelParams<kFused>
                     const uint32_t q_par = (uint32_t)pi & 1u, oe_par = (uint32_t)(pi - 1) & 1u;
                     if (ps.has_b)
                         mma_issuer<true>(P, tmem, sQ, sK, sV, sBar, ps.n_kv, B_Q, q_par, st, pi > 0, oe_par, abort);
-                    else if (P.key_pingpong && ps.n_kv >= 2 && pi == p_count - 1)   // key tiles ping-pong
+                    else if (kKpp && ps.n_kv >= 2 && pi == p_count - 1)   // key tiles ping-pong
                         mma_issuer_kpp(P, tmem, sQ, sK, sV, sBar, ps.n_kv, B_Q, q_par, st, pi > 0, oe_par, abort);
                     else
                         mma_issuer<false>(P, tmem, sQ, sK, sV, sBar, ps.n_kv, B_Q, q_par, st, pi > 0, oe_par, abort);
@@ -2062,9 +2064,9 @@ __device__ __forceinline__ void attn_tc_body(const typename KernelParams<kFused>
                 const PairSpan ps = pi == 0 ? ps0 : pair_span(P, p_first + pi, sp, s_r);
                 // one query tile over two or more key tiles (the CTA's last pair): the two
                 // warpgroups take alternate key tiles (mma_issuer_kpp) and merge at the end
-                const bool kpp = P.key_pingpong && !ps.has_b && ps.n_kv >= 2 && pi == p_count - 1;
+                const bool kpp = kKpp && !ps.has_b && ps.n_kv >= 2 && pi == p_count - 1;
                 if (x == 0 || ps.has_b || kpp) {
-                    softmax_tile<true, kSif>(P, tmem, sBar, x, warp & 3, lane, x && !kpp ? ps.t0b : ps.t0a, l, bl,
+                    softmax_tile<true, kSif, kKpp>(P, tmem, sBar, x, warp & 3, lane, x && !kpp ? ps.t0b : ps.t0a, l, bl,
                                  b, hk, sp, ps, done, (uint32_t)pi & 1u, p_count > 1, abort,
                                  pi == p_count - 1 ? sQ : 0u, kpp);
                     done += kpp ? (uint32_t)((ps.n_kv + 1 - x) / 2) : (uint32_t)ps.n_kv;
@@ -2106,10 +2108,17 @@ __global__ void __launch_bounds__(kThreads, 1) attn_tc_sif_kernel(const __grid_c
     attn_tc_body<false, false, true>(KP);
 }
 
+// Decode steps (AttnParams::key_pingpong): the plain kernel whose last pair, when it has one
+// query tile, splits its key tiles between the two softmax warpgroups.
+__global__ void __launch_bounds__(kThreads, 1) attn_tc_decode_kernel(const __grid_constant__ TcParams KP) {
+    attn_tc_body<false, false, false, true>(KP);
+}
+
 // The kernel of an instantiation.
-template <bool kFused, bool kMulti, bool kSif>
+template <bool kFused, bool kMulti, bool kSif, bool kKpp = false>
 const void* tc_kernel_fn() {
     if constexpr (kSif) return reinterpret_cast<const void*>(&attn_tc_sif_kernel);
+    else if constexpr (kKpp) return reinterpret_cast<const void*>(&attn_tc_decode_kernel);
     else return reinterpret_cast<const void*>(&attn_tc_kernel<kFused, kMulti>);
 }
 
@@ -2234,19 +2243,19 @@ namespace {
 
 // Host-side preparation shared by the plain and the fused launch: function attributes once
 // per process, the register-split guard, the tensor maps and the scalar parameters.
-template <bool kFused, bool kMulti = false, bool kSif = false>
+template <bool kFused, bool kMulti = false, bool kSif = false, bool kKpp = false>
 cudaError_t prepare_tc(const AttnParams& a, TcParams& p, dim3& grid) {
     constexpr int threads = kFused ? kThreadsFused : kThreads;
     constexpr int high = kFused ? kRegsHighFused : kRegsHigh;
     constexpr int low_total = kFused ? 128 * (kRegsLowFused + kRegsLoadFused) : 128 * kRegsLow;
     // once per process (one device per context; function-local statics: thread-safe)
     static const cudaError_t smem_err = cudaFuncSetAttribute(
-        tc_kernel_fn<kFused, kMulti, kSif>(), cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+        tc_kernel_fn<kFused, kMulti, kSif, kKpp>(), cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
     if (smem_err != cudaSuccess) return smem_err;
     {   // the register split must not ask for more than the launch holds
         static const int launch_regs = []() {
             cudaFuncAttributes fa{};
-            return cudaFuncGetAttributes(&fa, tc_kernel_fn<kFused, kMulti, kSif>()) == cudaSuccess ? fa.numRegs : -1;
+            return cudaFuncGetAttributes(&fa, tc_kernel_fn<kFused, kMulti, kSif, kKpp>()) == cudaSuccess ? fa.numRegs : -1;
         }();
         if (launch_regs < 0) return cudaErrorInvalidDeviceFunction;
         if (launch_regs * threads < low_total + 256 * high) return cudaErrorInvalidConfiguration;
@@ -2295,8 +2304,9 @@ cudaError_t prepare_tc(const AttnParams& a, TcParams& p, dim3& grid) {
     p.part_lse = a.part_lse;
     p.tickets = kFused || p.n_split == 1 || p.n_split > kMaxMergeSplits ? nullptr : a.tickets;
     p.sif_k = a.sif_k;
-    p.key_pingpong = kFused ? 0 : a.key_pingpong;
+
     if (kSif != (a.sif_k > 0) || a.sif_k < 0 || (kSif && (kFused || p.n_split != 1))) return cudaErrorInvalidValue;
+    if (kKpp != (a.key_pingpong != 0) || (kKpp && (kFused || kSif))) return cudaErrorInvalidValue;
     if (a.batch < 1 || a.batch > kMaxReq) return cudaErrorInvalidValue;
     std::memcpy(p.req, a.req, sizeof(ReqParam) * (size_t)a.batch);
     const int64_t pairs = ((a.sq + tq - 1) / tq + 1) / 2;
@@ -2347,7 +2357,7 @@ cudaError_t launch_attn_tc(const AttnParams& a, cudaStream_t s, Hook before) {
         attn_tc_sif_kernel<<<grid, kThreads, kSmemBytes, s>>>(p);
         return cudaGetLastError();
     }
-    cudaError_t e = prepare_tc<false>(a, p, grid);
+    cudaError_t e = a.key_pingpong ? prepare_tc<false, false, false, true>(a, p, grid) : prepare_tc<false>(a, p, grid);
     if (e != cudaSuccess) return e;
     before();
     if (a.dependent) {          // starts while the kernel before it runs (the producer waits)
@@ -2361,8 +2371,11 @@ cudaError_t launch_attn_tc(const AttnParams& a, cudaStream_t s, Hook before) {
         attr[0].val.programmaticStreamSerializationAllowed = 1;
         cfg.attrs = attr;
         cfg.numAttrs = 1;
-        e = cudaLaunchKernelEx(&cfg, attn_tc_kernel<false>, p);
+        e = a.key_pingpong ? cudaLaunchKernelEx(&cfg, attn_tc_decode_kernel, p)
+                           : cudaLaunchKernelEx(&cfg, attn_tc_kernel<false>, p);
         if (e != cudaSuccess) return e;
+    } else if (a.key_pingpong) {
+        attn_tc_decode_kernel<<<grid, kThreads, kSmemBytes, s>>>(p);
     } else {
         attn_tc_kernel<false><<<grid, kThreads, kSmemBytes, s>>>(p);
     }
