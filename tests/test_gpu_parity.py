@@ -306,6 +306,13 @@ def test_attend_llama8b_layer(impl):
     _attend_case(L8B_1, attn_impl=impl)
 
 
+def test_attend_cuda_cores_large_launch():
+    # 4 layers x 8 KV heads x 16 CTAs of 16 query rows: a launch large enough that the
+    # CUDA-core kernel keeps 16 rows a CTA (smaller launches take 4); a ragged row count
+    wl = _small(L8B_1, layers=4, chunks_per_request=2, pool_chunks=2, n_suffix=61)
+    _attend_case(wl, attn_impl=1)
+
+
 @pytest.mark.parametrize("sq", [1, 7, 33, 100])
 def test_attend_ragged_suffix(sq):
     wl = _small(L8B_1, chunks_per_request=3, pool_chunks=3, chunk_tokens=300, ratio_k=10)
