@@ -925,8 +925,9 @@ def run_ours(args):
         # extraction attention (the C2 Extractor's masked attention) over one chunk
         "extract": extract_line(wl, world, ext_ms, ext_kernel_ms, hbm, bf16, src),
         # every kernel the library launched in the timed steps (counted by its trace of the
-        # identical traced pass)
-        "gpu_launches": sum(v[1] for v in kern.values()),
+        # identical traced pass; a fused record covers two launches, the suffix angles kernel
+        # and the fused kernel)
+        "gpu_launches": sum(v[1] for v in kern.values()) + kern.get("fused", (0.0, 0))[1],
         "clocks": clk,
     }
     if not args.no_long_decode:
