@@ -37,3 +37,31 @@ def test_fused_step_reports_compose_and_attention_rooflines():
     assert r["roofline_attend"]["kernel"] == "attn_tc_kernel"
     unfused = bench.step_rooflines(False, {}, 0.0606, 0.0585, f, 6790.3, 1904.5, "measured")
     assert {o["kernel"] for o in unfused.values()} == {"compose_bulk_kernel", "attn_tc_kernel"}
+
+
+def test_compose_bytes_count_every_slot_once():
+    # read and write of K and V per composed slot and layer, plus one int32 position per
+    # slot, with the slot count from the oracle's definition of m = ceil(n / k)
+    for name in ("llama8b", "long70b", "sweep_k10", "tiny_f32"):
+        wl = synth.workload(name)
+        f = bench.workload_facts(wl)
+        m = orc.n_slots(wl.chunk_tokens, wl.ratio_k)
+        slots = wl.batch * wl.chunks_per_request * m
+        eb = 4 if wl.dtype == "f32" else 2
+        want = 2 * 2 * slots * wl.n_kv_heads * wl.head_dim * eb * wl.layers + 4 * slots
+        assert f["compose_bytes"] == want, name
+
+
+@pytest.mark.parametrize("name,keys,tc", [("llama8b", 1360, False), ("sweep_k1", 32907, True),
+                                          ("batched", 1163, True), ("long70b", 2315, True),
+                                          ("tiny_f32", 160, False)])
+def test_decode_line_names_the_route_kernel(name, keys, tc):
+    # the library's rule: bf16 at head_dim 128 on the tensor cores when the (layer, request,
+    # KV head) units fit in one wave of SMs or a request has 32 key tiles or more
+    wl = synth.workload(name)
+    line = bench.decode_line(wl, 1, 0.05, 0.04, keys * wl.batch, 6790.3, "measured")
+    kernel = line["roofline"]["kernel"]
+    assert kernel.startswith("attn_tc_decode_kernel" if tc else "decode_kernel"), kernel
+    # algorithmic bytes: K and V of every key, every layer and KV head, once
+    eb = 4 if wl.dtype == "f32" else 2
+    assert line["roofline"]["bytes_per_launch"] == keys * wl.batch * wl.layers * wl.n_kv_heads * wl.head_dim * eb * 2
