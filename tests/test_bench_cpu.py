@@ -65,3 +65,26 @@ def test_decode_line_names_the_route_kernel(name, keys, tc):
     # algorithmic bytes: K and V of every key, every layer and KV head, once
     eb = 4 if wl.dtype == "f32" else 2
     assert line["roofline"]["bytes_per_launch"] == keys * wl.batch * wl.layers * wl.n_kv_heads * wl.head_dim * eb * 2
+
+
+def test_reference_arm_line_matches_the_contract():
+    # the oracle arm: one JSON line with impl "reference", the GPU arm's metric, unit and
+    # config object, its own cpu_baseline and an e2e object with no host-device bytes
+    import json
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    res = subprocess.run([sys.executable, os.path.join(root, "bench.py"), "--impl", "reference",
+                          "--steps", "3", "--warmup", "3"], capture_output=True, text=True,
+                         timeout=300, cwd=root)
+    assert res.returncode == 0, res.stderr[-2000:]
+    line = json.loads(res.stdout.strip().splitlines()[-1])
+    assert line["impl"] == "reference"
+    assert line["metric"] == "composed KV tokens/s" and line["unit"] == "tokens/s"
+    assert line["higher_is_better"] is True and line["steps"] == 3 and line["warmup"] == 3
+    assert line["config"] == bench.job_config(synth.workload("llama8b"), 1)
+    assert line["value"] > 0 and line["ms_per_step"] > 0
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["value"] == line["value"]
+    assert line["e2e"] == {"value": line["value"], "unit": line["unit"],
+                           "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
