@@ -168,7 +168,7 @@ struct FusedTcParams {
     int32_t n_occ;           // occurrences of the launch
     int64_t pool_slots;
     RopeTurns rope;
-    int32_t req_occ[kMaxReq + 1];
+    int32_t req_occ[kMaxFusedReq + 1];
     FusedOcc occ[kMaxFusedOcc];
 };
 
@@ -1834,7 +1834,7 @@ struct SfxAngles {
     float2* tab;
     int32_t sq, batch;
     RopeTurns rope;
-    ReqParam req[kMaxReq];
+    ReqParam req[kMaxFusedReq];
 };
 __global__ void __launch_bounds__(256) suffix_angles_kernel(const __grid_constant__ SfxAngles A) {
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
@@ -2383,7 +2383,7 @@ cudaError_t launch_attn_tc(const AttnParams& a, cudaStream_t s, Hook before) {
 }
 
 namespace {
-thread_local FusedTcParams g_fused;          // the prepared launch (18 KB: kept off the stack)
+thread_local FusedTcParams g_fused;          // the prepared launch (kept off the stack)
 thread_local SfxAngles g_angles;
 thread_local dim3 g_fused_grid;
 thread_local bool g_fused_ready = false;
@@ -2398,7 +2398,8 @@ cudaError_t prepare_attn_fused(const AttnParams& a, const FusedSpec& f) {
     cudaError_t e = g_fused_multi ? prepare_tc<true, true>(a, p.t, g_fused_grid)
                                   : prepare_tc<true, false>(a, p.t, g_fused_grid);
     if (e != cudaSuccess) return e;
-    if (a.layer0 != 0 || p.t.sq_pitch != a.sq || f.req_occ[0] != 0 || f.req_occ[a.batch] > kMaxFusedOcc)
+    if (a.batch > kMaxFusedReq || a.layer0 != 0 || p.t.sq_pitch != a.sq || f.req_occ[0] != 0 ||
+        f.req_occ[a.batch] > kMaxFusedOcc)
         return cudaErrorInvalidValue;
     const int64_t prow = (int64_t)a.lq * f.pool_slots;
     const int64_t crow = (int64_t)a.lq * a.rows;

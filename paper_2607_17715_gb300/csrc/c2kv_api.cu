@@ -1120,8 +1120,8 @@ c2kv_status c2kv_compose_attend(c2kv_ctx* c, int32_t batch, const int32_t* req_p
         c2kv_cache* cache = nullptr;
         st = compose_plan(c, batch, req_ptr, chunk_ids, positions, suffix_capacity, &cache, occ);
         if (st != C2KV_OK) return st;
-        // The fused kernel takes pool-resident chunks on the tensor-core route, one attention
-        // launch (at most kMaxReq requests) and at most kMaxFusedOcc occurrences; anything
+        // The fused kernel takes pool-resident chunks on the tensor-core route, at most
+        // kMaxFusedReq requests and at most kMaxFusedOcc occurrences; anything
         // else runs compose and then attention.  By default it runs only when one pair of
         // query tiles covers each (layer, request, KV head).  With more pairs, forcing it
         // (C2KV_FUSE_ALWAYS) runs them in turn in one CTA per (layer, request, KV head), the
@@ -1137,7 +1137,7 @@ c2kv_status c2kv_compose_attend(c2kv_ctx* c, int32_t batch, const int32_t* req_p
                     c->cfg.attn_impl != C2KV_ATTN_SIMT &&
                     c2kv::attn_tc_supported(c->cfg.dtype, c->cfg.head_dim, c->cfg.n_q_heads,
                                             c->cfg.n_kv_heads) &&
-                    batch <= c2kv::kMaxReq && occ.size() <= (size_t)c2kv::kMaxFusedOcc;
+                    batch <= c2kv::kMaxFusedReq && occ.size() <= (size_t)c2kv::kMaxFusedOcc;
         const bool pairs_in_turn = pairs > 1 && c->cfg.attn_split <= 1;
         bool host_chunks = false;
         for (const auto& o : occ) host_chunks = host_chunks || o.host;

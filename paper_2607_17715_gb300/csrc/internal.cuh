@@ -272,7 +272,13 @@ struct FusedOcc {
     int32_t n;               // original chunk length
     int32_t k;               // ratio
 };
-constexpr int kMaxFusedOcc = 512;
+// The fused launch carries its occurrence table and per-request ranges in its parameter block,
+// and a launch's latency grows with that block (about 0.4 us per KB on a GB300: the 32-layer
+// fused step took 92.7 us with room for 512 occurrences and 256 requests, 88.1 us with 32
+// occurrences).  So the fused route takes at most 128 occurrences of at most 32 requests;
+// larger calls compose, then attend.
+constexpr int kMaxFusedOcc = 128;
+constexpr int kMaxFusedReq = 32;
 struct FusedSpec {
     const void* pool_k;      // [L][pool_slots][Hkv][128]
     const void* pool_v;
@@ -287,7 +293,7 @@ struct FusedSpec {
                              // KV head), the last pair first, which composes the cache
     int64_t pool_slots;
     RopeTurns rope;
-    int32_t req_occ[kMaxReq + 1];   // request i of the launch: occurrences [req_occ[i], req_occ[i+1])
+    int32_t req_occ[kMaxFusedReq + 1];   // request i of the launch: occurrences [req_occ[i], req_occ[i+1])
     FusedOcc occ[kMaxFusedOcc];
 };
 // Host preparation (tensor maps, parameters) of a fused launch, then the launch.  The fused

@@ -403,8 +403,9 @@ def test_fused_traced_and_on_a_side_stream_give_the_same_bits():
 
 @pytest.mark.parametrize("n_req,per_req", [(300, 1), (130, 4)])
 def test_compose_attend_many_requests_or_occurrences(n_req, per_req):
-    # more than 256 requests, or more than 512 occurrences: the call composes, then attends
-    # in groups of 256 requests; sampled requests against the oracle
+    # more requests (32) or occurrences (128) than the fused launch takes, even forced: the
+    # call composes, then attends in groups of 256 requests; sampled requests against the
+    # oracle
     c2kv = H.lib()
     wl = synth.scaled(L8B, layers=1, chunk_tokens=64, ratio_k=4, pool_chunks=5, n_suffix=3,
                       batch=n_req)
