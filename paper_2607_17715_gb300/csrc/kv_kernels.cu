@@ -34,8 +34,13 @@ namespace {
 // the CTA to the tile (tile items / IPT threads, 32 to 256), so a launch of small tiles
 // keeps every thread's loads in flight and spreads evenly over the SMs.
 // ---------------------------------------------------------------------------------------
-template <typename T, int VPH>
-__global__ void __launch_bounds__(256) compose_kernel(const __grid_constant__ ComposeParams P) {
+template <int N>
+struct BulkParams;
+
+// N: the capacity of the launch's occurrence table (a parameter block sized to the launch: a
+// launch's latency grows with its parameter bytes).
+template <typename T, int VPH, int N>
+__global__ void __launch_bounds__(256) compose_kernel(const __grid_constant__ BulkParams<N> P) {
     using V = Vec16<T>;
     constexpr int E = V::N;
     constexpr int HALF = VPH * E;
@@ -663,6 +668,24 @@ cudaError_t launch_bulk(const ComposeParams& p, int layers, cudaStream_t s, Hook
     return launch_bulk_n<T, VPH, 512>(p, layers, s, pre);
 }
 
+// The 16-byte compose kernel with its occurrence table sized to the launch.
+template <typename T, int VPH, int N>
+cudaError_t launch_16b_n(const ComposeParams& p, dim3 grid, int threads, cudaStream_t s, Hook pre) {
+    BulkParams<N> bp;
+    static_cast<ComposeHead&>(bp) = p;
+    for (int i = 0; i < p.n_occ; ++i) bp.occ[i] = p.occ[i];
+    pre();
+    compose_kernel<T, VPH, N><<<grid, threads, 0, s>>>(bp);
+    return cudaGetLastError();
+}
+
+template <typename T, int VPH>
+cudaError_t launch_16b(const ComposeParams& p, dim3 grid, int threads, cudaStream_t s, Hook pre) {
+    if (p.n_occ <= 16) return launch_16b_n<T, VPH, 16>(p, grid, threads, s, pre);
+    if (p.n_occ <= 128) return launch_16b_n<T, VPH, 128>(p, grid, threads, s, pre);
+    return launch_16b_n<T, VPH, kMaxOcc>(p, grid, threads, s, pre);
+}
+
 cudaError_t launch_compose(const ComposeParams& p, int dtype, int d, int layers, cudaStream_t s,
                            int max_ctas, Hook pre) {
     if (p.n_tiles == 0 || p.n_occ == 0) return cudaSuccess;
@@ -682,13 +705,11 @@ cudaError_t launch_compose(const ComposeParams& p, int dtype, int d, int layers,
     // one thread per four items of a tile (item = slot, head, vector pair), in whole warps
     const int items = p.tile_slots * p.hkv * vph_of(dtype, d);
     const int threads = std::min(256, std::max(32, (items / 4 + 31) / 32 * 32));
-    pre();
-    if (dtype == kDtypeBf16 && d == 128) compose_kernel<__nv_bfloat16, 8><<<grid, threads, 0, s>>>(p);
-    else if (dtype == kDtypeBf16 && d == 64) compose_kernel<__nv_bfloat16, 4><<<grid, threads, 0, s>>>(p);
-    else if (dtype == kDtypeF32 && d == 128) compose_kernel<float, 16><<<grid, threads, 0, s>>>(p);
-    else if (dtype == kDtypeF32 && d == 64) compose_kernel<float, 8><<<grid, threads, 0, s>>>(p);
-    else return cudaErrorInvalidValue;
-    return cudaGetLastError();
+    if (dtype == kDtypeBf16 && d == 128) return launch_16b<__nv_bfloat16, 8>(p, grid, threads, s, pre);
+    if (dtype == kDtypeBf16 && d == 64) return launch_16b<__nv_bfloat16, 4>(p, grid, threads, s, pre);
+    if (dtype == kDtypeF32 && d == 128) return launch_16b<float, 16>(p, grid, threads, s, pre);
+    if (dtype == kDtypeF32 && d == 64) return launch_16b<float, 8>(p, grid, threads, s, pre);
+    return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_compress(const CompressParams& p, int dtype, int d, cudaStream_t s) {
