@@ -260,8 +260,8 @@ c2kv_status c2kv_attend(c2kv_ctx* ctx, c2kv_cache* cache, int32_t layer, const v
  *     c2kv_compose(ctx, batch, req_ptr, chunk_ids, positions, suffix_capacity, cache_out)
  *     c2kv_attend(ctx, *cache_out, -1, q, k_suf, v_suf, n_suffix, out, lse)
  * (the composed cache, its positions, the suffix rows, O and lse), for every layer.  On
- * the tensor-core route (bf16, d 128) with every chunk in the device pool, at most 256
- * requests, at most 512 chunk occurrences and LOCAL_ROPE storage, one fused kernel does all of it: the
+ * the tensor-core route (bf16, d 128) with every chunk in the device pool, at most 32
+ * requests, at most 128 chunk occurrences and LOCAL_ROPE storage, one fused kernel does all of it: the
  * attention reads each composed slot straight from the pool, turns K by its occurrence's
  * offset in shared memory (Sec. 3.2.4 re-rotation), turns the queries and the suffix keys by
  * their positions, and writes the composed cache as it goes, so the cache is written once
