@@ -504,3 +504,39 @@ def test_unfused_route_traced_equals_untraced():
         assert torch.equal(lse_a, lse_b)
     finally:
         c2kv.c2kv_destroy(ctx)
+
+
+@pytest.mark.parametrize("n_req,per_req,want_fused", [
+    (32, 4, True),        # 32 requests, 128 occurrences: the fused launch's limits
+    (33, 3, False),       # one request more than it takes
+    (16, 9, False),       # 144 occurrences
+])
+def test_fused_route_limits(n_req, per_req, want_fused):
+    # forced fusion on one pair of query tiles per (layer, request, KV head): the fused launch
+    # takes at most 32 requests and 128 occurrences (its parameter block is kept small),
+    # larger calls compose, then attend; either way sampled requests match the oracle
+    c2kv = H.lib()
+    wl = synth.scaled(L8B, layers=1, chunk_tokens=64, ratio_k=4, pool_chunks=5, n_suffix=3,
+                      batch=n_req)
+    chunks = H.oracle_chunks_meanpool(wl, list(range(5)))
+    ctx = H.make_ctx(wl, pool_slots=200, fuse=2)
+    try:
+        dev = H.load_stored(ctx, wl, chunks)
+        rng = np.random.default_rng(11)
+        reqs = [([int(x) for x in rng.integers(0, 5, per_req)], [64 * i for i in range(per_req)])
+                for _ in range(n_req)]
+        q, ks, vs = synth.suffix(wl, layers=1)
+        c2kv.c2kv_profile_enable(ctx, True)
+        cache, out, _ = _run(ctx, wl, dev, reqs, q, ks, vs, 3, fused=True)
+        kinds = c2kv.c2kv_profile_read(ctx)
+        assert (kinds["fused"][1] == 1) == want_fused
+        assert (kinds["compose"][1] >= 1) == (not want_fused)
+        got = out.double().cpu().numpy()
+        for r in (0, n_req - 1):
+            ids, offs = reqs[r]
+            ref = orc.run_request(chunks, ids, offs, q[:, r], ks[:, r], vs[:, r], wl.rope_theta,
+                                  wl.dtype)
+            H.check_attention(got[:, r], ref["out"], wl, f"O req {r}")
+        c2kv.c2kv_cache_release(ctx, cache)
+    finally:
+        c2kv.c2kv_destroy(ctx)
